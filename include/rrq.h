@@ -1,0 +1,143 @@
+/*
+ * rrq.h -- C ABI of the GB300 (sm_103a) Recurrent Residual Quantization
+ * library: construction of the 2/4/6/8-bit RRQ package from bf16 weights and
+ * prefix reconstruction of bf16 weights from it.
+ *
+ * The operation (paper: "Recurrent Residual Quantization", Section 3):
+ *   - Section 3.1, Eq. 1-3: a group of consecutive weights shares a scale s
+ *     and zero-point; each weight gets an integer code Q, and the residual is
+ *     the weight minus its dequantized value.
+ *   - Section 3.2, Eq. 4-7 and Algorithm 1: the base stage quantizes W; each
+ *     of the following stages quantizes the running residual of the previous
+ *     one and subtracts its dequantized value.  With four 2-bit stages the
+ *     package serves the 2-, 4-, 6- and 8-bit operating points.
+ *   - Section 3.2, Eq. 8 (and Appendix C): the weight at prefix t is the
+ *     base plus the first t residual stages.
+ *   - Section 5.1: 2-bit round-to-nearest stages, group size 128.
+ *
+ * Arithmetic (identical, bit for bit, to the definition below; every step
+ * is one IEEE-754 binary32 operation rounded to nearest-even, no fused
+ * multiply-add, subnormals kept):
+ *     lo = min(v), hi = max(v) over the group, ordering -0 before +0
+ *     s  = fl(fl(hi - lo) / 3)                       3 = 2^2 - 1 steps
+ *     Q  = s == 0 ? 0 : clamp(rhe(fl(fl(v - lo) / s)), 0, 3)
+ *     L  = fl(lo + fl(Q * s))                        dequantized value
+ *     v' = fl(v - L)                                 running residual
+ *   v starts as the bf16 weight widened to binary32; rhe = round half to
+ *   even.  The stored zero of a stage is lo (the real offset m = -z*s).
+ *   Reconstruction with k stages: acc = L_0; acc = fl(acc + L_i) for
+ *   i = 1..k-1; output = bf16 round-to-nearest-even of acc.
+ *
+ * Layout (all buffers are caller-owned device memory of the current device):
+ *   W         bf16 [rows, cols] row-major; a group is `group` consecutive
+ *             elements of a row, so the flattened group index of element
+ *             c = r*cols + j is c / group.
+ *   codes[k]  uint8 [rows*cols/4] for stage k: element c is at byte c/4,
+ *             bits 2*(c%4) and 2*(c%4)+1 (least significant first).
+ *   scales[k] float [rows*cols/group], zeros[k] float [rows*cols/group].
+ *
+ * Calls are asynchronous on `stream` (a cudaStream_t; NULL = the legacy
+ * default stream).  Outputs are valid once the stream reaches the call.  The
+ * library never allocates, frees or synchronizes in these calls; only
+ * rrq_get_device_status synchronizes.  A bad argument returns an error code
+ * synchronously and launches nothing.  Functions are thread-safe.
+ */
+#ifndef RRQ_H
+#define RRQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+struct CUstream_st;                        /* cudaStream_t is struct CUstream_st* */
+typedef struct CUstream_st* rrq_stream_t;
+
+typedef enum {
+  RRQ_OK = 0,
+  RRQ_ERR_INVALID_ARG = 1, /* null pointer, non-positive size, cols % group != 0,
+                              n_stages or k out of range, pointer not device memory
+                              of the current device, aliasing outputs */
+  RRQ_ERR_UNSUPPORTED = 2, /* group not in {32, 64, 128, 256} */
+  RRQ_ERR_MISALIGNED = 3,  /* a pointer breaks the alignment stated below */
+  RRQ_ERR_CUDA = 4,        /* a CUDA runtime call or kernel launch failed; see
+                              rrq_last_cuda_error() */
+  RRQ_ERR_TIMEOUT = 5      /* a kernel gave up waiting for its own data copies
+                              (reported by rrq_get_device_status) */
+} rrq_status;
+
+#define RRQ_MAX_STAGES 4
+
+/* Build the RRQ package of one bf16 weight matrix (Algorithm 1 without a base
+ * checkpoint; Eq. 1-7).
+ *   W_bf16      device, bf16 bit patterns [rows, cols], 16-byte aligned; read only.
+ *   rows, cols  >= 1; cols % group == 0; rows*cols < 2^40.
+ *   group       32, 64, 128 or 256 (the paper uses 128).
+ *   n_stages    1..4: stage 0 is the 2-bit base, stages 1..n_stages-1 are
+ *               2-bit residual stages.
+ *   out_codes   host array of n_stages device pointers, each to
+ *               rrq_codes_bytes(rows, cols) bytes, 8-byte aligned.
+ *   out_scales, out_zeros
+ *               host arrays of n_stages device pointers, each to
+ *               rrq_meta_count(rows, cols, group) floats, 4-byte aligned.
+ * No output may overlap another output or W.  One fused kernel computes all
+ * stages; the running residual never leaves registers. */
+rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int group,
+                        int n_stages, uint8_t* const out_codes[],
+                        float* const out_scales[], float* const out_zeros[],
+                        rrq_stream_t stream);
+
+/* Prefix reconstruction with the first k stages (Eq. 8; Appendix C):
+ * k = 1, 2, 3, 4 give the 2-, 4-, 6-, 8-bit operating points.
+ *   codes, scales, zeros  host arrays of >= k device pointers laid out as
+ *                         written by rrq_quantize (8-, 4-, 4-byte aligned).
+ *   rows, cols, group     as given to rrq_quantize.
+ *   k                     1..4.
+ *   out_bf16              device, bf16 bit patterns [rows, cols], 16-byte
+ *                         aligned, not overlapping any input. */
+rrq_status rrq_reconstruct(const uint8_t* const codes[], const float* const scales[],
+                           const float* const zeros[], int64_t rows, int64_t cols,
+                           int group, int k, uint16_t* out_bf16, rrq_stream_t stream);
+
+/* Bytes of one stage's code array: rows*cols/4 (rows*cols is a multiple of
+ * 32 for every valid shape).  0 for invalid sizes. */
+size_t rrq_codes_bytes(int64_t rows, int64_t cols);
+
+/* Number of groups = entries of one stage's scale (and zero) array:
+ * rows*cols/group.  0 for invalid sizes. */
+size_t rrq_meta_count(int64_t rows, int64_t cols, int group);
+
+/* Total package bytes for n_stages stages: n_stages * (codes + 8 * groups). */
+size_t rrq_package_bytes(int64_t rows, int64_t cols, int group, int n_stages);
+
+/* Synchronizes `stream`, then reads and clears the current device's status
+ * word.  Returns RRQ_ERR_TIMEOUT if a kernel on this device gave up on a
+ * bounded wait since the last call (its outputs are then incomplete),
+ * RRQ_ERR_CUDA if the synchronization failed, RRQ_OK otherwise. */
+rrq_status rrq_get_device_status(rrq_stream_t stream);
+
+/* Longest time a kernel waits for one of its own bulk copies before it
+ * records RRQ_ERR_TIMEOUT and returns (default 1,000,000 us).  0 makes every
+ * such wait give up at once; tests use it to exercise the error path.  The
+ * setting is process-wide and applies to later launches. */
+void rrq_set_wait_limit_us(uint32_t microseconds);
+
+/* Test hook, process-wide: RRQ_DEBUG_FORCE_EXACT makes rrq_quantize take the
+ * per-element IEEE-division path for every group instead of only for the
+ * groups its check sends there; results are identical either way. */
+#define RRQ_DEBUG_FORCE_EXACT 1u
+void rrq_set_debug_flags(uint32_t flags);
+
+/* Human-readable name of a status code (static storage). */
+const char* rrq_status_string(rrq_status status);
+
+/* The cudaError_t (as int) behind the calling thread's last RRQ_ERR_CUDA. */
+int rrq_last_cuda_error(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* RRQ_H */

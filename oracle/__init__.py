@@ -1,0 +1,160 @@
+"""RRQ CPU oracle: TEST INFRASTRUCTURE ONLY.
+
+Only the tests, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline
+leg (and its ``--impl reference`` arm) may import this package.  The product
+path -- the CUDA library under ``paper_2608_04048_gb300`` -- never imports it,
+and the two share no code.
+
+This module compiles ``rrq_oracle.c`` with gcc (``-O2 -ffp-contract=off``, no
+fast-math) and exposes it to numpy through ctypes.  The arithmetic itself lives
+in the C file, which cites the paper's equations step by step (Section 3.1
+Eq. 1-3, Section 3.2 Eq. 4-8, Algorithm 1).
+
+Every function here is pinned by ``tests/test_oracle_pins.py`` (hand-worked
+groups, brute-force nearest level, invariants) and
+``tests/test_oracle_mutants.py`` (planted mistakes fail the pins).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import tempfile
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "rrq_oracle.c")
+_HDR = os.path.join(_HERE, "rrq_oracle.h")
+_BUILD_DIR = os.path.join(_HERE, "_build")
+LIB_PATH = os.path.join(_BUILD_DIR, "liboracle_rrq.so")
+
+CFLAGS = ["-O2", "-std=c11", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+
+
+def compile_oracle(src: str = _SRC, out: str = LIB_PATH, extra_flags=()) -> str:
+    """Compile an oracle source file into a shared library (atomic replace)."""
+    os.makedirs(os.path.dirname(out), exist_ok=True)
+    fd, tmp = tempfile.mkstemp(suffix=".so", dir=os.path.dirname(out))
+    os.close(fd)
+    cmd = ["gcc", *CFLAGS, *extra_flags, "-I", _HERE, "-o", tmp, src, "-lm"]
+    try:
+        subprocess.run(cmd, check=True, capture_output=True, text=True)
+    except subprocess.CalledProcessError as e:  # pragma: no cover - build failure
+        os.unlink(tmp)
+        raise RuntimeError(f"oracle build failed: {' '.join(cmd)}\n{e.stderr}") from e
+    os.replace(tmp, out)
+    return out
+
+
+def build() -> str:
+    """Build the oracle library if it is missing or older than its sources."""
+    if os.path.exists(LIB_PATH):
+        t = os.path.getmtime(LIB_PATH)
+        if t >= os.path.getmtime(_SRC) and t >= os.path.getmtime(_HDR):
+            return LIB_PATH
+    return compile_oracle()
+
+
+_u8p = ctypes.POINTER(ctypes.c_uint8)
+_f32p = ctypes.POINTER(ctypes.c_float)
+_u16p = ctypes.POINTER(ctypes.c_uint16)
+
+
+class Oracle:
+    """ctypes view of one compiled oracle library (the committed one, or a
+    test's mutated copy)."""
+
+    def __init__(self, lib_path: str):
+        lib = ctypes.CDLL(lib_path)
+        lib.rrq_oracle_quantize_group.argtypes = [
+            _f32p, ctypes.c_int, ctypes.c_int, _u8p, _f32p, _f32p, _f32p]
+        lib.rrq_oracle_quantize_group.restype = ctypes.c_int
+        lib.rrq_oracle_quantize.argtypes = [
+            _u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int,
+            ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p)]
+        lib.rrq_oracle_quantize.restype = ctypes.c_int
+        lib.rrq_oracle_reconstruct.argtypes = [
+            ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p),
+            ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _u16p]
+        lib.rrq_oracle_reconstruct.restype = ctypes.c_int
+        lib.rrq_oracle_f32_to_bf16.argtypes = [ctypes.c_float]
+        lib.rrq_oracle_f32_to_bf16.restype = ctypes.c_uint16
+        self.lib = lib
+
+    # -- one group, float input, unpacked codes --------------------------------
+    def quantize_group(self, x, n_stages: int = 4):
+        """Returns (Q[n_stages, g] uint8, scale[n_stages] f32, zero[n_stages] f32,
+        resid[n_stages, g] f32) for one group of float32 values."""
+        x = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+        g = x.size
+        Q = np.zeros((n_stages, g), np.uint8)
+        s = np.zeros(n_stages, np.float32)
+        z = np.zeros(n_stages, np.float32)
+        r = np.zeros((n_stages, g), np.float32)
+        rc = self.lib.rrq_oracle_quantize_group(
+            x.ctypes.data_as(_f32p), g, n_stages, Q.ctypes.data_as(_u8p),
+            s.ctypes.data_as(_f32p), z.ctypes.data_as(_f32p), r.ctypes.data_as(_f32p))
+        if rc != 0:
+            raise ValueError("oracle rejected the group")
+        return Q, s, z, r
+
+    # -- a bf16 matrix, packed package -----------------------------------------
+    def quantize(self, W_bits, group: int = 128, n_stages: int = 4):
+        """W_bits: uint16 array [rows, cols] of bf16 bit patterns.
+        Returns (codes, scales, zeros): lists of n_stages numpy arrays."""
+        W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+        rows, cols = W_bits.shape
+        n = rows * cols
+        codes = [np.zeros((n + 3) // 4, np.uint8) for _ in range(n_stages)]
+        scales = [np.zeros(n // group, np.float32) for _ in range(n_stages)]
+        zeros = [np.zeros(n // group, np.float32) for _ in range(n_stages)]
+        cp = (_u8p * n_stages)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (_f32p * n_stages)(*[a.ctypes.data_as(_f32p) for a in scales])
+        zp = (_f32p * n_stages)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        rc = self.lib.rrq_oracle_quantize(W_bits.ctypes.data_as(_u16p), rows, cols,
+                                          group, n_stages, cp, sp, zp)
+        if rc != 0:
+            raise ValueError("oracle rejected the matrix")
+        return codes, scales, zeros
+
+    def reconstruct(self, codes, scales, zeros, rows: int, cols: int, group: int, k: int):
+        """bf16 bit patterns [rows, cols] of the prefix-k reconstruction."""
+        codes = [np.ascontiguousarray(c, dtype=np.uint8) for c in codes[:k]]
+        scales = [np.ascontiguousarray(a, dtype=np.float32) for a in scales[:k]]
+        zeros = [np.ascontiguousarray(a, dtype=np.float32) for a in zeros[:k]]
+        out = np.zeros((rows, cols), np.uint16)
+        cp = (_u8p * k)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in scales])
+        zp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        rc = self.lib.rrq_oracle_reconstruct(cp, sp, zp, rows, cols, group, k,
+                                             out.ctypes.data_as(_u16p))
+        if rc != 0:
+            raise ValueError("oracle rejected the reconstruction")
+        return out
+
+    def f32_to_bf16(self, f: float) -> int:
+        return int(self.lib.rrq_oracle_f32_to_bf16(ctypes.c_float(f)))
+
+
+_default = None
+
+
+def load() -> Oracle:
+    """The committed oracle, built on first use."""
+    global _default
+    if _default is None:
+        _default = Oracle(build())
+    return _default
+
+
+def quantize_group(x, n_stages: int = 4):
+    return load().quantize_group(x, n_stages)
+
+
+def quantize(W_bits, group: int = 128, n_stages: int = 4):
+    return load().quantize(W_bits, group, n_stages)
+
+
+def reconstruct(codes, scales, zeros, rows, cols, group, k):
+    return load().reconstruct(codes, scales, zeros, rows, cols, group, k)

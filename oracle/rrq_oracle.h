@@ -1,0 +1,59 @@
+/*
+ * Plain CPU oracle for Recurrent Residual Quantization (RRQ) with 2-bit
+ * round-to-nearest stages: TEST INFRASTRUCTURE ONLY.
+ *
+ * Only the test suite, the smoke check and the benchmark's CPU-baseline leg
+ * may load this library.  The product path (the CUDA library) never calls it
+ * and shares no code, header, table or helper with it.
+ *
+ * The arithmetic follows the paper's representation statement (Section 3.1,
+ * Eq. 1-3), the recursion (Section 3.2, Eq. 4-7), Algorithm 1 (build without
+ * a base checkpoint) and the prefix reconstruction (Eq. 8), in IEEE-754
+ * binary32, one operation at a time, with no fused multiply-add and
+ * round-half-to-even for the code rounding.  See rrq_oracle.c for the
+ * readings taken where the paper leaves a detail open.
+ */
+#ifndef RRQ_ORACLE_H
+#define RRQ_ORACLE_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* One group of g float values through n_stages 2-bit stages.
+ *   x      [g]               input values (any finite binary32)
+ *   Q      [n_stages][g]     unpacked codes 0..3 (output)
+ *   scale  [n_stages]        per-stage scale s_k (output)
+ *   zero   [n_stages]        per-stage offset m_k = group minimum (output)
+ *   resid  [n_stages][g]     residual after each stage (output, may be NULL)
+ * Returns 0, or -1 on a bad argument (g < 1, n_stages < 1). */
+int rrq_oracle_quantize_group(const float* x, int g, int n_stages, uint8_t* Q,
+                              float* scale, float* zero, float* resid);
+
+/* A row-major bf16 matrix [rows, cols] (raw bf16 bit patterns), groups of
+ * `group` consecutive columns.  Outputs, for each stage k < n_stages:
+ *   codes[k]  uint8 [rows*cols/4]: element c at byte c/4, bits 2*(c%4)..+1
+ *   scales[k] float [rows*cols/group]
+ *   zeros[k]  float [rows*cols/group]
+ * Returns 0, or -1 on a bad argument (cols % group != 0, group < 1, ...). */
+int rrq_oracle_quantize(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                        int n_stages, uint8_t* const* codes, float* const* scales,
+                        float* const* zeros);
+
+/* Prefix reconstruction with the first k stages (k = 1 is the 2-bit base),
+ * written as bf16 bit patterns [rows*cols].  Returns 0 or -1. */
+int rrq_oracle_reconstruct(const uint8_t* const* codes, const float* const* scales,
+                           const float* const* zeros, int64_t rows, int64_t cols,
+                           int group, int k, uint16_t* out);
+
+/* The two scalar conversions the oracle uses, exported for tests. */
+float rrq_oracle_bf16_to_f32(uint16_t h);
+uint16_t rrq_oracle_f32_to_bf16(float f);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif

@@ -1,0 +1,52 @@
+"""Planted mistakes in a copy of the oracle must each break at least one pin.
+
+Each mutant edits one plausible step of rrq_oracle.c (a rounding rule, a
+dropped term, a wrong sign, a transposed operand, a wrong index), compiles the
+copy on the CPU and runs the pins of tests/_pins.py against it.  This shows
+that the pins, not the oracle agreeing with itself, are what fix its
+arithmetic."""
+import os
+
+import pytest
+
+import oracle
+import _pins
+
+SRC = os.path.join(os.path.dirname(oracle.__file__), "rrq_oracle.c")
+
+MUTANTS = {
+    "ties_round_up": ("return (fmodf(f, 2.0f) == 0.0f) ? f : f + 1.0f;", "return f + 1.0f;"),
+    "ties_round_down": ("return (fmodf(f, 2.0f) == 0.0f) ? f : f + 1.0f;", "return f;"),
+    "four_steps_not_three": ("float s = range / 3.0f;", "float s = range / 4.0f;"),
+    "level_drops_offset": ("level[q] = lo + qs;", "level[q] = qs;"),
+    "residual_sign": ("v[j] = v[j] - level[code];", "v[j] = v[j] + level[code];"),
+    "transposed_difference": ("float d = v[j] - lo;", "float d = lo - v[j];"),
+    "zero_sign_order_ignored": ("if (a == b && signbit(a) && !signbit(b)) return 1;", ""),
+    "no_clamp": ("if (code > 3) code = 3;", "if (code > 4) code = 4;"),
+    "packing_bit_order": ("codes[k][c / 4] |= (uint8_t)(Q[(size_t)k * group + j] << (2 * (c % 4)));",
+                          "codes[k][c / 4] |= (uint8_t)(Q[(size_t)k * group + j] << (2 * (3 - c % 4)));"),
+    "recon_drops_base": ("acc = (i == 0) ? value : acc + value;", "acc = (i == 0) ? 0.0f : acc + value;"),
+    "recon_bf16_truncates": ("u += 0x7fffu + ((u >> 16) & 1u);", ""),
+    "max_is_min": ("if (before(hi, v[j])) hi = v[j];", "if (before(v[j], hi)) hi = v[j];"),
+    "range_of_input_not_residual": ("if (before(v[j], lo)) lo = v[j];\n      if (before(hi, v[j])) hi = v[j];",
+                                    "if (before(x[j], lo)) lo = x[j];\n      if (before(hi, x[j])) hi = x[j];"),
+    "scale_rounds_range_twice": ("float range = hi - lo;", "float range = (float)(double)(hi - lo) * 1.0000001f;"),
+    "level_from_code_minus_one": ("float qs = (float)q * s;\n      level[q]", "float qs = (float)(q > 0 ? q - 1 : 0) * s;\n      level[q]"),
+}
+
+
+@pytest.fixture(scope="module")
+def source():
+    with open(SRC) as f:
+        return f.read()
+
+
+@pytest.mark.parametrize("name", sorted(MUTANTS))
+def test_mutant_is_caught(name, source, tmp_path):
+    old, new = MUTANTS[name]
+    assert source.count(old) == 1, f"mutation site for {name} not found exactly once"
+    src = tmp_path / "rrq_oracle.c"
+    src.write_text(source.replace(old, new))
+    lib = oracle.compile_oracle(str(src), str(tmp_path / "libmutant.so"))
+    fails = _pins.all_failures(oracle.Oracle(lib))
+    assert fails, f"mutant {name} passed every pin"
