@@ -1,0 +1,168 @@
+"""Thin ctypes binding of the RRQ C ABI (include/rrq.h).
+
+Argument marshalling only: every step of quantization and reconstruction runs
+in the CUDA kernels of librrq.so.  PyTorch supplies device memory and the
+current CUDA stream.  There is no CPU fallback: if the library is missing or
+the tensors are not on a CUDA device, the call raises.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from dataclasses import dataclass
+
+import torch
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_LIB = None
+
+_STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
+           3: "RRQ_ERR_MISALIGNED", 4: "RRQ_ERR_CUDA", 5: "RRQ_ERR_TIMEOUT"}
+
+#: symbols declared in include/rrq.h
+EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_codes_bytes", "rrq_meta_count",
+           "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
+           "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
+
+
+class RRQError(RuntimeError):
+    def __init__(self, status: int, what: str = ""):
+        self.status = status
+        msg = _STATUS.get(status, f"status {status}")
+        if status == 4 and _LIB is not None:
+            msg += f" (cudaError {_LIB.rrq_last_cuda_error()})"
+        super().__init__(f"{what}: {msg}" if what else msg)
+
+
+def library_path() -> str:
+    return os.path.join(_HERE, "_build", "librrq.so")
+
+
+def load_library():
+    """Load librrq.so (built in-tree by paper_2608_04048_gb300.build)."""
+    global _LIB
+    if _LIB is not None:
+        return _LIB
+    path = library_path()
+    if not os.path.exists(path):
+        raise RuntimeError(f"{path} is missing: build it with "
+                           "`python -m paper_2608_04048_gb300.build` (or __graft_entry__.build())")
+    lib = ctypes.CDLL(path)
+    vp, i64, i32, u32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int, ctypes.c_uint32
+    ptr_array = ctypes.POINTER(ctypes.c_void_p)
+    lib.rrq_quantize.argtypes = [vp, i64, i64, i32, i32, ptr_array, ptr_array, ptr_array, vp]
+    lib.rrq_quantize.restype = i32
+    lib.rrq_reconstruct.argtypes = [ptr_array, ptr_array, ptr_array, i64, i64, i32, i32, vp, vp]
+    lib.rrq_reconstruct.restype = i32
+    lib.rrq_codes_bytes.argtypes = [i64, i64]
+    lib.rrq_codes_bytes.restype = ctypes.c_size_t
+    lib.rrq_meta_count.argtypes = [i64, i64, i32]
+    lib.rrq_meta_count.restype = ctypes.c_size_t
+    lib.rrq_package_bytes.argtypes = [i64, i64, i32, i32]
+    lib.rrq_package_bytes.restype = ctypes.c_size_t
+    lib.rrq_get_device_status.argtypes = [vp]
+    lib.rrq_get_device_status.restype = i32
+    lib.rrq_set_wait_limit_us.argtypes = [u32]
+    lib.rrq_set_wait_limit_us.restype = None
+    lib.rrq_set_debug_flags.argtypes = [u32]
+    lib.rrq_set_debug_flags.restype = None
+    lib.rrq_status_string.argtypes = [i32]
+    lib.rrq_status_string.restype = ctypes.c_char_p
+    lib.rrq_last_cuda_error.argtypes = []
+    lib.rrq_last_cuda_error.restype = i32
+    _LIB = lib
+    return lib
+
+
+def _stream_handle(stream) -> int:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return int(stream.cuda_stream) if hasattr(stream, "cuda_stream") else int(stream)
+
+
+def _ptrs(tensors, n) -> ctypes.Array:
+    return (ctypes.c_void_p * n)(*[t.data_ptr() for t in tensors[:n]])
+
+
+@dataclass
+class Package:
+    """An RRQ package on the device: per stage a code array (uint8, n/4),
+    a scale array and a zero array (float32, n/group)."""
+    codes: list
+    scales: list
+    zeros: list
+    rows: int
+    cols: int
+    group: int
+    n_stages: int
+
+    @classmethod
+    def empty(cls, rows, cols, group=128, n_stages=4, device=None) -> "Package":
+        device = device or torch.device("cuda", torch.cuda.current_device())
+        n = rows * cols
+        return cls([torch.empty(n // 4, dtype=torch.uint8, device=device) for _ in range(n_stages)],
+                   [torch.empty(n // group, dtype=torch.float32, device=device) for _ in range(n_stages)],
+                   [torch.empty(n // group, dtype=torch.float32, device=device) for _ in range(n_stages)],
+                   rows, cols, group, n_stages)
+
+    def nbytes(self) -> int:
+        return sum(t.numel() * t.element_size() for t in self.codes + self.scales + self.zeros)
+
+
+def rrq_quantize(W: torch.Tensor, group: int = 128, n_stages: int = 4, out: Package | None = None,
+                 stream=None) -> Package:
+    """Build the RRQ package of a 2-D bf16 CUDA tensor (rows x cols, groups of
+    `group` consecutive columns) through the C ABI."""
+    lib = load_library()
+    if W.dtype != torch.bfloat16 or W.dim() != 2 or not W.is_cuda:
+        raise TypeError("W must be a 2-D bfloat16 CUDA tensor")
+    if not W.is_contiguous():
+        raise ValueError("W must be contiguous (row-major)")
+    rows, cols = W.shape
+    if out is None:
+        out = Package.empty(rows, cols, group, n_stages, W.device)
+    rc = lib.rrq_quantize(W.data_ptr(), rows, cols, group, n_stages, _ptrs(out.codes, n_stages),
+                          _ptrs(out.scales, n_stages), _ptrs(out.zeros, n_stages), _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_quantize")
+    return out
+
+
+def rrq_reconstruct(pkg: Package, k: int, out: torch.Tensor | None = None, stream=None) -> torch.Tensor:
+    """bf16 weights of the prefix with the first k stages (k=1..4 -> 2/4/6/8 bits)."""
+    lib = load_library()
+    if out is None:
+        out = torch.empty((pkg.rows, pkg.cols), dtype=torch.bfloat16, device=pkg.codes[0].device)
+    if out.dtype != torch.bfloat16 or not out.is_cuda or not out.is_contiguous():
+        raise TypeError("out must be a contiguous bfloat16 CUDA tensor")
+    n = min(k, len(pkg.codes)) if k >= 1 else 1
+    rc = lib.rrq_reconstruct(_ptrs(pkg.codes, n), _ptrs(pkg.scales, n), _ptrs(pkg.zeros, n),
+                             pkg.rows, pkg.cols, pkg.group, k, out.data_ptr(), _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_reconstruct")
+    return out
+
+
+def rrq_codes_bytes(rows: int, cols: int) -> int:
+    return int(load_library().rrq_codes_bytes(rows, cols))
+
+
+def rrq_meta_count(rows: int, cols: int, group: int) -> int:
+    return int(load_library().rrq_meta_count(rows, cols, group))
+
+
+def rrq_package_bytes(rows: int, cols: int, group: int, n_stages: int) -> int:
+    return int(load_library().rrq_package_bytes(rows, cols, group, n_stages))
+
+
+def rrq_get_device_status(stream=None) -> int:
+    """Synchronizes the stream; returns 0 (RRQ_OK) or a status code."""
+    return int(load_library().rrq_get_device_status(_stream_handle(stream)))
+
+
+def rrq_set_wait_limit_us(us: int) -> None:
+    load_library().rrq_set_wait_limit_us(us)
+
+
+def rrq_set_debug_flags(flags: int) -> None:
+    load_library().rrq_set_debug_flags(flags)

@@ -1,0 +1,97 @@
+"""The C-ABI library loads and exports every function include/rrq.h declares;
+argument checks that run before any CUDA call reject bad input (CPU only,
+nothing is computed)."""
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2608_04048_gb300 import binding, build
+
+HEADER = os.path.join(os.path.dirname(os.path.dirname(os.path.abspath(__file__))), "include", "rrq.h")
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(rrq_[a-z_0-9]+)\s*\(", text)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    build.build()
+    return binding.load_library()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    assert "rrq_quantize" in names and "rrq_reconstruct" in names
+    assert set(names) == set(binding.EXPORTS)
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for name in declared_functions():
+        assert hasattr(lib, name), name
+        assert ctypes.cast(getattr(lib, name), ctypes.c_void_p).value
+
+
+def test_size_helpers(lib):
+    assert binding.rrq_codes_bytes(4096, 4096) == 4096 * 4096 // 4
+    assert binding.rrq_meta_count(4096, 4096, 128) == 4096 * 4096 // 128
+    assert binding.rrq_package_bytes(4096, 4096, 128, 4) == 4 * (4096 * 1024 + 8 * 4096 * 32)
+    assert binding.rrq_meta_count(4, 100, 128) == 0
+    assert binding.rrq_codes_bytes(0, 128) == 0
+    assert binding.rrq_package_bytes(4, 128, 128, 5) == 0
+
+
+def test_status_strings(lib):
+    for code in range(6):
+        assert lib.rrq_status_string(code).startswith(b"RRQ_")
+
+
+def _call_quantize(lib, W, rows, cols, group, n_stages, codes, scales, zeros):
+    arr = lambda xs: (ctypes.c_void_p * len(xs))(*xs)
+    return lib.rrq_quantize(W, rows, cols, group, n_stages, arr(codes), arr(scales), arr(zeros), None)
+
+
+def test_quantize_argument_checks_run_before_cuda(lib):
+    base = 1 << 20
+    ok = dict(W=base, rows=4, cols=256, group=128, n_stages=2,
+              codes=[base + 0x10000, base + 0x20000], scales=[base + 0x30000, base + 0x40000],
+              zeros=[base + 0x50000, base + 0x60000])
+
+    def call(**kw):
+        a = dict(ok)
+        a.update(kw)
+        return _call_quantize(lib, a["W"], a["rows"], a["cols"], a["group"], a["n_stages"],
+                              a["codes"], a["scales"], a["zeros"])
+
+    assert call(W=None) == 1
+    assert call(rows=0) == 1
+    assert call(n_stages=0) == 1
+    assert call(n_stages=5) == 1
+    assert call(group=48) == 2
+    assert call(group=512) == 2
+    assert call(cols=192) == 1                      # cols % group != 0
+    assert call(W=base + 8) == 3                    # bf16 input must be 16-byte aligned
+    assert call(codes=[base + 0x10004, base + 0x20000]) == 3
+    assert call(scales=[base + 0x30002, base + 0x40000]) == 3
+    assert call(codes=[base + 0x10000, base + 0x10040]) == 1   # overlapping outputs
+    assert call(zeros=[base + 0x50000, base + 0x100]) == 1     # output overlaps W
+
+
+def test_reconstruct_argument_checks_run_before_cuda(lib):
+    base = 1 << 20
+    arr = lambda xs: (ctypes.c_void_p * len(xs))(*xs)
+    codes, scales, zeros = arr([base]), arr([base + 0x10000]), arr([base + 0x20000])
+    assert lib.rrq_reconstruct(codes, scales, zeros, 4, 256, 128, 0, base + 0x40000, None) == 1
+    assert lib.rrq_reconstruct(codes, scales, zeros, 4, 256, 100, 1, base + 0x40000, None) == 2
+    assert lib.rrq_reconstruct(codes, scales, zeros, 4, 256, 128, 1, base + 0x40008, None) == 3
+    assert lib.rrq_reconstruct(codes, scales, zeros, 4, 256, 128, 1, base + 0x80, None) == 1
+
+
+def test_binding_refuses_cpu_tensors(lib):
+    import torch
+    with pytest.raises(TypeError):
+        binding.rrq_quantize(torch.zeros(4, 128, dtype=torch.bfloat16))
