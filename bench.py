@@ -1,0 +1,483 @@
+"""Benchmark of the RRQ hot path on GB300: package construction (rrq_quantize)
+and prefix reconstruction (rrq_reconstruct, k = 1..4) over a synthetic
+Qwen3-8B-shaped linear stack (36 layers x {q,k,v,o,gate,up,down}, 6.95e9
+bf16 weights, Student-t(3) weights with 0.1% +-20 sigma outliers per row,
+group 128, four 2-bit stages).
+
+One step = rrq_quantize of every matrix of the stack, then rrq_reconstruct of
+every matrix at k = 1, 2, 3, 4.  The metric is bf16 weight bytes of the stack
+processed per second of step time (GB/s).  Inputs (13.9 GB) are far larger
+than L2, so no L2 flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+Under torchrun every rank builds and processes its own stack (independent
+matrices, no data-path collective): weak scaling, value = all ranks' bytes /
+max over ranks of the timed region.  Rank 0 prints one JSON line.
+
+--impl reference times the CPU oracle (the plain C implementation in oracle/,
+as it stands, single-threaded) on a bounded sample of the same workload; it is
+the slow reference arm, not a target.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import threading
+import time
+
+import numpy as np
+import torch
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+GROUP = 128
+STAGES = 4
+KS = (1, 2, 3, 4)
+WORKLOAD = "qwen3_8b_stack"
+METRIC = "RRQ package construction GB/s of bf16 weights and % of HBM peak; s per 8B-shaped stack"
+
+
+def alg_bytes_quantize(n: int, g: int = GROUP, S: int = STAGES) -> float:
+    """Algorithmic bytes of one rrq_quantize over n weights: bf16 read once,
+    S stages of 2-bit codes, fp32 scale and zero per group."""
+    return 2.0 * n + S * (n / 4.0 + 8.0 * n / g)
+
+
+def alg_bytes_reconstruct(n: int, k: int, g: int = GROUP) -> float:
+    """Algorithmic bytes of one rrq_reconstruct at prefix k: k code planes and
+    metadata read, bf16 written."""
+    return 2.0 * n + k * (n / 4.0 + 8.0 * n / g)
+
+
+def measured_peaks() -> dict:
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": float(d["hbm_gbs"]), "source": "measured"}
+    return {"hbm_gbs": 6800.0, "source": "fallback"}
+
+
+# ---------------------------------------------------------------------------
+# clocks during the timed region
+# ---------------------------------------------------------------------------
+class ClockSampler:
+    QUERY = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+             "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+             "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.device_index = device_index
+        self.proc = None
+        self.path = None
+
+    def __enter__(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.device_index}", f"--query-gpu={self.QUERY}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except (FileNotFoundError, OSError):
+            self.proc = None
+        time.sleep(0.3)
+        return self
+
+    def __exit__(self, *exc):
+        if self.proc is not None:
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+
+    def summary(self) -> dict:
+        if self.proc is None or not self.path:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    smax.append(float(parts[2]))
+                except ValueError:
+                    continue
+                for name, val in zip(names, parts[5:9]):
+                    if val.lower().startswith("active"):
+                        reasons.add(name)
+        os.unlink(self.path)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        # samples under load: the upper half of the clock distribution is
+        # not needed; report the median of all samples taken in the region
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(smax),
+                "samples": len(sm), "reasons": sorted(reasons)}
+
+
+# ---------------------------------------------------------------------------
+# distributed helpers (one process per GPU, launched by torchrun)
+# ---------------------------------------------------------------------------
+def dist_env():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def shard_seed_offset(rank: int) -> int:
+    """Each rank builds its own stack of independent matrices: seeds shifted
+    by a per-rank offset far above the stack's own seed range."""
+    return 1_000_003 * rank
+
+
+def max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch.distributed as dist
+    t = torch.tensor([x], dtype=torch.float64, device="cuda" if dist.get_backend() == "nccl" else "cpu")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def barrier(world: int):
+    if world > 1:
+        import torch.distributed as dist
+        dist.barrier()
+
+
+# ---------------------------------------------------------------------------
+# the GPU arm
+# ---------------------------------------------------------------------------
+def build_stack(specs, device, seed_offset: int):
+    from paper_2608_04048_gb300 import binding, workloads
+    mats, pkgs = [], []
+    for sp in specs:
+        W = workloads.generate(sp.rows, sp.cols, sp.seed + seed_offset, sp.dist, device)
+        mats.append(W)
+        pkgs.append(binding.Package.empty(sp.rows, sp.cols, GROUP, STAGES, device))
+    return mats, pkgs
+
+
+def run_gpu(args, world, rank, local) -> dict | None:
+    from paper_2608_04048_gb300 import binding, build, workloads
+    build.build()
+    torch.cuda.set_device(local)
+    device = torch.device("cuda", local)
+    specs = workloads.config_matrices(args.workload)
+    n_total = sum(sp.numel for sp in specs)
+    mats, pkgs = build_stack(specs, device, shard_seed_offset(rank))
+    max_n = max(sp.numel for sp in specs)
+    out = torch.empty(max_n, dtype=torch.bfloat16, device=device)
+    outs = [out[:sp.numel].view(sp.rows, sp.cols) for sp in specs]
+    stream = torch.cuda.current_stream(device)
+    binding.rrq_get_device_status()
+
+    def quantize_all():
+        for W, pkg in zip(mats, pkgs):
+            binding.rrq_quantize(W, GROUP, STAGES, out=pkg, stream=stream)
+
+    def reconstruct_all():
+        for k in KS:
+            for pkg, o in zip(pkgs, outs):
+                binding.rrq_reconstruct(pkg, k, out=o, stream=stream)
+
+    for _ in range(args.warmup):
+        quantize_all()
+        reconstruct_all()
+    torch.cuda.synchronize()
+    if binding.rrq_get_device_status() != 0:
+        raise RuntimeError("a kernel reported a timeout during warm-up")
+
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
+           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    barrier(world)
+    torch.cuda.synchronize()
+    with ClockSampler(local) as clocks:
+        t0 = torch.cuda.Event(enable_timing=True)
+        t1 = torch.cuda.Event(enable_timing=True)
+        t0.record(stream)
+        for a, b, c in ev:
+            a.record(stream)
+            quantize_all()
+            b.record(stream)
+            reconstruct_all()
+            c.record(stream)
+        t1.record(stream)
+        torch.cuda.synchronize()
+    barrier(world)
+    status = binding.rrq_get_device_status()
+    if status != 0:
+        raise RuntimeError(f"kernel status {status} in the timed region")
+    elapsed_ms = t0.elapsed_time(t1)
+    q_ms = [a.elapsed_time(b) for a, b, _ in ev]
+    r_ms = [b.elapsed_time(c) for _, b, c in ev]
+    elapsed_ms = max_over_ranks(elapsed_ms, world)
+
+    e2e = run_e2e(args, mats, pkgs, outs, specs, stream, world) if not args.no_e2e else None
+    if rank != 0:
+        return None
+
+    peaks = measured_peaks()
+    step_s = elapsed_ms / 1e3 / args.steps
+    bytes_bf16 = 2.0 * n_total
+    value = world * bytes_bf16 / step_s / 1e9
+    q_s = statistics.mean(q_ms) / 1e3
+    r_s = statistics.mean(r_ms) / 1e3
+    q_alg = sum(alg_bytes_quantize(sp.numel) for sp in specs)
+    r_alg = sum(alg_bytes_reconstruct(sp.numel, k) for sp in specs for k in KS)
+    q_gbs = q_alg / q_s / 1e9
+    r_gbs = r_alg / r_s / 1e9
+    dominant = "rrq_reconstruct" if r_s > q_s else "rrq_quantize"
+    achieved = r_gbs if dominant == "rrq_reconstruct" else q_gbs
+    launches = len(specs) * (1 + len(KS))
+    traffic = recorded_traffic(dominant, q_alg / len(specs), r_alg / (len(specs) * len(KS)))
+    line = {
+        "metric": METRIC,
+        "value": round(value, 2),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(elapsed_ms / args.steps, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {
+            "workload": f"{args.workload}: 36 layers x (q 4096x4096, k/v 1024x4096, o 4096x4096, "
+                        "gate/up 12288x4096, down 4096x12288), bf16, Student-t(3) std 0.02 + 0.1% +-0.4 "
+                        "outliers per row, group 128 along the input dim, 4 x 2-bit stages",
+            "step": "rrq_quantize on all 252 matrices, then rrq_reconstruct on all 252 at k=1,2,3,4",
+            "weights_per_rank": n_total,
+            "l2": "inputs 13.9 GB per rank, far larger than the 126 MB L2; no flush",
+            "parallelism": f"{world} independent rank(s), one stack each",
+        },
+        "breakdown": {
+            "quantize_s_per_stack": round(q_s, 6),
+            "quantize_alg_gbs": round(q_gbs, 1),
+            "quantize_bf16_in_gbs": round(bytes_bf16 / q_s / 1e9, 1),
+            "quantize_weights_per_s": round(n_total / q_s, 1),
+            "reconstruct_k1to4_s": round(r_s, 6),
+            "reconstruct_alg_gbs": round(r_gbs, 1),
+            "quantize_frac_of_measured_hbm": round(q_gbs / peaks["hbm_gbs"], 4),
+            "reconstruct_frac_of_measured_hbm": round(r_gbs / peaks["hbm_gbs"], 4),
+            "quantize_frac_of_nominal_8tbs": round(q_gbs / 8000.0, 4),
+            "paper_context_s": {"full_all_rtn_package_qwen3_8b_a100": 1293, "four_rtn_passes_a100": 412},
+        },
+        "roofline": {
+            "kernel": dominant,
+            "bound": "hbm",
+            "achieved": round(achieved, 1),
+            "peak": peaks["hbm_gbs"],
+            "peak_source": f"{peaks['source']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+            "unit": "GB/s",
+            "frac": round(achieved / peaks["hbm_gbs"], 4),
+            "traffic": traffic,
+        },
+        "clocks": clocks.summary(),
+        "gpu_launches": launches * args.steps,
+        "e2e": e2e,
+    }
+    return line
+
+
+def recorded_traffic(kernel: str, q_bytes_per_launch: float, r_bytes_per_launch: float):
+    """DRAM bytes per launch of `kernel` from the committed ncu summary
+    (profiles/traffic.json), scaled to this workload's average launch by the
+    ratio of DRAM to algorithmic bytes measured there; None when the kernel
+    source changed since the capture."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        rec = json.load(f)
+    entry = rec.get(kernel)
+    if not entry or entry.get("source_sha256") != kernel_source_hash():
+        return None
+    per_alg = entry["dram_bytes"] / entry["alg_bytes"]
+    alg = q_bytes_per_launch if kernel == "rrq_quantize" else r_bytes_per_launch
+    return round(per_alg * alg)
+
+
+def kernel_source_hash() -> str:
+    h = hashlib.sha256()
+    csrc = os.path.join(ROOT, "paper_2608_04048_gb300", "csrc")
+    for name in sorted(os.listdir(csrc)):
+        with open(os.path.join(csrc, name), "rb") as f:
+            h.update(name.encode())
+            h.update(f.read())
+    return h.hexdigest()
+
+
+def run_e2e(args, mats, pkgs, outs, specs, stream, world) -> dict:
+    """Same metric through the public API with host buffers: every step copies
+    each matrix from pinned host memory to the device, builds its package,
+    copies the package back, reconstructs at k=1..4 and copies each result
+    back to a pinned host buffer, all inside the timed region."""
+    from paper_2608_04048_gb300 import binding
+    def pinned_like(t):
+        h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+        h.copy_(t)
+        return h
+    host_W = [pinned_like(W) for W in mats]
+    host_pkg = [[torch.empty(t.shape, dtype=t.dtype, pin_memory=True) for t in p.codes + p.scales + p.zeros]
+                for p in pkgs]
+    max_n = max(sp.numel for sp in specs)
+    host_out = torch.empty(max_n, dtype=torch.bfloat16).pin_memory()
+    h2d = sum(W.numel() * 2 for W in mats)
+    d2h = sum(t.numel() * t.element_size() for p in host_pkg for t in p) + \
+        len(KS) * sum(sp.numel * 2 for sp in specs)
+
+    def step():
+        for i, (W, pkg) in enumerate(zip(mats, pkgs)):
+            W.copy_(host_W[i], non_blocking=True)
+            binding.rrq_quantize(W, GROUP, STAGES, out=pkg, stream=stream)
+            for h, d in zip(host_pkg[i], pkg.codes + pkg.scales + pkg.zeros):
+                h.copy_(d, non_blocking=True)
+        for k in KS:
+            for i, (pkg, o) in enumerate(zip(pkgs, outs)):
+                binding.rrq_reconstruct(pkg, k, out=o, stream=stream)
+                host_out[:o.numel()].view(o.shape).copy_(o, non_blocking=True)
+    step()
+    torch.cuda.synchronize()
+    steps = max(1, args.e2e_steps)
+    barrier(world)
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        step()
+    torch.cuda.synchronize()
+    dt = max_over_ranks(time.perf_counter() - t0, world)
+    n_total = sum(sp.numel for sp in specs)
+    return {"value": round(world * 2.0 * n_total * steps / dt / 1e9, 2), "unit": "GB/s",
+            "h2d_bytes_per_step": h2d, "d2h_bytes_per_step": d2h,
+            "steps": steps, "s_per_step": round(dt / steps, 4)}
+
+
+# ---------------------------------------------------------------------------
+# CPU oracle: baseline leg and the --impl reference arm
+# ---------------------------------------------------------------------------
+def oracle_sample(seconds_target: float, seed_offset: int = 0):
+    """Times the single-threaded C oracle on whole matrices of the stack's
+    first layer (quantize plus reconstruct at k=1..4), adding matrices until
+    about `seconds_target` of CPU work; returns (bf16 bytes, seconds, names)."""
+    import oracle
+    from paper_2608_04048_gb300 import workloads
+    specs = workloads.config_matrices(WORKLOAD)
+    order = [1, 2, 0, 3, 6, 4, 5]  # k, v, q, o, down, gate, up of layer 0
+    done_bytes, spent, names = 0.0, 0.0, []
+    for i in order:
+        sp = specs[i]
+        W = workloads.generate(sp.rows, sp.cols, sp.seed + seed_offset, sp.dist, "cpu")
+        Wb = W.view(torch.int16).numpy().view(np.uint16)
+        t = time.perf_counter()
+        pkg = oracle.quantize(Wb, GROUP, STAGES)
+        for k in KS:
+            oracle.reconstruct(*pkg, sp.rows, sp.cols, GROUP, k)
+        spent += time.perf_counter() - t
+        done_bytes += 2.0 * sp.numel
+        names.append(f"{sp.name} {sp.rows}x{sp.cols}")
+        if spent >= seconds_target:
+            break
+    return done_bytes, spent, names
+
+
+def cpu_baseline(seconds_target: float) -> dict:
+    import oracle
+    oracle.build()
+    b, s, names = oracle_sample(seconds_target)
+    return {"value": round(b / s / 1e9, 5), "unit": "GB/s", "cores": 1, "kind": "oracle",
+            "sample": f"single-threaded C oracle, quantize + reconstruct k=1..4 of layer-0 matrices "
+                      f"{', '.join(names)} ({b / 2:.0f} weights, {s:.1f} s)",
+            "host_cpus": os.cpu_count()}
+
+
+def run_reference(args, world, rank):
+    if rank != 0:
+        return None
+    import oracle
+    oracle.build()
+    for _ in range(args.warmup):
+        oracle_sample(0.0)
+    total_b, total_s, names = 0.0, 0.0, None
+    for _ in range(args.steps):
+        b, s, names = oracle_sample(0.0)
+        total_b += b
+        total_s += s
+    value = total_b / total_s / 1e9
+    return {
+        "impl": "reference",
+        "metric": METRIC,
+        "value": round(value, 5),
+        "unit": "GB/s",
+        "n_gpus": world,
+        "steps": args.steps,
+        "warmup": args.warmup,
+        "ms_per_step": round(total_s / args.steps * 1e3, 3),
+        "higher_is_better": True,
+        "scaling": "weak",
+        "vs_baseline": None,
+        "dtype": "f32",
+        "data": "synthetic",
+        "config": {"workload": f"{WORKLOAD}: bounded sample of the same stack, {', '.join(names)}",
+                   "step": "oracle quantize + reconstruct k=1..4 of the sampled matrix on the host"},
+        "cpu_baseline": {"value": round(value, 5), "unit": "GB/s", "cores": 1, "kind": "oracle",
+                         "sample": f"{', '.join(names)} per step"},
+        "e2e": {"value": round(value, 5), "unit": "GB/s", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+
+
+def main(argv=None):
+    ap = argparse.ArgumentParser(description=__doc__.split("\n\n")[0])
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--e2e-steps", type=int, default=2)
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    args = ap.parse_args(argv)
+
+    world, rank, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+        backend = "nccl" if torch.cuda.is_available() else "gloo"
+        if backend == "nccl":
+            torch.cuda.set_device(local)
+        dist.init_process_group(backend=backend)
+    try:
+        if args.impl == "reference":
+            line = run_reference(args, world, rank)
+        else:
+            if not torch.cuda.is_available():
+                raise SystemExit("bench.py needs a CUDA device (use --impl reference for the CPU oracle)")
+            line = run_gpu(args, world, rank, local)
+            if line is not None:
+                line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+        if line is not None:
+            print(json.dumps(line), flush=True)
+    finally:
+        if world > 1:
+            import torch.distributed as dist
+            dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()
