@@ -101,6 +101,41 @@ rrq_status rrq_reconstruct(const uint8_t* const codes[], const float* const scal
                            const float* const zeros[], int64_t rows, int64_t cols,
                            int group, int k, uint16_t* out_bf16, rrq_stream_t stream);
 
+/* One matrix of rrq_quantize_batch: the arguments of rrq_quantize for it. */
+typedef struct {
+  const uint16_t* W_bf16;                /* device, bf16 [rows, cols], 16-byte aligned */
+  int64_t rows, cols;                    /* cols % group == 0 */
+  uint8_t* codes[RRQ_MAX_STAGES];        /* first n_stages entries used */
+  float* scales[RRQ_MAX_STAGES];
+  float* zeros[RRQ_MAX_STAGES];
+} rrq_quantize_item;
+
+/* rrq_quantize for `count` matrices (count >= 1) that share `group` and
+ * `n_stages`: the same result as count separate calls, computed by one kernel
+ * launch per 64 matrices whose warps take the chunks of all of them in turn
+ * (no launch gaps, balanced across small and large matrices).  `items` is a
+ * host array, read during the call only.  Every rule of rrq_quantize holds per
+ * matrix; in addition no output may overlap any input or output of another
+ * matrix of the batch.  The library allocates nothing: the matrix
+ * descriptors travel in the kernel parameters. */
+rrq_status rrq_quantize_batch(const rrq_quantize_item* items, int count, int group,
+                              int n_stages, rrq_stream_t stream);
+
+/* One matrix of rrq_reconstruct_batch. */
+typedef struct {
+  const uint8_t* codes[RRQ_MAX_STAGES];  /* first k entries used */
+  const float* scales[RRQ_MAX_STAGES];
+  const float* zeros[RRQ_MAX_STAGES];
+  int64_t rows, cols;
+  uint16_t* out_bf16;                    /* device, bf16 [rows, cols], 16-byte aligned */
+} rrq_reconstruct_item;
+
+/* rrq_reconstruct at prefix k for `count` matrices sharing `group`, one kernel
+ * launch per 64 matrices; outputs may not overlap any input or output of the
+ * batch. */
+rrq_status rrq_reconstruct_batch(const rrq_reconstruct_item* items, int count, int group, int k,
+                                 rrq_stream_t stream);
+
 /* Bytes of one stage's code array: rows*cols/4 (rows*cols is a multiple of
  * 32 for every valid shape).  0 for invalid sizes. */
 size_t rrq_codes_bytes(int64_t rows, int64_t cols);

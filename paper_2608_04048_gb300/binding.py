@@ -20,9 +20,27 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
            3: "RRQ_ERR_MISALIGNED", 4: "RRQ_ERR_CUDA", 5: "RRQ_ERR_TIMEOUT"}
 
 #: symbols declared in include/rrq.h
-EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_codes_bytes", "rrq_meta_count",
+EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
+           "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
            "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
+
+
+MAX_STAGES = 4
+
+
+class QuantizeItem(ctypes.Structure):
+    """rrq_quantize_item of include/rrq.h"""
+    _fields_ = [("W_bf16", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
+                ("zeros", ctypes.c_void_p * MAX_STAGES)]
+
+
+class ReconstructItem(ctypes.Structure):
+    """rrq_reconstruct_item of include/rrq.h"""
+    _fields_ = [("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
+                ("zeros", ctypes.c_void_p * MAX_STAGES), ("rows", ctypes.c_int64),
+                ("cols", ctypes.c_int64), ("out_bf16", ctypes.c_void_p)]
 
 
 class RRQError(RuntimeError):
@@ -54,6 +72,10 @@ def load_library():
     lib.rrq_quantize.restype = i32
     lib.rrq_reconstruct.argtypes = [ptr_array, ptr_array, ptr_array, i64, i64, i32, i32, vp, vp]
     lib.rrq_reconstruct.restype = i32
+    lib.rrq_quantize_batch.argtypes = [ctypes.POINTER(QuantizeItem), i32, i32, i32, vp]
+    lib.rrq_quantize_batch.restype = i32
+    lib.rrq_reconstruct_batch.argtypes = [ctypes.POINTER(ReconstructItem), i32, i32, i32, vp]
+    lib.rrq_reconstruct_batch.restype = i32
     lib.rrq_codes_bytes.argtypes = [i64, i64]
     lib.rrq_codes_bytes.restype = ctypes.c_size_t
     lib.rrq_meta_count.argtypes = [i64, i64, i32]
@@ -135,12 +157,73 @@ def rrq_reconstruct(pkg: Package, k: int, out: torch.Tensor | None = None, strea
         out = torch.empty((pkg.rows, pkg.cols), dtype=torch.bfloat16, device=pkg.codes[0].device)
     if out.dtype != torch.bfloat16 or not out.is_cuda or not out.is_contiguous():
         raise TypeError("out must be a contiguous bfloat16 CUDA tensor")
-    n = min(k, len(pkg.codes)) if k >= 1 else 1
-    rc = lib.rrq_reconstruct(_ptrs(pkg.codes, n), _ptrs(pkg.scales, n), _ptrs(pkg.zeros, n),
+    if not 1 <= k <= pkg.n_stages:
+        raise ValueError(f"k must be in 1..{pkg.n_stages}")
+    rc = lib.rrq_reconstruct(_ptrs(pkg.codes, k), _ptrs(pkg.scales, k), _ptrs(pkg.zeros, k),
                              pkg.rows, pkg.cols, pkg.group, k, out.data_ptr(), _stream_handle(stream))
     if rc != 0:
         raise RRQError(rc, "rrq_reconstruct")
     return out
+
+
+def quantize_items(mats, pkgs) -> ctypes.Array:
+    """Host array of rrq_quantize_item for matrices and their packages (build
+    once and reuse: the pointers stay valid while the tensors live)."""
+    items = (QuantizeItem * len(mats))()
+    for it, W, pkg in zip(items, mats, pkgs):
+        if W.dtype != torch.bfloat16 or W.dim() != 2 or not W.is_cuda or not W.is_contiguous():
+            raise TypeError("every W must be a contiguous 2-D bfloat16 CUDA tensor")
+        it.W_bf16 = W.data_ptr()
+        it.rows, it.cols = W.shape
+        for k in range(pkg.n_stages):
+            it.codes[k] = pkg.codes[k].data_ptr()
+            it.scales[k] = pkg.scales[k].data_ptr()
+            it.zeros[k] = pkg.zeros[k].data_ptr()
+    return items
+
+
+def reconstruct_items(pkgs, outs) -> ctypes.Array:
+    items = (ReconstructItem * len(pkgs))()
+    for it, pkg, out in zip(items, pkgs, outs):
+        if out.dtype != torch.bfloat16 or not out.is_cuda or not out.is_contiguous():
+            raise TypeError("every out must be a contiguous bfloat16 CUDA tensor")
+        for k in range(pkg.n_stages):
+            it.codes[k] = pkg.codes[k].data_ptr()
+            it.scales[k] = pkg.scales[k].data_ptr()
+            it.zeros[k] = pkg.zeros[k].data_ptr()
+        it.rows, it.cols = pkg.rows, pkg.cols
+        it.out_bf16 = out.data_ptr()
+    return items
+
+
+def rrq_quantize_batch(mats, pkgs=None, group: int = 128, n_stages: int = 4, stream=None, items=None):
+    """rrq_quantize for a list of matrices in one call (one launch per 64).
+    Returns the packages; `items` may be a prebuilt quantize_items() array."""
+    lib = load_library()
+    if pkgs is None:
+        pkgs = [Package.empty(W.shape[0], W.shape[1], group, n_stages, W.device) for W in mats]
+    if items is None:
+        items = quantize_items(mats, pkgs)
+    rc = lib.rrq_quantize_batch(items, len(items), group, n_stages, _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_quantize_batch")
+    return pkgs
+
+
+def rrq_reconstruct_batch(pkgs, k: int, outs=None, stream=None, items=None):
+    """rrq_reconstruct at prefix k for a list of packages in one call."""
+    lib = load_library()
+    if outs is None:
+        outs = [torch.empty((p.rows, p.cols), dtype=torch.bfloat16, device=p.codes[0].device) for p in pkgs]
+    if items is None:
+        items = reconstruct_items(pkgs, outs)
+    group = pkgs[0].group
+    if any(not 1 <= k <= p.n_stages for p in pkgs):
+        raise ValueError("k exceeds the stages of a package")
+    rc = lib.rrq_reconstruct_batch(items, len(items), group, k, _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_reconstruct_batch")
+    return outs
 
 
 def rrq_codes_bytes(rows: int, cols: int) -> int:

@@ -1,10 +1,12 @@
 // C ABI of the RRQ library (declared in include/rrq.h): argument checks,
 // per-device set-up and kernel launches.  Every check runs before anything is
 // launched, so a rejected call has no effect on the device.
+#include <algorithm>
 #include <atomic>
 #include <cstdint>
 #include <cstring>
 #include <mutex>
+#include <vector>
 
 #include <cuda_runtime.h>
 
@@ -67,21 +69,206 @@ bool shape_ok(int64_t rows, int64_t cols) {
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
-// Device (or managed) memory that the current device can address.
+// Device (or managed) memory of the current device.  With unified virtual
+// addressing a 2 MiB page of device virtual memory never holds host memory,
+// so answers are cached per page (a direct-mapped table of recent pages).
+struct PageCache {
+  static constexpr int kSlots = 4096;
+  std::atomic<uint64_t> slot[kSlots];  // (page << 8) | (device + 1), 0 = empty
+  PageCache() {
+    for (auto& s : slot) s.store(0, std::memory_order_relaxed);
+  }
+};
+PageCache g_pages;
+
 bool on_device(const void* p, int dev) {
+  const uint64_t page = reinterpret_cast<uintptr_t>(p) >> 21;
+  const uint64_t tag = (page << 8) | static_cast<uint64_t>(dev + 1);
+  std::atomic<uint64_t>& s = g_pages.slot[page % PageCache::kSlots];
+  if (s.load(std::memory_order_relaxed) == tag) return true;
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
-    cudaGetLastError();  // clear the sticky-free error of an unknown pointer
+    cudaGetLastError();  // clear the error of an unknown pointer
     return false;
   }
-  if (a.type == cudaMemoryTypeManaged) return true;
-  return a.type == cudaMemoryTypeDevice && a.device == dev;
+  const bool ok = (a.type == cudaMemoryTypeDevice && a.device == dev) || a.type == cudaMemoryTypeManaged;
+  if (ok && a.type == cudaMemoryTypeDevice) s.store(tag, std::memory_order_relaxed);
+  return ok;
 }
 
+// Byte ranges touched by a call; outputs may not overlap anything else.
 struct Range {
   uintptr_t lo, hi;
+  bool output;
 };
-bool overlap(Range a, Range b) { return a.lo < b.hi && b.lo < a.hi; }
+
+bool ranges_disjoint(std::vector<Range>& r) {
+  std::sort(r.begin(), r.end(), [](const Range& a, const Range& b) { return a.lo < b.lo; });
+  uintptr_t max_hi_any = 0, max_hi_out = 0;
+  for (const Range& x : r) {
+    if (x.hi == x.lo) continue;
+    if (x.output ? x.lo < max_hi_any : x.lo < max_hi_out) return false;
+    max_hi_any = std::max(max_hi_any, x.hi);
+    if (x.output) max_hi_out = std::max(max_hi_out, x.hi);
+  }
+  return true;
+}
+
+Range range_of(const void* p, uint64_t bytes, bool output) {
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  return {a, a + bytes, output};
+}
+
+// ---------------------------------------------------------------------------
+// quantize
+// ---------------------------------------------------------------------------
+rrq_status check_quantize_item(const rrq_quantize_item& it, int group, int n_stages) {
+  if (!it.W_bf16 || !shape_ok(it.rows, it.cols)) return RRQ_ERR_INVALID_ARG;
+  if (it.cols % group != 0) return RRQ_ERR_INVALID_ARG;
+  for (int k = 0; k < n_stages; ++k)
+    if (!it.codes[k] || !it.scales[k] || !it.zeros[k]) return RRQ_ERR_INVALID_ARG;
+  if (!aligned(it.W_bf16, 16)) return RRQ_ERR_MISALIGNED;
+  for (int k = 0; k < n_stages; ++k)
+    if (!aligned(it.codes[k], 8) || !aligned(it.scales[k], 4) || !aligned(it.zeros[k], 4))
+      return RRQ_ERR_MISALIGNED;
+  return RRQ_OK;
+}
+
+void add_quantize_ranges(const rrq_quantize_item& it, int group, int n_stages, std::vector<Range>& r) {
+  const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
+  r.push_back(range_of(it.W_bf16, 2 * n, false));
+  for (int k = 0; k < n_stages; ++k) {
+    r.push_back(range_of(it.codes[k], n / 4, true));
+    r.push_back(range_of(it.scales[k], 4 * (n / group), true));
+    r.push_back(range_of(it.zeros[k], 4 * (n / group), true));
+  }
+}
+
+rrq_status quantize_batch(const rrq_quantize_item* items, int count, int group, int n_stages,
+                          rrq_stream_t stream) {
+  if (!items || count < 1 || n_stages < 1 || n_stages > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  std::vector<Range> ranges;
+  ranges.reserve(static_cast<size_t>(count) * (1 + 3 * n_stages));
+  for (int i = 0; i < count; ++i) {
+    if (rrq_status rc = check_quantize_item(items[i], group, n_stages)) return rc;
+    add_quantize_ranges(items[i], group, n_stages, ranges);
+  }
+  if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
+
+  int dev = 0;
+  DeviceState* st = nullptr;
+  if (rrq_status rc = current_device(&dev, &st)) return rc;
+  for (int i = 0; i < count; ++i) {
+    const rrq_quantize_item& it = items[i];
+    if (!on_device(it.W_bf16, dev)) return RRQ_ERR_INVALID_ARG;
+    for (int k = 0; k < n_stages; ++k)
+      if (!on_device(it.codes[k], dev) || !on_device(it.scales[k], dev) || !on_device(it.zeros[k], dev))
+        return RRQ_ERR_INVALID_ARG;
+  }
+
+  static thread_local rrq::QuantizeBatch p;  // ~8 KiB: kept off the stack
+  for (int base = 0; base < count; base += rrq::kMaxBatch) {
+    const int m = std::min(rrq::kMaxBatch, count - base);
+    std::memset(&p, 0, sizeof p);
+    p.count = m;
+    p.n_stages = n_stages;
+    p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
+    p.flags = g_debug_flags.load(std::memory_order_relaxed);
+    p.status = st->status;
+    int64_t chunks = 0;
+    for (int i = 0; i < m; ++i) {
+      const rrq_quantize_item& it = items[base + i];
+      rrq::QuantizeItem& q = p.item[i];
+      q.W = it.W_bf16;
+      q.n = it.rows * it.cols;
+      q.chunk_begin = chunks;
+      chunks += (q.n + rrq::kChunkElems - 1) / rrq::kChunkElems;
+      for (int k = 0; k < rrq::kMaxStages; ++k) {
+        const int kk = k < n_stages ? k : n_stages - 1;
+        q.codes[k] = it.codes[kk];
+        q.scales[k] = it.scales[kk];
+        q.zeros[k] = it.zeros[kk];
+      }
+    }
+    p.total_chunks = chunks;
+    cudaError_t e = rrq::quantize_launch(group, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+    if (e != cudaSuccess) return fail_cuda(e);
+  }
+  return RRQ_OK;
+}
+
+// ---------------------------------------------------------------------------
+// reconstruct
+// ---------------------------------------------------------------------------
+rrq_status check_reconstruct_item(const rrq_reconstruct_item& it, int group, int k) {
+  if (!it.out_bf16 || !shape_ok(it.rows, it.cols)) return RRQ_ERR_INVALID_ARG;
+  if (it.cols % group != 0) return RRQ_ERR_INVALID_ARG;
+  for (int i = 0; i < k; ++i)
+    if (!it.codes[i] || !it.scales[i] || !it.zeros[i]) return RRQ_ERR_INVALID_ARG;
+  if (!aligned(it.out_bf16, 16)) return RRQ_ERR_MISALIGNED;
+  for (int i = 0; i < k; ++i)
+    if (!aligned(it.codes[i], 8) || !aligned(it.scales[i], 4) || !aligned(it.zeros[i], 4))
+      return RRQ_ERR_MISALIGNED;
+  return RRQ_OK;
+}
+
+rrq_status reconstruct_batch(const rrq_reconstruct_item* items, int count, int group, int k,
+                             rrq_stream_t stream) {
+  if (!items || count < 1 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  std::vector<Range> ranges;
+  ranges.reserve(static_cast<size_t>(count) * (1 + 3 * k));
+  for (int i = 0; i < count; ++i) {
+    const rrq_reconstruct_item& it = items[i];
+    if (rrq_status rc = check_reconstruct_item(it, group, k)) return rc;
+    const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
+    ranges.push_back(range_of(it.out_bf16, 2 * n, true));
+    for (int j = 0; j < k; ++j) {
+      ranges.push_back(range_of(it.codes[j], n / 4, false));
+      ranges.push_back(range_of(it.scales[j], 4 * (n / group), false));
+      ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
+    }
+  }
+  if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
+
+  int dev = 0;
+  DeviceState* st = nullptr;
+  if (rrq_status rc = current_device(&dev, &st)) return rc;
+  for (int i = 0; i < count; ++i) {
+    const rrq_reconstruct_item& it = items[i];
+    if (!on_device(it.out_bf16, dev)) return RRQ_ERR_INVALID_ARG;
+    for (int j = 0; j < k; ++j)
+      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) || !on_device(it.zeros[j], dev))
+        return RRQ_ERR_INVALID_ARG;
+  }
+
+  static thread_local rrq::ReconstructBatch p;
+  for (int base = 0; base < count; base += rrq::kMaxBatch) {
+    const int m = std::min(rrq::kMaxBatch, count - base);
+    std::memset(&p, 0, sizeof p);
+    p.count = m;
+    int64_t chunks = 0;
+    for (int i = 0; i < m; ++i) {
+      const rrq_reconstruct_item& it = items[base + i];
+      rrq::ReconstructItem& q = p.item[i];
+      for (int j = 0; j < rrq::kMaxStages; ++j) {
+        const int jj = j < k ? j : k - 1;
+        q.codes[j] = it.codes[jj];
+        q.scales[j] = it.scales[jj];
+        q.zeros[j] = it.zeros[jj];
+      }
+      q.out = it.out_bf16;
+      q.n = it.rows * it.cols;
+      q.chunk_begin = chunks;
+      chunks += (q.n + rrq::kChunkElems - 1) / rrq::kChunkElems;
+    }
+    p.total_chunks = chunks;
+    cudaError_t e = rrq::reconstruct_launch(group, k, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+    if (e != cudaSuccess) return fail_cuda(e);
+  }
+  return RRQ_OK;
+}
 
 }  // namespace
 
@@ -107,108 +294,44 @@ size_t rrq_package_bytes(int64_t rows, int64_t cols, int group, int n_stages) {
 rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int group,
                         int n_stages, uint8_t* const out_codes[], float* const out_scales[],
                         float* const out_zeros[], rrq_stream_t stream) {
-  if (!W_bf16 || !out_codes || !out_scales || !out_zeros) return RRQ_ERR_INVALID_ARG;
-  if (!shape_ok(rows, cols) || n_stages < 1 || n_stages > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
-  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
-  if (cols % group != 0) return RRQ_ERR_INVALID_ARG;
-  for (int k = 0; k < n_stages; ++k)
-    if (!out_codes[k] || !out_scales[k] || !out_zeros[k]) return RRQ_ERR_INVALID_ARG;
-  if (!aligned(W_bf16, 16)) return RRQ_ERR_MISALIGNED;
-  for (int k = 0; k < n_stages; ++k)
-    if (!aligned(out_codes[k], 8) || !aligned(out_scales[k], 4) || !aligned(out_zeros[k], 4))
-      return RRQ_ERR_MISALIGNED;
-
-  const int64_t n = rows * cols;
-  const size_t code_bytes = static_cast<size_t>(n / 4);
-  const size_t meta_bytes = static_cast<size_t>(n / group) * sizeof(float);
-  Range ranges[1 + 3 * RRQ_MAX_STAGES];
-  int nr = 0;
-  ranges[nr++] = {reinterpret_cast<uintptr_t>(W_bf16), reinterpret_cast<uintptr_t>(W_bf16) + 2 * n};
+  if (!out_codes || !out_scales || !out_zeros || n_stages < 1 || n_stages > RRQ_MAX_STAGES)
+    return RRQ_ERR_INVALID_ARG;
+  rrq_quantize_item it{};
+  it.W_bf16 = W_bf16;
+  it.rows = rows;
+  it.cols = cols;
   for (int k = 0; k < n_stages; ++k) {
-    const uintptr_t c = reinterpret_cast<uintptr_t>(out_codes[k]);
-    const uintptr_t s = reinterpret_cast<uintptr_t>(out_scales[k]);
-    const uintptr_t z = reinterpret_cast<uintptr_t>(out_zeros[k]);
-    ranges[nr++] = {c, c + code_bytes};
-    ranges[nr++] = {s, s + meta_bytes};
-    ranges[nr++] = {z, z + meta_bytes};
+    it.codes[k] = out_codes[k];
+    it.scales[k] = out_scales[k];
+    it.zeros[k] = out_zeros[k];
   }
-  for (int a = 0; a < nr; ++a)
-    for (int b = a + 1; b < nr; ++b)
-      if (overlap(ranges[a], ranges[b])) return RRQ_ERR_INVALID_ARG;
+  return quantize_batch(&it, 1, group, n_stages, stream);
+}
 
-  int dev = 0;
-  DeviceState* st = nullptr;
-  if (rrq_status rc = current_device(&dev, &st)) return rc;
-  if (!on_device(W_bf16, dev)) return RRQ_ERR_INVALID_ARG;
-  for (int k = 0; k < n_stages; ++k)
-    if (!on_device(out_codes[k], dev) || !on_device(out_scales[k], dev) || !on_device(out_zeros[k], dev))
-      return RRQ_ERR_INVALID_ARG;
-
-  rrq::QuantizeParams p{};
-  p.W = W_bf16;
-  p.n = n;
-  for (int k = 0; k < rrq::kMaxStages; ++k) {
-    const int kk = k < n_stages ? k : n_stages - 1;
-    p.codes[k] = out_codes[kk];
-    p.scales[k] = out_scales[kk];
-    p.zeros[k] = out_zeros[kk];
-  }
-  p.n_stages = n_stages;
-  p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
-  p.flags = g_debug_flags.load(std::memory_order_relaxed);
-  p.status = st->status;
-  cudaError_t e = rrq::quantize_launch(group, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
-  if (e != cudaSuccess) return fail_cuda(e);
-  return RRQ_OK;
+rrq_status rrq_quantize_batch(const rrq_quantize_item* items, int count, int group, int n_stages,
+                              rrq_stream_t stream) {
+  return quantize_batch(items, count, group, n_stages, stream);
 }
 
 rrq_status rrq_reconstruct(const uint8_t* const codes[], const float* const scales[],
                            const float* const zeros[], int64_t rows, int64_t cols, int group,
                            int k, uint16_t* out_bf16, rrq_stream_t stream) {
-  if (!codes || !scales || !zeros || !out_bf16) return RRQ_ERR_INVALID_ARG;
-  if (!shape_ok(rows, cols) || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
-  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
-  if (cols % group != 0) return RRQ_ERR_INVALID_ARG;
-  for (int i = 0; i < k; ++i)
-    if (!codes[i] || !scales[i] || !zeros[i]) return RRQ_ERR_INVALID_ARG;
-  if (!aligned(out_bf16, 16)) return RRQ_ERR_MISALIGNED;
-  for (int i = 0; i < k; ++i)
-    if (!aligned(codes[i], 8) || !aligned(scales[i], 4) || !aligned(zeros[i], 4)) return RRQ_ERR_MISALIGNED;
-
-  const int64_t n = rows * cols;
-  const Range out{reinterpret_cast<uintptr_t>(out_bf16), reinterpret_cast<uintptr_t>(out_bf16) + 2 * n};
+  if (!codes || !scales || !zeros || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  rrq_reconstruct_item it{};
   for (int i = 0; i < k; ++i) {
-    const uintptr_t c = reinterpret_cast<uintptr_t>(codes[i]);
-    const uintptr_t s = reinterpret_cast<uintptr_t>(scales[i]);
-    const uintptr_t z = reinterpret_cast<uintptr_t>(zeros[i]);
-    const size_t mb = static_cast<size_t>(n / group) * sizeof(float);
-    if (overlap(out, {c, c + static_cast<size_t>(n / 4)}) || overlap(out, {s, s + mb}) ||
-        overlap(out, {z, z + mb}))
-      return RRQ_ERR_INVALID_ARG;
+    it.codes[i] = codes[i];
+    it.scales[i] = scales[i];
+    it.zeros[i] = zeros[i];
   }
+  it.rows = rows;
+  it.cols = cols;
+  it.out_bf16 = out_bf16;
+  return reconstruct_batch(&it, 1, group, k, stream);
+}
 
-  int dev = 0;
-  DeviceState* st = nullptr;
-  if (rrq_status rc = current_device(&dev, &st)) return rc;
-  if (!on_device(out_bf16, dev)) return RRQ_ERR_INVALID_ARG;
-  for (int i = 0; i < k; ++i)
-    if (!on_device(codes[i], dev) || !on_device(scales[i], dev) || !on_device(zeros[i], dev))
-      return RRQ_ERR_INVALID_ARG;
-
-  rrq::ReconstructParams p{};
-  for (int i = 0; i < rrq::kMaxStages; ++i) {
-    const int ii = i < k ? i : k - 1;
-    p.codes[i] = codes[ii];
-    p.scales[i] = scales[ii];
-    p.zeros[i] = zeros[ii];
-  }
-  p.n = n;
-  p.out = out_bf16;
-  p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
-  p.status = st->status;
-  cudaError_t e = rrq::reconstruct_launch(group, k, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
-  if (e != cudaSuccess) return fail_cuda(e);
-  return RRQ_OK;
+rrq_status rrq_reconstruct_batch(const rrq_reconstruct_item* items, int count, int group, int k,
+                                 rrq_stream_t stream) {
+  return reconstruct_batch(items, count, group, k, stream);
 }
 
 rrq_status rrq_get_device_status(rrq_stream_t stream) {

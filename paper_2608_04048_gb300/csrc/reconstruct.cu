@@ -3,11 +3,22 @@
 //     acc = L_0;  acc = fl(acc + L_i) for i = 1..k-1;  out = bf16_rne(acc)
 // with L_i = fl(zero_i + fl(Q_i * scale_i)) the dequantized value of stage i.
 //
-// A warp owns a chunk of 1024 consecutive weights, a lane owns 32 consecutive
-// weights (one 8-byte code word per stage, one scale and one zero per stage).
-// Code words and metadata are loaded one chunk ahead into registers; the
-// 2 KiB of bf16 output of a chunk is staged in shared memory and written by a
-// 1-D bulk copy (TMA store), double-buffered per warp.
+// A warp owns a chunk of 1024 consecutive weights of one matrix, a lane owns
+// 32 consecutive weights (one 8-byte code word per stage, one scale and one
+// zero per stage).  The chunks of all matrices of a launch form one sequence
+// taken in turn by the warps of a persistent grid.  Each lane copies its code
+// words and metadata asynchronously (cp.async) into a per-warp ring of
+// shared-memory buffers kRing - 1 chunks ahead of use, so that many chunks'
+// loads are in flight without holding registers; the 2 KiB of bf16 output of
+// a chunk is staged in shared memory and written by a 1-D bulk copy (TMA
+// store), double-buffered per warp.
+//
+// fl(Q*s) is one fused multiply-add: with t the float whose bits are
+// 0x4B000000 | (Q << 2j), t = 2^23 + Q*4^j exactly, and
+// fma(t, s*4^-j, -2^23*s*4^-j) = RN(Q*s) because the scalings by powers of
+// two are exact for s in [2^-100, 2^100].  So four codes of one byte need one
+// shift and one logic operation each, no shift per code.  Groups with a scale
+// outside that range use the plain form RN((t - 2^23) * s).
 #include <cuda_bf16.h>
 
 #include "rrq_device.cuh"
@@ -17,44 +28,31 @@ namespace {
 
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
-constexpr int kSmemBytes = kWarps * 2 * kChunkBytes;
-constexpr float kTwo23 = 8388608.0f;  // bits 0x4B000000 | q encode 2^23 + q for 0 <= q < 2^23
+constexpr int kRing = 4;               // chunks of inputs per warp in shared memory
+constexpr int kStageBytes = 512;       // one stage of one chunk: codes 256 B, scales 128 B, zeros 128 B
+constexpr float kTwo23 = 8388608.0f;   // bits 0x4B000000 | q encode 2^23 + q for 0 <= q < 2^23
 
 template <int K>
-struct ChunkInputs {
-  uint2 code[K];
-  float scale[K];
-  float zero[K];
-};
+__host__ __device__ constexpr int warp_smem_bytes() { return kRing * K * kStageBytes + 2 * kChunkBytes; }
+template <int K>
+__host__ __device__ constexpr int smem_bytes() { return kWarps * warp_smem_bytes<K>(); }
 
-template <int G, int K>
-__device__ __forceinline__ void load_chunk(const ReconstructParams& p, int64_t e0, bool valid,
-                                           ChunkInputs<K>& in) {
-#pragma unroll
-  for (int i = 0; i < K; ++i) {
-    if (valid) {
-      in.code[i] = __ldcs(reinterpret_cast<const uint2*>(p.codes[i] + (e0 >> 2)));
-      in.scale[i] = __ldg(p.scales[i] + e0 / G);
-      in.zero[i] = __ldg(p.zeros[i] + e0 / G);
-    } else {
-      in.code[i] = make_uint2(0u, 0u);
-      in.scale[i] = 0.0f;
-      in.zero[i] = 0.0f;
-    }
-  }
+__device__ __forceinline__ bool prescale_ok(float s) {
+  return s == 0.0f || (s >= 0x1p-100f && s <= 0x1p+100f);
 }
 
 template <int G, int K>
-__global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const ReconstructParams p) {
+__global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_constant__ ReconstructBatch p) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  uint8_t* stage_buf = smem + warp * (2 * kChunkBytes);
+  uint8_t* ring = smem + warp * warp_smem_bytes<K>();
+  uint8_t* stage_buf = ring + kRing * K * kStageBytes;
+  constexpr int kBufBytes = K * kStageBytes;
 
-  const int64_t n_chunks = (p.n + kChunkElems - 1) / kChunkElems;
   const int64_t first = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kWarps;
-  if (first >= n_chunks) return;
+  if (first >= p.total_chunks) return;
 
   // Slot j of a lane handles its 16-byte output piece (j + rot) & 3, so that
   // the shared-memory stores of a quarter warp hit distinct bank groups; the
@@ -63,37 +61,93 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const Reconstr
   const uint32_t sel_lo = rot == 0 ? 0x3210u : rot == 1 ? 0x5432u : rot == 2 ? 0x7654u : 0x1076u;
   const uint32_t sel_hi = rot == 0 ? 0x7654u : rot == 1 ? 0x1076u : rot == 2 ? 0x3210u : 0x5432u;
 
-  ChunkInputs<K> cur;
-  {
-    const int64_t e0 = first * kChunkElems + static_cast<int64_t>(lane) * kLaneElems;
-    load_chunk<G, K>(p, e0, e0 < p.n, cur);
-  }
-  uint32_t it = 0;
-  for (int64_t chunk = first; chunk < n_chunks; chunk += stride, ++it) {
-    const int64_t e0 = chunk * kChunkElems + static_cast<int64_t>(lane) * kLaneElems;
-    ChunkInputs<K> nxt;
-    {
-      const int64_t e1 = e0 + stride * kChunkElems;
-      load_chunk<G, K>(p, e1, e1 < p.n, nxt);
+  int m_load = 0, m_work = 0;
+  auto item_of = [&](int64_t chunk, int& m) -> const ReconstructItem& {
+    while (m + 1 < p.count && chunk >= p.item[m + 1].chunk_begin) ++m;
+    return p.item[m];
+  };
+
+  // Copies this lane's inputs of `chunk` into ring buffer `buf` (one commit
+  // group per call, empty past the end; lanes past a matrix's end get zeros).
+  auto issue = [&](int64_t chunk, int buf) {
+    if (chunk < p.total_chunks) {
+      const ReconstructItem& it = item_of(chunk, m_load);
+      const int64_t e = (chunk - it.chunk_begin) * kChunkElems + static_cast<int64_t>(lane) * kLaneElems;
+      const bool valid = e < it.n;
+      const uint32_t base = smem_u32(ring + buf * kBufBytes);
+#pragma unroll
+      for (int i = 0; i < K; ++i) {
+        const uint32_t sb = base + i * kStageBytes;
+        cp_async_8(sb + lane * 8, valid ? it.codes[i] + (e >> 2) : it.codes[i], valid ? 8u : 0u);
+        cp_async_4(sb + 256 + lane * 4, valid ? it.scales[i] + e / G : it.scales[i], valid ? 4u : 0u);
+        cp_async_4(sb + 384 + lane * 4, valid ? it.zeros[i] + e / G : it.zeros[i], valid ? 4u : 0u);
+      }
+    }
+    cp_async_commit();
+  };
+
+#pragma unroll
+  for (int j = 0; j < kRing - 1; ++j) issue(first + j * stride, j);
+
+  uint32_t iter = 0;
+  for (int64_t chunk = first; chunk < p.total_chunks; chunk += stride, ++iter) {
+    issue(chunk + (kRing - 1) * stride, (iter + kRing - 1) % kRing);
+    cp_async_wait<kRing - 1>();  // this lane's copies of `chunk` have landed
+
+    const uint8_t* buf = ring + (iter % kRing) * kBufBytes;
+    uint2 code[K];
+    float scale[K], zero[K];
+    bool ok = true;
+#pragma unroll
+    for (int i = 0; i < K; ++i) {
+      code[i] = *reinterpret_cast<const uint2*>(buf + i * kStageBytes + lane * 8);
+      scale[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + 256 + lane * 4);
+      zero[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + 384 + lane * 4);
+      ok = ok && prescale_ok(scale[i]);
     }
 
     f32x2 acc[16];
+    if (__all_sync(kFullMask, ok)) {
 #pragma unroll
-    for (int i = 0; i < K; ++i) {
-      const uint32_t w0 = __byte_perm(cur.code[i].x, cur.code[i].y, sel_lo);
-      const uint32_t w1 = __byte_perm(cur.code[i].x, cur.code[i].y, sel_hi);
-      const f32x2 LO = pack2(cur.zero[i], cur.zero[i]);
-      const f32x2 S = pack2(cur.scale[i], cur.scale[i]);
-      const float c = __fmul_rn(-kTwo23, cur.scale[i]);  // exact: power-of-two scaling
-      const f32x2 C = pack2(c, c);
+      for (int i = 0; i < K; ++i) {
+        const uint32_t w0 = __byte_perm(code[i].x, code[i].y, sel_lo);
+        const uint32_t w1 = __byte_perm(code[i].x, code[i].y, sel_hi);
+        const float s = scale[i];
+        const f32x2 LO = pack2(zero[i], zero[i]);
+        const f32x2 S01 = pack2(s, __fmul_rn(s, 0x1p-2f));
+        const f32x2 S23 = pack2(__fmul_rn(s, 0x1p-4f), __fmul_rn(s, 0x1p-6f));
+        const f32x2 C01 = pack2(__fmul_rn(s, -0x1p23f), __fmul_rn(s, -0x1p21f));
+        const f32x2 C23 = pack2(__fmul_rn(s, -0x1p19f), __fmul_rn(s, -0x1p17f));
 #pragma unroll
-      for (int m = 0; m < 16; ++m) {  // pair m: slot m/4, elements 2*(m%4), +1
-        const uint32_t word = m < 8 ? w0 : w1;
-        const int sh = 4 * (m & 7);
-        const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
-        // fl(Q*s) as one fused multiply-add (t = 2^23 + Q), then fl(zero + step)
-        const f32x2 level = add2(LO, fma2(t, S, C));
-        acc[m] = (i == 0) ? level : add2(acc[m], level);
+        for (int j = 0; j < 8; ++j) {  // byte j: elements 4j..4j+3 (pairs 2j, 2j+1)
+          const uint32_t word = j < 4 ? w0 : w1;
+          const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
+          const f32x2 t01 = pack2u(0x4B000000u | (b & 0x03u), 0x4B000000u | (b & 0x0Cu));
+          const f32x2 t23 = pack2u(0x4B000000u | (b & 0x30u), 0x4B000000u | (b & 0xC0u));
+          const f32x2 l01 = add2(LO, fma2(t01, S01, C01));
+          const f32x2 l23 = add2(LO, fma2(t23, S23, C23));
+          acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
+          acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
+        }
+      }
+    } else {
+      const f32x2 Z = pack2(0.0f, 0.0f), T23 = pack2(kTwo23, kTwo23);
+#pragma unroll
+      for (int i = 0; i < K; ++i) {
+        const uint32_t w0 = __byte_perm(code[i].x, code[i].y, sel_lo);
+        const uint32_t w1 = __byte_perm(code[i].x, code[i].y, sel_hi);
+        const f32x2 LO = pack2(zero[i], zero[i]);
+        const f32x2 S = pack2(scale[i], scale[i]);
+#pragma unroll
+        for (int m = 0; m < 16; ++m) {
+          const uint32_t word = m < 8 ? w0 : w1;
+          const int sh = 4 * (m & 7);
+          const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+          // RN(Q*s) through an fma with a zero addend (the compiler would fuse
+          // a separate multiply into the following add)
+          const f32x2 level = add2(LO, fma2(sub2(t, T23), S, Z));
+          acc[m] = (i == 0) ? level : add2(acc[m], level);
+        }
       }
     }
 
@@ -107,46 +161,46 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const Reconstr
       outw[m] = *reinterpret_cast<const uint32_t*>(&h);
     }
 
-    const int b = it & 1;
-    if (lane == 0) bulk_wait_read<1>();  // the store that last used buffer b has read it
+    const ReconstructItem& it = item_of(chunk, m_work);
+    const int bsel = iter & 1;
+    if (lane == 0) bulk_wait_read<1>();  // the store that last used this buffer has read it
     __syncwarp();
-    uint4* dst = reinterpret_cast<uint4*>(stage_buf + b * kChunkBytes + lane * 64);
+    uint4* dst = reinterpret_cast<uint4*>(stage_buf + bsel * kChunkBytes + lane * 64);
 #pragma unroll
     for (int j = 0; j < 4; ++j)
       dst[(j + rot) & 3] = make_uint4(outw[4 * j], outw[4 * j + 1], outw[4 * j + 2], outw[4 * j + 3]);
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) {
-      const int64_t e = chunk * kChunkElems;
-      const int64_t left = p.n - e;
+      const int64_t e = (chunk - it.chunk_begin) * kChunkElems;
+      const int64_t left = it.n - e;
       const uint32_t bytes = static_cast<uint32_t>((left < kChunkElems ? left : kChunkElems) * 2);
-      bulk_store(p.out + e, smem_u32(stage_buf + b * kChunkBytes), bytes);
+      bulk_store(it.out + e, smem_u32(stage_buf + bsel * kChunkBytes), bytes);
       bulk_commit();
     }
-    cur = nxt;
   }
+  cp_async_wait<0>();
   if (lane == 0) bulk_wait<0>();
 }
 
 template <int G, int K>
-cudaError_t launch_gk(const ReconstructParams& p, cudaStream_t stream, int sms) {
+cudaError_t launch_gk(const ReconstructBatch& p, cudaStream_t stream, int sms) {
   static int blocks_per_sm = 0;
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, reconstruct_kernel<G, K>, kThreads, kSmemBytes);
+        &blocks_per_sm, reconstruct_kernel<G, K>, kThreads, smem_bytes<K>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
-  const int64_t n_chunks = (p.n + kChunkElems - 1) / kChunkElems;
-  const int64_t want = (n_chunks + kWarps - 1) / kWarps;
+  const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  reconstruct_kernel<G, K><<<grid, kThreads, kSmemBytes, stream>>>(p);
+  reconstruct_kernel<G, K><<<grid, kThreads, smem_bytes<K>(), stream>>>(p);
   return cudaGetLastError();
 }
 
 template <int G>
-cudaError_t launch_g(int k, const ReconstructParams& p, cudaStream_t stream, int sms) {
+cudaError_t launch_g(int k, const ReconstructBatch& p, cudaStream_t stream, int sms) {
   switch (k) {
     case 1: return launch_gk<G, 1>(p, stream, sms);
     case 2: return launch_gk<G, 2>(p, stream, sms);
@@ -158,9 +212,24 @@ cudaError_t launch_g(int k, const ReconstructParams& p, cudaStream_t stream, int
 
 }  // namespace
 
-cudaError_t reconstruct_prepare() { return cudaSuccess; }  // < 48 KiB shared memory
+template <int G>
+cudaError_t prepare_g() {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<3>()))) return e;
+  return cudaFuncSetAttribute(reconstruct_kernel<G, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<4>());
+}
 
-cudaError_t reconstruct_launch(int group, int k, const ReconstructParams& p, cudaStream_t stream,
+cudaError_t reconstruct_prepare() {
+  cudaError_t e;
+  if ((e = prepare_g<32>())) return e;
+  if ((e = prepare_g<64>())) return e;
+  if ((e = prepare_g<128>())) return e;
+  return prepare_g<256>();
+}
+
+cudaError_t reconstruct_launch(int group, int k, const ReconstructBatch& p, cudaStream_t stream,
                                int sms) {
   switch (group) {
     case 32: return launch_g<32>(k, p, stream, sms);

@@ -12,31 +12,46 @@ constexpr int kMaxStages = 4;
 constexpr int kLaneElems = 32;                    // weights owned by one lane per chunk
 constexpr int kChunkElems = 32 * kLaneElems;      // weights per warp chunk (1024)
 constexpr int kChunkBytes = kChunkElems * 2;      // bf16 bytes per warp chunk (2 KiB)
+constexpr int kMaxBatch = 64;                     // matrices per kernel launch (kernel parameters)
 
 constexpr unsigned kStatusTimeout = 1u;           // bit set in the device status word
 constexpr uint32_t kDebugForceExact = 1u;         // same value as RRQ_DEBUG_FORCE_EXACT
 constexpr uint32_t kDrainLimitUs = 1000000u;      // wait for own copies before leaving
 
-struct QuantizeParams {
+// One matrix of a quantize launch.  Chunks of all matrices of a launch are
+// numbered consecutively; chunk_begin is this matrix's first chunk.
+struct QuantizeItem {
   const uint16_t* W;               // bf16 bits, n elements
   int64_t n;                       // rows * cols (multiple of 32)
+  int64_t chunk_begin;
   uint8_t* codes[kMaxStages];      // n/4 bytes each
   float* scales[kMaxStages];       // n/group each
   float* zeros[kMaxStages];        // n/group each
+};
+
+struct QuantizeBatch {
+  int count;                       // 1..kMaxBatch
   int n_stages;                    // 1..4
   uint32_t wait_limit_us;
   uint32_t flags;                  // kDebugForceExact
   unsigned* status;                // device status word
+  int64_t total_chunks;
+  QuantizeItem item[kMaxBatch];
 };
 
-struct ReconstructParams {
+struct ReconstructItem {
   const uint8_t* codes[kMaxStages];
   const float* scales[kMaxStages];
   const float* zeros[kMaxStages];
-  int64_t n;
   uint16_t* out;                   // bf16 bits, n elements
-  uint32_t wait_limit_us;
-  unsigned* status;
+  int64_t n;
+  int64_t chunk_begin;
+};
+
+struct ReconstructBatch {
+  int count;
+  int64_t total_chunks;
+  ReconstructItem item[kMaxBatch];
 };
 
 // One-time per-device set-up of kernel attributes (dynamic shared memory).
@@ -44,8 +59,8 @@ cudaError_t quantize_prepare();
 cudaError_t reconstruct_prepare();
 
 // Launch on `stream`; `sms` = multiprocessor count of the current device.
-cudaError_t quantize_launch(int group, const QuantizeParams& p, cudaStream_t stream, int sms);
-cudaError_t reconstruct_launch(int group, int k, const ReconstructParams& p, cudaStream_t stream,
+cudaError_t quantize_launch(int group, const QuantizeBatch& p, cudaStream_t stream, int sms);
+cudaError_t reconstruct_launch(int group, int k, const ReconstructBatch& p, cudaStream_t stream,
                                int sms);
 
 }  // namespace rrq

@@ -189,3 +189,43 @@ def test_nonzero_current_stream():
     ref = oracle.quantize(bf16_bits(W), 128, 4)
     assert_package_equal(gpu_package_host(pkg), ref, 4, "stream")
     assert np.array_equal(bf16_bits(out), oracle.reconstruct(*ref, 1024, 1024, 128, 4))
+
+
+def test_batch_matches_oracle_across_launches():
+    """rrq_quantize_batch / rrq_reconstruct_batch over 70 matrices of mixed
+    shapes (two launches of the 64-matrix batch kernel, chunks of different
+    matrices interleaved across warps): every package and reconstruction
+    equals the oracle's."""
+    rng = np.random.default_rng(0)
+    shapes = [(int(rng.integers(1, 40)), 128 * int(rng.integers(1, 12))) for _ in range(70)]
+    mats = [workloads.generate(r, c, 100 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+    pkgs = binding.rrq_quantize_batch(mats, group=128, n_stages=4)
+    outs = {k: binding.rrq_reconstruct_batch(pkgs, k) for k in (1, 2, 3, 4)}
+    torch.cuda.synchronize()
+    for i, (W, pkg) in enumerate(zip(mats, pkgs)):
+        ref = oracle.quantize(bf16_bits(W), 128, 4)
+        assert_package_equal(gpu_package_host(pkg), ref, 4, f"batch item {i}")
+        for k in (1, 2, 3, 4):
+            want = oracle.reconstruct(*ref, W.shape[0], W.shape[1], 128, k)
+            assert np.array_equal(bf16_bits(outs[k][i]), want), f"batch item {i} k={k}"
+
+
+def test_batch_rejects_overlapping_outputs():
+    mats = [workloads.generate(8, 256, i, "normal", "cuda") for i in range(2)]
+    pkgs = [binding.Package.empty(8, 256, 128, 4) for _ in range(2)]
+    pkgs[1].codes[0] = pkgs[0].codes[0]  # two matrices writing the same codes
+    with pytest.raises(binding.RRQError) as e:
+        binding.rrq_quantize_batch(mats, pkgs, 128, 4)
+    assert e.value.status == 1
+
+
+@pytest.mark.parametrize("group", GROUPS)
+def test_batch_group_sizes(group):
+    mats = [workloads.generate(17 + i, group * (1 + i), 7 * i + group, "t3", "cuda") for i in range(5)]
+    pkgs = binding.rrq_quantize_batch(mats, group=group, n_stages=3)
+    outs = binding.rrq_reconstruct_batch(pkgs, 3)
+    torch.cuda.synchronize()
+    for W, pkg, out in zip(mats, pkgs, outs):
+        ref = oracle.quantize(bf16_bits(W), group, 3)
+        assert_package_equal(gpu_package_host(pkg), ref, 3, f"batch g{group}")
+        assert np.array_equal(bf16_bits(out), oracle.reconstruct(*ref, W.shape[0], W.shape[1], group, 3))
