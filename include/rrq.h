@@ -78,10 +78,10 @@ typedef enum {
  *   n_stages    1..4: stage 0 is the 2-bit base, stages 1..n_stages-1 are
  *               2-bit residual stages.
  *   out_codes   host array of n_stages device pointers, each to
- *               rrq_codes_bytes(rows, cols) bytes, 8-byte aligned.
+ *               rrq_codes_bytes(rows, cols) bytes, 16-byte aligned.
  *   out_scales, out_zeros
  *               host arrays of n_stages device pointers, each to
- *               rrq_meta_count(rows, cols, group) floats, 4-byte aligned.
+ *               rrq_meta_count(rows, cols, group) floats, 16-byte aligned.
  * No output may overlap another output or W.  One fused kernel computes all
  * stages; the running residual never leaves registers. */
 rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int group,
@@ -92,7 +92,8 @@ rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int 
 /* Prefix reconstruction with the first k stages (Eq. 8; Appendix C):
  * k = 1, 2, 3, 4 give the 2-, 4-, 6-, 8-bit operating points.
  *   codes, scales, zeros  host arrays of >= k device pointers laid out as
- *                         written by rrq_quantize (8-, 4-, 4-byte aligned).
+ *                         written by rrq_quantize (16-byte aligned; the
+ *                         kernel copies whole chunks with bulk copies).
  *   rows, cols, group     as given to rrq_quantize.
  *   k                     1..4.
  *   out_bf16              device, bf16 bit patterns [rows, cols], 16-byte

@@ -129,7 +129,7 @@ rrq_status check_quantize_item(const rrq_quantize_item& it, int group, int n_sta
     if (!it.codes[k] || !it.scales[k] || !it.zeros[k]) return RRQ_ERR_INVALID_ARG;
   if (!aligned(it.W_bf16, 16)) return RRQ_ERR_MISALIGNED;
   for (int k = 0; k < n_stages; ++k)
-    if (!aligned(it.codes[k], 8) || !aligned(it.scales[k], 4) || !aligned(it.zeros[k], 4))
+    if (!aligned(it.codes[k], 16) || !aligned(it.scales[k], 16) || !aligned(it.zeros[k], 16))
       return RRQ_ERR_MISALIGNED;
   return RRQ_OK;
 }
@@ -208,7 +208,7 @@ rrq_status check_reconstruct_item(const rrq_reconstruct_item& it, int group, int
     if (!it.codes[i] || !it.scales[i] || !it.zeros[i]) return RRQ_ERR_INVALID_ARG;
   if (!aligned(it.out_bf16, 16)) return RRQ_ERR_MISALIGNED;
   for (int i = 0; i < k; ++i)
-    if (!aligned(it.codes[i], 8) || !aligned(it.scales[i], 4) || !aligned(it.zeros[i], 4))
+    if (!aligned(it.codes[i], 16) || !aligned(it.scales[i], 16) || !aligned(it.zeros[i], 16))
       return RRQ_ERR_MISALIGNED;
   return RRQ_OK;
 }
@@ -248,6 +248,8 @@ rrq_status reconstruct_batch(const rrq_reconstruct_item* items, int count, int g
     const int m = std::min(rrq::kMaxBatch, count - base);
     std::memset(&p, 0, sizeof p);
     p.count = m;
+    p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
+    p.status = st->status;
     int64_t chunks = 0;
     for (int i = 0; i < m; ++i) {
       const rrq_reconstruct_item& it = items[base + i];

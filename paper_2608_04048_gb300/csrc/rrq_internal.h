@@ -50,6 +50,8 @@ struct ReconstructItem {
 
 struct ReconstructBatch {
   int count;
+  uint32_t wait_limit_us;
+  unsigned* status;                // device status word
   int64_t total_chunks;
   ReconstructItem item[kMaxBatch];
 };

@@ -76,6 +76,7 @@ def test_quantize_argument_checks_run_before_cuda(lib):
     assert call(cols=192) == 1                      # cols % group != 0
     assert call(W=base + 8) == 3                    # bf16 input must be 16-byte aligned
     assert call(codes=[base + 0x10004, base + 0x20000]) == 3
+    assert call(codes=[base + 0x10008, base + 0x20000]) == 3   # package arrays: 16-byte aligned
     assert call(scales=[base + 0x30002, base + 0x40000]) == 3
     assert call(codes=[base + 0x10000, base + 0x10040]) == 1   # overlapping outputs
     assert call(zeros=[base + 0x50000, base + 0x100]) == 1     # output overlaps W

@@ -158,10 +158,14 @@ def test_timeout_path_reports_and_recovers():
     stays usable and the next call is exact again."""
     W = workloads.generate(512, 1024, 21, "normal", "cuda")
     binding.rrq_get_device_status()  # clear
+    pkg = binding.rrq_quantize(W, 128, 4)
     binding.rrq_set_wait_limit_us(0)
     try:
         binding.rrq_quantize(W, 128, 4)
         assert binding.rrq_get_device_status() == 5
+        # reconstruction has no bounded waits (its copies complete in hardware)
+        out = binding.rrq_reconstruct(pkg, 4)
+        assert binding.rrq_get_device_status() == 0
     finally:
         binding.rrq_set_wait_limit_us(1_000_000)
     assert binding.rrq_get_device_status() == 0
