@@ -44,6 +44,12 @@ STAGES = 4
 KS = (1, 2, 3, 4)
 WORKLOAD = "qwen3_8b_stack"
 METRIC = "RRQ package construction GB/s of bf16 weights and % of HBM peak; s per 8B-shaped stack"
+WORKLOAD_TEXT = {
+    "qwen3_8b_stack": "qwen3_8b_stack: 36 layers x (q 4096x4096, k/v 1024x4096, o 4096x4096, gate/up "
+                      "12288x4096, down 4096x12288), bf16, Student-t(3) std 0.02 + 0.1% +-0.4 outliers per "
+                      "row, group 128 along the input dim, 4 x 2-bit stages",
+    "qwen3_8b_layer": "qwen3_8b_layer: one layer of the 36-layer stack's shapes and distribution",
+}
 
 
 def alg_bytes_quantize(n: int, g: int = GROUP, S: int = STAGES) -> float:
@@ -261,12 +267,11 @@ def run_gpu(args, world, rank, local) -> dict | None:
         "dtype": "f32",
         "data": "synthetic",
         "config": {
-            "workload": f"{args.workload}: 36 layers x (q 4096x4096, k/v 1024x4096, o 4096x4096, "
-                        "gate/up 12288x4096, down 4096x12288), bf16, Student-t(3) std 0.02 + 0.1% +-0.4 "
-                        "outliers per row, group 128 along the input dim, 4 x 2-bit stages",
-            "step": "rrq_quantize_batch on all 252 matrices, then rrq_reconstruct_batch on all 252 at k=1,2,3,4",
+            "workload": WORKLOAD_TEXT.get(args.workload, args.workload),
+            "step": f"rrq_quantize_batch on all {len(specs)} matrices, then rrq_reconstruct_batch on all "
+                    f"{len(specs)} at k=1,2,3,4",
             "weights_per_rank": n_total,
-            "l2": "inputs 13.9 GB per rank, far larger than the 126 MB L2; no flush",
+            "l2": f"inputs {2 * n_total / 1e9:.2f} GB per rank, larger than the 126 MB L2; no flush",
             "parallelism": f"{world} independent rank(s), one stack each",
         },
         "breakdown": {
