@@ -73,14 +73,18 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
     if (chunk < p.total_chunks) {
       const ReconstructItem& it = item_of(chunk, m_load);
       const int64_t e = (chunk - it.chunk_begin) * kChunkElems + static_cast<int64_t>(lane) * kLaneElems;
-      const bool valid = e < it.n;
-      const uint32_t base = smem_u32(ring + buf * kBufBytes);
+      const bool valid = e < it.n;  // false only in the last chunk of a matrix
+      // byte offsets shared by every stage's arrays (invalid lanes read nothing)
+      const uint64_t off_code = valid ? static_cast<uint64_t>(e) >> 2 : 0;
+      const uint64_t off_meta = valid ? (static_cast<uint64_t>(e) / G) * 4 : 0;
+      const uint32_t n8 = valid ? 8u : 0u, n4 = valid ? 4u : 0u;
+      const uint32_t base = smem_u32(ring + buf * K * kStageBytes) + lane * 8;
+      const uint32_t mbase = smem_u32(ring + buf * K * kStageBytes) + 256 + lane * 4;
 #pragma unroll
       for (int i = 0; i < K; ++i) {
-        const uint32_t sb = base + i * kStageBytes;
-        cp_async_8(sb + lane * 8, valid ? it.codes[i] + (e >> 2) : it.codes[i], valid ? 8u : 0u);
-        cp_async_4(sb + 256 + lane * 4, valid ? it.scales[i] + e / G : it.scales[i], valid ? 4u : 0u);
-        cp_async_4(sb + 384 + lane * 4, valid ? it.zeros[i] + e / G : it.zeros[i], valid ? 4u : 0u);
+        cp_async_8(base + i * kStageBytes, reinterpret_cast<const char*>(it.codes[i]) + off_code, n8);
+        cp_async_4(mbase + i * kStageBytes, reinterpret_cast<const char*>(it.scales[i]) + off_meta, n4);
+        cp_async_4(mbase + i * kStageBytes + 128, reinterpret_cast<const char*>(it.zeros[i]) + off_meta, n4);
       }
     }
     cp_async_commit();
