@@ -137,6 +137,32 @@ typedef struct {
 rrq_status rrq_reconstruct_batch(const rrq_reconstruct_item* items, int count, int group, int k,
                                  rrq_stream_t stream);
 
+/* All prefixes at once (Eq. 8 for t = 0..k-1; Appendix C): one pass over the
+ * first k stages writes the reconstruction after every stage, out_bf16[j]
+ * receiving the prefix with j+1 stages (the 2-, 4-, 6-, 8-bit weights for
+ * k = 4).  Bit-identical to k separate rrq_reconstruct calls with k = 1..j+1,
+ * reading the package once instead of k times.  out_bf16 is a host array of
+ * k device pointers (16-byte aligned, not overlapping each other or any
+ * input). */
+rrq_status rrq_reconstruct_prefixes(const uint8_t* const codes[], const float* const scales[],
+                                    const float* const zeros[], int64_t rows, int64_t cols,
+                                    int group, int k, uint16_t* const out_bf16[],
+                                    rrq_stream_t stream);
+
+/* One matrix of rrq_reconstruct_prefixes_batch. */
+typedef struct {
+  const uint8_t* codes[RRQ_MAX_STAGES];  /* first k entries used */
+  const float* scales[RRQ_MAX_STAGES];
+  const float* zeros[RRQ_MAX_STAGES];
+  int64_t rows, cols;
+  uint16_t* out_bf16[RRQ_MAX_STAGES];    /* out_bf16[j]: prefix with j+1 stages */
+} rrq_prefixes_item;
+
+/* rrq_reconstruct_prefixes for `count` matrices sharing `group` and `k`, one
+ * kernel launch per 64 matrices. */
+rrq_status rrq_reconstruct_prefixes_batch(const rrq_prefixes_item* items, int count, int group,
+                                          int k, rrq_stream_t stream);
+
 /* Bytes of one stage's code array: rows*cols/4 (rows*cols is a multiple of
  * 32 for every valid shape).  0 for invalid sizes. */
 size_t rrq_codes_bytes(int64_t rows, int64_t cols);

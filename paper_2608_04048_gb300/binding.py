@@ -21,6 +21,7 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
 
 #: symbols declared in include/rrq.h
 EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
+           "rrq_reconstruct_prefixes", "rrq_reconstruct_prefixes_batch",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
            "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
@@ -41,6 +42,13 @@ class ReconstructItem(ctypes.Structure):
     _fields_ = [("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
                 ("zeros", ctypes.c_void_p * MAX_STAGES), ("rows", ctypes.c_int64),
                 ("cols", ctypes.c_int64), ("out_bf16", ctypes.c_void_p)]
+
+
+class PrefixesItem(ctypes.Structure):
+    """rrq_prefixes_item of include/rrq.h"""
+    _fields_ = [("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
+                ("zeros", ctypes.c_void_p * MAX_STAGES), ("rows", ctypes.c_int64),
+                ("cols", ctypes.c_int64), ("out_bf16", ctypes.c_void_p * MAX_STAGES)]
 
 
 class RRQError(RuntimeError):
@@ -76,6 +84,11 @@ def load_library():
     lib.rrq_quantize_batch.restype = i32
     lib.rrq_reconstruct_batch.argtypes = [ctypes.POINTER(ReconstructItem), i32, i32, i32, vp]
     lib.rrq_reconstruct_batch.restype = i32
+    lib.rrq_reconstruct_prefixes.argtypes = [ptr_array, ptr_array, ptr_array, i64, i64, i32, i32,
+                                             ptr_array, vp]
+    lib.rrq_reconstruct_prefixes.restype = i32
+    lib.rrq_reconstruct_prefixes_batch.argtypes = [ctypes.POINTER(PrefixesItem), i32, i32, i32, vp]
+    lib.rrq_reconstruct_prefixes_batch.restype = i32
     lib.rrq_codes_bytes.argtypes = [i64, i64]
     lib.rrq_codes_bytes.restype = ctypes.c_size_t
     lib.rrq_meta_count.argtypes = [i64, i64, i32]
@@ -223,6 +236,58 @@ def rrq_reconstruct_batch(pkgs, k: int, outs=None, stream=None, items=None):
     rc = lib.rrq_reconstruct_batch(items, len(items), group, k, _stream_handle(stream))
     if rc != 0:
         raise RRQError(rc, "rrq_reconstruct_batch")
+    return outs
+
+
+def _new_outs(pkg, k):
+    return [torch.empty((pkg.rows, pkg.cols), dtype=torch.bfloat16, device=pkg.codes[0].device)
+            for _ in range(k)]
+
+
+def rrq_reconstruct_prefixes(pkg: Package, k: int, outs=None, stream=None):
+    """bf16 weights of every prefix 1..k in one pass: outs[j] has j+1 stages."""
+    lib = load_library()
+    if not 1 <= k <= pkg.n_stages:
+        raise ValueError(f"k must be in 1..{pkg.n_stages}")
+    outs = outs if outs is not None else _new_outs(pkg, k)
+    for o in outs:
+        if o.dtype != torch.bfloat16 or not o.is_cuda or not o.is_contiguous():
+            raise TypeError("outputs must be contiguous bfloat16 CUDA tensors")
+    rc = lib.rrq_reconstruct_prefixes(_ptrs(pkg.codes, k), _ptrs(pkg.scales, k), _ptrs(pkg.zeros, k),
+                                      pkg.rows, pkg.cols, pkg.group, k, _ptrs(outs, k),
+                                      _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_reconstruct_prefixes")
+    return outs
+
+
+def prefixes_items(pkgs, outs, k) -> ctypes.Array:
+    items = (PrefixesItem * len(pkgs))()
+    for it, pkg, o in zip(items, pkgs, outs):
+        for j in range(k):
+            it.codes[j] = pkg.codes[j].data_ptr()
+            it.scales[j] = pkg.scales[j].data_ptr()
+            it.zeros[j] = pkg.zeros[j].data_ptr()
+            if o[j].dtype != torch.bfloat16 or not o[j].is_cuda or not o[j].is_contiguous():
+                raise TypeError("outputs must be contiguous bfloat16 CUDA tensors")
+            it.out_bf16[j] = o[j].data_ptr()
+        it.rows, it.cols = pkg.rows, pkg.cols
+    return items
+
+
+def rrq_reconstruct_prefixes_batch(pkgs, k: int, outs=None, stream=None, items=None):
+    """rrq_reconstruct_prefixes for a list of packages: outs[i][j] is matrix
+    i's prefix with j+1 stages."""
+    lib = load_library()
+    if any(not 1 <= k <= p.n_stages for p in pkgs):
+        raise ValueError("k exceeds the stages of a package")
+    if outs is None:
+        outs = [_new_outs(p, k) for p in pkgs]
+    if items is None:
+        items = prefixes_items(pkgs, outs, k)
+    rc = lib.rrq_reconstruct_prefixes_batch(items, len(items), pkgs[0].group, k, _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_reconstruct_prefixes_batch")
     return outs
 
 

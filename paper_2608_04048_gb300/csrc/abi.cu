@@ -201,29 +201,43 @@ rrq_status quantize_batch(const rrq_quantize_item* items, int count, int group, 
 // ---------------------------------------------------------------------------
 // reconstruct
 // ---------------------------------------------------------------------------
-rrq_status check_reconstruct_item(const rrq_reconstruct_item& it, int group, int k) {
-  if (!it.out_bf16 || !shape_ok(it.rows, it.cols)) return RRQ_ERR_INVALID_ARG;
+// A reconstruct request for one matrix: k stages in, n_out outputs
+// (n_out = 1: the prefix with k stages; n_out = k: every prefix).
+struct ReconView {
+  const uint8_t* const* codes;
+  const float* const* scales;
+  const float* const* zeros;
+  int64_t rows, cols;
+  uint16_t* const* out;
+};
+
+rrq_status check_reconstruct_item(const ReconView& it, int group, int k, int n_out) {
+  if (!shape_ok(it.rows, it.cols)) return RRQ_ERR_INVALID_ARG;
   if (it.cols % group != 0) return RRQ_ERR_INVALID_ARG;
   for (int i = 0; i < k; ++i)
     if (!it.codes[i] || !it.scales[i] || !it.zeros[i]) return RRQ_ERR_INVALID_ARG;
-  if (!aligned(it.out_bf16, 16)) return RRQ_ERR_MISALIGNED;
+  for (int j = 0; j < n_out; ++j)
+    if (!it.out[j]) return RRQ_ERR_INVALID_ARG;
+  for (int j = 0; j < n_out; ++j)
+    if (!aligned(it.out[j], 16)) return RRQ_ERR_MISALIGNED;
   for (int i = 0; i < k; ++i)
     if (!aligned(it.codes[i], 16) || !aligned(it.scales[i], 16) || !aligned(it.zeros[i], 16))
       return RRQ_ERR_MISALIGNED;
   return RRQ_OK;
 }
 
-rrq_status reconstruct_batch(const rrq_reconstruct_item* items, int count, int group, int k,
+rrq_status reconstruct_views(const ReconView* items, int count, int group, int k, bool all_prefixes,
                              rrq_stream_t stream) {
   if (!items || count < 1 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
   if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  const int n_out = all_prefixes ? k : 1;
   std::vector<Range> ranges;
-  ranges.reserve(static_cast<size_t>(count) * (1 + 3 * k));
+  ranges.reserve(static_cast<size_t>(count) * (n_out + 3 * k));
   for (int i = 0; i < count; ++i) {
-    const rrq_reconstruct_item& it = items[i];
-    if (rrq_status rc = check_reconstruct_item(it, group, k)) return rc;
+    const ReconView& it = items[i];
+    if (rrq_status rc = check_reconstruct_item(it, group, k, n_out)) return rc;
     const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
-    ranges.push_back(range_of(it.out_bf16, 2 * n, true));
+    for (int j = 0; j < n_out; ++j) ranges.push_back(range_of(it.out[j], 2 * n, true));
     for (int j = 0; j < k; ++j) {
       ranges.push_back(range_of(it.codes[j], n / 4, false));
       ranges.push_back(range_of(it.scales[j], 4 * (n / group), false));
@@ -236,8 +250,9 @@ rrq_status reconstruct_batch(const rrq_reconstruct_item* items, int count, int g
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
   for (int i = 0; i < count; ++i) {
-    const rrq_reconstruct_item& it = items[i];
-    if (!on_device(it.out_bf16, dev)) return RRQ_ERR_INVALID_ARG;
+    const ReconView& it = items[i];
+    for (int j = 0; j < n_out; ++j)
+      if (!on_device(it.out[j], dev)) return RRQ_ERR_INVALID_ARG;
     for (int j = 0; j < k; ++j)
       if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) || !on_device(it.zeros[j], dev))
         return RRQ_ERR_INVALID_ARG;
@@ -252,21 +267,22 @@ rrq_status reconstruct_batch(const rrq_reconstruct_item* items, int count, int g
     p.status = st->status;
     int64_t chunks = 0;
     for (int i = 0; i < m; ++i) {
-      const rrq_reconstruct_item& it = items[base + i];
+      const ReconView& it = items[base + i];
       rrq::ReconstructItem& q = p.item[i];
       for (int j = 0; j < rrq::kMaxStages; ++j) {
         const int jj = j < k ? j : k - 1;
         q.codes[j] = it.codes[jj];
         q.scales[j] = it.scales[jj];
         q.zeros[j] = it.zeros[jj];
+        q.out[j] = it.out[j < n_out ? j : n_out - 1];
       }
-      q.out = it.out_bf16;
       q.n = it.rows * it.cols;
       q.chunk_begin = chunks;
       chunks += (q.n + rrq::kChunkElems - 1) / rrq::kChunkElems;
     }
     p.total_chunks = chunks;
-    cudaError_t e = rrq::reconstruct_launch(group, k, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+    cudaError_t e = rrq::reconstruct_launch(group, k, all_prefixes, p,
+                                            reinterpret_cast<cudaStream_t>(stream), st->sms);
     if (e != cudaSuccess) return fail_cuda(e);
   }
   return RRQ_OK;
@@ -318,22 +334,37 @@ rrq_status rrq_quantize_batch(const rrq_quantize_item* items, int count, int gro
 rrq_status rrq_reconstruct(const uint8_t* const codes[], const float* const scales[],
                            const float* const zeros[], int64_t rows, int64_t cols, int group,
                            int k, uint16_t* out_bf16, rrq_stream_t stream) {
-  if (!codes || !scales || !zeros || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
-  rrq_reconstruct_item it{};
-  for (int i = 0; i < k; ++i) {
-    it.codes[i] = codes[i];
-    it.scales[i] = scales[i];
-    it.zeros[i] = zeros[i];
-  }
-  it.rows = rows;
-  it.cols = cols;
-  it.out_bf16 = out_bf16;
-  return reconstruct_batch(&it, 1, group, k, stream);
+  if (!codes || !scales || !zeros || !out_bf16 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  uint16_t* const outs[1] = {out_bf16};
+  const ReconView v{codes, scales, zeros, rows, cols, outs};
+  return reconstruct_views(&v, 1, group, k, false, stream);
 }
 
 rrq_status rrq_reconstruct_batch(const rrq_reconstruct_item* items, int count, int group, int k,
                                  rrq_stream_t stream) {
-  return reconstruct_batch(items, count, group, k, stream);
+  if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  std::vector<ReconView> v(static_cast<size_t>(count));
+  for (int i = 0; i < count; ++i)
+    v[i] = {items[i].codes, items[i].scales, items[i].zeros, items[i].rows, items[i].cols, &items[i].out_bf16};
+  return reconstruct_views(v.data(), count, group, k, false, stream);
+}
+
+rrq_status rrq_reconstruct_prefixes(const uint8_t* const codes[], const float* const scales[],
+                                    const float* const zeros[], int64_t rows, int64_t cols,
+                                    int group, int k, uint16_t* const out_bf16[],
+                                    rrq_stream_t stream) {
+  if (!codes || !scales || !zeros || !out_bf16 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  const ReconView v{codes, scales, zeros, rows, cols, out_bf16};
+  return reconstruct_views(&v, 1, group, k, true, stream);
+}
+
+rrq_status rrq_reconstruct_prefixes_batch(const rrq_prefixes_item* items, int count, int group,
+                                          int k, rrq_stream_t stream) {
+  if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  std::vector<ReconView> v(static_cast<size_t>(count));
+  for (int i = 0; i < count; ++i)
+    v[i] = {items[i].codes, items[i].scales, items[i].zeros, items[i].rows, items[i].cols, items[i].out_bf16};
+  return reconstruct_views(v.data(), count, group, k, true, stream);
 }
 
 rrq_status rrq_get_device_status(rrq_stream_t stream) {

@@ -41,7 +41,9 @@ __device__ __forceinline__ bool prescale_ok(float s) {
   return s == 0.0f || (s >= 0x1p-100f && s <= 0x1p+100f);
 }
 
-template <int G, int K>
+// kAllPrefixes: write the reconstruction after every stage i < K (prefixes
+// 1..K in one pass over the package) instead of only after stage K-1.
+template <int G, int K, bool kAllPrefixes>
 __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_constant__ ReconstructBatch p) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31;
@@ -93,7 +95,7 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
 #pragma unroll
   for (int j = 0; j < kRing - 1; ++j) issue(first + j * stride, j);
 
-  uint32_t iter = 0;
+  uint32_t iter = 0, n_store = 0;
   for (int64_t chunk = first; chunk < p.total_chunks; chunk += stride, ++iter) {
     issue(chunk + (kRing - 1) * stride, (iter + kRing - 1) % kRing);
     cp_async_wait<kRing - 1>();  // this lane's copies of `chunk` have landed
@@ -110,14 +112,47 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
       ok = ok && prescale_ok(scale[i]);
     }
 
-    f32x2 acc[16];
-    if (__all_sync(kFullMask, ok)) {
+    const bool all_ok = __all_sync(kFullMask, ok);
+    const ReconstructItem& it = item_of(chunk, m_work);
+    const int64_t c0 = (chunk - it.chunk_begin) * kChunkElems;
+
+    // bf16 round-to-nearest-even of acc, staged in shared memory and written
+    // by one bulk copy (two staging buffers per warp, used in turn)
+    auto emit = [&](const f32x2 (&acc)[16], uint16_t* out) {
+      uint32_t outw[16];
 #pragma unroll
-      for (int i = 0; i < K; ++i) {
-        const uint32_t w0 = __byte_perm(code[i].x, code[i].y, sel_lo);
-        const uint32_t w1 = __byte_perm(code[i].x, code[i].y, sel_hi);
+      for (int m = 0; m < 16; ++m) {
+        float a, b;
+        unpack2(acc[m], a, b);
+        const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+        outw[m] = *reinterpret_cast<const uint32_t*>(&h);
+      }
+      const int bsel = n_store & 1;
+      ++n_store;
+      if (lane == 0) bulk_wait_read<1>();  // the store that last used this buffer has read it
+      __syncwarp();
+      uint4* dst = reinterpret_cast<uint4*>(stage_buf + bsel * kChunkBytes + lane * 64);
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        dst[(j + rot) & 3] = make_uint4(outw[4 * j], outw[4 * j + 1], outw[4 * j + 2], outw[4 * j + 3]);
+      fence_proxy_async_smem();
+      __syncwarp();
+      if (lane == 0) {
+        const int64_t left = it.n - c0;
+        const uint32_t bytes = static_cast<uint32_t>((left < kChunkElems ? left : kChunkElems) * 2);
+        bulk_store(out + c0, smem_u32(stage_buf + bsel * kChunkBytes), bytes);
+        bulk_commit();
+      }
+    };
+
+    f32x2 acc[16];
+#pragma unroll
+    for (int i = 0; i < K; ++i) {
+      const uint32_t w0 = __byte_perm(code[i].x, code[i].y, sel_lo);
+      const uint32_t w1 = __byte_perm(code[i].x, code[i].y, sel_hi);
+      const f32x2 LO = pack2(zero[i], zero[i]);
+      if (all_ok) {
         const float s = scale[i];
-        const f32x2 LO = pack2(zero[i], zero[i]);
         const f32x2 S01 = pack2(s, __fmul_rn(s, 0x1p-2f));
         const f32x2 S23 = pack2(__fmul_rn(s, 0x1p-4f), __fmul_rn(s, 0x1p-6f));
         const f32x2 C01 = pack2(__fmul_rn(s, -0x1p23f), __fmul_rn(s, -0x1p21f));
@@ -133,14 +168,8 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
           acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
           acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
         }
-      }
-    } else {
-      const f32x2 Z = pack2(0.0f, 0.0f), T23 = pack2(kTwo23, kTwo23);
-#pragma unroll
-      for (int i = 0; i < K; ++i) {
-        const uint32_t w0 = __byte_perm(code[i].x, code[i].y, sel_lo);
-        const uint32_t w1 = __byte_perm(code[i].x, code[i].y, sel_hi);
-        const f32x2 LO = pack2(zero[i], zero[i]);
+      } else {
+        const f32x2 Z = pack2(0.0f, 0.0f), T23 = pack2(kTwo23, kTwo23);
         const f32x2 S = pack2(scale[i], scale[i]);
 #pragma unroll
         for (int m = 0; m < 16; ++m) {
@@ -153,77 +182,57 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
           acc[m] = (i == 0) ? level : add2(acc[m], level);
         }
       }
+      if (kAllPrefixes) emit(acc, it.out[i]);
     }
-
-    // bf16 round-to-nearest-even, two weights per word
-    uint32_t outw[16];
-#pragma unroll
-    for (int m = 0; m < 16; ++m) {
-      float a, b;
-      unpack2(acc[m], a, b);
-      const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
-      outw[m] = *reinterpret_cast<const uint32_t*>(&h);
-    }
-
-    const ReconstructItem& it = item_of(chunk, m_work);
-    const int bsel = iter & 1;
-    if (lane == 0) bulk_wait_read<1>();  // the store that last used this buffer has read it
-    __syncwarp();
-    uint4* dst = reinterpret_cast<uint4*>(stage_buf + bsel * kChunkBytes + lane * 64);
-#pragma unroll
-    for (int j = 0; j < 4; ++j)
-      dst[(j + rot) & 3] = make_uint4(outw[4 * j], outw[4 * j + 1], outw[4 * j + 2], outw[4 * j + 3]);
-    fence_proxy_async_smem();
-    __syncwarp();
-    if (lane == 0) {
-      const int64_t e = (chunk - it.chunk_begin) * kChunkElems;
-      const int64_t left = it.n - e;
-      const uint32_t bytes = static_cast<uint32_t>((left < kChunkElems ? left : kChunkElems) * 2);
-      bulk_store(it.out + e, smem_u32(stage_buf + bsel * kChunkBytes), bytes);
-      bulk_commit();
-    }
+    if (!kAllPrefixes) emit(acc, it.out[0]);
   }
   cp_async_wait<0>();
   if (lane == 0) bulk_wait<0>();
 }
 
-template <int G, int K>
+template <int G, int K, bool A>
 cudaError_t launch_gk(const ReconstructBatch& p, cudaStream_t stream, int sms) {
   static int blocks_per_sm = 0;
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, reconstruct_kernel<G, K>, kThreads, smem_bytes<K>());
+        &blocks_per_sm, reconstruct_kernel<G, K, A>, kThreads, smem_bytes<K>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
   const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  reconstruct_kernel<G, K><<<grid, kThreads, smem_bytes<K>(), stream>>>(p);
+  reconstruct_kernel<G, K, A><<<grid, kThreads, smem_bytes<K>(), stream>>>(p);
   return cudaGetLastError();
 }
 
-template <int G>
+template <int G, bool A>
 cudaError_t launch_g(int k, const ReconstructBatch& p, cudaStream_t stream, int sms) {
   switch (k) {
-    case 1: return launch_gk<G, 1>(p, stream, sms);
-    case 2: return launch_gk<G, 2>(p, stream, sms);
-    case 3: return launch_gk<G, 3>(p, stream, sms);
-    case 4: return launch_gk<G, 4>(p, stream, sms);
+    case 1: return launch_gk<G, 1, A>(p, stream, sms);
+    case 2: return launch_gk<G, 2, A>(p, stream, sms);
+    case 3: return launch_gk<G, 3, A>(p, stream, sms);
+    case 4: return launch_gk<G, 4, A>(p, stream, sms);
     default: return cudaErrorInvalidValue;
   }
 }
 
-}  // namespace
+template <int G, bool A>
+cudaError_t prepare_ga() {
+  cudaError_t e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 1, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 2, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 3, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<3>()))) return e;
+  return cudaFuncSetAttribute(reconstruct_kernel<G, 4, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<4>());
+}
 
 template <int G>
 cudaError_t prepare_g() {
-  cudaError_t e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()))) return e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 2>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()))) return e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 3>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<3>()))) return e;
-  return cudaFuncSetAttribute(reconstruct_kernel<G, 4>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<4>());
+  cudaError_t e = prepare_ga<G, false>();
+  return e != cudaSuccess ? e : prepare_ga<G, true>();
 }
+
+}  // namespace
 
 cudaError_t reconstruct_prepare() {
   cudaError_t e;
@@ -233,13 +242,22 @@ cudaError_t reconstruct_prepare() {
   return prepare_g<256>();
 }
 
-cudaError_t reconstruct_launch(int group, int k, const ReconstructBatch& p, cudaStream_t stream,
-                               int sms) {
+cudaError_t reconstruct_launch(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                               cudaStream_t stream, int sms) {
+  if (all_prefixes) {
+    switch (group) {
+      case 32: return launch_g<32, true>(k, p, stream, sms);
+      case 64: return launch_g<64, true>(k, p, stream, sms);
+      case 128: return launch_g<128, true>(k, p, stream, sms);
+      case 256: return launch_g<256, true>(k, p, stream, sms);
+      default: return cudaErrorInvalidValue;
+    }
+  }
   switch (group) {
-    case 32: return launch_g<32>(k, p, stream, sms);
-    case 64: return launch_g<64>(k, p, stream, sms);
-    case 128: return launch_g<128>(k, p, stream, sms);
-    case 256: return launch_g<256>(k, p, stream, sms);
+    case 32: return launch_g<32, false>(k, p, stream, sms);
+    case 64: return launch_g<64, false>(k, p, stream, sms);
+    case 128: return launch_g<128, false>(k, p, stream, sms);
+    case 256: return launch_g<256, false>(k, p, stream, sms);
     default: return cudaErrorInvalidValue;
   }
 }

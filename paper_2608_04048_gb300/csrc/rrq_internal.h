@@ -43,7 +43,7 @@ struct ReconstructItem {
   const uint8_t* codes[kMaxStages];
   const float* scales[kMaxStages];
   const float* zeros[kMaxStages];
-  uint16_t* out;                   // bf16 bits, n elements
+  uint16_t* out[kMaxStages];       // bf16 bits, n elements; out[0] only unless all prefixes
   int64_t n;
   int64_t chunk_begin;
 };
@@ -62,7 +62,8 @@ cudaError_t reconstruct_prepare();
 
 // Launch on `stream`; `sms` = multiprocessor count of the current device.
 cudaError_t quantize_launch(int group, const QuantizeBatch& p, cudaStream_t stream, int sms);
-cudaError_t reconstruct_launch(int group, int k, const ReconstructBatch& p, cudaStream_t stream,
-                               int sms);
+// all_prefixes: write prefixes 1..k to out[0..k-1] (else prefix k to out[0]).
+cudaError_t reconstruct_launch(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                               cudaStream_t stream, int sms);
 
 }  // namespace rrq

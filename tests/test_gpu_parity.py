@@ -233,3 +233,32 @@ def test_batch_group_sizes(group):
         ref = oracle.quantize(bf16_bits(W), group, 3)
         assert_package_equal(gpu_package_host(pkg), ref, 3, f"batch g{group}")
         assert np.array_equal(bf16_bits(out), oracle.reconstruct(*ref, W.shape[0], W.shape[1], group, 3))
+
+
+@pytest.mark.parametrize("group", GROUPS)
+def test_prefixes_single_matches_oracle(group):
+    """rrq_reconstruct_prefixes: one pass writes every prefix, each equal to
+    the oracle's reconstruction with that many stages."""
+    W = _edge_matrix(24, 8 * group, group, seed=7 + group)
+    pkg = binding.rrq_quantize(W, group, 4)
+    for k in (1, 2, 3, 4):
+        outs = binding.rrq_reconstruct_prefixes(pkg, k)
+        torch.cuda.synchronize()
+        ref = oracle.quantize(bf16_bits(W), group, 4)
+        for j, o in enumerate(outs):
+            want = oracle.reconstruct(*ref, W.shape[0], W.shape[1], group, j + 1)
+            assert np.array_equal(bf16_bits(o), want), f"g{group} k={k} prefix {j + 1}"
+
+
+def test_prefixes_batch_matches_oracle():
+    rng = np.random.default_rng(3)
+    shapes = [(int(rng.integers(1, 30)), 128 * int(rng.integers(1, 10))) for _ in range(67)]
+    mats = [workloads.generate(r, c, 300 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+    pkgs = binding.rrq_quantize_batch(mats, group=128, n_stages=4)
+    outs = binding.rrq_reconstruct_prefixes_batch(pkgs, 4)
+    torch.cuda.synchronize()
+    for i, W in enumerate(mats):
+        ref = oracle.quantize(bf16_bits(W), 128, 4)
+        for j in range(4):
+            want = oracle.reconstruct(*ref, W.shape[0], W.shape[1], 128, j + 1)
+            assert np.array_equal(bf16_bits(outs[i][j]), want), f"item {i} prefix {j + 1}"
