@@ -262,6 +262,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
         return None
 
     peaks = measured_peaks()
+    clock_summary = clocks.summary()
     step_s = elapsed_ms / 1e3 / args.steps
     bytes_bf16 = 2.0 * n_total
     value = world * bytes_bf16 / step_s / 1e9
@@ -273,7 +274,6 @@ def run_gpu(args, world, rank, local) -> dict | None:
     q_gbs = q_alg / q_s / 1e9
     r_gbs = r_alg / r_s / 1e9
     dominant = "rrq_reconstruct_prefixes" if r_s > q_s else "rrq_quantize"
-    achieved = r_gbs if dominant == "rrq_reconstruct" else q_gbs
     per_launch = 64  # matrices per kernel launch of the batch entry points
     launches = math.ceil(len(specs) / per_launch) * 2
     traffic = recorded_traffic(dominant, q_alg / (launches / 2), r_alg / (launches / 2))
@@ -312,21 +312,40 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "quantize_frac_of_nominal_8tbs": round(q_gbs / 8000.0, 4),
             "paper_context_s": {"full_all_rtn_package_qwen3_8b_a100": 1293, "four_rtn_passes_a100": 412},
         },
-        "roofline": {
-            "kernel": dominant,
-            "bound": "hbm",
-            "achieved": round(achieved, 1),
-            "peak": peaks["hbm_gbs"],
-            "peak_source": f"{peaks['source']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
-            "unit": "GB/s",
-            "frac": round(achieved / peaks["hbm_gbs"], 4),
-            "traffic": traffic,
-        },
-        "clocks": clocks.summary(),
+        "roofline": roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic,
+                                   clock_summary.get("sm_mhz")),
+        "clocks": clock_summary,
         "gpu_launches": launches * args.steps,
         "e2e": e2e,
     }
     return line
+
+
+FP32_OPS_PER_WEIGHT_STAGE = 8   # d, q0, remainder, q1, t, fl(Q s), level, residual
+
+
+def fp32_peak_tops(sm_mhz: float | None) -> float:
+    """fp32 pipe peak in tera-operations/s: 152 SMs x 128 fp32 lanes x SM clock
+    (125 per SM per clock measured with a packed-fma throughput loop)."""
+    return 152 * 128 * (sm_mhz or 2070.0) * 1e6 / 1e12
+
+
+def roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic, sm_mhz=None):
+    """Roofline of the dominant kernel.  Quantize needs 32 fp32 operations per
+    3.25 algorithmic bytes (9.8 op/B): above the GB300 ridge (fp32 peak / HBM
+    bandwidth = 40.7 T / 6.69 TB/s = 6.1 op/B), so its bound is the fp32 pipe
+    ("alu"); reconstruction is bound by HBM."""
+    if dominant == "rrq_quantize":
+        ops = n_total * STAGES * FP32_OPS_PER_WEIGHT_STAGE
+        achieved = ops / q_s / 1e12
+        peak = fp32_peak_tops(sm_mhz)
+        return {"kernel": dominant, "bound": "alu", "achieved": round(achieved, 2), "peak": round(peak, 2),
+                "peak_source": "derived: 152 SMs x 128 fp32 lanes x SM clock (fp32 operations)",
+                "unit": "Top/s", "frac": round(achieved / peak, 4),
+                "hbm_frac_of_measured": round(q_gbs / peaks["hbm_gbs"], 4), "traffic": traffic}
+    return {"kernel": dominant, "bound": "hbm", "achieved": round(r_gbs, 1), "peak": peaks["hbm_gbs"],
+            "peak_source": f"{peaks['source']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+            "unit": "GB/s", "frac": round(r_gbs / peaks["hbm_gbs"], 4), "traffic": traffic}
 
 
 def recorded_traffic(kernel: str, q_bytes_per_launch: float, r_bytes_per_launch: float):
