@@ -8,7 +8,8 @@ and the two share no code.
 This module compiles ``rrq_oracle.c`` with gcc (``-O2 -ffp-contract=off``, no
 fast-math) and exposes it to numpy through ctypes.  The arithmetic itself lives
 in the C file, which cites the paper's equations step by step (Section 3.1
-Eq. 1-3, Section 3.2 Eq. 4-8, Algorithm 1).
+Eq. 1-3, Section 3.2 Eq. 4-8, Algorithm 1), for the asymmetric min/max grid
+and for the symmetric grid with binary32 or binary16 scales.
 
 Every function here is pinned by ``tests/test_oracle_pins.py`` (hand-worked
 groups, brute-force nearest level, invariants) and
@@ -80,6 +81,21 @@ class Oracle:
         lib.rrq_oracle_reconstruct.restype = ctypes.c_int
         lib.rrq_oracle_f32_to_bf16.argtypes = [ctypes.c_float]
         lib.rrq_oracle_f32_to_bf16.restype = ctypes.c_uint16
+        lib.rrq_oracle_quantize_group_sym.argtypes = [
+            _f32p, ctypes.c_int, ctypes.c_int, ctypes.c_int, _u8p, _f32p, _f32p]
+        lib.rrq_oracle_quantize_group_sym.restype = ctypes.c_int
+        lib.rrq_oracle_quantize_sym.argtypes = [
+            _u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            ctypes.POINTER(_u8p), ctypes.POINTER(ctypes.c_void_p)]
+        lib.rrq_oracle_quantize_sym.restype = ctypes.c_int
+        lib.rrq_oracle_reconstruct_sym.argtypes = [
+            ctypes.POINTER(_u8p), ctypes.POINTER(ctypes.c_void_p), ctypes.c_int64, ctypes.c_int64,
+            ctypes.c_int, ctypes.c_int, ctypes.c_int, _u16p]
+        lib.rrq_oracle_reconstruct_sym.restype = ctypes.c_int
+        lib.rrq_oracle_f32_to_f16.argtypes = [ctypes.c_float]
+        lib.rrq_oracle_f32_to_f16.restype = ctypes.c_uint16
+        lib.rrq_oracle_f16_to_f32.argtypes = [ctypes.c_uint16]
+        lib.rrq_oracle_f16_to_f32.restype = ctypes.c_float
         self.lib = lib
 
     # -- one group, float input, unpacked codes --------------------------------
@@ -136,6 +152,61 @@ class Oracle:
     def f32_to_bf16(self, f: float) -> int:
         return int(self.lib.rrq_oracle_f32_to_bf16(ctypes.c_float(f)))
 
+    def f32_to_f16(self, f: float) -> int:
+        return int(self.lib.rrq_oracle_f32_to_f16(ctypes.c_float(f)))
+
+    def f16_to_f32(self, h: int) -> float:
+        return float(self.lib.rrq_oracle_f16_to_f32(ctypes.c_uint16(h)))
+
+    # -- symmetric grid ----------------------------------------------------------
+    def quantize_group_sym(self, x, n_stages: int = 4, scale_f16: bool = False):
+        """Returns (Q[n_stages, g] uint8, scale[n_stages] f32 (the value used),
+        resid[n_stages, g] f32) for one group under the symmetric grid."""
+        x = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+        g = x.size
+        Q = np.zeros((n_stages, g), np.uint8)
+        s = np.zeros(n_stages, np.float32)
+        r = np.zeros((n_stages, g), np.float32)
+        rc = self.lib.rrq_oracle_quantize_group_sym(
+            x.ctypes.data_as(_f32p), g, n_stages, int(scale_f16), Q.ctypes.data_as(_u8p),
+            s.ctypes.data_as(_f32p), r.ctypes.data_as(_f32p))
+        if rc != 0:
+            raise ValueError("oracle rejected the group")
+        return Q, s, r
+
+    def quantize_sym(self, W_bits, group: int = 128, n_stages: int = 4, scale_f16: bool = True):
+        """Symmetric package of a bf16 matrix: (codes, scales) with scales
+        float32 arrays, or uint16 binary16 bit patterns when scale_f16."""
+        W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+        rows, cols = W_bits.shape
+        n = rows * cols
+        sdt = np.uint16 if scale_f16 else np.float32
+        codes = [np.zeros((n + 3) // 4, np.uint8) for _ in range(n_stages)]
+        scales = [np.zeros(n // group, sdt) for _ in range(n_stages)]
+        cp = (_u8p * n_stages)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (ctypes.c_void_p * n_stages)(*[a.ctypes.data for a in scales])
+        rc = self.lib.rrq_oracle_quantize_sym(W_bits.ctypes.data_as(_u16p), rows, cols, group,
+                                              n_stages, int(scale_f16), cp, sp)
+        if rc != 0:
+            raise ValueError("oracle rejected the matrix")
+        return codes, scales
+
+    def reconstruct_sym(self, codes, scales, rows: int, cols: int, group: int, k: int,
+                        scale_f16: bool = True):
+        """bf16 bit patterns [rows, cols] of the prefix-k reconstruction of a
+        symmetric package."""
+        sdt = np.uint16 if scale_f16 else np.float32
+        codes = [np.ascontiguousarray(c, dtype=np.uint8) for c in codes[:k]]
+        scales = [np.ascontiguousarray(a, dtype=sdt) for a in scales[:k]]
+        out = np.zeros((rows, cols), np.uint16)
+        cp = (_u8p * k)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (ctypes.c_void_p * k)(*[a.ctypes.data for a in scales])
+        rc = self.lib.rrq_oracle_reconstruct_sym(cp, sp, rows, cols, group, k, int(scale_f16),
+                                                 out.ctypes.data_as(_u16p))
+        if rc != 0:
+            raise ValueError("oracle rejected the reconstruction")
+        return out
+
 
 _default = None
 
@@ -158,3 +229,11 @@ def quantize(W_bits, group: int = 128, n_stages: int = 4):
 
 def reconstruct(codes, scales, zeros, rows, cols, group, k):
     return load().reconstruct(codes, scales, zeros, rows, cols, group, k)
+
+
+def quantize_sym(W_bits, group: int = 128, n_stages: int = 4, scale_f16: bool = True):
+    return load().quantize_sym(W_bits, group, n_stages, scale_f16)
+
+
+def reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16: bool = True):
+    return load().reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16)

@@ -34,6 +34,21 @@
  *   - Reconstruction sums stage values in stage order in binary32:
  *     acc = L_0; acc = fl(acc + L_i) for i = 1..k-1; then bf16 round to
  *     nearest-even.
+ *
+ * Symmetric grid (the paper's timed and packaged configuration: "symmetric"
+ * quantization type in Table 4, no stored zero-points and a 16-bit scale per
+ * group of 128 in Appendix G), readings where the paper gives no formula:
+ *   - the zero-point of Eq. 1-3 is the implicit constant z = 2 (half of the
+ *     4 levels), so the dequantized value of code Q is (Q - 2) * s and the
+ *     levels are {-2s, -s, 0, s};
+ *   - s = fl(fl(2 * amax) / 3) with amax = max |x| over the group, so that
+ *     the extreme magnitude sits 1.5 steps from 0;
+ *   - Q = clamp(rhe(fl(x / s)) + 2, 0, 3) (the clamp is active at the
+ *     positive end: fl(amax / s) rounds to 2); if s == 0 every code is 2;
+ *   - with 16-bit scales, s is rounded to IEEE binary16 (nearest-even) first
+ *     and the stage quantizes against the stored value, so that construction
+ *     and reconstruction use the same scale;
+ *   - (Q - 2) * s is exact in binary32, so the residual is fl(x - (Q-2)*s).
  */
 #include "rrq_oracle.h"
 
@@ -58,6 +73,49 @@ uint16_t rrq_oracle_f32_to_bf16(float f) {
   return (uint16_t)(u >> 16);
 }
 
+/* Round half to even of a double holding an integer plus a fraction that is
+ * exact (at most 53 significant bits, 0 <= u). */
+static double rhe_double(double u) {
+  double f = floor(u);
+  double frac = u - f;
+  if (frac > 0.5) return f + 1.0;
+  if (frac < 0.5) return f;
+  return (fmod(f, 2.0) == 0.0) ? f : f + 1.0;
+}
+
+/* IEEE 754 binary16 (1 sign, 5 exponent, 10 fraction bits, bias 15) nearest
+ * to f, ties to even; subnormals kept; magnitudes from 65520 (the midpoint
+ * between the largest finite 65504 and 2^16) up round to infinity. */
+uint16_t rrq_oracle_f32_to_f16(float f) {
+  const uint16_t sign = signbit(f) ? 0x8000u : 0u;
+  if (isnan(f)) return (uint16_t)(sign | 0x7e00u);
+  const double a = fabs((double)f);
+  if (a >= 65520.0) return (uint16_t)(sign | 0x7c00u);
+  if (a < ldexp(1.0, -14)) {
+    /* subnormal range: multiples of 2^-24; 1024 * 2^-24 is the smallest
+     * normal, whose encoding is 1024 as well */
+    const double n = rhe_double(a * ldexp(1.0, 24)); /* exact scaling */
+    return (uint16_t)(sign | (uint16_t)n);
+  }
+  int e;
+  const double m = frexp(a, &e); /* a = m * 2^e, 0.5 <= m < 1 */
+  int exp = e - 1;               /* a = (2m) * 2^exp, 1 <= 2m < 2 */
+  double frac = rhe_double((2.0 * m - 1.0) * 1024.0); /* 10 fraction bits */
+  if (frac == 1024.0) { frac = 0.0; exp += 1; }         /* rounded up to 2^(exp+1) */
+  if (exp + 15 >= 31) return (uint16_t)(sign | 0x7c00u);
+  return (uint16_t)(sign | (uint16_t)((exp + 15) << 10) | (uint16_t)frac);
+}
+
+float rrq_oracle_f16_to_f32(uint16_t h) {
+  const int e = (h >> 10) & 0x1f;
+  const int frac = h & 0x3ff;
+  double v;
+  if (e == 0) v = ldexp((double)frac, -24);
+  else if (e == 31) v = frac ? NAN : INFINITY;
+  else v = ldexp((double)(1024 + frac), e - 25);
+  return (float)((h & 0x8000u) ? -v : v);
+}
+
 /* a comes strictly before b in the order  ... < -0 < +0 < ...  */
 static int before(float a, float b) {
   if (a < b) return 1;
@@ -73,6 +131,16 @@ static float round_half_even(float u) {
   if (frac < 0.5f) return f;
   /* exact tie: go to the even neighbour */
   return (fmodf(f, 2.0f) == 0.0f) ? f : f + 1.0f;
+}
+
+/* element c's 2-bit code goes to byte c/4, bits 2*(c%4) and up */
+static void put_code(uint8_t* codes, int64_t c, int q) {
+  codes[c / 4] |= (uint8_t)(q << (2 * (c % 4)));
+}
+
+/* rhe for either sign: rounding half to even is odd-symmetric */
+static float round_half_even_signed(float u) {
+  return u < 0.0f ? -round_half_even(-u) : round_half_even(u);
 }
 
 int rrq_oracle_quantize_group(const float* x, int g, int n_stages, uint8_t* Q,
@@ -145,10 +213,7 @@ int rrq_oracle_quantize(const uint16_t* W, int64_t rows, int64_t cols, int group
     for (int j = 0; j < group; ++j) x[j] = rrq_oracle_bf16_to_f32(W[base + j]);
     rrq_oracle_quantize_group(x, group, n_stages, Q, s, z, NULL);
     for (int k = 0; k < n_stages; ++k) {
-      for (int j = 0; j < group; ++j) {
-        const int64_t c = base + j;
-        codes[k][c / 4] |= (uint8_t)(Q[(size_t)k * group + j] << (2 * (c % 4)));
-      }
+      for (int j = 0; j < group; ++j) put_code(codes[k], base + j, Q[(size_t)k * group + j]);
       scales[k][gi] = s[k];
       zeros[k][gi] = z[k];
     }
@@ -172,6 +237,96 @@ int rrq_oracle_reconstruct(const uint8_t* const* codes, const float* const* scal
       float qs = (float)q * scales[i][gi];
       float value = zeros[i][gi] + qs; /* stage i's dequantized value */
       acc = (i == 0) ? value : acc + value;
+    }
+    out[c] = rrq_oracle_f32_to_bf16(acc);
+  }
+  return 0;
+}
+
+int rrq_oracle_quantize_group_sym(const float* x, int g, int n_stages, int scale_f16,
+                                  uint8_t* Q, float* scale, float* resid) {
+  if (g < 1 || n_stages < 1 || !x || !Q || !scale) return -1;
+  float* v = (float*)malloc(sizeof(float) * (size_t)g);
+  if (!v) return -1;
+  for (int j = 0; j < g; ++j) v[j] = x[j];
+
+  for (int k = 0; k < n_stages; ++k) {
+    /* largest magnitude of the values this stage quantizes */
+    float amax = 0.0f;
+    for (int j = 0; j < g; ++j)
+      if (fabsf(v[j]) > amax) amax = fabsf(v[j]);
+    float span = 2.0f * amax; /* exact: power-of-two scaling */
+    float s = span / 3.0f;    /* levels -2s..s: amax is 1.5 steps from 0 */
+    if (scale_f16) s = rrq_oracle_f16_to_f32(rrq_oracle_f32_to_f16(s));
+
+    for (int j = 0; j < g; ++j) {
+      int code = 2; /* implicit zero-point */
+      if (s != 0.0f) {
+        float u = v[j] / s; /* Eq. 1 with z = 2 applied after rounding */
+        code = (int)round_half_even_signed(u) + 2;
+        code = code < 0 ? 0 : code;
+        code = code > 3 ? 3 : code;
+      }
+      Q[(size_t)k * g + j] = (uint8_t)code;
+      float level = (float)(code - 2) * s; /* (Q - z) s, Eq. 3; exact */
+      v[j] = v[j] - level;
+    }
+    scale[k] = s;
+    if (resid)
+      for (int j = 0; j < g; ++j) resid[(size_t)k * g + j] = v[j];
+  }
+  free(v);
+  return 0;
+}
+
+int rrq_oracle_quantize_sym(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                            int n_stages, int scale_f16, uint8_t* const* codes,
+                            void* const* scales) {
+  if (!W || !codes || !scales) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || n_stages < 1) return -1;
+  if (cols % group != 0) return -1;
+  const int64_t n = rows * cols;
+  const int64_t n_groups = n / group;
+
+  float* x = (float*)malloc(sizeof(float) * (size_t)group);
+  uint8_t* Q = (uint8_t*)malloc((size_t)n_stages * (size_t)group);
+  float* s = (float*)malloc(sizeof(float) * (size_t)n_stages);
+  if (!x || !Q || !s) {
+    free(x); free(Q); free(s);
+    return -1;
+  }
+  for (int k = 0; k < n_stages; ++k) memset(codes[k], 0, (size_t)((n + 3) / 4));
+
+  for (int64_t gi = 0; gi < n_groups; ++gi) {
+    const int64_t base = gi * group;
+    for (int j = 0; j < group; ++j) x[j] = rrq_oracle_bf16_to_f32(W[base + j]);
+    rrq_oracle_quantize_group_sym(x, group, n_stages, scale_f16, Q, s, NULL);
+    for (int k = 0; k < n_stages; ++k) {
+      for (int j = 0; j < group; ++j) put_code(codes[k], base + j, Q[(size_t)k * group + j]);
+      if (scale_f16) ((uint16_t*)scales[k])[gi] = rrq_oracle_f32_to_f16(s[k]);
+      else ((float*)scales[k])[gi] = s[k];
+    }
+  }
+  free(x); free(Q); free(s);
+  return 0;
+}
+
+int rrq_oracle_reconstruct_sym(const uint8_t* const* codes, const void* const* scales,
+                               int64_t rows, int64_t cols, int group, int k, int scale_f16,
+                               uint16_t* out) {
+  if (!codes || !scales || !out) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || k < 1) return -1;
+  if (cols % group != 0) return -1;
+  const int64_t n = rows * cols;
+  for (int64_t c = 0; c < n; ++c) {
+    const int64_t gi = c / group;
+    float acc = 0.0f;
+    for (int i = 0; i < k; ++i) {
+      const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;
+      const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])
+                                : ((const float*)scales[i])[gi];
+      float level = (float)(q - 2) * s; /* stage i's dequantized value */
+      acc = (i == 0) ? level : acc + level;
     }
     out[c] = rrq_oracle_f32_to_bf16(acc);
   }

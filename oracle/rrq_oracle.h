@@ -48,9 +48,32 @@ int rrq_oracle_reconstruct(const uint8_t* const* codes, const float* const* scal
                            const float* const* zeros, int64_t rows, int64_t cols,
                            int group, int k, uint16_t* out);
 
-/* The two scalar conversions the oracle uses, exported for tests. */
+/* Symmetric grid (levels (Q-2)*s, s = 2*max|x|/3, no zero stored; see
+ * rrq_oracle.c).  scale_f16 != 0 rounds each scale to binary16 and
+ * quantizes against the rounded value.
+ *   scale  [n_stages]  the scale each stage used (a binary16 value when
+ *                      scale_f16), as binary32 */
+int rrq_oracle_quantize_group_sym(const float* x, int g, int n_stages, int scale_f16,
+                                  uint8_t* Q, float* scale, float* resid);
+
+/* Matrix form of the symmetric grid: codes[k] as for rrq_oracle_quantize;
+ * scales[k] is float[rows*cols/group], or uint16_t binary16 bit patterns
+ * when scale_f16. */
+int rrq_oracle_quantize_sym(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                            int n_stages, int scale_f16, uint8_t* const* codes,
+                            void* const* scales);
+
+/* Prefix-k reconstruction of a symmetric package:
+ * acc = (Q_0 - 2) s_0; acc = fl(acc + (Q_i - 2) s_i); bf16. */
+int rrq_oracle_reconstruct_sym(const uint8_t* const* codes, const void* const* scales,
+                               int64_t rows, int64_t cols, int group, int k, int scale_f16,
+                               uint16_t* out);
+
+/* The scalar conversions the oracle uses, exported for tests. */
 float rrq_oracle_bf16_to_f32(uint16_t h);
 uint16_t rrq_oracle_f32_to_bf16(float f);
+uint16_t rrq_oracle_f32_to_f16(float f);
+float rrq_oracle_f16_to_f32(uint16_t h);
 
 #ifdef __cplusplus
 }

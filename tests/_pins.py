@@ -15,7 +15,11 @@ Sources of truth:
     checked with exact rationals;
   * invariants of the method: half-step bound per stage, exact reconstruction
     of groups already on a 4-level grid, L-infinity error shrinking by >= 3x
-    per stage (Eq. 5-8), prefix reconstruction equal to input minus residual.
+    per stage (Eq. 5-8), prefix reconstruction equal to input minus residual;
+  * library conversions: bf16 rounding against torch, binary16 rounding
+    against numpy's float16.
+The symmetric grid (levels (Q-2)s, s = 2 max|x| / 3, binary32 or binary16
+scales) has its own worked groups, brute force and invariants below.
 """
 from __future__ import annotations
 
@@ -333,8 +337,255 @@ def pin_bf16_rounding(orc, seed=13, count=4000) -> list[str]:
     return [f"bf16({hex(int(u[i]))}) = {hex(int(got[i]))}, want {hex(int(want[i]))}" for i in bad[:5]]
 
 
+def pin_f16_rounding(orc, seed=17, count=6000) -> list[str]:
+    """The oracle's binary32 -> binary16 conversion is IEEE round-to-nearest-
+    even with subnormals and overflow to infinity, the same as numpy's
+    float16 cast (a library routine): random values across the whole binary16
+    range, exact ties (normal and subnormal), and the edges 65504 / 65520 /
+    2^-24 / 2^-25.  binary16 -> binary32 is checked for every finite pattern."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    # random binary32 values whose exponent lands around the binary16 range
+    e = rng.integers(127 - 30, 127 + 17, count).astype(np.uint32)
+    u = (rng.integers(0, 2, count).astype(np.uint32) << 31) | (e << 23) | \
+        rng.integers(0, 2 ** 23, count).astype(np.uint32)
+    # exact ties: a binary16 value plus half its spacing
+    h = rng.integers(0, 0x7BFF, 400).astype(np.uint16)
+    lo = h.view(np.float16).astype(np.float64)
+    hi = (h + 1).astype(np.uint16).view(np.float16).astype(np.float64)
+    ties = ((lo + hi) / 2).astype(np.float32)  # exact: at most 12 significant bits
+    edges = np.array([65504.0, 65519.99, 65520.0, 65536.0, 2.0 ** -24, 2.0 ** -25,
+                      2.0 ** -25 * 1.0000001, 3 * 2.0 ** -26, 2.0 ** -14, 0.0, -0.0, 1e-30],
+                     np.float32)
+    f = np.concatenate([u.view(np.float32), ties, -ties, edges])
+    with np.errstate(over="ignore"):
+        want = f.astype(np.float16).view(np.uint16)
+    got = np.array([orc.f32_to_f16(float(v)) for v in f], np.uint16)
+    for i in np.nonzero(got != want)[0][:5]:
+        fails.append(f"f16({f[i]!r}) = {hex(int(got[i]))}, want {hex(int(want[i]))}")
+    allh = np.arange(0, 0x10000, dtype=np.uint32).astype(np.uint16)
+    allh = allh[(allh & 0x7C00) != 0x7C00]
+    wantf = allh.view(np.float16).astype(np.float32)
+    gotf = np.array([orc.f16_to_f32(int(x)) for x in allh], np.float32)
+    bad = np.nonzero(gotf.view(np.uint32) != wantf.view(np.uint32))[0]
+    for i in bad[:5]:
+        fails.append(f"f16 decode {hex(int(allh[i]))} = {gotf[i]!r}, want {wantf[i]!r}")
+    return fails
+
+
+# ---------------------------------------------------------------------------
+# symmetric grid: hand-worked groups
+# ---------------------------------------------------------------------------
+# WS1 (binary32 scales), x = [-1.5, -1, 0.5, 1.5]:
+#   stage 0: amax = 1.5, s = fl(3/3) = 1; x/s = -1.5 -> rhe -2 -> Q 0;
+#            -1 -> Q 1; 0.5 -> rhe 0 (tie to even) -> Q 2; 1.5 -> rhe 2 ->
+#            Q 4, clamped to 3 (level s = 1).  r = [0.5, 0, 0.5, 0.5].
+#   stage 1: amax = 0.5, s = fl(1/3) = 0x3EAAAAAB; fl(0.5/s) = 1.5 exactly
+#            (0.49999998 / 0.33333334 = 1.49999996, within half an ulp of
+#            1.5), so rhe gives 2 and the clamp 3; 0 -> Q 2.
+#            r = 0.5 - s = 0x3E2AAAAA (exact), and 0.
+#   prefix k=1: (Q-2)s = [-2, -1, 0, 1]; k=2 adds [s, 0, s, s]:
+#            fl(-2 + s) = 0xBFD55555 -> bf16 0xBFD5; s -> 0x3EAB;
+#            fl(1 + s) = 0x3FAAAAAB -> 0x3FAB.
+WS1 = dict(x=[-1.5, -1.0, 0.5, 1.5], Q=[[0, 1, 2, 3], [3, 2, 3, 3]],
+           scale_bits=[0x3F800000, 0x3EAAAAAB],
+           resid_bits=[[0x3F000000, 0x00000000, 0x3F000000, 0x3F000000],
+                       [0x3E2AAAAA, 0x00000000, 0x3E2AAAAA, 0x3E2AAAAA]],
+           recon=[[0xC000, 0xBF80, 0x0000, 0x3F80], [0xBFD5, 0xBF80, 0x3EAB, 0x3FAB]])
+# WS2 (binary16 scales), a = 0.10009765625 = 1640 * 2^-14 (bf16 0x3DCD),
+# x = [a, 0, -a, a/2]:
+#   stage 0: fl(2a/3) = 0.066731770..., as binary16 (spacing 2^-14 in
+#            [2^-4, 2^-3)) 1093.33 * 2^-14 -> 1093 * 2^-14 = 0x2C45.
+#            In units of 2^-14: 1640/1093 = 1.5005 -> rhe 2 -> Q 3, r = 547;
+#            0 -> Q 2, r = 0; -1.5005 -> rhe -2 -> Q 0, r = -1640 + 2186 = 546;
+#            820/1093 = 0.750 -> rhe 1 -> Q 3, r = 820 - 1093 = -273.
+#            (547 > 1093/2: rounding the scale down to binary16 lets the top
+#            element exceed the half step.)
+#   stage 1: amax = 547 * 2^-14; fl(2*547/3 * 2^-14) in binary16 (spacing
+#            2^-16 in [2^-6, 2^-5)): 1458.67 * 2^-16 -> 1459 * 2^-16 = 0x25B3.
+#            In units of 2^-16, r = [2188, 0, 2184, -1092]:
+#            2188/1459 = 1.4997 -> rhe 1 -> Q 3, r = 729; 0 -> Q 2;
+#            2184/1459 = 1.4969 -> Q 3, r = 725; -1092/1459 = -0.748 -> rhe -1
+#            -> Q 1, r = -1092 + 1459 = 367.
+WS2 = dict(x=[0.10009765625, 0.0, -0.10009765625, 0.050048828125],
+           Q=[[3, 2, 0, 3], [3, 2, 3, 1]], scale_f16=[0x2C45, 0x25B3],
+           resid=[[547 * 2.0 ** -14, 0.0, 546 * 2.0 ** -14, -273 * 2.0 ** -14],
+                  [729 * 2.0 ** -16, 0.0, 725 * 2.0 ** -16, 367 * 2.0 ** -16]])
+# WS3: x = [-3, -1, 0.75, 1.5]: amax 3, s = 2; x/s = [-1.5, -0.5, 0.375, 0.75]
+#   -> rhe [-2, -0 (tie to even), 0, 1] -> Q [0, 2, 2, 3];
+#   levels [-4, 0, 0, 2], r = [1, -1, 0.75, -0.5] (|r| = s/2 at the ties).
+WS3 = dict(x=[-3.0, -1.0, 0.75, 1.5], Q0=[0, 2, 2, 3], scale0=2.0, resid0=[1.0, -1.0, 0.75, -0.5])
+
+
+def pin_sym_worked_groups(orc) -> list[str]:
+    fails = []
+    Q, s, r = orc.quantize_group_sym(np.array(WS1["x"], np.float32), 2, False)
+    if Q.tolist() != WS1["Q"]:
+        fails.append(f"WS1: codes {Q.tolist()}")
+    if [bits_of(v) for v in s] != WS1["scale_bits"]:
+        fails.append(f"WS1: scales {[hex(bits_of(v)) for v in s]}")
+    if [[bits_of(v) for v in row] for row in r] != WS1["resid_bits"]:
+        fails.append(f"WS1: residuals {[[hex(bits_of(v)) for v in row] for row in r]}")
+    W = bf16_bits_of_f32(np.array(WS1["x"], np.float32)).reshape(1, 4)
+    codes, scales = orc.quantize_sym(W, group=4, n_stages=2, scale_f16=False)
+    for k in (1, 2):
+        rec = orc.reconstruct_sym(codes, scales, 1, 4, 4, k, scale_f16=False)[0]
+        if rec.tolist() != WS1["recon"][k - 1]:
+            fails.append(f"WS1: recon k={k} {[hex(v) for v in rec]}")
+
+    Q, s, r = orc.quantize_group_sym(np.array(WS2["x"], np.float32), 2, True)
+    if Q.tolist() != WS2["Q"]:
+        fails.append(f"WS2: codes {Q.tolist()}")
+    if [orc.f32_to_f16(float(v)) for v in s] != WS2["scale_f16"]:
+        fails.append(f"WS2: scales {[float(v) for v in s]}")
+    if r.astype(np.float64).tolist() != WS2["resid"]:
+        fails.append(f"WS2: residuals {r.tolist()}")
+    W = bf16_bits_of_f32(np.array(WS2["x"], np.float32)).reshape(1, 4)
+    codes, scales = orc.quantize_sym(W, group=4, n_stages=2, scale_f16=True)
+    if [int(a[0]) for a in scales] != WS2["scale_f16"]:
+        fails.append(f"WS2: stored binary16 scales {[hex(int(a[0])) for a in scales]}")
+    packed = [int(c[0]) for c in codes]
+    want = [sum(q << (2 * j) for j, q in enumerate(row)) for row in WS2["Q"]]
+    if packed != want:
+        fails.append(f"WS2: packed {packed} != {want}")
+
+    Q, s, r = orc.quantize_group_sym(np.array(WS3["x"], np.float32), 1, False)
+    if Q[0].tolist() != WS3["Q0"] or float(s[0]) != WS3["scale0"] or r[0].tolist() != WS3["resid0"]:
+        fails.append(f"WS3: {Q[0].tolist()} {s[0]} {r[0].tolist()}")
+
+    # signed zeros only: s = 0, every code 2, residual keeps each sign,
+    # reconstruction +0
+    x = np.array([-0.0, 0.0, -0.0, 0.0], np.float32)
+    for f16 in (False, True):
+        Q, s, r = orc.quantize_group_sym(x, 4, f16)
+        if (Q != 2).any() or (s != 0).any() or [bits_of(v) for v in r[3]] != [0x80000000, 0, 0x80000000, 0]:
+            fails.append(f"zero group f16={f16}: {Q.tolist()} {s.tolist()} {[hex(bits_of(v)) for v in r[3]]}")
+    return fails
+
+
+# ---------------------------------------------------------------------------
+# symmetric grid: brute force and invariants
+# ---------------------------------------------------------------------------
+def pin_sym_brute_force_exact(orc, seed=19, count=300) -> list[str]:
+    """Dyadic groups with amax = 1.5 * 2^e, so s = 2^e exactly (also as
+    binary16), and values m * 2^(e-2), |m| <= 6: every step is exact.  Each
+    code must select the level of {-2s, -s, 0, s} nearest the value, an exact
+    tie going to the even code, and the residual must be exact."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    for _ in range(count):
+        g = int(rng.integers(2, 17))
+        e = int(rng.integers(-6, 4))
+        ms = list(rng.integers(-6, 7, size=g))
+        ms[0] = 6 if rng.random() < 0.5 else -6
+        rng.shuffle(ms)
+        s = Fraction(2) ** e
+        xs = [Fraction(int(m)) * Fraction(2) ** (e - 2) for m in ms]
+        x = np.array([float(v) for v in xs], np.float32)
+        for f16 in (False, True):
+            Q, sc, r = orc.quantize_group_sym(x, 1, f16)
+            if Fraction(float(sc[0])) != s:
+                fails.append(f"sym exact: s={sc[0]} want {float(s)}")
+                break
+            for j, v in enumerate(xs):
+                dist = [abs(v - (q - 2) * s) for q in range(4)]
+                best = min(dist)
+                cands = [q for q in range(4) if dist[q] == best]
+                want = cands[0] if len(cands) == 1 else [q for q in cands if q % 2 == 0][0]
+                if int(Q[0, j]) != want:
+                    fails.append(f"sym nearest level: x={float(v)} s={float(s)} Q={int(Q[0, j])} want {want}")
+                    break
+                if Fraction(float(r[0, j])) != v - (want - 2) * s:
+                    fails.append(f"sym exact residual wrong at x={float(v)}")
+                    break
+        if len(fails) > 5:
+            break
+    return fails
+
+
+def _is_f16(v) -> bool:
+    return float(np.float32(v).astype(np.float16)) == float(v)
+
+
+def pin_sym_invariants(orc, seed=23, count=120, g=128) -> list[str]:
+    """Random bf16 groups (Gaussian, Student-t, outliers), 4 stages:
+    s_k = 2 max|r_{k-1}| / 3 to binary32 rounding (binary16: to half a
+    binary16 spacing, and representable); |r_k| <= s_k / 2 up to rounding
+    (binary16: up to the scale's relative rounding, 2^-11, times 1.5);
+    max |r_k| <= max |r_{k-1}| / 3 up to the same; codes in 0..3."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    for x in _random_groups(rng, count, g):
+        for f16 in (False, True):
+            Q, s, r = orc.quantize_group_sym(x, 4, f16)
+            prev = x.astype(np.float64)
+            for k in range(4):
+                amax = float(np.max(np.abs(prev)))
+                sk = float(s[k])
+                ideal = 2 * amax / 3
+                rel = 2.0 ** -11 if f16 else 2.0 ** -23
+                if abs(sk - ideal) > rel * ideal * 1.01 + (2.0 ** -25 if f16 else 1e-45):
+                    fails.append(f"sym stage {k} f16={f16}: scale {sk} vs 2*amax/3 {ideal}")
+                if f16 and not _is_f16(sk):
+                    fails.append(f"sym stage {k}: scale {sk} not a binary16 value")
+                rk = r[k].astype(np.float64)
+                slack = 3 * rel + 2.0 ** -22
+                if np.max(np.abs(rk)) > 0.5 * sk * (1 + slack) + 1e-45:
+                    fails.append(f"sym stage {k} f16={f16}: |r| {np.max(np.abs(rk))} > s/2 {0.5 * sk}")
+                if np.max(np.abs(rk)) > amax / 3 * (1 + 2 * slack) + 1e-45:
+                    fails.append(f"sym stage {k} f16={f16}: max|r| not reduced 3x")
+                lev = (Q[k].astype(np.float64) - 2) * sk
+                if np.max(np.abs(prev - lev - rk)) > 2.0 ** -23 * amax + 1e-45:
+                    fails.append(f"sym stage {k}: residual is not value minus level")
+                prev = rk
+            if len(fails) > 5:
+                return fails
+    return fails
+
+
+def pin_sym_prefix_reconstruction(orc, seed=29, rows=5, g=64) -> list[str]:
+    """Eq. 8 for the symmetric package: packed codes and stored scales equal
+    the per-group results (binary16 scales stored as their bit patterns), and
+    the prefix-k reconstruction is x minus the residual after stage k-1 up to
+    summation and bf16 rounding."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 3 * g
+    xs = np.concatenate(_random_groups(rng, rows * 3, g)).reshape(rows, cols)
+    W = bf16_bits_of_f32(xs)
+    n = rows * cols
+    for f16 in (False, True):
+        codes, scales = orc.quantize_sym(W, group=g, n_stages=4, scale_f16=f16)
+        resid = []
+        for gi in range(n // g):
+            x = xs.reshape(-1)[gi * g:(gi + 1) * g]
+            Q, s, r = orc.quantize_group_sym(x, 4, f16)
+            resid.append(r)
+            c = np.arange(gi * g, (gi + 1) * g)
+            for k in range(4):
+                if not np.array_equal((codes[k][c // 4] >> (2 * (c % 4))) & 3, Q[k]):
+                    fails.append(f"sym group {gi} stage {k}: packed codes disagree")
+                stored = orc.f16_to_f32(int(scales[k][gi])) if f16 else float(scales[k][gi])
+                if bits_of(stored) != bits_of(s[k]):
+                    fails.append(f"sym group {gi} stage {k}: stored scale disagrees")
+        for k in range(1, 5):
+            rec = orc.reconstruct_sym(codes, scales, rows, cols, g, k, scale_f16=f16).reshape(-1)
+            recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+            for gi in range(n // g):
+                x = xs.reshape(-1)[gi * g:(gi + 1) * g].astype(np.float64)
+                want = x - resid[gi][k - 1]
+                err = np.abs(recf[gi * g:(gi + 1) * g] - want)
+                tol = np.abs(want) * 2 ** -8 + 8 * 2 ** -24 * (np.abs(x).max() + 1e-30)
+                if np.any(err > tol):
+                    fails.append(f"sym group {gi} f16={f16}: prefix k={k} is not x - r_(k-1)")
+                    break
+    return fails
+
+
 ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_brute_force_tiny,
-            pin_invariants, pin_exact_grid, pin_prefix_reconstruction]
+            pin_invariants, pin_exact_grid, pin_prefix_reconstruction, pin_f16_rounding,
+            pin_sym_worked_groups, pin_sym_brute_force_exact, pin_sym_invariants,
+            pin_sym_prefix_reconstruction]
 
 
 def all_failures(orc) -> list[str]:

@@ -23,8 +23,8 @@ MUTANTS = {
     "transposed_difference": ("float d = v[j] - lo;", "float d = lo - v[j];"),
     "zero_sign_order_ignored": ("if (a == b && signbit(a) && !signbit(b)) return 1;", ""),
     "no_clamp": ("if (code > 3) code = 3;", "if (code > 4) code = 4;"),
-    "packing_bit_order": ("codes[k][c / 4] |= (uint8_t)(Q[(size_t)k * group + j] << (2 * (c % 4)));",
-                          "codes[k][c / 4] |= (uint8_t)(Q[(size_t)k * group + j] << (2 * (3 - c % 4)));"),
+    "packing_bit_order": ("codes[c / 4] |= (uint8_t)(q << (2 * (c % 4)));",
+                          "codes[c / 4] |= (uint8_t)(q << (2 * (3 - c % 4)));"),
     "recon_drops_base": ("acc = (i == 0) ? value : acc + value;", "acc = (i == 0) ? 0.0f : acc + value;"),
     "recon_bf16_truncates": ("u += 0x7fffu + ((u >> 16) & 1u);", ""),
     "max_is_min": ("if (before(hi, v[j])) hi = v[j];", "if (before(v[j], hi)) hi = v[j];"),
@@ -32,6 +32,21 @@ MUTANTS = {
                                     "if (before(x[j], lo)) lo = x[j];\n      if (before(hi, x[j])) hi = x[j];"),
     "scale_rounds_range_twice": ("float range = hi - lo;", "float range = (float)(double)(hi - lo) * 1.0000001f;"),
     "level_from_code_minus_one": ("float qs = (float)q * s;\n      level[q]", "float qs = (float)(q > 0 ? q - 1 : 0) * s;\n      level[q]"),
+    # symmetric grid and binary16 scales
+    "sym_zero_point_one": ("code = (int)round_half_even_signed(u) + 2;", "code = (int)round_half_even_signed(u) + 1;"),
+    "sym_no_top_clamp": ("code = code > 3 ? 3 : code;", "code = code & 3;"),
+    "sym_scale_not_rounded_to_f16": ("if (scale_f16) s = rrq_oracle_f16_to_f32(rrq_oracle_f32_to_f16(s));", ""),
+    "sym_span_not_doubled": ("float span = 2.0f * amax;", "float span = amax;"),
+    "sym_round_half_up": ("return u < 0.0f ? -round_half_even(-u) : round_half_even(u);", "return floorf(u + 0.5f);"),
+    "sym_amax_signed": ("if (fabsf(v[j]) > amax) amax = fabsf(v[j]);", "if (v[j] > amax) amax = v[j];"),
+    "sym_level_without_zero_point": ("float level = (float)(code - 2) * s;", "float level = (float)code * s;"),
+    "sym_recon_zero_point_one": ("float level = (float)(q - 2) * s;", "float level = (float)(q - 1) * s;"),
+    "sym_recon_drops_base": ("acc = (i == 0) ? level : acc + level;", "acc = (i == 0) ? 0.0f : acc + level;"),
+    "f16_truncates": ("double frac = rhe_double((2.0 * m - 1.0) * 1024.0);", "double frac = floor((2.0 * m - 1.0) * 1024.0);"),
+    "f16_bias_14": ("(uint16_t)((exp + 15) << 10)", "(uint16_t)((exp + 14) << 10)"),
+    "f16_flushes_subnormals": ("const double n = rhe_double(a * ldexp(1.0, 24));", "const double n = 0.0;"),
+    "f16_decode_exponent": ("else v = ldexp((double)(1024 + frac), e - 25);", "else v = ldexp((double)(1024 + frac), e - 24);"),
+    "f16_ties_away": ("return (fmod(f, 2.0) == 0.0) ? f : f + 1.0;", "return f + 1.0;"),
 }
 
 
