@@ -60,7 +60,8 @@ typedef enum {
   RRQ_ERR_INVALID_ARG = 1, /* null pointer, non-positive size, cols % group != 0,
                               n_stages or k out of range, pointer not device memory
                               of the current device, aliasing outputs */
-  RRQ_ERR_UNSUPPORTED = 2, /* group not in {32, 64, 128, 256} */
+  RRQ_ERR_UNSUPPORTED = 2, /* group not in {32, 64, 128, 256}, or a format
+                              combination the library does not build */
   RRQ_ERR_MISALIGNED = 3,  /* a pointer breaks the alignment stated below */
   RRQ_ERR_CUDA = 4,        /* a CUDA runtime call or kernel launch failed; see
                               rrq_last_cuda_error() */
@@ -162,6 +163,94 @@ typedef struct {
  * kernel launch per 64 matrices. */
 rrq_status rrq_reconstruct_prefixes_batch(const rrq_prefixes_item* items, int count, int group,
                                           int k, rrq_stream_t stream);
+
+/* ------------------------------------------------------------------------
+ * Package formats.  The calls above build and read the asymmetric package
+ * with binary32 scales and zeros.  The format-generic calls below also build
+ * and read the symmetric package, the paper's timed and stored
+ * configuration ("symmetric" quantization type, Table 4; no stored
+ * zero-points and a 16-bit scale per group of 128, Appendix G).
+ *
+ * Symmetric grid (RRQ_GRID_SYM), per group and stage (bit for bit; binary32
+ * steps rounded to nearest-even):
+ *     amax = max |v| over the group
+ *     s    = fl(fl(2 * amax) / 3)          amax sits 1.5 steps from 0
+ *     s    = binary16_rne(s)               only with RRQ_SCALE_F16: the stage
+ *                                          quantizes against the stored scale
+ *     Q    = s == 0 ? 2 : clamp(rhe(fl(v / s)) + 2, 0, 3)
+ *     L    = (Q - 2) * s                   levels -2s, -s, 0, s (exact)
+ *     v'   = fl(v - L)
+ *   The zero-point is the implicit constant 2 (Eq. 1-3 with z = 2): nothing
+ *   is stored for it.  Reconstruction: acc = L_0; acc = fl(acc + L_i);
+ *   bf16 round-to-nearest-even.  Inputs need 2 * max|W| finite; with
+ *   RRQ_SCALE_F16 also max|W| < 98,000 (the scale must stay finite in
+ *   binary16), otherwise the results are unspecified.
+ * ------------------------------------------------------------------------ */
+typedef enum {
+  RRQ_GRID_ASYM = 0, /* zero = group minimum, levels lo + Q*s (the calls above) */
+  RRQ_GRID_SYM = 1   /* implicit zero-point 2, levels (Q - 2)*s, no zeros stored */
+} rrq_grid;
+
+typedef enum {
+  RRQ_SCALE_F32 = 0, /* IEEE binary32 scale, 4 bytes per group and stage */
+  RRQ_SCALE_F16 = 1  /* IEEE binary16 scale, 2 bytes per group and stage
+                        (RRQ_GRID_SYM only) */
+} rrq_scale_type;
+
+typedef struct {
+  int group;      /* 32, 64, 128 or 256 */
+  int n_stages;   /* 1..4 stages held by the package */
+  int grid;       /* rrq_grid */
+  int scale_type; /* rrq_scale_type */
+} rrq_format;
+
+/* One matrix of rrq_quantize_ex.  scales[k] points to float (RRQ_SCALE_F32)
+ * or uint16_t binary16 bit patterns (RRQ_SCALE_F16), rrq_meta_count entries,
+ * 16-byte aligned.  zeros[k] is used by RRQ_GRID_ASYM only (ignored, may be
+ * NULL, for RRQ_GRID_SYM). */
+typedef struct {
+  const uint16_t* W_bf16;                /* device, bf16 [rows, cols], 16-byte aligned */
+  int64_t rows, cols;                    /* cols % group == 0 */
+  uint8_t* codes[RRQ_MAX_STAGES];        /* first n_stages entries used */
+  void* scales[RRQ_MAX_STAGES];
+  float* zeros[RRQ_MAX_STAGES];
+} rrq_quantize_desc;
+
+/* Build the packages of `count` matrices in format *fmt (Algorithm 1 without
+ * a base checkpoint; Eq. 1-7).  Same rules as rrq_quantize_batch (one launch
+ * per 64 matrices, no overlap between any output and any input or output of
+ * the batch).  RRQ_ERR_UNSUPPORTED for a group outside {32, 64, 128, 256}
+ * or RRQ_SCALE_F16 with RRQ_GRID_ASYM; RRQ_ERR_INVALID_ARG for an unknown
+ * grid or scale type.  With RRQ_GRID_ASYM and RRQ_SCALE_F32 the result equals
+ * rrq_quantize_batch's. */
+rrq_status rrq_quantize_ex(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
+                           rrq_stream_t stream);
+
+/* One matrix of rrq_reconstruct_ex: the package (first k stages) and the
+ * outputs, out_bf16[0] only, or out_bf16[0..k-1] when all prefixes are
+ * requested (out_bf16[j] = prefix with j+1 stages). */
+typedef struct {
+  const uint8_t* codes[RRQ_MAX_STAGES];
+  const void* scales[RRQ_MAX_STAGES];    /* float or binary16, as in rrq_quantize_desc */
+  const float* zeros[RRQ_MAX_STAGES];    /* RRQ_GRID_ASYM only */
+  int64_t rows, cols;
+  uint16_t* out_bf16[RRQ_MAX_STAGES];    /* device, bf16 [rows, cols], 16-byte aligned */
+} rrq_reconstruct_desc;
+
+/* Prefix reconstruction (Eq. 8; Appendix C) of `count` packages in format
+ * *fmt: the prefix with k stages (all_prefixes == 0), or every prefix 1..k in
+ * one pass over the package (all_prefixes != 0).  1 <= k <= fmt->n_stages.
+ * Same rules as rrq_reconstruct_batch / rrq_reconstruct_prefixes_batch. */
+rrq_status rrq_reconstruct_ex(const rrq_reconstruct_desc* items, int count, const rrq_format* fmt,
+                              int k, int all_prefixes, rrq_stream_t stream);
+
+/* Bytes of one stage's scale array in format *fmt: groups * (4 or 2).
+ * 0 for invalid arguments. */
+size_t rrq_scales_bytes(int64_t rows, int64_t cols, const rrq_format* fmt);
+
+/* Total package bytes in format *fmt: n_stages * (codes + scales + zeros),
+ * zeros only for RRQ_GRID_ASYM.  0 for invalid arguments. */
+size_t rrq_package_bytes_ex(int64_t rows, int64_t cols, const rrq_format* fmt);
 
 /* Bytes of one stage's code array: rows*cols/4 (rows*cols is a multiple of
  * 32 for every valid shape).  0 for invalid sizes. */

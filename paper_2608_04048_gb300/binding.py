@@ -22,12 +22,37 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
 #: symbols declared in include/rrq.h
 EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
            "rrq_reconstruct_prefixes", "rrq_reconstruct_prefixes_batch",
+           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_scales_bytes", "rrq_package_bytes_ex",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
            "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
 
 
 MAX_STAGES = 4
+
+#: rrq_grid / rrq_scale_type of include/rrq.h
+GRID_ASYM, GRID_SYM = 0, 1
+SCALE_F32, SCALE_F16 = 0, 1
+
+
+class Format(ctypes.Structure):
+    """rrq_format of include/rrq.h"""
+    _fields_ = [("group", ctypes.c_int), ("n_stages", ctypes.c_int), ("grid", ctypes.c_int),
+                ("scale_type", ctypes.c_int)]
+
+
+class QuantizeDesc(ctypes.Structure):
+    """rrq_quantize_desc of include/rrq.h"""
+    _fields_ = [("W_bf16", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
+                ("zeros", ctypes.c_void_p * MAX_STAGES)]
+
+
+class ReconstructDesc(ctypes.Structure):
+    """rrq_reconstruct_desc of include/rrq.h"""
+    _fields_ = [("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
+                ("zeros", ctypes.c_void_p * MAX_STAGES), ("rows", ctypes.c_int64),
+                ("cols", ctypes.c_int64), ("out_bf16", ctypes.c_void_p * MAX_STAGES)]
 
 
 class QuantizeItem(ctypes.Structure):
@@ -89,6 +114,15 @@ def load_library():
     lib.rrq_reconstruct_prefixes.restype = i32
     lib.rrq_reconstruct_prefixes_batch.argtypes = [ctypes.POINTER(PrefixesItem), i32, i32, i32, vp]
     lib.rrq_reconstruct_prefixes_batch.restype = i32
+    fmt_p = ctypes.POINTER(Format)
+    lib.rrq_quantize_ex.argtypes = [ctypes.POINTER(QuantizeDesc), i32, fmt_p, vp]
+    lib.rrq_quantize_ex.restype = i32
+    lib.rrq_reconstruct_ex.argtypes = [ctypes.POINTER(ReconstructDesc), i32, fmt_p, i32, i32, vp]
+    lib.rrq_reconstruct_ex.restype = i32
+    lib.rrq_scales_bytes.argtypes = [i64, i64, fmt_p]
+    lib.rrq_scales_bytes.restype = ctypes.c_size_t
+    lib.rrq_package_bytes_ex.argtypes = [i64, i64, fmt_p]
+    lib.rrq_package_bytes_ex.restype = ctypes.c_size_t
     lib.rrq_codes_bytes.argtypes = [i64, i64]
     lib.rrq_codes_bytes.restype = ctypes.c_size_t
     lib.rrq_meta_count.argtypes = [i64, i64, i32]
@@ -121,8 +155,10 @@ def _ptrs(tensors, n) -> ctypes.Array:
 
 @dataclass
 class Package:
-    """An RRQ package on the device: per stage a code array (uint8, n/4),
-    a scale array and a zero array (float32, n/group)."""
+    """An RRQ package on the device: per stage a code array (uint8, n/4) and
+    a scale array (n/group; float32, or float16 = IEEE binary16 for
+    SCALE_F16), plus a zero array (float32, n/group) for the asymmetric grid
+    (empty list for the symmetric grid)."""
     codes: list
     scales: list
     zeros: list
@@ -130,15 +166,23 @@ class Package:
     cols: int
     group: int
     n_stages: int
+    grid: int = GRID_ASYM
+    scale_type: int = SCALE_F32
 
     @classmethod
-    def empty(cls, rows, cols, group=128, n_stages=4, device=None) -> "Package":
+    def empty(cls, rows, cols, group=128, n_stages=4, device=None, grid=GRID_ASYM,
+              scale_type=SCALE_F32) -> "Package":
         device = device or torch.device("cuda", torch.cuda.current_device())
         n = rows * cols
+        sdt = torch.float16 if scale_type == SCALE_F16 else torch.float32
+        zeros = [] if grid == GRID_SYM else \
+            [torch.empty(n // group, dtype=torch.float32, device=device) for _ in range(n_stages)]
         return cls([torch.empty(n // 4, dtype=torch.uint8, device=device) for _ in range(n_stages)],
-                   [torch.empty(n // group, dtype=torch.float32, device=device) for _ in range(n_stages)],
-                   [torch.empty(n // group, dtype=torch.float32, device=device) for _ in range(n_stages)],
-                   rows, cols, group, n_stages)
+                   [torch.empty(n // group, dtype=sdt, device=device) for _ in range(n_stages)],
+                   zeros, rows, cols, group, n_stages, grid, scale_type)
+
+    def format(self) -> Format:
+        return Format(self.group, self.n_stages, self.grid, self.scale_type)
 
     def nbytes(self) -> int:
         return sum(t.numel() * t.element_size() for t in self.codes + self.scales + self.zeros)
@@ -289,6 +333,85 @@ def rrq_reconstruct_prefixes_batch(pkgs, k: int, outs=None, stream=None, items=N
     if rc != 0:
         raise RRQError(rc, "rrq_reconstruct_prefixes_batch")
     return outs
+
+
+def quantize_descs(mats, pkgs) -> ctypes.Array:
+    """Host array of rrq_quantize_desc for matrices and their packages."""
+    items = (QuantizeDesc * len(mats))()
+    for it, W, pkg in zip(items, mats, pkgs):
+        if W.dtype != torch.bfloat16 or W.dim() != 2 or not W.is_cuda or not W.is_contiguous():
+            raise TypeError("every W must be a contiguous 2-D bfloat16 CUDA tensor")
+        it.W_bf16 = W.data_ptr()
+        it.rows, it.cols = W.shape
+        for k in range(pkg.n_stages):
+            it.codes[k] = pkg.codes[k].data_ptr()
+            it.scales[k] = pkg.scales[k].data_ptr()
+            it.zeros[k] = pkg.zeros[k].data_ptr() if pkg.zeros else None
+    return items
+
+
+def rrq_quantize_ex(mats, group: int = 128, n_stages: int = 4, grid: int = GRID_SYM,
+                    scale_type: int = SCALE_F16, pkgs=None, stream=None, items=None):
+    """Packages of a list of bf16 matrices in any supported format (one
+    launch per 64 matrices).  Default: the symmetric grid with binary16
+    scales."""
+    lib = load_library()
+    if pkgs is None:
+        pkgs = [Package.empty(W.shape[0], W.shape[1], group, n_stages, W.device, grid, scale_type)
+                for W in mats]
+    if items is None:
+        items = quantize_descs(mats, pkgs)
+    fmt = Format(group, n_stages, grid, scale_type)
+    rc = lib.rrq_quantize_ex(items, len(items), ctypes.byref(fmt), _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_quantize_ex")
+    return pkgs
+
+
+def reconstruct_descs(pkgs, outs, k) -> ctypes.Array:
+    """Host array of rrq_reconstruct_desc; outs[i] is a list of 1 or k outputs."""
+    items = (ReconstructDesc * len(pkgs))()
+    for it, pkg, o in zip(items, pkgs, outs):
+        for j in range(k):
+            it.codes[j] = pkg.codes[j].data_ptr()
+            it.scales[j] = pkg.scales[j].data_ptr()
+            it.zeros[j] = pkg.zeros[j].data_ptr() if pkg.zeros else None
+        for j, t in enumerate(o):
+            if t.dtype != torch.bfloat16 or not t.is_cuda or not t.is_contiguous():
+                raise TypeError("outputs must be contiguous bfloat16 CUDA tensors")
+            it.out_bf16[j] = t.data_ptr()
+        it.rows, it.cols = pkg.rows, pkg.cols
+    return items
+
+
+def rrq_reconstruct_ex(pkgs, k: int, all_prefixes: bool = False, outs=None, stream=None, items=None):
+    """Prefix reconstruction of packages of one format: outs[i] = [prefix k]
+    or, with all_prefixes, [prefix 1, ..., prefix k]."""
+    lib = load_library()
+    if any(not 1 <= k <= p.n_stages for p in pkgs):
+        raise ValueError("k exceeds the stages of a package")
+    if outs is None:
+        outs = [_new_outs(p, k if all_prefixes else 1) for p in pkgs]
+    if items is None:
+        items = reconstruct_descs(pkgs, outs, k)
+    fmt = pkgs[0].format()
+    rc = lib.rrq_reconstruct_ex(items, len(items), ctypes.byref(fmt), k, int(all_prefixes),
+                                _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_reconstruct_ex")
+    return outs
+
+
+def rrq_scales_bytes(rows: int, cols: int, group: int, grid: int, scale_type: int,
+                     n_stages: int = 4) -> int:
+    return int(load_library().rrq_scales_bytes(rows, cols,
+                                               ctypes.byref(Format(group, n_stages, grid, scale_type))))
+
+
+def rrq_package_bytes_ex(rows: int, cols: int, group: int, n_stages: int, grid: int,
+                         scale_type: int) -> int:
+    return int(load_library().rrq_package_bytes_ex(
+        rows, cols, ctypes.byref(Format(group, n_stages, grid, scale_type))))
 
 
 def rrq_codes_bytes(rows: int, cols: int) -> int:

@@ -119,40 +119,71 @@ Range range_of(const void* p, uint64_t bytes, bool output) {
   return {a, a + bytes, output};
 }
 
+// A validated package format.
+struct Fmt {
+  int group = 0;
+  int n_stages = 0;
+  rrq::Format kind = rrq::kAsymF32;
+  bool sym() const { return kind != rrq::kAsymF32; }
+  uint64_t scale_bytes() const { return kind == rrq::kSymF16 ? 2 : 4; }
+};
+
+rrq_status parse_format(const rrq_format* f, Fmt* out) {
+  if (!f || f->n_stages < 1 || f->n_stages > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  if (f->grid != RRQ_GRID_ASYM && f->grid != RRQ_GRID_SYM) return RRQ_ERR_INVALID_ARG;
+  if (f->scale_type != RRQ_SCALE_F32 && f->scale_type != RRQ_SCALE_F16) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(f->group)) return RRQ_ERR_UNSUPPORTED;
+  out->group = f->group;
+  out->n_stages = f->n_stages;
+  if (f->grid == RRQ_GRID_ASYM) {
+    if (f->scale_type != RRQ_SCALE_F32) return RRQ_ERR_UNSUPPORTED;
+    out->kind = rrq::kAsymF32;
+  } else {
+    out->kind = f->scale_type == RRQ_SCALE_F16 ? rrq::kSymF16 : rrq::kSymF32;
+  }
+  return RRQ_OK;
+}
+
+Fmt asym_format(int group, int n_stages) {
+  Fmt f;
+  f.group = group;
+  f.n_stages = n_stages;
+  return f;
+}
+
 // ---------------------------------------------------------------------------
 // quantize
 // ---------------------------------------------------------------------------
-rrq_status check_quantize_item(const rrq_quantize_item& it, int group, int n_stages) {
+rrq_status check_quantize_item(const rrq_quantize_desc& it, const Fmt& f) {
   if (!it.W_bf16 || !shape_ok(it.rows, it.cols)) return RRQ_ERR_INVALID_ARG;
-  if (it.cols % group != 0) return RRQ_ERR_INVALID_ARG;
-  for (int k = 0; k < n_stages; ++k)
-    if (!it.codes[k] || !it.scales[k] || !it.zeros[k]) return RRQ_ERR_INVALID_ARG;
+  if (it.cols % f.group != 0) return RRQ_ERR_INVALID_ARG;
+  for (int k = 0; k < f.n_stages; ++k)
+    if (!it.codes[k] || !it.scales[k] || (!f.sym() && !it.zeros[k])) return RRQ_ERR_INVALID_ARG;
   if (!aligned(it.W_bf16, 16)) return RRQ_ERR_MISALIGNED;
-  for (int k = 0; k < n_stages; ++k)
-    if (!aligned(it.codes[k], 16) || !aligned(it.scales[k], 16) || !aligned(it.zeros[k], 16))
+  for (int k = 0; k < f.n_stages; ++k)
+    if (!aligned(it.codes[k], 16) || !aligned(it.scales[k], 16) || (!f.sym() && !aligned(it.zeros[k], 16)))
       return RRQ_ERR_MISALIGNED;
   return RRQ_OK;
 }
 
-void add_quantize_ranges(const rrq_quantize_item& it, int group, int n_stages, std::vector<Range>& r) {
+void add_quantize_ranges(const rrq_quantize_desc& it, const Fmt& f, std::vector<Range>& r) {
   const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
   r.push_back(range_of(it.W_bf16, 2 * n, false));
-  for (int k = 0; k < n_stages; ++k) {
+  for (int k = 0; k < f.n_stages; ++k) {
     r.push_back(range_of(it.codes[k], n / 4, true));
-    r.push_back(range_of(it.scales[k], 4 * (n / group), true));
-    r.push_back(range_of(it.zeros[k], 4 * (n / group), true));
+    r.push_back(range_of(it.scales[k], f.scale_bytes() * (n / f.group), true));
+    if (!f.sym()) r.push_back(range_of(it.zeros[k], 4 * (n / f.group), true));
   }
 }
 
-rrq_status quantize_batch(const rrq_quantize_item* items, int count, int group, int n_stages,
-                          rrq_stream_t stream) {
-  if (!items || count < 1 || n_stages < 1 || n_stages > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
-  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& f, rrq_stream_t stream) {
+  if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  const int n_stages = f.n_stages;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (1 + 3 * n_stages));
   for (int i = 0; i < count; ++i) {
-    if (rrq_status rc = check_quantize_item(items[i], group, n_stages)) return rc;
-    add_quantize_ranges(items[i], group, n_stages, ranges);
+    if (rrq_status rc = check_quantize_item(items[i], f)) return rc;
+    add_quantize_ranges(items[i], f, ranges);
   }
   if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
 
@@ -160,10 +191,11 @@ rrq_status quantize_batch(const rrq_quantize_item* items, int count, int group, 
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
   for (int i = 0; i < count; ++i) {
-    const rrq_quantize_item& it = items[i];
+    const rrq_quantize_desc& it = items[i];
     if (!on_device(it.W_bf16, dev)) return RRQ_ERR_INVALID_ARG;
     for (int k = 0; k < n_stages; ++k)
-      if (!on_device(it.codes[k], dev) || !on_device(it.scales[k], dev) || !on_device(it.zeros[k], dev))
+      if (!on_device(it.codes[k], dev) || !on_device(it.scales[k], dev) ||
+          (!f.sym() && !on_device(it.zeros[k], dev)))
         return RRQ_ERR_INVALID_ARG;
   }
 
@@ -178,7 +210,7 @@ rrq_status quantize_batch(const rrq_quantize_item* items, int count, int group, 
     p.status = st->status;
     int64_t chunks = 0;
     for (int i = 0; i < m; ++i) {
-      const rrq_quantize_item& it = items[base + i];
+      const rrq_quantize_desc& it = items[base + i];
       rrq::QuantizeItem& q = p.item[i];
       q.W = it.W_bf16;
       q.n = it.rows * it.cols;
@@ -188,11 +220,11 @@ rrq_status quantize_batch(const rrq_quantize_item* items, int count, int group, 
         const int kk = k < n_stages ? k : n_stages - 1;
         q.codes[k] = it.codes[kk];
         q.scales[k] = it.scales[kk];
-        q.zeros[k] = it.zeros[kk];
+        q.zeros[k] = f.sym() ? nullptr : it.zeros[kk];
       }
     }
     p.total_chunks = chunks;
-    cudaError_t e = rrq::quantize_launch(group, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+    cudaError_t e = rrq::quantize_launch(f.group, f.kind, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
     if (e != cudaSuccess) return fail_cuda(e);
   }
   return RRQ_OK;
@@ -205,43 +237,43 @@ rrq_status quantize_batch(const rrq_quantize_item* items, int count, int group, 
 // (n_out = 1: the prefix with k stages; n_out = k: every prefix).
 struct ReconView {
   const uint8_t* const* codes;
-  const float* const* scales;
+  const void* const* scales;
   const float* const* zeros;
   int64_t rows, cols;
   uint16_t* const* out;
 };
 
-rrq_status check_reconstruct_item(const ReconView& it, int group, int k, int n_out) {
+rrq_status check_reconstruct_item(const ReconView& it, const Fmt& f, int k, int n_out) {
   if (!shape_ok(it.rows, it.cols)) return RRQ_ERR_INVALID_ARG;
-  if (it.cols % group != 0) return RRQ_ERR_INVALID_ARG;
+  if (it.cols % f.group != 0) return RRQ_ERR_INVALID_ARG;
   for (int i = 0; i < k; ++i)
-    if (!it.codes[i] || !it.scales[i] || !it.zeros[i]) return RRQ_ERR_INVALID_ARG;
+    if (!it.codes[i] || !it.scales[i] || (!f.sym() && !it.zeros[i])) return RRQ_ERR_INVALID_ARG;
   for (int j = 0; j < n_out; ++j)
     if (!it.out[j]) return RRQ_ERR_INVALID_ARG;
   for (int j = 0; j < n_out; ++j)
     if (!aligned(it.out[j], 16)) return RRQ_ERR_MISALIGNED;
   for (int i = 0; i < k; ++i)
-    if (!aligned(it.codes[i], 16) || !aligned(it.scales[i], 16) || !aligned(it.zeros[i], 16))
+    if (!aligned(it.codes[i], 16) || !aligned(it.scales[i], 16) || (!f.sym() && !aligned(it.zeros[i], 16)))
       return RRQ_ERR_MISALIGNED;
   return RRQ_OK;
 }
 
-rrq_status reconstruct_views(const ReconView* items, int count, int group, int k, bool all_prefixes,
+rrq_status reconstruct_views(const ReconView* items, int count, const Fmt& f, int k, bool all_prefixes,
                              rrq_stream_t stream) {
-  if (!items || count < 1 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
-  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  if (!items || count < 1 || k < 1 || k > RRQ_MAX_STAGES || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
+  const int group = f.group;
   const int n_out = all_prefixes ? k : 1;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (n_out + 3 * k));
   for (int i = 0; i < count; ++i) {
     const ReconView& it = items[i];
-    if (rrq_status rc = check_reconstruct_item(it, group, k, n_out)) return rc;
+    if (rrq_status rc = check_reconstruct_item(it, f, k, n_out)) return rc;
     const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
     for (int j = 0; j < n_out; ++j) ranges.push_back(range_of(it.out[j], 2 * n, true));
     for (int j = 0; j < k; ++j) {
       ranges.push_back(range_of(it.codes[j], n / 4, false));
-      ranges.push_back(range_of(it.scales[j], 4 * (n / group), false));
-      ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
+      ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
+      if (!f.sym()) ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
     }
   }
   if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
@@ -254,7 +286,8 @@ rrq_status reconstruct_views(const ReconView* items, int count, int group, int k
     for (int j = 0; j < n_out; ++j)
       if (!on_device(it.out[j], dev)) return RRQ_ERR_INVALID_ARG;
     for (int j = 0; j < k; ++j)
-      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) || !on_device(it.zeros[j], dev))
+      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) ||
+          (!f.sym() && !on_device(it.zeros[j], dev)))
         return RRQ_ERR_INVALID_ARG;
   }
 
@@ -273,7 +306,7 @@ rrq_status reconstruct_views(const ReconView* items, int count, int group, int k
         const int jj = j < k ? j : k - 1;
         q.codes[j] = it.codes[jj];
         q.scales[j] = it.scales[jj];
-        q.zeros[j] = it.zeros[jj];
+        q.zeros[j] = f.sym() ? nullptr : it.zeros[jj];
         q.out[j] = it.out[j < n_out ? j : n_out - 1];
       }
       q.n = it.rows * it.cols;
@@ -281,7 +314,7 @@ rrq_status reconstruct_views(const ReconView* items, int count, int group, int k
       chunks += (q.n + rrq::kChunkElems - 1) / rrq::kChunkElems;
     }
     p.total_chunks = chunks;
-    cudaError_t e = rrq::reconstruct_launch(group, k, all_prefixes, p,
+    cudaError_t e = rrq::reconstruct_launch(group, f.kind, k, all_prefixes, p,
                                             reinterpret_cast<cudaStream_t>(stream), st->sms);
     if (e != cudaSuccess) return fail_cuda(e);
   }
@@ -314,7 +347,8 @@ rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int 
                         float* const out_zeros[], rrq_stream_t stream) {
   if (!out_codes || !out_scales || !out_zeros || n_stages < 1 || n_stages > RRQ_MAX_STAGES)
     return RRQ_ERR_INVALID_ARG;
-  rrq_quantize_item it{};
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  rrq_quantize_desc it{};
   it.W_bf16 = W_bf16;
   it.rows = rows;
   it.cols = cols;
@@ -323,30 +357,58 @@ rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int 
     it.scales[k] = out_scales[k];
     it.zeros[k] = out_zeros[k];
   }
-  return quantize_batch(&it, 1, group, n_stages, stream);
+  return quantize_batch(&it, 1, asym_format(group, n_stages), stream);
 }
 
 rrq_status rrq_quantize_batch(const rrq_quantize_item* items, int count, int group, int n_stages,
                               rrq_stream_t stream) {
-  return quantize_batch(items, count, group, n_stages, stream);
+  if (!items || count < 1 || n_stages < 1 || n_stages > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  std::vector<rrq_quantize_desc> d(static_cast<size_t>(count));
+  for (int i = 0; i < count; ++i) {
+    d[i].W_bf16 = items[i].W_bf16;
+    d[i].rows = items[i].rows;
+    d[i].cols = items[i].cols;
+    for (int k = 0; k < RRQ_MAX_STAGES; ++k) {
+      d[i].codes[k] = items[i].codes[k];
+      d[i].scales[k] = items[i].scales[k];
+      d[i].zeros[k] = items[i].zeros[k];
+    }
+  }
+  return quantize_batch(d.data(), count, asym_format(group, n_stages), stream);
+}
+
+rrq_status rrq_quantize_ex(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
+                           rrq_stream_t stream) {
+  Fmt f;
+  if (rrq_status rc = parse_format(fmt, &f)) return rc;
+  return quantize_batch(items, count, f, stream);
 }
 
 rrq_status rrq_reconstruct(const uint8_t* const codes[], const float* const scales[],
                            const float* const zeros[], int64_t rows, int64_t cols, int group,
                            int k, uint16_t* out_bf16, rrq_stream_t stream) {
   if (!codes || !scales || !zeros || !out_bf16 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
   uint16_t* const outs[1] = {out_bf16};
-  const ReconView v{codes, scales, zeros, rows, cols, outs};
-  return reconstruct_views(&v, 1, group, k, false, stream);
+  const void* sc[RRQ_MAX_STAGES] = {};
+  for (int i = 0; i < k; ++i) sc[i] = scales[i];
+  const ReconView v{codes, sc, zeros, rows, cols, outs};
+  return reconstruct_views(&v, 1, asym_format(group, k), k, false, stream);
 }
 
 rrq_status rrq_reconstruct_batch(const rrq_reconstruct_item* items, int count, int group, int k,
                                  rrq_stream_t stream) {
-  if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  if (!items || count < 1 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
   std::vector<ReconView> v(static_cast<size_t>(count));
-  for (int i = 0; i < count; ++i)
-    v[i] = {items[i].codes, items[i].scales, items[i].zeros, items[i].rows, items[i].cols, &items[i].out_bf16};
-  return reconstruct_views(v.data(), count, group, k, false, stream);
+  std::vector<const void*> sc(static_cast<size_t>(count) * RRQ_MAX_STAGES);
+  for (int i = 0; i < count; ++i) {
+    for (int j = 0; j < RRQ_MAX_STAGES; ++j) sc[i * RRQ_MAX_STAGES + j] = items[i].scales[j];
+    v[i] = {items[i].codes, &sc[i * RRQ_MAX_STAGES], items[i].zeros, items[i].rows, items[i].cols,
+            &items[i].out_bf16};
+  }
+  return reconstruct_views(v.data(), count, asym_format(group, k), k, false, stream);
 }
 
 rrq_status rrq_reconstruct_prefixes(const uint8_t* const codes[], const float* const scales[],
@@ -354,17 +416,51 @@ rrq_status rrq_reconstruct_prefixes(const uint8_t* const codes[], const float* c
                                     int group, int k, uint16_t* const out_bf16[],
                                     rrq_stream_t stream) {
   if (!codes || !scales || !zeros || !out_bf16 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
-  const ReconView v{codes, scales, zeros, rows, cols, out_bf16};
-  return reconstruct_views(&v, 1, group, k, true, stream);
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  const void* sc[RRQ_MAX_STAGES] = {};
+  for (int i = 0; i < k; ++i) sc[i] = scales[i];
+  const ReconView v{codes, sc, zeros, rows, cols, out_bf16};
+  return reconstruct_views(&v, 1, asym_format(group, k), k, true, stream);
 }
 
 rrq_status rrq_reconstruct_prefixes_batch(const rrq_prefixes_item* items, int count, int group,
                                           int k, rrq_stream_t stream) {
+  if (!items || count < 1 || k < 1 || k > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  std::vector<ReconView> v(static_cast<size_t>(count));
+  std::vector<const void*> sc(static_cast<size_t>(count) * RRQ_MAX_STAGES);
+  for (int i = 0; i < count; ++i) {
+    for (int j = 0; j < RRQ_MAX_STAGES; ++j) sc[i * RRQ_MAX_STAGES + j] = items[i].scales[j];
+    v[i] = {items[i].codes, &sc[i * RRQ_MAX_STAGES], items[i].zeros, items[i].rows, items[i].cols,
+            items[i].out_bf16};
+  }
+  return reconstruct_views(v.data(), count, asym_format(group, k), k, true, stream);
+}
+
+rrq_status rrq_reconstruct_ex(const rrq_reconstruct_desc* items, int count, const rrq_format* fmt,
+                              int k, int all_prefixes, rrq_stream_t stream) {
+  Fmt f;
+  if (rrq_status rc = parse_format(fmt, &f)) return rc;
   if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
   std::vector<ReconView> v(static_cast<size_t>(count));
   for (int i = 0; i < count; ++i)
     v[i] = {items[i].codes, items[i].scales, items[i].zeros, items[i].rows, items[i].cols, items[i].out_bf16};
-  return reconstruct_views(v.data(), count, group, k, true, stream);
+  return reconstruct_views(v.data(), count, f, k, all_prefixes != 0, stream);
+}
+
+size_t rrq_scales_bytes(int64_t rows, int64_t cols, const rrq_format* fmt) {
+  Fmt f;
+  if (parse_format(fmt, &f) != RRQ_OK) return 0;
+  return rrq_meta_count(rows, cols, f.group) * static_cast<size_t>(f.scale_bytes());
+}
+
+size_t rrq_package_bytes_ex(int64_t rows, int64_t cols, const rrq_format* fmt) {
+  Fmt f;
+  if (parse_format(fmt, &f) != RRQ_OK) return 0;
+  const size_t m = rrq_meta_count(rows, cols, f.group);
+  if (m == 0) return 0;
+  const size_t per_stage = rrq_codes_bytes(rows, cols) + m * (f.scale_bytes() + (f.sym() ? 0 : 4));
+  return static_cast<size_t>(f.n_stages) * per_stage;
 }
 
 rrq_status rrq_get_device_status(rrq_stream_t stream) {

@@ -19,7 +19,21 @@
 // two are exact for s in [2^-100, 2^100].  So four codes of one byte need one
 // shift and one logic operation each, no shift per code.  Groups with a scale
 // outside that range use the plain form RN((t - 2^23) * s).
+//
+// Symmetric grid (implicit zero-point 2): L_i = (Q_i - 2) * s_i, exact in
+// binary32, so acc + L_i is one fma(u, s, acc) with u = Q - 2 taken exactly
+// as t - (2^23 + 2*4^j) from the same prescaled t; the base stage is the
+// exact product u * s.  binary16 scales are read as the 4-byte word holding
+// the lane's scale and its neighbour's (the copy is cut to 2 bytes at the end
+// of an array with an odd number of groups) and widened exactly.
+//
+// This header holds the kernel template; reconstruct_asym_f32.cu,
+// reconstruct_sym_f32.cu and reconstruct_sym_f16.cu each instantiate one
+// package format (they compile in parallel).
+#pragma once
+
 #include <cuda_bf16.h>
+#include <cuda_fp16.h>
 
 #include "rrq_device.cuh"
 
@@ -43,8 +57,10 @@ __device__ __forceinline__ bool prescale_ok(float s) {
 
 // kAllPrefixes: write the reconstruction after every stage i < K (prefixes
 // 1..K in one pass over the package) instead of only after stage K-1.
-template <int G, int K, bool kAllPrefixes>
+template <int G, int K, bool kAllPrefixes, int F>
 __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_constant__ ReconstructBatch p) {
+  constexpr bool kSym = F != kAsymF32;
+  constexpr bool kF16 = F == kSymF16;
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -78,15 +94,23 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
       const bool valid = e < it.n;  // false only in the last chunk of a matrix
       // byte offsets shared by every stage's arrays (invalid lanes read nothing)
       const uint64_t off_code = valid ? static_cast<uint64_t>(e) >> 2 : 0;
-      const uint64_t off_meta = valid ? (static_cast<uint64_t>(e) / G) * 4 : 0;
+      const uint64_t gi = static_cast<uint64_t>(e) / G;
+      uint64_t off_meta = valid ? gi * 4 : 0;
+      uint32_t n_scale = valid ? 4u : 0u;
+      if (kF16) {  // the aligned 4-byte word holding this group's 2-byte scale
+        off_meta = valid ? (gi * 2) & ~uint64_t{3} : 0;
+        const uint64_t left = static_cast<uint64_t>(it.n / G) * 2 - off_meta;
+        n_scale = valid ? (left < 4 ? 2u : 4u) : 0u;
+      }
       const uint32_t n8 = valid ? 8u : 0u, n4 = valid ? 4u : 0u;
       const uint32_t base = smem_u32(ring + buf * K * kStageBytes) + lane * 8;
       const uint32_t mbase = smem_u32(ring + buf * K * kStageBytes) + 256 + lane * 4;
 #pragma unroll
       for (int i = 0; i < K; ++i) {
         cp_async_8(base + i * kStageBytes, reinterpret_cast<const char*>(it.codes[i]) + off_code, n8);
-        cp_async_4(mbase + i * kStageBytes, reinterpret_cast<const char*>(it.scales[i]) + off_meta, n4);
-        cp_async_4(mbase + i * kStageBytes + 128, reinterpret_cast<const char*>(it.zeros[i]) + off_meta, n4);
+        cp_async_4(mbase + i * kStageBytes, reinterpret_cast<const char*>(it.scales[i]) + off_meta, n_scale);
+        if (!kSym)
+          cp_async_4(mbase + i * kStageBytes + 128, reinterpret_cast<const char*>(it.zeros[i]) + off_meta, n4);
       }
     }
     cp_async_commit();
@@ -107,8 +131,15 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
 #pragma unroll
     for (int i = 0; i < K; ++i) {
       code[i] = *reinterpret_cast<const uint2*>(buf + i * kStageBytes + lane * 8);
-      scale[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + 256 + lane * 4);
-      zero[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + 384 + lane * 4);
+      if (kF16) {
+        // group index parity of this lane: chunks start on an even group
+        const uint32_t w = *reinterpret_cast<const uint32_t*>(buf + i * kStageBytes + 256 + lane * 4);
+        const uint32_t h = ((lane / (G / 32)) & 1) ? (w >> 16) : (w & 0xffffu);
+        scale[i] = __half2float(__ushort_as_half(static_cast<unsigned short>(h)));
+      } else {
+        scale[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + 256 + lane * 4);
+      }
+      zero[i] = kSym ? 0.0f : *reinterpret_cast<const float*>(buf + i * kStageBytes + 384 + lane * 4);
       ok = ok && prescale_ok(scale[i]);
     }
 
@@ -151,7 +182,34 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
       const uint32_t w0 = __byte_perm(code[i].x, code[i].y, sel_lo);
       const uint32_t w1 = __byte_perm(code[i].x, code[i].y, sel_hi);
       const f32x2 LO = pack2(zero[i], zero[i]);
-      if (all_ok) {
+      if (kSym) {
+        // u = Q - 2 (times 4^j in the prescaled form), exact; L = u * s exact
+        const float s = scale[i];
+        if (all_ok) {
+          const f32x2 S01 = pack2(s, __fmul_rn(s, 0x1p-2f));
+          const f32x2 S23 = pack2(__fmul_rn(s, 0x1p-4f), __fmul_rn(s, 0x1p-6f));
+          const f32x2 K01 = pack2(kTwo23 + 2.0f, kTwo23 + 8.0f);
+          const f32x2 K23 = pack2(kTwo23 + 32.0f, kTwo23 + 128.0f);
+#pragma unroll
+          for (int j = 0; j < 8; ++j) {
+            const uint32_t word = j < 4 ? w0 : w1;
+            const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
+            const f32x2 u01 = sub2(pack2u(0x4B000000u | (b & 0x03u), 0x4B000000u | (b & 0x0Cu)), K01);
+            const f32x2 u23 = sub2(pack2u(0x4B000000u | (b & 0x30u), 0x4B000000u | (b & 0xC0u)), K23);
+            acc[2 * j] = (i == 0) ? mul2(u01, S01) : fma2(u01, S01, acc[2 * j]);
+            acc[2 * j + 1] = (i == 0) ? mul2(u23, S23) : fma2(u23, S23, acc[2 * j + 1]);
+          }
+        } else {
+          const f32x2 K2 = pack2(kTwo23 + 2.0f, kTwo23 + 2.0f), S = pack2(s, s);
+#pragma unroll
+          for (int m = 0; m < 16; ++m) {
+            const uint32_t word = m < 8 ? w0 : w1;
+            const int sh = 4 * (m & 7);
+            const f32x2 u = sub2(pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u)), K2);
+            acc[m] = (i == 0) ? mul2(u, S) : fma2(u, S, acc[m]);
+          }
+        }
+      } else if (all_ok) {
         const float s = scale[i];
         const f32x2 S01 = pack2(s, __fmul_rn(s, 0x1p-2f));
         const f32x2 S23 = pack2(__fmul_rn(s, 0x1p-4f), __fmul_rn(s, 0x1p-6f));
@@ -190,76 +248,79 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
   if (lane == 0) bulk_wait<0>();
 }
 
-template <int G, int K, bool A>
+template <int G, int K, bool A, int F>
 cudaError_t launch_gk(const ReconstructBatch& p, cudaStream_t stream, int sms) {
   static int blocks_per_sm = 0;
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, reconstruct_kernel<G, K, A>, kThreads, smem_bytes<K>());
+        &blocks_per_sm, reconstruct_kernel<G, K, A, F>, kThreads, smem_bytes<K>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
   const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  reconstruct_kernel<G, K, A><<<grid, kThreads, smem_bytes<K>(), stream>>>(p);
+  reconstruct_kernel<G, K, A, F><<<grid, kThreads, smem_bytes<K>(), stream>>>(p);
   return cudaGetLastError();
 }
 
-template <int G, bool A>
+template <int G, bool A, int F>
 cudaError_t launch_g(int k, const ReconstructBatch& p, cudaStream_t stream, int sms) {
   switch (k) {
-    case 1: return launch_gk<G, 1, A>(p, stream, sms);
-    case 2: return launch_gk<G, 2, A>(p, stream, sms);
-    case 3: return launch_gk<G, 3, A>(p, stream, sms);
-    case 4: return launch_gk<G, 4, A>(p, stream, sms);
+    case 1: return launch_gk<G, 1, A, F>(p, stream, sms);
+    case 2: return launch_gk<G, 2, A, F>(p, stream, sms);
+    case 3: return launch_gk<G, 3, A, F>(p, stream, sms);
+    case 4: return launch_gk<G, 4, A, F>(p, stream, sms);
     default: return cudaErrorInvalidValue;
   }
 }
 
-template <int G, bool A>
+template <int G, bool A, int F>
 cudaError_t prepare_ga() {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 1, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()))) return e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 2, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()))) return e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 3, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<3>()))) return e;
-  return cudaFuncSetAttribute(reconstruct_kernel<G, 4, A>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<4>());
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 1, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 2, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 3, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<3>()))) return e;
+  return cudaFuncSetAttribute(reconstruct_kernel<G, 4, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<4>());
 }
 
-template <int G>
+template <int G, int F>
 cudaError_t prepare_g() {
-  cudaError_t e = prepare_ga<G, false>();
-  return e != cudaSuccess ? e : prepare_ga<G, true>();
+  cudaError_t e = prepare_ga<G, false, F>();
+  return e != cudaSuccess ? e : prepare_ga<G, true, F>();
 }
 
-}  // namespace
-
-cudaError_t reconstruct_prepare() {
+// Set-up and launch of one format (instantiated by one translation unit each).
+template <int F>
+cudaError_t prepare_format() {
   cudaError_t e;
-  if ((e = prepare_g<32>())) return e;
-  if ((e = prepare_g<64>())) return e;
-  if ((e = prepare_g<128>())) return e;
-  return prepare_g<256>();
+  if ((e = prepare_g<32, F>())) return e;
+  if ((e = prepare_g<64, F>())) return e;
+  if ((e = prepare_g<128, F>())) return e;
+  return prepare_g<256, F>();
 }
 
-cudaError_t reconstruct_launch(int group, int k, bool all_prefixes, const ReconstructBatch& p,
-                               cudaStream_t stream, int sms) {
+template <int F>
+cudaError_t launch_format(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                          cudaStream_t stream, int sms) {
   if (all_prefixes) {
     switch (group) {
-      case 32: return launch_g<32, true>(k, p, stream, sms);
-      case 64: return launch_g<64, true>(k, p, stream, sms);
-      case 128: return launch_g<128, true>(k, p, stream, sms);
-      case 256: return launch_g<256, true>(k, p, stream, sms);
+      case 32: return launch_g<32, true, F>(k, p, stream, sms);
+      case 64: return launch_g<64, true, F>(k, p, stream, sms);
+      case 128: return launch_g<128, true, F>(k, p, stream, sms);
+      case 256: return launch_g<256, true, F>(k, p, stream, sms);
       default: return cudaErrorInvalidValue;
     }
   }
   switch (group) {
-    case 32: return launch_g<32, false>(k, p, stream, sms);
-    case 64: return launch_g<64, false>(k, p, stream, sms);
-    case 128: return launch_g<128, false>(k, p, stream, sms);
-    case 256: return launch_g<256, false>(k, p, stream, sms);
+    case 32: return launch_g<32, false, F>(k, p, stream, sms);
+    case 64: return launch_g<64, false, F>(k, p, stream, sms);
+    case 128: return launch_g<128, false, F>(k, p, stream, sms);
+    case 256: return launch_g<256, false, F>(k, p, stream, sms);
     default: return cudaErrorInvalidValue;
   }
 }
+
+}  // namespace
 
 }  // namespace rrq

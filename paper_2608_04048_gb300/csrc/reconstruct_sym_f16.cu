@@ -1,0 +1,14 @@
+// Prefix reconstruction kernels for one package format (see
+// reconstruct_kernel.cuh for the arithmetic and the work decomposition).
+#include "reconstruct_kernel.cuh"
+
+namespace rrq {
+
+cudaError_t reconstruct_prepare_sym_f16() { return prepare_format<kSymF16>(); }
+
+cudaError_t reconstruct_launch_sym_f16(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                                  cudaStream_t stream, int sms) {
+  return launch_format<kSymF16>(group, k, all_prefixes, p, stream, sms);
+}
+
+}  // namespace rrq

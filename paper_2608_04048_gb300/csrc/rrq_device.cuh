@@ -109,6 +109,10 @@ __device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src, uint32
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
                : "memory");
 }
+// streaming (evict-first) 16-bit global store
+__device__ __forceinline__ void stcs_u16(uint16_t* p, uint16_t v) {
+  asm volatile("st.global.cs.u16 [%0], %1;" ::"l"(p), "h"(v) : "memory");
+}
 __device__ __forceinline__ void cp_async_commit() {
   asm volatile("cp.async.commit_group;" ::: "memory");
 }
@@ -190,7 +194,27 @@ __device__ __forceinline__ void lane_minmax(const f32x2 (&v)[16], float& lo, flo
   hi = fmaxf(hi0, hi1);
 }
 
+// max |v| over 16 packed pairs held by one lane
+__device__ __forceinline__ float lane_amax(const f32x2 (&v)[16]) {
+  float m0 = 0.0f, m1 = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 16; i += 2) {
+    float a, b, c, d;
+    unpack2(v[i], a, b);
+    unpack2(v[i + 1], c, d);
+    m0 = fmaxf(m0, fmaxf(fabsf(a), fabsf(b)));
+    m1 = fmaxf(m1, fmaxf(fabsf(c), fabsf(d)));
+  }
+  return fmaxf(m0, m1);
+}
+
 // reductions over the L consecutive lanes that share one group (L | 32)
+template <int L>
+__device__ __forceinline__ float group_max(float x) {
+#pragma unroll
+  for (int off = 1; off < L; off <<= 1) x = fmaxf(x, __shfl_xor_sync(kFullMask, x, off));
+  return x;
+}
 template <int L>
 __device__ __forceinline__ void group_minmax(float& lo, float& hi) {
 #pragma unroll

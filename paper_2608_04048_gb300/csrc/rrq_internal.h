@@ -14,6 +14,13 @@ constexpr int kChunkElems = 32 * kLaneElems;      // weights per warp chunk (102
 constexpr int kChunkBytes = kChunkElems * 2;      // bf16 bytes per warp chunk (2 KiB)
 constexpr int kMaxBatch = 64;                     // matrices per kernel launch (kernel parameters)
 
+// Package formats built by the kernels (grid x scale type of include/rrq.h).
+enum Format : int {
+  kAsymF32 = 0,  // zero = group minimum, binary32 scale and zero
+  kSymF32 = 1,   // implicit zero-point 2, binary32 scale
+  kSymF16 = 2,   // implicit zero-point 2, binary16 scale
+};
+
 constexpr unsigned kStatusTimeout = 1u;           // bit set in the device status word
 constexpr uint32_t kDebugForceExact = 1u;         // same value as RRQ_DEBUG_FORCE_EXACT
 constexpr uint32_t kDrainLimitUs = 1000000u;      // wait for own copies before leaving
@@ -25,8 +32,8 @@ struct QuantizeItem {
   int64_t n;                       // rows * cols (multiple of 32)
   int64_t chunk_begin;
   uint8_t* codes[kMaxStages];      // n/4 bytes each
-  float* scales[kMaxStages];       // n/group each
-  float* zeros[kMaxStages];        // n/group each
+  void* scales[kMaxStages];        // n/group float or binary16 each
+  float* zeros[kMaxStages];        // n/group each (asymmetric grid only)
 };
 
 struct QuantizeBatch {
@@ -41,8 +48,8 @@ struct QuantizeBatch {
 
 struct ReconstructItem {
   const uint8_t* codes[kMaxStages];
-  const float* scales[kMaxStages];
-  const float* zeros[kMaxStages];
+  const void* scales[kMaxStages];  // float or binary16
+  const float* zeros[kMaxStages];  // asymmetric grid only
   uint16_t* out[kMaxStages];       // bf16 bits, n elements; out[0] only unless all prefixes
   int64_t n;
   int64_t chunk_begin;
@@ -58,12 +65,36 @@ struct ReconstructBatch {
 
 // One-time per-device set-up of kernel attributes (dynamic shared memory).
 cudaError_t quantize_prepare();
-cudaError_t reconstruct_prepare();
+cudaError_t reconstruct_prepare_asym_f32();
+cudaError_t reconstruct_prepare_sym_f32();
+cudaError_t reconstruct_prepare_sym_f16();
 
 // Launch on `stream`; `sms` = multiprocessor count of the current device.
-cudaError_t quantize_launch(int group, const QuantizeBatch& p, cudaStream_t stream, int sms);
+cudaError_t quantize_launch(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream, int sms);
 // all_prefixes: write prefixes 1..k to out[0..k-1] (else prefix k to out[0]).
-cudaError_t reconstruct_launch(int group, int k, bool all_prefixes, const ReconstructBatch& p,
-                               cudaStream_t stream, int sms);
+// One translation unit per format (they compile in parallel).
+cudaError_t reconstruct_launch_asym_f32(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                                        cudaStream_t stream, int sms);
+cudaError_t reconstruct_launch_sym_f32(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                                       cudaStream_t stream, int sms);
+cudaError_t reconstruct_launch_sym_f16(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                                       cudaStream_t stream, int sms);
+
+inline cudaError_t reconstruct_prepare() {
+  cudaError_t e;
+  if ((e = reconstruct_prepare_asym_f32())) return e;
+  if ((e = reconstruct_prepare_sym_f32())) return e;
+  return reconstruct_prepare_sym_f16();
+}
+
+inline cudaError_t reconstruct_launch(int group, Format fmt, int k, bool all_prefixes,
+                                      const ReconstructBatch& p, cudaStream_t stream, int sms) {
+  switch (fmt) {
+    case kAsymF32: return reconstruct_launch_asym_f32(group, k, all_prefixes, p, stream, sms);
+    case kSymF32: return reconstruct_launch_sym_f32(group, k, all_prefixes, p, stream, sms);
+    case kSymF16: return reconstruct_launch_sym_f16(group, k, all_prefixes, p, stream, sms);
+  }
+  return cudaErrorInvalidValue;
+}
 
 }  // namespace rrq

@@ -86,3 +86,65 @@ def check_sampled(W: torch.Tensor, pkg: binding.Package, idx: np.ndarray, ks=(1,
             bad = np.nonzero(got.reshape(-1) != want.reshape(-1))[0]
             raise AssertionError(f"{where} sampled reconstruct k={k}: {bad.size} mismatches")
         del out
+
+
+# ---------------------------------------------------------------------------
+# symmetric grid (binary32 or binary16 scales)
+# ---------------------------------------------------------------------------
+def _cmp_bytes(a, b, what):
+    a8 = np.ascontiguousarray(a).view(np.uint8)
+    b8 = np.ascontiguousarray(b).view(np.uint8)
+    if a8.shape != b8.shape or not np.array_equal(a8, b8):
+        bad = np.nonzero(a8 != b8)[0] if a8.shape == b8.shape else []
+        raise AssertionError(f"{what}: {len(bad)} byte mismatches, first at {bad[0] if len(bad) else None}")
+
+
+def scales_host(pkg):
+    """Stored scales as numpy: float32, or uint16 binary16 bit patterns."""
+    torch.cuda.synchronize()
+    if pkg.scale_type == binding.SCALE_F16:
+        return [s.view(torch.int16).cpu().numpy().view(np.uint16) for s in pkg.scales]
+    return [s.cpu().numpy() for s in pkg.scales]
+
+
+def check_full_sym(W: torch.Tensor, group: int, n_stages: int, f16: bool, where=""):
+    """Symmetric package of W through rrq_quantize_ex against the oracle (codes
+    and scales bit for bit), then every prefix through rrq_reconstruct_ex, one
+    at a time and all at once."""
+    rows, cols = W.shape
+    st = binding.SCALE_F16 if f16 else binding.SCALE_F32
+    (pkg,) = binding.rrq_quantize_ex([W], group, n_stages, binding.GRID_SYM, st)
+    rc, rs = oracle.quantize_sym(bf16_bits(W), group, n_stages, f16)
+    gs = scales_host(pkg)
+    for k in range(n_stages):
+        _cmp_bytes(pkg.codes[k].cpu().numpy(), rc[k], f"{where} stage {k} codes")
+        _cmp_bytes(gs[k], rs[k], f"{where} stage {k} scales")
+    allp = binding.rrq_reconstruct_ex([pkg], n_stages, all_prefixes=True)[0]
+    for k in range(1, n_stages + 1):
+        one = binding.rrq_reconstruct_ex([pkg], k)[0][0]
+        torch.cuda.synchronize()
+        want = oracle.reconstruct_sym(rc, rs, rows, cols, group, k, f16)
+        _cmp_bytes(bf16_bits(one), want, f"{where} reconstruct k={k}")
+        _cmp_bytes(bf16_bits(allp[k - 1]), want, f"{where} all-prefix reconstruct k={k}")
+    return pkg
+
+
+def check_sampled_sym(W: torch.Tensor, pkg, idx: np.ndarray, outs=None, where=""):
+    """Sampled groups of a symmetric package (and optionally of its prefix
+    reconstructions outs[j] = prefix j+1) against the oracle run on exactly
+    those groups."""
+    g, S = pkg.group, pkg.n_stages
+    f16 = pkg.scale_type == binding.SCALE_F16
+    it = torch.from_numpy(idx).to(W.device)
+    Wg = W.reshape(-1, g).index_select(0, it)
+    rc, rs = oracle.quantize_sym(bf16_bits(Wg), g, S, f16)
+    for k in range(S):
+        gc = pkg.codes[k].view(-1, g // 4).index_select(0, it).cpu().numpy().reshape(-1)
+        _cmp_bytes(gc, rc[k], f"{where} stage {k} codes")
+        s = pkg.scales[k].index_select(0, it)
+        gs = s.view(torch.int16).cpu().numpy().view(np.uint16) if f16 else s.cpu().numpy()
+        _cmp_bytes(gs, rs[k], f"{where} stage {k} scales")
+    for j, o in enumerate(outs or []):
+        got = bf16_bits(o.reshape(-1, g).index_select(0, it))
+        want = oracle.reconstruct_sym(rc, rs, idx.size, g, g, j + 1, f16)
+        _cmp_bytes(got, want, f"{where} sampled prefix {j + 1}")

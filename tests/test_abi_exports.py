@@ -96,3 +96,60 @@ def test_binding_refuses_cpu_tensors(lib):
     import torch
     with pytest.raises(TypeError):
         binding.rrq_quantize(torch.zeros(4, 128, dtype=torch.bfloat16))
+
+
+def _fmt(group=128, n_stages=4, grid=1, scale_type=1):
+    return binding.Format(group, n_stages, grid, scale_type)
+
+
+def test_format_size_helpers(lib):
+    n, g = 4096 * 4096, 128
+    assert binding.rrq_scales_bytes(4096, 4096, g, binding.GRID_SYM, binding.SCALE_F16) == 2 * n // g
+    assert binding.rrq_scales_bytes(4096, 4096, g, binding.GRID_SYM, binding.SCALE_F32) == 4 * n // g
+    assert binding.rrq_scales_bytes(4096, 4096, g, binding.GRID_ASYM, binding.SCALE_F32) == 4 * n // g
+    assert binding.rrq_scales_bytes(4096, 4096, g, binding.GRID_ASYM, binding.SCALE_F16) == 0
+    # symmetric binary16 package: 2 bits + 16/128 bits per weight and stage
+    assert binding.rrq_package_bytes_ex(4096, 4096, g, 4, binding.GRID_SYM, binding.SCALE_F16) == \
+        4 * (n // 4 + 2 * n // g)
+    assert binding.rrq_package_bytes_ex(4096, 4096, g, 4, binding.GRID_ASYM, binding.SCALE_F32) == \
+        binding.rrq_package_bytes(4096, 4096, g, 4)
+    assert binding.rrq_package_bytes_ex(4096, 4096, g, 5, binding.GRID_SYM, binding.SCALE_F16) == 0
+
+
+def test_ex_argument_checks_run_before_cuda(lib):
+    import torch
+    base = 1 << 20
+    no_device = 4 if not torch.cuda.is_available() else 1  # past the checks: CUDA error or not device memory
+
+    def quantize(fmt, scales=(0x30000, 0x40000), zeros=(0, 0), W=base, count=1):
+        d = binding.QuantizeDesc()
+        d.W_bf16, d.rows, d.cols = W, 4, 256
+        d.codes[0], d.codes[1] = base + 0x10000, base + 0x20000
+        d.scales[0], d.scales[1] = base + scales[0], base + scales[1]
+        d.zeros[0] = base + zeros[0] if zeros[0] else None
+        d.zeros[1] = base + zeros[1] if zeros[1] else None
+        items = (binding.QuantizeDesc * 1)(d)
+        return lib.rrq_quantize_ex(items, count, ctypes.byref(fmt) if fmt is not None else None, None)
+
+    assert quantize(None) == 1
+    assert quantize(_fmt(n_stages=2, grid=2)) == 1
+    assert quantize(_fmt(n_stages=2, scale_type=3)) == 1
+    assert quantize(_fmt(n_stages=2, grid=0, scale_type=1)) == 2   # binary16 scales need the symmetric grid
+    assert quantize(_fmt(group=48, n_stages=2)) == 2
+    assert quantize(_fmt(n_stages=2), count=0) == 1
+    assert quantize(_fmt(n_stages=2, grid=0, scale_type=0)) == 1   # asymmetric grid needs zeros
+    assert quantize(_fmt(n_stages=2), scales=(0x30002, 0x40000)) == 3
+    # 8 groups: binary16 scales span 16 bytes, binary32 scales 32 bytes
+    assert quantize(_fmt(n_stages=2, scale_type=0), scales=(0x30000, 0x30010)) == 1
+    assert quantize(_fmt(n_stages=2, scale_type=1), scales=(0x30000, 0x30010)) == no_device
+    assert quantize(_fmt(n_stages=2, scale_type=1), scales=(0x30000, 0x3000F)) == 3
+
+    r = binding.ReconstructDesc()
+    r.codes[0], r.scales[0], r.rows, r.cols = base, base + 0x10000, 4, 256
+    r.out_bf16[0] = base + 0x40000
+    items = (binding.ReconstructDesc * 1)(r)
+    assert lib.rrq_reconstruct_ex(items, 1, ctypes.byref(_fmt(n_stages=1)), 2, 0, None) == 1  # k > n_stages
+    assert lib.rrq_reconstruct_ex(items, 1, ctypes.byref(_fmt(n_stages=1)), 1, 1, None) == no_device
+    r.out_bf16[0] = base + 0x10004
+    items = (binding.ReconstructDesc * 1)(r)
+    assert lib.rrq_reconstruct_ex(items, 1, ctypes.byref(_fmt(n_stages=1)), 1, 0, None) == 3
