@@ -64,6 +64,55 @@ def alg_bytes_prefixes(n: int, k: int, g: int = GROUP) -> float:
     return 2.0 * k * n + k * (n / 4.0 + 8.0 * n / g)
 
 
+def alg_bytes_quantize_sym16(n: int, g: int = GROUP, S: int = STAGES) -> float:
+    """Symmetric package with binary16 scales: bf16 in, per stage n/4 code
+    bytes and 2 n/g scale bytes out."""
+    return n * (2 + S * (0.25 + 2.0 / g))
+
+
+def alg_bytes_prefixes_sym16(n: int, k: int, g: int = GROUP) -> float:
+    return n * (k * (0.25 + 2.0 / g) + 2 * k)
+
+
+def time_sym_f16(mats, p_outs, specs, stream, reps: int = 3) -> dict:
+    """The same stack in the paper's stored format (symmetric grid, binary16
+    scales): rrq_quantize_ex, then rrq_reconstruct_ex of every prefix, each
+    timed with CUDA events after one warm-up (breakdown context; the step
+    above is the asymmetric binary32 package)."""
+    from paper_2608_04048_gb300 import binding
+    G, F16 = binding.GRID_SYM, binding.SCALE_F16
+    pkgs = [binding.Package.empty(sp.rows, sp.cols, GROUP, STAGES, mats[0].device, G, F16) for sp in specs]
+    q_items = binding.quantize_descs(mats, pkgs)
+    r_items = binding.reconstruct_descs(pkgs, p_outs, len(KS))
+    quant = lambda: binding.rrq_quantize_ex(mats, GROUP, STAGES, G, F16, pkgs, stream, q_items)
+    recon = lambda: binding.rrq_reconstruct_ex(pkgs, len(KS), True, p_outs, stream, r_items)
+    quant(); recon()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    ev[0].record(stream)
+    for _ in range(reps):
+        quant()
+    ev[1].record(stream)
+    for _ in range(reps):
+        recon()
+    ev[2].record(stream)
+    torch.cuda.synchronize()
+    if binding.rrq_get_device_status() != 0:
+        raise RuntimeError("a kernel reported a timeout (symmetric format)")
+    q_s = ev[0].elapsed_time(ev[1]) / reps / 1e3
+    r_s = ev[1].elapsed_time(ev[2]) / reps / 1e3
+    q_alg = sum(alg_bytes_quantize_sym16(sp.numel) for sp in specs)
+    r_alg = sum(alg_bytes_prefixes_sym16(sp.numel, len(KS)) for sp in specs)
+    hbm = measured_peaks()["hbm_gbs"]
+    del pkgs
+    return {"format": "symmetric grid, binary16 scales (rrq_quantize_ex / rrq_reconstruct_ex)",
+            "quantize_s_per_stack": round(q_s, 6), "quantize_alg_gbs": round(q_alg / q_s / 1e9, 1),
+            "quantize_frac_of_measured_hbm": round(q_alg / q_s / 1e9 / hbm, 4),
+            "reconstruct_prefixes_k1to4_s": round(r_s, 6),
+            "reconstruct_prefixes_alg_gbs": round(r_alg / r_s / 1e9, 1),
+            "reconstruct_frac_of_measured_hbm": round(r_alg / r_s / 1e9 / hbm, 4),
+            "step_bf16_gbs": round(2.0 * sum(sp.numel for sp in specs) / (q_s + r_s) / 1e9, 2)}
+
+
 def alg_bytes_reconstruct(n: int, k: int, g: int = GROUP) -> float:
     """Algorithmic bytes of one rrq_reconstruct at prefix k: k code planes and
     metadata read, bf16 written."""
@@ -257,6 +306,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
     torch.cuda.synchronize()
     each_k_s = a.elapsed_time(b) / 2 / 1e3
 
+    sym = time_sym_f16(mats, p_outs, specs, stream) if not args.no_sym else None
     e2e = run_e2e(args, mats, pkgs, p_outs, specs, stream, world) if not args.no_e2e else None
     if rank != 0:
         return None
@@ -311,6 +361,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "reconstruct_frac_of_measured_hbm": round(r_gbs / peaks["hbm_gbs"], 4),
             "quantize_frac_of_nominal_8tbs": round(q_gbs / 8000.0, 4),
             "paper_context_s": {"full_all_rtn_package_qwen3_8b_a100": 1293, "four_rtn_passes_a100": 412},
+            "sym_f16": sym,
         },
         "roofline": roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic,
                                    clock_summary.get("sm_mhz")),
@@ -321,7 +372,9 @@ def run_gpu(args, world, rank, local) -> dict | None:
     return line
 
 
-FP32_OPS_PER_WEIGHT_STAGE = 8   # d, q0, remainder, q1, t, fl(Q s), level, residual
+# operations of the definition per weight and stage: v - lo, / s, rhe, Q * s,
+# lo + Q s, v - L, and the min and max that give the next stage's range
+FP32_OPS_PER_WEIGHT_STAGE = 8
 
 
 def fp32_peak_tops(sm_mhz: float | None) -> float:
@@ -508,6 +561,7 @@ def main(argv=None):
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-sym", action="store_true", help="skip the symmetric binary16 breakdown")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args(argv)
 
