@@ -92,6 +92,10 @@ class Oracle:
             ctypes.POINTER(_u8p), ctypes.POINTER(ctypes.c_void_p), ctypes.c_int64, ctypes.c_int64,
             ctypes.c_int, ctypes.c_int, ctypes.c_int, _u16p]
         lib.rrq_oracle_reconstruct_sym.restype = ctypes.c_int
+        lib.rrq_oracle_quantize_from_base.argtypes = [
+            _u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            ctypes.c_int, ctypes.POINTER(_u8p), ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(_f32p)]
+        lib.rrq_oracle_quantize_from_base.restype = ctypes.c_int
         lib.rrq_oracle_f32_to_f16.argtypes = [ctypes.c_float]
         lib.rrq_oracle_f32_to_f16.restype = ctypes.c_uint16
         lib.rrq_oracle_f16_to_f32.argtypes = [ctypes.c_uint16]
@@ -191,6 +195,34 @@ class Oracle:
             raise ValueError("oracle rejected the matrix")
         return codes, scales
 
+    def quantize_from_base(self, W_bits, base, group: int = 128, n_stages: int = 4,
+                           sym: bool = False, scale_f16: bool = False):
+        """Algorithm 1 with a base checkpoint.  base = (codes0, scales0, zeros0)
+        (zeros0 None for the symmetric grid).  Returns the whole package
+        (codes, scales, zeros), stage 0 being the given base; zeros is None for
+        the symmetric grid."""
+        W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+        rows, cols = W_bits.shape
+        n = rows * cols
+        sdt = np.uint16 if scale_f16 else np.float32
+        codes = [np.ascontiguousarray(base[0], dtype=np.uint8).copy()] + \
+            [np.zeros((n + 3) // 4, np.uint8) for _ in range(n_stages - 1)]
+        scales = [np.ascontiguousarray(base[1], dtype=sdt).copy()] + \
+            [np.zeros(n // group, sdt) for _ in range(n_stages - 1)]
+        cp = (_u8p * n_stages)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (ctypes.c_void_p * n_stages)(*[a.ctypes.data for a in scales])
+        zeros = None
+        zp = None
+        if not sym:
+            zeros = [np.ascontiguousarray(base[2], dtype=np.float32).copy()] + \
+                [np.zeros(n // group, np.float32) for _ in range(n_stages - 1)]
+            zp = (_f32p * n_stages)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        rc = self.lib.rrq_oracle_quantize_from_base(W_bits.ctypes.data_as(_u16p), rows, cols, group,
+                                                    n_stages, int(sym), int(scale_f16), cp, sp, zp)
+        if rc != 0:
+            raise ValueError("oracle rejected the base-checkpoint build")
+        return codes, scales, zeros
+
     def reconstruct_sym(self, codes, scales, rows: int, cols: int, group: int, k: int,
                         scale_f16: bool = True):
         """bf16 bit patterns [rows, cols] of the prefix-k reconstruction of a
@@ -237,3 +269,8 @@ def quantize_sym(W_bits, group: int = 128, n_stages: int = 4, scale_f16: bool = 
 
 def reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16: bool = True):
     return load().reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16)
+
+
+def quantize_from_base(W_bits, base, group: int = 128, n_stages: int = 4, sym: bool = False,
+                       scale_f16: bool = False):
+    return load().quantize_from_base(W_bits, base, group, n_stages, sym, scale_f16)

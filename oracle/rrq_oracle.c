@@ -49,6 +49,12 @@
  *     and the stage quantizes against the stored value, so that construction
  *     and reconstruction use the same scale;
  *   - (Q - 2) * s is exact in binary32, so the residual is fl(x - (Q-2)*s).
+ *
+ * Algorithm 1 with a base checkpoint: stage 0 of the package is given (codes,
+ * scales and, for the asymmetric grid, zeros, in the package's own format);
+ * it is dequantized with the same level formula as a computed stage 0, the
+ * running residual starts as fl(x - L_0), and stages 1.. are quantized from it
+ * exactly as in the build without a checkpoint.
  */
 #include "rrq_oracle.h"
 
@@ -330,5 +336,57 @@ int rrq_oracle_reconstruct_sym(const uint8_t* const* codes, const void* const* s
     }
     out[c] = rrq_oracle_f32_to_bf16(acc);
   }
+  return 0;
+}
+
+/* dequantized value of one given base code (the level formula of the grid) */
+static float base_level(int grid_sym, int q, float s, float z) {
+  if (grid_sym) return (float)(q - 2) * s;
+  float qs = (float)q * s;
+  return z + qs;
+}
+
+int rrq_oracle_quantize_from_base(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                                  int n_stages, int grid_sym, int scale_f16,
+                                  uint8_t* const* codes, void* const* scales,
+                                  float* const* zeros) {
+  if (!W || !codes || !scales || (!grid_sym && !zeros)) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || n_stages < 2) return -1;
+  if (cols % group != 0 || (scale_f16 && !grid_sym)) return -1;
+  const int64_t n = rows * cols;
+  const int64_t n_groups = n / group;
+  const int rs = n_stages - 1; /* residual stages computed here */
+
+  float* r = (float*)malloc(sizeof(float) * (size_t)group);
+  uint8_t* Q = (uint8_t*)malloc((size_t)rs * (size_t)group);
+  float* s = (float*)malloc(sizeof(float) * (size_t)rs);
+  float* z = (float*)malloc(sizeof(float) * (size_t)rs);
+  if (!r || !Q || !s || !z) {
+    free(r); free(Q); free(s); free(z);
+    return -1;
+  }
+  for (int k = 1; k < n_stages; ++k) memset(codes[k], 0, (size_t)((n + 3) / 4));
+
+  for (int64_t gi = 0; gi < n_groups; ++gi) {
+    const int64_t base = gi * group;
+    const float s0 = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[0])[gi])
+                               : ((const float*)scales[0])[gi];
+    const float z0 = grid_sym ? 0.0f : zeros[0][gi];
+    for (int j = 0; j < group; ++j) {
+      const int64_t c = base + j;
+      const int q0 = (codes[0][c / 4] >> (2 * (c % 4))) & 3;
+      const float x = rrq_oracle_bf16_to_f32(W[c]);
+      r[j] = x - base_level(grid_sym, q0, s0, z0); /* R_0 = W - W_0 */
+    }
+    if (grid_sym) rrq_oracle_quantize_group_sym(r, group, rs, scale_f16, Q, s, NULL);
+    else rrq_oracle_quantize_group(r, group, rs, Q, s, z, NULL);
+    for (int k = 1; k < n_stages; ++k) {
+      for (int j = 0; j < group; ++j) put_code(codes[k], base + j, Q[(size_t)(k - 1) * group + j]);
+      if (scale_f16) ((uint16_t*)scales[k])[gi] = rrq_oracle_f32_to_f16(s[k - 1]);
+      else ((float*)scales[k])[gi] = s[k - 1];
+      if (!grid_sym) zeros[k][gi] = z[k - 1];
+    }
+  }
+  free(r); free(Q); free(s); free(z);
   return 0;
 }

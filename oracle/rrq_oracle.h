@@ -69,6 +69,15 @@ int rrq_oracle_reconstruct_sym(const uint8_t* const* codes, const void* const* s
                                int64_t rows, int64_t cols, int group, int k, int scale_f16,
                                uint16_t* out);
 
+/* Algorithm 1 with a base checkpoint: codes[0], scales[0] (and zeros[0] for
+ * the asymmetric grid) are inputs holding stage 0 in the package's format;
+ * stages 1..n_stages-1 are written (n_stages >= 2).  grid_sym selects the
+ * symmetric grid (zeros unused, may be NULL); scale_f16 requires grid_sym. */
+int rrq_oracle_quantize_from_base(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                                  int n_stages, int grid_sym, int scale_f16,
+                                  uint8_t* const* codes, void* const* scales,
+                                  float* const* zeros);
+
 /* The scalar conversions the oracle uses, exported for tests. */
 float rrq_oracle_bf16_to_f32(uint16_t h);
 uint16_t rrq_oracle_f32_to_bf16(float f);

@@ -582,10 +582,127 @@ def pin_sym_prefix_reconstruction(orc, seed=29, rows=5, g=64) -> list[str]:
     return fails
 
 
+# ---------------------------------------------------------------------------
+# Algorithm 1 with a base checkpoint
+# ---------------------------------------------------------------------------
+# WB1 (asymmetric), x = [-1, 0, 0.5, 2], given base: every code 0, scale 1,
+# zero -1 (not the RTN base): L0 = -1 for all, R0 = [0, 1, 1.5, 3].
+#   stage 1: lo 0, hi 3, s 1, codes rhe([0, 1, 1.5, 3]) = [0, 1, 2, 3] (1.5 ties
+#            to 2), r = [0, 0, -0.5, 0];
+#   stage 2: lo -0.5, hi 0, s = fl(0.5/3) = 0x3E2AAAAB; fl(0.5/s) = 3 exactly
+#            (2.99999991 rounds up), so Q = [3, 3, 0, 3]; fl(3s) = 0.5, level
+#            -0.5 + 0.5 = 0, r = +0 everywhere;
+#   stage 3: constant +0 group, s = 0, zero +0, codes 0.
+#   prefixes: k=1 [-1]*4; k=2 [-1, 0, 1, 2]; k=3 = x.
+WB1 = dict(x=[-1.0, 0.0, 0.5, 2.0], base=([0x00], [1.0], [-1.0]),
+           Q=[[0, 1, 2, 3], [3, 3, 0, 3], [0, 0, 0, 0]],
+           scale_bits=[0x3F800000, 0x3E2AAAAB, 0x00000000], zero_bits=[0x00000000, 0xBF000000, 0x00000000],
+           recon=[[0xBF80] * 4, [0xBF80, 0x0000, 0x3F80, 0x4000], [0xBF80, 0x0000, 0x3F00, 0x4000]])
+# WB2 (symmetric, binary16), x = [0.75, -0.25, 0.5, -1], given base codes
+# [3, 2, 3, 0] with scale 0.5 (0x3800): L0 = (Q-2) 0.5 = [0.5, 0, 0.5, -1],
+# R0 = [0.25, -0.25, +0, +0].
+#   stage 1: amax 0.25, fl(0.5/3) as binary16 (spacing 2^-13 in [1/8, 1/4)):
+#            1365.33 -> 1365 * 2^-13 = 0x3155.  In units of 2^-13: 2048/1365 =
+#            1.5004 -> rhe 2 -> clamped Q 3, r = 2048 - 1365 = 683;
+#            -1.5004 -> rhe -2 -> Q 0, r = -2048 + 2730 = 682; zeros -> Q 2.
+WB2 = dict(x=[0.75, -0.25, 0.5, -1.0], base=([3 | (2 << 2) | (3 << 4) | (0 << 6)], [0x3800]),
+           Q1=[3, 0, 2, 2], scale1=0x3155)
+
+
+def _as_base(codes_byte, scales, zeros=None, f16=False):
+    return (np.array(codes_byte, np.uint8), np.array(scales, np.uint16 if f16 else np.float32),
+            None if zeros is None else np.array(zeros, np.float32))
+
+
+def pin_base_worked_groups(orc) -> list[str]:
+    fails = []
+    W = bf16_bits_of_f32(np.array(WB1["x"], np.float32)).reshape(1, 4)
+    codes, scales, zeros = orc.quantize_from_base(W, _as_base(*WB1["base"]), group=4, n_stages=4)
+    got_q = [[int((codes[k][0] >> (2 * j)) & 3) for j in range(4)] for k in (1, 2, 3)]
+    if got_q != WB1["Q"]:
+        fails.append(f"WB1: codes {got_q}")
+    if [bits_of(scales[k][0]) for k in (1, 2, 3)] != WB1["scale_bits"]:
+        fails.append(f"WB1: scales {[hex(bits_of(scales[k][0])) for k in (1, 2, 3)]}")
+    if [bits_of(zeros[k][0]) for k in (1, 2, 3)] != WB1["zero_bits"]:
+        fails.append(f"WB1: zeros {[hex(bits_of(zeros[k][0])) for k in (1, 2, 3)]}")
+    for k in (1, 2, 3):
+        rec = orc.reconstruct(codes, scales, zeros, 1, 4, 4, k)[0]
+        if rec.tolist() != WB1["recon"][k - 1]:
+            fails.append(f"WB1: recon k={k} {[hex(v) for v in rec]}")
+
+    W = bf16_bits_of_f32(np.array(WB2["x"], np.float32)).reshape(1, 4)
+    codes, scales, _ = orc.quantize_from_base(W, _as_base(*WB2["base"], f16=True), group=4,
+                                              n_stages=2, sym=True, scale_f16=True)
+    got = [int((codes[1][0] >> (2 * j)) & 3) for j in range(4)]
+    if got != WB2["Q1"] or int(scales[1][0]) != WB2["scale1"]:
+        fails.append(f"WB2: codes {got} scale {hex(int(scales[1][0]))}")
+    if int(codes[0][0]) != WB2["base"][0][0] or int(scales[0][0]) != WB2["base"][1][0]:
+        fails.append("WB2: the given base was not kept as stage 0")
+    return fails
+
+
+def pin_base_branch_equivalence(orc, seed=31, rows=4, g=64) -> list[str]:
+    """Algorithm 1's two branches are one recursion once the base is fixed:
+    given the base stage the build itself computes (RTN), the checkpoint
+    branch yields the same residual stages, for every format."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 4 * g
+    xs = np.concatenate(_random_groups(rng, rows * 4, g)).reshape(rows, cols)
+    W = bf16_bits_of_f32(xs)
+    c, s, z = orc.quantize(W, group=g, n_stages=4)
+    c2, s2, z2 = orc.quantize_from_base(W, (c[0], s[0], z[0]), group=g, n_stages=4)
+    for k in range(4):
+        if not (np.array_equal(c[k], c2[k]) and np.array_equal(s[k].view(np.uint32), s2[k].view(np.uint32))
+                and np.array_equal(z[k].view(np.uint32), z2[k].view(np.uint32))):
+            fails.append(f"asym: stage {k} differs between the two branches")
+    for f16 in (False, True):
+        c, s = orc.quantize_sym(W, group=g, n_stages=4, scale_f16=f16)
+        c2, s2, _ = orc.quantize_from_base(W, (c[0], s[0], None), group=g, n_stages=4, sym=True, scale_f16=f16)
+        for k in range(4):
+            if not (np.array_equal(c[k], c2[k]) and np.array_equal(s[k].view(np.uint8), s2[k].view(np.uint8))):
+                fails.append(f"sym f16={f16}: stage {k} differs between the two branches")
+    return fails
+
+
+def pin_base_residual_invariants(orc, seed=37, rows=3, g=128) -> list[str]:
+    """With an arbitrary given base (random codes, scales and zeros), the
+    prefix-1 reconstruction is the base's own dequantization, and every
+    residual stage obeys the half-step bound relative to the range of what it
+    quantizes, so the reconstruction error of the last prefix is at most half
+    of the last stage's step (asymmetric grid)."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 2 * g
+    xs = np.concatenate(_random_groups(rng, rows * 2, g)).reshape(rows, cols)
+    W = bf16_bits_of_f32(xs)
+    n = rows * cols
+    base = (rng.integers(0, 256, n // 4).astype(np.uint8),
+            rng.uniform(0.001, 0.05, n // g).astype(np.float32),
+            rng.uniform(-0.1, 0.0, n // g).astype(np.float32))
+    codes, scales, zeros = orc.quantize_from_base(W, base, group=g, n_stages=4)
+    rec1 = orc.reconstruct(codes, scales, zeros, rows, cols, g, 1).reshape(-1)
+    c = np.arange(n)
+    q0 = (base[0][c // 4] >> (2 * (c % 4))) & 3
+    lev = (base[2][c // g] + (q0.astype(np.float32) * base[1][c // g]).astype(np.float32)).astype(np.float32)
+    want1 = ((lev.view(np.uint32) + 0x7FFF + ((lev.view(np.uint32) >> 16) & 1)) >> 16).astype(np.uint16)
+    if not np.array_equal(rec1, want1):
+        fails.append("prefix 1 is not the given base's dequantization")
+    rec4 = orc.reconstruct(codes, scales, zeros, rows, cols, g, 4).reshape(-1)
+    recf = (rec4.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    err = np.abs(recf - xs.reshape(-1).astype(np.float64))
+    bound = 0.5 * scales[3][c // g].astype(np.float64) * (1 + 2 ** -20) + \
+        np.abs(xs.reshape(-1)) * 2 ** -8 + 2 ** -30
+    if np.any(err > bound):
+        fails.append(f"last-prefix error {err.max()} exceeds half the last step")
+    return fails
+
+
 ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_brute_force_tiny,
             pin_invariants, pin_exact_grid, pin_prefix_reconstruction, pin_f16_rounding,
             pin_sym_worked_groups, pin_sym_brute_force_exact, pin_sym_invariants,
-            pin_sym_prefix_reconstruction]
+            pin_sym_prefix_reconstruction, pin_base_worked_groups, pin_base_branch_equivalence,
+            pin_base_residual_invariants]
 
 
 def all_failures(orc) -> list[str]:

@@ -47,6 +47,13 @@ MUTANTS = {
     "f16_flushes_subnormals": ("const double n = rhe_double(a * ldexp(1.0, 24));", "const double n = 0.0;"),
     "f16_decode_exponent": ("else v = ldexp((double)(1024 + frac), e - 25);", "else v = ldexp((double)(1024 + frac), e - 24);"),
     "f16_ties_away": ("return (fmod(f, 2.0) == 0.0) ? f : f + 1.0;", "return f + 1.0;"),
+    # Algorithm 1 with a base checkpoint
+    "base_drops_zero": ("  return z + qs;", "  return qs;"),
+    "base_sym_zero_point_one": ("if (grid_sym) return (float)(q - 2) * s;", "if (grid_sym) return (float)(q - 1) * s;"),
+    "base_residual_sign": ("r[j] = x - base_level(grid_sym, q0, s0, z0);", "r[j] = x + base_level(grid_sym, q0, s0, z0);"),
+    "base_ignored": ("r[j] = x - base_level(grid_sym, q0, s0, z0);", "r[j] = x - 0.0f * base_level(grid_sym, q0, s0, z0);"),
+    "base_code_bit_order": ("const int q0 = (codes[0][c / 4] >> (2 * (c % 4))) & 3;",
+                            "const int q0 = (codes[0][c / 4] >> (2 * (3 - c % 4))) & 3;"),
 }
 
 
