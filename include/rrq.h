@@ -226,6 +226,20 @@ typedef struct {
 rrq_status rrq_quantize_ex(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
                            rrq_stream_t stream);
 
+/* Algorithm 1 with a base checkpoint (Section 3.2: the construction can start
+ * from an existing low-bit checkpoint by skipping the base quantization):
+ * stage 0 of every item's package is an INPUT in format *fmt -- codes[0],
+ * scales[0] and, for RRQ_GRID_ASYM, zeros[0] (a 2-bit checkpoint from any
+ * quantizer, stored in this layout) -- dequantized with the grid's level
+ * formula (lo + Q*s, or (Q - 2)*s); the running residual starts at
+ * R_0 = fl(W - L_0) and stages 1..n_stages-1 are computed from it exactly as
+ * rrq_quantize_ex computes them from its own stage 0 (given the base that
+ * rrq_quantize_ex would compute, the results are identical).
+ * fmt->n_stages >= 2.  The stage-0 arrays are read only; they may overlap
+ * other inputs but no output.  Other rules as for rrq_quantize_ex. */
+rrq_status rrq_quantize_from_base(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
+                                  rrq_stream_t stream);
+
 /* One matrix of rrq_reconstruct_ex: the package (first k stages) and the
  * outputs, out_bf16[0] only, or out_bf16[0..k-1] when all prefixes are
  * requested (out_bf16[j] = prefix with j+1 stages). */

@@ -22,7 +22,7 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
 #: symbols declared in include/rrq.h
 EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
            "rrq_reconstruct_prefixes", "rrq_reconstruct_prefixes_batch",
-           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_scales_bytes", "rrq_package_bytes_ex",
+           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_scales_bytes", "rrq_package_bytes_ex",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
            "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
@@ -117,6 +117,8 @@ def load_library():
     fmt_p = ctypes.POINTER(Format)
     lib.rrq_quantize_ex.argtypes = [ctypes.POINTER(QuantizeDesc), i32, fmt_p, vp]
     lib.rrq_quantize_ex.restype = i32
+    lib.rrq_quantize_from_base.argtypes = [ctypes.POINTER(QuantizeDesc), i32, fmt_p, vp]
+    lib.rrq_quantize_from_base.restype = i32
     lib.rrq_reconstruct_ex.argtypes = [ctypes.POINTER(ReconstructDesc), i32, fmt_p, i32, i32, vp]
     lib.rrq_reconstruct_ex.restype = i32
     lib.rrq_scales_bytes.argtypes = [i64, i64, fmt_p]
@@ -365,6 +367,19 @@ def rrq_quantize_ex(mats, group: int = 128, n_stages: int = 4, grid: int = GRID_
     rc = lib.rrq_quantize_ex(items, len(items), ctypes.byref(fmt), _stream_handle(stream))
     if rc != 0:
         raise RRQError(rc, "rrq_quantize_ex")
+    return pkgs
+
+
+def rrq_quantize_from_base(mats, pkgs, stream=None, items=None):
+    """Algorithm 1 with a base checkpoint: each package's stage 0 (codes[0],
+    scales[0], zeros[0]) is given; stages 1.. are computed in place."""
+    lib = load_library()
+    if items is None:
+        items = quantize_descs(mats, pkgs)
+    fmt = pkgs[0].format()
+    rc = lib.rrq_quantize_from_base(items, len(items), ctypes.byref(fmt), _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_quantize_from_base")
     return pkgs
 
 

@@ -52,6 +52,7 @@ rrq_status current_device(int* dev_out, DeviceState** state) {
     if ((e = cudaGetSymbolAddress(&addr, rrq_device_status))) return fail_cuda(e);
     d.status = static_cast<unsigned*>(addr);
     if ((e = rrq::quantize_prepare())) return fail_cuda(e);
+    if ((e = rrq::quantize_prepare_base())) return fail_cuda(e);
     if ((e = rrq::reconstruct_prepare())) return fail_cuda(e);
     d.ready = true;
   }
@@ -166,24 +167,28 @@ rrq_status check_quantize_item(const rrq_quantize_desc& it, const Fmt& f) {
   return RRQ_OK;
 }
 
-void add_quantize_ranges(const rrq_quantize_desc& it, const Fmt& f, std::vector<Range>& r) {
+// from_base: stage 0 is an input (Algorithm 1 with a base checkpoint).
+void add_quantize_ranges(const rrq_quantize_desc& it, const Fmt& f, bool from_base, std::vector<Range>& r) {
   const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
   r.push_back(range_of(it.W_bf16, 2 * n, false));
   for (int k = 0; k < f.n_stages; ++k) {
-    r.push_back(range_of(it.codes[k], n / 4, true));
-    r.push_back(range_of(it.scales[k], f.scale_bytes() * (n / f.group), true));
-    if (!f.sym()) r.push_back(range_of(it.zeros[k], 4 * (n / f.group), true));
+    const bool out = !(from_base && k == 0);
+    r.push_back(range_of(it.codes[k], n / 4, out));
+    r.push_back(range_of(it.scales[k], f.scale_bytes() * (n / f.group), out));
+    if (!f.sym()) r.push_back(range_of(it.zeros[k], 4 * (n / f.group), out));
   }
 }
 
-rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& f, rrq_stream_t stream) {
+rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& f, rrq_stream_t stream,
+                          bool from_base = false) {
   if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  if (from_base && f.n_stages < 2) return RRQ_ERR_INVALID_ARG;
   const int n_stages = f.n_stages;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (1 + 3 * n_stages));
   for (int i = 0; i < count; ++i) {
     if (rrq_status rc = check_quantize_item(items[i], f)) return rc;
-    add_quantize_ranges(items[i], f, ranges);
+    add_quantize_ranges(items[i], f, from_base, ranges);
   }
   if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
 
@@ -224,7 +229,9 @@ rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& 
       }
     }
     p.total_chunks = chunks;
-    cudaError_t e = rrq::quantize_launch(f.group, f.kind, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+    const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+    cudaError_t e = from_base ? rrq::quantize_launch_base(f.group, f.kind, p, s, st->sms)
+                              : rrq::quantize_launch(f.group, f.kind, p, s, st->sms);
     if (e != cudaSuccess) return fail_cuda(e);
   }
   return RRQ_OK;
@@ -435,6 +442,13 @@ rrq_status rrq_reconstruct_prefixes_batch(const rrq_prefixes_item* items, int co
             items[i].out_bf16};
   }
   return reconstruct_views(v.data(), count, asym_format(group, k), k, true, stream);
+}
+
+rrq_status rrq_quantize_from_base(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
+                                  rrq_stream_t stream) {
+  Fmt f;
+  if (rrq_status rc = parse_format(fmt, &f)) return rc;
+  return quantize_batch(items, count, f, stream, true);
 }
 
 rrq_status rrq_reconstruct_ex(const rrq_reconstruct_desc* items, int count, const rrq_format* fmt,

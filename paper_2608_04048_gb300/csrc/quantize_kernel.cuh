@@ -1,0 +1,578 @@
+// RRQ package construction: one fused sm_103a kernel computes every stage of
+// Algorithm 1 for a batch of bf16 weight matrices (without a base checkpoint,
+// or from a given base stage).
+//
+// Per stage k (Section 3.1 Eq. 1-3 applied to x for k = 0 and to the running
+// residual for k >= 1, Section 3.2 Eq. 4-7), for every group:
+//     lo = min v, hi = max v                     (-0 ordered before +0)
+//     s  = fl(fl(hi - lo) / 3)                   2-bit grid: 3 steps
+//     Q  = s == 0 ? 0 : clamp(rhe(fl(fl(v - lo) / s)), 0, 3)
+//     v' = fl(v - fl(lo + fl(Q * s)))            residual, kept in registers
+// Codes are packed 4 per byte (element c at bits 2*(c%4) of byte c/4); the
+// per-group scale s and zero lo are stored as binary32.
+//
+// Work decomposition: a warp owns a chunk of 1024 consecutive weights of one
+// matrix at a time (2 KiB of bf16), a lane owns 32 consecutive weights, and
+// the group/32 consecutive lanes that hold one group reduce with shuffles.
+// The chunks of all matrices of a launch form one sequence that the warps of
+// a persistent grid take in turn, so small matrices share the machine.  Each
+// warp streams its chunks through a private ring of shared-memory buffers
+// filled by 1-D bulk copies (TMA) completing on mbarriers.
+//
+// Scale.  s = RN((hi - lo) / 3) is computed as q = RN(D * RN(1/3)), then one
+// fused correction q + RN(D - 3q) * RN(1/3) (Markstein's step); this equals
+// the IEEE quotient for every binary32 D (checked exhaustively over all
+// significands).
+//
+// Code.  rhe(fl(d / s)) from a two-float reciprocal r_hi + r_lo = 1/s
+// (rcp.approx and a Newton step give r_hi; r_lo = RN(RN(1 - s*r_hi) * r_hi)),
+// relative error <= 2^-45.6: q = RN(d*r_hi + RN(d*r_lo)) (one multiply, one
+// fma) where the value before the last rounding is within x * 2^-45.3 of
+// x = d/s.  rhe(fl(x)) changes only where x crosses B1 = 0.5 + 2^-25,
+// B2 = 1.5 - 2^-24 or B3 = 2.5 + 2^-23 (the binary32 rounding boundaries next
+// to the ties 0.5, 1.5, 2.5), and rhe(RN(y)) changes at the same points, so
+// rhe(q) equals rhe(fl(d/s)) unless some float d lies within that error of
+// B_q * s.  In units of the last bit of B_q * s (an exact product of a 24-bit
+// and a 25/26-bit integer) the error is below 10 units.  How close a float can
+// come to B_q * s depends only on the significand m of s: within 64 units only
+// for m < 2^23 + 64, |m - 3*2^22| < 64 or m > 2^24 - 64 (about 1 scale in
+// 30,000).  Those groups, and scales outside [2^-90, 2^90], take the
+// per-element IEEE-division path.  Results are bit-identical to the definition
+// above in every case.
+//
+// Rounding to an integer uses t = RN(q + 2^23) = 2^23 + rhe(q) (the code is
+// the low bits of t), and the dequantized step fl(Q*s) is one fused
+// multiply-add fma(t, s, -2^23*s) with a single rounding.  (Separate packed
+// multiply and add instructions are not used for it: the compiler fuses them
+// into one fma even with -fmad=false.)
+//
+// Symmetric grid (the paper's "symmetric" configuration, Table 4 and
+// Appendix G; implicit zero-point 2, no zero stored):
+//     amax = max |v|,  s = fl(fl(2 amax) / 3)  [binary16-rounded if stored so]
+//     Q  = s == 0 ? 2 : clamp(rhe(fl(v / s)) + 2, 0, 3)
+//     v' = fl(v - (Q - 2) s)                   (Q - 2) s is exact
+// The code uses the same two-float quotient q ~ v/s; min(q, 1) applies the
+// upper clamp (rhe(x) >= 1 already means Q = 3; |x| <= 2.25 keeps the lower
+// end at Q >= 0), t = RN(min(q, 1) + C) with C = 1.5 * 2^23 + 2 gives
+// C + rhe (C is even), whose low two bits are Q, and u = t - C = Q - 2 exactly;
+// the residual is one fma(u, -s, v) = RN(v - (Q - 2) s).  The boundaries that
+// matter are +-B1 and -B2 (the same magnitudes as above), so binary32 scales
+// use the same significand test.  A binary16 scale has at most 11 significant
+// bits: then B_q * s has more than 24 significant bits with an odd top part,
+// no float d equals it, and the distance from any float to it is at least one
+// unit of 2^(exponent(s) - 48 + 13), far above the quotient's error -- every
+// binary16 scale takes the fast path.
+//
+// Algorithm 1 with a base checkpoint (kBase): stage 0 of the package is given.
+// Each lane loads its 8-byte base code word, base scale (and zero) one chunk
+// ahead, dequantizes stage 0 in registers with the grid's level formula,
+// starts the running residual at fl(x - L_0) and computes stages 1.. only.
+//
+// This header holds the kernel template; quantize.cu instantiates the build
+// without a base checkpoint, quantize_base.cu the build from one.
+#pragma once
+
+#include <cuda_fp16.h>
+
+#include "rrq_device.cuh"
+
+namespace rrq {
+namespace {
+
+#ifndef RRQ_QUANTIZE_CTAS_PER_SM
+#define RRQ_QUANTIZE_CTAS_PER_SM 3
+#endif
+#ifndef RRQ_QUANTIZE_RING
+#define RRQ_QUANTIZE_RING 4
+#endif
+constexpr int kWarps = 8;                  // warps per CTA
+constexpr int kThreads = kWarps * 32;
+constexpr int kRing = RRQ_QUANTIZE_RING;   // bulk-copy buffers per warp
+constexpr int kSmemBytes = kWarps * kRing * kChunkBytes + kWarps * kRing * 8;
+constexpr float kTwo23 = 8388608.0f;       // RN(x + 2^23) = 2^23 + rhe(x) for 0 <= x < 2^22
+constexpr float kThird = 0x1.555556p-2f;   // RN(1/3)
+constexpr float kSymRound = 12582914.0f;   // 1.5 * 2^23 + 2: RN(x + C) = C + rhe(x), low bits 2 + rhe(x)
+
+// RN(D / 3) for finite D >= 0 (exhaustively equal to IEEE division).
+__device__ __forceinline__ float div3(float D) {
+  const float q = __fmul_rn(D, kThird);
+  const float e = __fmaf_rn(-q, 3.0f, D);
+  return __fmaf_rn(e, kThird, q);
+}
+
+// 1/s as r_hi + r_lo with relative error below 2^-45.6 (s in [2^-90, 2^90]):
+// r_hi from rcp.approx and one Newton step (relative error ~2^-23),
+// r_lo = RN(1 - s*r_hi) * r_hi carries the rest.
+__device__ __forceinline__ void recip2(float s, float& r_hi, float& r_lo) {
+  float r0;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r0) : "f"(s));
+  const float e0 = __fmaf_rn(-s, r0, 1.0f);
+  r_hi = __fmaf_rn(r0, e0, r0);
+  const float e1 = __fmaf_rn(-s, r_hi, 1.0f);
+  r_lo = __fmul_rn(e1, r_hi);
+}
+
+// Per-element IEEE-division path: code and residual of one value.
+__device__ __forceinline__ int exact_code(float v, float lo, float s) {
+  if (s == 0.0f) return 0;
+  const float d = __fsub_rn(v, lo);
+  const float u = __fdiv_rn(d, s);
+  int q = __float2int_rn(u);  // round half to even
+  q = q < 0 ? 0 : q;
+  return q > 3 ? 3 : q;
+}
+struct ExactPair {
+  f32x2 w;
+  uint32_t q0, q1;
+};
+__device__ __noinline__ ExactPair exact_pair(f32x2 v, float lo, float s) {
+  float a, b;
+  unpack2(v, a, b);
+  const int qa = exact_code(a, lo, s), qb = exact_code(b, lo, s);
+  const float wa = __fsub_rn(a, __fadd_rn(lo, __fmul_rn(__int2float_rn(qa), s)));
+  const float wb = __fsub_rn(b, __fadd_rn(lo, __fmul_rn(__int2float_rn(qb), s)));
+  return {pack2(wa, wb), static_cast<uint32_t>(qa), static_cast<uint32_t>(qb)};
+}
+
+// Symmetric grid, per-element IEEE-division path.
+__device__ __forceinline__ int exact_code_sym(float v, float s) {
+  if (s == 0.0f) return 2;
+  int q = __float2int_rn(__fdiv_rn(v, s)) + 2;  // round half to even, zero-point 2
+  q = q < 0 ? 0 : q;
+  return q > 3 ? 3 : q;
+}
+__device__ __noinline__ ExactPair exact_pair_sym(f32x2 v, float s) {
+  float a, b;
+  unpack2(v, a, b);
+  const int qa = exact_code_sym(a, s), qb = exact_code_sym(b, s);
+  const float wa = __fsub_rn(a, __fmul_rn(__int2float_rn(qa - 2), s));
+  const float wb = __fsub_rn(b, __fmul_rn(__int2float_rn(qb - 2), s));
+  return {pack2(wa, wb), static_cast<uint32_t>(qa), static_cast<uint32_t>(qb)};
+}
+
+// Scales for which the corrected quotient is proven exact (see the file
+// comment): significand away from the three near-boundary bands, exponent in
+// [2^-90, 2^90].
+__device__ __forceinline__ bool corrected_quotient_safe(float s) {
+  const uint32_t bits = __float_as_uint(s);
+  const uint32_t e = bits >> 23;  // s > 0: no sign bit
+  // exponent field in [127-90, 127+89]
+  const bool range_ok = (e - (127u - 90u)) < 180u;
+  // significand field f = m - 2^23 within 64 of 0, 2^22 or 2^23 (mod 2^22)
+  const bool band = (((bits & 0x7fffffu) + 64u) & 0x3fffffu) < 128u;
+  return range_ok && !band;
+}
+
+// Appends the 2-bit code in the low bits of t to acc from the top: after
+// eight calls the codes of elements 0..7 sit at bits 16..31, element 0 lowest.
+__device__ __forceinline__ uint32_t push_code(uint32_t acc, uint32_t t) {
+  return __funnelshift_r(acc, t, 2);
+}
+
+// Stores the packed codes of stage k of this lane's 32 weights: acc[m] holds
+// the codes of slots 4m..4m+3 in its high half, in slot order.
+__device__ __forceinline__ void store_codes(uint8_t* codes, int64_t e0, const uint32_t (&acc)[4],
+                                            uint32_t sel_lo, uint32_t sel_hi) {
+  const uint32_t c0 = __byte_perm(acc[0], acc[1], 0x7632);
+  const uint32_t c1 = __byte_perm(acc[2], acc[3], 0x7632);
+  const uint2 out = make_uint2(__byte_perm(c0, c1, sel_lo), __byte_perm(c0, c1, sel_hi));
+  __stcs(reinterpret_cast<uint2*>(codes + (e0 >> 2)), out);
+}
+
+// A lane's stage-0 words of a given base checkpoint: its 32 codes (8 bytes),
+// its group's scale and zero.
+struct BaseWords {
+  uint2 code;
+  float scale;
+  float zero;
+};
+
+template <int G, int F>
+__device__ __forceinline__ BaseWords load_base(const QuantizeItem& it, int64_t e0) {
+  BaseWords b{make_uint2(0u, 0u), 0.0f, 0.0f};
+  if (e0 < it.n) {
+    b.code = __ldg(reinterpret_cast<const uint2*>(it.codes[0] + (e0 >> 2)));
+    if (F == kSymF16)
+      b.scale = __half2float(__ldg(static_cast<const __half*>(it.scales[0]) + e0 / G));
+    else
+      b.scale = __ldg(static_cast<const float*>(it.scales[0]) + e0 / G);
+    if (F == kAsymF32) b.zero = __ldg(it.zeros[0] + e0 / G);
+  }
+  return b;
+}
+
+// v <- fl(v - L_0) for the given base stage.  The code word is rotated so
+// that slot j's 8 codes sit at bits 16j (the lane reads its pieces rotated).
+template <int F>
+__device__ __forceinline__ void subtract_base(f32x2 (&v)[16], const BaseWords& b, uint32_t ld_lo,
+                                              uint32_t ld_hi) {
+  const uint32_t w0 = __byte_perm(b.code.x, b.code.y, ld_lo);
+  const uint32_t w1 = __byte_perm(b.code.x, b.code.y, ld_hi);
+  const float s = b.scale;
+  if (F == kAsymF32) {
+    // fl(Q s) = fma(2^23 + Q, s, -2^23 s) when 2^23 s is exact, else
+    // fma(t - 2^23, s, 0); then fl(zero + fl(Q s)) and fl(v - L_0)
+    const bool scaled_ok = s == 0.0f || (fabsf(s) >= 0x1p-100f && fabsf(s) <= 0x1p+100f);
+    const f32x2 S = pack2(s, s), Z = pack2(b.zero, b.zero), T23 = pack2(kTwo23, kTwo23);
+    const float c = __fmul_rn(-kTwo23, s);
+    const f32x2 C = pack2(c, c), Z0 = pack2(0.0f, 0.0f);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const uint32_t word = i < 8 ? w0 : w1;
+      const int sh = 4 * (i & 7);
+      const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+      const f32x2 qs = scaled_ok ? fma2(t, S, C) : fma2(sub2(t, T23), S, Z0);
+      v[i] = sub2(v[i], add2(Z, qs));
+    }
+  } else {
+    // (Q - 2) s is exact: fl(v - (Q-2) s) is one fma
+    const f32x2 NS = pack2(-s, -s), K2 = pack2(kTwo23 + 2.0f, kTwo23 + 2.0f);
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+      const uint32_t word = i < 8 ? w0 : w1;
+      const int sh = 4 * (i & 7);
+      const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+      v[i] = fma2(sub2(t, K2), NS, v[i]);
+    }
+  }
+}
+
+template <int G, bool kBase>
+__device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, const QuantizeItem& it,
+                                                    int64_t e0, int lane, uint4 (&raw)[4],
+                                                    uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
+                                                    uint32_t ld_lo, uint32_t ld_hi) {
+  constexpr int L = G / 32;  // lanes per group
+  const bool valid = e0 < it.n;
+  if (!valid) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) raw[j] = make_uint4(0u, 0u, 0u, 0u);
+  }
+
+  // bf16 -> binary32 (exact), pairs of consecutive weights, slot order
+  f32x2 v[16];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const uint32_t w4[4] = {raw[j].x, raw[j].y, raw[j].z, raw[j].w};
+#pragma unroll
+    for (int m = 0; m < 4; ++m) v[4 * j + m] = pack2u(w4[m] << 16, w4[m] & 0xffff0000u);
+  }
+  if constexpr (kBase) subtract_base<kAsymF32>(v, bw, ld_lo, ld_hi);  // R_0 = W - W_0
+
+  float lo, hi;
+  lane_minmax(v, lo, hi);
+  group_minmax<L>(lo, hi);
+
+#pragma unroll 1
+  for (int k = kBase ? 1 : 0; k < p.n_stages; ++k) {
+    // A zero minimum: the stored offset is -0 if the group holds a -0.
+    if (__any_sync(kFullMask, lo == 0.0f)) {
+      uint32_t neg = 0;
+      if (lo == 0.0f) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          neg |= (static_cast<uint32_t>(v[i]) == 0x80000000u) |
+                 (static_cast<uint32_t>(v[i] >> 32) == 0x80000000u);
+      }
+      neg = group_or<L>(neg);
+      if (lo == 0.0f) lo = neg ? -0.0f : 0.0f;
+    }
+
+    const float s = div3(__fsub_rn(hi, lo));
+    const bool fast = !(p.flags & kDebugForceExact) && (s == 0.0f || corrected_quotient_safe(s));
+    uint32_t acc[4] = {0u, 0u, 0u, 0u};
+    // min/max of the new residual (next stage's range), gathered in the loop
+    float mn0 = __int_as_float(0x7f800000), mn1 = mn0, mx0 = -mn0, mx1 = mx0;
+    if (fast) {
+      float r_hi = 0.0f, r_lo = 0.0f;
+      if (s > 0.0f) recip2(s, r_hi, r_lo);
+      const float c = __fmul_rn(-kTwo23, s);  // exact: power-of-two scaling
+      const f32x2 LO = pack2(lo, lo), RH = pack2(r_hi, r_hi), RL = pack2(r_lo, r_lo), S = pack2(s, s);
+      const f32x2 T23 = pack2(kTwo23, kTwo23), C = pack2(c, c);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const f32x2 d = sub2(v[i], LO);
+        const f32x2 q = fma2(d, RH, mul2(d, RL));  // d/s to 2^-45.3
+        const f32x2 t = add2(q, T23);              // 2^23 + rhe(q)
+        const f32x2 step = fma2(t, S, C);    // fl(Q*s)
+        v[i] = sub2(v[i], add2(LO, step));   // v - fl(lo + fl(Q*s))
+        acc[i >> 2] = push_code(push_code(acc[i >> 2], static_cast<uint32_t>(t)),
+                                static_cast<uint32_t>(t >> 32));
+        float a, b;
+        unpack2(v[i], a, b);
+        if (i & 1) {
+          mn1 = fminf(mn1, fminf(a, b));
+          mx1 = fmaxf(mx1, fmaxf(a, b));
+        } else {
+          mn0 = fminf(mn0, fminf(a, b));
+          mx0 = fmaxf(mx0, fmaxf(a, b));
+        }
+      }
+    } else {  // this group: IEEE division element by element
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const ExactPair x = exact_pair(v[i], lo, s);
+        v[i] = x.w;
+        acc[i >> 2] = push_code(push_code(acc[i >> 2], x.q0), x.q1);
+      }
+      lane_minmax(v, mn0, mx0);
+    }
+
+    if (valid) {
+      store_codes(it.codes[k], e0, acc, sel_lo, sel_hi);
+      if ((lane & (L - 1)) == 0) {
+        __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s);
+        __stcs(it.zeros[k] + e0 / G, lo);
+      }
+    }
+    if (k + 1 < p.n_stages) {  // range of the residual = next stage's lo, hi
+      lo = fminf(mn0, mn1);
+      hi = fmaxf(mx0, mx1);
+      group_minmax<L>(lo, hi);
+    }
+  }
+}
+
+// Symmetric grid; kF16: the scale is rounded to binary16, stored as such, and
+// the stage quantizes against the rounded value.
+template <int G, bool kF16, bool kBase>
+__device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const QuantizeItem& it,
+                                                   int64_t e0, int lane, uint4 (&raw)[4],
+                                                   uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
+                                                   uint32_t ld_lo, uint32_t ld_hi) {
+  constexpr int L = G / 32;  // lanes per group
+  const bool valid = e0 < it.n;
+  if (!valid) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) raw[j] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  f32x2 v[16];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const uint32_t w4[4] = {raw[j].x, raw[j].y, raw[j].z, raw[j].w};
+#pragma unroll
+    for (int m = 0; m < 4; ++m) v[4 * j + m] = pack2u(w4[m] << 16, w4[m] & 0xffff0000u);
+  }
+  if constexpr (kBase) subtract_base<kSymF32>(v, bw, ld_lo, ld_hi);  // R_0 = W - W_0
+  float amax = group_max<L>(lane_amax(v));
+
+#pragma unroll 1
+  for (int k = kBase ? 1 : 0; k < p.n_stages; ++k) {
+    float s = div3(__fmul_rn(amax, 2.0f));  // 2 * amax is exact
+    uint16_t s16 = 0;
+    if (kF16) {
+      s16 = __half_as_ushort(__float2half_rn(s));
+      s = __half2float(__ushort_as_half(s16));
+    }
+    const bool fast = !(p.flags & kDebugForceExact) && (kF16 || s == 0.0f || corrected_quotient_safe(s));
+    uint32_t acc[4] = {0u, 0u, 0u, 0u};
+    float mx0 = 0.0f, mx1 = 0.0f;  // max |new residual|, gathered in the loop
+    if (fast) {
+      float r_hi = 0.0f, r_lo = 0.0f;
+      if (s > 0.0f) recip2(s, r_hi, r_lo);
+      const f32x2 RH = pack2(r_hi, r_hi), RL = pack2(r_lo, r_lo), NS = pack2(-s, -s);
+      const f32x2 C = pack2(kSymRound, kSymRound);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const f32x2 q = fma2(v[i], RH, mul2(v[i], RL));  // v/s to 2^-45.3
+        float qa, qb;
+        unpack2(q, qa, qb);
+        const f32x2 t = add2(pack2(fminf(qa, 1.0f), fminf(qb, 1.0f)), C);  // C + rhe, clamped
+        const f32x2 u = sub2(t, C);                                       // Q - 2, exact
+        v[i] = fma2(u, NS, v[i]);                                         // v - (Q-2) s
+        acc[i >> 2] = push_code(push_code(acc[i >> 2], static_cast<uint32_t>(t)),
+                                static_cast<uint32_t>(t >> 32));
+        float a, b;
+        unpack2(v[i], a, b);
+        if (i & 1) mx1 = fmaxf(mx1, fmaxf(fabsf(a), fabsf(b)));
+        else mx0 = fmaxf(mx0, fmaxf(fabsf(a), fabsf(b)));
+      }
+    } else {  // this group: IEEE division element by element
+#pragma unroll
+      for (int i = 0; i < 16; ++i) {
+        const ExactPair x = exact_pair_sym(v[i], s);
+        v[i] = x.w;
+        acc[i >> 2] = push_code(push_code(acc[i >> 2], x.q0), x.q1);
+      }
+      mx0 = lane_amax(v);
+    }
+
+    if (valid) {
+      store_codes(it.codes[k], e0, acc, sel_lo, sel_hi);
+      if ((lane & (L - 1)) == 0) {
+        if (kF16) stcs_u16(static_cast<uint16_t*>(it.scales[k]) + e0 / G, s16);
+        else __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s);
+      }
+    }
+    if (k + 1 < p.n_stages) amax = group_max<L>(fmaxf(mx0, mx1));
+  }
+}
+
+template <int G, int F, bool kBase>
+__device__ __forceinline__ void quantize_chunk(const QuantizeBatch& p, const QuantizeItem& it,
+                                               int64_t e0, int lane, uint4 (&raw)[4],
+                                               uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
+                                               uint32_t ld_lo, uint32_t ld_hi) {
+  if constexpr (F == kAsymF32)
+    quantize_chunk_asym<G, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
+  else
+    quantize_chunk_sym<G, F == kSymF16, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
+}
+
+template <int G, int F, bool kBase>
+__global__ void __launch_bounds__(kThreads, RRQ_QUANTIZE_CTAS_PER_SM) quantize_kernel(const __grid_constant__ QuantizeBatch p) {
+  extern __shared__ __align__(128) uint8_t smem[];
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  uint8_t* ring = smem + warp * (kRing * kChunkBytes);
+  const uint32_t ring_s = smem_u32(ring);
+  const uint32_t bar0 = smem_u32(smem + kWarps * kRing * kChunkBytes) + warp * kRing * 8;
+
+  const int64_t first = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
+  const int64_t stride = static_cast<int64_t>(gridDim.x) * kWarps;
+  if (first >= p.total_chunks) return;  // warp-uniform: nothing issued, nothing to wait for
+
+  if (lane == 0) {
+#pragma unroll
+    for (int b = 0; b < kRing; ++b) mbar_init(bar0 + 8 * b, 1);
+    fence_mbarrier_init();
+  }
+  __syncwarp();
+
+  // matrix of a chunk: chunks only move forward, so a running index suffices
+  int m_issue = 0, m_work = 0;
+  auto item_of = [&](int64_t chunk, int& m) -> const QuantizeItem& {
+    while (m + 1 < p.count && chunk >= p.item[m + 1].chunk_begin) ++m;
+    return p.item[m];
+  };
+  auto issue = [&](int64_t chunk, int b) {  // lane 0 only
+    const QuantizeItem& it = item_of(chunk, m_issue);
+    const int64_t e = (chunk - it.chunk_begin) * kChunkElems;
+    const int64_t left = it.n - e;
+    const uint32_t bytes = static_cast<uint32_t>((left < kChunkElems ? left : kChunkElems) * 2);
+    mbar_arrive_expect_tx(bar0 + 8 * b, bytes);
+    bulk_load(ring_s + b * kChunkBytes, it.W + e, bytes, bar0 + 8 * b);
+  };
+  if (lane == 0) {
+#pragma unroll
+    for (int b = 0; b < kRing; ++b) {
+      const int64_t c = first + b * stride;
+      if (c < p.total_chunks) issue(c, b);
+    }
+  }
+
+  // Lane l reads its four 16-byte pieces in rotated order so that a quarter
+  // warp touches eight distinct bank groups; slot j holds piece (j+rot)&3.
+  const int rot = (lane >> 1) & 3;
+  const uint32_t sel_lo = rot == 0 ? 0x3210u : rot == 1 ? 0x1076u : rot == 2 ? 0x7654u : 0x5432u;
+  const uint32_t sel_hi = rot == 0 ? 0x7654u : rot == 1 ? 0x5432u : rot == 2 ? 0x3210u : 0x1076u;
+  // the inverse rotation, for a base code word read in memory order
+  const uint32_t ld_lo = rot == 0 ? 0x3210u : rot == 1 ? 0x5432u : rot == 2 ? 0x7654u : 0x1076u;
+  const uint32_t ld_hi = rot == 0 ? 0x7654u : rot == 1 ? 0x1076u : rot == 2 ? 0x3210u : 0x5432u;
+
+  // base words of this warp's chunks, loaded one chunk ahead
+  int m_base = 0;
+  auto base_of = [&](int64_t chunk) -> BaseWords {
+    if (!kBase || chunk >= p.total_chunks) return BaseWords{make_uint2(0u, 0u), 0.0f, 0.0f};
+    const QuantizeItem& it = item_of(chunk, m_base);
+    return load_base<G, F>(it, (chunk - it.chunk_begin) * kChunkElems + static_cast<int64_t>(lane) * kLaneElems);
+  };
+  BaseWords bw_next = base_of(first);
+
+  uint32_t iter = 0;
+  for (int64_t chunk = first; chunk < p.total_chunks; chunk += stride, ++iter) {
+    const int b = iter % kRing;
+    const bool ready = mbar_wait(bar0 + 8 * b, (iter / kRing) & 1, p.wait_limit_us);
+    if (!__all_sync(kFullMask, ready)) {
+      // Give up: record it, wait (bounded) for this warp's copies in flight
+      // so that none lands in freed shared memory, and leave.
+      if (lane == 0) {
+        atomicOr(p.status, kStatusTimeout);
+        for (int j = 0; j < kRing; ++j) {
+          if (chunk + j * stride >= p.total_chunks) break;
+          const uint32_t jt = iter + j;
+          mbar_wait(bar0 + 8 * (jt % kRing), (jt / kRing) & 1, kDrainLimitUs);
+        }
+      }
+      __syncwarp();
+      return;
+    }
+    const uint4* src = reinterpret_cast<const uint4*>(ring + b * kChunkBytes + lane * 64);
+    uint4 raw[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j) raw[j] = src[(j + rot) & 3];
+    __syncwarp();
+    if (lane == 0) {
+      const int64_t next = chunk + kRing * stride;
+      if (next < p.total_chunks) {
+        fence_proxy_async_smem();
+        issue(next, b);
+      }
+    }
+    const QuantizeItem& it = item_of(chunk, m_work);
+    const int64_t e0 = (chunk - it.chunk_begin) * kChunkElems + static_cast<int64_t>(lane) * kLaneElems;
+    const BaseWords bw = bw_next;
+    if (kBase) bw_next = base_of(chunk + stride);  // in flight while this chunk computes
+    quantize_chunk<G, F, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
+  }
+}
+
+template <int G, int F, bool kBase>
+cudaError_t launch_gf(const QuantizeBatch& p, cudaStream_t stream, int sms) {
+  static int blocks_per_sm = 0;  // same for every device of this build
+  if (blocks_per_sm == 0) {
+    cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
+        &blocks_per_sm, quantize_kernel<G, F, kBase>, kThreads, kSmemBytes);
+    if (e != cudaSuccess) return e;
+    if (blocks_per_sm < 1) blocks_per_sm = 1;
+  }
+  const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
+  const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
+  const int grid = static_cast<int>(want < cap ? want : cap);
+  quantize_kernel<G, F, kBase><<<grid, kThreads, kSmemBytes, stream>>>(p);
+  return cudaGetLastError();
+}
+
+template <int F, bool kBase>
+cudaError_t launch_f(int group, const QuantizeBatch& p, cudaStream_t stream, int sms) {
+  switch (group) {
+    case 32: return launch_gf<32, F, kBase>(p, stream, sms);
+    case 64: return launch_gf<64, F, kBase>(p, stream, sms);
+    case 128: return launch_gf<128, F, kBase>(p, stream, sms);
+    case 256: return launch_gf<256, F, kBase>(p, stream, sms);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int F, bool kBase>
+cudaError_t prepare_f() {
+  cudaError_t e;
+  const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  if ((e = cudaFuncSetAttribute(quantize_kernel<32, F, kBase>, a, kSmemBytes))) return e;
+  if ((e = cudaFuncSetAttribute(quantize_kernel<64, F, kBase>, a, kSmemBytes))) return e;
+  if ((e = cudaFuncSetAttribute(quantize_kernel<128, F, kBase>, a, kSmemBytes))) return e;
+  return cudaFuncSetAttribute(quantize_kernel<256, F, kBase>, a, kSmemBytes);
+}
+
+// Set-up and launch of every format, with or without a base checkpoint
+// (instantiated by quantize.cu and quantize_base.cu).
+template <bool kBase>
+cudaError_t prepare_all() {
+  cudaError_t e;
+  if ((e = prepare_f<kAsymF32, kBase>())) return e;
+  if ((e = prepare_f<kSymF32, kBase>())) return e;
+  return prepare_f<kSymF16, kBase>();
+}
+
+template <bool kBase>
+cudaError_t launch_all(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream, int sms) {
+  switch (fmt) {
+    case kAsymF32: return launch_f<kAsymF32, kBase>(group, p, stream, sms);
+    case kSymF32: return launch_f<kSymF32, kBase>(group, p, stream, sms);
+    case kSymF16: return launch_f<kSymF16, kBase>(group, p, stream, sms);
+  }
+  return cudaErrorInvalidValue;
+}
+
+}  // namespace
+}  // namespace rrq

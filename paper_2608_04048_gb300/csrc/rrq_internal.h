@@ -65,12 +65,17 @@ struct ReconstructBatch {
 
 // One-time per-device set-up of kernel attributes (dynamic shared memory).
 cudaError_t quantize_prepare();
+cudaError_t quantize_prepare_base();
 cudaError_t reconstruct_prepare_asym_f32();
 cudaError_t reconstruct_prepare_sym_f32();
 cudaError_t reconstruct_prepare_sym_f16();
 
 // Launch on `stream`; `sms` = multiprocessor count of the current device.
 cudaError_t quantize_launch(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream, int sms);
+// Stage 0 given (item codes[0], scales[0], zeros[0] are inputs); stages
+// 1..n_stages-1 computed.
+cudaError_t quantize_launch_base(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream,
+                                 int sms);
 // all_prefixes: write prefixes 1..k to out[0..k-1] (else prefix k to out[0]).
 // One translation unit per format (they compile in parallel).
 cudaError_t reconstruct_launch_asym_f32(int group, int k, bool all_prefixes, const ReconstructBatch& p,
