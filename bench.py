@@ -113,6 +113,30 @@ def time_sym_f16(mats, p_outs, specs, stream, reps: int = 3) -> dict:
             "step_bf16_gbs": round(2.0 * sum(sp.numel for sp in specs) / (q_s + r_s) / 1e9, 2)}
 
 
+def time_from_base(mats, pkgs, specs, stream, reps: int = 3) -> dict:
+    """Algorithm 1 from a base checkpoint on the same stack: each package's
+    stage 0 (left by the timed step) is taken as the given base and stages
+    1..3 are rebuilt by rrq_quantize_from_base (reads W and the base stage,
+    writes three stages: the same 3.25 B/weight as the full build)."""
+    from paper_2608_04048_gb300 import binding
+    items = binding.quantize_descs(mats, pkgs)
+    run = lambda: binding.rrq_quantize_from_base(mats, pkgs, stream, items)
+    run()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        run()
+    b.record(stream)
+    torch.cuda.synchronize()
+    if binding.rrq_get_device_status() != 0:
+        raise RuntimeError("a kernel reported a timeout (from base)")
+    t = a.elapsed_time(b) / reps / 1e3
+    alg = sum(alg_bytes_quantize(sp.numel) for sp in specs)
+    return {"call": "rrq_quantize_from_base (asymmetric, binary32), stage 0 given",
+            "s_per_stack": round(t, 6), "alg_gbs": round(alg / t / 1e9, 1),
+            "frac_of_measured_hbm": round(alg / t / 1e9 / measured_peaks()["hbm_gbs"], 4)}
+
+
 def alg_bytes_reconstruct(n: int, k: int, g: int = GROUP) -> float:
     """Algorithmic bytes of one rrq_reconstruct at prefix k: k code planes and
     metadata read, bf16 written."""
@@ -307,6 +331,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
     each_k_s = a.elapsed_time(b) / 2 / 1e3
 
     sym = time_sym_f16(mats, p_outs, specs, stream) if not args.no_sym else None
+    from_base = time_from_base(mats, pkgs, specs, stream) if not args.no_sym else None
     e2e = run_e2e(args, mats, pkgs, p_outs, specs, stream, world) if not args.no_e2e else None
     if rank != 0:
         return None
@@ -362,6 +387,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "quantize_frac_of_nominal_8tbs": round(q_gbs / 8000.0, 4),
             "paper_context_s": {"full_all_rtn_package_qwen3_8b_a100": 1293, "four_rtn_passes_a100": 412},
             "sym_f16": sym,
+            "from_base": from_base,
         },
         "roofline": roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic,
                                    clock_summary.get("sm_mhz")),
@@ -561,7 +587,8 @@ def main(argv=None):
     ap.add_argument("--workload", default=WORKLOAD)
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--no-sym", action="store_true", help="skip the symmetric binary16 breakdown")
+    ap.add_argument("--no-sym", action="store_true",
+                    help="skip the symmetric binary16 and base-checkpoint breakdown")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args(argv)
 
