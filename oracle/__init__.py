@@ -96,6 +96,11 @@ class Oracle:
             _u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int,
             ctypes.c_int, ctypes.POINTER(_u8p), ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(_f32p)]
         lib.rrq_oracle_quantize_from_base.restype = ctypes.c_int
+        lib.rrq_oracle_gemv.argtypes = [
+            ctypes.POINTER(_u8p), ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(_f32p),
+            ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            _u16p, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
+        lib.rrq_oracle_gemv.restype = ctypes.c_int
         lib.rrq_oracle_f32_to_f16.argtypes = [ctypes.c_float]
         lib.rrq_oracle_f32_to_f16.restype = ctypes.c_uint16
         lib.rrq_oracle_f16_to_f32.argtypes = [ctypes.c_uint16]
@@ -223,6 +228,30 @@ class Oracle:
             raise ValueError("oracle rejected the base-checkpoint build")
         return codes, scales, zeros
 
+    def gemv(self, codes, scales, zeros, rows: int, cols: int, group: int, k: int, A_bits,
+             sym: bool = False, scale_f16: bool = False):
+        """Y [batch, rows] float64 = A [batch, cols] (bf16 bit patterns) times
+        the transposed prefix-k weights (binary32 stage sums)."""
+        A_bits = np.ascontiguousarray(np.atleast_2d(A_bits), dtype=np.uint16)
+        batch = A_bits.shape[0]
+        assert A_bits.shape[1] == cols
+        sdt = np.uint16 if scale_f16 else np.float32
+        codes = [np.ascontiguousarray(c, dtype=np.uint8) for c in codes[:k]]
+        scales = [np.ascontiguousarray(a, dtype=sdt) for a in scales[:k]]
+        cp = (_u8p * k)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (ctypes.c_void_p * k)(*[a.ctypes.data for a in scales])
+        zp = None
+        if not sym:
+            zeros = [np.ascontiguousarray(a, dtype=np.float32) for a in zeros[:k]]
+            zp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        Y = np.zeros((batch, rows), np.float64)
+        rc = self.lib.rrq_oracle_gemv(cp, sp, zp, rows, cols, group, k, int(sym), int(scale_f16),
+                                      A_bits.ctypes.data_as(_u16p), batch,
+                                      Y.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
+        if rc != 0:
+            raise ValueError("oracle rejected the product")
+        return Y
+
     def reconstruct_sym(self, codes, scales, rows: int, cols: int, group: int, k: int,
                         scale_f16: bool = True):
         """bf16 bit patterns [rows, cols] of the prefix-k reconstruction of a
@@ -269,6 +298,10 @@ def quantize_sym(W_bits, group: int = 128, n_stages: int = 4, scale_f16: bool = 
 
 def reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16: bool = True):
     return load().reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16)
+
+
+def gemv(codes, scales, zeros, rows, cols, group, k, A_bits, sym: bool = False, scale_f16: bool = False):
+    return load().gemv(codes, scales, zeros, rows, cols, group, k, A_bits, sym, scale_f16)
 
 
 def quantize_from_base(W_bits, base, group: int = 128, n_stages: int = 4, sym: bool = False,

@@ -50,6 +50,12 @@
  *     and reconstruction use the same scale;
  *   - (Q - 2) * s is exact in binary32, so the residual is fl(x - (Q-2)*s).
  *
+ * Stage-wise product (Appendix C: A W~_(t) = A W^_0 + sum_k A R^_k): with
+ * the prefix-k weight W~[r][c] = the binary32 stage sum of the reconstruction
+ * (before its bf16 rounding), Y[b][r] = sum_c W~[r][c] * A[b][c], the
+ * products and the sum taken in binary64 (each product of a binary32 and a
+ * bf16 value is exact there).
+ *
  * Algorithm 1 with a base checkpoint: stage 0 of the package is given (codes,
  * scales and, for the asymmetric grid, zeros, in the package's own format);
  * it is dequantized with the same level formula as a computed stage 0, the
@@ -388,5 +394,32 @@ int rrq_oracle_quantize_from_base(const uint16_t* W, int64_t rows, int64_t cols,
     }
   }
   free(r); free(Q); free(s); free(z);
+  return 0;
+}
+
+int rrq_oracle_gemv(const uint8_t* const* codes, const void* const* scales,
+                    const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
+                    int grid_sym, int scale_f16, const uint16_t* A, int batch, double* Y) {
+  if (!codes || !scales || (!grid_sym && !zeros) || !A || !Y) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || k < 1 || batch < 1) return -1;
+  if (cols % group != 0 || (scale_f16 && !grid_sym)) return -1;
+  for (int b = 0; b < batch; ++b)
+    for (int64_t r = 0; r < rows; ++r) Y[(size_t)b * rows + r] = 0.0;
+  for (int64_t r = 0; r < rows; ++r) {
+    for (int64_t j = 0; j < cols; ++j) {
+      const int64_t c = r * cols + j;
+      const int64_t gi = c / group;
+      float w = 0.0f; /* prefix weight W~[r][j] */
+      for (int i = 0; i < k; ++i) {
+        const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;
+        const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])
+                                  : ((const float*)scales[i])[gi];
+        const float lv = base_level(grid_sym, q, s, grid_sym ? 0.0f : zeros[i][gi]);
+        w = (i == 0) ? lv : w + lv;
+      }
+      for (int b = 0; b < batch; ++b)
+        Y[(size_t)b * rows + r] += (double)w * (double)rrq_oracle_bf16_to_f32(A[(size_t)b * cols + j]);
+    }
+  }
   return 0;
 }

@@ -78,6 +78,14 @@ int rrq_oracle_quantize_from_base(const uint16_t* W, int64_t rows, int64_t cols,
                                   uint8_t* const* codes, void* const* scales,
                                   float* const* zeros);
 
+/* Product of activations with the prefix-k weights (Appendix C):
+ * Y[b][r] = sum_c W~[r][c] * A[b][c] in binary64, W~ = the binary32 stage sum
+ * of the first k stages (the reconstruction before bf16 rounding).
+ *   A  bf16 bit patterns [batch][cols];  Y  double [batch][rows]. */
+int rrq_oracle_gemv(const uint8_t* const* codes, const void* const* scales,
+                    const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
+                    int grid_sym, int scale_f16, const uint16_t* A, int batch, double* Y);
+
 /* The scalar conversions the oracle uses, exported for tests. */
 float rrq_oracle_bf16_to_f32(uint16_t h);
 uint16_t rrq_oracle_f32_to_bf16(float f);

@@ -49,6 +49,12 @@ def bf16_bits_of_f32(x: np.ndarray) -> np.ndarray:
     return (u >> 16).astype(np.uint16)
 
 
+def bf16_round_bits(x) -> np.ndarray:
+    """bf16 bit patterns of float32 values rounded to nearest-even."""
+    u = np.asarray(x, np.float32).view(np.uint32)
+    return ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+
+
 def _golden_cases():
     with open(GOLDEN) as f:
         return {c["name"]: c for c in json.load(f)["cases"]}
@@ -698,11 +704,95 @@ def pin_base_residual_invariants(orc, seed=37, rows=3, g=128) -> list[str]:
     return fails
 
 
+# ---------------------------------------------------------------------------
+# stage-wise product with the prefix weights (Appendix C)
+# ---------------------------------------------------------------------------
+# GV1: the WE1 package (x = [-1, 0, 0.5, 2]; prefix 1 = [-1, 0, 1, 2], prefix 2
+# = x exactly) times A = [[2, -1, 4, 0.25], [1, 1, 1, 1]]:
+#   k=1: [-2 + 0 + 4 + 0.5, -1 + 0 + 1 + 2] = [2.5, 2];  k=2: [-2 + 0 + 2 + 0.5, 1.5].
+# GV2: the WS1 symmetric package (x = [-1.5, -1, 0.5, 1.5], binary32 scales),
+#   k=1 levels [-2, -1, 0, 1] -> A[0] . = -4 + 1 + 0 + 0.25 = -2.75.
+GV_A = [[2.0, -1.0, 4.0, 0.25], [1.0, 1.0, 1.0, 1.0]]
+
+
+def pin_gemv_worked(orc) -> list[str]:
+    fails = []
+    A = bf16_bits_of_f32(np.array(GV_A, np.float32))
+    W = bf16_bits_of_f32(np.array([-1.0, 0.0, 0.5, 2.0], np.float32)).reshape(1, 4)
+    codes, scales, zeros = orc.quantize(W, group=4, n_stages=2)
+    for k, want in ((1, [2.5, 2.0]), (2, [0.5, 1.5])):
+        Y = orc.gemv(codes, scales, zeros, 1, 4, 4, k, A)
+        if Y[:, 0].tolist() != want:
+            fails.append(f"GV1 k={k}: {Y[:, 0].tolist()} != {want}")
+    W = bf16_bits_of_f32(np.array(WS1["x"], np.float32)).reshape(1, 4)
+    codes, scales = orc.quantize_sym(W, group=4, n_stages=2, scale_f16=False)
+    Y = orc.gemv(codes, scales, None, 1, 4, 4, 1, A[:1], sym=True)
+    if Y[0, 0] != -2.75:
+        fails.append(f"GV2: {Y[0, 0]} != -2.75")
+    return fails
+
+
+def pin_gemv_is_input_minus_residual(orc, seed=41, rows=6, g=64) -> list[str]:
+    """Eq. 8 with Eq. 5-7 in product form: A W~_(k) = A X - A R_(k-1) (the
+    prefix-k weight is the input minus the residual after stage k-1, taken
+    from the stage-by-stage quantizer), up to the binary32 rounding of the
+    stage sums; for every format."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 3 * g
+    xs = np.concatenate(_random_groups(rng, rows * 3, g)).reshape(rows, cols)
+    W = bf16_bits_of_f32(xs)
+    A = bf16_round_bits(rng.normal(0, 1, (3, cols)).astype(np.float32))
+    Af = (A.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    for sym, f16 in ((False, False), (True, False), (True, True)):
+        if sym:
+            codes, scales = orc.quantize_sym(W, group=g, n_stages=4, scale_f16=f16)
+            zeros = None
+        else:
+            codes, scales, zeros = orc.quantize(W, group=g, n_stages=4)
+        resid = []
+        for gi in range(rows * cols // g):
+            x = xs.reshape(-1)[gi * g:(gi + 1) * g]
+            r = orc.quantize_group_sym(x, 4, f16)[2] if sym else orc.quantize_group(x, 4)[3]
+            resid.append(r)
+        resid = np.concatenate(resid, axis=1).astype(np.float64)  # [4, n]
+        for k in range(1, 5):
+            Y = orc.gemv(codes, scales, zeros, rows, cols, g, k, A, sym, f16)
+            wk = (xs.reshape(-1).astype(np.float64) - resid[k - 1]).reshape(rows, cols)
+            want = Af @ wk.T
+            tol = np.abs(Af) @ (np.abs(xs).astype(np.float64) + np.abs(wk)).T * (k + 1) * 2.0 ** -23
+            if np.any(np.abs(Y - want) > tol + 1e-300):
+                fails.append(f"sym={sym} f16={f16} k={k}: A W~ != A X - A R")
+    return fails
+
+
+def pin_gemv_vs_bf16_reconstruction(orc, seed=43, rows=5, g=128) -> list[str]:
+    """The product equals A times the bf16 reconstruction (a separately
+    pinned routine) up to the bf16 rounding of each weight (2^-9 relative)."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 2 * g
+    xs = np.concatenate(_random_groups(rng, rows * 2, g)).reshape(rows, cols)
+    W = bf16_bits_of_f32(xs)
+    codes, scales, zeros = orc.quantize(W, group=g, n_stages=4)
+    A = bf16_round_bits(rng.normal(0, 1, (2, cols)).astype(np.float32))
+    Af = (A.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    for k in range(1, 5):
+        rec = orc.reconstruct(codes, scales, zeros, rows, cols, g, k)
+        recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        Y = orc.gemv(codes, scales, zeros, rows, cols, g, k, A)
+        tol = np.abs(Af) @ np.abs(recf).T * 2.0 ** -8 + 1e-300
+        if np.any(np.abs(Y - Af @ recf.T) > tol):
+            fails.append(f"k={k}: product differs from A x bf16 reconstruction beyond bf16 rounding")
+    return fails
+
+
 ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_brute_force_tiny,
             pin_invariants, pin_exact_grid, pin_prefix_reconstruction, pin_f16_rounding,
             pin_sym_worked_groups, pin_sym_brute_force_exact, pin_sym_invariants,
             pin_sym_prefix_reconstruction, pin_base_worked_groups, pin_base_branch_equivalence,
-            pin_base_residual_invariants]
+            pin_base_residual_invariants, pin_gemv_worked, pin_gemv_is_input_minus_residual,
+            pin_gemv_vs_bf16_reconstruction]
 
 
 def all_failures(orc) -> list[str]:

@@ -54,6 +54,15 @@ MUTANTS = {
     "base_ignored": ("r[j] = x - base_level(grid_sym, q0, s0, z0);", "r[j] = x - 0.0f * base_level(grid_sym, q0, s0, z0);"),
     "base_code_bit_order": ("const int q0 = (codes[0][c / 4] >> (2 * (c % 4))) & 3;",
                             "const int q0 = (codes[0][c / 4] >> (2 * (3 - c % 4))) & 3;"),
+    # stage-wise product
+    "gemv_drops_base": ("w = (i == 0) ? lv : w + lv;", "w = (i == 0) ? 0.0f : w + lv;"),
+    "gemv_reversed_activation": ("(double)rrq_oracle_bf16_to_f32(A[(size_t)b * cols + j]);",
+                                 "(double)rrq_oracle_bf16_to_f32(A[(size_t)b * cols + (cols - 1 - j)]);"),
+    "gemv_wrong_output_row": ("Y[(size_t)b * rows + r] += (double)w", "Y[(size_t)b * rows + (rows - 1 - r)] += (double)w"),
+    "gemv_bf16_weight": ("Y[(size_t)b * rows + r] += (double)w *",
+                         "Y[(size_t)b * rows + r] += (double)rrq_oracle_bf16_to_f32(rrq_oracle_f32_to_bf16(w)) *"),
+    "gemv_one_stage_short": ("      for (int i = 0; i < k; ++i) {\n        const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;\n        const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])\n                                  : ((const float*)scales[i])[gi];\n        const float lv",
+                             "      for (int i = 0; i < k - (k > 1); ++i) {\n        const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;\n        const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])\n                                  : ((const float*)scales[i])[gi];\n        const float lv"),
 }
 
 
