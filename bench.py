@@ -137,6 +137,37 @@ def time_from_base(mats, pkgs, specs, stream, reps: int = 3) -> dict:
             "frac_of_measured_hbm": round(alg / t / 1e9 / measured_peaks()["hbm_gbs"], 4)}
 
 
+def time_gemv(pkgs, specs, stream, batch: int = 1, reps: int = 5) -> dict:
+    """Decode product over the whole stack (Appendix C): rrq_gemv of every
+    matrix's package at prefix k = 1..4 with one activation row, timed with
+    CUDA events.  Algorithmic bytes: the first k stages of the package
+    (k x (1/4 + 8/g) B per weight), the bf16 activations and the fp32 output."""
+    from paper_2608_04048_gb300 import binding
+    dev = pkgs[0].codes[0].device
+    gen = torch.Generator(device=dev).manual_seed(77)
+    acts = [torch.randn((batch, sp.cols), generator=gen, device=dev).to(torch.bfloat16) for sp in specs]
+    ys = [torch.empty((batch, sp.rows), dtype=torch.float32, device=dev) for sp in specs]
+    hbm = measured_peaks()["hbm_gbs"]
+    out = {"call": f"rrq_gemv over all {len(specs)} matrices, batch {batch} (asymmetric binary32 package)"}
+    for k in KS:
+        items = binding.gemv_descs(pkgs, acts, ys, k)
+        run = lambda: binding.rrq_gemv(pkgs, acts, k, ys, stream, items)
+        run()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            run()
+        b.record(stream)
+        torch.cuda.synchronize()
+        t = a.elapsed_time(b) / reps / 1e3
+        alg = sum(sp.numel * k * (0.25 + 8.0 / GROUP) + 2 * batch * sp.cols + 4 * batch * sp.rows
+                  for sp in specs)
+        out[f"k{k}"] = {"s_per_stack": round(t, 6), "alg_gbs": round(alg / t / 1e9, 1),
+                        "frac_of_measured_hbm": round(alg / t / 1e9 / hbm, 4),
+                        "weights_per_s": round(sum(sp.numel for sp in specs) / t, 1)}
+    return out
+
+
 def alg_bytes_reconstruct(n: int, k: int, g: int = GROUP) -> float:
     """Algorithmic bytes of one rrq_reconstruct at prefix k: k code planes and
     metadata read, bf16 written."""
@@ -332,6 +363,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
 
     sym = time_sym_f16(mats, p_outs, specs, stream) if not args.no_sym else None
     from_base = time_from_base(mats, pkgs, specs, stream) if not args.no_sym else None
+    gemv = time_gemv(pkgs, specs, stream) if not args.no_sym else None
     e2e = run_e2e(args, mats, pkgs, p_outs, specs, stream, world) if not args.no_e2e else None
     if rank != 0:
         return None
@@ -388,6 +420,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "paper_context_s": {"full_all_rtn_package_qwen3_8b_a100": 1293, "four_rtn_passes_a100": 412},
             "sym_f16": sym,
             "from_base": from_base,
+            "gemv_decode": gemv,
         },
         "roofline": roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic,
                                    clock_summary.get("sm_mhz")),
@@ -588,7 +621,7 @@ def main(argv=None):
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-sym", action="store_true",
-                    help="skip the symmetric binary16 and base-checkpoint breakdown")
+                    help="skip the symmetric binary16, base-checkpoint and product breakdown")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     args = ap.parse_args(argv)
 

@@ -258,6 +258,33 @@ typedef struct {
 rrq_status rrq_reconstruct_ex(const rrq_reconstruct_desc* items, int count, const rrq_format* fmt,
                               int k, int all_prefixes, rrq_stream_t stream);
 
+/* One matrix of rrq_gemv: its package (first k stages, format of the call),
+ * the activations and the output. */
+typedef struct {
+  const uint8_t* codes[RRQ_MAX_STAGES];
+  const void* scales[RRQ_MAX_STAGES];    /* float or binary16 */
+  const float* zeros[RRQ_MAX_STAGES];    /* RRQ_GRID_ASYM only */
+  int64_t rows, cols;                    /* the weight matrix [rows, cols] */
+  const uint16_t* A_bf16;                /* device, bf16 [batch, cols] row-major, 16-byte aligned */
+  float* Y;                              /* device, float [batch, rows] row-major, 16-byte aligned */
+} rrq_gemv_desc;
+
+#define RRQ_MAX_GEMV_BATCH 8
+
+/* Product of activations with the prefix-k weights, without materialising
+ * them (Appendix C: A W~_(t) = A W^_0 + sum_k A R^_k):
+ *     Y[b][r] = sum_c W~[r][c] * A[b][c],   b < batch, r < rows
+ * where W~[r][c] is the binary32 prefix sum of the first k stages (acc = L_0;
+ * acc = fl(acc + L_i), the value rrq_reconstruct rounds to bf16).  The kernel
+ * reads only the package (k x (2 + 64/g) bits per weight for RRQ_GRID_ASYM,
+ * k x (2 + 16/g) for the binary16 symmetric format) and sums each row in a
+ * fixed order in binary32 (deterministic; |Y - exact| <= gamma_cols *
+ * sum_c |W~ A|).  For decoding: 1 <= batch <= RRQ_MAX_GEMV_BATCH activation
+ * rows; 1 <= k <= fmt->n_stages.  Y must not overlap any input or another Y.
+ * One launch per 64 matrices; other rules as for rrq_reconstruct_ex. */
+rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
+                    rrq_stream_t stream);
+
 /* Bytes of one stage's scale array in format *fmt: groups * (4 or 2).
  * 0 for invalid arguments. */
 size_t rrq_scales_bytes(int64_t rows, int64_t cols, const rrq_format* fmt);

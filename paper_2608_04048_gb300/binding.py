@@ -22,7 +22,7 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
 #: symbols declared in include/rrq.h
 EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
            "rrq_reconstruct_prefixes", "rrq_reconstruct_prefixes_batch",
-           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_scales_bytes", "rrq_package_bytes_ex",
+           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_gemv", "rrq_scales_bytes", "rrq_package_bytes_ex",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
            "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
@@ -46,6 +46,16 @@ class QuantizeDesc(ctypes.Structure):
     _fields_ = [("W_bf16", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
                 ("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
                 ("zeros", ctypes.c_void_p * MAX_STAGES)]
+
+
+class GemvDesc(ctypes.Structure):
+    """rrq_gemv_desc of include/rrq.h"""
+    _fields_ = [("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
+                ("zeros", ctypes.c_void_p * MAX_STAGES), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("A_bf16", ctypes.c_void_p), ("Y", ctypes.c_void_p)]
+
+
+MAX_GEMV_BATCH = 8
 
 
 class ReconstructDesc(ctypes.Structure):
@@ -119,6 +129,8 @@ def load_library():
     lib.rrq_quantize_ex.restype = i32
     lib.rrq_quantize_from_base.argtypes = [ctypes.POINTER(QuantizeDesc), i32, fmt_p, vp]
     lib.rrq_quantize_from_base.restype = i32
+    lib.rrq_gemv.argtypes = [ctypes.POINTER(GemvDesc), i32, fmt_p, i32, i32, vp]
+    lib.rrq_gemv.restype = i32
     lib.rrq_reconstruct_ex.argtypes = [ctypes.POINTER(ReconstructDesc), i32, fmt_p, i32, i32, vp]
     lib.rrq_reconstruct_ex.restype = i32
     lib.rrq_scales_bytes.argtypes = [i64, i64, fmt_p]
@@ -381,6 +393,44 @@ def rrq_quantize_from_base(mats, pkgs, stream=None, items=None):
     if rc != 0:
         raise RRQError(rc, "rrq_quantize_from_base")
     return pkgs
+
+
+def gemv_descs(pkgs, acts, ys, k) -> ctypes.Array:
+    """Host array of rrq_gemv_desc: acts[i] bf16 [batch, cols], ys[i] float32
+    [batch, rows]."""
+    items = (GemvDesc * len(pkgs))()
+    for it, pkg, A, Y in zip(items, pkgs, acts, ys):
+        if A.dtype != torch.bfloat16 or A.dim() != 2 or not A.is_cuda or not A.is_contiguous():
+            raise TypeError("activations must be contiguous 2-D bfloat16 CUDA tensors")
+        if Y.dtype != torch.float32 or not Y.is_cuda or not Y.is_contiguous():
+            raise TypeError("outputs must be contiguous float32 CUDA tensors")
+        for j in range(k):
+            it.codes[j] = pkg.codes[j].data_ptr()
+            it.scales[j] = pkg.scales[j].data_ptr()
+            it.zeros[j] = pkg.zeros[j].data_ptr() if pkg.zeros else None
+        it.rows, it.cols = pkg.rows, pkg.cols
+        it.A_bf16, it.Y = A.data_ptr(), Y.data_ptr()
+    return items
+
+
+def rrq_gemv(pkgs, acts, k: int, ys=None, stream=None, items=None):
+    """Y_i = A_i W~_i^T for each package i at prefix k (Appendix C), A_i bf16
+    [batch, cols] with 1 <= batch <= 8; returns float32 [batch, rows] each."""
+    lib = load_library()
+    batch = acts[0].shape[0]
+    if any(not 1 <= k <= p.n_stages for p in pkgs):
+        raise ValueError("k exceeds the stages of a package")
+    if any(A.shape[0] != batch for A in acts):
+        raise ValueError("every activation matrix must have the same batch")
+    if ys is None:
+        ys = [torch.empty((batch, p.rows), dtype=torch.float32, device=p.codes[0].device) for p in pkgs]
+    if items is None:
+        items = gemv_descs(pkgs, acts, ys, k)
+    fmt = pkgs[0].format()
+    rc = lib.rrq_gemv(items, len(items), ctypes.byref(fmt), k, batch, _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_gemv")
+    return ys
 
 
 def reconstruct_descs(pkgs, outs, k) -> ctypes.Array:

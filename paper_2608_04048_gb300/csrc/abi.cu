@@ -53,6 +53,7 @@ rrq_status current_device(int* dev_out, DeviceState** state) {
     d.status = static_cast<unsigned*>(addr);
     if ((e = rrq::quantize_prepare())) return fail_cuda(e);
     if ((e = rrq::quantize_prepare_base())) return fail_cuda(e);
+    if ((e = rrq::gemv_prepare())) return fail_cuda(e);
     if ((e = rrq::reconstruct_prepare())) return fail_cuda(e);
     d.ready = true;
   }
@@ -328,6 +329,81 @@ rrq_status reconstruct_views(const ReconView* items, int count, const Fmt& f, in
   return RRQ_OK;
 }
 
+// ---------------------------------------------------------------------------
+// stage-wise product
+// ---------------------------------------------------------------------------
+rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k, int batch,
+                      rrq_stream_t stream) {
+  if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
+  if (batch < 1 || batch > rrq::kMaxGemvBatch) return RRQ_ERR_INVALID_ARG;
+  const int group = f.group;
+  std::vector<Range> ranges;
+  ranges.reserve(static_cast<size_t>(count) * (2 + 3 * k));
+  for (int i = 0; i < count; ++i) {
+    const rrq_gemv_desc& it = items[i];
+    if (!shape_ok(it.rows, it.cols) || it.cols % group != 0 || !it.A_bf16 || !it.Y) return RRQ_ERR_INVALID_ARG;
+    for (int j = 0; j < k; ++j)
+      if (!it.codes[j] || !it.scales[j] || (!f.sym() && !it.zeros[j])) return RRQ_ERR_INVALID_ARG;
+    if (!aligned(it.A_bf16, 16) || !aligned(it.Y, 16)) return RRQ_ERR_MISALIGNED;
+    for (int j = 0; j < k; ++j)
+      if (!aligned(it.codes[j], 16) || !aligned(it.scales[j], 16) || (!f.sym() && !aligned(it.zeros[j], 16)))
+        return RRQ_ERR_MISALIGNED;
+    const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
+    ranges.push_back(range_of(it.A_bf16, 2 * static_cast<uint64_t>(batch) * it.cols, false));
+    ranges.push_back(range_of(it.Y, 4 * static_cast<uint64_t>(batch) * it.rows, true));
+    for (int j = 0; j < k; ++j) {
+      ranges.push_back(range_of(it.codes[j], n / 4, false));
+      ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
+      if (!f.sym()) ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
+    }
+  }
+  if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
+
+  int dev = 0;
+  DeviceState* st = nullptr;
+  if (rrq_status rc = current_device(&dev, &st)) return rc;
+  for (int i = 0; i < count; ++i) {
+    const rrq_gemv_desc& it = items[i];
+    if (!on_device(it.A_bf16, dev) || !on_device(it.Y, dev)) return RRQ_ERR_INVALID_ARG;
+    for (int j = 0; j < k; ++j)
+      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) ||
+          (!f.sym() && !on_device(it.zeros[j], dev)))
+        return RRQ_ERR_INVALID_ARG;
+  }
+
+  int log2g = 0;
+  while ((1 << log2g) < group) ++log2g;
+  static thread_local rrq::GemvBatch p;
+  for (int base = 0; base < count; base += rrq::kMaxBatch) {
+    const int m = std::min(rrq::kMaxBatch, count - base);
+    std::memset(&p, 0, sizeof p);
+    p.count = m;
+    p.k = k;
+    p.log2g = log2g;
+    int64_t rows = 0;
+    for (int i = 0; i < m; ++i) {
+      const rrq_gemv_desc& it = items[base + i];
+      rrq::GemvItem& q = p.item[i];
+      for (int j = 0; j < rrq::kMaxStages; ++j) {
+        const int jj = j < k ? j : k - 1;
+        q.codes[j] = it.codes[jj];
+        q.scales[j] = it.scales[jj];
+        q.zeros[j] = f.sym() ? nullptr : it.zeros[jj];
+      }
+      q.A = it.A_bf16;
+      q.Y = it.Y;
+      q.rows = it.rows;
+      q.cols = it.cols;
+      q.row_begin = rows;
+      rows += it.rows;
+    }
+    p.total_rows = rows;
+    cudaError_t e = rrq::gemv_launch(f.kind, batch, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+    if (e != cudaSuccess) return fail_cuda(e);
+  }
+  return RRQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -449,6 +525,13 @@ rrq_status rrq_quantize_from_base(const rrq_quantize_desc* items, int count, con
   Fmt f;
   if (rrq_status rc = parse_format(fmt, &f)) return rc;
   return quantize_batch(items, count, f, stream, true);
+}
+
+rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
+                    rrq_stream_t stream) {
+  Fmt f;
+  if (rrq_status rc = parse_format(fmt, &f)) return rc;
+  return gemv_batch(items, count, f, k, batch, stream);
 }
 
 rrq_status rrq_reconstruct_ex(const rrq_reconstruct_desc* items, int count, const rrq_format* fmt,

@@ -63,6 +63,29 @@ struct ReconstructBatch {
   ReconstructItem item[kMaxBatch];
 };
 
+// One matrix of a stage-wise product launch: Y = A * W~^T with W~ the prefix
+// weights of the package's first k stages.  Rows of all matrices of a launch
+// are numbered consecutively; row_begin is this matrix's first.
+struct GemvItem {
+  const uint8_t* codes[kMaxStages];
+  const void* scales[kMaxStages];  // float or binary16
+  const float* zeros[kMaxStages];  // asymmetric grid only
+  const uint16_t* A;               // bf16 [batch, cols]
+  float* Y;                        // [batch, rows]
+  int64_t rows, cols;
+  int64_t row_begin;
+};
+
+struct GemvBatch {
+  int count;
+  int k;                           // stages summed, 1..4
+  int log2g;                       // group = 1 << log2g
+  int64_t total_rows;
+  GemvItem item[kMaxBatch];
+};
+
+constexpr int kMaxGemvBatch = 8;   // activation rows (tokens) per call
+
 // One-time per-device set-up of kernel attributes (dynamic shared memory).
 cudaError_t quantize_prepare();
 cudaError_t quantize_prepare_base();
@@ -84,6 +107,10 @@ cudaError_t reconstruct_launch_sym_f32(int group, int k, bool all_prefixes, cons
                                        cudaStream_t stream, int sms);
 cudaError_t reconstruct_launch_sym_f16(int group, int k, bool all_prefixes, const ReconstructBatch& p,
                                        cudaStream_t stream, int sms);
+
+cudaError_t gemv_prepare();
+// batch = activation rows, 1..kMaxGemvBatch
+cudaError_t gemv_launch(Format fmt, int batch, const GemvBatch& p, cudaStream_t stream, int sms);
 
 inline cudaError_t reconstruct_prepare() {
   cudaError_t e;

@@ -1,0 +1,159 @@
+"""GPU parity for the stage-wise product with the prefix weights (rrq_gemv,
+Appendix C): Y = A W~^T from the package alone, against the oracle's binary64
+product of the same binary32 prefix weights.
+
+Tolerance, from the kernel's arithmetic: every product W~ a is exact inside
+its fma and every partial sum is rounded once; a lane sums its 32 columns of
+each 1024-column chunk into two accumulators (16 columns each, chunks in
+turn), then adds the two and the warp adds 32 lanes in 5 butterfly steps, so
+no term passes through more than d = cols/64 + 8 roundings and
+|Y - exact| <= d * 2^-24 * sum_c |W~ a| (first order).  sum_c |W~ a| is
+bounded with the bf16 reconstruction: |W~| <= |bf16(W~)| (1 + 2^-8)."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_04048_gb300 import binding, build, workloads
+from gpu_helpers import bf16_bits
+
+pytestmark = pytest.mark.gpu
+
+GROUPS = (32, 64, 128, 256)
+FORMATS = [(binding.GRID_ASYM, binding.SCALE_F32), (binding.GRID_SYM, binding.SCALE_F32),
+           (binding.GRID_SYM, binding.SCALE_F16)]
+FMT_IDS = ["asym_f32", "sym_f32", "sym_f16"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    build.build()
+    binding.load_library()
+    binding.rrq_set_debug_flags(0)
+
+
+def _host_pkg(pkg, rows_idx=None):
+    """Package arrays on the host, optionally only the given rows."""
+    torch.cuda.synchronize()
+    g, cols = pkg.group, pkg.cols
+    f16 = pkg.scale_type == binding.SCALE_F16
+
+    def take(t, per_row):
+        a = t.view(torch.int16).cpu().numpy().view(np.uint16) if (f16 and t.dtype == torch.float16) \
+            else t.cpu().numpy()
+        if rows_idx is None:
+            return a
+        return a.reshape(-1, per_row)[rows_idx].reshape(-1)
+    codes = [take(c, cols // 4) for c in pkg.codes]
+    scales = [take(s, cols // g) for s in pkg.scales]
+    zeros = [take(z, cols // g) for z in pkg.zeros] if pkg.zeros else None
+    return codes, scales, zeros
+
+
+def _check(pkg, A, Y, k, rows_idx=None, where=""):
+    """Y (GPU, float32 [batch, rows]) against the oracle on the given rows."""
+    sym, f16 = pkg.grid == binding.GRID_SYM, pkg.scale_type == binding.SCALE_F16
+    codes, scales, zeros = _host_pkg(pkg, rows_idx)
+    nr = pkg.rows if rows_idx is None else len(rows_idx)
+    Ab = bf16_bits(A)
+    want = oracle.gemv(codes, scales, zeros, nr, pkg.cols, pkg.group, k, Ab, sym, f16)
+    if sym:
+        rec = oracle.reconstruct_sym(codes, scales, nr, pkg.cols, pkg.group, k, f16)
+    else:
+        rec = oracle.reconstruct(codes, scales, zeros, nr, pkg.cols, pkg.group, k)
+    recf = np.abs((rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+    Af = np.abs((Ab.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+    d = pkg.cols // 64 + 8
+    tol = d * 2.0 ** -24 * (Af @ recf.T) * (1 + 2.0 ** -8) + 1e-30
+    got = Y.cpu().numpy().astype(np.float64)
+    if rows_idx is not None:
+        got = got[:, rows_idx]
+    err = np.abs(got - want)
+    bad = np.argwhere(err > tol)
+    assert bad.size == 0, (f"{where}: {len(bad)} outputs beyond the bound, first {tuple(bad[0])}: "
+                           f"gpu {got[tuple(bad[0])]!r} oracle {want[tuple(bad[0])]!r} tol {tol[tuple(bad[0])]!r}")
+
+
+def _acts(batch, cols, seed, dev="cuda"):
+    g = torch.Generator(device=dev).manual_seed(seed)
+    return torch.randn((batch, cols), generator=g, device=dev, dtype=torch.float32).to(torch.bfloat16)
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FMT_IDS)
+@pytest.mark.parametrize("group", GROUPS)
+@pytest.mark.parametrize("batch", [1, 3, 8])
+def test_formats_groups_batches(batch, group, fmt):
+    rows, cols = 45, 9 * group  # cols not a multiple of 1024 for g <= 64: ragged chunks
+    W = workloads.generate(rows, cols, 70 + group, "t3_rowout", "cuda")
+    (pkg,) = binding.rrq_quantize_ex([W], group, 4, *fmt)
+    A = _acts(batch, cols, seed=batch * 100 + group)
+    for k in (1, 2, 3, 4):
+        (Y,) = binding.rrq_gemv([pkg], [A], k)
+        _check(pkg, A, Y, k, where=f"{fmt} g{group} B{batch} k{k}")
+
+
+@pytest.mark.parametrize("shape", [(1, 32), (3, 96), (7, 2304), (33, 1024 + 32), (5, 12288), (2049, 128)])
+def test_shapes(shape):
+    rows, cols = shape
+    g = 32 if cols % 64 else 128 if cols % 128 == 0 else 64
+    W = workloads.generate(rows, cols, rows + cols, "t3", "cuda")
+    (pkg,) = binding.rrq_quantize_ex([W], g, 4, binding.GRID_ASYM, binding.SCALE_F32)
+    A = _acts(2, cols, seed=rows)
+    for k in (1, 4):
+        (Y,) = binding.rrq_gemv([pkg], [A], k)
+        _check(pkg, A, Y, k, where=f"{shape} k{k}")
+
+
+def test_deterministic_and_matches_asym_original_package():
+    """Two calls give identical bits; a package built by rrq_quantize (the
+    asymmetric original call) is read the same way."""
+    W = workloads.generate(300, 4096, 3, "t3_rowout", "cuda")
+    pkg = binding.rrq_quantize(W, 128, 4)
+    A = _acts(4, 4096, seed=5)
+    Y1 = binding.rrq_gemv([pkg], [A], 4)[0]
+    Y2 = binding.rrq_gemv([pkg], [A], 4)[0]
+    torch.cuda.synchronize()
+    assert torch.equal(Y1.view(torch.int32), Y2.view(torch.int32))
+    _check(pkg, A, Y1, 4, where="asym original")
+
+
+def test_batch_across_launches():
+    rng = np.random.default_rng(12)
+    shapes = [(int(rng.integers(1, 40)), 128 * int(rng.integers(1, 20))) for _ in range(70)]
+    mats = [workloads.generate(r, c, 1200 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+    pkgs = binding.rrq_quantize_ex(mats, 128, 4, binding.GRID_SYM, binding.SCALE_F16)
+    acts = [_acts(2, c, seed=i) for i, (r, c) in enumerate(shapes)]
+    ys = binding.rrq_gemv(pkgs, acts, 3)
+    for i, (p, A, Y) in enumerate(zip(pkgs, acts, ys)):
+        _check(p, A, Y, 3, where=f"item {i}")
+
+
+def test_qwen3_8b_layer_sampled_rows():
+    """A full-size Qwen3-8B-shaped layer (7 matrices, one call) at batch 1,
+    every prefix; 64 sampled rows of every matrix against the oracle."""
+    specs = workloads.config_matrices("qwen3_8b_layer")
+    mats = [workloads.generate_spec(sp, "cuda") for sp in specs]
+    pkgs = binding.rrq_quantize_batch(mats, group=128, n_stages=4)
+    acts = [_acts(1, sp.cols, seed=50 + i) for i, sp in enumerate(specs)]
+    for k in (1, 2, 3, 4):
+        ys = binding.rrq_gemv(pkgs, acts, k)
+        for i, (sp, p, A, Y) in enumerate(zip(specs, pkgs, acts, ys)):
+            rng = np.random.default_rng(i * 10 + k)
+            idx = np.unique(np.concatenate([[0, sp.rows - 1], rng.integers(0, sp.rows, 62)]))
+            _check(p, A, Y, k, rows_idx=idx, where=f"{sp.name} k{k}")
+
+
+def test_errors():
+    W = workloads.generate(8, 256, 1, "normal", "cuda")
+    pkg = binding.rrq_quantize(W, 128, 2)
+    A = _acts(9, 256, seed=1)
+    with pytest.raises(binding.RRQError) as e:
+        binding.rrq_gemv([pkg], [A], 1)
+    assert e.value.status == 1
+    with pytest.raises(ValueError):
+        binding.rrq_gemv([pkg], [A[:2]], 3)
+    A2 = _acts(2, 256, seed=2)
+    Yover = A2.view(torch.float32).reshape(-1)[:16].view(2, 8)  # Y over the activations
+    with pytest.raises(binding.RRQError) as e:
+        binding.rrq_gemv([pkg], [A2], 1, ys=[Yover])
+    assert e.value.status == 1
