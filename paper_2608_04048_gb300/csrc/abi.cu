@@ -53,7 +53,6 @@ rrq_status current_device(int* dev_out, DeviceState** state) {
     d.status = static_cast<unsigned*>(addr);
     if ((e = rrq::quantize_prepare())) return fail_cuda(e);
     if ((e = rrq::quantize_prepare_base())) return fail_cuda(e);
-    if ((e = rrq::gemv_prepare())) return fail_cuda(e);
     if ((e = rrq::reconstruct_prepare())) return fail_cuda(e);
     d.ready = true;
   }
@@ -378,9 +377,8 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
     const int m = std::min(rrq::kMaxBatch, count - base);
     std::memset(&p, 0, sizeof p);
     p.count = m;
-    p.k = k;
     p.log2g = log2g;
-    int64_t rows = 0;
+    int64_t blocks = 0, max_cols = 0;
     for (int i = 0; i < m; ++i) {
       const rrq_gemv_desc& it = items[base + i];
       rrq::GemvItem& q = p.item[i];
@@ -390,16 +388,47 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
         q.scales[j] = it.scales[jj];
         q.zeros[j] = f.sym() ? nullptr : it.zeros[jj];
       }
-      q.A = it.A_bf16;
-      q.Y = it.Y;
       q.rows = it.rows;
       q.cols = it.cols;
-      q.row_begin = rows;
-      rows += it.rows;
+      q.blk_begin = blocks;
+      blocks += (it.rows + rrq::kGemvRows - 1) / rrq::kGemvRows;
+      max_cols = std::max(max_cols, it.cols);
     }
-    p.total_rows = rows;
-    cudaError_t e = rrq::gemv_launch(f.kind, batch, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
-    if (e != cudaSuccess) return fail_cuda(e);
+    p.total_blocks = blocks;
+    // one contiguous range of blocks per CTA, with equal shares of rows x cols
+    p.grid = static_cast<int>(std::min<int64_t>({blocks, st->sms, rrq::kMaxGemvGrid}));
+    {
+      int64_t total = 0;
+      for (int i = 0; i < m; ++i) total += items[base + i].rows * items[base + i].cols;
+      int c = 0;
+      int64_t done = 0, blk = 0;
+      p.cta_begin[0] = 0;
+      for (int i = 0; i < m && c < p.grid; ++i) {
+        const rrq_gemv_desc& it = items[base + i];
+        const int64_t nblk = (it.rows + rrq::kGemvRows - 1) / rrq::kGemvRows;
+        for (int64_t b = 0; b < nblk; ++b, ++blk) {
+          const int64_t r = std::min<int64_t>(rrq::kGemvRows, it.rows - b * rrq::kGemvRows);
+          done += r * it.cols;
+          // close CTA c's range once its share is reached
+          while (c + 1 < p.grid && done * p.grid >= (c + 1) * total) p.cta_begin[++c] = blk + 1;
+        }
+      }
+      while (c < p.grid) p.cta_begin[++c] = blocks;
+      p.cta_begin[p.grid] = blocks;
+    }
+    // activation rows per launch: as many as shared memory holds
+    const int per = rrq::gemv_rows_per_launch(k, max_cols);
+    if (per < 1) return RRQ_ERR_UNSUPPORTED;
+    for (int b0 = 0; b0 < batch; b0 += per) {
+      const int nb = std::min(per, batch - b0);
+      for (int i = 0; i < m; ++i) {
+        const rrq_gemv_desc& it = items[base + i];
+        p.item[i].A = it.A_bf16 + static_cast<int64_t>(b0) * it.cols;
+        p.item[i].Y = it.Y + static_cast<int64_t>(b0) * it.rows;
+      }
+      cudaError_t e = rrq::gemv_launch(f.kind, k, nb, max_cols, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+      if (e != cudaSuccess) return fail_cuda(e);
+    }
   }
   return RRQ_OK;
 }

@@ -64,25 +64,31 @@ struct ReconstructBatch {
 };
 
 // One matrix of a stage-wise product launch: Y = A * W~^T with W~ the prefix
-// weights of the package's first k stages.  Rows of all matrices of a launch
-// are numbered consecutively; row_begin is this matrix's first.
+// weights of the package's first k stages.  Each matrix's rows are cut into
+// blocks of 16; the blocks of all matrices of a launch are numbered
+// consecutively and blk_begin is this matrix's first.
 struct GemvItem {
   const uint8_t* codes[kMaxStages];
   const void* scales[kMaxStages];  // float or binary16
   const float* zeros[kMaxStages];  // asymmetric grid only
-  const uint16_t* A;               // bf16 [batch, cols]
-  float* Y;                        // [batch, rows]
+  const uint16_t* A;               // bf16 [activation rows, cols] (this launch's first row)
+  float* Y;                        // [activation rows, rows] (this launch's first row)
   int64_t rows, cols;
-  int64_t row_begin;
+  int64_t blk_begin;
 };
+
+constexpr int kMaxGemvGrid = 256;  // CTAs of one launch (at most one per multiprocessor)
 
 struct GemvBatch {
   int count;
-  int k;                           // stages summed, 1..4
   int log2g;                       // group = 1 << log2g
-  int64_t total_rows;
+  int grid;                        // CTAs of the launch
+  int64_t total_blocks;
+  int64_t cta_begin[kMaxGemvGrid + 1];  // CTA c takes blocks [cta_begin[c], cta_begin[c+1])
   GemvItem item[kMaxBatch];
 };
+
+constexpr int kGemvRows = 16;      // rows per block
 
 constexpr int kMaxGemvBatch = 8;   // activation rows (tokens) per call
 
@@ -108,9 +114,24 @@ cudaError_t reconstruct_launch_sym_f32(int group, int k, bool all_prefixes, cons
 cudaError_t reconstruct_launch_sym_f16(int group, int k, bool all_prefixes, const ReconstructBatch& p,
                                        cudaStream_t stream, int sms);
 
-cudaError_t gemv_prepare();
-// batch = activation rows, 1..kMaxGemvBatch
-cudaError_t gemv_launch(Format fmt, int batch, const GemvBatch& p, cudaStream_t stream, int sms);
+// Activation rows one launch can hold in shared memory for matrices of up to
+// max_cols columns with k stages (0: too wide).
+int gemv_rows_per_launch(int k, int64_t max_cols);
+// nb activation rows (1..kMaxGemvBatch, within gemv_rows_per_launch); one
+// translation unit per format.
+cudaError_t gemv_launch_asym_f32(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
+cudaError_t gemv_launch_sym_f32(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
+cudaError_t gemv_launch_sym_f16(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
+
+inline cudaError_t gemv_launch(Format fmt, int k, int nb, int64_t max_cols, const GemvBatch& p,
+                               cudaStream_t stream, int sms) {
+  switch (fmt) {
+    case kAsymF32: return gemv_launch_asym_f32(k, nb, max_cols, p, stream, sms);
+    case kSymF32: return gemv_launch_sym_f32(k, nb, max_cols, p, stream, sms);
+    case kSymF16: return gemv_launch_sym_f16(k, nb, max_cols, p, stream, sms);
+  }
+  return cudaErrorInvalidValue;
+}
 
 inline cudaError_t reconstruct_prepare() {
   cudaError_t e;
