@@ -471,17 +471,30 @@ def recorded_traffic(kernel: str, q_bytes_per_launch: float, r_bytes_per_launch:
     with open(path) as f:
         rec = json.load(f)
     entry = rec.get(kernel)
-    if not entry or entry.get("source_sha256") != kernel_source_hash():
+    if not entry or kernel not in KERNEL_SOURCES or entry.get("source_sha256") != kernel_source_hash(kernel):
         return None
     per_alg = entry["dram_bytes"] / entry["alg_bytes"]
     alg = q_bytes_per_launch if kernel == "rrq_quantize" else r_bytes_per_launch
     return round(per_alg * alg)
 
 
-def kernel_source_hash() -> str:
+# the source files each recorded kernel is compiled from
+KERNEL_SOURCES = {
+    "rrq_quantize": ["quantize_kernel.cuh", "quantize.cu"],
+    "rrq_quantize_ex_sym_f16": ["quantize_kernel.cuh", "quantize.cu"],
+    "rrq_reconstruct_prefixes": ["reconstruct_kernel.cuh", "reconstruct_asym_f32.cu"],
+    "rrq_reconstruct_ex_sym_f16": ["reconstruct_kernel.cuh", "reconstruct_sym_f16.cu"],
+    "rrq_gemv_k1": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
+    "rrq_gemv_k4": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
+}
+
+
+def kernel_source_hash(kernel: str) -> str:
+    """SHA-256 over the sources of one kernel (its own files plus the shared
+    device helpers and the host/device interface header)."""
     h = hashlib.sha256()
     csrc = os.path.join(ROOT, "paper_2608_04048_gb300", "csrc")
-    for name in sorted(os.listdir(csrc)):
+    for name in KERNEL_SOURCES[kernel] + ["rrq_device.cuh", "rrq_internal.h"]:
         with open(os.path.join(csrc, name), "rb") as f:
             h.update(name.encode())
             h.update(f.read())
