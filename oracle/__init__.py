@@ -101,6 +101,21 @@ class Oracle:
             ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
             _u16p, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
         lib.rrq_oracle_gemv.restype = ctypes.c_int
+        _i32p = ctypes.POINTER(ctypes.c_int)
+        lib.rrq_oracle_quantize_group_bits.argtypes = [
+            _f32p, ctypes.c_int, ctypes.c_int, _i32p, _u8p, _f32p, _f32p, _f32p]
+        lib.rrq_oracle_quantize_group_bits.restype = ctypes.c_int
+        lib.rrq_oracle_quantize_bits.argtypes = [
+            _u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _i32p,
+            ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p)]
+        lib.rrq_oracle_quantize_bits.restype = ctypes.c_int
+        lib.rrq_oracle_reconstruct_bits.argtypes = [
+            ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p),
+            ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _i32p, _u16p]
+        lib.rrq_oracle_reconstruct_bits.restype = ctypes.c_int
+        lib.rrq_oracle_group_pmr.argtypes = [_u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
+                                             ctypes.POINTER(ctypes.c_double)]
+        lib.rrq_oracle_group_pmr.restype = ctypes.c_int
         lib.rrq_oracle_f32_to_f16.argtypes = [ctypes.c_float]
         lib.rrq_oracle_f32_to_f16.restype = ctypes.c_uint16
         lib.rrq_oracle_f16_to_f32.argtypes = [ctypes.c_uint16]
@@ -252,6 +267,64 @@ class Oracle:
             raise ValueError("oracle rejected the product")
         return Y
 
+    # -- heterogeneous stage widths (asymmetric grid) ----------------------------
+    def quantize_group_bits(self, x, bits):
+        """(Q, scale, zero, resid) for one group with per-stage widths."""
+        x = np.ascontiguousarray(np.asarray(x, dtype=np.float32))
+        g, S = x.size, len(bits)
+        b = (ctypes.c_int * S)(*bits)
+        Q = np.zeros((S, g), np.uint8)
+        s = np.zeros(S, np.float32)
+        z = np.zeros(S, np.float32)
+        r = np.zeros((S, g), np.float32)
+        rc = self.lib.rrq_oracle_quantize_group_bits(
+            x.ctypes.data_as(_f32p), g, S, b, Q.ctypes.data_as(_u8p), s.ctypes.data_as(_f32p),
+            z.ctypes.data_as(_f32p), r.ctypes.data_as(_f32p))
+        if rc != 0:
+            raise ValueError("oracle rejected the group")
+        return Q, s, z, r
+
+    def quantize_bits(self, W_bits, group, bits):
+        """(codes, scales, zeros) with stage k's codes packed at bits[k] bits."""
+        W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+        rows, cols = W_bits.shape
+        n, S = rows * cols, len(bits)
+        codes = [np.zeros((n * b + 7) // 8, np.uint8) for b in bits]
+        scales = [np.zeros(n // group, np.float32) for _ in bits]
+        zeros = [np.zeros(n // group, np.float32) for _ in bits]
+        cp = (_u8p * S)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (_f32p * S)(*[a.ctypes.data_as(_f32p) for a in scales])
+        zp = (_f32p * S)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        rc = self.lib.rrq_oracle_quantize_bits(W_bits.ctypes.data_as(_u16p), rows, cols, group, S,
+                                               (ctypes.c_int * S)(*bits), cp, sp, zp)
+        if rc != 0:
+            raise ValueError("oracle rejected the matrix")
+        return codes, scales, zeros
+
+    def reconstruct_bits(self, codes, scales, zeros, rows, cols, group, k, bits):
+        codes = [np.ascontiguousarray(c, dtype=np.uint8) for c in codes[:k]]
+        scales = [np.ascontiguousarray(a, dtype=np.float32) for a in scales[:k]]
+        zeros = [np.ascontiguousarray(a, dtype=np.float32) for a in zeros[:k]]
+        out = np.zeros((rows, cols), np.uint16)
+        cp = (_u8p * k)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in scales])
+        zp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        rc = self.lib.rrq_oracle_reconstruct_bits(cp, sp, zp, rows, cols, group, k,
+                                                  (ctypes.c_int * k)(*bits[:k]), out.ctypes.data_as(_u16p))
+        if rc != 0:
+            raise ValueError("oracle rejected the reconstruction")
+        return out
+
+    def group_pmr(self, W_bits, group):
+        W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+        rows, cols = W_bits.shape
+        out = np.zeros(rows * cols // group, np.float64)
+        rc = self.lib.rrq_oracle_group_pmr(W_bits.ctypes.data_as(_u16p), rows, cols, group,
+                                           out.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
+        if rc != 0:
+            raise ValueError("oracle rejected the matrix")
+        return out
+
     def reconstruct_sym(self, codes, scales, rows: int, cols: int, group: int, k: int,
                         scale_f16: bool = True):
         """bf16 bit patterns [rows, cols] of the prefix-k reconstruction of a
@@ -302,6 +375,18 @@ def reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16: bool = True)
 
 def gemv(codes, scales, zeros, rows, cols, group, k, A_bits, sym: bool = False, scale_f16: bool = False):
     return load().gemv(codes, scales, zeros, rows, cols, group, k, A_bits, sym, scale_f16)
+
+
+def quantize_bits(W_bits, group, bits):
+    return load().quantize_bits(W_bits, group, bits)
+
+
+def reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits):
+    return load().reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits)
+
+
+def group_pmr(W_bits, group):
+    return load().group_pmr(W_bits, group)
 
 
 def quantize_from_base(W_bits, base, group: int = 128, n_stages: int = 4, sym: bool = False,

@@ -56,6 +56,16 @@
  * products and the sum taken in binary64 (each product of a binary32 and a
  * bf16 value is exact there).
  *
+ * Heterogeneous stage widths (Section 3.2: stage k may use b_k bits, B_t is
+ * the sum of the widths; the split analysis of Section 3.3 / Table 3 uses
+ * zero-point grids): stage k of the asymmetric grid with b bits has
+ * m = 2^b - 1 steps, s = fl(fl(hi - lo) / m), Q = clamp(rhe(fl(fl(v - lo)/s)),
+ * 0, m), level fl(lo + fl(Q s)); codes are packed LSB-first, element c of the
+ * stage at bits b*c .. b*c + b - 1 of the stage's byte array.
+ *
+ * Group peak-to-mean ratio (Section 3.1 and Table 9's K/MAE): for a group,
+ * max |x| / (sum |x| / g), taken in binary64; 0 for an all-zero group.
+ *
  * Algorithm 1 with a base checkpoint: stage 0 of the package is given (codes,
  * scales and, for the asymmetric grid, zeros, in the package's own format);
  * it is dequantized with the same level formula as a computed stage 0, the
@@ -420,6 +430,132 @@ int rrq_oracle_gemv(const uint8_t* const* codes, const void* const* scales,
       for (int b = 0; b < batch; ++b)
         Y[(size_t)b * rows + r] += (double)w * (double)rrq_oracle_bf16_to_f32(A[(size_t)b * cols + j]);
     }
+  }
+  return 0;
+}
+
+/* Asymmetric 2^b-level stages with per-stage widths; see the file comment. */
+int rrq_oracle_quantize_group_bits(const float* x, int g, int n_stages, const int* bits,
+                                   uint8_t* Q, float* scale, float* zero, float* resid) {
+  if (g < 1 || n_stages < 1 || !x || !bits || !Q || !scale || !zero) return -1;
+  for (int k = 0; k < n_stages; ++k)
+    if (bits[k] < 1 || bits[k] > 4) return -1;
+  float* v = (float*)malloc(sizeof(float) * (size_t)g);
+  if (!v) return -1;
+  for (int j = 0; j < g; ++j) v[j] = x[j];
+
+  for (int k = 0; k < n_stages; ++k) {
+    const int m = (1 << bits[k]) - 1; /* steps of a b-bit grid */
+    float lo = v[0], hi = v[0]; /* range of this stage's values, -0 before +0 */
+    for (int j = 1; j < g; ++j) {
+      lo = before(v[j], lo) ? v[j] : lo;
+      hi = before(hi, v[j]) ? v[j] : hi;
+    }
+    const float span = hi - lo;
+    float s = span / (float)m;
+    for (int j = 0; j < g; ++j) {
+      int code = 0;
+      if (s != 0.0f) {
+        const float dist = v[j] - lo;
+        const float u = dist / s;
+        code = (int)round_half_even(u);
+        code = code < 0 ? 0 : (code > m ? m : code);
+      }
+      Q[(size_t)k * g + j] = (uint8_t)code;
+      float qs = (float)code * s;
+      float lv = lo + qs;
+      v[j] = v[j] - lv;
+    }
+    scale[k] = s;
+    zero[k] = lo;
+    if (resid)
+      for (int j = 0; j < g; ++j) resid[(size_t)k * g + j] = v[j];
+  }
+  free(v);
+  return 0;
+}
+
+/* element c's b-bit code at bits b*c.. of the stage's byte array (LSB first) */
+static void put_bits(uint8_t* codes, int64_t c, int b, int q) {
+  for (int t = 0; t < b; ++t) {
+    const int64_t bit = c * b + t;
+    if ((q >> t) & 1) codes[bit / 8] |= (uint8_t)(1u << (bit % 8));
+  }
+}
+static int get_bits(const uint8_t* codes, int64_t c, int b) {
+  int q = 0;
+  for (int t = 0; t < b; ++t) {
+    const int64_t bit = c * b + t;
+    q |= ((codes[bit / 8] >> (bit % 8)) & 1) << t;
+  }
+  return q;
+}
+
+int rrq_oracle_quantize_bits(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                             int n_stages, const int* bits, uint8_t* const* codes,
+                             float* const* scales, float* const* zeros) {
+  if (!W || !bits || !codes || !scales || !zeros) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || n_stages < 1 || cols % group != 0) return -1;
+  const int64_t n = rows * cols;
+  const int64_t n_groups = n / group;
+  float* x = (float*)malloc(sizeof(float) * (size_t)group);
+  uint8_t* Q = (uint8_t*)malloc((size_t)n_stages * (size_t)group);
+  float* s = (float*)malloc(sizeof(float) * (size_t)n_stages);
+  float* z = (float*)malloc(sizeof(float) * (size_t)n_stages);
+  if (!x || !Q || !s || !z) {
+    free(x); free(Q); free(s); free(z);
+    return -1;
+  }
+  for (int k = 0; k < n_stages; ++k) memset(codes[k], 0, (size_t)((n * bits[k] + 7) / 8));
+  for (int64_t gi = 0; gi < n_groups; ++gi) {
+    const int64_t base = gi * group;
+    for (int j = 0; j < group; ++j) x[j] = rrq_oracle_bf16_to_f32(W[base + j]);
+    if (rrq_oracle_quantize_group_bits(x, group, n_stages, bits, Q, s, z, NULL) != 0) {
+      free(x); free(Q); free(s); free(z);
+      return -1;
+    }
+    for (int k = 0; k < n_stages; ++k) {
+      for (int j = 0; j < group; ++j) put_bits(codes[k], base + j, bits[k], Q[(size_t)k * group + j]);
+      scales[k][gi] = s[k];
+      zeros[k][gi] = z[k];
+    }
+  }
+  free(x); free(Q); free(s); free(z);
+  return 0;
+}
+
+int rrq_oracle_reconstruct_bits(const uint8_t* const* codes, const float* const* scales,
+                                const float* const* zeros, int64_t rows, int64_t cols, int group,
+                                int k, const int* bits, uint16_t* out) {
+  if (!codes || !scales || !zeros || !bits || !out) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || k < 1 || cols % group != 0) return -1;
+  const int64_t n = rows * cols;
+  for (int64_t c = 0; c < n; ++c) {
+    const int64_t gi = c / group;
+    float acc = 0.0f;
+    for (int i = 0; i < k; ++i) {
+      const int q = get_bits(codes[i], c, bits[i]);
+      float qs = (float)q * scales[i][gi];
+      float lv = zeros[i][gi] + qs;
+      if (i == 0) acc = lv;
+      else acc = acc + lv;
+    }
+    out[c] = rrq_oracle_f32_to_bf16(acc);
+  }
+  return 0;
+}
+
+int rrq_oracle_group_pmr(const uint16_t* W, int64_t rows, int64_t cols, int group, double* pmr) {
+  if (!W || !pmr || rows < 1 || cols < 1 || group < 1 || cols % group != 0) return -1;
+  const int64_t n_groups = rows * cols / group;
+  for (int64_t gi = 0; gi < n_groups; ++gi) {
+    double peak = 0.0, sum = 0.0;
+    for (int j = 0; j < group; ++j) {
+      const double a = fabs((double)rrq_oracle_bf16_to_f32(W[gi * group + j]));
+      if (a > peak) peak = a;
+      sum += a;
+    }
+    pmr[gi] = sum > 0.0 ? peak / (sum / (double)group) : 0.0;
   }
   return 0;
 }

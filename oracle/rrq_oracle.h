@@ -86,6 +86,23 @@ int rrq_oracle_gemv(const uint8_t* const* codes, const void* const* scales,
                     const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
                     int grid_sym, int scale_f16, const uint16_t* A, int batch, double* Y);
 
+/* Asymmetric stages with per-stage widths bits[k] in 1..4 (2^b levels,
+ * 2^b - 1 steps).  Group form as rrq_oracle_quantize_group; matrix form packs
+ * stage k's codes LSB-first, element c at bits bits[k]*c.., into
+ * codes[k] (rows*cols*bits[k]/8 bytes). */
+int rrq_oracle_quantize_group_bits(const float* x, int g, int n_stages, const int* bits,
+                                   uint8_t* Q, float* scale, float* zero, float* resid);
+int rrq_oracle_quantize_bits(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                             int n_stages, const int* bits, uint8_t* const* codes,
+                             float* const* scales, float* const* zeros);
+int rrq_oracle_reconstruct_bits(const uint8_t* const* codes, const float* const* scales,
+                                const float* const* zeros, int64_t rows, int64_t cols, int group,
+                                int k, const int* bits, uint16_t* out);
+
+/* Per-group peak-to-mean ratio max|x| / (sum|x| / g) of a bf16 matrix, in
+ * binary64 (0 for an all-zero group): pmr[rows*cols/group]. */
+int rrq_oracle_group_pmr(const uint16_t* W, int64_t rows, int64_t cols, int group, double* pmr);
+
 /* The scalar conversions the oracle uses, exported for tests. */
 float rrq_oracle_bf16_to_f32(uint16_t h);
 uint16_t rrq_oracle_f32_to_bf16(float f);

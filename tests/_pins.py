@@ -787,12 +787,164 @@ def pin_gemv_vs_bf16_reconstruction(orc, seed=43, rows=5, g=128) -> list[str]:
     return fails
 
 
+# ---------------------------------------------------------------------------
+# heterogeneous stage widths (asymmetric grid) and the group peak-to-mean ratio
+# ---------------------------------------------------------------------------
+# WH1: x = [-1, 0, 0.5, 2], widths [1, 3] (a 1-bit base, a 3-bit residual):
+#   stage 0: lo -1, hi 2, one step s = 3; d/s = [0, 1/3, 1/2, 1] -> rhe
+#            [0, 0, 0 (tie to even), 1]; levels [-1, -1, -1, 2], r = [0, 1, 1.5, 0];
+#   stage 1: lo 0, hi 1.5, seven steps s = fl(1.5/7); 1/s = 4.67 -> 5,
+#            1.5/s = 6.99999986 rounds to 7.0 -> 7, zeros -> 0.
+WH1 = dict(x=[-1.0, 0.0, 0.5, 2.0], bits=[1, 3], Q=[[0, 0, 0, 1], [0, 5, 7, 0]], s0=3.0, z=[-1.0, 0.0],
+           r0=[0.0, 1.0, 1.5, 0.0])
+
+
+def pin_bits_worked_and_two_bit_case(orc) -> list[str]:
+    fails = []
+    Q, s, z, r = orc.quantize_group_bits(np.array(WH1["x"], np.float32), WH1["bits"])
+    if Q.tolist() != WH1["Q"] or float(s[0]) != WH1["s0"] or z.tolist() != WH1["z"] or r[0].tolist() != WH1["r0"]:
+        fails.append(f"WH1: {Q.tolist()} {s.tolist()} {z.tolist()} {r[0].tolist()}")
+    if bits_of(s[1]) != bits_of(np.float32(1.5) / np.float32(7.0)):
+        fails.append(f"WH1: stage-1 scale {s[1]!r}")
+    # every width 2: the 2-bit quantizer (separately pinned) bit for bit
+    rng = np.random.default_rng(47)
+    for x in _random_groups(rng, 30, 128):
+        a = orc.quantize_group(x, 4)
+        b = orc.quantize_group_bits(x, [2, 2, 2, 2])
+        for u, v in zip(a, b):
+            if not np.array_equal(np.asarray(u).view(np.uint8), np.asarray(v).view(np.uint8)):
+                fails.append("widths [2, 2, 2, 2] differ from the 2-bit quantizer")
+                return fails
+    W = bf16_bits_of_f32(np.concatenate(_random_groups(rng, 6, 64)).reshape(3, 128))
+    a = orc.quantize(W, 64, 4)
+    b = orc.quantize_bits(W, 64, [2, 2, 2, 2])
+    for u, v in zip(a, b):
+        for uu, vv in zip(u, v):
+            if not np.array_equal(uu.view(np.uint8), vv.view(np.uint8)):
+                fails.append("packed widths [2, 2, 2, 2] differ from the 2-bit package")
+                return fails
+    return fails
+
+
+def pin_bits_brute_force_exact(orc, seed=53, count=200) -> list[str]:
+    """Dyadic groups for widths 1, 3, 4: lo = a/16, s = 2^e, values
+    lo + m 2^(e-2) with both ends present (range = (2^b - 1) 2^e): every step
+    exact; each code is the nearest of the 2^b levels, ties to the even code."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    for i in range(count):
+        b = (1, 3, 4)[i % 3]
+        steps = (1 << b) - 1
+        g = int(rng.integers(2, 17))
+        e = int(rng.integers(-4, 2))
+        lo = Fraction(int(rng.integers(-16, 17)), 16)
+        ms = list(rng.integers(0, 4 * steps + 1, size=g))
+        ms[0], ms[-1] = 0, 4 * steps
+        rng.shuffle(ms)
+        s = Fraction(2) ** e
+        xs = [lo + Fraction(int(m)) * Fraction(2) ** (e - 2) for m in ms]
+        Q, sc, z, r = orc.quantize_group_bits(np.array([float(v) for v in xs], np.float32), [b])
+        if Fraction(float(sc[0])) != s or Fraction(float(z[0])) != lo:
+            fails.append(f"b={b}: s={sc[0]} z={z[0]}")
+            continue
+        for j, v in enumerate(xs):
+            dist = [abs(v - (lo + q * s)) for q in range(steps + 1)]
+            best = min(dist)
+            cands = [q for q in range(steps + 1) if dist[q] == best]
+            want = cands[0] if len(cands) == 1 else [q for q in cands if q % 2 == 0][0]
+            if int(Q[0, j]) != want or Fraction(float(r[0, j])) != v - (lo + want * s):
+                fails.append(f"b={b}: x={float(v)} Q={int(Q[0, j])} want {want}")
+                break
+        if len(fails) > 5:
+            break
+    return fails
+
+
+def pin_bits_invariants_and_packing(orc, seed=59, g=64) -> list[str]:
+    """Random groups, widths [1, 3], [3, 1], [4, 2, 1], [2, 4]: zero = group
+    minimum, s = range / (2^b - 1) to rounding, half-step bound, the L-inf
+    error shrinks by 2^b - 1 per stage (to rounding); the packed codes equal
+    the per-group codes read back with numpy's little-endian bit unpacking;
+    prefix k reconstructs x - r_(k-1) to summation and bf16 rounding."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    rows, cols = 4, 2 * g
+    xs = np.concatenate(_random_groups(rng, rows * 2, g)).reshape(rows, cols)
+    W = bf16_bits_of_f32(xs)
+    for bits in ([1, 3], [3, 1], [4, 2, 1], [2, 4]):
+        codes, scales, zeros = orc.quantize_bits(W, g, bits)
+        for gi in range(rows * cols // g):
+            x = xs.reshape(-1)[gi * g:(gi + 1) * g]
+            Q, s, z, r = orc.quantize_group_bits(x, bits)
+            prev = x.astype(np.float64)
+            for k, b in enumerate(bits):
+                steps = (1 << b) - 1
+                lo, hi = float(np.min(prev)), float(np.max(prev))
+                if float(z[k]) != lo or abs(float(s[k]) - (hi - lo) / steps) > 2 ** -22 * (hi - lo) + 1e-45:
+                    fails.append(f"{bits} stage {k}: zero/scale")
+                rk = r[k].astype(np.float64)
+                bound = 0.5 * float(s[k]) + 2 ** -21 * (abs(lo) + (steps + 1) * float(s[k])) + 1e-45
+                if np.max(np.abs(rk)) > bound:
+                    fails.append(f"{bits} stage {k}: half step")
+                if np.max(np.abs(rk)) > np.max(np.abs(prev)) / steps * (1 + 2 ** -18) + 2 ** -20 * (abs(lo) + (steps + 1) * float(s[k])):
+                    fails.append(f"{bits} stage {k}: max|r| not reduced by 2^b - 1")
+                bitsarr = np.unpackbits(codes[k], bitorder="little")
+                c0 = gi * g
+                got = [int(sum(int(bitsarr[(c0 + j) * b + t]) << t for t in range(b))) for j in range(g)]
+                if got != Q[k].tolist():
+                    fails.append(f"{bits} stage {k}: packed codes")
+                prev = rk
+            if len(fails) > 5:
+                return fails
+        for k in range(1, len(bits) + 1):
+            rec = orc.reconstruct_bits(codes, scales, zeros, rows, cols, g, k, bits).reshape(-1)
+            recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+            for gi in range(rows * cols // g):
+                x = xs.reshape(-1)[gi * g:(gi + 1) * g].astype(np.float64)
+                r = orc.quantize_group_bits(x.astype(np.float32), bits)[3]
+                want = x - r[k - 1]
+                tol = np.abs(want) * 2 ** -8 + 8 * 2 ** -24 * (np.abs(x).max() + 1e-30)
+                if np.any(np.abs(recf[gi * g:(gi + 1) * g] - want) > tol):
+                    fails.append(f"{bits}: prefix {k} is not x - r")
+                    break
+    return fails
+
+
+def pin_group_pmr(orc, seed=61) -> list[str]:
+    """Closed forms of max|x| / mean|x|: a constant nonzero group gives 1, a
+    group with one nonzero gives g, j equal magnitudes (any signs) and zeros
+    give g / j, an all-zero group 0; random groups match the definition to
+    binary64 rounding."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    g = 128
+    rows = []
+    rows.append(np.full(g, 0.5, np.float32))
+    one = np.zeros(g, np.float32); one[17] = -3.0; rows.append(one)
+    j = 5
+    some = np.zeros(g, np.float32); some[:j] = [0.25, -0.25, 0.25, -0.25, 0.25]; rows.append(some)
+    rows.append(np.zeros(g, np.float32))
+    W = bf16_bits_of_f32(np.stack(rows)).reshape(1, 4 * g)
+    p = orc.group_pmr(W, g)
+    want = [1.0, float(g), g / j, 0.0]
+    if p.tolist() != want:
+        fails.append(f"closed forms {p.tolist()} != {want}")
+    xs = np.concatenate(_random_groups(rng, 8, g)).reshape(2, 4 * g)
+    p = orc.group_pmr(bf16_bits_of_f32(xs), g)
+    a = np.abs(xs.astype(np.float64)).reshape(-1, g)
+    ref = a.max(1) / a.mean(1)
+    if np.max(np.abs(p - ref) / ref) > 1e-12:
+        fails.append("random groups: pmr differs from max/mean")
+    return fails
+
+
 ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_brute_force_tiny,
             pin_invariants, pin_exact_grid, pin_prefix_reconstruction, pin_f16_rounding,
             pin_sym_worked_groups, pin_sym_brute_force_exact, pin_sym_invariants,
             pin_sym_prefix_reconstruction, pin_base_worked_groups, pin_base_branch_equivalence,
             pin_base_residual_invariants, pin_gemv_worked, pin_gemv_is_input_minus_residual,
-            pin_gemv_vs_bf16_reconstruction]
+            pin_gemv_vs_bf16_reconstruction, pin_bits_worked_and_two_bit_case, pin_bits_brute_force_exact,
+            pin_bits_invariants_and_packing, pin_group_pmr]
 
 
 def all_failures(orc) -> list[str]:

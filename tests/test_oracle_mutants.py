@@ -61,6 +61,17 @@ MUTANTS = {
     "gemv_wrong_output_row": ("Y[(size_t)b * rows + r] += (double)w", "Y[(size_t)b * rows + (rows - 1 - r)] += (double)w"),
     "gemv_bf16_weight": ("Y[(size_t)b * rows + r] += (double)w *",
                          "Y[(size_t)b * rows + r] += (double)rrq_oracle_bf16_to_f32(rrq_oracle_f32_to_bf16(w)) *"),
+    # heterogeneous widths and the peak-to-mean ratio
+    "bits_steps_pow2": ("const int m = (1 << bits[k]) - 1; /* steps of a b-bit grid */",
+                        "const int m = (1 << bits[k]); /* steps of a b-bit grid */"),
+    "bits_pack_msb_first": ("if ((q >> t) & 1) codes[bit / 8] |= (uint8_t)(1u << (bit % 8));",
+                            "if ((q >> t) & 1) codes[bit / 8] |= (uint8_t)(1u << (7 - bit % 8));"),
+    "bits_clamp_one_low": ("code = code < 0 ? 0 : (code > m ? m : code);", "code = code < 0 ? 0 : (code > m - 1 ? m - 1 : code);"),
+    "bits_read_reversed": ("q |= ((codes[bit / 8] >> (bit % 8)) & 1) << t;", "q |= ((codes[bit / 8] >> (bit % 8)) & 1) << (b - 1 - t);"),
+    "bits_level_drops_zero": ("      float lv = lo + qs;\n      v[j] = v[j] - lv;", "      float lv = qs;\n      v[j] = v[j] - lv;"),
+    "pmr_sum_not_mean": ("pmr[gi] = sum > 0.0 ? peak / (sum / (double)group) : 0.0;", "pmr[gi] = sum > 0.0 ? peak / sum : 0.0;"),
+    "pmr_signed_values": ("const double a = fabs((double)rrq_oracle_bf16_to_f32(W[gi * group + j]));",
+                          "const double a = (double)rrq_oracle_bf16_to_f32(W[gi * group + j]);"),
     "gemv_one_stage_short": ("      for (int i = 0; i < k; ++i) {\n        const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;\n        const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])\n                                  : ((const float*)scales[i])[gi];\n        const float lv",
                              "      for (int i = 0; i < k - (k > 1); ++i) {\n        const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;\n        const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])\n                                  : ((const float*)scales[i])[gi];\n        const float lv"),
 }
