@@ -202,7 +202,21 @@ typedef struct {
   int n_stages;   /* 1..4 stages held by the package */
   int grid;       /* rrq_grid */
   int scale_type; /* rrq_scale_type */
+  int bits[RRQ_MAX_STAGES]; /* code width of each stage, 1..4 (0 = 2); see below */
 } rrq_format;
+
+/* Heterogeneous stage widths (Section 3.2: stage k may have its own width
+ * b_k, the operating point after t stages is b_0 + ... + b_t bits; Table 3
+ * compares 1+3, 2+2 and 3+1 splits).  A stage of width b on the asymmetric
+ * grid has 2^b levels and m = 2^b - 1 steps:
+ *     s = fl(fl(hi - lo) / m),  Q = s == 0 ? 0 : clamp(rhe(fl(fl(v - lo) / s)), 0, m),
+ *     L = fl(lo + fl(Q * s)),   v' = fl(v - L)
+ * (b = 2 is the grid above).  Stage k's codes are packed least significant
+ * bit first, element c at bits b_k*c .. b_k*c + b_k - 1 of a byte array of
+ * rows*cols*b_k/8 bytes (rrq_stage_codes_bytes).  Widths other than 2 are
+ * supported with RRQ_GRID_ASYM and RRQ_SCALE_F32 by rrq_quantize_ex and
+ * rrq_reconstruct_ex; other combinations and calls return
+ * RRQ_ERR_UNSUPPORTED. */
 
 /* One matrix of rrq_quantize_ex.  scales[k] points to float (RRQ_SCALE_F32)
  * or uint16_t binary16 bit patterns (RRQ_SCALE_F16), rrq_meta_count entries,
@@ -285,12 +299,35 @@ typedef struct {
 rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
                     rrq_stream_t stream);
 
+/* One matrix of rrq_group_pmr. */
+typedef struct {
+  const uint16_t* W_bf16;  /* device, bf16 [rows, cols], 16-byte aligned */
+  int64_t rows, cols;      /* cols % group == 0 */
+  float* pmr;              /* device, float [rows*cols/group], 16-byte aligned */
+  float* stats;            /* device, float [2]: max and mean of pmr over the
+                              matrix's groups; NULL to skip */
+} rrq_pmr_desc;
+
+/* Group peak-to-mean ratio (Section 3.1; the group-maximum K/MAE of Table 9),
+ * the outlier statistic for choosing a stage split (Section 3.3):
+ *     pmr[g] = max |x| / (sum |x| / group) over group g (0 if all zero),
+ * max |x| exact, the sum in binary32 (|pmr - exact| <= group * 2^-24 * pmr
+ * to first order), and per matrix stats = {max_g pmr[g], mean_g pmr[g]}
+ * (fixed-order reduction, deterministic).  Same rules as rrq_quantize_batch
+ * for shapes, alignment, overlap and the stream. */
+rrq_status rrq_group_pmr(const rrq_pmr_desc* items, int count, int group, rrq_stream_t stream);
+
+/* Bytes of one stage's code array at width `bits` (1..4): rows*cols*bits/8.
+ * 0 for invalid arguments. */
+size_t rrq_stage_codes_bytes(int64_t rows, int64_t cols, int bits);
+
 /* Bytes of one stage's scale array in format *fmt: groups * (4 or 2).
  * 0 for invalid arguments. */
 size_t rrq_scales_bytes(int64_t rows, int64_t cols, const rrq_format* fmt);
 
-/* Total package bytes in format *fmt: n_stages * (codes + scales + zeros),
- * zeros only for RRQ_GRID_ASYM.  0 for invalid arguments. */
+/* Total package bytes in format *fmt: the sum over its stages of codes (at
+ * the stage's width) + scales + zeros, zeros only for RRQ_GRID_ASYM.  0 for
+ * invalid arguments. */
 size_t rrq_package_bytes_ex(int64_t rows, int64_t cols, const rrq_format* fmt);
 
 /* Bytes of one stage's code array: rows*cols/4 (rows*cols is a multiple of

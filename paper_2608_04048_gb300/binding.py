@@ -22,7 +22,8 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
 #: symbols declared in include/rrq.h
 EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
            "rrq_reconstruct_prefixes", "rrq_reconstruct_prefixes_batch",
-           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_gemv", "rrq_scales_bytes", "rrq_package_bytes_ex",
+           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_gemv",
+           "rrq_stage_codes_bytes", "rrq_group_pmr", "rrq_scales_bytes", "rrq_package_bytes_ex",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
            "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
@@ -36,9 +37,9 @@ SCALE_F32, SCALE_F16 = 0, 1
 
 
 class Format(ctypes.Structure):
-    """rrq_format of include/rrq.h"""
+    """rrq_format of include/rrq.h (bits: per-stage code widths, 0 = 2)"""
     _fields_ = [("group", ctypes.c_int), ("n_stages", ctypes.c_int), ("grid", ctypes.c_int),
-                ("scale_type", ctypes.c_int)]
+                ("scale_type", ctypes.c_int), ("bits", ctypes.c_int * MAX_STAGES)]
 
 
 class QuantizeDesc(ctypes.Structure):
@@ -56,6 +57,12 @@ class GemvDesc(ctypes.Structure):
 
 
 MAX_GEMV_BATCH = 8
+
+
+class PmrDesc(ctypes.Structure):
+    """rrq_pmr_desc of include/rrq.h"""
+    _fields_ = [("W_bf16", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("pmr", ctypes.c_void_p), ("stats", ctypes.c_void_p)]
 
 
 class ReconstructDesc(ctypes.Structure):
@@ -133,6 +140,10 @@ def load_library():
     lib.rrq_gemv.restype = i32
     lib.rrq_reconstruct_ex.argtypes = [ctypes.POINTER(ReconstructDesc), i32, fmt_p, i32, i32, vp]
     lib.rrq_reconstruct_ex.restype = i32
+    lib.rrq_group_pmr.argtypes = [ctypes.POINTER(PmrDesc), i32, i32, vp]
+    lib.rrq_group_pmr.restype = i32
+    lib.rrq_stage_codes_bytes.argtypes = [i64, i64, i32]
+    lib.rrq_stage_codes_bytes.restype = ctypes.c_size_t
     lib.rrq_scales_bytes.argtypes = [i64, i64, fmt_p]
     lib.rrq_scales_bytes.restype = ctypes.c_size_t
     lib.rrq_package_bytes_ex.argtypes = [i64, i64, fmt_p]
@@ -182,21 +193,24 @@ class Package:
     n_stages: int
     grid: int = GRID_ASYM
     scale_type: int = SCALE_F32
+    bits: tuple = (2, 2, 2, 2)
 
     @classmethod
     def empty(cls, rows, cols, group=128, n_stages=4, device=None, grid=GRID_ASYM,
-              scale_type=SCALE_F32) -> "Package":
+              scale_type=SCALE_F32, bits=None) -> "Package":
         device = device or torch.device("cuda", torch.cuda.current_device())
         n = rows * cols
+        bits = tuple(bits) if bits else (2,) * n_stages
         sdt = torch.float16 if scale_type == SCALE_F16 else torch.float32
         zeros = [] if grid == GRID_SYM else \
             [torch.empty(n // group, dtype=torch.float32, device=device) for _ in range(n_stages)]
-        return cls([torch.empty(n // 4, dtype=torch.uint8, device=device) for _ in range(n_stages)],
+        return cls([torch.empty(n * bits[k] // 8, dtype=torch.uint8, device=device) for k in range(n_stages)],
                    [torch.empty(n // group, dtype=sdt, device=device) for _ in range(n_stages)],
-                   zeros, rows, cols, group, n_stages, grid, scale_type)
+                   zeros, rows, cols, group, n_stages, grid, scale_type, bits + (2,) * (4 - len(bits)))
 
     def format(self) -> Format:
-        return Format(self.group, self.n_stages, self.grid, self.scale_type)
+        return Format(self.group, self.n_stages, self.grid, self.scale_type,
+                      (ctypes.c_int * MAX_STAGES)(*self.bits[:MAX_STAGES]))
 
     def nbytes(self) -> int:
         return sum(t.numel() * t.element_size() for t in self.codes + self.scales + self.zeros)
@@ -365,17 +379,18 @@ def quantize_descs(mats, pkgs) -> ctypes.Array:
 
 
 def rrq_quantize_ex(mats, group: int = 128, n_stages: int = 4, grid: int = GRID_SYM,
-                    scale_type: int = SCALE_F16, pkgs=None, stream=None, items=None):
+                    scale_type: int = SCALE_F16, pkgs=None, stream=None, items=None, bits=None):
     """Packages of a list of bf16 matrices in any supported format (one
     launch per 64 matrices).  Default: the symmetric grid with binary16
-    scales."""
+    scales.  bits: per-stage code widths (asymmetric grid), default 2."""
     lib = load_library()
     if pkgs is None:
-        pkgs = [Package.empty(W.shape[0], W.shape[1], group, n_stages, W.device, grid, scale_type)
+        pkgs = [Package.empty(W.shape[0], W.shape[1], group, n_stages, W.device, grid, scale_type, bits)
                 for W in mats]
     if items is None:
         items = quantize_descs(mats, pkgs)
-    fmt = Format(group, n_stages, grid, scale_type)
+    fmt = pkgs[0].format()
+    fmt.group, fmt.n_stages, fmt.grid, fmt.scale_type = group, n_stages, grid, scale_type
     rc = lib.rrq_quantize_ex(items, len(items), ctypes.byref(fmt), _stream_handle(stream))
     if rc != 0:
         raise RRQError(rc, "rrq_quantize_ex")
@@ -465,6 +480,30 @@ def rrq_reconstruct_ex(pkgs, k: int, all_prefixes: bool = False, outs=None, stre
     if rc != 0:
         raise RRQError(rc, "rrq_reconstruct_ex")
     return outs
+
+
+def rrq_group_pmr(mats, group: int = 128, stream=None):
+    """Per-group peak-to-mean ratios (float32 [rows*cols/group]) and per-matrix
+    [max, mean] (float32 [2]) of a list of bf16 matrices."""
+    lib = load_library()
+    items = (PmrDesc * len(mats))()
+    pmrs, stats = [], []
+    for it, W in zip(items, mats):
+        if W.dtype != torch.bfloat16 or W.dim() != 2 or not W.is_cuda or not W.is_contiguous():
+            raise TypeError("every W must be a contiguous 2-D bfloat16 CUDA tensor")
+        pm = torch.empty(W.numel() // group, dtype=torch.float32, device=W.device)
+        st = torch.empty(4, dtype=torch.float32, device=W.device)
+        it.W_bf16, (it.rows, it.cols), it.pmr, it.stats = W.data_ptr(), W.shape, pm.data_ptr(), st.data_ptr()
+        pmrs.append(pm)
+        stats.append(st[:2])
+    rc = lib.rrq_group_pmr(items, len(items), group, _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_group_pmr")
+    return pmrs, stats
+
+
+def rrq_stage_codes_bytes(rows: int, cols: int, bits: int) -> int:
+    return int(load_library().rrq_stage_codes_bytes(rows, cols, bits))
 
 
 def rrq_scales_bytes(rows: int, cols: int, group: int, grid: int, scale_type: int,

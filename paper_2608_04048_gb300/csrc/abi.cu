@@ -125,21 +125,30 @@ struct Fmt {
   int group = 0;
   int n_stages = 0;
   rrq::Format kind = rrq::kAsymF32;
-  bool sym() const { return kind != rrq::kAsymF32; }
+  int bits[RRQ_MAX_STAGES] = {2, 2, 2, 2};
+  bool sym() const { return kind == rrq::kSymF32 || kind == rrq::kSymF16; }
   uint64_t scale_bytes() const { return kind == rrq::kSymF16 ? 2 : 4; }
+  uint64_t code_bytes(uint64_t n, int k) const { return n * static_cast<uint64_t>(bits[k]) / 8; }
 };
 
 rrq_status parse_format(const rrq_format* f, Fmt* out) {
   if (!f || f->n_stages < 1 || f->n_stages > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
   if (f->grid != RRQ_GRID_ASYM && f->grid != RRQ_GRID_SYM) return RRQ_ERR_INVALID_ARG;
   if (f->scale_type != RRQ_SCALE_F32 && f->scale_type != RRQ_SCALE_F16) return RRQ_ERR_INVALID_ARG;
+  bool two_bit = true;
+  for (int k = 0; k < f->n_stages; ++k) {
+    if (f->bits[k] < 0 || f->bits[k] > 4) return RRQ_ERR_INVALID_ARG;
+    out->bits[k] = f->bits[k] == 0 ? 2 : f->bits[k];
+    two_bit = two_bit && out->bits[k] == 2;
+  }
   if (!group_supported(f->group)) return RRQ_ERR_UNSUPPORTED;
   out->group = f->group;
   out->n_stages = f->n_stages;
   if (f->grid == RRQ_GRID_ASYM) {
     if (f->scale_type != RRQ_SCALE_F32) return RRQ_ERR_UNSUPPORTED;
-    out->kind = rrq::kAsymF32;
+    out->kind = two_bit ? rrq::kAsymF32 : rrq::kAsymBits;
   } else {
+    if (!two_bit) return RRQ_ERR_UNSUPPORTED;  // other widths: asymmetric grid only
     out->kind = f->scale_type == RRQ_SCALE_F16 ? rrq::kSymF16 : rrq::kSymF32;
   }
   return RRQ_OK;
@@ -173,7 +182,7 @@ void add_quantize_ranges(const rrq_quantize_desc& it, const Fmt& f, bool from_ba
   r.push_back(range_of(it.W_bf16, 2 * n, false));
   for (int k = 0; k < f.n_stages; ++k) {
     const bool out = !(from_base && k == 0);
-    r.push_back(range_of(it.codes[k], n / 4, out));
+    r.push_back(range_of(it.codes[k], f.code_bytes(n, k), out));
     r.push_back(range_of(it.scales[k], f.scale_bytes() * (n / f.group), out));
     if (!f.sym()) r.push_back(range_of(it.zeros[k], 4 * (n / f.group), out));
   }
@@ -183,6 +192,7 @@ rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& 
                           bool from_base = false) {
   if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
   if (from_base && f.n_stages < 2) return RRQ_ERR_INVALID_ARG;
+  if (from_base && f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
   const int n_stages = f.n_stages;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (1 + 3 * n_stages));
@@ -210,6 +220,7 @@ rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& 
     std::memset(&p, 0, sizeof p);
     p.count = m;
     p.n_stages = n_stages;
+    for (int k = 0; k < RRQ_MAX_STAGES; ++k) p.bits[k] = f.bits[k];
     p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
     p.flags = g_debug_flags.load(std::memory_order_relaxed);
     p.status = st->status;
@@ -278,7 +289,7 @@ rrq_status reconstruct_views(const ReconView* items, int count, const Fmt& f, in
     const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
     for (int j = 0; j < n_out; ++j) ranges.push_back(range_of(it.out[j], 2 * n, true));
     for (int j = 0; j < k; ++j) {
-      ranges.push_back(range_of(it.codes[j], n / 4, false));
+      ranges.push_back(range_of(it.codes[j], f.code_bytes(n, j), false));
       ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
       if (!f.sym()) ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
     }
@@ -303,6 +314,7 @@ rrq_status reconstruct_views(const ReconView* items, int count, const Fmt& f, in
     const int m = std::min(rrq::kMaxBatch, count - base);
     std::memset(&p, 0, sizeof p);
     p.count = m;
+    for (int j = 0; j < RRQ_MAX_STAGES; ++j) p.bits[j] = f.bits[j];
     p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
     p.status = st->status;
     int64_t chunks = 0;
@@ -335,6 +347,7 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
                       rrq_stream_t stream) {
   if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
   if (batch < 1 || batch > rrq::kMaxGemvBatch) return RRQ_ERR_INVALID_ARG;
+  if (f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
   const int group = f.group;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (2 + 3 * k));
@@ -433,9 +446,59 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
   return RRQ_OK;
 }
 
+rrq_status pmr_batch(const rrq_pmr_desc* items, int count, int group, rrq_stream_t stream) {
+  if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
+  std::vector<Range> ranges;
+  for (int i = 0; i < count; ++i) {
+    const rrq_pmr_desc& it = items[i];
+    if (!it.W_bf16 || !it.pmr || !shape_ok(it.rows, it.cols) || it.cols % group != 0) return RRQ_ERR_INVALID_ARG;
+    if (!aligned(it.W_bf16, 16) || !aligned(it.pmr, 16) || (it.stats && !aligned(it.stats, 4)))
+      return RRQ_ERR_MISALIGNED;
+    const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
+    ranges.push_back(range_of(it.W_bf16, 2 * n, false));
+    ranges.push_back(range_of(it.pmr, 4 * (n / group), true));
+    if (it.stats) ranges.push_back(range_of(it.stats, 8, true));
+  }
+  if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
+  int dev = 0;
+  DeviceState* st = nullptr;
+  if (rrq_status rc = current_device(&dev, &st)) return rc;
+  for (int i = 0; i < count; ++i)
+    if (!on_device(items[i].W_bf16, dev) || !on_device(items[i].pmr, dev) ||
+        (items[i].stats && !on_device(items[i].stats, dev)))
+      return RRQ_ERR_INVALID_ARG;
+  static thread_local rrq::PmrBatch p;
+  for (int base = 0; base < count; base += rrq::kMaxBatch) {
+    const int m = std::min(rrq::kMaxBatch, count - base);
+    std::memset(&p, 0, sizeof p);
+    p.count = m;
+    p.group = group;
+    int64_t chunks = 0;
+    for (int i = 0; i < m; ++i) {
+      const rrq_pmr_desc& it = items[base + i];
+      rrq::PmrItem& q = p.item[i];
+      q.W = it.W_bf16;
+      q.pmr = it.pmr;
+      q.stats = it.stats;
+      q.n = it.rows * it.cols;
+      q.chunk_begin = chunks;
+      chunks += (q.n + rrq::kChunkElems - 1) / rrq::kChunkElems;
+    }
+    p.total_chunks = chunks;
+    cudaError_t e = rrq::pmr_launch(group, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
+    if (e != cudaSuccess) return fail_cuda(e);
+  }
+  return RRQ_OK;
+}
+
 }  // namespace
 
 extern "C" {
+
+rrq_status rrq_group_pmr(const rrq_pmr_desc* items, int count, int group, rrq_stream_t stream) {
+  return pmr_batch(items, count, group, stream);
+}
 
 size_t rrq_codes_bytes(int64_t rows, int64_t cols) {
   if (!shape_ok(rows, cols)) return 0;
@@ -574,6 +637,11 @@ rrq_status rrq_reconstruct_ex(const rrq_reconstruct_desc* items, int count, cons
   return reconstruct_views(v.data(), count, f, k, all_prefixes != 0, stream);
 }
 
+size_t rrq_stage_codes_bytes(int64_t rows, int64_t cols, int bits) {
+  if (!shape_ok(rows, cols) || bits < 1 || bits > 4) return 0;
+  return static_cast<size_t>(rows * cols) * static_cast<size_t>(bits) / 8;
+}
+
 size_t rrq_scales_bytes(int64_t rows, int64_t cols, const rrq_format* fmt) {
   Fmt f;
   if (parse_format(fmt, &f) != RRQ_OK) return 0;
@@ -585,8 +653,10 @@ size_t rrq_package_bytes_ex(int64_t rows, int64_t cols, const rrq_format* fmt) {
   if (parse_format(fmt, &f) != RRQ_OK) return 0;
   const size_t m = rrq_meta_count(rows, cols, f.group);
   if (m == 0) return 0;
-  const size_t per_stage = rrq_codes_bytes(rows, cols) + m * (f.scale_bytes() + (f.sym() ? 0 : 4));
-  return static_cast<size_t>(f.n_stages) * per_stage;
+  size_t total = 0;
+  for (int k = 0; k < f.n_stages; ++k)
+    total += rrq_stage_codes_bytes(rows, cols, f.bits[k]) + m * (f.scale_bytes() + (f.sym() ? 0 : 4));
+  return total;
 }
 
 rrq_status rrq_get_device_status(rrq_stream_t stream) {

@@ -73,7 +73,7 @@ struct Cursor {
 template <int F, int K, int B>
 __global__ void __launch_bounds__(kThreads, 1)
 gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
-  constexpr bool kSym = F != kAsymF32;
+  constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
   constexpr int kBuf = K * kStageBytes;
   constexpr int kRing = ring_depth<K>();

@@ -68,6 +68,17 @@
 // ahead, dequantizes stage 0 in registers with the grid's level formula,
 // starts the running residual at fl(x - L_0) and computes stages 1.. only.
 //
+// Heterogeneous stage widths (kAsymBits): stage k has b_k in 1..4 bits, 2^b - 1
+// steps.  The band test above covers the 2-bit boundaries only; for any
+// width the kernel instead checks each element: with q the two-float
+// quotient, if q is farther than 2^-17 from every half-integer (while
+// ulp(q) <= 2^-20 for q < 16 and |q - x| < 2^-40), x, RN(x) and q round to the
+// same integer and the fast code is exact; the few elements within the margin
+// (and groups with a scale outside [2^-90, 2^90]) take the IEEE-division
+// path.  Codes are packed least significant bit first, element c at bits
+// b*c.., so a lane's 32 weights fill b words; for this format the lane reads
+// its shared-memory pieces in natural order.
+//
 // This header holds the kernel template; quantize.cu instantiates the build
 // without a base checkpoint, quantize_base.cu the build from one.
 #pragma once
@@ -167,6 +178,163 @@ __device__ __forceinline__ bool corrected_quotient_safe(float s) {
 // eight calls the codes of elements 0..7 sit at bits 16..31, element 0 lowest.
 __device__ __forceinline__ uint32_t push_code(uint32_t acc, uint32_t t) {
   return __funnelshift_r(acc, t, 2);
+}
+
+// b-bit stages: the per-element IEEE-division path for m = 2^b - 1 steps.
+__device__ __noinline__ ExactPair exact_pair_bits(f32x2 v, float lo, float s, int m) {
+  float a, b;
+  unpack2(v, a, b);
+  int qa = 0, qb = 0;
+  if (s != 0.0f) {
+    qa = __float2int_rn(__fdiv_rn(__fsub_rn(a, lo), s));  // round half to even
+    qb = __float2int_rn(__fdiv_rn(__fsub_rn(b, lo), s));
+    qa = qa < 0 ? 0 : (qa > m ? m : qa);
+    qb = qb < 0 ? 0 : (qb > m ? m : qb);
+  }
+  const float wa = __fsub_rn(a, __fadd_rn(lo, __fmul_rn(__int2float_rn(qa), s)));
+  const float wb = __fsub_rn(b, __fadd_rn(lo, __fmul_rn(__int2float_rn(qb), s)));
+  return {pack2(wa, wb), static_cast<uint32_t>(qa), static_cast<uint32_t>(qb)};
+}
+
+constexpr float kTieMargin = 0.5f - 0x1p-17f;  // |q - rhe(q)| beyond this: near a half-integer
+
+// One b-bit stage of a lane's 32 values (natural order): codes into words
+// (element j at bits B*j), residuals in place, min/max of the new residuals.
+template <int B>
+__device__ __forceinline__ void stage_bits(f32x2 (&v)[16], float lo, float s, bool fast,
+                                           uint32_t (&words)[4], float& mn, float& mx) {
+  constexpr int M = (1 << B) - 1;
+  constexpr uint32_t kMask = static_cast<uint32_t>(M);
+#pragma unroll
+  for (int w = 0; w < 4; ++w) words[w] = 0u;
+  float mn0 = __int_as_float(0x7f800000), mn1 = mn0, mx0 = -mn0, mx1 = mx0;
+  auto place = [&](int j, uint32_t code) {  // element j's code at bits B*j
+    const int bit = B * j, w = bit >> 5, sh = bit & 31;
+    words[w] |= code << sh;
+    if (sh + B > 32) words[w + 1] |= code >> (32 - sh);
+  };
+  float r_hi = 0.0f, r_lo = 0.0f;
+  if (fast && s > 0.0f) recip2(s, r_hi, r_lo);
+  const float c = __fmul_rn(-kTwo23, s);
+  const f32x2 LO = pack2(lo, lo), RH = pack2(r_hi, r_hi), RL = pack2(r_lo, r_lo), S = pack2(s, s);
+  const f32x2 T23 = pack2(kTwo23, kTwo23), C = pack2(c, c);
+#pragma unroll
+  for (int i = 0; i < 16; ++i) {
+    uint32_t ca, cb;
+    bool exact = !fast;
+    f32x2 t = T23;
+    if (fast) {
+      const f32x2 d = sub2(v[i], LO);
+      const f32x2 q = fma2(d, RH, mul2(d, RL));  // d/s to 2^-45.3
+      t = add2(q, T23);                          // 2^23 + rhe(q)
+      float fa, fb;
+      unpack2(sub2(q, sub2(t, T23)), fa, fb);    // q - rhe(q), exact
+      exact = fabsf(fa) > kTieMargin || fabsf(fb) > kTieMargin;
+    }
+    if (exact) {
+      const ExactPair x = exact_pair_bits(v[i], lo, s, M);
+      v[i] = x.w;
+      ca = x.q0;
+      cb = x.q1;
+    } else {
+      v[i] = sub2(v[i], add2(LO, fma2(t, S, C)));  // v - fl(lo + fl(Q s))
+      ca = static_cast<uint32_t>(t) & kMask;
+      cb = static_cast<uint32_t>(t >> 32) & kMask;
+    }
+    place(2 * i, ca);
+    place(2 * i + 1, cb);
+    float a, b;
+    unpack2(v[i], a, b);
+    if (i & 1) {
+      mn1 = fminf(mn1, fminf(a, b));
+      mx1 = fmaxf(mx1, fmaxf(a, b));
+    } else {
+      mn0 = fminf(mn0, fminf(a, b));
+      mx0 = fmaxf(mx0, fmaxf(a, b));
+    }
+  }
+  mn = fminf(mn0, mn1);
+  mx = fmaxf(mx0, mx1);
+}
+
+template <int B>
+__device__ __forceinline__ void store_words(uint8_t* codes, int64_t e0, const uint32_t (&w)[4]) {
+  uint8_t* dst = codes + (e0 >> 5) * (4 * B);  // 4B bytes per 32 weights
+  if (B == 4) {
+    __stcs(reinterpret_cast<uint4*>(dst), make_uint4(w[0], w[1], w[2], w[3]));
+  } else if (B == 2) {
+    __stcs(reinterpret_cast<uint2*>(dst), make_uint2(w[0], w[1]));
+  } else {
+#pragma unroll
+    for (int j = 0; j < B; ++j) __stcs(reinterpret_cast<unsigned int*>(dst) + j, w[j]);
+  }
+}
+
+// Asymmetric grid with per-stage widths (values in natural order).
+template <int G>
+__device__ __forceinline__ void quantize_chunk_bits(const QuantizeBatch& p, const QuantizeItem& it,
+                                                    int64_t e0, int lane, uint4 (&raw)[4]) {
+  constexpr int L = G / 32;  // lanes per group
+  const bool valid = e0 < it.n;
+  if (!valid) {
+#pragma unroll
+    for (int j = 0; j < 4; ++j) raw[j] = make_uint4(0u, 0u, 0u, 0u);
+  }
+  f32x2 v[16];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    const uint32_t w4[4] = {raw[j].x, raw[j].y, raw[j].z, raw[j].w};
+#pragma unroll
+    for (int m = 0; m < 4; ++m) v[4 * j + m] = pack2u(w4[m] << 16, w4[m] & 0xffff0000u);
+  }
+  float lo, hi;
+  lane_minmax(v, lo, hi);
+  group_minmax<L>(lo, hi);
+
+#pragma unroll 1
+  for (int k = 0; k < p.n_stages; ++k) {
+    if (__any_sync(kFullMask, lo == 0.0f)) {  // a zero minimum is -0 if the group holds a -0
+      uint32_t neg = 0;
+      if (lo == 0.0f) {
+#pragma unroll
+        for (int i = 0; i < 16; ++i)
+          neg |= (static_cast<uint32_t>(v[i]) == 0x80000000u) |
+                 (static_cast<uint32_t>(v[i] >> 32) == 0x80000000u);
+      }
+      neg = group_or<L>(neg);
+      if (lo == 0.0f) lo = neg ? -0.0f : 0.0f;
+    }
+    const int b = p.bits[k];
+    const float range = __fsub_rn(hi, lo);
+    const float s = b == 2 ? div3(range) : b == 1 ? range : __fdiv_rn(range, static_cast<float>((1 << b) - 1));
+    const uint32_t e = __float_as_uint(s) >> 23;
+    const bool fast = !(p.flags & kDebugForceExact) && (s == 0.0f || (e - (127u - 90u)) < 180u);
+    uint32_t words[4];
+    float mn, mx;
+    switch (b) {
+      case 1: stage_bits<1>(v, lo, s, fast, words, mn, mx); break;
+      case 3: stage_bits<3>(v, lo, s, fast, words, mn, mx); break;
+      case 4: stage_bits<4>(v, lo, s, fast, words, mn, mx); break;
+      default: stage_bits<2>(v, lo, s, fast, words, mn, mx); break;
+    }
+    if (valid) {
+      switch (b) {
+        case 1: store_words<1>(it.codes[k], e0, words); break;
+        case 3: store_words<3>(it.codes[k], e0, words); break;
+        case 4: store_words<4>(it.codes[k], e0, words); break;
+        default: store_words<2>(it.codes[k], e0, words); break;
+      }
+      if ((lane & (L - 1)) == 0) {
+        __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s);
+        __stcs(it.zeros[k] + e0 / G, lo);
+      }
+    }
+    if (k + 1 < p.n_stages) {
+      lo = mn;
+      hi = mx;
+      group_minmax<L>(lo, hi);
+    }
+  }
 }
 
 // Stores the packed codes of stage k of this lane's 32 weights: acc[m] holds
@@ -415,12 +583,16 @@ __device__ __forceinline__ void quantize_chunk(const QuantizeBatch& p, const Qua
                                                uint32_t ld_lo, uint32_t ld_hi) {
   if constexpr (F == kAsymF32)
     quantize_chunk_asym<G, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
+  else if constexpr (F == kAsymBits)
+    quantize_chunk_bits<G>(p, it, e0, lane, raw);
   else
     quantize_chunk_sym<G, F == kSymF16, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
 }
 
+// (the width-generic stages need more registers: two CTAs per SM)
 template <int G, int F, bool kBase>
-__global__ void __launch_bounds__(kThreads, RRQ_QUANTIZE_CTAS_PER_SM) quantize_kernel(const __grid_constant__ QuantizeBatch p) {
+__global__ void __launch_bounds__(kThreads, F == kAsymBits ? 2 : RRQ_QUANTIZE_CTAS_PER_SM)
+quantize_kernel(const __grid_constant__ QuantizeBatch p) {
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -463,7 +635,8 @@ __global__ void __launch_bounds__(kThreads, RRQ_QUANTIZE_CTAS_PER_SM) quantize_k
 
   // Lane l reads its four 16-byte pieces in rotated order so that a quarter
   // warp touches eight distinct bank groups; slot j holds piece (j+rot)&3.
-  const int rot = (lane >> 1) & 3;
+  // (The heterogeneous-width format packs its codes in natural order.)
+  const int rot = F == kAsymBits ? 0 : (lane >> 1) & 3;
   const uint32_t sel_lo = rot == 0 ? 0x3210u : rot == 1 ? 0x1076u : rot == 2 ? 0x7654u : 0x5432u;
   const uint32_t sel_hi = rot == 0 ? 0x7654u : rot == 1 ? 0x5432u : rot == 2 ? 0x3210u : 0x1076u;
   // the inverse rotation, for a base code word read in memory order
@@ -561,7 +734,9 @@ cudaError_t prepare_all() {
   cudaError_t e;
   if ((e = prepare_f<kAsymF32, kBase>())) return e;
   if ((e = prepare_f<kSymF32, kBase>())) return e;
-  return prepare_f<kSymF16, kBase>();
+  if ((e = prepare_f<kSymF16, kBase>())) return e;
+  if constexpr (!kBase) return prepare_f<kAsymBits, false>();
+  return cudaSuccess;
 }
 
 template <bool kBase>
@@ -570,6 +745,9 @@ cudaError_t launch_all(int group, Format fmt, const QuantizeBatch& p, cudaStream
     case kAsymF32: return launch_f<kAsymF32, kBase>(group, p, stream, sms);
     case kSymF32: return launch_f<kSymF32, kBase>(group, p, stream, sms);
     case kSymF16: return launch_f<kSymF16, kBase>(group, p, stream, sms);
+    case kAsymBits:
+      if constexpr (!kBase) return launch_f<kAsymBits, false>(group, p, stream, sms);
+      break;
   }
   return cudaErrorInvalidValue;
 }

@@ -27,9 +27,14 @@
 // the lane's scale and its neighbour's (the copy is cut to 2 bytes at the end
 // of an array with an odd number of groups) and widened exactly.
 //
+// Heterogeneous stage widths (kAsymBits): a lane copies the 4b bytes of its
+// b-bit codes per stage, extracts each code by shift and mask and forms
+// fl(zero + fl(Q s)) as fma(t - 2^23, s, 0) + zero; values are kept in natural
+// order.
+//
 // This header holds the kernel template; reconstruct_asym_f32.cu,
-// reconstruct_sym_f32.cu and reconstruct_sym_f16.cu each instantiate one
-// package format (they compile in parallel).
+// reconstruct_sym_f32.cu, reconstruct_sym_f16.cu and reconstruct_asym_bits.cu
+// each instantiate one package format (they compile in parallel).
 #pragma once
 
 #include <cuda_bf16.h>
@@ -43,13 +48,38 @@ namespace {
 constexpr int kWarps = 8;
 constexpr int kThreads = kWarps * 32;
 constexpr int kRing = 4;               // chunks of inputs per warp in shared memory
-constexpr int kStageBytes = 512;       // one stage of one chunk: codes 256 B, scales 128 B, zeros 128 B
 constexpr float kTwo23 = 8388608.0f;   // bits 0x4B000000 | q encode 2^23 + q for 0 <= q < 2^23
 
-template <int K>
-__host__ __device__ constexpr int warp_smem_bytes() { return kRing * K * kStageBytes + 2 * kChunkBytes; }
-template <int K>
-__host__ __device__ constexpr int smem_bytes() { return kWarps * warp_smem_bytes<K>(); }
+// One stage of one chunk in shared memory: codes (8 B per lane, 16 B for the
+// heterogeneous-width format), then scales 128 B, zeros 128 B.
+template <int F>
+__host__ __device__ constexpr int code_bytes() { return F == kAsymBits ? 512 : 256; }
+template <int F>
+__host__ __device__ constexpr int stage_bytes() { return code_bytes<F>() + 256; }
+template <int K, int F>
+__host__ __device__ constexpr int warp_smem_bytes() { return kRing * K * stage_bytes<F>() + 2 * kChunkBytes; }
+template <int K, int F>
+__host__ __device__ constexpr int smem_bytes() { return kWarps * warp_smem_bytes<K, F>(); }
+
+// Stage values of 32 codes of width B (element j at bits B*j of w), natural
+// order: acc = level (first stage) or fl(acc + level).
+template <int B>
+__device__ __forceinline__ void dequant_bits(const uint4& w4, float s, float z, bool first, f32x2 (&acc)[16]) {
+  const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
+  auto code = [&](int j) -> uint32_t {
+    const int bit = B * j, i = bit >> 5, sh = bit & 31;
+    uint32_t c = w[i] >> sh;
+    if (sh + B > 32) c |= w[i + 1] << (32 - sh);
+    return c & ((1u << B) - 1u);
+  };
+  const f32x2 S = pack2(s, s), Z = pack2(z, z), T23 = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f);
+#pragma unroll
+  for (int m = 0; m < 16; ++m) {
+    const f32x2 t = pack2u(0x4B000000u | code(2 * m), 0x4B000000u | code(2 * m + 1));
+    const f32x2 level = add2(Z, fma2(sub2(t, T23), S, Z0));  // fl(zero + fl(Q s))
+    acc[m] = first ? level : add2(acc[m], level);
+  }
+}
 
 __device__ __forceinline__ bool prescale_ok(float s) {
   return s == 0.0f || (s >= 0x1p-100f && s <= 0x1p+100f);
@@ -59,12 +89,14 @@ __device__ __forceinline__ bool prescale_ok(float s) {
 // 1..K in one pass over the package) instead of only after stage K-1.
 template <int G, int K, bool kAllPrefixes, int F>
 __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_constant__ ReconstructBatch p) {
-  constexpr bool kSym = F != kAsymF32;
+  constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  uint8_t* ring = smem + warp * warp_smem_bytes<K>();
+  constexpr int kStageBytes = stage_bytes<F>();
+  constexpr int kCB = code_bytes<F>();
+  uint8_t* ring = smem + warp * warp_smem_bytes<K, F>();
   uint8_t* stage_buf = ring + kRing * K * kStageBytes;
   constexpr int kBufBytes = K * kStageBytes;
 
@@ -75,7 +107,7 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
   // Slot j of a lane handles its 16-byte output piece (j + rot) & 3, so that
   // the shared-memory stores of a quarter warp hit distinct bank groups; the
   // code words are rotated right by 16*rot bits to match.
-  const int rot = (lane >> 1) & 3;
+  const int rot = F == kAsymBits ? 0 : (lane >> 1) & 3;
   const uint32_t sel_lo = rot == 0 ? 0x3210u : rot == 1 ? 0x5432u : rot == 2 ? 0x7654u : 0x1076u;
   const uint32_t sel_hi = rot == 0 ? 0x7654u : rot == 1 ? 0x1076u : rot == 2 ? 0x3210u : 0x5432u;
 
@@ -103,11 +135,26 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
         n_scale = valid ? (left < 4 ? 2u : 4u) : 0u;
       }
       const uint32_t n8 = valid ? 8u : 0u, n4 = valid ? 4u : 0u;
-      const uint32_t base = smem_u32(ring + buf * K * kStageBytes) + lane * 8;
-      const uint32_t mbase = smem_u32(ring + buf * K * kStageBytes) + 256 + lane * 4;
+      const uint32_t base = smem_u32(ring + buf * K * kStageBytes) + lane * (F == kAsymBits ? 16 : 8);
+      const uint32_t mbase = smem_u32(ring + buf * K * kStageBytes) + kCB + lane * 4;
 #pragma unroll
       for (int i = 0; i < K; ++i) {
-        cp_async_8(base + i * kStageBytes, reinterpret_cast<const char*>(it.codes[i]) + off_code, n8);
+        if (F == kAsymBits) {  // 4b bytes of b-bit codes for the lane's 32 weights
+          const int b = p.bits[i];
+          const char* src = reinterpret_cast<const char*>(it.codes[i]) + (valid ? (static_cast<uint64_t>(e) >> 5) * 4 * b : 0);
+          const uint32_t dst = base + i * kStageBytes;
+          if (b == 4) cp_async_16(dst, src, valid ? 16u : 0u);
+          else if (b == 2) cp_async_8(dst, src, n8);
+          else {
+            cp_async_4(dst, src, n4);
+            if (b == 3) {
+              cp_async_4(dst + 4, src + 4, n4);
+              cp_async_4(dst + 8, src + 8, n4);
+            }
+          }
+        } else {
+          cp_async_8(base + i * kStageBytes, reinterpret_cast<const char*>(it.codes[i]) + off_code, n8);
+        }
         cp_async_4(mbase + i * kStageBytes, reinterpret_cast<const char*>(it.scales[i]) + off_meta, n_scale);
         if (!kSym)
           cp_async_4(mbase + i * kStageBytes + 128, reinterpret_cast<const char*>(it.zeros[i]) + off_meta, n4);
@@ -130,16 +177,16 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
     bool ok = true;
 #pragma unroll
     for (int i = 0; i < K; ++i) {
-      code[i] = *reinterpret_cast<const uint2*>(buf + i * kStageBytes + lane * 8);
+      code[i] = F == kAsymBits ? make_uint2(0u, 0u) : *reinterpret_cast<const uint2*>(buf + i * kStageBytes + lane * 8);
       if (kF16) {
         // group index parity of this lane: chunks start on an even group
-        const uint32_t w = *reinterpret_cast<const uint32_t*>(buf + i * kStageBytes + 256 + lane * 4);
+        const uint32_t w = *reinterpret_cast<const uint32_t*>(buf + i * kStageBytes + kCB + lane * 4);
         const uint32_t h = ((lane / (G / 32)) & 1) ? (w >> 16) : (w & 0xffffu);
         scale[i] = __half2float(__ushort_as_half(static_cast<unsigned short>(h)));
       } else {
-        scale[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + 256 + lane * 4);
+        scale[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + kCB + lane * 4);
       }
-      zero[i] = kSym ? 0.0f : *reinterpret_cast<const float*>(buf + i * kStageBytes + 384 + lane * 4);
+      zero[i] = kSym ? 0.0f : *reinterpret_cast<const float*>(buf + i * kStageBytes + kCB + 128 + lane * 4);
       ok = ok && prescale_ok(scale[i]);
     }
 
@@ -182,7 +229,15 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
       const uint32_t w0 = __byte_perm(code[i].x, code[i].y, sel_lo);
       const uint32_t w1 = __byte_perm(code[i].x, code[i].y, sel_hi);
       const f32x2 LO = pack2(zero[i], zero[i]);
-      if (kSym) {
+      if (F == kAsymBits) {
+        const uint4 w4 = *reinterpret_cast<const uint4*>(buf + i * kStageBytes + lane * 16);
+        switch (p.bits[i]) {
+          case 1: dequant_bits<1>(w4, scale[i], zero[i], i == 0, acc); break;
+          case 3: dequant_bits<3>(w4, scale[i], zero[i], i == 0, acc); break;
+          case 4: dequant_bits<4>(w4, scale[i], zero[i], i == 0, acc); break;
+          default: dequant_bits<2>(w4, scale[i], zero[i], i == 0, acc); break;
+        }
+      } else if (kSym) {
         // u = Q - 2 (times 4^j in the prescaled form), exact; L = u * s exact
         const float s = scale[i];
         if (all_ok) {
@@ -253,14 +308,14 @@ cudaError_t launch_gk(const ReconstructBatch& p, cudaStream_t stream, int sms) {
   static int blocks_per_sm = 0;
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, reconstruct_kernel<G, K, A, F>, kThreads, smem_bytes<K>());
+        &blocks_per_sm, reconstruct_kernel<G, K, A, F>, kThreads, smem_bytes<K, F>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
   const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  reconstruct_kernel<G, K, A, F><<<grid, kThreads, smem_bytes<K>(), stream>>>(p);
+  reconstruct_kernel<G, K, A, F><<<grid, kThreads, smem_bytes<K, F>(), stream>>>(p);
   return cudaGetLastError();
 }
 
@@ -278,10 +333,10 @@ cudaError_t launch_g(int k, const ReconstructBatch& p, cudaStream_t stream, int 
 template <int G, bool A, int F>
 cudaError_t prepare_ga() {
   cudaError_t e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 1, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1>()))) return e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 2, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2>()))) return e;
-  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 3, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<3>()))) return e;
-  return cudaFuncSetAttribute(reconstruct_kernel<G, 4, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<4>());
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 1, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<1, F>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 2, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<2, F>()))) return e;
+  if ((e = cudaFuncSetAttribute(reconstruct_kernel<G, 3, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<3, F>()))) return e;
+  return cudaFuncSetAttribute(reconstruct_kernel<G, 4, A, F>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_bytes<4, F>());
 }
 
 template <int G, int F>

@@ -109,6 +109,10 @@ __device__ __forceinline__ void cp_async_4(uint32_t dst, const void* src, uint32
   asm volatile("cp.async.ca.shared.global [%0], [%1], 4, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
                : "memory");
 }
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void* src, uint32_t src_bytes) {
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src), "r"(src_bytes)
+               : "memory");
+}
 // streaming (evict-first) 16-bit global store
 __device__ __forceinline__ void stcs_u16(uint16_t* p, uint16_t v) {
   asm volatile("st.global.cs.u16 [%0], %1;" ::"l"(p), "h"(v) : "memory");

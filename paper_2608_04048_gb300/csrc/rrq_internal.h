@@ -19,6 +19,7 @@ enum Format : int {
   kAsymF32 = 0,  // zero = group minimum, binary32 scale and zero
   kSymF32 = 1,   // implicit zero-point 2, binary32 scale
   kSymF16 = 2,   // implicit zero-point 2, binary16 scale
+  kAsymBits = 3, // zero = group minimum, binary32 scale and zero, per-stage widths 1..4
 };
 
 constexpr unsigned kStatusTimeout = 1u;           // bit set in the device status word
@@ -39,6 +40,7 @@ struct QuantizeItem {
 struct QuantizeBatch {
   int count;                       // 1..kMaxBatch
   int n_stages;                    // 1..4
+  int bits[kMaxStages];            // code width per stage (kAsymBits), else 2
   uint32_t wait_limit_us;
   uint32_t flags;                  // kDebugForceExact
   unsigned* status;                // device status word
@@ -57,6 +59,7 @@ struct ReconstructItem {
 
 struct ReconstructBatch {
   int count;
+  int bits[kMaxStages];            // code width per stage (kAsymBits), else 2
   uint32_t wait_limit_us;
   unsigned* status;                // device status word
   int64_t total_chunks;
@@ -92,12 +95,31 @@ constexpr int kGemvRows = 16;      // rows per block
 
 constexpr int kMaxGemvBatch = 8;   // activation rows (tokens) per call
 
+// One matrix of a group peak-to-mean ratio launch.
+struct PmrItem {
+  const uint16_t* W;               // bf16, n elements
+  float* pmr;                      // n/group
+  float* stats;                    // [2] max and mean over the groups, or null
+  int64_t n;
+  int64_t chunk_begin;
+};
+
+struct PmrBatch {
+  int count;
+  int group;
+  int64_t total_chunks;
+  PmrItem item[kMaxBatch];
+};
+
+cudaError_t pmr_launch(int group, const PmrBatch& p, cudaStream_t stream, int sms);
+
 // One-time per-device set-up of kernel attributes (dynamic shared memory).
 cudaError_t quantize_prepare();
 cudaError_t quantize_prepare_base();
 cudaError_t reconstruct_prepare_asym_f32();
 cudaError_t reconstruct_prepare_sym_f32();
 cudaError_t reconstruct_prepare_sym_f16();
+cudaError_t reconstruct_prepare_asym_bits();
 
 // Launch on `stream`; `sms` = multiprocessor count of the current device.
 cudaError_t quantize_launch(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream, int sms);
@@ -113,6 +135,8 @@ cudaError_t reconstruct_launch_sym_f32(int group, int k, bool all_prefixes, cons
                                        cudaStream_t stream, int sms);
 cudaError_t reconstruct_launch_sym_f16(int group, int k, bool all_prefixes, const ReconstructBatch& p,
                                        cudaStream_t stream, int sms);
+cudaError_t reconstruct_launch_asym_bits(int group, int k, bool all_prefixes, const ReconstructBatch& p,
+                                         cudaStream_t stream, int sms);
 
 // Activation rows one launch can hold in shared memory for matrices of up to
 // max_cols columns with k stages (0: too wide).
@@ -129,6 +153,7 @@ inline cudaError_t gemv_launch(Format fmt, int k, int nb, int64_t max_cols, cons
     case kAsymF32: return gemv_launch_asym_f32(k, nb, max_cols, p, stream, sms);
     case kSymF32: return gemv_launch_sym_f32(k, nb, max_cols, p, stream, sms);
     case kSymF16: return gemv_launch_sym_f16(k, nb, max_cols, p, stream, sms);
+    case kAsymBits: break;
   }
   return cudaErrorInvalidValue;
 }
@@ -137,7 +162,8 @@ inline cudaError_t reconstruct_prepare() {
   cudaError_t e;
   if ((e = reconstruct_prepare_asym_f32())) return e;
   if ((e = reconstruct_prepare_sym_f32())) return e;
-  return reconstruct_prepare_sym_f16();
+  if ((e = reconstruct_prepare_sym_f16())) return e;
+  return reconstruct_prepare_asym_bits();
 }
 
 inline cudaError_t reconstruct_launch(int group, Format fmt, int k, bool all_prefixes,
@@ -146,6 +172,7 @@ inline cudaError_t reconstruct_launch(int group, Format fmt, int k, bool all_pre
     case kAsymF32: return reconstruct_launch_asym_f32(group, k, all_prefixes, p, stream, sms);
     case kSymF32: return reconstruct_launch_sym_f32(group, k, all_prefixes, p, stream, sms);
     case kSymF16: return reconstruct_launch_sym_f16(group, k, all_prefixes, p, stream, sms);
+    case kAsymBits: return reconstruct_launch_asym_bits(group, k, all_prefixes, p, stream, sms);
   }
   return cudaErrorInvalidValue;
 }
