@@ -168,6 +168,64 @@ def time_gemv(pkgs, specs, stream, batch: int = 1, reps: int = 5) -> dict:
     return out
 
 
+def time_bits(mats, p_outs, specs, stream, bits, reps: int = 3) -> dict:
+    """A heterogeneous-width package of the same stack (asymmetric grid,
+    stage widths `bits`): rrq_quantize_ex and all-prefix rrq_reconstruct_ex,
+    CUDA events after one warm-up.  Bytes: 2 + sum_k (b_k/8 + 8/g) per weight
+    to build; sum_k (b_k/8 + 8/g) + 2 S to reconstruct every prefix."""
+    from paper_2608_04048_gb300 import binding
+    S = len(bits)
+    pkgs = [binding.Package.empty(sp.rows, sp.cols, GROUP, S, mats[0].device, binding.GRID_ASYM,
+                                  binding.SCALE_F32, list(bits)) for sp in specs]
+    q_items = binding.quantize_descs(mats, pkgs)
+    outs = [o[:S] for o in p_outs]
+    r_items = binding.reconstruct_descs(pkgs, outs, S)
+    quant = lambda: binding.rrq_quantize_ex(mats, GROUP, S, binding.GRID_ASYM, binding.SCALE_F32,
+                                            pkgs, stream, q_items, bits=list(bits))
+    recon = lambda: binding.rrq_reconstruct_ex(pkgs, S, True, outs, stream, r_items)
+    quant(); recon()
+    ev = [torch.cuda.Event(enable_timing=True) for _ in range(3)]
+    ev[0].record(stream)
+    for _ in range(reps):
+        quant()
+    ev[1].record(stream)
+    for _ in range(reps):
+        recon()
+    ev[2].record(stream)
+    torch.cuda.synchronize()
+    if binding.rrq_get_device_status() != 0:
+        raise RuntimeError("a kernel reported a timeout (widths)")
+    q_s = ev[0].elapsed_time(ev[1]) / reps / 1e3
+    r_s = ev[1].elapsed_time(ev[2]) / reps / 1e3
+    per = sum(b / 8 + 8.0 / GROUP for b in bits)
+    n = sum(sp.numel for sp in specs)
+    hbm = measured_peaks()["hbm_gbs"]
+    del pkgs
+    return {"quantize_s_per_stack": round(q_s, 6), "quantize_alg_gbs": round(n * (2 + per) / q_s / 1e9, 1),
+            "quantize_frac_of_measured_hbm": round(n * (2 + per) / q_s / 1e9 / hbm, 4),
+            "reconstruct_prefixes_s": round(r_s, 6),
+            "reconstruct_prefixes_alg_gbs": round(n * (per + 2 * S) / r_s / 1e9, 1),
+            "reconstruct_frac_of_measured_hbm": round(n * (per + 2 * S) / r_s / 1e9 / hbm, 4)}
+
+
+def time_pmr(mats, specs, stream, reps: int = 5) -> dict:
+    """rrq_group_pmr over the stack (2 B per weight read, 4 B per group
+    written)."""
+    from paper_2608_04048_gb300 import binding
+    binding.rrq_group_pmr(mats, GROUP, stream)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        binding.rrq_group_pmr(mats, GROUP, stream)
+    b.record(stream)
+    torch.cuda.synchronize()
+    t = a.elapsed_time(b) / reps / 1e3
+    n = sum(sp.numel for sp in specs)
+    alg = n * (2 + 4.0 / GROUP)
+    return {"s_per_stack": round(t, 6), "alg_gbs": round(alg / t / 1e9, 1),
+            "frac_of_measured_hbm": round(alg / t / 1e9 / measured_peaks()["hbm_gbs"], 4)}
+
+
 def alg_bytes_reconstruct(n: int, k: int, g: int = GROUP) -> float:
     """Algorithmic bytes of one rrq_reconstruct at prefix k: k code planes and
     metadata read, bf16 written."""
@@ -364,6 +422,9 @@ def run_gpu(args, world, rank, local) -> dict | None:
     sym = time_sym_f16(mats, p_outs, specs, stream) if not args.no_sym else None
     from_base = time_from_base(mats, pkgs, specs, stream) if not args.no_sym else None
     gemv = time_gemv(pkgs, specs, stream) if not args.no_sym else None
+    bits = {"+".join(map(str, b)): time_bits(mats, p_outs, specs, stream, b) for b in ((1, 3), (3, 1))} \
+        if not args.no_sym else None
+    pmr = time_pmr(mats, specs, stream) if not args.no_sym else None
     e2e = run_e2e(args, mats, pkgs, p_outs, specs, stream, world) if not args.no_e2e else None
     if rank != 0:
         return None
@@ -421,6 +482,8 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "sym_f16": sym,
             "from_base": from_base,
             "gemv_decode": gemv,
+            "widths": bits,
+            "group_pmr": pmr,
         },
         "roofline": roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic,
                                    clock_summary.get("sm_mhz")),
