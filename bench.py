@@ -377,27 +377,30 @@ def run_gpu(args, world, rank, local) -> dict | None:
         for k in KS:
             binding.rrq_reconstruct_batch(pkgs, k, outs, stream=stream, items=r_items)
 
+    f_items = binding.quantize_prefixes_descs(mats, pkgs, p_outs)
+
+    def step():
+        # the package and its 2/4/6/8-bit reconstructions in one pass over W
+        binding.rrq_quantize_prefixes(mats, GROUP, STAGES, binding.GRID_ASYM, binding.SCALE_F32,
+                                      pkgs, p_outs, stream, f_items)
+
     for _ in range(args.warmup):
-        quantize_all()
-        reconstruct_all()
+        step()
     torch.cuda.synchronize()
     if binding.rrq_get_device_status() != 0:
         raise RuntimeError("a kernel reported a timeout during warm-up")
 
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True),
-           torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
     barrier(world)
     torch.cuda.synchronize()
     with ClockSampler(local) as clocks:
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record(stream)
-        for a, b, c in ev:
+        for a, b in ev:
             a.record(stream)
-            quantize_all()
+            step()
             b.record(stream)
-            reconstruct_all()
-            c.record(stream)
         t1.record(stream)
         torch.cuda.synchronize()
     barrier(world)
@@ -405,9 +408,21 @@ def run_gpu(args, world, rank, local) -> dict | None:
     if status != 0:
         raise RuntimeError(f"kernel status {status} in the timed region")
     elapsed_ms = t0.elapsed_time(t1)
-    q_ms = [a.elapsed_time(b) for a, b, _ in ev]
-    r_ms = [b.elapsed_time(c) for _, b, c in ev]
+    f_ms = [a.elapsed_time(b) for a, b in ev]
     elapsed_ms = max_over_ranks(elapsed_ms, world)
+
+    # the same outputs by two calls (package, then every prefix): breakdown only
+    def timed(fn, reps=3):
+        fn()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            fn()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps
+    q_ms = [timed(quantize_all)]
+    r_ms = [timed(reconstruct_all)]
 
     # separate rrq_reconstruct calls per k (context for the breakdown, not the step)
     reconstruct_each_k()
@@ -436,15 +451,16 @@ def run_gpu(args, world, rank, local) -> dict | None:
     value = world * bytes_bf16 / step_s / 1e9
     q_s = statistics.mean(q_ms) / 1e3
     r_s = statistics.mean(r_ms) / 1e3
+    f_s = statistics.mean(f_ms) / 1e3
+    f_alg = sum(alg_bytes_quantize(sp.numel) + STAGES * 2 * sp.numel for sp in specs)
     q_alg = sum(alg_bytes_quantize(sp.numel) for sp in specs)
     r_alg = sum(alg_bytes_prefixes(sp.numel, len(KS)) for sp in specs)
     r_each_alg = sum(alg_bytes_reconstruct(sp.numel, k) for sp in specs for k in KS)
     q_gbs = q_alg / q_s / 1e9
     r_gbs = r_alg / r_s / 1e9
-    dominant = "rrq_reconstruct_prefixes" if r_s > q_s else "rrq_quantize"
     per_launch = 64  # matrices per kernel launch of the batch entry points
-    launches = math.ceil(len(specs) / per_launch) * 2
-    traffic = recorded_traffic(dominant, q_alg / (launches / 2), r_alg / (launches / 2))
+    launches = math.ceil(len(specs) / per_launch)
+    traffic = recorded_traffic("rrq_quantize_prefixes", f_alg / launches, f_alg / launches)
     line = {
         "metric": METRIC,
         "value": round(value, 2),
@@ -460,13 +476,19 @@ def run_gpu(args, world, rank, local) -> dict | None:
         "data": "synthetic",
         "config": {
             "workload": WORKLOAD_TEXT.get(args.workload, args.workload),
-            "step": f"rrq_quantize_batch on all {len(specs)} matrices, then "
-                    f"rrq_reconstruct_prefixes_batch writing the k=1,2,3,4 reconstructions of all {len(specs)}",
+            "step": f"rrq_quantize_prefixes on all {len(specs)} matrices: the package and the "
+                    f"k=1,2,3,4 bf16 reconstructions of every matrix in one pass",
             "weights_per_rank": n_total,
             "l2": f"inputs {2 * n_total / 1e9:.2f} GB per rank, larger than the 126 MB L2; no flush",
             "parallelism": f"{world} independent rank(s), one stack each",
         },
         "breakdown": {
+            "step_alg_gbs": round(f_alg / f_s / 1e9, 1),
+            "step_frac_of_measured_hbm": round(f_alg / f_s / 1e9 / peaks["hbm_gbs"], 4),
+            "two_calls_s_per_stack": round(q_s + r_s, 6),
+            "two_calls_bf16_gbs": round(bytes_bf16 / (q_s + r_s) / 1e9, 2),
+            "quantize_alu_frac": round(n_total * STAGES * FP32_OPS_PER_WEIGHT_STAGE / q_s / 1e12
+                                       / fp32_peak_tops(clock_summary.get("sm_mhz")), 4),
             "quantize_s_per_stack": round(q_s, 6),
             "quantize_alg_gbs": round(q_gbs, 1),
             "quantize_bf16_in_gbs": round(bytes_bf16 / q_s / 1e9, 1),
@@ -485,8 +507,11 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "widths": bits,
             "group_pmr": pmr,
         },
-        "roofline": roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic,
-                                   clock_summary.get("sm_mhz")),
+        "roofline": {"kernel": "rrq_quantize_prefixes (quantize_kernel, build with prefixes)",
+                     "bound": "hbm", "achieved": round(f_alg / f_s / 1e9, 1), "peak": peaks["hbm_gbs"],
+                     "peak_source": f"{peaks['source']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
+                     "unit": "GB/s", "frac": round(f_alg / f_s / 1e9 / peaks["hbm_gbs"], 4),
+                     "alg_bytes_per_weight": 3.25 + 2 * STAGES, "traffic": traffic},
         "clocks": clock_summary,
         "gpu_launches": launches * args.steps,
         "e2e": e2e,
@@ -505,24 +530,6 @@ def fp32_peak_tops(sm_mhz: float | None) -> float:
     return 152 * 128 * (sm_mhz or 2070.0) * 1e6 / 1e12
 
 
-def roofline_entry(dominant, q_s, r_s, q_gbs, r_gbs, n_total, peaks, traffic, sm_mhz=None):
-    """Roofline of the dominant kernel.  Quantize needs 32 fp32 operations per
-    3.25 algorithmic bytes (9.8 op/B): above the GB300 ridge (fp32 peak / HBM
-    bandwidth = 40.7 T / 6.69 TB/s = 6.1 op/B), so its bound is the fp32 pipe
-    ("alu"); reconstruction is bound by HBM."""
-    if dominant == "rrq_quantize":
-        ops = n_total * STAGES * FP32_OPS_PER_WEIGHT_STAGE
-        achieved = ops / q_s / 1e12
-        peak = fp32_peak_tops(sm_mhz)
-        return {"kernel": dominant, "bound": "alu", "achieved": round(achieved, 2), "peak": round(peak, 2),
-                "peak_source": "derived: 152 SMs x 128 fp32 lanes x SM clock (fp32 operations)",
-                "unit": "Top/s", "frac": round(achieved / peak, 4),
-                "hbm_frac_of_measured": round(q_gbs / peaks["hbm_gbs"], 4), "traffic": traffic}
-    return {"kernel": dominant, "bound": "hbm", "achieved": round(r_gbs, 1), "peak": peaks["hbm_gbs"],
-            "peak_source": f"{peaks['source']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
-            "unit": "GB/s", "frac": round(r_gbs / peaks["hbm_gbs"], 4), "traffic": traffic}
-
-
 def recorded_traffic(kernel: str, q_bytes_per_launch: float, r_bytes_per_launch: float):
     """DRAM bytes per launch of `kernel` from the committed ncu summary
     (profiles/traffic.json), scaled to this workload's average launch by the
@@ -537,7 +544,7 @@ def recorded_traffic(kernel: str, q_bytes_per_launch: float, r_bytes_per_launch:
     if not entry or kernel not in KERNEL_SOURCES or entry.get("source_sha256") != kernel_source_hash(kernel):
         return None
     per_alg = entry["dram_bytes"] / entry["alg_bytes"]
-    alg = q_bytes_per_launch if kernel == "rrq_quantize" else r_bytes_per_launch
+    alg = r_bytes_per_launch if kernel == "rrq_reconstruct_prefixes" else q_bytes_per_launch
     return round(per_alg * alg)
 
 
@@ -547,6 +554,7 @@ KERNEL_SOURCES = {
     "rrq_quantize_ex_sym_f16": ["quantize_kernel.cuh", "quantize.cu"],
     "rrq_reconstruct_prefixes": ["reconstruct_kernel.cuh", "reconstruct_asym_f32.cu"],
     "rrq_reconstruct_ex_sym_f16": ["reconstruct_kernel.cuh", "reconstruct_sym_f16.cu"],
+    "rrq_quantize_prefixes": ["quantize_kernel.cuh", "quantize_emit.cu"],
     "rrq_gemv_k1": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
     "rrq_gemv_k4": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
 }
@@ -566,9 +574,10 @@ def kernel_source_hash(kernel: str) -> str:
 
 def run_e2e(args, mats, pkgs, p_outs, specs, stream, world) -> dict:
     """Same metric through the public API with host buffers: every step copies
-    each matrix from pinned host memory to the device, builds its package,
-    copies the package back, reconstructs every prefix k=1..4 and copies each
-    result back to a pinned host buffer, all inside the timed region."""
+    each matrix from pinned host memory to the device, builds its package and
+    its k=1..4 reconstructions (rrq_quantize_prefixes), and copies the package
+    and every reconstruction back to pinned host buffers, all inside the timed
+    region."""
     from paper_2608_04048_gb300 import binding
     def pinned_like(t):
         h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
@@ -583,17 +592,16 @@ def run_e2e(args, mats, pkgs, p_outs, specs, stream, world) -> dict:
     d2h = sum(t.numel() * t.element_size() for p in host_pkg for t in p) + \
         len(KS) * sum(sp.numel * 2 for sp in specs)
 
-    q_items = binding.quantize_items(mats, pkgs)
-    p_items = binding.prefixes_items(pkgs, p_outs, len(KS))
+    f_items = binding.quantize_prefixes_descs(mats, pkgs, p_outs)
 
     def step():
         for W, h in zip(mats, host_W):
             W.copy_(h, non_blocking=True)
-        binding.rrq_quantize_batch(mats, pkgs, GROUP, STAGES, stream=stream, items=q_items)
+        binding.rrq_quantize_prefixes(mats, GROUP, STAGES, binding.GRID_ASYM, binding.SCALE_F32,
+                                      pkgs, p_outs, stream, f_items)
         for i, pkg in enumerate(pkgs):
             for h, d in zip(host_pkg[i], pkg.codes + pkg.scales + pkg.zeros):
                 h.copy_(d, non_blocking=True)
-        binding.rrq_reconstruct_prefixes_batch(pkgs, len(KS), p_outs, stream=stream, items=p_items)
         for outs_i in p_outs:
             for o in outs_i:
                 host_out[:o.numel()].view(o.shape).copy_(o, non_blocking=True)

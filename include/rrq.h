@@ -240,6 +240,29 @@ typedef struct {
 rrq_status rrq_quantize_ex(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
                            rrq_stream_t stream);
 
+/* One matrix of rrq_quantize_prefixes: rrq_quantize_desc plus the outputs
+ * for the reconstruction after every stage. */
+typedef struct {
+  const uint16_t* W_bf16;                /* device, bf16 [rows, cols], 16-byte aligned */
+  int64_t rows, cols;
+  uint8_t* codes[RRQ_MAX_STAGES];
+  void* scales[RRQ_MAX_STAGES];
+  float* zeros[RRQ_MAX_STAGES];          /* RRQ_GRID_ASYM only */
+  uint16_t* out_bf16[RRQ_MAX_STAGES];    /* out_bf16[j]: prefix with j+1 stages, bf16 [rows, cols],
+                                            16-byte aligned; first n_stages entries used */
+} rrq_quantize_prefixes_desc;
+
+/* Build the package and its reconstructions in one pass (Algorithm 1 without
+ * a base checkpoint with Eq. 8 at every prefix): the same package as
+ * rrq_quantize_ex, and out_bf16[j] the same bits as rrq_reconstruct_ex at
+ * prefix j+1 on it -- the stage levels the construction computes are the
+ * values the reconstruction sums, so the 2/4/6/8-bit weights come with the
+ * package from one read of W (11.25 B per weight moved at group 128 with 4
+ * stages, against 12.5 B for the two calls).  Formats: any with 2-bit
+ * stages.  No output may overlap any input or output of the batch. */
+rrq_status rrq_quantize_prefixes(const rrq_quantize_prefixes_desc* items, int count,
+                                 const rrq_format* fmt, rrq_stream_t stream);
+
 /* Algorithm 1 with a base checkpoint (Section 3.2: the construction can start
  * from an existing low-bit checkpoint by skipping the base quantization):
  * stage 0 of every item's package is an INPUT in format *fmt -- codes[0],

@@ -23,7 +23,7 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
 EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
            "rrq_reconstruct_prefixes", "rrq_reconstruct_prefixes_batch",
            "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_gemv",
-           "rrq_stage_codes_bytes", "rrq_group_pmr", "rrq_scales_bytes", "rrq_package_bytes_ex",
+           "rrq_stage_codes_bytes", "rrq_group_pmr", "rrq_quantize_prefixes", "rrq_scales_bytes", "rrq_package_bytes_ex",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
            "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
@@ -63,6 +63,13 @@ class PmrDesc(ctypes.Structure):
     """rrq_pmr_desc of include/rrq.h"""
     _fields_ = [("W_bf16", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
                 ("pmr", ctypes.c_void_p), ("stats", ctypes.c_void_p)]
+
+
+class QuantizePrefixesDesc(ctypes.Structure):
+    """rrq_quantize_prefixes_desc of include/rrq.h"""
+    _fields_ = [("W_bf16", ctypes.c_void_p), ("rows", ctypes.c_int64), ("cols", ctypes.c_int64),
+                ("codes", ctypes.c_void_p * MAX_STAGES), ("scales", ctypes.c_void_p * MAX_STAGES),
+                ("zeros", ctypes.c_void_p * MAX_STAGES), ("out_bf16", ctypes.c_void_p * MAX_STAGES)]
 
 
 class ReconstructDesc(ctypes.Structure):
@@ -134,6 +141,8 @@ def load_library():
     fmt_p = ctypes.POINTER(Format)
     lib.rrq_quantize_ex.argtypes = [ctypes.POINTER(QuantizeDesc), i32, fmt_p, vp]
     lib.rrq_quantize_ex.restype = i32
+    lib.rrq_quantize_prefixes.argtypes = [ctypes.POINTER(QuantizePrefixesDesc), i32, fmt_p, vp]
+    lib.rrq_quantize_prefixes.restype = i32
     lib.rrq_quantize_from_base.argtypes = [ctypes.POINTER(QuantizeDesc), i32, fmt_p, vp]
     lib.rrq_quantize_from_base.restype = i32
     lib.rrq_gemv.argtypes = [ctypes.POINTER(GemvDesc), i32, fmt_p, i32, i32, vp]
@@ -395,6 +404,43 @@ def rrq_quantize_ex(mats, group: int = 128, n_stages: int = 4, grid: int = GRID_
     if rc != 0:
         raise RRQError(rc, "rrq_quantize_ex")
     return pkgs
+
+
+def quantize_prefixes_descs(mats, pkgs, outs) -> ctypes.Array:
+    """Host array of rrq_quantize_prefixes_desc; outs[i][j] is matrix i's
+    prefix with j+1 stages (bf16, the matrix's shape)."""
+    items = (QuantizePrefixesDesc * len(mats))()
+    for it, W, pkg, o in zip(items, mats, pkgs, outs):
+        if W.dtype != torch.bfloat16 or W.dim() != 2 or not W.is_cuda or not W.is_contiguous():
+            raise TypeError("every W must be a contiguous 2-D bfloat16 CUDA tensor")
+        it.W_bf16 = W.data_ptr()
+        it.rows, it.cols = W.shape
+        for k in range(pkg.n_stages):
+            it.codes[k] = pkg.codes[k].data_ptr()
+            it.scales[k] = pkg.scales[k].data_ptr()
+            it.zeros[k] = pkg.zeros[k].data_ptr() if pkg.zeros else None
+            if o[k].dtype != torch.bfloat16 or not o[k].is_cuda or not o[k].is_contiguous():
+                raise TypeError("outputs must be contiguous bfloat16 CUDA tensors")
+            it.out_bf16[k] = o[k].data_ptr()
+    return items
+
+
+def rrq_quantize_prefixes(mats, group: int = 128, n_stages: int = 4, grid: int = GRID_ASYM,
+                          scale_type: int = SCALE_F32, pkgs=None, outs=None, stream=None, items=None):
+    """Package of each matrix and its bf16 reconstruction after every stage,
+    in one pass: returns (pkgs, outs) with outs[i][j] = prefix j+1."""
+    lib = load_library()
+    if pkgs is None:
+        pkgs = [Package.empty(W.shape[0], W.shape[1], group, n_stages, W.device, grid, scale_type) for W in mats]
+    if outs is None:
+        outs = [_new_outs(p, n_stages) for p in pkgs]
+    if items is None:
+        items = quantize_prefixes_descs(mats, pkgs, outs)
+    fmt = Format(group, n_stages, grid, scale_type)
+    rc = lib.rrq_quantize_prefixes(items, len(items), ctypes.byref(fmt), _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_quantize_prefixes")
+    return pkgs, outs
 
 
 def rrq_quantize_from_base(mats, pkgs, stream=None, items=None):

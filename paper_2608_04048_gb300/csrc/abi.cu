@@ -53,6 +53,7 @@ rrq_status current_device(int* dev_out, DeviceState** state) {
     d.status = static_cast<unsigned*>(addr);
     if ((e = rrq::quantize_prepare())) return fail_cuda(e);
     if ((e = rrq::quantize_prepare_base())) return fail_cuda(e);
+    if ((e = rrq::quantize_prepare_emit())) return fail_cuda(e);
     if ((e = rrq::reconstruct_prepare())) return fail_cuda(e);
     d.ready = true;
   }
@@ -164,7 +165,47 @@ Fmt asym_format(int group, int n_stages) {
 // ---------------------------------------------------------------------------
 // quantize
 // ---------------------------------------------------------------------------
-rrq_status check_quantize_item(const rrq_quantize_desc& it, const Fmt& f) {
+// A quantize request for one matrix, from either descriptor type; out is
+// all-null except for the build with prefixes.
+struct QView {
+  const uint16_t* W_bf16;
+  int64_t rows, cols;
+  uint8_t* codes[RRQ_MAX_STAGES];
+  void* scales[RRQ_MAX_STAGES];
+  float* zeros[RRQ_MAX_STAGES];
+  uint16_t* out[RRQ_MAX_STAGES];
+};
+
+QView view_of(const rrq_quantize_desc& d) {
+  QView v{};
+  v.W_bf16 = d.W_bf16;
+  v.rows = d.rows;
+  v.cols = d.cols;
+  for (int k = 0; k < RRQ_MAX_STAGES; ++k) {
+    v.codes[k] = d.codes[k];
+    v.scales[k] = d.scales[k];
+    v.zeros[k] = d.zeros[k];
+  }
+  return v;
+}
+
+QView view_of(const rrq_quantize_prefixes_desc& d) {
+  QView v{};
+  v.W_bf16 = d.W_bf16;
+  v.rows = d.rows;
+  v.cols = d.cols;
+  for (int k = 0; k < RRQ_MAX_STAGES; ++k) {
+    v.codes[k] = d.codes[k];
+    v.scales[k] = d.scales[k];
+    v.zeros[k] = d.zeros[k];
+    v.out[k] = d.out_bf16[k];
+  }
+  return v;
+}
+
+enum QMode { kBuild, kFromBase, kEmit };
+
+rrq_status check_quantize_item(const QView& it, const Fmt& f, QMode mode) {
   if (!it.W_bf16 || !shape_ok(it.rows, it.cols)) return RRQ_ERR_INVALID_ARG;
   if (it.cols % f.group != 0) return RRQ_ERR_INVALID_ARG;
   for (int k = 0; k < f.n_stages; ++k)
@@ -173,13 +214,22 @@ rrq_status check_quantize_item(const rrq_quantize_desc& it, const Fmt& f) {
   for (int k = 0; k < f.n_stages; ++k)
     if (!aligned(it.codes[k], 16) || !aligned(it.scales[k], 16) || (!f.sym() && !aligned(it.zeros[k], 16)))
       return RRQ_ERR_MISALIGNED;
+  if (mode == kEmit) {
+    for (int k = 0; k < f.n_stages; ++k)
+      if (!it.out[k]) return RRQ_ERR_INVALID_ARG;
+    for (int k = 0; k < f.n_stages; ++k)
+      if (!aligned(it.out[k], 16)) return RRQ_ERR_MISALIGNED;
+  }
   return RRQ_OK;
 }
 
-// from_base: stage 0 is an input (Algorithm 1 with a base checkpoint).
-void add_quantize_ranges(const rrq_quantize_desc& it, const Fmt& f, bool from_base, std::vector<Range>& r) {
+// kFromBase: stage 0 is an input (Algorithm 1 with a base checkpoint).
+void add_quantize_ranges(const QView& it, const Fmt& f, QMode mode, std::vector<Range>& r) {
+  const bool from_base = mode == kFromBase;
   const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
   r.push_back(range_of(it.W_bf16, 2 * n, false));
+  if (mode == kEmit)
+    for (int k = 0; k < f.n_stages; ++k) r.push_back(range_of(it.out[k], 2 * n, true));
   for (int k = 0; k < f.n_stages; ++k) {
     const bool out = !(from_base && k == 0);
     r.push_back(range_of(it.codes[k], f.code_bytes(n, k), out));
@@ -188,17 +238,17 @@ void add_quantize_ranges(const rrq_quantize_desc& it, const Fmt& f, bool from_ba
   }
 }
 
-rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& f, rrq_stream_t stream,
-                          bool from_base = false) {
+rrq_status quantize_batch(const QView* items, int count, const Fmt& f, rrq_stream_t stream, QMode mode) {
   if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  const bool from_base = mode == kFromBase;
   if (from_base && f.n_stages < 2) return RRQ_ERR_INVALID_ARG;
-  if (from_base && f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
+  if (mode != kBuild && f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
   const int n_stages = f.n_stages;
   std::vector<Range> ranges;
-  ranges.reserve(static_cast<size_t>(count) * (1 + 3 * n_stages));
+  ranges.reserve(static_cast<size_t>(count) * (1 + 4 * n_stages));
   for (int i = 0; i < count; ++i) {
-    if (rrq_status rc = check_quantize_item(items[i], f)) return rc;
-    add_quantize_ranges(items[i], f, from_base, ranges);
+    if (rrq_status rc = check_quantize_item(items[i], f, mode)) return rc;
+    add_quantize_ranges(items[i], f, mode, ranges);
   }
   if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
 
@@ -206,8 +256,11 @@ rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& 
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
   for (int i = 0; i < count; ++i) {
-    const rrq_quantize_desc& it = items[i];
+    const QView& it = items[i];
     if (!on_device(it.W_bf16, dev)) return RRQ_ERR_INVALID_ARG;
+    if (mode == kEmit)
+      for (int k = 0; k < n_stages; ++k)
+        if (!on_device(it.out[k], dev)) return RRQ_ERR_INVALID_ARG;
     for (int k = 0; k < n_stages; ++k)
       if (!on_device(it.codes[k], dev) || !on_device(it.scales[k], dev) ||
           (!f.sym() && !on_device(it.zeros[k], dev)))
@@ -226,7 +279,7 @@ rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& 
     p.status = st->status;
     int64_t chunks = 0;
     for (int i = 0; i < m; ++i) {
-      const rrq_quantize_desc& it = items[base + i];
+      const QView& it = items[base + i];
       rrq::QuantizeItem& q = p.item[i];
       q.W = it.W_bf16;
       q.n = it.rows * it.cols;
@@ -237,12 +290,14 @@ rrq_status quantize_batch(const rrq_quantize_desc* items, int count, const Fmt& 
         q.codes[k] = it.codes[kk];
         q.scales[k] = it.scales[kk];
         q.zeros[k] = f.sym() ? nullptr : it.zeros[kk];
+        q.out[k] = mode == kEmit ? it.out[kk] : nullptr;
       }
     }
     p.total_chunks = chunks;
     const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
-    cudaError_t e = from_base ? rrq::quantize_launch_base(f.group, f.kind, p, s, st->sms)
-                              : rrq::quantize_launch(f.group, f.kind, p, s, st->sms);
+    cudaError_t e = mode == kFromBase ? rrq::quantize_launch_base(f.group, f.kind, p, s, st->sms)
+                    : mode == kEmit   ? rrq::quantize_launch_emit(f.group, f.kind, p, s, st->sms)
+                                      : rrq::quantize_launch(f.group, f.kind, p, s, st->sms);
     if (e != cudaSuccess) return fail_cuda(e);
   }
   return RRQ_OK;
@@ -492,6 +547,16 @@ rrq_status pmr_batch(const rrq_pmr_desc* items, int count, int group, rrq_stream
   return RRQ_OK;
 }
 
+template <typename Desc>
+rrq_status quantize_descs(const Desc* items, int count, const rrq_format* fmt, rrq_stream_t stream, QMode mode) {
+  Fmt f;
+  if (rrq_status rc = parse_format(fmt, &f)) return rc;
+  if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
+  std::vector<QView> v(static_cast<size_t>(count));
+  for (int i = 0; i < count; ++i) v[i] = view_of(items[i]);
+  return quantize_batch(v.data(), count, f, stream, mode);
+}
+
 }  // namespace
 
 extern "C" {
@@ -523,7 +588,7 @@ rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int 
   if (!out_codes || !out_scales || !out_zeros || n_stages < 1 || n_stages > RRQ_MAX_STAGES)
     return RRQ_ERR_INVALID_ARG;
   if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
-  rrq_quantize_desc it{};
+  QView it{};
   it.W_bf16 = W_bf16;
   it.rows = rows;
   it.cols = cols;
@@ -532,15 +597,16 @@ rrq_status rrq_quantize(const uint16_t* W_bf16, int64_t rows, int64_t cols, int 
     it.scales[k] = out_scales[k];
     it.zeros[k] = out_zeros[k];
   }
-  return quantize_batch(&it, 1, asym_format(group, n_stages), stream);
+  return quantize_batch(&it, 1, asym_format(group, n_stages), stream, kBuild);
 }
 
 rrq_status rrq_quantize_batch(const rrq_quantize_item* items, int count, int group, int n_stages,
                               rrq_stream_t stream) {
   if (!items || count < 1 || n_stages < 1 || n_stages > RRQ_MAX_STAGES) return RRQ_ERR_INVALID_ARG;
   if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
-  std::vector<rrq_quantize_desc> d(static_cast<size_t>(count));
+  std::vector<QView> d(static_cast<size_t>(count));
   for (int i = 0; i < count; ++i) {
+    d[i] = QView{};
     d[i].W_bf16 = items[i].W_bf16;
     d[i].rows = items[i].rows;
     d[i].cols = items[i].cols;
@@ -550,14 +616,17 @@ rrq_status rrq_quantize_batch(const rrq_quantize_item* items, int count, int gro
       d[i].zeros[k] = items[i].zeros[k];
     }
   }
-  return quantize_batch(d.data(), count, asym_format(group, n_stages), stream);
+  return quantize_batch(d.data(), count, asym_format(group, n_stages), stream, kBuild);
 }
 
 rrq_status rrq_quantize_ex(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
                            rrq_stream_t stream) {
-  Fmt f;
-  if (rrq_status rc = parse_format(fmt, &f)) return rc;
-  return quantize_batch(items, count, f, stream);
+  return quantize_descs(items, count, fmt, stream, kBuild);
+}
+
+rrq_status rrq_quantize_prefixes(const rrq_quantize_prefixes_desc* items, int count, const rrq_format* fmt,
+                                 rrq_stream_t stream) {
+  return quantize_descs(items, count, fmt, stream, kEmit);
 }
 
 rrq_status rrq_reconstruct(const uint8_t* const codes[], const float* const scales[],
@@ -614,9 +683,7 @@ rrq_status rrq_reconstruct_prefixes_batch(const rrq_prefixes_item* items, int co
 
 rrq_status rrq_quantize_from_base(const rrq_quantize_desc* items, int count, const rrq_format* fmt,
                                   rrq_stream_t stream) {
-  Fmt f;
-  if (rrq_status rc = parse_format(fmt, &f)) return rc;
-  return quantize_batch(items, count, f, stream, true);
+  return quantize_descs(items, count, fmt, stream, kFromBase);
 }
 
 rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,

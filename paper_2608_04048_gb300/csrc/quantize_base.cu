@@ -5,11 +5,11 @@
 
 namespace rrq {
 
-cudaError_t quantize_prepare_base() { return prepare_all<true>(); }
+cudaError_t quantize_prepare_base() { return prepare_all<kModeBase>(); }
 
 cudaError_t quantize_launch_base(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream,
                                  int sms) {
-  return launch_all<true>(group, fmt, p, stream, sms);
+  return launch_all<kModeBase>(group, fmt, p, stream, sms);
 }
 
 }  // namespace rrq

@@ -79,10 +79,19 @@
 // b*c.., so a lane's 32 weights fill b words; for this format the lane reads
 // its shared-memory pieces in natural order.
 //
+// Build with prefixes (kModeEmit): the stage levels the build computes are
+// exactly the values the reconstruction sums (fl(lo + fl(Q s)), or (Q-2) s),
+// so the kernel also keeps the binary32 prefix sums acc = L_0,
+// acc = fl(acc + L_k) in registers and writes the bf16 reconstruction after
+// every stage -- the package and its 2/4/6/8-bit weights in one pass over W,
+// bit-identical to rrq_reconstruct on the package.
+//
 // This header holds the kernel template; quantize.cu instantiates the build
-// without a base checkpoint, quantize_base.cu the build from one.
+// without a base checkpoint, quantize_base.cu the build from one,
+// quantize_emit.cu the build that also writes every prefix.
 #pragma once
 
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
 #include "rrq_device.cuh"
@@ -133,16 +142,25 @@ __device__ __forceinline__ int exact_code(float v, float lo, float s) {
   return q > 3 ? 3 : q;
 }
 struct ExactPair {
-  f32x2 w;
+  f32x2 w;         // residuals
+  f32x2 l;         // stage levels
   uint32_t q0, q1;
+};
+
+// What a launch computes.
+enum Mode : int {
+  kModeBuild = 0,  // every stage from W (Algorithm 1, no base checkpoint)
+  kModeBase = 1,   // stage 0 given, stages 1.. from R_0 = W - W_0
+  kModeEmit = 2,   // every stage from W, plus the bf16 reconstruction after every stage
 };
 __device__ __noinline__ ExactPair exact_pair(f32x2 v, float lo, float s) {
   float a, b;
   unpack2(v, a, b);
   const int qa = exact_code(a, lo, s), qb = exact_code(b, lo, s);
-  const float wa = __fsub_rn(a, __fadd_rn(lo, __fmul_rn(__int2float_rn(qa), s)));
-  const float wb = __fsub_rn(b, __fadd_rn(lo, __fmul_rn(__int2float_rn(qb), s)));
-  return {pack2(wa, wb), static_cast<uint32_t>(qa), static_cast<uint32_t>(qb)};
+  const float la = __fadd_rn(lo, __fmul_rn(__int2float_rn(qa), s));
+  const float lb = __fadd_rn(lo, __fmul_rn(__int2float_rn(qb), s));
+  return {pack2(__fsub_rn(a, la), __fsub_rn(b, lb)), pack2(la, lb), static_cast<uint32_t>(qa),
+          static_cast<uint32_t>(qb)};
 }
 
 // Symmetric grid, per-element IEEE-division path.
@@ -156,9 +174,9 @@ __device__ __noinline__ ExactPair exact_pair_sym(f32x2 v, float s) {
   float a, b;
   unpack2(v, a, b);
   const int qa = exact_code_sym(a, s), qb = exact_code_sym(b, s);
-  const float wa = __fsub_rn(a, __fmul_rn(__int2float_rn(qa - 2), s));
-  const float wb = __fsub_rn(b, __fmul_rn(__int2float_rn(qb - 2), s));
-  return {pack2(wa, wb), static_cast<uint32_t>(qa), static_cast<uint32_t>(qb)};
+  const float la = __fmul_rn(__int2float_rn(qa - 2), s), lb = __fmul_rn(__int2float_rn(qb - 2), s);
+  return {pack2(__fsub_rn(a, la), __fsub_rn(b, lb)), pack2(la, lb), static_cast<uint32_t>(qa),
+          static_cast<uint32_t>(qb)};
 }
 
 // Scales for which the corrected quotient is proven exact (see the file
@@ -191,9 +209,10 @@ __device__ __noinline__ ExactPair exact_pair_bits(f32x2 v, float lo, float s, in
     qa = qa < 0 ? 0 : (qa > m ? m : qa);
     qb = qb < 0 ? 0 : (qb > m ? m : qb);
   }
-  const float wa = __fsub_rn(a, __fadd_rn(lo, __fmul_rn(__int2float_rn(qa), s)));
-  const float wb = __fsub_rn(b, __fadd_rn(lo, __fmul_rn(__int2float_rn(qb), s)));
-  return {pack2(wa, wb), static_cast<uint32_t>(qa), static_cast<uint32_t>(qb)};
+  const float la = __fadd_rn(lo, __fmul_rn(__int2float_rn(qa), s));
+  const float lb = __fadd_rn(lo, __fmul_rn(__int2float_rn(qb), s));
+  return {pack2(__fsub_rn(a, la), __fsub_rn(b, lb)), pack2(la, lb), static_cast<uint32_t>(qa),
+          static_cast<uint32_t>(qb)};
 }
 
 constexpr float kTieMargin = 0.5f - 0x1p-17f;  // |q - rhe(q)| beyond this: near a half-integer
@@ -405,13 +424,37 @@ __device__ __forceinline__ void subtract_base(f32x2 (&v)[16], const BaseWords& b
   }
 }
 
-template <int G, bool kBase>
+// bf16 of the prefix sums of this lane's 32 weights (slot order), each 16-byte
+// piece stored at its place in memory (slot j holds piece (j + rot) & 3).
+__device__ __forceinline__ void emit_prefix(uint16_t* out, int64_t e0, const f32x2 (&w)[16], int rot) {
+#pragma unroll
+  for (int j = 0; j < 4; ++j) {
+    uint32_t h[4];
+#pragma unroll
+    for (int m = 0; m < 4; ++m) {
+      float a, b;
+      unpack2(w[4 * j + m], a, b);
+      const __nv_bfloat162 x = __floats2bfloat162_rn(a, b);
+      h[m] = *reinterpret_cast<const uint32_t*>(&x);
+    }
+    __stcs(reinterpret_cast<uint4*>(out + e0 + 8 * ((j + rot) & 3)), make_uint4(h[0], h[1], h[2], h[3]));
+  }
+}
+
+template <int G, int M>
 __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, const QuantizeItem& it,
                                                     int64_t e0, int lane, uint4 (&raw)[4],
                                                     uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
-                                                    uint32_t ld_lo, uint32_t ld_hi) {
+                                                    uint32_t ld_lo, uint32_t ld_hi, int rot) {
+  constexpr bool kBase = M == kModeBase;
+  constexpr bool kEmit = M == kModeEmit;
   constexpr int L = G / 32;  // lanes per group
   const bool valid = e0 < it.n;
+  // prefix sums (kModeEmit), starting at -0: fl(-0 + x) = x for every x,
+  // including both zeros, so the first stage needs no special case
+  f32x2 wsum[kEmit ? 16 : 1];
+#pragma unroll
+  for (int i = 0; i < (kEmit ? 16 : 1); ++i) wsum[i] = pack2(-0.0f, -0.0f);
   if (!valid) {
 #pragma unroll
     for (int j = 0; j < 4; ++j) raw[j] = make_uint4(0u, 0u, 0u, 0u);
@@ -463,7 +506,9 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
         const f32x2 q = fma2(d, RH, mul2(d, RL));  // d/s to 2^-45.3
         const f32x2 t = add2(q, T23);              // 2^23 + rhe(q)
         const f32x2 step = fma2(t, S, C);    // fl(Q*s)
-        v[i] = sub2(v[i], add2(LO, step));   // v - fl(lo + fl(Q*s))
+        const f32x2 lv = add2(LO, step);     // fl(lo + fl(Q*s))
+        v[i] = sub2(v[i], lv);               // v - fl(lo + fl(Q*s))
+        if constexpr (kEmit) wsum[i] = add2(wsum[i], lv);
         acc[i >> 2] = push_code(push_code(acc[i >> 2], static_cast<uint32_t>(t)),
                                 static_cast<uint32_t>(t >> 32));
         float a, b;
@@ -481,6 +526,7 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
       for (int i = 0; i < 16; ++i) {
         const ExactPair x = exact_pair(v[i], lo, s);
         v[i] = x.w;
+        if constexpr (kEmit) wsum[i] = add2(wsum[i], x.l);
         acc[i >> 2] = push_code(push_code(acc[i >> 2], x.q0), x.q1);
       }
       lane_minmax(v, mn0, mx0);
@@ -492,6 +538,7 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
         __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s);
         __stcs(it.zeros[k] + e0 / G, lo);
       }
+      if constexpr (kEmit) emit_prefix(it.out[k], e0, wsum, rot);
     }
     if (k + 1 < p.n_stages) {  // range of the residual = next stage's lo, hi
       lo = fminf(mn0, mn1);
@@ -503,13 +550,20 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
 
 // Symmetric grid; kF16: the scale is rounded to binary16, stored as such, and
 // the stage quantizes against the rounded value.
-template <int G, bool kF16, bool kBase>
+template <int G, bool kF16, int M>
 __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const QuantizeItem& it,
                                                    int64_t e0, int lane, uint4 (&raw)[4],
                                                    uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
-                                                   uint32_t ld_lo, uint32_t ld_hi) {
+                                                   uint32_t ld_lo, uint32_t ld_hi, int rot) {
+  constexpr bool kBase = M == kModeBase;
+  constexpr bool kEmit = M == kModeEmit;
   constexpr int L = G / 32;  // lanes per group
   const bool valid = e0 < it.n;
+  // prefix sums (kModeEmit), starting at -0: fl(-0 + x) = x for every x,
+  // including both zeros, so the first stage needs no special case
+  f32x2 wsum[kEmit ? 16 : 1];
+#pragma unroll
+  for (int i = 0; i < (kEmit ? 16 : 1); ++i) wsum[i] = pack2(-0.0f, -0.0f);
   if (!valid) {
 #pragma unroll
     for (int j = 0; j < 4; ++j) raw[j] = make_uint4(0u, 0u, 0u, 0u);
@@ -538,7 +592,7 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
     if (fast) {
       float r_hi = 0.0f, r_lo = 0.0f;
       if (s > 0.0f) recip2(s, r_hi, r_lo);
-      const f32x2 RH = pack2(r_hi, r_hi), RL = pack2(r_lo, r_lo), NS = pack2(-s, -s);
+      const f32x2 RH = pack2(r_hi, r_hi), RL = pack2(r_lo, r_lo), NS = pack2(-s, -s), S = pack2(s, s);
       const f32x2 C = pack2(kSymRound, kSymRound);
 #pragma unroll
       for (int i = 0; i < 16; ++i) {
@@ -548,6 +602,7 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
         const f32x2 t = add2(pack2(fminf(qa, 1.0f), fminf(qb, 1.0f)), C);  // C + rhe, clamped
         const f32x2 u = sub2(t, C);                                       // Q - 2, exact
         v[i] = fma2(u, NS, v[i]);                                         // v - (Q-2) s
+        if constexpr (kEmit) wsum[i] = fma2(u, S, wsum[i]);  // + (Q-2) s, exact product
         acc[i >> 2] = push_code(push_code(acc[i >> 2], static_cast<uint32_t>(t)),
                                 static_cast<uint32_t>(t >> 32));
         float a, b;
@@ -560,6 +615,7 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
       for (int i = 0; i < 16; ++i) {
         const ExactPair x = exact_pair_sym(v[i], s);
         v[i] = x.w;
+        if constexpr (kEmit) wsum[i] = add2(wsum[i], x.l);
         acc[i >> 2] = push_code(push_code(acc[i >> 2], x.q0), x.q1);
       }
       mx0 = lane_amax(v);
@@ -571,28 +627,31 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
         if (kF16) stcs_u16(static_cast<uint16_t*>(it.scales[k]) + e0 / G, s16);
         else __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s);
       }
+      if constexpr (kEmit) emit_prefix(it.out[k], e0, wsum, rot);
     }
     if (k + 1 < p.n_stages) amax = group_max<L>(fmaxf(mx0, mx1));
   }
 }
 
-template <int G, int F, bool kBase>
+template <int G, int F, int M>
 __device__ __forceinline__ void quantize_chunk(const QuantizeBatch& p, const QuantizeItem& it,
                                                int64_t e0, int lane, uint4 (&raw)[4],
                                                uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
-                                               uint32_t ld_lo, uint32_t ld_hi) {
+                                               uint32_t ld_lo, uint32_t ld_hi, int rot) {
   if constexpr (F == kAsymF32)
-    quantize_chunk_asym<G, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
+    quantize_chunk_asym<G, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot);
   else if constexpr (F == kAsymBits)
     quantize_chunk_bits<G>(p, it, e0, lane, raw);
   else
-    quantize_chunk_sym<G, F == kSymF16, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
+    quantize_chunk_sym<G, F == kSymF16, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot);
 }
 
-// (the width-generic stages need more registers: two CTAs per SM)
-template <int G, int F, bool kBase>
-__global__ void __launch_bounds__(kThreads, F == kAsymBits ? 2 : RRQ_QUANTIZE_CTAS_PER_SM)
+// (the width-generic stages and the prefix sums need more registers: two
+// CTAs per SM)
+template <int G, int F, int M>
+__global__ void __launch_bounds__(kThreads, (F == kAsymBits || M == kModeEmit) ? 2 : RRQ_QUANTIZE_CTAS_PER_SM)
 quantize_kernel(const __grid_constant__ QuantizeBatch p) {
+  constexpr bool kBase = M == kModeBase;
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -686,67 +745,67 @@ quantize_kernel(const __grid_constant__ QuantizeBatch p) {
     const int64_t e0 = (chunk - it.chunk_begin) * kChunkElems + static_cast<int64_t>(lane) * kLaneElems;
     const BaseWords bw = bw_next;
     if (kBase) bw_next = base_of(chunk + stride);  // in flight while this chunk computes
-    quantize_chunk<G, F, kBase>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi);
+    quantize_chunk<G, F, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot);
   }
 }
 
-template <int G, int F, bool kBase>
+template <int G, int F, int M>
 cudaError_t launch_gf(const QuantizeBatch& p, cudaStream_t stream, int sms) {
   static int blocks_per_sm = 0;  // same for every device of this build
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, quantize_kernel<G, F, kBase>, kThreads, kSmemBytes);
+        &blocks_per_sm, quantize_kernel<G, F, M>, kThreads, kSmemBytes);
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
   const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  quantize_kernel<G, F, kBase><<<grid, kThreads, kSmemBytes, stream>>>(p);
+  quantize_kernel<G, F, M><<<grid, kThreads, kSmemBytes, stream>>>(p);
   return cudaGetLastError();
 }
 
-template <int F, bool kBase>
+template <int F, int M>
 cudaError_t launch_f(int group, const QuantizeBatch& p, cudaStream_t stream, int sms) {
   switch (group) {
-    case 32: return launch_gf<32, F, kBase>(p, stream, sms);
-    case 64: return launch_gf<64, F, kBase>(p, stream, sms);
-    case 128: return launch_gf<128, F, kBase>(p, stream, sms);
-    case 256: return launch_gf<256, F, kBase>(p, stream, sms);
+    case 32: return launch_gf<32, F, M>(p, stream, sms);
+    case 64: return launch_gf<64, F, M>(p, stream, sms);
+    case 128: return launch_gf<128, F, M>(p, stream, sms);
+    case 256: return launch_gf<256, F, M>(p, stream, sms);
     default: return cudaErrorInvalidValue;
   }
 }
 
-template <int F, bool kBase>
+template <int F, int M>
 cudaError_t prepare_f() {
   cudaError_t e;
   const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-  if ((e = cudaFuncSetAttribute(quantize_kernel<32, F, kBase>, a, kSmemBytes))) return e;
-  if ((e = cudaFuncSetAttribute(quantize_kernel<64, F, kBase>, a, kSmemBytes))) return e;
-  if ((e = cudaFuncSetAttribute(quantize_kernel<128, F, kBase>, a, kSmemBytes))) return e;
-  return cudaFuncSetAttribute(quantize_kernel<256, F, kBase>, a, kSmemBytes);
+  if ((e = cudaFuncSetAttribute(quantize_kernel<32, F, M>, a, kSmemBytes))) return e;
+  if ((e = cudaFuncSetAttribute(quantize_kernel<64, F, M>, a, kSmemBytes))) return e;
+  if ((e = cudaFuncSetAttribute(quantize_kernel<128, F, M>, a, kSmemBytes))) return e;
+  return cudaFuncSetAttribute(quantize_kernel<256, F, M>, a, kSmemBytes);
 }
 
-// Set-up and launch of every format, with or without a base checkpoint
-// (instantiated by quantize.cu and quantize_base.cu).
-template <bool kBase>
+// Set-up and launch of every format in one mode (instantiated by quantize.cu,
+// quantize_base.cu and quantize_emit.cu).
+template <int M>
 cudaError_t prepare_all() {
   cudaError_t e;
-  if ((e = prepare_f<kAsymF32, kBase>())) return e;
-  if ((e = prepare_f<kSymF32, kBase>())) return e;
-  if ((e = prepare_f<kSymF16, kBase>())) return e;
-  if constexpr (!kBase) return prepare_f<kAsymBits, false>();
+  if ((e = prepare_f<kAsymF32, M>())) return e;
+  if ((e = prepare_f<kSymF32, M>())) return e;
+  if ((e = prepare_f<kSymF16, M>())) return e;
+  if constexpr (M == kModeBuild) return prepare_f<kAsymBits, kModeBuild>();
   return cudaSuccess;
 }
 
-template <bool kBase>
+template <int M>
 cudaError_t launch_all(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream, int sms) {
   switch (fmt) {
-    case kAsymF32: return launch_f<kAsymF32, kBase>(group, p, stream, sms);
-    case kSymF32: return launch_f<kSymF32, kBase>(group, p, stream, sms);
-    case kSymF16: return launch_f<kSymF16, kBase>(group, p, stream, sms);
+    case kAsymF32: return launch_f<kAsymF32, M>(group, p, stream, sms);
+    case kSymF32: return launch_f<kSymF32, M>(group, p, stream, sms);
+    case kSymF16: return launch_f<kSymF16, M>(group, p, stream, sms);
     case kAsymBits:
-      if constexpr (!kBase) return launch_f<kAsymBits, false>(group, p, stream, sms);
+      if constexpr (M == kModeBuild) return launch_f<kAsymBits, kModeBuild>(group, p, stream, sms);
       break;
   }
   return cudaErrorInvalidValue;

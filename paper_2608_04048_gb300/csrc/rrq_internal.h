@@ -35,6 +35,7 @@ struct QuantizeItem {
   uint8_t* codes[kMaxStages];      // n/4 bytes each
   void* scales[kMaxStages];        // n/group float or binary16 each
   float* zeros[kMaxStages];        // n/group each (asymmetric grid only)
+  uint16_t* out[kMaxStages];       // bf16 prefix after each stage (build with prefixes only)
 };
 
 struct QuantizeBatch {
@@ -116,6 +117,7 @@ cudaError_t pmr_launch(int group, const PmrBatch& p, cudaStream_t stream, int sm
 // One-time per-device set-up of kernel attributes (dynamic shared memory).
 cudaError_t quantize_prepare();
 cudaError_t quantize_prepare_base();
+cudaError_t quantize_prepare_emit();
 cudaError_t reconstruct_prepare_asym_f32();
 cudaError_t reconstruct_prepare_sym_f32();
 cudaError_t reconstruct_prepare_sym_f16();
@@ -126,6 +128,10 @@ cudaError_t quantize_launch(int group, Format fmt, const QuantizeBatch& p, cudaS
 // Stage 0 given (item codes[0], scales[0], zeros[0] are inputs); stages
 // 1..n_stages-1 computed.
 cudaError_t quantize_launch_base(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream,
+                                 int sms);
+// Every stage computed, and the bf16 reconstruction after stage k written to
+// item out[k].
+cudaError_t quantize_launch_emit(int group, Format fmt, const QuantizeBatch& p, cudaStream_t stream,
                                  int sms);
 // all_prefixes: write prefixes 1..k to out[0..k-1] (else prefix k to out[0]).
 // One translation unit per format (they compile in parallel).

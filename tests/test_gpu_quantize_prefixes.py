@@ -1,0 +1,106 @@
+"""GPU parity for the build with prefixes (rrq_quantize_prefixes: Algorithm 1
+and Eq. 8 at every prefix in one pass): for every format the package equals
+rrq_quantize_ex's and every bf16 prefix equals rrq_reconstruct_ex's on it, bit
+for bit (both of which the other parity tests tie to the CPU oracle), and a
+direct comparison with the oracle."""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from paper_2608_04048_gb300 import binding, build, workloads
+from gpu_helpers import bf16_bits, scales_host
+from test_gpu_parity import _edge_matrix
+
+pytestmark = pytest.mark.gpu
+
+GROUPS = (32, 64, 128, 256)
+FORMATS = [(binding.GRID_ASYM, binding.SCALE_F32), (binding.GRID_SYM, binding.SCALE_F32),
+           (binding.GRID_SYM, binding.SCALE_F16)]
+FMT_IDS = ["asym_f32", "sym_f32", "sym_f16"]
+
+
+@pytest.fixture(scope="module", autouse=True)
+def lib():
+    build.build()
+    binding.load_library()
+    binding.rrq_set_debug_flags(0)
+    binding.rrq_set_wait_limit_us(1_000_000)
+    yield
+    binding.rrq_set_debug_flags(0)
+
+
+def _same(a, b):
+    return torch.equal(a.contiguous().view(torch.uint8), b.contiguous().view(torch.uint8))
+
+
+def check(mats, group, S, fmt, where=""):
+    pkgs, outs = binding.rrq_quantize_prefixes(mats, group, S, *fmt)
+    refs = binding.rrq_quantize_ex(mats, group, S, *fmt)
+    routs = binding.rrq_reconstruct_ex(refs, S, all_prefixes=True)
+    torch.cuda.synchronize()
+    assert binding.rrq_get_device_status() == 0
+    for i, (p, r) in enumerate(zip(pkgs, refs)):
+        for k in range(S):
+            assert _same(p.codes[k], r.codes[k]), f"{where} item {i} stage {k} codes"
+            assert _same(p.scales[k], r.scales[k]), f"{where} item {i} stage {k} scales"
+            if p.zeros:
+                assert _same(p.zeros[k], r.zeros[k]), f"{where} item {i} stage {k} zeros"
+            assert _same(outs[i][k], routs[i][k]), f"{where} item {i} prefix {k + 1}"
+    return pkgs, outs
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FMT_IDS)
+@pytest.mark.parametrize("group", GROUPS)
+def test_formats_and_groups(group, fmt):
+    mats = [workloads.generate(133, 5 * group, 31 + group, d, "cuda") for d in ("t3_rowout", "normal")]
+    check(mats, group, 4, fmt, where=f"g{group} {fmt}")
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FMT_IDS)
+def test_fewer_stages_and_shapes(fmt):
+    for shape in ((1, 32), (31, 32), (7, 2304), (2049, 128)):
+        for g in GROUPS:
+            if shape[1] % g:
+                continue
+            for S in (1, 2, 3):
+                W = workloads.generate(shape[0], shape[1], S + shape[0], "t3", "cuda")
+                check([W], g, S, fmt, where=f"{shape} g{g} S{S}")
+
+
+@pytest.mark.parametrize("group", GROUPS)
+def test_edge_groups_and_forced_exact(group):
+    W = _edge_matrix(24, 8 * group, group, seed=300 + group)
+    check([W], group, 4, FORMATS[0], where=f"edge g{group}")
+    binding.rrq_set_debug_flags(1)
+    try:
+        for fmt in FORMATS:
+            Wf = W if fmt[1] == binding.SCALE_F32 else workloads.generate(24, 8 * group, 3, "t3_rowout", "cuda")
+            check([Wf], group, 4, fmt, where=f"forced exact g{group} {fmt}")
+    finally:
+        binding.rrq_set_debug_flags(0)
+
+
+def test_against_oracle_and_across_launches():
+    rng = np.random.default_rng(31)
+    shapes = [(int(rng.integers(1, 30)), 128 * int(rng.integers(1, 10))) for _ in range(70)]
+    mats = [workloads.generate(r, c, 2000 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+    pkgs, outs = check(mats, 128, 4, FORMATS[0], where="batch")
+    for i in (0, 33, 69):
+        W = mats[i]
+        ref = oracle.quantize(bf16_bits(W), 128, 4)
+        for k in range(1, 5):
+            want = oracle.reconstruct(*ref, W.shape[0], W.shape[1], 128, k)
+            assert np.array_equal(bf16_bits(outs[i][k - 1]), want), f"item {i} prefix {k}"
+
+
+def test_errors():
+    W = workloads.generate(8, 256, 1, "normal", "cuda")
+    with pytest.raises(binding.RRQError) as e:
+        binding.rrq_quantize_prefixes([W], 128, 2, outs=[[torch.empty(0, dtype=torch.bfloat16, device="cuda")] * 2])
+    assert e.value.status == 1
+    pkg = binding.Package.empty(8, 256, 128, 2)
+    o = torch.empty((8, 256), dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(binding.RRQError) as e:  # two prefixes into one buffer
+        binding.rrq_quantize_prefixes([W], 128, 2, pkgs=[pkg], outs=[[o, o]])
+    assert e.value.status == 1
