@@ -109,6 +109,9 @@ constexpr int kWarps = 8;                  // warps per CTA
 constexpr int kThreads = kWarps * 32;
 constexpr int kRing = RRQ_QUANTIZE_RING;   // bulk-copy buffers per warp
 constexpr int kSmemBytes = kWarps * kRing * kChunkBytes + kWarps * kRing * 8;
+// plus, when the prefixes are written, two 2 KiB output staging buffers per warp
+template <int M>
+__host__ __device__ constexpr int smem_bytes();
 constexpr float kTwo23 = 8388608.0f;       // RN(x + 2^23) = 2^23 + rhe(x) for 0 <= x < 2^22
 constexpr float kThird = 0x1.555556p-2f;   // RN(1/3)
 constexpr float kSymRound = 12582914.0f;   // 1.5 * 2^23 + 2: RN(x + C) = C + rhe(x), low bits 2 + rhe(x)
@@ -265,11 +268,11 @@ __device__ __forceinline__ void stage_bits(f32x2 (&v)[16], float lo, float s, bo
     float a, b;
     unpack2(v[i], a, b);
     if (i & 1) {
-      mn1 = fminf(mn1, fminf(a, b));
-      mx1 = fmaxf(mx1, fmaxf(a, b));
+      mn1 = min3(mn1, a, b);
+      mx1 = max3(mx1, a, b);
     } else {
-      mn0 = fminf(mn0, fminf(a, b));
-      mx0 = fmaxf(mx0, fmaxf(a, b));
+      mn0 = min3(mn0, a, b);
+      mx0 = max3(mx0, a, b);
     }
   }
   mn = fminf(mn0, mn1);
@@ -424,20 +427,39 @@ __device__ __forceinline__ void subtract_base(f32x2 (&v)[16], const BaseWords& b
   }
 }
 
-// bf16 of the prefix sums of this lane's 32 weights (slot order), each 16-byte
-// piece stored at its place in memory (slot j holds piece (j + rot) & 3).
-__device__ __forceinline__ void emit_prefix(uint16_t* out, int64_t e0, const f32x2 (&w)[16], int rot) {
+// Output staging of the build with prefixes: two 2 KiB buffers per warp used
+// in turn; every lane writes its 32 bf16 values (slot j -> piece (j + rot) & 3,
+// conflict-free), lane 0 writes the chunk out with one bulk copy.
+struct Emitter {
+  uint8_t* stage;   // this warp's two buffers
+  uint32_t n_store; // stores issued so far
+};
+
+// bf16 of the prefix sums of this lane's 32 weights to out[c0 ..] (warp-wide:
+// every lane calls it, also lanes past the end of the matrix).
+__device__ __forceinline__ void emit_prefix(Emitter& em, uint16_t* out, int64_t c0, int64_t n,
+                                            const f32x2 (&w)[16], int lane, int rot) {
+  uint32_t h[16];
 #pragma unroll
-  for (int j = 0; j < 4; ++j) {
-    uint32_t h[4];
+  for (int m = 0; m < 16; ++m) {
+    float a, b;
+    unpack2(w[m], a, b);
+    const __nv_bfloat162 x = __floats2bfloat162_rn(a, b);
+    h[m] = *reinterpret_cast<const uint32_t*>(&x);
+  }
+  uint8_t* buf = em.stage + (em.n_store & 1) * kChunkBytes;
+  ++em.n_store;
+  if (lane == 0) bulk_wait_read<1>();  // the copy that last used this buffer has read it
+  __syncwarp();
+  uint4* dst = reinterpret_cast<uint4*>(buf + lane * 64);
 #pragma unroll
-    for (int m = 0; m < 4; ++m) {
-      float a, b;
-      unpack2(w[4 * j + m], a, b);
-      const __nv_bfloat162 x = __floats2bfloat162_rn(a, b);
-      h[m] = *reinterpret_cast<const uint32_t*>(&x);
-    }
-    __stcs(reinterpret_cast<uint4*>(out + e0 + 8 * ((j + rot) & 3)), make_uint4(h[0], h[1], h[2], h[3]));
+  for (int j = 0; j < 4; ++j) dst[(j + rot) & 3] = make_uint4(h[4 * j], h[4 * j + 1], h[4 * j + 2], h[4 * j + 3]);
+  fence_proxy_async_smem();
+  __syncwarp();
+  if (lane == 0) {
+    const int64_t left = n - c0;
+    bulk_store(out + c0, smem_u32(buf), static_cast<uint32_t>((left < kChunkElems ? left : kChunkElems) * 2));
+    bulk_commit();
   }
 }
 
@@ -445,7 +467,7 @@ template <int G, int M>
 __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, const QuantizeItem& it,
                                                     int64_t e0, int lane, uint4 (&raw)[4],
                                                     uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
-                                                    uint32_t ld_lo, uint32_t ld_hi, int rot) {
+                                                    uint32_t ld_lo, uint32_t ld_hi, int rot, Emitter& em) {
   constexpr bool kBase = M == kModeBase;
   constexpr bool kEmit = M == kModeEmit;
   constexpr int L = G / 32;  // lanes per group
@@ -474,8 +496,24 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
   lane_minmax(v, lo, hi);
   group_minmax<L>(lo, hi);
 
+  // A stage's codes, scale, offset and prefix are written in the next stage's
+  // prologue (the last stage's after the loop): independent stores that fill
+  // the latency of the next range, scale and reciprocal.
+  uint32_t acc[4] = {0u, 0u, 0u, 0u};
+  float s_out = 0.0f, lo_out = 0.0f;
+  auto write_stage = [&](int k) {
+    if (valid) {
+      store_codes(it.codes[k], e0, acc, sel_lo, sel_hi);
+      if ((lane & (L - 1)) == 0) {
+        __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s_out);
+        __stcs(it.zeros[k] + e0 / G, lo_out);
+      }
+    }
+    if constexpr (kEmit) emit_prefix(em, it.out[k], e0 - lane * kLaneElems, it.n, wsum, lane, rot);
+  };
+  const int k0 = kBase ? 1 : 0;
 #pragma unroll 1
-  for (int k = kBase ? 1 : 0; k < p.n_stages; ++k) {
+  for (int k = k0; k < p.n_stages; ++k) {
     // A zero minimum: the stored offset is -0 if the group holds a -0.
     if (__any_sync(kFullMask, lo == 0.0f)) {
       uint32_t neg = 0;
@@ -491,12 +529,15 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
 
     const float s = div3(__fsub_rn(hi, lo));
     const bool fast = !(p.flags & kDebugForceExact) && (s == 0.0f || corrected_quotient_safe(s));
-    uint32_t acc[4] = {0u, 0u, 0u, 0u};
+    float r_hi, r_lo;
+    recip2(s, r_hi, r_lo);
+    if (!(s > 0.0f)) r_hi = r_lo = 0.0f;  // s = 0: every quotient 0
+    if (k > k0) write_stage(k - 1);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[j] = 0u;
     // min/max of the new residual (next stage's range), gathered in the loop
     float mn0 = __int_as_float(0x7f800000), mn1 = mn0, mx0 = -mn0, mx1 = mx0;
     if (fast) {
-      float r_hi = 0.0f, r_lo = 0.0f;
-      if (s > 0.0f) recip2(s, r_hi, r_lo);
       const float c = __fmul_rn(-kTwo23, s);  // exact: power-of-two scaling
       const f32x2 LO = pack2(lo, lo), RH = pack2(r_hi, r_hi), RL = pack2(r_lo, r_lo), S = pack2(s, s);
       const f32x2 T23 = pack2(kTwo23, kTwo23), C = pack2(c, c);
@@ -514,11 +555,11 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
         float a, b;
         unpack2(v[i], a, b);
         if (i & 1) {
-          mn1 = fminf(mn1, fminf(a, b));
-          mx1 = fmaxf(mx1, fmaxf(a, b));
+          mn1 = min3(mn1, a, b);
+          mx1 = max3(mx1, a, b);
         } else {
-          mn0 = fminf(mn0, fminf(a, b));
-          mx0 = fmaxf(mx0, fmaxf(a, b));
+          mn0 = min3(mn0, a, b);
+          mx0 = max3(mx0, a, b);
         }
       }
     } else {  // this group: IEEE division element by element
@@ -531,21 +572,15 @@ __device__ __forceinline__ void quantize_chunk_asym(const QuantizeBatch& p, cons
       }
       lane_minmax(v, mn0, mx0);
     }
-
-    if (valid) {
-      store_codes(it.codes[k], e0, acc, sel_lo, sel_hi);
-      if ((lane & (L - 1)) == 0) {
-        __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s);
-        __stcs(it.zeros[k] + e0 / G, lo);
-      }
-      if constexpr (kEmit) emit_prefix(it.out[k], e0, wsum, rot);
-    }
+    s_out = s;
+    lo_out = lo;
     if (k + 1 < p.n_stages) {  // range of the residual = next stage's lo, hi
       lo = fminf(mn0, mn1);
       hi = fmaxf(mx0, mx1);
       group_minmax<L>(lo, hi);
     }
   }
+  if (p.n_stages > k0) write_stage(p.n_stages - 1);
 }
 
 // Symmetric grid; kF16: the scale is rounded to binary16, stored as such, and
@@ -554,7 +589,7 @@ template <int G, bool kF16, int M>
 __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const QuantizeItem& it,
                                                    int64_t e0, int lane, uint4 (&raw)[4],
                                                    uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
-                                                   uint32_t ld_lo, uint32_t ld_hi, int rot) {
+                                                   uint32_t ld_lo, uint32_t ld_hi, int rot, Emitter& em) {
   constexpr bool kBase = M == kModeBase;
   constexpr bool kEmit = M == kModeEmit;
   constexpr int L = G / 32;  // lanes per group
@@ -578,8 +613,24 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
   if constexpr (kBase) subtract_base<kSymF32>(v, bw, ld_lo, ld_hi);  // R_0 = W - W_0
   float amax = group_max<L>(lane_amax(v));
 
+  // A stage's codes, scale and prefix are written in the next stage's
+  // prologue (the last stage's after the loop), filling its latency.
+  uint32_t acc[4] = {0u, 0u, 0u, 0u};
+  float s_out = 0.0f;
+  uint16_t s16_out = 0;
+  auto write_stage = [&](int k) {
+    if (valid) {
+      store_codes(it.codes[k], e0, acc, sel_lo, sel_hi);
+      if ((lane & (L - 1)) == 0) {
+        if (kF16) stcs_u16(static_cast<uint16_t*>(it.scales[k]) + e0 / G, s16_out);
+        else __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s_out);
+      }
+    }
+    if constexpr (kEmit) emit_prefix(em, it.out[k], e0 - lane * kLaneElems, it.n, wsum, lane, rot);
+  };
+  const int k0 = kBase ? 1 : 0;
 #pragma unroll 1
-  for (int k = kBase ? 1 : 0; k < p.n_stages; ++k) {
+  for (int k = k0; k < p.n_stages; ++k) {
     float s = div3(__fmul_rn(amax, 2.0f));  // 2 * amax is exact
     uint16_t s16 = 0;
     if (kF16) {
@@ -587,11 +638,14 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
       s = __half2float(__ushort_as_half(s16));
     }
     const bool fast = !(p.flags & kDebugForceExact) && (kF16 || s == 0.0f || corrected_quotient_safe(s));
-    uint32_t acc[4] = {0u, 0u, 0u, 0u};
+    float r_hi, r_lo;
+    recip2(s, r_hi, r_lo);
+    if (!(s > 0.0f)) r_hi = r_lo = 0.0f;  // s = 0: every quotient 0
+    if (k > k0) write_stage(k - 1);
+#pragma unroll
+    for (int j = 0; j < 4; ++j) acc[j] = 0u;
     float mx0 = 0.0f, mx1 = 0.0f;  // max |new residual|, gathered in the loop
     if (fast) {
-      float r_hi = 0.0f, r_lo = 0.0f;
-      if (s > 0.0f) recip2(s, r_hi, r_lo);
       const f32x2 RH = pack2(r_hi, r_hi), RL = pack2(r_lo, r_lo), NS = pack2(-s, -s), S = pack2(s, s);
       const f32x2 C = pack2(kSymRound, kSymRound);
 #pragma unroll
@@ -607,8 +661,8 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
                                 static_cast<uint32_t>(t >> 32));
         float a, b;
         unpack2(v[i], a, b);
-        if (i & 1) mx1 = fmaxf(mx1, fmaxf(fabsf(a), fabsf(b)));
-        else mx0 = fmaxf(mx0, fmaxf(fabsf(a), fabsf(b)));
+        if (i & 1) mx1 = max3(mx1, fabsf(a), fabsf(b));
+        else mx0 = max3(mx0, fabsf(a), fabsf(b));
       }
     } else {  // this group: IEEE division element by element
 #pragma unroll
@@ -620,30 +674,24 @@ __device__ __forceinline__ void quantize_chunk_sym(const QuantizeBatch& p, const
       }
       mx0 = lane_amax(v);
     }
-
-    if (valid) {
-      store_codes(it.codes[k], e0, acc, sel_lo, sel_hi);
-      if ((lane & (L - 1)) == 0) {
-        if (kF16) stcs_u16(static_cast<uint16_t*>(it.scales[k]) + e0 / G, s16);
-        else __stcs(static_cast<float*>(it.scales[k]) + e0 / G, s);
-      }
-      if constexpr (kEmit) emit_prefix(it.out[k], e0, wsum, rot);
-    }
+    s_out = s;
+    s16_out = s16;
     if (k + 1 < p.n_stages) amax = group_max<L>(fmaxf(mx0, mx1));
   }
+  if (p.n_stages > k0) write_stage(p.n_stages - 1);
 }
 
 template <int G, int F, int M>
 __device__ __forceinline__ void quantize_chunk(const QuantizeBatch& p, const QuantizeItem& it,
                                                int64_t e0, int lane, uint4 (&raw)[4],
                                                uint32_t sel_lo, uint32_t sel_hi, const BaseWords& bw,
-                                               uint32_t ld_lo, uint32_t ld_hi, int rot) {
+                                               uint32_t ld_lo, uint32_t ld_hi, int rot, Emitter& em) {
   if constexpr (F == kAsymF32)
-    quantize_chunk_asym<G, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot);
+    quantize_chunk_asym<G, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot, em);
   else if constexpr (F == kAsymBits)
     quantize_chunk_bits<G>(p, it, e0, lane, raw);
   else
-    quantize_chunk_sym<G, F == kSymF16, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot);
+    quantize_chunk_sym<G, F == kSymF16, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot, em);
 }
 
 // (the width-generic stages and the prefix sums need more registers: two
@@ -658,6 +706,7 @@ quantize_kernel(const __grid_constant__ QuantizeBatch p) {
   uint8_t* ring = smem + warp * (kRing * kChunkBytes);
   const uint32_t ring_s = smem_u32(ring);
   const uint32_t bar0 = smem_u32(smem + kWarps * kRing * kChunkBytes) + warp * kRing * 8;
+  Emitter em{smem + kSmemBytes + warp * 2 * kChunkBytes, 0u};  // used by the build with prefixes
 
   const int64_t first = static_cast<int64_t>(blockIdx.x) * kWarps + warp;
   const int64_t stride = static_cast<int64_t>(gridDim.x) * kWarps;
@@ -725,6 +774,7 @@ quantize_kernel(const __grid_constant__ QuantizeBatch p) {
           const uint32_t jt = iter + j;
           mbar_wait(bar0 + 8 * (jt % kRing), (jt / kRing) & 1, kDrainLimitUs);
         }
+        if (M == kModeEmit) bulk_wait<0>();  // this warp's output copies
       }
       __syncwarp();
       return;
@@ -745,8 +795,14 @@ quantize_kernel(const __grid_constant__ QuantizeBatch p) {
     const int64_t e0 = (chunk - it.chunk_begin) * kChunkElems + static_cast<int64_t>(lane) * kLaneElems;
     const BaseWords bw = bw_next;
     if (kBase) bw_next = base_of(chunk + stride);  // in flight while this chunk computes
-    quantize_chunk<G, F, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot);
+    quantize_chunk<G, F, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot, em);
   }
+  if (M == kModeEmit && lane == 0) bulk_wait<0>();  // output copies done before the CTA exits
+}
+
+template <int M>
+__host__ __device__ constexpr int smem_bytes() {
+  return kSmemBytes + (M == kModeEmit ? kWarps * 2 * kChunkBytes : 0);
 }
 
 template <int G, int F, int M>
@@ -754,14 +810,14 @@ cudaError_t launch_gf(const QuantizeBatch& p, cudaStream_t stream, int sms) {
   static int blocks_per_sm = 0;  // same for every device of this build
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
-        &blocks_per_sm, quantize_kernel<G, F, M>, kThreads, kSmemBytes);
+        &blocks_per_sm, quantize_kernel<G, F, M>, kThreads, smem_bytes<M>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
   }
   const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  quantize_kernel<G, F, M><<<grid, kThreads, kSmemBytes, stream>>>(p);
+  quantize_kernel<G, F, M><<<grid, kThreads, smem_bytes<M>(), stream>>>(p);
   return cudaGetLastError();
 }
 
@@ -780,10 +836,10 @@ template <int F, int M>
 cudaError_t prepare_f() {
   cudaError_t e;
   const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-  if ((e = cudaFuncSetAttribute(quantize_kernel<32, F, M>, a, kSmemBytes))) return e;
-  if ((e = cudaFuncSetAttribute(quantize_kernel<64, F, M>, a, kSmemBytes))) return e;
-  if ((e = cudaFuncSetAttribute(quantize_kernel<128, F, M>, a, kSmemBytes))) return e;
-  return cudaFuncSetAttribute(quantize_kernel<256, F, M>, a, kSmemBytes);
+  if ((e = cudaFuncSetAttribute(quantize_kernel<32, F, M>, a, smem_bytes<M>()))) return e;
+  if ((e = cudaFuncSetAttribute(quantize_kernel<64, F, M>, a, smem_bytes<M>()))) return e;
+  if ((e = cudaFuncSetAttribute(quantize_kernel<128, F, M>, a, smem_bytes<M>()))) return e;
+  return cudaFuncSetAttribute(quantize_kernel<256, F, M>, a, smem_bytes<M>());
 }
 
 // Set-up and launch of every format in one mode (instantiated by quantize.cu,

@@ -206,8 +206,8 @@ __device__ __forceinline__ float lane_amax(const f32x2 (&v)[16]) {
     float a, b, c, d;
     unpack2(v[i], a, b);
     unpack2(v[i + 1], c, d);
-    m0 = fmaxf(m0, fmaxf(fabsf(a), fabsf(b)));
-    m1 = fmaxf(m1, fmaxf(fabsf(c), fabsf(d)));
+    m0 = max3(m0, fabsf(a), fabsf(b));
+    m1 = max3(m1, fabsf(c), fabsf(d));
   }
   return fmaxf(m0, m1);
 }
