@@ -101,6 +101,11 @@ class Oracle:
             ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
             _u16p, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
         lib.rrq_oracle_gemv.restype = ctypes.c_int
+        lib.rrq_oracle_prefill.argtypes = [
+            ctypes.POINTER(_u8p), ctypes.POINTER(ctypes.c_void_p), ctypes.POINTER(_f32p),
+            ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, ctypes.c_int, ctypes.c_int,
+            _u16p, ctypes.c_int64, ctypes.POINTER(ctypes.c_double)]
+        lib.rrq_oracle_prefill.restype = ctypes.c_int
         _i32p = ctypes.POINTER(ctypes.c_int)
         lib.rrq_oracle_quantize_group_bits.argtypes = [
             _f32p, ctypes.c_int, ctypes.c_int, _i32p, _u8p, _f32p, _f32p, _f32p]
@@ -267,6 +272,30 @@ class Oracle:
             raise ValueError("oracle rejected the product")
         return Y
 
+    def prefill(self, codes, scales, zeros, rows: int, cols: int, group: int, k: int, A_bits,
+                sym: bool = False, scale_f16: bool = False):
+        """Y [tokens, rows] float64 = A [tokens, cols] (bf16 bit patterns) times
+        the transposed bf16 prefix-k reconstruction, summed in binary64."""
+        A_bits = np.ascontiguousarray(np.atleast_2d(A_bits), dtype=np.uint16)
+        tokens = A_bits.shape[0]
+        assert A_bits.shape[1] == cols
+        sdt = np.uint16 if scale_f16 else np.float32
+        codes = [np.ascontiguousarray(c, dtype=np.uint8) for c in codes[:k]]
+        scales = [np.ascontiguousarray(a, dtype=sdt) for a in scales[:k]]
+        cp = (_u8p * k)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (ctypes.c_void_p * k)(*[a.ctypes.data for a in scales])
+        zp = None
+        if not sym:
+            zeros = [np.ascontiguousarray(a, dtype=np.float32) for a in zeros[:k]]
+            zp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        Y = np.zeros((tokens, rows), np.float64)
+        rc = self.lib.rrq_oracle_prefill(cp, sp, zp, rows, cols, group, k, int(sym), int(scale_f16),
+                                         A_bits.ctypes.data_as(_u16p), tokens,
+                                         Y.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
+        if rc != 0:
+            raise ValueError("oracle rejected the prefill product")
+        return Y
+
     # -- heterogeneous stage widths (asymmetric grid) ----------------------------
     def quantize_group_bits(self, x, bits):
         """(Q, scale, zero, resid) for one group with per-stage widths."""
@@ -375,6 +404,10 @@ def reconstruct_sym(codes, scales, rows, cols, group, k, scale_f16: bool = True)
 
 def gemv(codes, scales, zeros, rows, cols, group, k, A_bits, sym: bool = False, scale_f16: bool = False):
     return load().gemv(codes, scales, zeros, rows, cols, group, k, A_bits, sym, scale_f16)
+
+
+def prefill(codes, scales, zeros, rows, cols, group, k, A_bits, sym: bool = False, scale_f16: bool = False):
+    return load().prefill(codes, scales, zeros, rows, cols, group, k, A_bits, sym, scale_f16)
 
 
 def quantize_bits(W_bits, group, bits):

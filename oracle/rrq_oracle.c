@@ -56,6 +56,11 @@
  * products and the sum taken in binary64 (each product of a binary32 and a
  * bf16 value is exact there).
  *
+ * Prefill form of the same product (many activation rows, bf16 operands as
+ * a tensor-core GEMM takes them): the weight is the bf16 prefix
+ * reconstruction itself, Y[t][r] = sum_c bf16(W~[r][c]) * A[t][c] in
+ * binary64 (products of two bf16 values are exact there).
+ *
  * Heterogeneous stage widths (Section 3.2: stage k may use b_k bits, B_t is
  * the sum of the widths; the split analysis of Section 3.3 / Table 3 uses
  * zero-point grids): stage k of the asymmetric grid with b bits has
@@ -557,5 +562,46 @@ int rrq_oracle_group_pmr(const uint16_t* W, int64_t rows, int64_t cols, int grou
     }
     pmr[gi] = sum > 0.0 ? peak / (sum / (double)group) : 0.0;
   }
+  return 0;
+}
+
+/* bf16 prefix-k weight of flat element c: the binary32 stage sum of the
+ * first k stages (stage order), rounded to nearest-even bf16 -- the value the
+ * prefix reconstruction returns for that element. */
+static uint16_t prefill_weight(const uint8_t* const* codes, const void* const* scales,
+                               const float* const* zeros, int64_t c, int group, int k,
+                               int grid_sym, int scale_f16) {
+  const int64_t g = c / group;
+  float sum = 0.0f;
+  for (int st = 0; st < k; ++st) {
+    const int code = (codes[st][c / 4] >> (2 * (c % 4))) & 3;
+    const float sc = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[st])[g])
+                               : ((const float*)scales[st])[g];
+    const float level = base_level(grid_sym, code, sc, grid_sym ? 0.0f : zeros[st][g]);
+    sum = st == 0 ? level : sum + level;
+  }
+  return rrq_oracle_f32_to_bf16(sum);
+}
+
+int rrq_oracle_prefill(const uint8_t* const* codes, const void* const* scales,
+                       const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
+                       int grid_sym, int scale_f16, const uint16_t* A, int64_t tokens, double* Y) {
+  if (!codes || !scales || (!grid_sym && !zeros) || !A || !Y) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || k < 1 || tokens < 1) return -1;
+  if (cols % group != 0 || (scale_f16 && !grid_sym)) return -1;
+  double* wrow = (double*)malloc(sizeof(double) * (size_t)cols);
+  if (!wrow) return -1;
+  for (int64_t r = 0; r < rows; ++r) {
+    for (int64_t j = 0; j < cols; ++j)
+      wrow[j] = (double)rrq_oracle_bf16_to_f32(
+          prefill_weight(codes, scales, zeros, r * cols + j, group, k, grid_sym, scale_f16));
+    for (int64_t t = 0; t < tokens; ++t) {
+      double dot = 0.0;
+      for (int64_t j = 0; j < cols; ++j)
+        dot += wrow[j] * (double)rrq_oracle_bf16_to_f32(A[(size_t)t * cols + j]);
+      Y[(size_t)t * rows + r] = dot;
+    }
+  }
+  free(wrow);
   return 0;
 }

@@ -86,6 +86,16 @@ int rrq_oracle_gemv(const uint8_t* const* codes, const void* const* scales,
                     const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
                     int grid_sym, int scale_f16, const uint16_t* A, int batch, double* Y);
 
+/* Product of many activation rows with the prefix-k weights, the prefill
+ * form of Appendix C's stage-wise product with bf16 operands (as a tensor-core
+ * GEMM takes them): Y[t][r] = sum_c bf16(W~[r][c]) * A[t][c] in binary64,
+ * bf16(W~) = the prefix-k reconstruction (the binary32 stage sum rounded to
+ * nearest-even bf16), each product of two bf16 values exact in binary64.
+ *   A  bf16 bit patterns [tokens][cols];  Y  double [tokens][rows]. */
+int rrq_oracle_prefill(const uint8_t* const* codes, const void* const* scales,
+                       const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
+                       int grid_sym, int scale_f16, const uint16_t* A, int64_t tokens, double* Y);
+
 /* Asymmetric stages with per-stage widths bits[k] in 1..4 (2^b levels,
  * 2^b - 1 steps).  Group form as rrq_oracle_quantize_group; matrix form packs
  * stage k's codes LSB-first, element c at bits bits[k]*c.., into

@@ -938,13 +938,122 @@ def pin_group_pmr(orc, seed=61) -> list[str]:
     return fails
 
 
+# ---------------------------------------------------------------------------
+# prefill product (bf16 operands: the prefix reconstruction is the weight)
+# ---------------------------------------------------------------------------
+# PF1: a hand-built one-stage package, codes [0, 1, 2, 3] (byte 0xE4, LSB
+#   first), scale s = 1 + 3*2^-9, zero 0.  Levels fl(Q s) = [0, 1.005859375,
+#   2.01171875, 3.017578125] (exact); their bf16 nearest-even values are
+#   [0, 1.0078125, 2.015625, 3.015625] (truncation would give [0, 1, 2,
+#   3.015625]).  A = [[1, 1, 1, 1], [0, 0, 0, 1], [1, -1, 0.5, 2]]:
+#   Y = [6.0390625, 3.015625, -1.0078125 + 1.0078125 + 6.03125 = 6.03125].
+# PF2: the same codes, symmetric grid, binary16 scale 1.0 (0x3C00): levels
+#   (Q - 2) = [-2, -1, 0, 1]; Y = [-2, 1, -2 + 1 + 0 + 2 = 1].
+PF1 = dict(byte=0xE4, scale=1.0 + 3 * 2.0 ** -9, Y=[6.0390625, 3.015625, 6.03125])
+PF_A = [[1.0, 1.0, 1.0, 1.0], [0.0, 0.0, 0.0, 1.0], [1.0, -1.0, 0.5, 2.0]]
+PF2_Y = [-2.0, 1.0, 1.0]
+
+
+def pin_prefill_worked(orc) -> list[str]:
+    fails = []
+    A = bf16_bits_of_f32(np.array(PF_A, np.float32))
+    codes = [np.array([PF1["byte"]], np.uint8)]
+    Y = orc.prefill(codes, [np.array([PF1["scale"]], np.float32)], [np.zeros(1, np.float32)], 1, 4, 4, 1, A)
+    if Y[:, 0].tolist() != PF1["Y"]:
+        fails.append(f"PF1: {Y[:, 0].tolist()} != {PF1['Y']}")
+    Y = orc.prefill(codes, [np.array([0x3C00], np.uint16)], None, 1, 4, 4, 1, A, sym=True, scale_f16=True)
+    if Y[:, 0].tolist() != PF2_Y:
+        fails.append(f"PF2: {Y[:, 0].tolist()} != {PF2_Y}")
+    return fails
+
+
+def pin_prefill_one_hot(orc, seed=67, rows=5, g=64) -> list[str]:
+    """One-hot activation rows pick single weights: with A[t] = e_(p(t)) for a
+    permutation p of the columns, Y[t][r] is the bf16 reconstruction (a
+    separately pinned routine) at [r][p(t)], exactly; every format, k = 1..4."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 2 * g
+    xs = np.concatenate(_random_groups(rng, rows * 2, g)).reshape(rows, cols)
+    W = bf16_bits_of_f32(xs)
+    perm = rng.permutation(cols)
+    A = np.zeros((cols, cols), np.float32)
+    A[np.arange(cols), perm] = 1.0
+    A = bf16_bits_of_f32(A)
+    for sym, f16 in ((False, False), (True, False), (True, True)):
+        if sym:
+            codes, scales = orc.quantize_sym(W, group=g, n_stages=4, scale_f16=f16)
+            zeros = None
+        else:
+            codes, scales, zeros = orc.quantize(W, group=g, n_stages=4)
+        for k in range(1, 5):
+            rec = (orc.reconstruct_sym(codes, scales, rows, cols, g, k, f16) if sym
+                   else orc.reconstruct(codes, scales, zeros, rows, cols, g, k))
+            recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+            Y = orc.prefill(codes, scales, zeros, rows, cols, g, k, A, sym, f16)
+            if not np.array_equal(Y, recf[:, perm].T):
+                fails.append(f"sym={sym} f16={f16} k={k}: one-hot rows do not select the reconstruction")
+    return fails
+
+
+def pin_prefill_integer_exact(orc, seed=71, rows=6, g=32) -> list[str]:
+    """Packages with scale 1 and integer zeros have integer levels z + Q, so
+    every prefix weight is a small integer (exact in bf16) and, with integer
+    activations, the product is an integer matrix: numpy's int64 matmul of the
+    weights unpacked here (LSB-first 2-bit codes, group-wise zeros) must equal
+    the oracle exactly."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 4 * g
+    n = rows * cols
+    q = rng.integers(0, 4, (4, n))
+    z = rng.integers(-3, 4, (4, n // g))
+    codes = [np.zeros(n // 4, np.uint8) for _ in range(4)]
+    for i in range(4):
+        for s in range(4):
+            codes[i] |= (q[i, s::4] << (2 * s)).astype(np.uint8)
+    scales = [np.ones(n // g, np.float32) for _ in range(4)]
+    zeros = [z[i].astype(np.float32) for i in range(4)]
+    A_int = rng.integers(-4, 5, (7, cols))
+    A = bf16_bits_of_f32(A_int.astype(np.float32))
+    for k in range(1, 5):
+        w = sum(q[i] + np.repeat(z[i], g) for i in range(k)).reshape(rows, cols)
+        Y = orc.prefill(codes, scales, zeros, rows, cols, g, k, A)
+        if not np.array_equal(Y, (A_int @ w.T).astype(np.float64)):
+            fails.append(f"k={k}: integer package product differs from the int64 matmul")
+    return fails
+
+
+def pin_prefill_vs_binary32_product(orc, seed=73, rows=4, g=128) -> list[str]:
+    """The bf16-weight product differs from the binary32-weight product (the
+    decode form, pinned above) by at most the bf16 rounding of each weight:
+    |Y_bf16 - Y_f32| <= 2^-9 sum |a| |w~| (plus the binary64 sums)."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 2 * g
+    xs = np.concatenate(_random_groups(rng, rows * 2, g)).reshape(rows, cols)
+    codes, scales, zeros = orc.quantize(bf16_bits_of_f32(xs), group=g, n_stages=4)
+    A = bf16_round_bits(rng.normal(0, 1, (9, cols)).astype(np.float32))
+    Af = (A.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    for k in range(1, 5):
+        Yb = orc.prefill(codes, scales, zeros, rows, cols, g, k, A)
+        Yf = orc.gemv(codes, scales, zeros, rows, cols, g, k, A)
+        rec = orc.reconstruct(codes, scales, zeros, rows, cols, g, k)
+        recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        tol = np.abs(Af) @ np.abs(recf).T * 2.0 ** -8 + 1e-300
+        if np.any(np.abs(Yb - Yf) > tol) or np.array_equal(Yb, Yf):
+            fails.append(f"k={k}: bf16-weight product not within bf16 rounding of the binary32 one")
+    return fails
+
+
 ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_brute_force_tiny,
             pin_invariants, pin_exact_grid, pin_prefix_reconstruction, pin_f16_rounding,
             pin_sym_worked_groups, pin_sym_brute_force_exact, pin_sym_invariants,
             pin_sym_prefix_reconstruction, pin_base_worked_groups, pin_base_branch_equivalence,
             pin_base_residual_invariants, pin_gemv_worked, pin_gemv_is_input_minus_residual,
             pin_gemv_vs_bf16_reconstruction, pin_bits_worked_and_two_bit_case, pin_bits_brute_force_exact,
-            pin_bits_invariants_and_packing, pin_group_pmr]
+            pin_bits_invariants_and_packing, pin_group_pmr, pin_prefill_worked, pin_prefill_one_hot,
+            pin_prefill_integer_exact, pin_prefill_vs_binary32_product]
 
 
 def all_failures(orc) -> list[str]:

@@ -74,6 +74,17 @@ MUTANTS = {
                           "const double a = (double)rrq_oracle_bf16_to_f32(W[gi * group + j]);"),
     "gemv_one_stage_short": ("      for (int i = 0; i < k; ++i) {\n        const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;\n        const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])\n                                  : ((const float*)scales[i])[gi];\n        const float lv",
                              "      for (int i = 0; i < k - (k > 1); ++i) {\n        const int q = (codes[i][c / 4] >> (2 * (c % 4))) & 3;\n        const float s = scale_f16 ? rrq_oracle_f16_to_f32(((const uint16_t*)scales[i])[gi])\n                                  : ((const float*)scales[i])[gi];\n        const float lv"),
+    # prefill product (bf16 weights)
+    "prefill_drops_base": ("sum = st == 0 ? level : sum + level;", "sum = st == 0 ? 0.0f : sum + level;"),
+    "prefill_weight_truncated": ("  return rrq_oracle_f32_to_bf16(sum);",
+                                 "  uint32_t u; memcpy(&u, &sum, 4); return (uint16_t)(u >> 16);"),
+    "prefill_reversed_activation": ("dot += wrow[j] * (double)rrq_oracle_bf16_to_f32(A[(size_t)t * cols + j]);",
+                                    "dot += wrow[j] * (double)rrq_oracle_bf16_to_f32(A[(size_t)t * cols + (cols - 1 - j)]);"),
+    "prefill_wrong_output_row": ("Y[(size_t)t * rows + r] = dot;", "Y[(size_t)t * rows + (rows - 1 - r)] = dot;"),
+    "prefill_one_stage_short": ("for (int st = 0; st < k; ++st) {", "for (int st = 0; st < k - (k > 1); ++st) {"),
+    "prefill_code_bit_order": ("const int code = (codes[st][c / 4] >> (2 * (c % 4))) & 3;",
+                               "const int code = (codes[st][c / 4] >> (2 * (3 - c % 4))) & 3;"),
+    "prefill_first_group_only": ("  const int64_t g = c / group;\n  float sum", "  const int64_t g = 0;\n  float sum"),
 }
 
 
