@@ -322,6 +322,25 @@ typedef struct {
 rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
                     rrq_stream_t stream);
 
+#define RRQ_MAX_PREFILL_TOKENS (1 << 24)
+
+/* Prefill form of the same product (Appendix C's stage-wise product for many
+ * activation rows) on the tensor cores, without materialising the weights:
+ *     Y[t][r] = sum_c bf16(W~)[r][c] * A[t][c],   t < tokens, r < rows
+ * where bf16(W~) is the prefix-k reconstruction, bit for bit the values
+ * rrq_reconstruct_ex returns (the tensor cores take bf16 operands).  The
+ * kernel forms those weights from the package tile by tile in shared memory
+ * and multiplies with tcgen05 MMAs, accumulating in binary32 (the order of
+ * the partial sums is the hardware's; the result is deterministic).  The
+ * items are rrq_gemv_desc with A_bf16 = [tokens, cols] and Y = float [tokens,
+ * rows], both row-major and 16-byte aligned.  1 <= tokens <=
+ * RRQ_MAX_PREFILL_TOKENS; 1 <= k <= fmt->n_stages; 2-bit stages only
+ * (RRQ_ERR_UNSUPPORTED for other widths).  Y must not overlap any input or
+ * another Y.  One launch per 16 matrices; other rules as for
+ * rrq_reconstruct_ex. */
+rrq_status rrq_prefill(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int64_t tokens,
+                       rrq_stream_t stream);
+
 /* One matrix of rrq_group_pmr. */
 typedef struct {
   const uint16_t* W_bf16;  /* device, bf16 [rows, cols], 16-byte aligned */

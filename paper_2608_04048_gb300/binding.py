@@ -22,7 +22,7 @@ _STATUS = {0: "RRQ_OK", 1: "RRQ_ERR_INVALID_ARG", 2: "RRQ_ERR_UNSUPPORTED",
 #: symbols declared in include/rrq.h
 EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconstruct_batch",
            "rrq_reconstruct_prefixes", "rrq_reconstruct_prefixes_batch",
-           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_gemv",
+           "rrq_quantize_ex", "rrq_reconstruct_ex", "rrq_quantize_from_base", "rrq_gemv", "rrq_prefill",
            "rrq_stage_codes_bytes", "rrq_group_pmr", "rrq_quantize_prefixes", "rrq_scales_bytes", "rrq_package_bytes_ex",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
@@ -147,6 +147,8 @@ def load_library():
     lib.rrq_quantize_from_base.restype = i32
     lib.rrq_gemv.argtypes = [ctypes.POINTER(GemvDesc), i32, fmt_p, i32, i32, vp]
     lib.rrq_gemv.restype = i32
+    lib.rrq_prefill.argtypes = [ctypes.POINTER(GemvDesc), i32, fmt_p, i32, ctypes.c_int64, vp]
+    lib.rrq_prefill.restype = i32
     lib.rrq_reconstruct_ex.argtypes = [ctypes.POINTER(ReconstructDesc), i32, fmt_p, i32, i32, vp]
     lib.rrq_reconstruct_ex.restype = i32
     lib.rrq_group_pmr.argtypes = [ctypes.POINTER(PmrDesc), i32, i32, vp]
@@ -491,6 +493,27 @@ def rrq_gemv(pkgs, acts, k: int, ys=None, stream=None, items=None):
     rc = lib.rrq_gemv(items, len(items), ctypes.byref(fmt), k, batch, _stream_handle(stream))
     if rc != 0:
         raise RRQError(rc, "rrq_gemv")
+    return ys
+
+
+def rrq_prefill(pkgs, acts, k: int, ys=None, stream=None, items=None):
+    """Y_i = A_i bf16(W~_i)^T for each package i at prefix k on the tensor
+    cores (Appendix C's product for many activation rows), A_i bf16 [tokens,
+    cols]; returns float32 [tokens, rows] each."""
+    lib = load_library()
+    tokens = acts[0].shape[0]
+    if any(not 1 <= k <= p.n_stages for p in pkgs):
+        raise ValueError("k exceeds the stages of a package")
+    if any(A.shape[0] != tokens for A in acts):
+        raise ValueError("every activation matrix must have the same number of tokens")
+    if ys is None:
+        ys = [torch.empty((tokens, p.rows), dtype=torch.float32, device=p.codes[0].device) for p in pkgs]
+    if items is None:
+        items = gemv_descs(pkgs, acts, ys, k)
+    fmt = pkgs[0].format()
+    rc = lib.rrq_prefill(items, len(items), ctypes.byref(fmt), k, tokens, _stream_handle(stream))
+    if rc != 0:
+        raise RRQError(rc, "rrq_prefill")
     return ys
 
 

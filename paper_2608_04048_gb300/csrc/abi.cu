@@ -501,6 +501,119 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
   return RRQ_OK;
 }
 
+// The driver's tensor-map encoder, looked up once through the runtime (no
+// link against the driver library).
+using EncodeTiledFn = CUresult (*)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*, const cuuint64_t*,
+                                   const cuuint64_t*, const cuuint32_t*, const cuuint32_t*, CUtensorMapInterleave,
+                                   CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn encode_tiled() {
+  static EncodeTiledFn fn = [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<EncodeTiledFn>(nullptr);
+    return reinterpret_cast<EncodeTiledFn>(ptr);
+  }();
+  return fn;
+}
+
+// Activations [tokens, cols] bf16 as a 2-D tensor map: boxes of 64 columns x
+// kPrefillBN tokens, 128-byte swizzle (the MMA's K-major operand layout),
+// zeros outside the matrix.
+bool encode_activations(CUtensorMap* map, const uint16_t* A, int64_t tokens, int64_t cols) {
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn) return false;
+  const cuuint64_t dim[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(tokens)};
+  const cuuint64_t stride[1] = {static_cast<cuuint64_t>(cols) * 2};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(rrq::kPrefillBK), static_cast<cuuint32_t>(rrq::kPrefillBN)};
+  const cuuint32_t estride[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(A), dim, stride, box, estride,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k, int64_t tokens,
+                         rrq_stream_t stream) {
+  if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
+  if (tokens < 1 || tokens > RRQ_MAX_PREFILL_TOKENS) return RRQ_ERR_INVALID_ARG;
+  if (f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
+  const int group = f.group;
+  std::vector<Range> ranges;
+  ranges.reserve(static_cast<size_t>(count) * (2 + 3 * k));
+  for (int i = 0; i < count; ++i) {
+    const rrq_gemv_desc& it = items[i];
+    if (!shape_ok(it.rows, it.cols) || it.cols % group != 0 || !it.A_bf16 || !it.Y) return RRQ_ERR_INVALID_ARG;
+    if (it.cols > (int64_t{1} << 31) - rrq::kPrefillBK) return RRQ_ERR_INVALID_ARG;
+    for (int j = 0; j < k; ++j)
+      if (!it.codes[j] || !it.scales[j] || (!f.sym() && !it.zeros[j])) return RRQ_ERR_INVALID_ARG;
+    if (!aligned(it.A_bf16, 16) || !aligned(it.Y, 16)) return RRQ_ERR_MISALIGNED;
+    for (int j = 0; j < k; ++j)
+      if (!aligned(it.codes[j], 16) || !aligned(it.scales[j], 16) || (!f.sym() && !aligned(it.zeros[j], 16)))
+        return RRQ_ERR_MISALIGNED;
+    const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
+    ranges.push_back(range_of(it.A_bf16, 2 * static_cast<uint64_t>(tokens) * it.cols, false));
+    ranges.push_back(range_of(it.Y, 4 * static_cast<uint64_t>(tokens) * it.rows, true));
+    for (int j = 0; j < k; ++j) {
+      ranges.push_back(range_of(it.codes[j], n / 4, false));
+      ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
+      if (!f.sym()) ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
+    }
+  }
+  if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
+
+  int dev = 0;
+  DeviceState* st = nullptr;
+  if (rrq_status rc = current_device(&dev, &st)) return rc;
+  for (int i = 0; i < count; ++i) {
+    const rrq_gemv_desc& it = items[i];
+    if (!on_device(it.A_bf16, dev) || !on_device(it.Y, dev)) return RRQ_ERR_INVALID_ARG;
+    for (int j = 0; j < k; ++j)
+      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) ||
+          (!f.sym() && !on_device(it.zeros[j], dev)))
+        return RRQ_ERR_INVALID_ARG;
+  }
+
+  int log2g = 0;
+  while ((1 << log2g) < group) ++log2g;
+  const int64_t token_tiles = (tokens + rrq::kPrefillBN - 1) / rrq::kPrefillBN;
+  static thread_local rrq::PrefillBatch p;
+  for (int base = 0; base < count; base += rrq::kMaxPrefillBatch) {
+    const int m = std::min(rrq::kMaxPrefillBatch, count - base);
+    std::memset(&p, 0, sizeof p);
+    p.count = m;
+    p.log2g = log2g;
+    p.tokens = tokens;
+    p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
+    p.status = st->status;
+    int64_t tiles = 0;
+    for (int i = 0; i < m; ++i) {
+      const rrq_gemv_desc& it = items[base + i];
+      rrq::PrefillItem& q = p.item[i];
+      for (int j = 0; j < rrq::kMaxStages; ++j) {
+        const int jj = j < k ? j : k - 1;
+        q.codes[j] = it.codes[jj];
+        q.scales[j] = it.scales[jj];
+        q.zeros[j] = f.sym() ? nullptr : it.zeros[jj];
+      }
+      q.Y = it.Y;
+      q.rows = it.rows;
+      q.cols = it.cols;
+      q.tile_begin = tiles;
+      q.token_tiles = static_cast<int32_t>(token_tiles);
+      tiles += (it.rows + rrq::kPrefillBM - 1) / rrq::kPrefillBM * token_tiles;
+      if (!encode_activations(&p.act[i], it.A_bf16, tokens, it.cols)) return RRQ_ERR_UNSUPPORTED;
+    }
+    if (tiles > 0x7fffffff) return RRQ_ERR_INVALID_ARG;
+    p.total_tiles = tiles;
+    cudaError_t e = rrq::prefill_launch(f.kind, k, p, reinterpret_cast<cudaStream_t>(stream));
+    if (e != cudaSuccess) return fail_cuda(e);
+  }
+  return RRQ_OK;
+}
+
 rrq_status pmr_batch(const rrq_pmr_desc* items, int count, int group, rrq_stream_t stream) {
   if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
   if (!group_supported(group)) return RRQ_ERR_UNSUPPORTED;
@@ -691,6 +804,13 @@ rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt
   Fmt f;
   if (rrq_status rc = parse_format(fmt, &f)) return rc;
   return gemv_batch(items, count, f, k, batch, stream);
+}
+
+rrq_status rrq_prefill(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int64_t tokens,
+                       rrq_stream_t stream) {
+  Fmt f;
+  if (rrq_status rc = parse_format(fmt, &f)) return rc;
+  return prefill_batch(items, count, f, k, tokens, stream);
 }
 
 rrq_status rrq_reconstruct_ex(const rrq_reconstruct_desc* items, int count, const rrq_format* fmt,

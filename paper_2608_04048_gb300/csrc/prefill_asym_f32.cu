@@ -1,0 +1,11 @@
+// Tensor-core prefill product for the asym f32 package format (see
+// prefill_kernel.cuh).
+#include "prefill_kernel.cuh"
+
+namespace rrq {
+
+cudaError_t prefill_launch_asym_f32(int k, const PrefillBatch& p, cudaStream_t stream) {
+  return prefill_launch_f<kAsymF32>(k, p, stream);
+}
+
+}  // namespace rrq

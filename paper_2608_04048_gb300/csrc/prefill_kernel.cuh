@@ -1,0 +1,369 @@
+// Prefill form of the stage-wise product (Appendix C, A W~_(t) = A W^_0 +
+// sum_k A R^_k, for many activation rows) on the fifth-generation tensor
+// cores:
+//
+//     Y[t][r] = sum_c A[t][c] * bf16(W~_k)[r][c]
+//
+// with bf16(W~_k) the prefix-k reconstruction (Eq. 8: acc = L_0; acc =
+// fl(acc + L_i); bf16 round to nearest-even), formed from the package inside
+// the kernel and never written to memory.  The tensor cores take bf16
+// operands, so the weight is the reconstruction exactly as rrq_reconstruct
+// returns it; products are accumulated in binary32 in tensor memory.
+//
+// One CTA computes a tile of 128 weight rows x 256 tokens (one
+// tcgen05.mma.cta_group::1.kind::f16 shape, M = 128, N = 256, K = 16) over
+// the whole K range, in stages of 64 columns through a 4-deep shared-memory
+// ring:
+//   - warp 8 loads the activation tile of a stage (256 tokens x 64 columns,
+//     bf16) with one 2-D TMA copy (128-byte swizzle);
+//   - warps 0-7 read the package words of the stage (codes, scales, zeros),
+//     form the 128 x 64 bf16 weight tile in registers and store it in the
+//     same K-major 128-byte-swizzled layout, then signal the stage;
+//   - one thread of warp 9 issues the four MMAs of the stage and commits
+//     them to the stage's "empty" barrier, which releases its buffers;
+//   - after the last stage warps 0-7 read the accumulator (tcgen05.ld, one
+//     TMEM lane = one weight row) and store Y with coalesced binary32 stores.
+// Every wait is bounded in wall time; on expiry the kernel sets the status
+// word, drains its own copies and MMAs (bounded) and frees its tensor memory.
+#pragma once
+
+#include <cuda_bf16.h>
+#include <cuda_fp16.h>
+
+#include "rrq_device.cuh"
+
+namespace rrq {
+namespace {
+
+constexpr int kPfStages = 4;                         // pipeline depth
+constexpr int kPfWTileBytes = kPrefillBM * 128;      // 128 rows x 64 bf16 (16 KiB)
+constexpr int kPfATileBytes = kPrefillBN * 128;      // 256 tokens x 64 bf16 (32 KiB)
+constexpr int kPfDqWarps = 8;                        // weight tiles, then the epilogue
+constexpr int kPfTmaWarp = 8;
+constexpr int kPfMmaWarp = 9;
+constexpr int kPfThreads = 10 * 32;
+constexpr uint32_t kPfTmemCols = kPrefillBN;         // binary32 accumulator, 128 lanes x 256 columns
+constexpr int kPfBarOffset = kPfStages * (kPfWTileBytes + kPfATileBytes);
+constexpr int kPfBars = 3 * kPfStages + 2;           // full_a, full_w, empty per stage; acc_full; drain
+constexpr int kPfSmemBytes = kPfBarOffset + 8 * kPfBars + 16 + 1024;  // + TMEM address, alignment slack
+
+// Instruction descriptor of tcgen05.mma .kind::f16: D binary32 (bits 4-5),
+// A and B bf16 (bits 7-9, 10-12), both K-major (bits 15, 16 clear),
+// N >> 3 at bits 17-22, M >> 4 at bits 24-28.
+constexpr uint32_t kPfIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
+                              (static_cast<uint32_t>(kPrefillBN >> 3) << 17) |
+                              (static_cast<uint32_t>(kPrefillBM >> 4) << 24);
+
+// Shared-memory matrix descriptor of a K-major tile with 128-byte swizzle:
+// rows 128 bytes apart, 8-row groups 1024 bytes apart (stride byte offset),
+// the tile base 1024-byte aligned (base offset 0), descriptor version 1,
+// layout type 2 (128-byte swizzle) in bits 61-63.  The leading byte offset
+// is not used by this layout (one swizzle row spans the MMA's K).
+__device__ __forceinline__ uint64_t sw128_desc(uint32_t saddr) {
+  return static_cast<uint64_t>((saddr & 0x3FFFFu) >> 4) | (static_cast<uint64_t>(1) << 16) |
+         (static_cast<uint64_t>(1024 >> 4) << 32) | (static_cast<uint64_t>(1) << 46) |
+         (static_cast<uint64_t>(2) << 61);
+}
+
+__device__ __forceinline__ void tmem_alloc(uint32_t slot, uint32_t ncols) {
+  asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(slot), "r"(ncols)
+               : "memory");
+}
+__device__ __forceinline__ void tmem_relinquish() {
+  asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void tmem_dealloc(uint32_t taddr, uint32_t ncols) {
+  asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(taddr), "r"(ncols) : "memory");
+}
+__device__ __forceinline__ void tc_fence_before() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void tc_fence_after() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+// D (tensor memory) = A B^T (+ D if acc != 0), A and B from shared memory.
+__device__ __forceinline__ void mma_bf16(uint32_t d, uint64_t a, uint64_t b, uint32_t idesc, uint32_t acc) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d),
+      "l"(a), "l"(b), "r"(idesc), "r"(acc)
+      : "memory");
+}
+// Arrives on `bar` once every MMA issued so far by this thread has completed.
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+// 2-D tiled TMA load: box at (x = column, y = row) of `map`, completing on `bar`.
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(x), "r"(y), "r"(bar)
+      : "memory");
+}
+// 32 consecutive binary32 columns of this thread's tensor-memory lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0, %1, %2, %3, %4, %5, %6, %7, %8, %9, %10, %11, %12, %13, %14, "
+      "%15, %16, %17, %18, %19, %20, %21, %22, %23, %24, %25, %26, %27, %28, %29, %30, %31}, [%32];"
+      : "=r"(v[0]), "=r"(v[1]), "=r"(v[2]), "=r"(v[3]), "=r"(v[4]), "=r"(v[5]), "=r"(v[6]), "=r"(v[7]),
+        "=r"(v[8]), "=r"(v[9]), "=r"(v[10]), "=r"(v[11]), "=r"(v[12]), "=r"(v[13]), "=r"(v[14]), "=r"(v[15]),
+        "=r"(v[16]), "=r"(v[17]), "=r"(v[18]), "=r"(v[19]), "=r"(v[20]), "=r"(v[21]), "=r"(v[22]), "=r"(v[23]),
+        "=r"(v[24]), "=r"(v[25]), "=r"(v[26]), "=r"(v[27]), "=r"(v[28]), "=r"(v[29]), "=r"(v[30]), "=r"(v[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+// bf16 prefix-k weights of 32 consecutive weights of one row (one group):
+// cw[i] holds their stage-i codes (LSB first, 2 bits each), sc/zr the
+// group's stage-i scale and zero.  Same operations, in the same order, as the
+// reconstruction kernel's general path, so the values are bit-identical.
+template <int F, int K>
+__device__ __forceinline__ void prefix_weights_bf16(const uint2 (&cw)[K], const float (&sc)[K], const float (&zr)[K],
+                                                    uint32_t (&h)[16]) {
+  constexpr bool kSym = F == kSymF32 || F == kSymF16;
+  f32x2 acc[16];
+#pragma unroll
+  for (int i = 0; i < K; ++i) {
+    const f32x2 S = pack2(sc[i], sc[i]);
+    if constexpr (kSym) {
+      const f32x2 K2 = pack2(8388608.0f + 2.0f, 8388608.0f + 2.0f);
+#pragma unroll
+      for (int m = 0; m < 16; ++m) {
+        const uint32_t word = m < 8 ? cw[i].x : cw[i].y;
+        const int sh = 4 * (m & 7);
+        // Q - 2, exact; (Q - 2) s is exact, so the fma rounds only the sum
+        const f32x2 u = sub2(pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u)), K2);
+        acc[m] = (i == 0) ? mul2(u, S) : fma2(u, S, acc[m]);
+      }
+    } else {
+      const f32x2 LO = pack2(zr[i], zr[i]), Z = pack2(0.0f, 0.0f);
+      const f32x2 T23 = pack2(8388608.0f, 8388608.0f);
+#pragma unroll
+      for (int m = 0; m < 16; ++m) {
+        const uint32_t word = m < 8 ? cw[i].x : cw[i].y;
+        const int sh = 4 * (m & 7);
+        const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+        // fl(zero + fl(Q s)): the product rounded on its own (fma, zero addend)
+        const f32x2 level = add2(LO, fma2(sub2(t, T23), S, Z));
+        acc[m] = (i == 0) ? level : add2(acc[m], level);
+      }
+    }
+  }
+#pragma unroll
+  for (int m = 0; m < 16; ++m) {
+    float a, b;
+    unpack2(acc[m], a, b);
+    const __nv_bfloat162 x = __floats2bfloat162_rn(a, b);
+    h[m] = *reinterpret_cast<const uint32_t*>(&x);
+  }
+}
+
+template <int F, int K>
+__global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_constant__ PrefillBatch p) {
+  extern __shared__ uint8_t smem_raw[];
+  const uint32_t raw_s = smem_u32(smem_raw);
+  const uint32_t base_s = (raw_s + 1023u) & ~1023u;  // swizzled tiles need 1024-byte alignment
+  uint8_t* const base = smem_raw + (base_s - raw_s);
+  const uint32_t w_s = base_s;                              // weight tiles
+  const uint32_t a_s = base_s + kPfStages * kPfWTileBytes;  // activation tiles
+  const uint32_t bar_s = base_s + kPfBarOffset;
+  const uint32_t acc_full = bar_s + 8 * (3 * kPfStages);
+  const uint32_t drain = acc_full + 8;
+  const uint32_t slot_s = bar_s + 8 * kPfBars;
+  const volatile uint32_t* slot = reinterpret_cast<const volatile uint32_t*>(base + kPfBarOffset + 8 * kPfBars);
+  auto full_a = [&](int s) { return bar_s + 8 * s; };
+  auto full_w = [&](int s) { return bar_s + 8 * (kPfStages + s); };
+  auto empty = [&](int s) { return bar_s + 8 * (2 * kPfStages + s); };
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+
+  // this CTA's tile
+  const int64_t tile = blockIdx.x;
+  int mi = 0;
+  while (mi + 1 < p.count && tile >= p.item[mi + 1].tile_begin) ++mi;
+  const PrefillItem& it = p.item[mi];
+  const int64_t j = tile - it.tile_begin;
+  const int64_t row0 = (j / it.token_tiles) * kPrefillBM;
+  const int64_t t0 = (j % it.token_tiles) * kPrefillBN;
+  const int nk = static_cast<int>((it.cols + kPrefillBK - 1) / kPrefillBK);
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < kPfStages; ++s) {
+      mbar_init(full_a(s), 1);
+      mbar_init(full_w(s), kPfDqWarps);
+      mbar_init(empty(s), 1);
+    }
+    mbar_init(acc_full, 1);
+    mbar_init(drain, 1);
+    fence_mbarrier_init();
+  }
+  if (warp == kPfMmaWarp) {
+    tmem_alloc(slot_s, kPfTmemCols);
+    tmem_relinquish();
+  }
+  tc_fence_before();
+  __syncthreads();
+  tc_fence_after();
+  const uint32_t tmem = *slot;
+
+  if (warp == kPfTmaWarp) {
+    if (lane == 0) {
+      bool ok = true;
+      int issued = 0;
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % kPfStages;
+        if (kb >= kPfStages && !mbar_wait(empty(s), ((kb / kPfStages) - 1) & 1, p.wait_limit_us)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(full_a(s), kPfATileBytes);
+        tma_load_2d(a_s + s * kPfATileBytes, &p.act[mi], kb * kPrefillBK, static_cast<int>(t0), full_a(s));
+        ++issued;
+      }
+      if (!ok) {  // let this thread's copies land before the CTA can leave
+        atomicOr(p.status, kStatusTimeout);
+        for (int kb = issued > kPfStages ? issued - kPfStages : 0; kb < issued; ++kb)
+          mbar_wait(full_a(kb % kPfStages), (kb / kPfStages) & 1, kDrainLimitUs);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kPfMmaWarp) {
+    if (lane == 0) {
+      bool ok = true;
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % kPfStages;
+        const uint32_t ph = (kb / kPfStages) & 1;
+        if (!mbar_wait(full_a(s), ph, p.wait_limit_us) || !mbar_wait(full_w(s), ph, p.wait_limit_us)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t wa = w_s + s * kPfWTileBytes, aa = a_s + s * kPfATileBytes;
+#pragma unroll
+        for (int kk = 0; kk < kPrefillBK / 16; ++kk)  // K = 16 per MMA: 32 bytes along the swizzle row
+          mma_bf16(tmem, sw128_desc(wa + 32 * kk), sw128_desc(aa + 32 * kk), kPfIdesc, (kb | kk) != 0);
+        mma_commit(empty(s));
+      }
+      if (ok) {
+        mma_commit(acc_full);
+      } else {  // no MMA may be in flight when the tensor memory is freed
+        atomicOr(p.status, kStatusTimeout);
+        mma_commit(drain);
+        mbar_wait(drain, 0, kDrainLimitUs);
+      }
+    }
+    __syncwarp();
+  } else {  // warps 0-7: weight tiles, then the epilogue
+    const int rl = threadIdx.x & (kPrefillBM - 1);  // tile row
+    const int half = threadIdx.x >> 7;               // columns 32 * half .. + 31 of a stage
+    const int64_t r = row0 + rl;
+    bool ok = true;
+    for (int kb = 0; kb < nk; ++kb) {
+      const int s = kb % kPfStages;
+      const int64_t c0 = static_cast<int64_t>(kb) * kPrefillBK + 32 * half;
+      const bool valid = r < it.rows && c0 < it.cols;
+      uint2 cw[K];
+      float sc[K], zr[K];
+#pragma unroll
+      for (int i = 0; i < K; ++i) {
+        cw[i] = make_uint2(0u, 0u);
+        sc[i] = 0.0f;
+        zr[i] = 0.0f;
+      }
+      if (valid) {  // 32 weights inside one group (group >= 32, c0 % 32 == 0)
+        const int64_t e = r * it.cols + c0;
+        const int64_t g = e >> p.log2g;
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+          cw[i] = __ldg(reinterpret_cast<const uint2*>(it.codes[i] + (e >> 2)));
+          if constexpr (F == kSymF16)
+            sc[i] = __half2float(__ushort_as_half(__ldg(static_cast<const unsigned short*>(it.scales[i]) + g)));
+          else
+            sc[i] = __ldg(static_cast<const float*>(it.scales[i]) + g);
+          if constexpr (F == kAsymF32) zr[i] = __ldg(it.zeros[i] + g);
+        }
+      }
+      // the MMAs of this stage's previous round have read its weight tile
+      bool ready = true;
+      if (kb >= kPfStages) ready = mbar_wait(empty(s), ((kb / kPfStages) - 1) & 1, p.wait_limit_us);
+      if (!__all_sync(kFullMask, ready)) {
+        ok = false;
+        break;
+      }
+      uint32_t h[16];
+      if (valid) {
+        prefix_weights_bf16<F, K>(cw, sc, zr, h);
+      } else {
+#pragma unroll
+        for (int m = 0; m < 16; ++m) h[m] = 0u;
+      }
+      // K-major, 128-byte swizzle: 16-byte piece c of row rl at piece c ^ (rl % 8)
+      uint8_t* const wrow = base + s * kPfWTileBytes + (rl >> 3) * 1024 + (rl & 7) * 128;
+#pragma unroll
+      for (int q = 0; q < 4; ++q) {
+        const int piece = (4 * half + q) ^ (rl & 7);
+        *reinterpret_cast<uint4*>(wrow + 16 * piece) = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
+      }
+      fence_proxy_async_smem();  // visible to the tensor cores (async proxy)
+      __syncwarp();
+      if (lane == 0) mbar_arrive(full_w(s));
+    }
+    bool have = false;
+    if (ok) have = mbar_wait(acc_full, 0, p.wait_limit_us);
+    have = __all_sync(kFullMask, have);
+    if (!have && lane == 0) atomicOr(p.status, kStatusTimeout);
+    tc_fence_after();
+    if (have) {
+      const int quarter = warp & 3;  // TMEM lanes 32 * quarter .. + 31 of this warp
+      const int cols_half = warp >> 2;
+      const int64_t row = row0 + 32 * quarter + lane;
+#pragma unroll 1
+      for (int c = 0; c < kPrefillBN / 2 / 32; ++c) {
+        const int col = cols_half * (kPrefillBN / 2) + 32 * c;
+        uint32_t v[32];
+        tmem_ld32(tmem + (static_cast<uint32_t>(32 * quarter) << 16) + static_cast<uint32_t>(col), v);
+        if (row < it.rows) {
+          const int64_t tb = t0 + col;
+          float* y = it.Y + tb * it.rows + row;
+#pragma unroll
+          for (int q = 0; q < 32; ++q)
+            if (tb + q < p.tokens) y[q * it.rows] = __uint_as_float(v[q]);
+        }
+      }
+    }
+  }
+  tc_fence_before();
+  __syncthreads();
+  if (warp == kPfMmaWarp) {
+    tc_fence_after();
+    tmem_dealloc(tmem, kPfTmemCols);
+  }
+}
+
+template <int F, int K>
+cudaError_t prefill_launch_k(const PrefillBatch& p, cudaStream_t stream) {
+  // (per launch: the attribute belongs to the current device)
+  cudaError_t e = cudaFuncSetAttribute(prefill_kernel<F, K>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPfSmemBytes);
+  if (e != cudaSuccess) return e;
+  prefill_kernel<F, K><<<static_cast<unsigned>(p.total_tiles), kPfThreads, kPfSmemBytes, stream>>>(p);
+  return cudaGetLastError();
+}
+
+template <int F>
+cudaError_t prefill_launch_f(int k, const PrefillBatch& p, cudaStream_t stream) {
+  switch (k) {
+    case 1: return prefill_launch_k<F, 1>(p, stream);
+    case 2: return prefill_launch_k<F, 2>(p, stream);
+    case 3: return prefill_launch_k<F, 3>(p, stream);
+    case 4: return prefill_launch_k<F, 4>(p, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+}  // namespace
+}  // namespace rrq

@@ -4,6 +4,7 @@
 #pragma once
 
 #include <cstdint>
+#include <cuda.h>  // CUtensorMap (the type only; no driver call is linked)
 #include <cuda_runtime.h>
 
 namespace rrq {
@@ -95,6 +96,50 @@ struct GemvBatch {
 constexpr int kGemvRows = 16;      // rows per block
 
 constexpr int kMaxGemvBatch = 8;   // activation rows (tokens) per call
+
+// One matrix of a prefill launch: Y = A bf16(W~)^T on the tensor cores, with
+// bf16(W~) the prefix-k reconstruction formed from the package in the
+// kernel.  A matrix is cut into tiles of kPrefillBM weight rows by
+// kPrefillBN tokens; the tiles of all matrices of a launch are numbered
+// consecutively (one CTA each) and tile_begin is this matrix's first.
+struct PrefillItem {
+  const uint8_t* codes[kMaxStages];
+  const void* scales[kMaxStages];  // float or binary16
+  const float* zeros[kMaxStages];  // asymmetric grid only
+  float* Y;                        // [tokens, rows]
+  int64_t rows, cols;
+  int64_t tile_begin;
+  int32_t token_tiles;
+};
+
+constexpr int kPrefillBM = 128;       // weight rows per tile (TMEM lanes, MMA M)
+constexpr int kPrefillBN = 256;       // tokens per tile (MMA N, TMEM columns)
+constexpr int kPrefillBK = 64;        // columns per pipeline stage (one 128-byte swizzle row)
+constexpr int kMaxPrefillBatch = 16;  // matrices per launch
+
+struct PrefillBatch {  // (64-byte aligned through its tensor maps)
+  CUtensorMap act[kMaxPrefillBatch];  // activations [tokens, cols] bf16: box 64 x 256, 128-byte swizzle
+  PrefillItem item[kMaxPrefillBatch];
+  int count;
+  int log2g;                          // group = 1 << log2g
+  int64_t tokens;
+  int64_t total_tiles;
+  uint32_t wait_limit_us;
+  unsigned* status;
+};
+
+cudaError_t prefill_launch_asym_f32(int k, const PrefillBatch& p, cudaStream_t stream);
+cudaError_t prefill_launch_sym_f32(int k, const PrefillBatch& p, cudaStream_t stream);
+cudaError_t prefill_launch_sym_f16(int k, const PrefillBatch& p, cudaStream_t stream);
+
+inline cudaError_t prefill_launch(Format fmt, int k, const PrefillBatch& p, cudaStream_t stream) {
+  switch (fmt) {
+    case kAsymF32: return prefill_launch_asym_f32(k, p, stream);
+    case kSymF32: return prefill_launch_sym_f32(k, p, stream);
+    case kSymF16: return prefill_launch_sym_f16(k, p, stream);
+    default: return cudaErrorInvalidValue;
+  }
+}
 
 // One matrix of a group peak-to-mean ratio launch.
 struct PmrItem {
