@@ -168,6 +168,45 @@ def time_gemv(pkgs, specs, stream, batch: int = 1, reps: int = 5) -> dict:
     return out
 
 
+def time_prefill(pkgs, specs, stream, tokens: int = 2048, reps: int = 2) -> dict:
+    """Prefill product over the whole stack (Appendix C's product for many
+    activation rows, on the tensor cores): rrq_prefill of each layer's 7
+    packages (one call per layer, buffers shared by the layers) with `tokens`
+    activation rows, at prefix k = 1..4, timed with CUDA events.  Work: 2 x
+    tokens x rows x cols flops per matrix, against the measured bf16 dense
+    peak (burst: the calls are timed alone)."""
+    from paper_2608_04048_gb300 import binding
+    dev = pkgs[0].codes[0].device
+    per = 7
+    layers = [list(range(i, min(i + per, len(specs)))) for i in range(0, len(specs), per)]
+    gen = torch.Generator(device=dev).manual_seed(78)
+    acts = [torch.randn((tokens, specs[j].cols), generator=gen, device=dev).to(torch.bfloat16) for j in layers[0]]
+    ys = [torch.empty((tokens, specs[j].rows), dtype=torch.float32, device=dev) for j in layers[0]]
+    peak = measured_peaks().get("bf16_tflops") or 1900.0
+    flops = 2.0 * tokens * sum(sp.numel for sp in specs)
+    out = {"call": f"rrq_prefill over all {len(specs)} matrices, {tokens} tokens, one call per layer "
+                   "(asymmetric binary32 package)", "tokens": tokens, "peak_tflops": peak}
+    for k in KS:
+        items = [binding.gemv_descs([pkgs[j] for j in L], acts[:len(L)], ys[:len(L)], k) for L in layers]
+
+        def run():
+            for L, it in zip(layers, items):
+                binding.rrq_prefill([pkgs[j] for j in L], acts[:len(L)], k, ys[:len(L)], stream, it)
+        run()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            run()
+        b.record(stream)
+        torch.cuda.synchronize()
+        t = a.elapsed_time(b) / reps / 1e3
+        out[f"k{k}"] = {"s_per_stack": round(t, 6), "tflops": round(flops / t / 1e12, 1),
+                        "frac_of_measured_bf16": round(flops / t / 1e12 / peak, 4)}
+    if binding.rrq_get_device_status() != 0:
+        raise RuntimeError("a kernel reported a timeout (prefill)")
+    return out
+
+
 def time_bits(mats, p_outs, specs, stream, bits, reps: int = 3) -> dict:
     """A heterogeneous-width package of the same stack (asymmetric grid,
     stage widths `bits`): rrq_quantize_ex and all-prefix rrq_reconstruct_ex,
@@ -437,6 +476,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
     sym = time_sym_f16(mats, p_outs, specs, stream) if not args.no_sym else None
     from_base = time_from_base(mats, pkgs, specs, stream) if not args.no_sym else None
     gemv = time_gemv(pkgs, specs, stream) if not args.no_sym else None
+    prefill = time_prefill(pkgs, specs, stream) if not args.no_sym else None
     bits = {"+".join(map(str, b)): time_bits(mats, p_outs, specs, stream, b) for b in ((1, 3), (3, 1))} \
         if not args.no_sym else None
     pmr = time_pmr(mats, specs, stream) if not args.no_sym else None
@@ -504,6 +544,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "sym_f16": sym,
             "from_base": from_base,
             "gemv_decode": gemv,
+            "prefill": prefill,
             "widths": bits,
             "group_pmr": pmr,
         },

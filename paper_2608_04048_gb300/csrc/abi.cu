@@ -521,14 +521,14 @@ EncodeTiledFn encode_tiled() {
 }
 
 // Activations [tokens, cols] bf16 as a 2-D tensor map: boxes of 64 columns x
-// kPrefillBN tokens, 128-byte swizzle (the MMA's K-major operand layout),
+// kPrefillMmaN tokens, 128-byte swizzle (the MMA's K-major operand layout),
 // zeros outside the matrix.
 bool encode_activations(CUtensorMap* map, const uint16_t* A, int64_t tokens, int64_t cols) {
   EncodeTiledFn fn = encode_tiled();
   if (!fn) return false;
   const cuuint64_t dim[2] = {static_cast<cuuint64_t>(cols), static_cast<cuuint64_t>(tokens)};
   const cuuint64_t stride[1] = {static_cast<cuuint64_t>(cols) * 2};
-  const cuuint32_t box[2] = {static_cast<cuuint32_t>(rrq::kPrefillBK), static_cast<cuuint32_t>(rrq::kPrefillBN)};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(rrq::kPrefillBK), static_cast<cuuint32_t>(rrq::kPrefillMmaN)};
   const cuuint32_t estride[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(A), dim, stride, box, estride,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
@@ -601,9 +601,10 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
       q.Y = it.Y;
       q.rows = it.rows;
       q.cols = it.cols;
+      const int64_t row_tiles = (it.rows + rrq::kPrefillBM - 1) / rrq::kPrefillBM;
       q.tile_begin = tiles;
-      q.token_tiles = static_cast<int32_t>(token_tiles);
-      tiles += (it.rows + rrq::kPrefillBM - 1) / rrq::kPrefillBM * token_tiles;
+      q.row_tiles = static_cast<int32_t>(row_tiles);
+      tiles += row_tiles * token_tiles;
       if (!encode_activations(&p.act[i], it.A_bf16, tokens, it.cols)) return RRQ_ERR_UNSUPPORTED;
     }
     if (tiles > 0x7fffffff) return RRQ_ERR_INVALID_ARG;

@@ -55,10 +55,6 @@ constexpr float kTwo23 = 8388608.0f;
 template <int K>
 __host__ __device__ constexpr int ring_bytes() { return kWarps * ring_depth<K>() * K * kStageBytes; }
 
-__device__ __forceinline__ bool prescale_ok(float s) {
-  return s == 0.0f || (s >= 0x1p-100f && s <= 0x1p+100f);
-}
-
 // swizzled position of 16-byte activation piece P of a row
 __device__ __forceinline__ uint32_t act_piece(uint32_t P) { return P ^ ((P >> 3) & 7u); }
 

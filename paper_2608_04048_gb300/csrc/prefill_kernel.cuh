@@ -10,18 +10,20 @@
 // operands, so the weight is the reconstruction exactly as rrq_reconstruct
 // returns it; products are accumulated in binary32 in tensor memory.
 //
-// One CTA computes a tile of 128 weight rows x 256 tokens (one
-// tcgen05.mma.cta_group::1.kind::f16 shape, M = 128, N = 256, K = 16) over
-// the whole K range, in stages of 64 columns through a 4-deep shared-memory
-// ring:
-//   - warp 8 loads the activation tile of a stage (256 tokens x 64 columns,
-//     bf16) with one 2-D TMA copy (128-byte swizzle);
-//   - warps 0-7 read the package words of the stage (codes, scales, zeros),
-//     form the 128 x 64 bf16 weight tile in registers and store it in the
-//     same K-major 128-byte-swizzled layout, then signal the stage;
-//   - one thread of warp 9 issues the four MMAs of the stage and commits
-//     them to the stage's "empty" barrier, which releases its buffers;
-//   - after the last stage warps 0-7 read the accumulator (tcgen05.ld, one
+// One CTA computes a tile of 128 weight rows x 512 tokens: two accumulators
+// of tcgen05.mma.cta_group::1.kind::f16 shape M = 128, N = 256 (K = 16 per
+// instruction), which fill the 512 columns of tensor memory, so every weight
+// tile formed from the package serves 512 tokens.  The K range is walked in
+// stages of 64 columns:
+//   - warp 8 loads the activation tile of a stage (512 tokens x 64 columns,
+//     bf16, two 2-D TMA boxes, 128-byte swizzle) into a 2-deep ring;
+//   - warps 0-7 read the package words of the stage one stage ahead (codes,
+//     scales, zeros), form the 128 x 64 bf16 weight tile in registers and
+//     store it in the same K-major 128-byte-swizzled layout into a 4-deep
+//     ring, then signal the stage;
+//   - one thread of warp 9 issues the MMAs of the stage and commits them to
+//     the two rings' "empty" barriers, which release the buffers;
+//   - after the last stage warps 0-7 read the accumulators (tcgen05.ld, one
 //     TMEM lane = one weight row) and store Y with coalesced binary32 stores.
 // Every wait is bounded in wall time; on expiry the kernel sets the status
 // word, drains its own copies and MMAs (bounded) and frees its tensor memory.
@@ -35,23 +37,26 @@
 namespace rrq {
 namespace {
 
-constexpr int kPfStages = 4;                         // pipeline depth
+constexpr int kPfWStages = 4;                        // weight-tile ring depth
+constexpr int kPfAStages = 2;                        // activation-tile ring depth
 constexpr int kPfWTileBytes = kPrefillBM * 128;      // 128 rows x 64 bf16 (16 KiB)
-constexpr int kPfATileBytes = kPrefillBN * 128;      // 256 tokens x 64 bf16 (32 KiB)
+constexpr int kPfAHalfBytes = kPrefillMmaN * 128;    // 256 tokens x 64 bf16 (32 KiB)
+constexpr int kPfATileBytes = 2 * kPfAHalfBytes;     // 512 tokens (64 KiB)
 constexpr int kPfDqWarps = 8;                        // weight tiles, then the epilogue
 constexpr int kPfTmaWarp = 8;
 constexpr int kPfMmaWarp = 9;
 constexpr int kPfThreads = 10 * 32;
-constexpr uint32_t kPfTmemCols = kPrefillBN;         // binary32 accumulator, 128 lanes x 256 columns
-constexpr int kPfBarOffset = kPfStages * (kPfWTileBytes + kPfATileBytes);
-constexpr int kPfBars = 3 * kPfStages + 2;           // full_a, full_w, empty per stage; acc_full; drain
+constexpr uint32_t kPfTmemCols = kPrefillBN;         // two binary32 accumulators, 128 lanes x 256 columns each
+constexpr int kPfBarOffset = kPfWStages * kPfWTileBytes + kPfAStages * kPfATileBytes;
+// full_w, empty_w per weight stage; full_a, empty_a per activation stage; acc_full; drain
+constexpr int kPfBars = 2 * kPfWStages + 2 * kPfAStages + 2;
 constexpr int kPfSmemBytes = kPfBarOffset + 8 * kPfBars + 16 + 1024;  // + TMEM address, alignment slack
 
 // Instruction descriptor of tcgen05.mma .kind::f16: D binary32 (bits 4-5),
 // A and B bf16 (bits 7-9, 10-12), both K-major (bits 15, 16 clear),
 // N >> 3 at bits 17-22, M >> 4 at bits 24-28.
 constexpr uint32_t kPfIdesc = (1u << 4) | (1u << 7) | (1u << 10) |
-                              (static_cast<uint32_t>(kPrefillBN >> 3) << 17) |
+                              (static_cast<uint32_t>(kPrefillMmaN >> 3) << 17) |
                               (static_cast<uint32_t>(kPrefillBM >> 4) << 24);
 
 // Shared-memory matrix descriptor of a K-major tile with 128-byte swizzle:
@@ -117,39 +122,92 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// bf16 prefix-k weights of 32 consecutive weights of one row (one group):
-// cw[i] holds their stage-i codes (LSB first, 2 bits each), sc/zr the
-// group's stage-i scale and zero.  Same operations, in the same order, as the
-// reconstruction kernel's general path, so the values are bit-identical.
+// Package words of the 32 consecutive weights (one group) a thread forms in
+// one stage.
+template <int K>
+struct PkgWords {
+  uint2 cw[K];   // stage-i codes, LSB first, 2 bits each
+  float sc[K];   // stage-i scale
+  float zr[K];   // stage-i zero (asymmetric grid)
+};
+
 template <int F, int K>
-__device__ __forceinline__ void prefix_weights_bf16(const uint2 (&cw)[K], const float (&sc)[K], const float (&zr)[K],
-                                                    uint32_t (&h)[16]) {
+__device__ __forceinline__ void load_words(const PrefillItem& it, int64_t r, int64_t c0, int log2g, bool valid,
+                                           PkgWords<K>& w) {
+#pragma unroll
+  for (int i = 0; i < K; ++i) {
+    w.cw[i] = make_uint2(0u, 0u);
+    w.sc[i] = 0.0f;
+    w.zr[i] = 0.0f;
+  }
+  if (!valid) return;
+  const int64_t e = r * it.cols + c0;
+  const int64_t g = e >> log2g;
+#pragma unroll
+  for (int i = 0; i < K; ++i) {
+    w.cw[i] = __ldg(reinterpret_cast<const uint2*>(it.codes[i] + (e >> 2)));
+    if constexpr (F == kSymF16)
+      w.sc[i] = __half2float(__ushort_as_half(__ldg(static_cast<const unsigned short*>(it.scales[i]) + g)));
+    else
+      w.sc[i] = __ldg(static_cast<const float*>(it.scales[i]) + g);
+    if constexpr (F == kAsymF32) w.zr[i] = __ldg(it.zeros[i] + g);
+  }
+}
+
+// bf16 prefix-k weights of those 32 weights: acc = L_0; acc = fl(acc + L_i);
+// bf16 nearest-even.  L_i = fl(zero + fl(Q s)) (asymmetric) or (Q - 2) s
+// (symmetric, exact).  Two evaluations of fl(Q s), both exact to the same
+// bits: with prescale_ok(s) each code stays in its bit field (value 4^j Q
+// for the j-th code of a byte) and one fma with s / 4^j and -2^23 s / 4^j
+// rounds Q s once; otherwise the code is shifted down and fma(Q, s, 0).
+template <int F, int K>
+__device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32_t (&h)[16]) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
+  constexpr float kT23 = 8388608.0f;
   f32x2 acc[16];
 #pragma unroll
   for (int i = 0; i < K; ++i) {
-    const f32x2 S = pack2(sc[i], sc[i]);
-    if constexpr (kSym) {
-      const f32x2 K2 = pack2(8388608.0f + 2.0f, 8388608.0f + 2.0f);
+    const float s = w.sc[i];
+    if (prescale_ok(s)) {
+      const f32x2 S01 = pack2(s, __fmul_rn(s, 0x1p-2f)), S23 = pack2(__fmul_rn(s, 0x1p-4f), __fmul_rn(s, 0x1p-6f));
+      const f32x2 LO = pack2(w.zr[i], w.zr[i]);
+      const f32x2 C01 = pack2(__fmul_rn(s, -0x1p23f), __fmul_rn(s, -0x1p21f));
+      const f32x2 C23 = pack2(__fmul_rn(s, -0x1p19f), __fmul_rn(s, -0x1p17f));
+      const f32x2 K01 = pack2(kT23 + 2.0f, kT23 + 8.0f), K23 = pack2(kT23 + 32.0f, kT23 + 128.0f);
 #pragma unroll
-      for (int m = 0; m < 16; ++m) {
-        const uint32_t word = m < 8 ? cw[i].x : cw[i].y;
-        const int sh = 4 * (m & 7);
-        // Q - 2, exact; (Q - 2) s is exact, so the fma rounds only the sum
-        const f32x2 u = sub2(pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u)), K2);
-        acc[m] = (i == 0) ? mul2(u, S) : fma2(u, S, acc[m]);
+      for (int j = 0; j < 8; ++j) {  // byte j: weights 4j..4j+3 (pairs 2j, 2j+1)
+        const uint32_t word = j < 4 ? w.cw[i].x : w.cw[i].y;
+        const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
+        const f32x2 t01 = pack2u(0x4B000000u | (b & 0x03u), 0x4B000000u | (b & 0x0Cu));
+        const f32x2 t23 = pack2u(0x4B000000u | (b & 0x30u), 0x4B000000u | (b & 0xC0u));
+        if constexpr (kSym) {  // 4^j (Q - 2), exact; times s / 4^j exact
+          const f32x2 u01 = sub2(t01, K01), u23 = sub2(t23, K23);
+          acc[2 * j] = (i == 0) ? mul2(u01, S01) : fma2(u01, S01, acc[2 * j]);
+          acc[2 * j + 1] = (i == 0) ? mul2(u23, S23) : fma2(u23, S23, acc[2 * j + 1]);
+        } else {
+          const f32x2 l01 = add2(LO, fma2(t01, S01, C01));
+          const f32x2 l23 = add2(LO, fma2(t23, S23, C23));
+          acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
+          acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
+        }
       }
     } else {
-      const f32x2 LO = pack2(zr[i], zr[i]), Z = pack2(0.0f, 0.0f);
-      const f32x2 T23 = pack2(8388608.0f, 8388608.0f);
+      const f32x2 S = pack2(s, s);
+      const f32x2 LO = pack2(w.zr[i], w.zr[i]), Z = pack2(0.0f, 0.0f);
+      const f32x2 T23 = pack2(kT23, kT23), K2 = pack2(kT23 + 2.0f, kT23 + 2.0f);
 #pragma unroll
       for (int m = 0; m < 16; ++m) {
-        const uint32_t word = m < 8 ? cw[i].x : cw[i].y;
+        const uint32_t word = m < 8 ? w.cw[i].x : w.cw[i].y;
         const int sh = 4 * (m & 7);
         const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
-        // fl(zero + fl(Q s)): the product rounded on its own (fma, zero addend)
-        const f32x2 level = add2(LO, fma2(sub2(t, T23), S, Z));
-        acc[m] = (i == 0) ? level : add2(acc[m], level);
+        if constexpr (kSym) {
+          const f32x2 u = sub2(t, K2);  // Q - 2, exact
+          acc[m] = (i == 0) ? mul2(u, S) : fma2(u, S, acc[m]);
+        } else {
+          // fl(zero + fl(Q s)): the product rounded on its own (fma, zero addend)
+          const f32x2 level = add2(LO, fma2(sub2(t, T23), S, Z));
+          acc[m] = (i == 0) ? level : add2(acc[m], level);
+        }
       }
     }
   }
@@ -168,35 +226,40 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   const uint32_t raw_s = smem_u32(smem_raw);
   const uint32_t base_s = (raw_s + 1023u) & ~1023u;  // swizzled tiles need 1024-byte alignment
   uint8_t* const base = smem_raw + (base_s - raw_s);
-  const uint32_t w_s = base_s;                              // weight tiles
-  const uint32_t a_s = base_s + kPfStages * kPfWTileBytes;  // activation tiles
+  const uint32_t w_s = base_s;                                // weight tiles
+  const uint32_t a_s = base_s + kPfWStages * kPfWTileBytes;   // activation tiles
   const uint32_t bar_s = base_s + kPfBarOffset;
-  const uint32_t acc_full = bar_s + 8 * (3 * kPfStages);
+  const uint32_t acc_full = bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages);
   const uint32_t drain = acc_full + 8;
   const uint32_t slot_s = bar_s + 8 * kPfBars;
   const volatile uint32_t* slot = reinterpret_cast<const volatile uint32_t*>(base + kPfBarOffset + 8 * kPfBars);
-  auto full_a = [&](int s) { return bar_s + 8 * s; };
-  auto full_w = [&](int s) { return bar_s + 8 * (kPfStages + s); };
-  auto empty = [&](int s) { return bar_s + 8 * (2 * kPfStages + s); };
+  auto full_w = [&](int s) { return bar_s + 8 * s; };
+  auto empty_w = [&](int s) { return bar_s + 8 * (kPfWStages + s); };
+  auto full_a = [&](int s) { return bar_s + 8 * (2 * kPfWStages + s); };
+  auto empty_a = [&](int s) { return bar_s + 8 * (2 * kPfWStages + kPfAStages + s); };
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // this CTA's tile
+  // this CTA's tile (token tile major)
   const int64_t tile = blockIdx.x;
   int mi = 0;
   while (mi + 1 < p.count && tile >= p.item[mi + 1].tile_begin) ++mi;
   const PrefillItem& it = p.item[mi];
   const int64_t j = tile - it.tile_begin;
-  const int64_t row0 = (j / it.token_tiles) * kPrefillBM;
-  const int64_t t0 = (j % it.token_tiles) * kPrefillBN;
+  const int64_t row0 = (j % it.row_tiles) * kPrefillBM;
+  const int64_t t0 = (j / it.row_tiles) * kPrefillBN;
+  const bool two = t0 + kPrefillMmaN < p.tokens;  // the second accumulator has tokens
   const int nk = static_cast<int>((it.cols + kPrefillBK - 1) / kPrefillBK);
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < kPfStages; ++s) {
-      mbar_init(full_a(s), 1);
+    for (int s = 0; s < kPfWStages; ++s) {
       mbar_init(full_w(s), kPfDqWarps);
-      mbar_init(empty(s), 1);
+      mbar_init(empty_w(s), 1);
+    }
+    for (int s = 0; s < kPfAStages; ++s) {
+      mbar_init(full_a(s), 1);
+      mbar_init(empty_a(s), 1);
     }
     mbar_init(acc_full, 1);
     mbar_init(drain, 1);
@@ -216,19 +279,22 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       bool ok = true;
       int issued = 0;
       for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % kPfStages;
-        if (kb >= kPfStages && !mbar_wait(empty(s), ((kb / kPfStages) - 1) & 1, p.wait_limit_us)) {
+        const int s = kb % kPfAStages;
+        if (kb >= kPfAStages && !mbar_wait(empty_a(s), ((kb / kPfAStages) - 1) & 1, p.wait_limit_us)) {
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(full_a(s), kPfATileBytes);
-        tma_load_2d(a_s + s * kPfATileBytes, &p.act[mi], kb * kPrefillBK, static_cast<int>(t0), full_a(s));
+        const uint32_t dst = a_s + s * kPfATileBytes;
+        mbar_arrive_expect_tx(full_a(s), two ? kPfATileBytes : kPfAHalfBytes);
+        tma_load_2d(dst, &p.act[mi], kb * kPrefillBK, static_cast<int>(t0), full_a(s));
+        if (two)
+          tma_load_2d(dst + kPfAHalfBytes, &p.act[mi], kb * kPrefillBK, static_cast<int>(t0 + kPrefillMmaN), full_a(s));
         ++issued;
       }
       if (!ok) {  // let this thread's copies land before the CTA can leave
         atomicOr(p.status, kStatusTimeout);
-        for (int kb = issued > kPfStages ? issued - kPfStages : 0; kb < issued; ++kb)
-          mbar_wait(full_a(kb % kPfStages), (kb / kPfStages) & 1, kDrainLimitUs);
+        for (int kb = issued > kPfAStages ? issued - kPfAStages : 0; kb < issued; ++kb)
+          mbar_wait(full_a(kb % kPfAStages), (kb / kPfAStages) & 1, kDrainLimitUs);
       }
     }
     __syncwarp();
@@ -236,18 +302,22 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     if (lane == 0) {
       bool ok = true;
       for (int kb = 0; kb < nk; ++kb) {
-        const int s = kb % kPfStages;
-        const uint32_t ph = (kb / kPfStages) & 1;
-        if (!mbar_wait(full_a(s), ph, p.wait_limit_us) || !mbar_wait(full_w(s), ph, p.wait_limit_us)) {
+        const int sw = kb % kPfWStages, sa = kb % kPfAStages;
+        if (!mbar_wait(full_a(sa), (kb / kPfAStages) & 1, p.wait_limit_us) ||
+            !mbar_wait(full_w(sw), (kb / kPfWStages) & 1, p.wait_limit_us)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t wa = w_s + s * kPfWTileBytes, aa = a_s + s * kPfATileBytes;
+        const uint32_t wa = w_s + sw * kPfWTileBytes, aa = a_s + sa * kPfATileBytes;
 #pragma unroll
-        for (int kk = 0; kk < kPrefillBK / 16; ++kk)  // K = 16 per MMA: 32 bytes along the swizzle row
-          mma_bf16(tmem, sw128_desc(wa + 32 * kk), sw128_desc(aa + 32 * kk), kPfIdesc, (kb | kk) != 0);
-        mma_commit(empty(s));
+        for (int kk = 0; kk < kPrefillBK / 16; ++kk) {  // K = 16 per MMA: 32 bytes along the swizzle row
+          const uint64_t wd = sw128_desc(wa + 32 * kk);
+          mma_bf16(tmem, wd, sw128_desc(aa + 32 * kk), kPfIdesc, (kb | kk) != 0);
+          if (two) mma_bf16(tmem + kPrefillMmaN, wd, sw128_desc(aa + kPfAHalfBytes + 32 * kk), kPfIdesc, (kb | kk) != 0);
+        }
+        mma_commit(empty_w(sw));
+        mma_commit(empty_a(sa));
       }
       if (ok) {
         mma_commit(acc_full);
@@ -263,41 +333,26 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     const int half = threadIdx.x >> 7;               // columns 32 * half .. + 31 of a stage
     const int64_t r = row0 + rl;
     bool ok = true;
+    PkgWords<K> cur, nxt;
+    load_words<F, K>(it, r, 32 * half, p.log2g, r < it.rows && 32 * half < it.cols, cur);
     for (int kb = 0; kb < nk; ++kb) {
-      const int s = kb % kPfStages;
+      const int s = kb % kPfWStages;
       const int64_t c0 = static_cast<int64_t>(kb) * kPrefillBK + 32 * half;
       const bool valid = r < it.rows && c0 < it.cols;
-      uint2 cw[K];
-      float sc[K], zr[K];
-#pragma unroll
-      for (int i = 0; i < K; ++i) {
-        cw[i] = make_uint2(0u, 0u);
-        sc[i] = 0.0f;
-        zr[i] = 0.0f;
-      }
-      if (valid) {  // 32 weights inside one group (group >= 32, c0 % 32 == 0)
-        const int64_t e = r * it.cols + c0;
-        const int64_t g = e >> p.log2g;
-#pragma unroll
-        for (int i = 0; i < K; ++i) {
-          cw[i] = __ldg(reinterpret_cast<const uint2*>(it.codes[i] + (e >> 2)));
-          if constexpr (F == kSymF16)
-            sc[i] = __half2float(__ushort_as_half(__ldg(static_cast<const unsigned short*>(it.scales[i]) + g)));
-          else
-            sc[i] = __ldg(static_cast<const float*>(it.scales[i]) + g);
-          if constexpr (F == kAsymF32) zr[i] = __ldg(it.zeros[i] + g);
-        }
+      if (kb + 1 < nk) {  // the next stage's words, in flight while this stage is formed
+        const int64_t c1 = c0 + kPrefillBK;
+        load_words<F, K>(it, r, c1, p.log2g, r < it.rows && c1 < it.cols, nxt);
       }
       // the MMAs of this stage's previous round have read its weight tile
       bool ready = true;
-      if (kb >= kPfStages) ready = mbar_wait(empty(s), ((kb / kPfStages) - 1) & 1, p.wait_limit_us);
+      if (kb >= kPfWStages) ready = mbar_wait(empty_w(s), ((kb / kPfWStages) - 1) & 1, p.wait_limit_us);
       if (!__all_sync(kFullMask, ready)) {
         ok = false;
         break;
       }
       uint32_t h[16];
       if (valid) {
-        prefix_weights_bf16<F, K>(cw, sc, zr, h);
+        prefix_weights_bf16<F, K>(cur, h);
       } else {
 #pragma unroll
         for (int m = 0; m < 16; ++m) h[m] = 0u;
@@ -312,23 +367,24 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       fence_proxy_async_smem();  // visible to the tensor cores (async proxy)
       __syncwarp();
       if (lane == 0) mbar_arrive(full_w(s));
+      cur = nxt;
     }
     bool have = false;
     if (ok) have = mbar_wait(acc_full, 0, p.wait_limit_us);
     have = __all_sync(kFullMask, have);
     if (!have && lane == 0) atomicOr(p.status, kStatusTimeout);
     tc_fence_after();
-    if (have) {
-      const int quarter = warp & 3;  // TMEM lanes 32 * quarter .. + 31 of this warp
-      const int cols_half = warp >> 2;
+    const int quarter = warp & 3;  // TMEM lanes 32 * quarter .. + 31 of this warp
+    const int acc_i = warp >> 2;   // accumulator: tokens t0 + 256 * acc_i ..
+    if (have && (acc_i == 0 || two)) {
       const int64_t row = row0 + 32 * quarter + lane;
 #pragma unroll 1
-      for (int c = 0; c < kPrefillBN / 2 / 32; ++c) {
-        const int col = cols_half * (kPrefillBN / 2) + 32 * c;
+      for (int c = 0; c < kPrefillMmaN / 32; ++c) {
+        const int col = acc_i * kPrefillMmaN + 32 * c;
         uint32_t v[32];
         tmem_ld32(tmem + (static_cast<uint32_t>(32 * quarter) << 16) + static_cast<uint32_t>(col), v);
+        const int64_t tb = t0 + col;
         if (row < it.rows) {
-          const int64_t tb = t0 + col;
           float* y = it.Y + tb * it.rows + row;
 #pragma unroll
           for (int q = 0; q < 32; ++q)

@@ -81,10 +81,6 @@ __device__ __forceinline__ void dequant_bits(const uint4& w4, float s, float z, 
   }
 }
 
-__device__ __forceinline__ bool prescale_ok(float s) {
-  return s == 0.0f || (s >= 0x1p-100f && s <= 0x1p+100f);
-}
-
 // kAllPrefixes: write the reconstruction after every stage i < K (prefixes
 // 1..K in one pass over the package) instead of only after stage K-1.
 template <int G, int K, bool kAllPrefixes, int F>

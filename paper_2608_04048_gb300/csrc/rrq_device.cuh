@@ -178,6 +178,13 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
   return d;
 }
 
+// A scale for which s/4, s/16, s/64 and s * 2^23 are exact binary32 values,
+// so that a code left in its bit field (value 4^j Q) times s / 4^j, minus
+// 2^23 s / 4^j, gives Q s with a single rounding inside one fma.
+__device__ __forceinline__ bool prescale_ok(float s) {
+  return s == 0.0f || (s >= 0x1p-100f && s <= 0x1p+100f);
+}
+
 // min and max over 16 packed pairs (32 values) held by one lane
 __device__ __forceinline__ void lane_minmax(const f32x2 (&v)[16], float& lo, float& hi) {
   float a, b, c, d;

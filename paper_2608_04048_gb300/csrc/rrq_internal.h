@@ -101,7 +101,8 @@ constexpr int kMaxGemvBatch = 8;   // activation rows (tokens) per call
 // bf16(W~) the prefix-k reconstruction formed from the package in the
 // kernel.  A matrix is cut into tiles of kPrefillBM weight rows by
 // kPrefillBN tokens; the tiles of all matrices of a launch are numbered
-// consecutively (one CTA each) and tile_begin is this matrix's first.
+// consecutively (one CTA each, token tile major: the CTAs that run together
+// share activation tiles) and tile_begin is this matrix's first.
 struct PrefillItem {
   const uint8_t* codes[kMaxStages];
   const void* scales[kMaxStages];  // float or binary16
@@ -109,16 +110,17 @@ struct PrefillItem {
   float* Y;                        // [tokens, rows]
   int64_t rows, cols;
   int64_t tile_begin;
-  int32_t token_tiles;
+  int32_t row_tiles;
 };
 
 constexpr int kPrefillBM = 128;       // weight rows per tile (TMEM lanes, MMA M)
-constexpr int kPrefillBN = 256;       // tokens per tile (MMA N, TMEM columns)
+constexpr int kPrefillMmaN = 256;     // tokens per MMA (MMA N; also the activation box)
+constexpr int kPrefillBN = 512;       // tokens per tile: two accumulators, all 512 TMEM columns
 constexpr int kPrefillBK = 64;        // columns per pipeline stage (one 128-byte swizzle row)
 constexpr int kMaxPrefillBatch = 16;  // matrices per launch
 
 struct PrefillBatch {  // (64-byte aligned through its tensor maps)
-  CUtensorMap act[kMaxPrefillBatch];  // activations [tokens, cols] bf16: box 64 x 256, 128-byte swizzle
+  CUtensorMap act[kMaxPrefillBatch];  // activations [tokens, cols] bf16: box 64 x kPrefillMmaN, 128-byte swizzle
   PrefillItem item[kMaxPrefillBatch];
   int count;
   int log2g;                          // group = 1 << log2g
