@@ -535,6 +535,21 @@ bool encode_activations(CUtensorMap* map, const uint16_t* A, int64_t tokens, int
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Codes of one stage [rows, cols/4] bytes as a 2-D tensor map: boxes of 16
+// bytes (64 weights) x kPrefillBM rows, no swizzle, zeros outside (needs
+// cols % 64 == 0 for 16-byte row strides).
+bool encode_codes(CUtensorMap* map, const uint8_t* codes, int64_t rows, int64_t cols) {
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn) return false;
+  const cuuint64_t dim[2] = {static_cast<cuuint64_t>(cols / 4), static_cast<cuuint64_t>(rows)};
+  const cuuint64_t stride[1] = {static_cast<cuuint64_t>(cols / 4)};
+  const cuuint32_t box[2] = {16, static_cast<cuuint32_t>(rrq::kPrefillBM)};
+  const cuuint32_t estride[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(codes), dim, stride, box, estride,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
+            CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k, int64_t tokens,
                          rrq_stream_t stream) {
   if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
@@ -589,6 +604,12 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
     p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
     p.status = st->status;
     int64_t tiles = 0;
+    p.codes_tma = 1;
+    p.scale_blocks = 1;
+    for (int i = 0; i < m; ++i) {
+      if (items[base + i].cols % 64 != 0) p.codes_tma = 0;
+      if ((items[base + i].cols / group) % (16 / f.scale_bytes()) != 0) p.scale_blocks = 0;
+    }
     for (int i = 0; i < m; ++i) {
       const rrq_gemv_desc& it = items[base + i];
       rrq::PrefillItem& q = p.item[i];
@@ -606,6 +627,9 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
       q.row_tiles = static_cast<int32_t>(row_tiles);
       tiles += row_tiles * token_tiles;
       if (!encode_activations(&p.act[i], it.A_bf16, tokens, it.cols)) return RRQ_ERR_UNSUPPORTED;
+      if (p.codes_tma)
+        for (int j = 0; j < k; ++j)
+          if (!encode_codes(&p.codes[i][j], it.codes[j], it.rows, it.cols)) return RRQ_ERR_UNSUPPORTED;
     }
     if (tiles > 0x7fffffff) return RRQ_ERR_INVALID_ARG;
     p.total_tiles = tiles;

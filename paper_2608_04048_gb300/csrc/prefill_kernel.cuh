@@ -17,10 +17,13 @@
 // stages of 64 columns:
 //   - warp 8 loads the activation tile of a stage (512 tokens x 64 columns,
 //     bf16, two 2-D TMA boxes, 128-byte swizzle) into a 2-deep ring;
-//   - warps 0-7 read the package words of the stage one stage ahead (codes,
-//     scales, zeros), form the 128 x 64 bf16 weight tile in registers and
-//     store it in the same K-major 128-byte-swizzled layout into a 4-deep
-//     ring, then signal the stage;
+//   - warp 10 loads the stage's codes of the row tile (one 2-D TMA box of
+//     16 bytes x 128 rows per package stage) into a 4-deep ring;
+//   - warps 0-7 take the codes from that ring (or load them themselves when
+//     a matrix's code rows are not 16-byte multiples) and the scales and
+//     zeros a stage ahead, form the 128 x 64 bf16 weight tile in registers
+//     and store it in the same K-major 128-byte-swizzled layout into a
+//     3-deep ring, then signal the stage;
 //   - one thread of warp 9 issues the MMAs of the stage and commits them to
 //     the two rings' "empty" barriers, which release the buffers;
 //   - after the last stage warps 0-7 read the accumulators (tcgen05.ld, one
@@ -37,19 +40,25 @@
 namespace rrq {
 namespace {
 
-constexpr int kPfWStages = 4;                        // weight-tile ring depth
+constexpr int kPfWStages = 3;                        // weight-tile ring depth
+constexpr int kPfCStages = 4;                        // code-tile ring depth
 constexpr int kPfAStages = 2;                        // activation-tile ring depth
 constexpr int kPfWTileBytes = kPrefillBM * 128;      // 128 rows x 64 bf16 (16 KiB)
 constexpr int kPfAHalfBytes = kPrefillMmaN * 128;    // 256 tokens x 64 bf16 (32 KiB)
 constexpr int kPfATileBytes = 2 * kPfAHalfBytes;     // 512 tokens (64 KiB)
+constexpr int kPfCTileBytes = kPrefillBM * 16;       // one package stage's codes of a stage (2 KiB)
+constexpr int kPfCStageBytes = kMaxStages * kPfCTileBytes;
 constexpr int kPfDqWarps = 8;                        // weight tiles, then the epilogue
 constexpr int kPfTmaWarp = 8;
 constexpr int kPfMmaWarp = 9;
-constexpr int kPfThreads = 10 * 32;
+constexpr int kPfCodeWarp = 10;
+constexpr int kPfThreads = 11 * 32;
 constexpr uint32_t kPfTmemCols = kPrefillBN;         // two binary32 accumulators, 128 lanes x 256 columns each
-constexpr int kPfBarOffset = kPfWStages * kPfWTileBytes + kPfAStages * kPfATileBytes;
-// full_w, empty_w per weight stage; full_a, empty_a per activation stage; acc_full; drain
-constexpr int kPfBars = 2 * kPfWStages + 2 * kPfAStages + 2;
+constexpr int kPfCOffset = kPfWStages * kPfWTileBytes + kPfAStages * kPfATileBytes;
+constexpr int kPfBarOffset = kPfCOffset + kPfCStages * kPfCStageBytes;
+// full_w, empty_w per weight stage; full_a, empty_a per activation stage;
+// full_c, empty_c per code stage; acc_full; drain
+constexpr int kPfBars = 2 * kPfWStages + 2 * kPfAStages + 2 * kPfCStages + 2;
 constexpr int kPfSmemBytes = kPfBarOffset + 8 * kPfBars + 16 + 1024;  // + TMEM address, alignment slack
 
 // Instruction descriptor of tcgen05.mma .kind::f16: D binary32 (bits 4-5),
@@ -122,6 +131,25 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+// Bounded wait that sleeps in the barrier instead of spinning: each try
+// suspends the thread until the phase completes or about a millisecond
+// passes, so waiting warps take no issue slots from the working ones.
+__device__ __forceinline__ bool pf_wait(uint32_t bar, uint32_t parity, uint32_t limit_us) {
+  if (limit_us == 0) return false;
+  const uint64_t t0 = globaltimer_ns();
+  const uint64_t limit_ns = static_cast<uint64_t>(limit_us) * 1000u;
+  while (true) {
+    uint32_t done;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
+        : "=r"(done)
+        : "r"(bar), "r"(parity), "r"(1000000u)
+        : "memory");
+    if (done) return true;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
 // Package words of the 32 consecutive weights (one group) a thread forms in
 // one stage.
 template <int K>
@@ -131,26 +159,55 @@ struct PkgWords {
   float zr[K];   // stage-i zero (asymmetric grid)
 };
 
+// Scales (and zeros) of 16 consecutive bytes of one row: 4 binary32 or 8
+// binary16 groups, loaded as one vector per package stage.
+template <int K>
+struct ScaleBlock {
+  uint4 s[K];
+  uint4 z[K];
+};
+
+template <int F>
+__host__ __device__ constexpr int groups_per_block() { return F == kSymF16 ? 8 : 4; }
+
 template <int F, int K>
-__device__ __forceinline__ void load_words(const PrefillItem& it, int64_t r, int64_t c0, int log2g, bool valid,
-                                           PkgWords<K>& w) {
+__device__ __forceinline__ void load_block(const PrefillItem& it, int64_t b, ScaleBlock<K>& sb) {
 #pragma unroll
   for (int i = 0; i < K; ++i) {
-    w.cw[i] = make_uint2(0u, 0u);
-    w.sc[i] = 0.0f;
-    w.zr[i] = 0.0f;
+    sb.s[i] = __ldg(static_cast<const uint4*>(it.scales[i]) + b);
+    if constexpr (F == kAsymF32) sb.z[i] = __ldg(reinterpret_cast<const uint4*>(it.zeros[i]) + b);
   }
-  if (!valid) return;
-  const int64_t e = r * it.cols + c0;
-  const int64_t g = e >> log2g;
+}
+
+__device__ __forceinline__ uint32_t pick_word(const uint4& v, int j) {
+  return (j & 2) ? ((j & 1) ? v.w : v.z) : ((j & 1) ? v.y : v.x);
+}
+
+// stage-i scale and zero of group gi (0 .. groups_per_block - 1) of a block
+template <int F, int K>
+__device__ __forceinline__ void from_block(const ScaleBlock<K>& sb, int gi, PkgWords<K>& w) {
 #pragma unroll
   for (int i = 0; i < K; ++i) {
-    w.cw[i] = __ldg(reinterpret_cast<const uint2*>(it.codes[i] + (e >> 2)));
+    if constexpr (F == kSymF16) {
+      const uint32_t word = pick_word(sb.s[i], gi >> 1);
+      w.sc[i] = __half2float(__ushort_as_half(static_cast<unsigned short>((gi & 1) ? (word >> 16) : (word & 0xffffu))));
+    } else {
+      w.sc[i] = __uint_as_float(pick_word(sb.s[i], gi));
+    }
+    w.zr[i] = (F == kAsymF32) ? __uint_as_float(pick_word(sb.z[i], gi)) : 0.0f;
+  }
+}
+
+// stage-i scale and zero of group g, one scalar load each
+template <int F, int K>
+__device__ __forceinline__ void load_scales(const PrefillItem& it, int64_t g, PkgWords<K>& w) {
+#pragma unroll
+  for (int i = 0; i < K; ++i) {
     if constexpr (F == kSymF16)
       w.sc[i] = __half2float(__ushort_as_half(__ldg(static_cast<const unsigned short*>(it.scales[i]) + g)));
     else
       w.sc[i] = __ldg(static_cast<const float*>(it.scales[i]) + g);
-    if constexpr (F == kAsymF32) w.zr[i] = __ldg(it.zeros[i] + g);
+    w.zr[i] = (F == kAsymF32) ? __ldg(it.zeros[i] + g) : 0.0f;
   }
 }
 
@@ -229,7 +286,8 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   const uint32_t w_s = base_s;                                // weight tiles
   const uint32_t a_s = base_s + kPfWStages * kPfWTileBytes;   // activation tiles
   const uint32_t bar_s = base_s + kPfBarOffset;
-  const uint32_t acc_full = bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages);
+  const uint32_t c_s = base_s + kPfCOffset;                  // code tiles
+  const uint32_t acc_full = bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages + 2 * kPfCStages);
   const uint32_t drain = acc_full + 8;
   const uint32_t slot_s = bar_s + 8 * kPfBars;
   const volatile uint32_t* slot = reinterpret_cast<const volatile uint32_t*>(base + kPfBarOffset + 8 * kPfBars);
@@ -237,6 +295,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   auto empty_w = [&](int s) { return bar_s + 8 * (kPfWStages + s); };
   auto full_a = [&](int s) { return bar_s + 8 * (2 * kPfWStages + s); };
   auto empty_a = [&](int s) { return bar_s + 8 * (2 * kPfWStages + kPfAStages + s); };
+  auto full_c = [&](int s) { return bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages + s); };
+  auto empty_c = [&](int s) { return bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages + kPfCStages + s); };
+  const bool codes_tma = p.codes_tma != 0;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -261,6 +322,10 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       mbar_init(full_a(s), 1);
       mbar_init(empty_a(s), 1);
     }
+    for (int s = 0; s < kPfCStages; ++s) {
+      mbar_init(full_c(s), 1);
+      mbar_init(empty_c(s), kPfDqWarps);
+    }
     mbar_init(acc_full, 1);
     mbar_init(drain, 1);
     fence_mbarrier_init();
@@ -280,7 +345,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       int issued = 0;
       for (int kb = 0; kb < nk; ++kb) {
         const int s = kb % kPfAStages;
-        if (kb >= kPfAStages && !mbar_wait(empty_a(s), ((kb / kPfAStages) - 1) & 1, p.wait_limit_us)) {
+        if (kb >= kPfAStages && !pf_wait(empty_a(s), ((kb / kPfAStages) - 1) & 1, p.wait_limit_us)) {
           ok = false;
           break;
         }
@@ -298,13 +363,37 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       }
     }
     __syncwarp();
+  } else if (warp == kPfCodeWarp) {
+    if (lane == 0 && codes_tma) {
+      bool ok = true;
+      int issued = 0;
+      for (int kb = 0; kb < nk; ++kb) {
+        const int s = kb % kPfCStages;
+        if (kb >= kPfCStages && !pf_wait(empty_c(s), ((kb / kPfCStages) - 1) & 1, p.wait_limit_us)) {
+          ok = false;
+          break;
+        }
+        mbar_arrive_expect_tx(full_c(s), K * kPfCTileBytes);
+#pragma unroll
+        for (int i = 0; i < K; ++i)
+          tma_load_2d(c_s + s * kPfCStageBytes + i * kPfCTileBytes, &p.codes[mi][i], kb * 16, static_cast<int>(row0),
+                      full_c(s));
+        ++issued;
+      }
+      if (!ok) {  // let this thread's copies land before the CTA can leave
+        atomicOr(p.status, kStatusTimeout);
+        for (int kb = issued > kPfCStages ? issued - kPfCStages : 0; kb < issued; ++kb)
+          mbar_wait(full_c(kb % kPfCStages), (kb / kPfCStages) & 1, kDrainLimitUs);
+      }
+    }
+    __syncwarp();
   } else if (warp == kPfMmaWarp) {
     if (lane == 0) {
       bool ok = true;
       for (int kb = 0; kb < nk; ++kb) {
         const int sw = kb % kPfWStages, sa = kb % kPfAStages;
-        if (!mbar_wait(full_a(sa), (kb / kPfAStages) & 1, p.wait_limit_us) ||
-            !mbar_wait(full_w(sw), (kb / kPfWStages) & 1, p.wait_limit_us)) {
+        if (!pf_wait(full_a(sa), (kb / kPfAStages) & 1, p.wait_limit_us) ||
+            !pf_wait(full_w(sw), (kb / kPfWStages) & 1, p.wait_limit_us)) {
           ok = false;
           break;
         }
@@ -333,19 +422,63 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     const int half = threadIdx.x >> 7;               // columns 32 * half .. + 31 of a stage
     const int64_t r = row0 + rl;
     bool ok = true;
-    PkgWords<K> cur, nxt;
-    load_words<F, K>(it, r, 32 * half, p.log2g, r < it.rows && 32 * half < it.cols, cur);
+    const bool blocked = p.scale_blocks != 0;
+    constexpr int kSB = groups_per_block<F>();
+    ScaleBlock<K> bc, bn;     // scale blocks in use and the next one (in flight)
+    int64_t blk_cur = -1, blk_nxt = -1;
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % kPfWStages;
       const int64_t c0 = static_cast<int64_t>(kb) * kPrefillBK + 32 * half;
       const bool valid = r < it.rows && c0 < it.cols;
-      if (kb + 1 < nk) {  // the next stage's words, in flight while this stage is formed
-        const int64_t c1 = c0 + kPrefillBK;
-        load_words<F, K>(it, r, c1, p.log2g, r < it.rows && c1 < it.cols, nxt);
+      PkgWords<K> cur;
+#pragma unroll
+      for (int i = 0; i < K; ++i) {
+        cur.cw[i] = make_uint2(0u, 0u);
+        cur.sc[i] = 0.0f;
+        cur.zr[i] = 0.0f;
+      }
+      if (valid) {
+        const int64_t e = r * it.cols + c0;
+        const int64_t g = e >> p.log2g;
+        if (blocked) {  // rows hold whole blocks, so a block never leaves its row
+          const int64_t blk = g / kSB;
+          if (blk != blk_cur) {
+            if (blk == blk_nxt) bc = bn;
+            else load_block<F, K>(it, blk, bc);
+            blk_cur = blk;
+            blk_nxt = -1;
+            if (((blk + 1) * kSB << p.log2g) < (r + 1) * it.cols) {  // prefetch the row's next block
+              load_block<F, K>(it, blk + 1, bn);
+              blk_nxt = blk + 1;
+            }
+          }
+          from_block<F, K>(bc, static_cast<int>(g % kSB), cur);
+        } else {
+          load_scales<F, K>(it, g, cur);
+        }
+        if (!codes_tma) {
+#pragma unroll
+          for (int i = 0; i < K; ++i) cur.cw[i] = __ldg(reinterpret_cast<const uint2*>(it.codes[i] + (e >> 2)));
+        }
+      }
+      if (codes_tma) {  // this stage's codes from the ring; the slot is free once read
+        const int sc = kb % kPfCStages;
+        const bool got = pf_wait(full_c(sc), (kb / kPfCStages) & 1, p.wait_limit_us);
+        if (!__all_sync(kFullMask, got)) {
+          ok = false;
+          break;
+        }
+        const uint8_t* ct = base + kPfCOffset + sc * kPfCStageBytes + rl * 16 + half * 8;
+#pragma unroll
+        for (int i = 0; i < K; ++i) cur.cw[i] = *reinterpret_cast<const uint2*>(ct + i * kPfCTileBytes);
+        // every lane's reads before the next copy (async proxy) into the slot
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(empty_c(sc));
       }
       // the MMAs of this stage's previous round have read its weight tile
       bool ready = true;
-      if (kb >= kPfWStages) ready = mbar_wait(empty_w(s), ((kb / kPfWStages) - 1) & 1, p.wait_limit_us);
+      if (kb >= kPfWStages) ready = pf_wait(empty_w(s), ((kb / kPfWStages) - 1) & 1, p.wait_limit_us);
       if (!__all_sync(kFullMask, ready)) {
         ok = false;
         break;
@@ -367,10 +500,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       fence_proxy_async_smem();  // visible to the tensor cores (async proxy)
       __syncwarp();
       if (lane == 0) mbar_arrive(full_w(s));
-      cur = nxt;
     }
     bool have = false;
-    if (ok) have = mbar_wait(acc_full, 0, p.wait_limit_us);
+    if (ok) have = pf_wait(acc_full, 0, p.wait_limit_us);
     have = __all_sync(kFullMask, have);
     if (!have && lane == 0) atomicOr(p.status, kStatusTimeout);
     tc_fence_after();

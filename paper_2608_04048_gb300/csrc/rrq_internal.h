@@ -121,7 +121,12 @@ constexpr int kMaxPrefillBatch = 16;  // matrices per launch
 
 struct PrefillBatch {  // (64-byte aligned through its tensor maps)
   CUtensorMap act[kMaxPrefillBatch];  // activations [tokens, cols] bf16: box 64 x kPrefillMmaN, 128-byte swizzle
+  // codes of stage i [rows, cols/4] bytes: box 16 x kPrefillBM (the codes of
+  // one 64-column stage of a row tile); used when codes_tma != 0
+  CUtensorMap codes[kMaxPrefillBatch][kMaxStages];
   PrefillItem item[kMaxPrefillBatch];
+  int codes_tma;                      // every matrix has cols % 64 == 0
+  int scale_blocks;                   // every matrix has 16-byte rows of scales (and zeros)
   int count;
   int log2g;                          // group = 1 << log2g
   int64_t tokens;

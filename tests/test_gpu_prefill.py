@@ -168,6 +168,24 @@ def test_deterministic_and_reconstruction_consistent():
     _status_ok()
 
 
+@pytest.mark.parametrize("shape", [(129, 4096, 257), (256, 4096, 257), (300, 2048, 600)])
+def test_repeated_runs_identical(shape):
+    """The ring protocols leave no race: five runs of the same call give the
+    same bits, and they match the oracle (ragged row and token tiles, the
+    code tiles by TMA)."""
+    rows, cols, tokens = shape
+    W = workloads.generate(rows, cols, rows + cols, "t3", "cuda")
+    (pkg,) = binding.rrq_quantize_ex([W], 128, 4, binding.GRID_ASYM, binding.SCALE_F32)
+    A = _acts(tokens, cols, seed=rows)
+    for k in (1, 4):
+        outs = [binding.rrq_prefill([pkg], [A], k)[0] for _ in range(5)]
+        torch.cuda.synchronize()
+        for Y in outs[1:]:
+            assert torch.equal(Y.view(torch.int32), outs[0].view(torch.int32)), f"{shape} k{k}: runs differ"
+        _check(pkg, A, outs[0], k, where=f"{shape} k{k}")
+    _status_ok()
+
+
 def test_batch_across_launches():
     rng = np.random.default_rng(21)
     shapes = [(int(rng.integers(1, 300)), 128 * int(rng.integers(1, 12))) for _ in range(20)]
