@@ -182,10 +182,12 @@ def time_prefill(pkgs, specs, stream, tokens: int = 2048, reps: int = 2) -> dict
     gen = torch.Generator(device=dev).manual_seed(78)
     acts = [torch.randn((tokens, specs[j].cols), generator=gen, device=dev).to(torch.bfloat16) for j in layers[0]]
     ys = [torch.empty((tokens, specs[j].rows), dtype=torch.float32, device=dev) for j in layers[0]]
-    peak = measured_peaks().get("bf16_tflops") or 1900.0
+    peaks = measured_peaks()
+    peak = peaks["bf16_tflops"]
     flops = 2.0 * tokens * sum(sp.numel for sp in specs)
     out = {"call": f"rrq_prefill over all {len(specs)} matrices, {tokens} tokens, one call per layer "
-                   "(asymmetric binary32 package)", "tokens": tokens, "peak_tflops": peak}
+                   "(asymmetric binary32 package)", "tokens": tokens, "peak_tflops": peak,
+           "peak_source": f"{peaks['source']} dense bf16 (burst)"}
     for k in KS:
         items = [binding.gemv_descs([pkgs[j] for j in L], acts[:len(L)], ys[:len(L)], k) for L in layers]
 
@@ -276,8 +278,9 @@ def measured_peaks() -> dict:
     if os.path.exists(p):
         with open(p) as f:
             d = json.load(f)
-        return {"hbm_gbs": float(d["hbm_gbs"]), "source": "measured"}
-    return {"hbm_gbs": 6800.0, "source": "fallback"}
+        return {"hbm_gbs": float(d["hbm_gbs"]), "bf16_tflops": float(d.get("bf16_tflops") or 1900.0),
+                "source": "measured"}
+    return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "source": "fallback"}
 
 
 # ---------------------------------------------------------------------------
