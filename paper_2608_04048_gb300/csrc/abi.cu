@@ -536,14 +536,14 @@ bool encode_activations(CUtensorMap* map, const uint16_t* A, int64_t tokens, int
 }
 
 // Codes of one stage [rows, cols/4] bytes as a 2-D tensor map: boxes of 16
-// bytes (64 weights) x kPrefillBM rows, no swizzle, zeros outside (needs
+// bytes (64 weights) x box_rows rows, no swizzle, zeros outside (needs
 // cols % 64 == 0 for 16-byte row strides).
-bool encode_codes(CUtensorMap* map, const uint8_t* codes, int64_t rows, int64_t cols) {
+bool encode_codes(CUtensorMap* map, const uint8_t* codes, int64_t rows, int64_t cols, int box_rows) {
   EncodeTiledFn fn = encode_tiled();
   if (!fn) return false;
   const cuuint64_t dim[2] = {static_cast<cuuint64_t>(cols / 4), static_cast<cuuint64_t>(rows)};
   const cuuint64_t stride[1] = {static_cast<cuuint64_t>(cols / 4)};
-  const cuuint32_t box[2] = {16, static_cast<cuuint32_t>(rrq::kPrefillBM)};
+  const cuuint32_t box[2] = {16, static_cast<cuuint32_t>(box_rows)};
   const cuuint32_t estride[2] = {1, 1};
   return fn(map, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<uint8_t*>(codes), dim, stride, box, estride,
             CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_128B,
@@ -594,6 +594,11 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
   int log2g = 0;
   while ((1 << log2g) < group) ++log2g;
   const int64_t token_tiles = (tokens + rrq::kPrefillBN - 1) / rrq::kPrefillBN;
+  // clusters share weight tiles across token tiles: 4 CTAs for the longer
+  // prefixes (forming weights costs most there), else 2 (measured best on
+  // Qwen3-8B-shaped layers at 2048 tokens)
+  const int cluster = (k >= 3 && token_tiles >= 3) ? 4 : token_tiles >= 2 ? 2 : 1;
+  const int64_t token_tiles_padded = (token_tiles + cluster - 1) / cluster * cluster;
   static thread_local rrq::PrefillBatch p;
   for (int base = 0; base < count; base += rrq::kMaxPrefillBatch) {
     const int m = std::min(rrq::kMaxPrefillBatch, count - base);
@@ -601,6 +606,7 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
     p.count = m;
     p.log2g = log2g;
     p.tokens = tokens;
+    p.cluster = cluster;
     p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
     p.status = st->status;
     int64_t tiles = 0;
@@ -625,11 +631,12 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
       const int64_t row_tiles = (it.rows + rrq::kPrefillBM - 1) / rrq::kPrefillBM;
       q.tile_begin = tiles;
       q.row_tiles = static_cast<int32_t>(row_tiles);
-      tiles += row_tiles * token_tiles;
+      tiles += row_tiles * token_tiles_padded;
       if (!encode_activations(&p.act[i], it.A_bf16, tokens, it.cols)) return RRQ_ERR_UNSUPPORTED;
       if (p.codes_tma)
         for (int j = 0; j < k; ++j)
-          if (!encode_codes(&p.codes[i][j], it.codes[j], it.rows, it.cols)) return RRQ_ERR_UNSUPPORTED;
+          if (!encode_codes(&p.codes[i][j], it.codes[j], it.rows, it.cols, rrq::kPrefillBM / cluster))
+            return RRQ_ERR_UNSUPPORTED;
     }
     if (tiles > 0x7fffffff) return RRQ_ERR_INVALID_ARG;
     p.total_tiles = tiles;

@@ -12,24 +12,33 @@
 //
 // One CTA computes a tile of 128 weight rows x 512 tokens: two accumulators
 // of tcgen05.mma.cta_group::1.kind::f16 shape M = 128, N = 256 (K = 16 per
-// instruction), which fill the 512 columns of tensor memory, so every weight
-// tile formed from the package serves 512 tokens.  The K range is walked in
-// stages of 64 columns:
+// instruction), which fill the 512 columns of tensor memory.  CS CTAs (1, 2
+// or 4) with the same 128 rows and consecutive token tiles form a cluster
+// that shares the weight tiles: each CTA forms 128/CS of the rows and sends
+// them to the others, so a weight tile formed from the package serves
+// 512 x CS tokens.  The K range is walked in stages of 64 columns:
 //   - warp 8 loads the activation tile of a stage (512 tokens x 64 columns,
 //     bf16, two 2-D TMA boxes, 128-byte swizzle) into a 2-deep ring;
-//   - warp 10 loads the stage's codes of the row tile (one 2-D TMA box of
-//     16 bytes x 128 rows per package stage) into a 4-deep ring;
+//   - warp 10 loads the stage's codes of this CTA's rows (one 2-D TMA box of
+//     16 bytes x 128/CS rows per package stage) into a 4-deep ring;
 //   - warps 0-7 take the codes from that ring (or load them themselves when
 //     a matrix's code rows are not 16-byte multiples) and the scales and
-//     zeros a stage ahead, form the 128 x 64 bf16 weight tile in registers
-//     and store it in the same K-major 128-byte-swizzled layout into a
-//     3-deep ring, then signal the stage;
+//     zeros as 16-byte blocks a block ahead, form this CTA's rows of the bf16
+//     weight tile in registers and store them in the K-major
+//     128-byte-swizzled layout into a 3-deep ring;
+//   - in a cluster, warp 11 then copies those rows (contiguous in the
+//     swizzled tile) into the same slot of every other CTA with one bulk
+//     copy each, which completes there as transaction bytes of the slot's
+//     "full" barrier; no thread issues a cluster-scope release;
 //   - one thread of warp 9 issues the MMAs of the stage and commits them to
-//     the two rings' "empty" barriers, which release the buffers;
+//     the activation ring's "empty" barrier and, multicast, to the weight
+//     ring's "empty" barrier of every CTA of the cluster, so that no CTA
+//     overwrites a slot before all have read it;
 //   - after the last stage warps 0-7 read the accumulators (tcgen05.ld, one
 //     TMEM lane = one weight row) and store Y with coalesced binary32 stores.
 // Every wait is bounded in wall time; on expiry the kernel sets the status
-// word, drains its own copies and MMAs (bounded) and frees its tensor memory.
+// word, drains its own copies and MMAs (bounded) and frees its tensor memory;
+// the CTAs of a cluster meet at a cluster barrier before any of them leaves.
 #pragma once
 
 #include <cuda_bf16.h>
@@ -52,13 +61,14 @@ constexpr int kPfDqWarps = 8;                        // weight tiles, then the e
 constexpr int kPfTmaWarp = 8;
 constexpr int kPfMmaWarp = 9;
 constexpr int kPfCodeWarp = 10;
-constexpr int kPfThreads = 11 * 32;
+constexpr int kPfShareWarp = 11;                     // clusters: sends this CTA's rows to the others
+constexpr int kPfThreads = 12 * 32;
 constexpr uint32_t kPfTmemCols = kPrefillBN;         // two binary32 accumulators, 128 lanes x 256 columns each
 constexpr int kPfCOffset = kPfWStages * kPfWTileBytes + kPfAStages * kPfATileBytes;
 constexpr int kPfBarOffset = kPfCOffset + kPfCStages * kPfCStageBytes;
 // full_w, empty_w per weight stage; full_a, empty_a per activation stage;
-// full_c, empty_c per code stage; acc_full; drain
-constexpr int kPfBars = 2 * kPfWStages + 2 * kPfAStages + 2 * kPfCStages + 2;
+// full_c, empty_c per code stage; acc_full; drain; share_done per weight stage
+constexpr int kPfBars = 2 * kPfWStages + 2 * kPfAStages + 2 * kPfCStages + 2 + kPfWStages;
 constexpr int kPfSmemBytes = kPfBarOffset + 8 * kPfBars + 16 + 1024;  // + TMEM address, alignment slack
 
 // Instruction descriptor of tcgen05.mma .kind::f16: D binary32 (bits 4-5),
@@ -111,6 +121,32 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
 }
+// Cluster forms: the address of the same shared-memory offset in CTA `rank`
+// of the cluster, an MMA commit that arrives on the barrier at the same
+// offset in every CTA of `mask`, and the cluster-wide barrier.
+__device__ __forceinline__ uint32_t cluster_addr(uint32_t saddr, uint32_t rank) {
+  uint32_t r;
+  asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(saddr), "r"(rank));
+  return r;
+}
+__device__ __forceinline__ void mma_commit_multicast(uint32_t bar, uint16_t mask) {
+  asm volatile(
+      "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(bar),
+      "h"(mask)
+      : "memory");
+}
+// shared -> shared bulk copy into CTA dst's memory (cluster addresses of the
+// destination and of its barrier), completing there as transaction bytes
+__device__ __forceinline__ void bulk_copy_cluster(uint32_t dst, uint32_t src, uint32_t bytes, uint32_t bar) {
+  asm volatile("cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(dst),
+               "r"(src), "r"(bytes), "r"(bar)
+               : "memory");
+}
+__device__ __forceinline__ void cluster_sync() {
+  asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+  asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
 // 2-D tiled TMA load: box at (x = column, y = row) of `map`, completing on `bar`.
 __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap* map, int x, int y, uint32_t bar) {
   asm volatile(
@@ -211,17 +247,18 @@ __device__ __forceinline__ void load_scales(const PrefillItem& it, int64_t g, Pk
   }
 }
 
-// bf16 prefix-k weights of those 32 weights: acc = L_0; acc = fl(acc + L_i);
+// bf16 prefix-k weights of the first NW (8, 16 or 32) of those weights: acc =
+// L_0; acc = fl(acc + L_i);
 // bf16 nearest-even.  L_i = fl(zero + fl(Q s)) (asymmetric) or (Q - 2) s
 // (symmetric, exact).  Two evaluations of fl(Q s), both exact to the same
 // bits: with prescale_ok(s) each code stays in its bit field (value 4^j Q
 // for the j-th code of a byte) and one fma with s / 4^j and -2^23 s / 4^j
 // rounds Q s once; otherwise the code is shifted down and fma(Q, s, 0).
-template <int F, int K>
-__device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32_t (&h)[16]) {
+template <int F, int K, int NW>
+__device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32_t (&h)[NW / 2]) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr float kT23 = 8388608.0f;
-  f32x2 acc[16];
+  f32x2 acc[NW / 2];
 #pragma unroll
   for (int i = 0; i < K; ++i) {
     const float s = w.sc[i];
@@ -232,7 +269,7 @@ __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32
       const f32x2 C23 = pack2(__fmul_rn(s, -0x1p19f), __fmul_rn(s, -0x1p17f));
       const f32x2 K01 = pack2(kT23 + 2.0f, kT23 + 8.0f), K23 = pack2(kT23 + 32.0f, kT23 + 128.0f);
 #pragma unroll
-      for (int j = 0; j < 8; ++j) {  // byte j: weights 4j..4j+3 (pairs 2j, 2j+1)
+      for (int j = 0; j < NW / 4; ++j) {  // byte j: weights 4j..4j+3 (pairs 2j, 2j+1)
         const uint32_t word = j < 4 ? w.cw[i].x : w.cw[i].y;
         const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
         const f32x2 t01 = pack2u(0x4B000000u | (b & 0x03u), 0x4B000000u | (b & 0x0Cu));
@@ -253,7 +290,7 @@ __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32
       const f32x2 LO = pack2(w.zr[i], w.zr[i]), Z = pack2(0.0f, 0.0f);
       const f32x2 T23 = pack2(kT23, kT23), K2 = pack2(kT23 + 2.0f, kT23 + 2.0f);
 #pragma unroll
-      for (int m = 0; m < 16; ++m) {
+      for (int m = 0; m < NW / 2; ++m) {
         const uint32_t word = m < 8 ? w.cw[i].x : w.cw[i].y;
         const int sh = 4 * (m & 7);
         const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
@@ -269,7 +306,7 @@ __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32
     }
   }
 #pragma unroll
-  for (int m = 0; m < 16; ++m) {
+  for (int m = 0; m < NW / 2; ++m) {
     float a, b;
     unpack2(acc[m], a, b);
     const __nv_bfloat162 x = __floats2bfloat162_rn(a, b);
@@ -277,8 +314,10 @@ __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32
   }
 }
 
-template <int F, int K>
+template <int F, int K, int CS>
 __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_constant__ PrefillBatch p) {
+  constexpr int kRows = kPrefillBM / CS;  // rows of the tile this CTA forms for the cluster
+  constexpr int kNW = 32 / CS;            // weights a thread forms per stage
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_s = smem_u32(smem_raw);
   const uint32_t base_s = (raw_s + 1023u) & ~1023u;  // swizzled tiles need 1024-byte alignment
@@ -289,7 +328,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   const uint32_t c_s = base_s + kPfCOffset;                  // code tiles
   const uint32_t acc_full = bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages + 2 * kPfCStages);
   const uint32_t drain = acc_full + 8;
-  const uint32_t slot_s = bar_s + 8 * kPfBars;
+  const uint32_t slot_s = bar_s + 8 * kPfBars;  // (after share_done)
   const volatile uint32_t* slot = reinterpret_cast<const volatile uint32_t*>(base + kPfBarOffset + 8 * kPfBars);
   auto full_w = [&](int s) { return bar_s + 8 * s; };
   auto empty_w = [&](int s) { return bar_s + 8 * (kPfWStages + s); };
@@ -297,26 +336,35 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   auto empty_a = [&](int s) { return bar_s + 8 * (2 * kPfWStages + kPfAStages + s); };
   auto full_c = [&](int s) { return bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages + s); };
   auto empty_c = [&](int s) { return bar_s + 8 * (2 * kPfWStages + 2 * kPfAStages + kPfCStages + s); };
+  auto share_done = [&](int s) { return drain + 8 + 8 * s; };
   const bool codes_tma = p.codes_tma != 0;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
 
-  // this CTA's tile (token tile major)
+  // this CTA's tile: clusters in token-tile-major order, rank = token tile
+  // within the cluster
   const int64_t tile = blockIdx.x;
   int mi = 0;
   while (mi + 1 < p.count && tile >= p.item[mi + 1].tile_begin) ++mi;
   const PrefillItem& it = p.item[mi];
   const int64_t j = tile - it.tile_begin;
-  const int64_t row0 = (j % it.row_tiles) * kPrefillBM;
-  const int64_t t0 = (j / it.row_tiles) * kPrefillBN;
+  const int rank = static_cast<int>(j % CS);
+  const int64_t cj = j / CS;
+  const int64_t row0 = (cj % it.row_tiles) * kPrefillBM;
+  const int64_t t0 = ((cj / it.row_tiles) * CS + rank) * kPrefillBN;
+  const bool active = t0 < p.tokens;              // (padding CTAs only form weights)
   const bool two = t0 + kPrefillMmaN < p.tokens;  // the second accumulator has tokens
   const int nk = static_cast<int>((it.cols + kPrefillBK - 1) / kPrefillBK);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < kPfWStages; ++s) {
-      mbar_init(full_w(s), kPfDqWarps);
-      mbar_init(empty_w(s), 1);
+      // one CTA: the producer warps; a cluster: one arrival that expects the
+      // other CTAs' rows as transaction bytes (this CTA's own rows are ready
+      // before it)
+      mbar_init(full_w(s), CS == 1 ? kPfDqWarps : 1);
+      mbar_init(empty_w(s), CS);              // every MMA thread of the cluster
+      mbar_init(share_done(s), kPfDqWarps);
     }
     for (int s = 0; s < kPfAStages; ++s) {
       mbar_init(full_a(s), 1);
@@ -338,9 +386,10 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem = *slot;
+  if constexpr (CS > 1) cluster_sync();  // every CTA's barriers exist before any remote access
 
   if (warp == kPfTmaWarp) {
-    if (lane == 0) {
+    if (lane == 0 && active) {
       bool ok = true;
       int issued = 0;
       for (int kb = 0; kb < nk; ++kb) {
@@ -373,11 +422,11 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
           ok = false;
           break;
         }
-        mbar_arrive_expect_tx(full_c(s), K * kPfCTileBytes);
+        mbar_arrive_expect_tx(full_c(s), K * kRows * 16);
 #pragma unroll
         for (int i = 0; i < K; ++i)
-          tma_load_2d(c_s + s * kPfCStageBytes + i * kPfCTileBytes, &p.codes[mi][i], kb * 16, static_cast<int>(row0),
-                      full_c(s));
+          tma_load_2d(c_s + s * kPfCStageBytes + i * kPfCTileBytes, &p.codes[mi][i], kb * 16,
+                      static_cast<int>(row0 + rank * kRows), full_c(s));
         ++issued;
       }
       if (!ok) {  // let this thread's copies land before the CTA can leave
@@ -392,24 +441,29 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       bool ok = true;
       for (int kb = 0; kb < nk; ++kb) {
         const int sw = kb % kPfWStages, sa = kb % kPfAStages;
-        if (!pf_wait(full_a(sa), (kb / kPfAStages) & 1, p.wait_limit_us) ||
+        if ((active && !pf_wait(full_a(sa), (kb / kPfAStages) & 1, p.wait_limit_us)) ||
             !pf_wait(full_w(sw), (kb / kPfWStages) & 1, p.wait_limit_us)) {
           ok = false;
           break;
         }
         tc_fence_after();
-        const uint32_t wa = w_s + sw * kPfWTileBytes, aa = a_s + sa * kPfATileBytes;
+        if (active) {
+          const uint32_t wa = w_s + sw * kPfWTileBytes, aa = a_s + sa * kPfATileBytes;
 #pragma unroll
-        for (int kk = 0; kk < kPrefillBK / 16; ++kk) {  // K = 16 per MMA: 32 bytes along the swizzle row
-          const uint64_t wd = sw128_desc(wa + 32 * kk);
-          mma_bf16(tmem, wd, sw128_desc(aa + 32 * kk), kPfIdesc, (kb | kk) != 0);
-          if (two) mma_bf16(tmem + kPrefillMmaN, wd, sw128_desc(aa + kPfAHalfBytes + 32 * kk), kPfIdesc, (kb | kk) != 0);
+          for (int kk = 0; kk < kPrefillBK / 16; ++kk) {  // K = 16 per MMA: 32 bytes along the swizzle row
+            const uint64_t wd = sw128_desc(wa + 32 * kk);
+            mma_bf16(tmem, wd, sw128_desc(aa + 32 * kk), kPfIdesc, (kb | kk) != 0);
+            if (two)
+              mma_bf16(tmem + kPrefillMmaN, wd, sw128_desc(aa + kPfAHalfBytes + 32 * kk), kPfIdesc, (kb | kk) != 0);
+          }
         }
-        mma_commit(empty_w(sw));
-        mma_commit(empty_a(sa));
+        // the weight slot is free in every CTA of the cluster once all their MMAs read it
+        if constexpr (CS > 1) mma_commit_multicast(empty_w(sw), static_cast<uint16_t>((1u << CS) - 1u));
+        else mma_commit(empty_w(sw));
+        if (active) mma_commit(empty_a(sa));
       }
       if (ok) {
-        mma_commit(acc_full);
+        if (active) mma_commit(acc_full);
       } else {  // no MMA may be in flight when the tensor memory is freed
         atomicOr(p.status, kStatusTimeout);
         mma_commit(drain);
@@ -417,10 +471,34 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       }
     }
     __syncwarp();
+  } else if (warp == kPfShareWarp) {
+    // clusters: once this CTA's producer warps have written their rows of a
+    // stage, send them to the same slot of every other CTA (one bulk copy
+    // each, counted there as transaction bytes) and expect the others' rows
+    if constexpr (CS > 1) {
+      if (lane == 0) {
+        constexpr uint32_t kBytes = kRows * 128;  // contiguous rows of the swizzled tile
+        for (int kb = 0; kb < nk; ++kb) {
+          const int s = kb % kPfWStages;
+          if (!pf_wait(share_done(s), (kb / kPfWStages) & 1, p.wait_limit_us)) {
+            atomicOr(p.status, kStatusTimeout);
+            break;
+          }
+          const uint32_t src = w_s + s * kPfWTileBytes + rank * kBytes;
+#pragma unroll
+          for (int d = 0; d < CS; ++d)
+            if (d != rank) bulk_copy_cluster(cluster_addr(src, d), src, kBytes, cluster_addr(full_w(s), d));
+          mbar_arrive_expect_tx(full_w(s), (CS - 1) * kBytes);
+        }
+      }
+    }
+    __syncwarp();
   } else {  // warps 0-7: weight tiles, then the epilogue
-    const int rl = threadIdx.x & (kPrefillBM - 1);  // tile row
-    const int half = threadIdx.x >> 7;               // columns 32 * half .. + 31 of a stage
-    const int64_t r = row0 + rl;
+    // thread -> (row of this CTA's share, kNW-column chunk of a stage)
+    const int chunk = threadIdx.x / kRows;
+    const int rl = threadIdx.x % kRows;
+    const int tr = rank * kRows + rl;  // row in the tile
+    const int64_t r = row0 + tr;
     bool ok = true;
     const bool blocked = p.scale_blocks != 0;
     constexpr int kSB = groups_per_block<F>();
@@ -428,7 +506,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     int64_t blk_cur = -1, blk_nxt = -1;
     for (int kb = 0; kb < nk; ++kb) {
       const int s = kb % kPfWStages;
-      const int64_t c0 = static_cast<int64_t>(kb) * kPrefillBK + 32 * half;
+      const int64_t c0 = static_cast<int64_t>(kb) * kPrefillBK + kNW * chunk;
       const bool valid = r < it.rows && c0 < it.cols;
       PkgWords<K> cur;
 #pragma unroll
@@ -456,9 +534,14 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         } else {
           load_scales<F, K>(it, g, cur);
         }
-        if (!codes_tma) {
+        if (!codes_tma) {  // kNW codes: kNW / 4 bytes (8-aligned for 32, 4 for 16, 2 for 8)
 #pragma unroll
-          for (int i = 0; i < K; ++i) cur.cw[i] = __ldg(reinterpret_cast<const uint2*>(it.codes[i] + (e >> 2)));
+          for (int i = 0; i < K; ++i) {
+            const uint8_t* cp = it.codes[i] + (e >> 2);
+            if constexpr (kNW == 32) cur.cw[i] = __ldg(reinterpret_cast<const uint2*>(cp));
+            else if constexpr (kNW == 16) cur.cw[i].x = __ldg(reinterpret_cast<const unsigned int*>(cp));
+            else cur.cw[i].x = __ldg(reinterpret_cast<const unsigned short*>(cp));
+          }
         }
       }
       if (codes_tma) {  // this stage's codes from the ring; the slot is free once read
@@ -468,47 +551,64 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
           ok = false;
           break;
         }
-        const uint8_t* ct = base + kPfCOffset + sc * kPfCStageBytes + rl * 16 + half * 8;
+        const uint8_t* ct = base + kPfCOffset + sc * kPfCStageBytes + rl * 16 + chunk * (kNW / 4);
 #pragma unroll
-        for (int i = 0; i < K; ++i) cur.cw[i] = *reinterpret_cast<const uint2*>(ct + i * kPfCTileBytes);
+        for (int i = 0; i < K; ++i) {
+          if constexpr (kNW == 32) cur.cw[i] = *reinterpret_cast<const uint2*>(ct + i * kPfCTileBytes);
+          else if constexpr (kNW == 16) cur.cw[i].x = *reinterpret_cast<const uint32_t*>(ct + i * kPfCTileBytes);
+          else cur.cw[i].x = *reinterpret_cast<const uint16_t*>(ct + i * kPfCTileBytes);
+        }
         // every lane's reads before the next copy (async proxy) into the slot
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0) mbar_arrive(empty_c(sc));
       }
-      // the MMAs of this stage's previous round have read its weight tile
+      // the MMAs of this stage's previous round (in every CTA of the
+      // cluster) have read its weight tile
       bool ready = true;
       if (kb >= kPfWStages) ready = pf_wait(empty_w(s), ((kb / kPfWStages) - 1) & 1, p.wait_limit_us);
       if (!__all_sync(kFullMask, ready)) {
         ok = false;
         break;
       }
-      uint32_t h[16];
+      uint32_t h[kNW / 2];
       if (valid) {
-        prefix_weights_bf16<F, K>(cur, h);
+        prefix_weights_bf16<F, K, kNW>(cur, h);
       } else {
 #pragma unroll
-        for (int m = 0; m < 16; ++m) h[m] = 0u;
+        for (int m = 0; m < kNW / 2; ++m) h[m] = 0u;
       }
-      // K-major, 128-byte swizzle: 16-byte piece c of row rl at piece c ^ (rl % 8)
-      uint8_t* const wrow = base + s * kPfWTileBytes + (rl >> 3) * 1024 + (rl & 7) * 128;
+      // K-major, 128-byte swizzle: 16-byte piece c of tile row tr at piece
+      // c ^ (tr % 8), in this stage's slot (the share warp copies this CTA's
+      // rows to the others)
+      uint8_t* const wrow = base + s * kPfWTileBytes + (tr >> 3) * 1024 + (tr & 7) * 128;
 #pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const int piece = (4 * half + q) ^ (rl & 7);
+      for (int q = 0; q < kNW / 8; ++q) {
+        const int piece = (chunk * (kNW / 8) + q) ^ (tr & 7);
         *reinterpret_cast<uint4*>(wrow + 16 * piece) = make_uint4(h[4 * q], h[4 * q + 1], h[4 * q + 2], h[4 * q + 3]);
       }
-      fence_proxy_async_smem();  // visible to the tensor cores (async proxy)
+      fence_proxy_async_smem();  // visible to the async proxy (tensor cores, bulk copies)
       __syncwarp();
-      if (lane == 0) mbar_arrive(full_w(s));
+      if (lane == 0) mbar_arrive(CS == 1 ? full_w(s) : share_done(s));
+    }
+    if constexpr (CS > 1) {
+      // the other CTAs' last commits to this CTA's weight-ring barriers have
+      // landed before it can leave
+      if (ok) {
+        for (int sl = 0; sl < kPfWStages && sl < nk; ++sl) {
+          const int last = sl + ((nk - 1 - sl) / kPfWStages) * kPfWStages;
+          if (!pf_wait(empty_w(sl), (last / kPfWStages) & 1, p.wait_limit_us)) ok = false;
+        }
+      }
     }
     bool have = false;
-    if (ok) have = pf_wait(acc_full, 0, p.wait_limit_us);
+    if (ok && active) have = pf_wait(acc_full, 0, p.wait_limit_us);
     have = __all_sync(kFullMask, have);
-    if (!have && lane == 0) atomicOr(p.status, kStatusTimeout);
+    if (!have && (active || !__all_sync(kFullMask, ok)) && lane == 0) atomicOr(p.status, kStatusTimeout);
     tc_fence_after();
     const int quarter = warp & 3;  // TMEM lanes 32 * quarter .. + 31 of this warp
     const int acc_i = warp >> 2;   // accumulator: tokens t0 + 256 * acc_i ..
-    if (have && (acc_i == 0 || two)) {
+    if (have && active && (acc_i == 0 || two)) {
       const int64_t row = row0 + 32 * quarter + lane;
 #pragma unroll 1
       for (int c = 0; c < kPrefillMmaN / 32; ++c) {
@@ -527,19 +627,47 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (CS > 1) cluster_sync();  // no CTA leaves while another may still write into it
   if (warp == kPfMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kPfTmemCols);
   }
 }
 
+template <int F, int K, int CS>
+cudaError_t prefill_launch_kc(const PrefillBatch& p, cudaStream_t stream) {
+  // (per launch: the attribute belongs to the current device)
+  cudaError_t e =
+      cudaFuncSetAttribute(prefill_kernel<F, K, CS>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPfSmemBytes);
+  if (e != cudaSuccess) return e;
+  if constexpr (CS == 1) {
+    prefill_kernel<F, K, 1><<<static_cast<unsigned>(p.total_tiles), kPfThreads, kPfSmemBytes, stream>>>(p);
+    return cudaGetLastError();
+  } else {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(static_cast<unsigned>(p.total_tiles), 1, 1);  // a multiple of CS
+    cfg.blockDim = dim3(kPfThreads, 1, 1);
+    cfg.dynamicSmemBytes = kPfSmemBytes;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = CS;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, prefill_kernel<F, K, CS>, p);
+  }
+}
+
 template <int F, int K>
 cudaError_t prefill_launch_k(const PrefillBatch& p, cudaStream_t stream) {
-  // (per launch: the attribute belongs to the current device)
-  cudaError_t e = cudaFuncSetAttribute(prefill_kernel<F, K>, cudaFuncAttributeMaxDynamicSharedMemorySize, kPfSmemBytes);
-  if (e != cudaSuccess) return e;
-  prefill_kernel<F, K><<<static_cast<unsigned>(p.total_tiles), kPfThreads, kPfSmemBytes, stream>>>(p);
-  return cudaGetLastError();
+  switch (p.cluster) {
+    case 1: return prefill_launch_kc<F, K, 1>(p, stream);
+    case 2: return prefill_launch_kc<F, K, 2>(p, stream);
+    case 4: return prefill_launch_kc<F, K, 4>(p, stream);
+    default: return cudaErrorInvalidValue;
+  }
 }
 
 template <int F>

@@ -100,9 +100,13 @@ constexpr int kMaxGemvBatch = 8;   // activation rows (tokens) per call
 // One matrix of a prefill launch: Y = A bf16(W~)^T on the tensor cores, with
 // bf16(W~) the prefix-k reconstruction formed from the package in the
 // kernel.  A matrix is cut into tiles of kPrefillBM weight rows by
-// kPrefillBN tokens; the tiles of all matrices of a launch are numbered
-// consecutively (one CTA each, token tile major: the CTAs that run together
-// share activation tiles) and tile_begin is this matrix's first.
+// kPrefillBN tokens.  `cluster` CTAs (1, 2 or 4) with the same row tile and
+// consecutive token tiles form a cluster that shares the weight tiles (each
+// forms 1/cluster of the rows); token tiles are padded to a multiple of
+// `cluster`.  The tiles of all matrices of a launch are numbered
+// consecutively (one CTA each, clusters in token-tile-major order: the CTAs
+// that run together share activation tiles) and tile_begin is this matrix's
+// first.
 struct PrefillItem {
   const uint8_t* codes[kMaxStages];
   const void* scales[kMaxStages];  // float or binary16
@@ -121,10 +125,12 @@ constexpr int kMaxPrefillBatch = 16;  // matrices per launch
 
 struct PrefillBatch {  // (64-byte aligned through its tensor maps)
   CUtensorMap act[kMaxPrefillBatch];  // activations [tokens, cols] bf16: box 64 x kPrefillMmaN, 128-byte swizzle
-  // codes of stage i [rows, cols/4] bytes: box 16 x kPrefillBM (the codes of
-  // one 64-column stage of a row tile); used when codes_tma != 0
+  // codes of stage i [rows, cols/4] bytes: box 16 x (kPrefillBM / cluster)
+  // (the codes of one 64-column stage of a CTA's share of a row tile); used
+  // when codes_tma != 0
   CUtensorMap codes[kMaxPrefillBatch][kMaxStages];
   PrefillItem item[kMaxPrefillBatch];
+  int cluster;                        // CTAs per cluster (1, 2, 4)
   int codes_tma;                      // every matrix has cols % 64 == 0
   int scale_blocks;                   // every matrix has 16-byte rows of scales (and zeros)
   int count;

@@ -134,7 +134,10 @@ def test_integer_packages_exact(shape):
     _status_ok()
 
 
-@pytest.mark.parametrize("shape", [(1, 32, 1), (3, 96, 7), (129, 4096, 257), (64, 12288, 64), (513, 128, 1000)])
+# token tiles of 512: 1 (no cluster), 2 (clusters of 2), 3 and 6 (clusters of
+# 4 with idle padding CTAs), 4
+@pytest.mark.parametrize("shape", [(1, 32, 1), (3, 96, 7), (129, 4096, 257), (64, 12288, 64), (513, 128, 1000),
+                                   (200, 1024, 1100), (77, 2048, 3000), (256, 4096, 2048)])
 def test_shapes(shape):
     rows, cols, tokens = shape
     g = 32 if cols % 64 else 128 if cols % 128 == 0 else 64
@@ -168,7 +171,8 @@ def test_deterministic_and_reconstruction_consistent():
     _status_ok()
 
 
-@pytest.mark.parametrize("shape", [(129, 4096, 257), (256, 4096, 257), (300, 2048, 600)])
+@pytest.mark.parametrize("shape", [(129, 4096, 257), (256, 4096, 257), (300, 2048, 600), (129, 4096, 1500),
+                                   (256, 2048, 2048)])
 def test_repeated_runs_identical(shape):
     """The ring protocols leave no race: five runs of the same call give the
     same bits, and they match the oracle (ragged row and token tiles, the
