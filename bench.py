@@ -621,7 +621,8 @@ def run_e2e(args, mats, pkgs, p_outs, specs, stream, world) -> dict:
     each matrix from pinned host memory to the device, builds its package and
     its k=1..4 reconstructions (rrq_quantize_prefixes), and copies the package
     and every reconstruction back to pinned host buffers, all inside the timed
-    region."""
+    region.  Layers are pipelined over three streams (copy in, build, copy
+    out); the timed region ends when every stream is done."""
     from paper_2608_04048_gb300 import binding
     def pinned_like(t):
         h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
@@ -636,19 +637,42 @@ def run_e2e(args, mats, pkgs, p_outs, specs, stream, world) -> dict:
     d2h = sum(t.numel() * t.element_size() for p in host_pkg for t in p) + \
         len(KS) * sum(sp.numel * 2 for sp in specs)
 
-    f_items = binding.quantize_prefixes_descs(mats, pkgs, p_outs)
+    # one layer (7 matrices) per chunk, on three streams: the copy in of chunk
+    # i+1 and the copy out of chunk i-1 overlap the build of chunk i
+    per = 7
+    chunks = [list(range(i, min(i + per, len(mats)))) for i in range(0, len(mats), per)]
+    c_items = [binding.quantize_prefixes_descs([mats[j] for j in L], [pkgs[j] for j in L], [p_outs[j] for j in L])
+               for L in chunks]
+    dev = mats[0].device
+    s_in, s_out = torch.cuda.Stream(dev), torch.cuda.Stream(dev)
+    ev = lambda: [torch.cuda.Event() for _ in chunks]
+    ev_in, ev_built, ev_out = ev(), ev(), ev()
+    started = [False]
 
     def step():
-        for W, h in zip(mats, host_W):
-            W.copy_(h, non_blocking=True)
-        binding.rrq_quantize_prefixes(mats, GROUP, STAGES, binding.GRID_ASYM, binding.SCALE_F32,
-                                      pkgs, p_outs, stream, f_items)
-        for i, pkg in enumerate(pkgs):
-            for h, d in zip(host_pkg[i], pkg.codes + pkg.scales + pkg.zeros):
-                h.copy_(d, non_blocking=True)
-        for outs_i in p_outs:
-            for o in outs_i:
-                host_out[:o.numel()].view(o.shape).copy_(o, non_blocking=True)
+        for ci, L in enumerate(chunks):
+            with torch.cuda.stream(s_in):
+                if started[0]:  # the previous step's build of this chunk has read W
+                    s_in.wait_event(ev_built[ci])
+                for j in L:
+                    mats[j].copy_(host_W[j], non_blocking=True)
+                ev_in[ci].record(s_in)
+            stream.wait_event(ev_in[ci])
+            if started[0]:  # the previous step's copy out of this chunk is done
+                stream.wait_event(ev_out[ci])
+            binding.rrq_quantize_prefixes([mats[j] for j in L], GROUP, STAGES, binding.GRID_ASYM,
+                                          binding.SCALE_F32, [pkgs[j] for j in L], [p_outs[j] for j in L],
+                                          stream, c_items[ci])
+            ev_built[ci].record(stream)
+            with torch.cuda.stream(s_out):
+                s_out.wait_event(ev_built[ci])
+                for j in L:
+                    for h, d in zip(host_pkg[j], pkgs[j].codes + pkgs[j].scales + pkgs[j].zeros):
+                        h.copy_(d, non_blocking=True)
+                    for o in p_outs[j]:
+                        host_out[:o.numel()].view(o.shape).copy_(o, non_blocking=True)
+                ev_out[ci].record(s_out)
+        started[0] = True
     step()
     torch.cuda.synchronize()
     steps = max(1, args.e2e_steps)
