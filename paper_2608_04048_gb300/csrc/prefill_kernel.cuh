@@ -46,6 +46,13 @@
 
 #include "rrq_device.cuh"
 
+#ifndef PF_PRODUCERS_CS4
+#define PF_PRODUCERS_CS4 4
+#endif
+#ifndef PF_PRODUCERS_CS2
+#define PF_PRODUCERS_CS2 4
+#endif
+
 namespace rrq {
 namespace {
 
@@ -57,7 +64,7 @@ constexpr int kPfAHalfBytes = kPrefillMmaN * 128;    // 256 tokens x 64 bf16 (32
 constexpr int kPfATileBytes = 2 * kPfAHalfBytes;     // 512 tokens (64 KiB)
 constexpr int kPfCTileBytes = kPrefillBM * 16;       // one package stage's codes of a stage (2 KiB)
 constexpr int kPfCStageBytes = kMaxStages * kPfCTileBytes;
-constexpr int kPfDqWarps = 8;                        // weight tiles, then the epilogue
+constexpr int kPfDqWarps = 8;                        // the epilogue (and weight tiles, below)
 constexpr int kPfTmaWarp = 8;
 constexpr int kPfMmaWarp = 9;
 constexpr int kPfCodeWarp = 10;
@@ -314,10 +321,17 @@ __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32
   }
 }
 
+// Warps (of 0-7) that form weight tiles: fewer when a CTA forms few rows,
+// so that each thread's fixed cost per stage covers more weights.
+template <int CS>
+__host__ __device__ constexpr int producer_warps() { return CS == 4 ? PF_PRODUCERS_CS4 : PF_PRODUCERS_CS2; }
+
 template <int F, int K, int CS>
 __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_constant__ PrefillBatch p) {
   constexpr int kRows = kPrefillBM / CS;  // rows of the tile this CTA forms for the cluster
-  constexpr int kNW = 32 / CS;            // weights a thread forms per stage
+  constexpr int kProd = CS == 1 ? kPfDqWarps : producer_warps<CS>();
+  constexpr int kNW = kRows * kPrefillBK / (kProd * 32);  // weights a thread forms per stage
+  static_assert(kNW == 8 || kNW == 16 || kNW == 32, "weights per producer thread");
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw_s = smem_u32(smem_raw);
   const uint32_t base_s = (raw_s + 1023u) & ~1023u;  // swizzled tiles need 1024-byte alignment
@@ -362,9 +376,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       // one CTA: the producer warps; a cluster: one arrival that expects the
       // other CTAs' rows as transaction bytes (this CTA's own rows are ready
       // before it)
-      mbar_init(full_w(s), CS == 1 ? kPfDqWarps : 1);
+      mbar_init(full_w(s), CS == 1 ? kProd : 1);
       mbar_init(empty_w(s), CS);              // every MMA thread of the cluster
-      mbar_init(share_done(s), kPfDqWarps);
+      mbar_init(share_done(s), kProd);
     }
     for (int s = 0; s < kPfAStages; ++s) {
       mbar_init(full_a(s), 1);
@@ -372,7 +386,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     }
     for (int s = 0; s < kPfCStages; ++s) {
       mbar_init(full_c(s), 1);
-      mbar_init(empty_c(s), kPfDqWarps);
+      mbar_init(empty_c(s), kProd);
     }
     mbar_init(acc_full, 1);
     mbar_init(drain, 1);
@@ -500,11 +514,12 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     const int tr = rank * kRows + rl;  // row in the tile
     const int64_t r = row0 + tr;
     bool ok = true;
+    const bool producer = warp < kProd;
     const bool blocked = p.scale_blocks != 0;
     constexpr int kSB = groups_per_block<F>();
     ScaleBlock<K> bc, bn;     // scale blocks in use and the next one (in flight)
     int64_t blk_cur = -1, blk_nxt = -1;
-    for (int kb = 0; kb < nk; ++kb) {
+    for (int kb = 0; producer && kb < nk; ++kb) {
       const int s = kb % kPfWStages;
       const int64_t c0 = static_cast<int64_t>(kb) * kPrefillBK + kNW * chunk;
       const bool valid = r < it.rows && c0 < it.cols;
@@ -594,7 +609,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     if constexpr (CS > 1) {
       // the other CTAs' last commits to this CTA's weight-ring barriers have
       // landed before it can leave
-      if (ok) {
+      if (ok && producer) {
         for (int sl = 0; sl < kPfWStages && sl < nk; ++sl) {
           const int last = sl + ((nk - 1 - sl) / kPfWStages) * kPfWStages;
           if (!pf_wait(empty_w(sl), (last / kPfWStages) & 1, p.wait_limit_us)) ok = false;
