@@ -616,8 +616,13 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
       if (items[base + i].cols % 64 != 0) p.codes_tma = 0;
       if ((items[base + i].cols / group) % (16 / f.scale_bytes()) != 0) p.scale_blocks = 0;
     }
+    // longest rows first: their tiles start in the first waves instead of
+    // forming a long last wave (the tile order is the launch's)
+    int order[rrq::kMaxPrefillBatch];
+    for (int i = 0; i < m; ++i) order[i] = base + i;
+    std::stable_sort(order, order + m, [&](int a, int b) { return items[a].cols > items[b].cols; });
     for (int i = 0; i < m; ++i) {
-      const rrq_gemv_desc& it = items[base + i];
+      const rrq_gemv_desc& it = items[order[i]];
       rrq::PrefillItem& q = p.item[i];
       for (int j = 0; j < rrq::kMaxStages; ++j) {
         const int jj = j < k ? j : k - 1;
