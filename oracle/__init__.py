@@ -118,6 +118,10 @@ class Oracle:
             ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p),
             ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _i32p, _u16p]
         lib.rrq_oracle_reconstruct_bits.restype = ctypes.c_int
+        lib.rrq_oracle_product_bits.argtypes = [
+            ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p), ctypes.c_int64, ctypes.c_int64,
+            ctypes.c_int, ctypes.c_int, _i32p, _u16p, ctypes.c_int64, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
+        lib.rrq_oracle_product_bits.restype = ctypes.c_int
         lib.rrq_oracle_group_pmr.argtypes = [_u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
                                              ctypes.POINTER(ctypes.c_double)]
         lib.rrq_oracle_group_pmr.restype = ctypes.c_int
@@ -330,6 +334,28 @@ class Oracle:
             raise ValueError("oracle rejected the matrix")
         return codes, scales, zeros
 
+    def product_bits(self, codes, scales, zeros, rows, cols, group, k, bits, A_bits, bf16_weights: bool):
+        """Y [tokens, rows] float64: activations (bf16 bit patterns) times the
+        prefix-k weights of a package with per-stage widths, binary32 (decode
+        form) or bf16-rounded (prefill form)."""
+        A_bits = np.ascontiguousarray(np.atleast_2d(A_bits), dtype=np.uint16)
+        tokens = A_bits.shape[0]
+        assert A_bits.shape[1] == cols
+        codes = [np.ascontiguousarray(c, dtype=np.uint8) for c in codes[:k]]
+        scales = [np.ascontiguousarray(a, dtype=np.float32) for a in scales[:k]]
+        zeros = [np.ascontiguousarray(a, dtype=np.float32) for a in zeros[:k]]
+        cp = (_u8p * k)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in scales])
+        zp = (_f32p * k)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        b = (ctypes.c_int * k)(*list(bits)[:k])
+        Y = np.zeros((tokens, rows), np.float64)
+        rc = self.lib.rrq_oracle_product_bits(cp, sp, zp, rows, cols, group, k, b, A_bits.ctypes.data_as(_u16p),
+                                              tokens, int(bf16_weights),
+                                              Y.ctypes.data_as(ctypes.POINTER(ctypes.c_double)))
+        if rc != 0:
+            raise ValueError("oracle rejected the product with per-stage widths")
+        return Y
+
     def reconstruct_bits(self, codes, scales, zeros, rows, cols, group, k, bits):
         codes = [np.ascontiguousarray(c, dtype=np.uint8) for c in codes[:k]]
         scales = [np.ascontiguousarray(a, dtype=np.float32) for a in scales[:k]]
@@ -416,6 +442,10 @@ def quantize_bits(W_bits, group, bits):
 
 def reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits):
     return load().reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits)
+
+
+def product_bits(codes, scales, zeros, rows, cols, group, k, bits, A_bits, bf16_weights: bool):
+    return load().product_bits(codes, scales, zeros, rows, cols, group, k, bits, A_bits, bf16_weights)
 
 
 def group_pmr(W_bits, group):

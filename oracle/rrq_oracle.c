@@ -605,3 +605,42 @@ int rrq_oracle_prefill(const uint8_t* const* codes, const void* const* scales,
   free(wrow);
   return 0;
 }
+
+/* Products with the prefix weights of a package with per-stage widths
+ * (asymmetric grid, codes LSB-first at bits[i] per weight): the prefix-k
+ * weight is the binary32 stage sum of zero + fl(Q s), as in
+ * rrq_oracle_reconstruct_bits; taken as it is (the decode form) or rounded
+ * to nearest-even bf16 (the prefill form, bf16_weights != 0), and
+ * Y[t][r] = sum_c w(r, c) A[t][c] in binary64. */
+int rrq_oracle_product_bits(const uint8_t* const* codes, const float* const* scales,
+                            const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
+                            const int* bits, const uint16_t* A, int64_t tokens, int bf16_weights,
+                            double* Y) {
+  if (!codes || !scales || !zeros || !bits || !A || !Y) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || k < 1 || tokens < 1 || cols % group != 0) return -1;
+  for (int i = 0; i < k; ++i)
+    if (bits[i] < 1 || bits[i] > 4) return -1;
+  double* wts = (double*)malloc(sizeof(double) * (size_t)cols);
+  if (!wts) return -1;
+  for (int64_t r = 0; r < rows; ++r) {
+    for (int64_t j = 0; j < cols; ++j) {
+      const int64_t c = r * cols + j;
+      const int64_t g = c / group;
+      float running = 0.0f;
+      for (int st = 0; st < k; ++st) {
+        const int code = get_bits(codes[st], c, bits[st]);
+        const float scaled = (float)code * scales[st][g];
+        const float lvl = zeros[st][g] + scaled;
+        running = st == 0 ? lvl : running + lvl;
+      }
+      wts[j] = bf16_weights ? (double)rrq_oracle_bf16_to_f32(rrq_oracle_f32_to_bf16(running)) : (double)running;
+    }
+    for (int64_t t = 0; t < tokens; ++t) {
+      double sum = 0.0;
+      for (int64_t j = 0; j < cols; ++j) sum += wts[j] * (double)rrq_oracle_bf16_to_f32(A[(size_t)t * cols + j]);
+      Y[(size_t)t * rows + r] = sum;
+    }
+  }
+  free(wts);
+  return 0;
+}

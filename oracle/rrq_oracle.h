@@ -96,6 +96,16 @@ int rrq_oracle_prefill(const uint8_t* const* codes, const void* const* scales,
                        const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
                        int grid_sym, int scale_f16, const uint16_t* A, int64_t tokens, double* Y);
 
+/* Products (decode form with binary32 weights, prefill form with bf16
+ * weights when bf16_weights != 0) with the prefix-k weights of a package with
+ * per-stage widths bits[i] in 1..4 (asymmetric grid):
+ * Y[t][r] = sum_c w(r, c) A[t][c] in binary64.
+ *   A  bf16 bit patterns [tokens][cols];  Y  double [tokens][rows]. */
+int rrq_oracle_product_bits(const uint8_t* const* codes, const float* const* scales,
+                            const float* const* zeros, int64_t rows, int64_t cols, int group, int k,
+                            const int* bits, const uint16_t* A, int64_t tokens, int bf16_weights,
+                            double* Y);
+
 /* Asymmetric stages with per-stage widths bits[k] in 1..4 (2^b levels,
  * 2^b - 1 steps).  Group form as rrq_oracle_quantize_group; matrix form packs
  * stage k's codes LSB-first, element c at bits bits[k]*c.., into

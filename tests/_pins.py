@@ -1046,6 +1046,113 @@ def pin_prefill_vs_binary32_product(orc, seed=73, rows=4, g=128) -> list[str]:
     return fails
 
 
+# ---------------------------------------------------------------------------
+# products with per-stage widths (decode form: binary32 weights; prefill form:
+# bf16 weights)
+# ---------------------------------------------------------------------------
+BITS_SPLITS = ([1, 3], [3, 1], [4, 2, 1], [2, 4], [1, 1, 1, 1])
+
+
+def _bits_package(orc, rng, rows, cols, g, bits):
+    xs = np.concatenate(_random_groups(rng, rows * cols // g, g)).reshape(rows, cols)
+    return orc.quantize_bits(bf16_bits_of_f32(xs), g, bits)
+
+
+def pin_product_bits_two_bit_case(orc, seed=79, rows=5, g=64) -> list[str]:
+    """With every width 2 the product equals the 2-bit products pinned above:
+    the decode form rrq_oracle_gemv and the prefill form rrq_oracle_prefill,
+    exactly."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 3 * g
+    xs = np.concatenate(_random_groups(rng, rows * 3, g)).reshape(rows, cols)
+    codes, scales, zeros = orc.quantize(bf16_bits_of_f32(xs), group=g, n_stages=4)
+    A = bf16_round_bits(rng.normal(0, 1, (3, cols)).astype(np.float32))
+    for k in range(1, 5):
+        yd = orc.product_bits(codes, scales, zeros, rows, cols, g, k, [2] * 4, A, False)
+        yp = orc.product_bits(codes, scales, zeros, rows, cols, g, k, [2] * 4, A, True)
+        if not np.array_equal(yd, orc.gemv(codes, scales, zeros, rows, cols, g, k, A)):
+            fails.append(f"k={k}: decode form with widths 2 differs from the 2-bit product")
+        if not np.array_equal(yp, orc.prefill(codes, scales, zeros, rows, cols, g, k, A)):
+            fails.append(f"k={k}: prefill form with widths 2 differs from the 2-bit prefill product")
+    return fails
+
+
+def pin_product_bits_one_hot(orc, seed=83, rows=4, g=32) -> list[str]:
+    """One-hot activation rows pick single weights: the prefill form returns the
+    width reconstruction (pinned above) exactly, and the decode form rounds to
+    it, for several splits and every prefix."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 4 * g
+    perm = rng.permutation(cols)
+    E = np.zeros((cols, cols), np.float32)
+    E[np.arange(cols), perm] = 1.0
+    E = bf16_bits_of_f32(E)
+    for bits in BITS_SPLITS:
+        codes, scales, zeros = _bits_package(orc, rng, rows, cols, g, bits)
+        for k in range(1, len(bits) + 1):
+            rec = orc.reconstruct_bits(codes, scales, zeros, rows, cols, g, k, bits)
+            recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+            yp = orc.product_bits(codes, scales, zeros, rows, cols, g, k, bits, E, True)
+            yd = orc.product_bits(codes, scales, zeros, rows, cols, g, k, bits, E, False)
+            if not np.array_equal(yp, recf[:, perm].T):
+                fails.append(f"{bits} k={k}: one-hot prefill form is not the width reconstruction")
+            if not np.array_equal(bf16_round_bits(yd.astype(np.float32)), rec[:, perm].T):
+                fails.append(f"{bits} k={k}: one-hot decode form does not round to the reconstruction")
+    return fails
+
+
+def pin_product_bits_integer_exact(orc, seed=89, rows=5, g=32) -> list[str]:
+    """Scale 1 and integer zeros make every level an integer: the products
+    (both forms) equal numpy's int64 matmul of weights whose codes are
+    unpacked here with numpy's little-endian bit order."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 4 * g
+    n = rows * cols
+    A_int = rng.integers(-4, 5, (6, cols))
+    A = bf16_bits_of_f32(A_int.astype(np.float32))
+    for bits in BITS_SPLITS:
+        q = [rng.integers(0, 1 << b, n) for b in bits]
+        z = [rng.integers(-3, 4, n // g) for _ in bits]
+        codes = []
+        for qi, b in zip(q, bits):
+            bitsarr = ((qi[:, None] >> np.arange(b)) & 1).astype(np.uint8).reshape(-1)
+            codes.append(np.packbits(bitsarr, bitorder="little"))
+        scales = [np.ones(n // g, np.float32) for _ in bits]
+        zeros = [zi.astype(np.float32) for zi in z]
+        for k in range(1, len(bits) + 1):
+            w = sum(q[i] + np.repeat(z[i], g) for i in range(k)).reshape(rows, cols)
+            want = (A_int @ w.T).astype(np.float64)
+            for bf in (False, True):
+                Y = orc.product_bits(codes, scales, zeros, rows, cols, g, k, bits, A, bf)
+                if not np.array_equal(Y, want):
+                    fails.append(f"{bits} k={k} bf16={bf}: integer product differs from the int64 matmul")
+    return fails
+
+
+def pin_product_bits_forms(orc, seed=97, rows=4, g=64) -> list[str]:
+    """The prefill form differs from the decode form by at most the bf16
+    rounding of each weight (2^-9 relative), and does differ."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 2 * g
+    A = bf16_round_bits(rng.normal(0, 1, (5, cols)).astype(np.float32))
+    Af = (A.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+    for bits in BITS_SPLITS[:3]:
+        codes, scales, zeros = _bits_package(orc, rng, rows, cols, g, bits)
+        k = len(bits)
+        rec = orc.reconstruct_bits(codes, scales, zeros, rows, cols, g, k, bits)
+        recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        yd = orc.product_bits(codes, scales, zeros, rows, cols, g, k, bits, A, False)
+        yp = orc.product_bits(codes, scales, zeros, rows, cols, g, k, bits, A, True)
+        tol = np.abs(Af) @ np.abs(recf).T * 2.0 ** -8 + 1e-300
+        if np.any(np.abs(yp - yd) > tol) or np.array_equal(yp, yd):
+            fails.append(f"{bits}: the two forms are not within bf16 rounding of each other")
+    return fails
+
+
 ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_brute_force_tiny,
             pin_invariants, pin_exact_grid, pin_prefix_reconstruction, pin_f16_rounding,
             pin_sym_worked_groups, pin_sym_brute_force_exact, pin_sym_invariants,
@@ -1053,7 +1160,8 @@ ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_bru
             pin_base_residual_invariants, pin_gemv_worked, pin_gemv_is_input_minus_residual,
             pin_gemv_vs_bf16_reconstruction, pin_bits_worked_and_two_bit_case, pin_bits_brute_force_exact,
             pin_bits_invariants_and_packing, pin_group_pmr, pin_prefill_worked, pin_prefill_one_hot,
-            pin_prefill_integer_exact, pin_prefill_vs_binary32_product]
+            pin_prefill_integer_exact, pin_prefill_vs_binary32_product, pin_product_bits_two_bit_case,
+            pin_product_bits_one_hot, pin_product_bits_integer_exact, pin_product_bits_forms]
 
 
 def all_failures(orc) -> list[str]:

@@ -85,6 +85,13 @@ MUTANTS = {
     "prefill_code_bit_order": ("const int code = (codes[st][c / 4] >> (2 * (c % 4))) & 3;",
                                "const int code = (codes[st][c / 4] >> (2 * (3 - c % 4))) & 3;"),
     "prefill_first_group_only": ("  const int64_t g = c / group;\n  float sum", "  const int64_t g = 0;\n  float sum"),
+    # products with per-stage widths
+    "pbits_drops_base": ("running = st == 0 ? lvl : running + lvl;", "running = st == 0 ? 0.0f : running + lvl;"),
+    "pbits_ignores_widths": ("const int code = get_bits(codes[st], c, bits[st]);", "const int code = get_bits(codes[st], c, 2);"),
+    "pbits_never_rounds": ("wts[j] = bf16_weights ? (double)rrq_oracle_bf16_to_f32(rrq_oracle_f32_to_bf16(running)) : (double)running;",
+                           "wts[j] = (double)running;"),
+    "pbits_wrong_output_row": ("Y[(size_t)t * rows + r] = sum;", "Y[(size_t)t * rows + (rows - 1 - r)] = sum;"),
+    "pbits_first_stage_zero": ("const float lvl = zeros[st][g] + scaled;", "const float lvl = zeros[0][g] + scaled;"),
 }
 
 
