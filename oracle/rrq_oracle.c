@@ -627,7 +627,7 @@ int rrq_oracle_product_bits(const uint8_t* const* codes, const float* const* sca
       const int64_t c = r * cols + j;
       const int64_t g = c / group;
       float running = 0.0f;
-      for (int st = 0; st < k; ++st) {
+      for (int st = 0; st != k; ++st) {
         const int code = get_bits(codes[st], c, bits[st]);
         const float scaled = (float)code * scales[st][g];
         const float lvl = zeros[st][g] + scaled;
