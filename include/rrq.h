@@ -334,10 +334,10 @@ rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt
  * the partial sums is the hardware's; the result is deterministic).  The
  * items are rrq_gemv_desc with A_bf16 = [tokens, cols] and Y = float [tokens,
  * rows], both row-major and 16-byte aligned.  1 <= tokens <=
- * RRQ_MAX_PREFILL_TOKENS; 1 <= k <= fmt->n_stages; 2-bit stages only
- * (RRQ_ERR_UNSUPPORTED for other widths).  Y must not overlap any input or
- * another Y.  One launch per 16 matrices; other rules as for
- * rrq_reconstruct_ex. */
+ * RRQ_MAX_PREFILL_TOKENS; 1 <= k <= fmt->n_stages.  Per-stage widths
+ * (fmt->bits, asymmetric grid) are taken with the reconstruction's weights of
+ * that format.  Y must not overlap any input or another Y.  One launch per 16
+ * matrices; other rules as for rrq_reconstruct_ex. */
 rrq_status rrq_prefill(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int64_t tokens,
                        rrq_stream_t stream);
 

@@ -554,7 +554,7 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
                          rrq_stream_t stream) {
   if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
   if (tokens < 1 || tokens > RRQ_MAX_PREFILL_TOKENS) return RRQ_ERR_INVALID_ARG;
-  if (f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
+  const bool widths = f.kind == rrq::kAsymBits;
   const int group = f.group;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (2 + 3 * k));
@@ -572,7 +572,7 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
     ranges.push_back(range_of(it.A_bf16, 2 * static_cast<uint64_t>(tokens) * it.cols, false));
     ranges.push_back(range_of(it.Y, 4 * static_cast<uint64_t>(tokens) * it.rows, true));
     for (int j = 0; j < k; ++j) {
-      ranges.push_back(range_of(it.codes[j], n / 4, false));
+      ranges.push_back(range_of(it.codes[j], f.code_bytes(n, j), false));
       ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
       if (!f.sym()) ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
     }
@@ -597,7 +597,8 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
   // clusters share weight tiles across token tiles: 4 CTAs for the longer
   // prefixes (forming weights costs most there), else 2 (measured best on
   // Qwen3-8B-shaped layers at 2048 tokens)
-  const int cluster = (k >= 3 && token_tiles >= 3) ? 4 : token_tiles >= 2 ? 2 : 1;
+  // (per-stage widths: one CTA, each thread forming whole 32-weight words)
+  const int cluster = widths ? 1 : (k >= 3 && token_tiles >= 3) ? 4 : token_tiles >= 2 ? 2 : 1;
   const int64_t token_tiles_padded = (token_tiles + cluster - 1) / cluster * cluster;
   static thread_local rrq::PrefillBatch p;
   for (int base = 0; base < count; base += rrq::kMaxPrefillBatch) {
@@ -610,8 +611,9 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
     p.wait_limit_us = g_wait_limit_us.load(std::memory_order_relaxed);
     p.status = st->status;
     int64_t tiles = 0;
-    p.codes_tma = 1;
+    p.codes_tma = widths ? 0 : 1;
     p.scale_blocks = 1;
+    for (int j = 0; j < rrq::kMaxStages; ++j) p.bits[j] = f.bits[j];
     for (int i = 0; i < m; ++i) {
       if (items[base + i].cols % 64 != 0) p.codes_tma = 0;
       if ((items[base + i].cols / group) % (16 / f.scale_bytes()) != 0) p.scale_blocks = 0;

@@ -22,7 +22,9 @@
 //   - warp 10 loads the stage's codes of this CTA's rows (one 2-D TMA box of
 //     16 bytes x 128/CS rows per package stage) into a 4-deep ring;
 //   - warps 0-7 take the codes from that ring (or load them themselves when
-//     a matrix's code rows are not 16-byte multiples) and the scales and
+//     a matrix's code rows are not 16-byte multiples, and for packages with
+//     per-stage widths: b words per 32 weights, formed by the
+//     reconstruction's width-generic routine) and the scales and
 //     zeros as 16-byte blocks a block ahead, form this CTA's rows of the bf16
 //     weight tile in registers and store them in the K-major
 //     128-byte-swizzled layout into a 3-deep ring;
@@ -198,6 +200,7 @@ __device__ __forceinline__ bool pf_wait(uint32_t bar, uint32_t parity, uint32_t 
 template <int K>
 struct PkgWords {
   uint2 cw[K];   // stage-i codes, LSB first, 2 bits each
+  uint4 cb[K];   // per-stage widths: stage-i codes, b 32-bit words (b = the stage's width)
   float sc[K];   // stage-i scale
   float zr[K];   // stage-i zero (asymmetric grid)
 };
@@ -218,7 +221,7 @@ __device__ __forceinline__ void load_block(const PrefillItem& it, int64_t b, Sca
 #pragma unroll
   for (int i = 0; i < K; ++i) {
     sb.s[i] = __ldg(static_cast<const uint4*>(it.scales[i]) + b);
-    if constexpr (F == kAsymF32) sb.z[i] = __ldg(reinterpret_cast<const uint4*>(it.zeros[i]) + b);
+    if constexpr (F == kAsymF32 || F == kAsymBits) sb.z[i] = __ldg(reinterpret_cast<const uint4*>(it.zeros[i]) + b);
   }
 }
 
@@ -237,7 +240,7 @@ __device__ __forceinline__ void from_block(const ScaleBlock<K>& sb, int gi, PkgW
     } else {
       w.sc[i] = __uint_as_float(pick_word(sb.s[i], gi));
     }
-    w.zr[i] = (F == kAsymF32) ? __uint_as_float(pick_word(sb.z[i], gi)) : 0.0f;
+    w.zr[i] = (F == kAsymF32 || F == kAsymBits) ? __uint_as_float(pick_word(sb.z[i], gi)) : 0.0f;
   }
 }
 
@@ -250,7 +253,7 @@ __device__ __forceinline__ void load_scales(const PrefillItem& it, int64_t g, Pk
       w.sc[i] = __half2float(__ushort_as_half(__ldg(static_cast<const unsigned short*>(it.scales[i]) + g)));
     else
       w.sc[i] = __ldg(static_cast<const float*>(it.scales[i]) + g);
-    w.zr[i] = (F == kAsymF32) ? __ldg(it.zeros[i] + g) : 0.0f;
+    w.zr[i] = (F == kAsymF32 || F == kAsymBits) ? __ldg(it.zeros[i] + g) : 0.0f;
   }
 }
 
@@ -527,6 +530,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
 #pragma unroll
       for (int i = 0; i < K; ++i) {
         cur.cw[i] = make_uint2(0u, 0u);
+        cur.cb[i] = make_uint4(0u, 0u, 0u, 0u);
         cur.sc[i] = 0.0f;
         cur.zr[i] = 0.0f;
       }
@@ -549,7 +553,17 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         } else {
           load_scales<F, K>(it, g, cur);
         }
-        if (!codes_tma) {  // kNW codes: kNW / 4 bytes (8-aligned for 32, 4 for 16, 2 for 8)
+        if constexpr (F == kAsymBits) {  // 32 weights of width b: b words at word b * (e / 32)
+#pragma unroll
+          for (int i = 0; i < K; ++i) {
+            const int b = p.bits[i];
+            const uint32_t* wp = reinterpret_cast<const uint32_t*>(it.codes[i]) + (e >> 5) * b;
+            cur.cb[i].x = __ldg(wp);
+            if (b > 1) cur.cb[i].y = __ldg(wp + 1);
+            if (b > 2) cur.cb[i].z = __ldg(wp + 2);
+            if (b > 3) cur.cb[i].w = __ldg(wp + 3);
+          }
+        } else if (!codes_tma) {  // kNW codes: kNW / 4 bytes (8-aligned for 32, 4 for 16, 2 for 8)
 #pragma unroll
           for (int i = 0; i < K; ++i) {
             const uint8_t* cp = it.codes[i] + (e >> 2);
@@ -588,7 +602,28 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
       }
       uint32_t h[kNW / 2];
       if (valid) {
-        prefix_weights_bf16<F, K, kNW>(cur, h);
+        if constexpr (F == kAsymBits) {
+          static_assert(kNW == 32, "per-stage widths take whole 32-weight words");
+          f32x2 acc[16];
+#pragma unroll
+          for (int i = 0; i < K; ++i) {
+            switch (p.bits[i]) {
+              case 1: dequant_bits<1>(cur.cb[i], cur.sc[i], cur.zr[i], i == 0, acc); break;
+              case 3: dequant_bits<3>(cur.cb[i], cur.sc[i], cur.zr[i], i == 0, acc); break;
+              case 4: dequant_bits<4>(cur.cb[i], cur.sc[i], cur.zr[i], i == 0, acc); break;
+              default: dequant_bits<2>(cur.cb[i], cur.sc[i], cur.zr[i], i == 0, acc); break;
+            }
+          }
+#pragma unroll
+          for (int m = 0; m < 16; ++m) {
+            float a, b;
+            unpack2(acc[m], a, b);
+            const __nv_bfloat162 x = __floats2bfloat162_rn(a, b);
+            h[m] = *reinterpret_cast<const uint32_t*>(&x);
+          }
+        } else {
+          prefix_weights_bf16<F, K, kNW>(cur, h);
+        }
       } else {
 #pragma unroll
         for (int m = 0; m < kNW / 2; ++m) h[m] = 0u;
@@ -677,11 +712,15 @@ cudaError_t prefill_launch_kc(const PrefillBatch& p, cudaStream_t stream) {
 
 template <int F, int K>
 cudaError_t prefill_launch_k(const PrefillBatch& p, cudaStream_t stream) {
-  switch (p.cluster) {
-    case 1: return prefill_launch_kc<F, K, 1>(p, stream);
-    case 2: return prefill_launch_kc<F, K, 2>(p, stream);
-    case 4: return prefill_launch_kc<F, K, 4>(p, stream);
-    default: return cudaErrorInvalidValue;
+  if constexpr (F == kAsymBits) {  // one CTA per cluster (the host asks for no more)
+    return p.cluster == 1 ? prefill_launch_kc<F, K, 1>(p, stream) : cudaErrorInvalidValue;
+  } else {
+    switch (p.cluster) {
+      case 1: return prefill_launch_kc<F, K, 1>(p, stream);
+      case 2: return prefill_launch_kc<F, K, 2>(p, stream);
+      case 4: return prefill_launch_kc<F, K, 4>(p, stream);
+      default: return cudaErrorInvalidValue;
+    }
   }
 }
 

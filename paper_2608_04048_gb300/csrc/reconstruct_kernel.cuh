@@ -61,25 +61,6 @@ __host__ __device__ constexpr int warp_smem_bytes() { return kRing * K * stage_b
 template <int K, int F>
 __host__ __device__ constexpr int smem_bytes() { return kWarps * warp_smem_bytes<K, F>(); }
 
-// Stage values of 32 codes of width B (element j at bits B*j of w), natural
-// order: acc = level (first stage) or fl(acc + level).
-template <int B>
-__device__ __forceinline__ void dequant_bits(const uint4& w4, float s, float z, bool first, f32x2 (&acc)[16]) {
-  const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
-  auto code = [&](int j) -> uint32_t {
-    const int bit = B * j, i = bit >> 5, sh = bit & 31;
-    uint32_t c = w[i] >> sh;
-    if (sh + B > 32) c |= w[i + 1] << (32 - sh);
-    return c & ((1u << B) - 1u);
-  };
-  const f32x2 S = pack2(s, s), Z = pack2(z, z), T23 = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f);
-#pragma unroll
-  for (int m = 0; m < 16; ++m) {
-    const f32x2 t = pack2u(0x4B000000u | code(2 * m), 0x4B000000u | code(2 * m + 1));
-    const f32x2 level = add2(Z, fma2(sub2(t, T23), S, Z0));  // fl(zero + fl(Q s))
-    acc[m] = first ? level : add2(acc[m], level);
-  }
-}
 
 // kAllPrefixes: write the reconstruction after every stage i < K (prefixes
 // 1..K in one pass over the package) instead of only after stage K-1.

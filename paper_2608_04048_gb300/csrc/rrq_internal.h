@@ -130,7 +130,8 @@ struct PrefillBatch {  // (64-byte aligned through its tensor maps)
   // when codes_tma != 0
   CUtensorMap codes[kMaxPrefillBatch][kMaxStages];
   PrefillItem item[kMaxPrefillBatch];
-  int cluster;                        // CTAs per cluster (1, 2, 4)
+  int cluster;                        // CTAs per cluster (1, 2, 4; 1 with per-stage widths)
+  int bits[kMaxStages];               // per-stage code widths (kAsymBits)
   int codes_tma;                      // every matrix has cols % 64 == 0
   int scale_blocks;                   // every matrix has 16-byte rows of scales (and zeros)
   int count;
@@ -144,12 +145,14 @@ struct PrefillBatch {  // (64-byte aligned through its tensor maps)
 cudaError_t prefill_launch_asym_f32(int k, const PrefillBatch& p, cudaStream_t stream);
 cudaError_t prefill_launch_sym_f32(int k, const PrefillBatch& p, cudaStream_t stream);
 cudaError_t prefill_launch_sym_f16(int k, const PrefillBatch& p, cudaStream_t stream);
+cudaError_t prefill_launch_asym_bits(int k, const PrefillBatch& p, cudaStream_t stream);
 
 inline cudaError_t prefill_launch(Format fmt, int k, const PrefillBatch& p, cudaStream_t stream) {
   switch (fmt) {
     case kAsymF32: return prefill_launch_asym_f32(k, p, stream);
     case kSymF32: return prefill_launch_sym_f32(k, p, stream);
     case kSymF16: return prefill_launch_sym_f16(k, p, stream);
+    case kAsymBits: return prefill_launch_asym_bits(k, p, stream);
     default: return cudaErrorInvalidValue;
   }
 }

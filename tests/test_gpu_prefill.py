@@ -222,6 +222,40 @@ def test_qwen3_8b_layer_sampled():
     _status_ok()
 
 
+@pytest.mark.parametrize("group", [32, 128])
+@pytest.mark.parametrize("bits", [(1, 3), (3, 1), (4, 2, 1), (2, 4), (1, 1, 1, 1), (4, 4)],
+                         ids=lambda b: "+".join(map(str, b)))
+def test_widths(bits, group):
+    """Packages with per-stage widths: every prefix against the oracle's
+    prefill form (bf16 prefix weights) within the same bound, and one-hot
+    rows returning the width reconstruction (rrq_reconstruct_ex) exactly."""
+    rows, cols, tokens = 200, 8 * group, 600
+    W = workloads.generate(rows, cols, 90 + sum(bits), "t3_rowout", "cuda")
+    (pkg,) = binding.rrq_quantize_ex([W], group, len(bits), binding.GRID_ASYM, binding.SCALE_F32, bits=bits)
+    A = _acts(tokens, cols, seed=len(bits) + group)
+    torch.cuda.synchronize()
+    codes = [c.cpu().numpy() for c in pkg.codes]
+    scales = [x.cpu().numpy() for x in pkg.scales]
+    zeros = [x.cpu().numpy() for x in pkg.zeros]
+    Ab = bf16_bits(A)
+    Af = np.abs((Ab.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+    perm = torch.randperm(cols, generator=torch.Generator().manual_seed(group))
+    E = torch.zeros((cols, cols), dtype=torch.bfloat16, device="cuda")
+    E[torch.arange(cols), perm.cuda()] = 1.0
+    for k in range(1, len(bits) + 1):
+        (Y,) = binding.rrq_prefill([pkg], [A], k)
+        want = oracle.product_bits(codes, scales, zeros, rows, cols, group, k, bits, Ab, True)
+        rec = oracle.reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits)
+        recf = np.abs((rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+        tol = (cols / 16 + 2) * 2.0 ** -23 * (Af @ recf.T) + 1e-30
+        err = np.abs(Y.cpu().numpy().astype(np.float64) - want)
+        assert not np.any(err > tol), f"{bits} g{group} k{k}: {int((err > tol).sum())} outputs beyond the bound"
+        (Yh,) = binding.rrq_prefill([pkg], [E], k)
+        rec_gpu = binding.rrq_reconstruct_ex([pkg], k)[0][0]
+        assert torch.equal(Yh, rec_gpu.float()[:, perm.cuda()].T.contiguous()), f"{bits} g{group} k{k}: one-hot"
+    _status_ok()
+
+
 def test_errors():
     W = workloads.generate(8, 256, 1, "normal", "cuda")
     pkg = binding.rrq_quantize(W, 128, 2)
@@ -232,10 +266,6 @@ def test_errors():
     with pytest.raises(binding.RRQError) as e:
         binding.rrq_prefill([pkg], [A], 1, ys=[Yover])
     assert e.value.status == 1
-    (bpkg,) = binding.rrq_quantize_ex([W], 128, 2, binding.GRID_ASYM, binding.SCALE_F32, bits=(1, 3))
-    with pytest.raises(binding.RRQError) as e:
-        binding.rrq_prefill([bpkg], [A], 1)
-    assert e.value.status == 2
     _status_ok()
 
 
