@@ -317,8 +317,10 @@ typedef struct {
  * k x (2 + 16/g) for the binary16 symmetric format) and sums each row in a
  * fixed order in binary32 (deterministic; |Y - exact| <= gamma_cols *
  * sum_c |W~ A|).  For decoding: 1 <= batch <= RRQ_MAX_GEMV_BATCH activation
- * rows; 1 <= k <= fmt->n_stages.  Y must not overlap any input or another Y.
- * One launch per 64 matrices; other rules as for rrq_reconstruct_ex. */
+ * rows; 1 <= k <= fmt->n_stages.  Per-stage widths (fmt->bits, asymmetric
+ * grid) are taken with the reconstruction's stage sum of that format.  Y must
+ * not overlap any input or another Y.  One launch per 64 matrices; other
+ * rules as for rrq_reconstruct_ex. */
 rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
                     rrq_stream_t stream);
 

@@ -402,7 +402,6 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
                       rrq_stream_t stream) {
   if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
   if (batch < 1 || batch > rrq::kMaxGemvBatch) return RRQ_ERR_INVALID_ARG;
-  if (f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
   const int group = f.group;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (2 + 3 * k));
@@ -419,7 +418,7 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
     ranges.push_back(range_of(it.A_bf16, 2 * static_cast<uint64_t>(batch) * it.cols, false));
     ranges.push_back(range_of(it.Y, 4 * static_cast<uint64_t>(batch) * it.rows, true));
     for (int j = 0; j < k; ++j) {
-      ranges.push_back(range_of(it.codes[j], n / 4, false));
+      ranges.push_back(range_of(it.codes[j], f.code_bytes(n, j), false));
       ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
       if (!f.sym()) ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
     }
@@ -446,6 +445,7 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
     std::memset(&p, 0, sizeof p);
     p.count = m;
     p.log2g = log2g;
+    for (int j = 0; j < rrq::kMaxStages; ++j) p.bits[j] = f.bits[j];
     int64_t blocks = 0, max_cols = 0;
     for (int i = 0; i < m; ++i) {
       const rrq_gemv_desc& it = items[base + i];
@@ -485,7 +485,7 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
       p.cta_begin[p.grid] = blocks;
     }
     // activation rows per launch: as many as shared memory holds
-    const int per = rrq::gemv_rows_per_launch(k, max_cols);
+    const int per = rrq::gemv_rows_per_launch(f.kind, k, max_cols);
     if (per < 1) return RRQ_ERR_UNSUPPORTED;
     for (int b0 = 0; b0 < batch; b0 += per) {
       const int nb = std::min(per, batch - b0);

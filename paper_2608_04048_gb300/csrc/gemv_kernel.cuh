@@ -48,12 +48,17 @@ static_assert(kRows == kWarps, "one row of a block per warp");
 // ring depth (chunks per warp in shared memory, two ahead of use)
 template <int K>
 __host__ __device__ constexpr int ring_depth() { return 3; }
-constexpr int kStageBytes = 512;       // one stage of one chunk: codes 256 B | scales 128 B | zeros 128 B
+// one stage of one chunk: codes (256 B at 2 bits, up to 512 B with per-stage
+// widths: 16 B per lane) | scales 128 B | zeros 128 B
+template <int F>
+__host__ __device__ constexpr int code_area() { return F == kAsymBits ? 512 : 256; }
+template <int F>
+__host__ __device__ constexpr int stage_bytes() { return code_area<F>() + 256; }
 constexpr int kMaxSmem = 227 * 1024;
 constexpr float kTwo23 = 8388608.0f;
 
-template <int K>
-__host__ __device__ constexpr int ring_bytes() { return kWarps * ring_depth<K>() * K * kStageBytes; }
+template <int F, int K>
+__host__ __device__ constexpr int ring_bytes() { return kWarps * ring_depth<K>() * K * stage_bytes<F>(); }
 
 // swizzled position of 16-byte activation piece P of a row
 __device__ __forceinline__ uint32_t act_piece(uint32_t P) { return P ^ ((P >> 3) & 7u); }
@@ -71,10 +76,12 @@ __global__ void __launch_bounds__(kThreads, 1)
 gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
+  constexpr int kStageBytes = stage_bytes<F>();
+  constexpr int kCA = code_area<F>();  // scales at kCA, zeros at kCA + 128
   constexpr int kBuf = K * kStageBytes;
   constexpr int kRing = ring_depth<K>();
   extern __shared__ __align__(128) uint8_t smem[];
-  float* act = reinterpret_cast<float*>(smem + ring_bytes<K>());  // [B][act_floats], swizzled pieces
+  float* act = reinterpret_cast<float*>(smem + ring_bytes<F, K>());  // [B][act_floats], swizzled pieces
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
   uint8_t* ring = smem + warp * kRing * kBuf;
@@ -140,9 +147,24 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
       const uint32_t base = ring_s + buf * kBuf;
 #pragma unroll
       for (int i = 0; i < K; ++i) {
-        cp_async_8(base + i * kStageBytes + lane * 8, cp[i] + off_code, n8);
-        cp_async_4(base + i * kStageBytes + 256 + lane * 4, sp[i] + off_meta, n_scale);
-        if (!kSym) cp_async_4(base + i * kStageBytes + 384 + lane * 4, zp[i] + off_meta, n4);
+        if constexpr (F == kAsymBits) {  // 4b bytes of b-bit codes for the lane's 32 weights
+          const int b = p.bits[i];
+          const char* src = cp[i] + (valid ? (e >> 5) * 4 * static_cast<uint64_t>(b) : 0);
+          const uint32_t dst = base + i * kStageBytes + lane * 16;
+          if (b == 4) cp_async_16(dst, src, valid ? 16u : 0u);
+          else if (b == 2) cp_async_8(dst, src, n8);
+          else {
+            cp_async_4(dst, src, n4);
+            if (b == 3) {
+              cp_async_4(dst + 4, src + 4, n4);
+              cp_async_4(dst + 8, src + 8, n4);
+            }
+          }
+        } else {
+          cp_async_8(base + i * kStageBytes + lane * 8, cp[i] + off_code, n8);
+        }
+        cp_async_4(base + i * kStageBytes + kCA + lane * 4, sp[i] + off_meta, n_scale);
+        if (!kSym) cp_async_4(base + i * kStageBytes + kCA + 128 + lane * 4, zp[i] + off_meta, n4);
       }
     }
     cp_async_commit();
@@ -197,17 +219,17 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
       bool fast = true;
 #pragma unroll
       for (int i = 0; i < K; ++i) {
-        code[i] = *reinterpret_cast<const uint2*>(buf + i * kStageBytes + lane * 8);
+        code[i] = F == kAsymBits ? make_uint2(0u, 0u) : *reinterpret_cast<const uint2*>(buf + i * kStageBytes + lane * 8);
         if (kF16) {
-          const uint32_t word = *reinterpret_cast<const uint32_t*>(buf + i * kStageBytes + 256 + lane * 4);
+          const uint32_t word = *reinterpret_cast<const uint32_t*>(buf + i * kStageBytes + kCA + lane * 4);
           const uint64_t gi = static_cast<uint64_t>(r * cols + col) >> p.log2g;
           const uint32_t h = (gi & 1) ? (word >> 16) : (word & 0xffffu);
           s[i] = __half2float(__ushort_as_half(static_cast<unsigned short>(h)));
         } else {
-          s[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + 256 + lane * 4);
+          s[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + kCA + lane * 4);
           fast = fast && prescale_ok(s[i]);
         }
-        z[i] = kSym ? 0.0f : *reinterpret_cast<const float*>(buf + i * kStageBytes + 384 + lane * 4);
+        z[i] = kSym ? 0.0f : *reinterpret_cast<const float*>(buf + i * kStageBytes + kCA + 128 + lane * 4);
       }
       if (col >= cols) continue;  // beyond the row's last column: nothing to add
       const uint8_t* abase = reinterpret_cast<const uint8_t*>(act) + static_cast<uint32_t>(ch) * (kChunkElems * 4);
@@ -223,7 +245,22 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
           }
         }
       };
-      if (fast) {
+      if constexpr (F == kAsymBits) {
+        // per-stage widths: the reconstruction's width-generic stage sum
+        f32x2 w[16];
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+          const uint4 w4 = *reinterpret_cast<const uint4*>(buf + i * kStageBytes + lane * 16);
+          switch (p.bits[i]) {
+            case 1: dequant_bits<1>(w4, s[i], z[i], i == 0, w); break;
+            case 3: dequant_bits<3>(w4, s[i], z[i], i == 0, w); break;
+            case 4: dequant_bits<4>(w4, s[i], z[i], i == 0, w); break;
+            default: dequant_bits<2>(w4, s[i], z[i], i == 0, w); break;
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < 8; ++q) dot(q, w[2 * q], w[2 * q + 1]);
+      } else if (fast) {
         // t = 2^23 + Q*4^j exactly; s*4^-j exact (see reconstruct_kernel.cuh)
         f32x2 S01[K], S23[K], C01[K], C23[K], Z[K];
 #pragma unroll
@@ -305,9 +342,9 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
 inline int64_t act_floats_of(int64_t max_cols) {
   return ((max_cols + kChunkElems - 1) / kChunkElems) * kChunkElems;
 }
-template <int K>
+template <int F, int K>
 int tokens_per_launch(int64_t max_cols) {
-  const int64_t t = (kMaxSmem - ring_bytes<K>()) / (act_floats_of(max_cols) * 4);
+  const int64_t t = (kMaxSmem - ring_bytes<F, K>()) / (act_floats_of(max_cols) * 4);
   return static_cast<int>(t < kMaxGemvBatch ? t : kMaxGemvBatch);
 }
 
@@ -315,7 +352,7 @@ template <int F, int K, int B>
 cudaError_t launch_fkb(const GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
   static int attr_bytes = 0;  // largest dynamic shared memory enabled so far (same for every device)
   const int act_floats = static_cast<int>(act_floats_of(max_cols));
-  const int smem = ring_bytes<K>() + nb * act_floats * 4;
+  const int smem = ring_bytes<F, K>() + nb * act_floats * 4;
   if (smem > attr_bytes) {
     cudaError_t e = cudaFuncSetAttribute(gemv_kernel<F, K, B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;

@@ -88,6 +88,7 @@ struct GemvBatch {
   int count;
   int log2g;                       // group = 1 << log2g
   int grid;                        // CTAs of the launch
+  int bits[kMaxStages];            // per-stage code widths (kAsymBits)
   int64_t total_blocks;
   int64_t cta_begin[kMaxGemvGrid + 1];  // CTA c takes blocks [cta_begin[c], cta_begin[c+1])
   GemvItem item[kMaxBatch];
@@ -207,12 +208,13 @@ cudaError_t reconstruct_launch_asym_bits(int group, int k, bool all_prefixes, co
 
 // Activation rows one launch can hold in shared memory for matrices of up to
 // max_cols columns with k stages (0: too wide).
-int gemv_rows_per_launch(int k, int64_t max_cols);
+int gemv_rows_per_launch(Format fmt, int k, int64_t max_cols);
 // nb activation rows (1..kMaxGemvBatch, within gemv_rows_per_launch); one
 // translation unit per format.
 cudaError_t gemv_launch_asym_f32(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
 cudaError_t gemv_launch_sym_f32(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
 cudaError_t gemv_launch_sym_f16(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
+cudaError_t gemv_launch_asym_bits(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
 
 inline cudaError_t gemv_launch(Format fmt, int k, int nb, int64_t max_cols, const GemvBatch& p,
                                cudaStream_t stream, int sms) {
@@ -220,7 +222,7 @@ inline cudaError_t gemv_launch(Format fmt, int k, int nb, int64_t max_cols, cons
     case kAsymF32: return gemv_launch_asym_f32(k, nb, max_cols, p, stream, sms);
     case kSymF32: return gemv_launch_sym_f32(k, nb, max_cols, p, stream, sms);
     case kSymF16: return gemv_launch_sym_f16(k, nb, max_cols, p, stream, sms);
-    case kAsymBits: break;
+    case kAsymBits: return gemv_launch_asym_bits(k, nb, max_cols, p, stream, sms);
   }
   return cudaErrorInvalidValue;
 }

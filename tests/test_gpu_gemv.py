@@ -143,6 +143,35 @@ def test_qwen3_8b_layer_sampled_rows():
             _check(p, A, Y, k, rows_idx=idx, where=f"{sp.name} k{k}")
 
 
+@pytest.mark.parametrize("group", [32, 128])
+@pytest.mark.parametrize("bits", [(1, 3), (3, 1), (4, 2, 1), (2, 4), (1, 1, 1, 1), (4, 4)],
+                         ids=lambda b: "+".join(map(str, b)))
+@pytest.mark.parametrize("batch", [1, 5])
+def test_widths(batch, bits, group):
+    """Packages with per-stage widths: every prefix against the oracle's
+    decode form (binary32 prefix weights) within the kernel's summation
+    bound (the same tree as the 2-bit formats)."""
+    rows, cols = 45, 9 * group
+    W = workloads.generate(rows, cols, 95 + sum(bits), "t3_rowout", "cuda")
+    (pkg,) = binding.rrq_quantize_ex([W], group, len(bits), binding.GRID_ASYM, binding.SCALE_F32, bits=bits)
+    A = _acts(batch, cols, seed=batch + group)
+    torch.cuda.synchronize()
+    codes = [c.cpu().numpy() for c in pkg.codes]
+    scales = [x.cpu().numpy() for x in pkg.scales]
+    zeros = [x.cpu().numpy() for x in pkg.zeros]
+    Ab = bf16_bits(A)
+    Af = np.abs((Ab.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+    for k in range(1, len(bits) + 1):
+        (Y,) = binding.rrq_gemv([pkg], [A], k)
+        want = oracle.product_bits(codes, scales, zeros, rows, cols, group, k, bits, Ab, False)
+        rec = oracle.reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits)
+        recf = np.abs((rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+        d = cols // 64 + 8
+        tol = d * 2.0 ** -24 * (Af @ recf.T) * (1 + 2.0 ** -8) + 1e-30
+        err = np.abs(Y.cpu().numpy().astype(np.float64) - want)
+        assert not np.any(err > tol), f"{bits} g{group} B{batch} k{k}: {int((err > tol).sum())} outputs beyond the bound"
+
+
 def test_errors():
     W = workloads.generate(8, 256, 1, "normal", "cuda")
     pkg = binding.rrq_quantize(W, 128, 2)
