@@ -122,6 +122,10 @@ class Oracle:
             ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p), ctypes.c_int64, ctypes.c_int64,
             ctypes.c_int, ctypes.c_int, _i32p, _u16p, ctypes.c_int64, ctypes.c_int, ctypes.POINTER(ctypes.c_double)]
         lib.rrq_oracle_product_bits.restype = ctypes.c_int
+        lib.rrq_oracle_quantize_from_base_bits.argtypes = [
+            _u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int, ctypes.c_int, _i32p,
+            ctypes.POINTER(_u8p), ctypes.POINTER(_f32p), ctypes.POINTER(_f32p)]
+        lib.rrq_oracle_quantize_from_base_bits.restype = ctypes.c_int
         lib.rrq_oracle_group_pmr.argtypes = [_u16p, ctypes.c_int64, ctypes.c_int64, ctypes.c_int,
                                              ctypes.POINTER(ctypes.c_double)]
         lib.rrq_oracle_group_pmr.restype = ctypes.c_int
@@ -334,6 +338,29 @@ class Oracle:
             raise ValueError("oracle rejected the matrix")
         return codes, scales, zeros
 
+    def quantize_from_base_bits(self, W_bits, base, group, bits):
+        """Algorithm 1 with a base checkpoint and per-stage widths: base =
+        (codes0, scales0, zeros0) at width bits[0]; returns the package
+        (codes, scales, zeros) with stage 0 the given base."""
+        W_bits = np.ascontiguousarray(W_bits, dtype=np.uint16)
+        rows, cols = W_bits.shape
+        n, S = rows * cols, len(bits)
+        codes = [np.ascontiguousarray(base[0], dtype=np.uint8).copy()] + \
+            [np.zeros((n * b + 7) // 8, np.uint8) for b in bits[1:]]
+        scales = [np.ascontiguousarray(base[1], dtype=np.float32).copy()] + [np.zeros(n // group, np.float32)
+                                                                              for _ in bits[1:]]
+        zeros = [np.ascontiguousarray(base[2], dtype=np.float32).copy()] + [np.zeros(n // group, np.float32)
+                                                                             for _ in bits[1:]]
+        cp = (_u8p * S)(*[c.ctypes.data_as(_u8p) for c in codes])
+        sp = (_f32p * S)(*[a.ctypes.data_as(_f32p) for a in scales])
+        zp = (_f32p * S)(*[a.ctypes.data_as(_f32p) for a in zeros])
+        b = (ctypes.c_int * S)(*bits)
+        rc = self.lib.rrq_oracle_quantize_from_base_bits(W_bits.ctypes.data_as(_u16p), rows, cols, group, S, b,
+                                                         cp, sp, zp)
+        if rc != 0:
+            raise ValueError("oracle rejected the base-checkpoint build with widths")
+        return codes, scales, zeros
+
     def product_bits(self, codes, scales, zeros, rows, cols, group, k, bits, A_bits, bf16_weights: bool):
         """Y [tokens, rows] float64: activations (bf16 bit patterns) times the
         prefix-k weights of a package with per-stage widths, binary32 (decode
@@ -442,6 +469,10 @@ def quantize_bits(W_bits, group, bits):
 
 def reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits):
     return load().reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits)
+
+
+def quantize_from_base_bits(W_bits, base, group, bits):
+    return load().quantize_from_base_bits(W_bits, base, group, bits)
 
 
 def product_bits(codes, scales, zeros, rows, cols, group, k, bits, A_bits, bf16_weights: bool):

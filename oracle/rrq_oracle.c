@@ -644,3 +644,49 @@ int rrq_oracle_product_bits(const uint8_t* const* codes, const float* const* sca
   free(wts);
   return 0;
 }
+
+/* Algorithm 1 with a base checkpoint, per-stage widths (asymmetric grid):
+ * stage 0 is given (bits[0]-bit codes, scale and zero in codes[0],
+ * scales[0], zeros[0]); R_0 = x - fl(zero + fl(Q s)); stages 1..n_stages-1
+ * quantize the running residual at widths bits[1..] exactly as
+ * rrq_oracle_quantize_group_bits does. */
+int rrq_oracle_quantize_from_base_bits(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                                       int n_stages, const int* bits, uint8_t* const* codes,
+                                       float* const* scales, float* const* zeros) {
+  if (!W || !bits || !codes || !scales || !zeros) return -1;
+  if (rows < 1 || cols < 1 || group < 1 || n_stages < 2 || cols % group != 0) return -1;
+  for (int k = 0; k < n_stages; ++k)
+    if (bits[k] < 1 || bits[k] > 4) return -1;
+  const int64_t n = rows * cols;
+  const int64_t n_groups = n / group;
+  const int rest = n_stages - 1;
+  float* r0 = (float*)malloc(sizeof(float) * (size_t)group);
+  uint8_t* Qr = (uint8_t*)malloc((size_t)rest * (size_t)group);
+  float* sr = (float*)malloc(sizeof(float) * (size_t)rest);
+  float* zr = (float*)malloc(sizeof(float) * (size_t)rest);
+  if (!r0 || !Qr || !sr || !zr) {
+    free(r0); free(Qr); free(sr); free(zr);
+    return -1;
+  }
+  for (int k = 1; k < n_stages; ++k) memset(codes[k], 0, (size_t)((n * bits[k] + 7) / 8));
+  for (int64_t gi = 0; gi < n_groups; ++gi) {
+    const int64_t first = gi * group;
+    for (int j = 0; j < group; ++j) {
+      const int q0 = get_bits(codes[0], first + j, bits[0]);
+      const float based = (float)q0 * scales[0][gi];
+      const float base_level_w = zeros[0][gi] + based;
+      r0[j] = rrq_oracle_bf16_to_f32(W[first + j]) - base_level_w; /* R_0 = W - W_0 */
+    }
+    if (rrq_oracle_quantize_group_bits(r0, group, rest, bits + 1, Qr, sr, zr, NULL) != 0) {
+      free(r0); free(Qr); free(sr); free(zr);
+      return -1;
+    }
+    for (int k = 1; k < n_stages; ++k) {
+      for (int j = 0; j < group; ++j) put_bits(codes[k], first + j, bits[k], Qr[(size_t)(k - 1) * group + j]);
+      scales[k][gi] = sr[k - 1];
+      zeros[k][gi] = zr[k - 1];
+    }
+  }
+  free(r0); free(Qr); free(sr); free(zr);
+  return 0;
+}

@@ -106,6 +106,13 @@ int rrq_oracle_product_bits(const uint8_t* const* codes, const float* const* sca
                             const int* bits, const uint16_t* A, int64_t tokens, int bf16_weights,
                             double* Y);
 
+/* Algorithm 1 with a base checkpoint for a package with per-stage widths
+ * (asymmetric grid): stage 0 given in codes[0] (bits[0] bits per weight,
+ * LSB-first), scales[0], zeros[0]; stages 1..n_stages-1 are written. */
+int rrq_oracle_quantize_from_base_bits(const uint16_t* W, int64_t rows, int64_t cols, int group,
+                                       int n_stages, const int* bits, uint8_t* const* codes,
+                                       float* const* scales, float* const* zeros);
+
 /* Asymmetric stages with per-stage widths bits[k] in 1..4 (2^b levels,
  * 2^b - 1 steps).  Group form as rrq_oracle_quantize_group; matrix form packs
  * stage k's codes LSB-first, element c at bits bits[k]*c.., into

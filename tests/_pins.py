@@ -1153,6 +1153,78 @@ def pin_product_bits_forms(orc, seed=97, rows=4, g=64) -> list[str]:
     return fails
 
 
+# ---------------------------------------------------------------------------
+# Algorithm 1 with a base checkpoint and per-stage widths
+# ---------------------------------------------------------------------------
+FB_SPLITS = ([1, 3], [3, 1], [4, 2, 1], [2, 4, 2, 1])
+
+
+def pin_base_bits_branch_equivalence(orc, seed=101, rows=4, g=64) -> list[str]:
+    """Given the RTN base of the width quantizer (pinned above), the base
+    branch rebuilds exactly the same package: Algorithm 1's two branches agree."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 3 * g
+    for bits in FB_SPLITS:
+        xs = np.concatenate(_random_groups(rng, rows * 3, g)).reshape(rows, cols)
+        W = bf16_bits_of_f32(xs)
+        codes, scales, zeros = orc.quantize_bits(W, g, bits)
+        fc, fs, fz = orc.quantize_from_base_bits(W, (codes[0], scales[0], zeros[0]), g, bits)
+        for k in range(len(bits)):
+            if not (np.array_equal(fc[k], codes[k]) and np.array_equal(fs[k].view(np.uint32), scales[k].view(np.uint32))
+                    and np.array_equal(fz[k].view(np.uint32), zeros[k].view(np.uint32))):
+                fails.append(f"{bits} stage {k}: base branch differs from the full build")
+    return fails
+
+
+def pin_base_bits_zero_base(orc, seed=103, rows=3, g=32) -> list[str]:
+    """A base whose every level is +0 (codes 0, zero +0, any scale) leaves
+    R_0 = x, so stages 1.. are the width quantizer of x with widths bits[1:]."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 4 * g
+    n = rows * cols
+    for bits in FB_SPLITS:
+        xs = np.concatenate(_random_groups(rng, rows * 4, g)).reshape(rows, cols)
+        W = bf16_bits_of_f32(xs)
+        base = (np.zeros((n * bits[0] + 7) // 8, np.uint8), rng.uniform(0.1, 2.0, n // g).astype(np.float32),
+                np.zeros(n // g, np.float32))
+        fc, fs, fz = orc.quantize_from_base_bits(W, base, g, bits)
+        rc, rs, rz = orc.quantize_bits(W, g, bits[1:])
+        for k in range(1, len(bits)):
+            if not (np.array_equal(fc[k], rc[k - 1]) and np.array_equal(fs[k].view(np.uint32), rs[k - 1].view(np.uint32))
+                    and np.array_equal(fz[k].view(np.uint32), rz[k - 1].view(np.uint32))):
+                fails.append(f"{bits} stage {k}: zero base does not reduce to the width quantizer of x")
+    return fails
+
+
+def pin_base_bits_random_base(orc, seed=107, rows=3, g=64) -> list[str]:
+    """With an arbitrary base (random codes, scales, zeros), the last prefix of
+    the base branch is within half a last step (plus the binary32 roundings
+    of the stage sums) of the input in every group."""
+    rng = np.random.default_rng(seed)
+    fails = []
+    cols = 2 * g
+    n = rows * cols
+    for bits in FB_SPLITS:
+        xs = np.concatenate(_random_groups(rng, rows * 2, g)).reshape(rows, cols)
+        W = bf16_bits_of_f32(xs)
+        b0 = bits[0]
+        q0 = rng.integers(0, 1 << b0, n)
+        c0 = np.packbits(((q0[:, None] >> np.arange(b0)) & 1).astype(np.uint8).reshape(-1), bitorder="little")
+        base = (c0, rng.uniform(0.0, 0.05, n // g).astype(np.float32), rng.normal(0, 0.05, n // g).astype(np.float32))
+        fc, fs, fz = orc.quantize_from_base_bits(W, base, g, bits)
+        k = len(bits)
+        rec = orc.reconstruct_bits(fc, fs, fz, rows, cols, g, k, bits)
+        recf = (rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64).reshape(-1)
+        x = (W.astype(np.uint32) << 16).view(np.float32).astype(np.float64).reshape(-1)
+        half = np.repeat(fs[k - 1].astype(np.float64), g) / 2
+        bound = half + np.abs(x) * 2.0 ** -8 + 1e-30
+        if np.any(np.abs(recf - x) > bound):
+            fails.append(f"{bits}: last prefix beyond half a last step")
+    return fails
+
+
 ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_brute_force_tiny,
             pin_invariants, pin_exact_grid, pin_prefix_reconstruction, pin_f16_rounding,
             pin_sym_worked_groups, pin_sym_brute_force_exact, pin_sym_invariants,
@@ -1161,7 +1233,8 @@ ALL_PINS = [pin_worked_groups, pin_bf16_rounding, pin_brute_force_exact, pin_bru
             pin_gemv_vs_bf16_reconstruction, pin_bits_worked_and_two_bit_case, pin_bits_brute_force_exact,
             pin_bits_invariants_and_packing, pin_group_pmr, pin_prefill_worked, pin_prefill_one_hot,
             pin_prefill_integer_exact, pin_prefill_vs_binary32_product, pin_product_bits_two_bit_case,
-            pin_product_bits_one_hot, pin_product_bits_integer_exact, pin_product_bits_forms]
+            pin_product_bits_one_hot, pin_product_bits_integer_exact, pin_product_bits_forms,
+            pin_base_bits_branch_equivalence, pin_base_bits_zero_base, pin_base_bits_random_base]
 
 
 def all_failures(orc) -> list[str]:

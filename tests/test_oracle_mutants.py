@@ -92,6 +92,15 @@ MUTANTS = {
                            "wts[j] = (double)running;"),
     "pbits_wrong_output_row": ("Y[(size_t)t * rows + r] = sum;", "Y[(size_t)t * rows + (rows - 1 - r)] = sum;"),
     "pbits_first_stage_zero": ("const float lvl = zeros[st][g] + scaled;", "const float lvl = zeros[0][g] + scaled;"),
+    # Algorithm 1 with a base checkpoint and per-stage widths
+    "fbb_residual_sign": ("r0[j] = rrq_oracle_bf16_to_f32(W[first + j]) - base_level_w;",
+                          "r0[j] = rrq_oracle_bf16_to_f32(W[first + j]) + base_level_w;"),
+    "fbb_base_drops_zero": ("const float base_level_w = zeros[0][gi] + based;", "const float base_level_w = based;"),
+    "fbb_base_read_at_width_two": ("const int q0 = get_bits(codes[0], first + j, bits[0]);",
+                                   "const int q0 = get_bits(codes[0], first + j, 2);"),
+    "fbb_widths_not_shifted": ("rrq_oracle_quantize_group_bits(r0, group, rest, bits + 1, Qr, sr, zr, NULL)",
+                               "rrq_oracle_quantize_group_bits(r0, group, rest, bits, Qr, sr, zr, NULL)"),
+    "fbb_first_scale_everywhere": ("scales[k][gi] = sr[k - 1];", "scales[k][gi] = sr[0];"),
 }
 
 
