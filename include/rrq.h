@@ -266,8 +266,9 @@ rrq_status rrq_quantize_prefixes(const rrq_quantize_prefixes_desc* items, int co
 /* Algorithm 1 with a base checkpoint (Section 3.2: the construction can start
  * from an existing low-bit checkpoint by skipping the base quantization):
  * stage 0 of every item's package is an INPUT in format *fmt -- codes[0],
- * scales[0] and, for RRQ_GRID_ASYM, zeros[0] (a 2-bit checkpoint from any
- * quantizer, stored in this layout) -- dequantized with the grid's level
+ * scales[0] and, for RRQ_GRID_ASYM, zeros[0] (a checkpoint from any
+ * quantizer at the width fmt->bits[0], stored in this layout) -- dequantized
+ * with the grid's level
  * formula (lo + Q*s, or (Q - 2)*s); the running residual starts at
  * R_0 = fl(W - L_0) and stages 1..n_stages-1 are computed from it exactly as
  * rrq_quantize_ex computes them from its own stage 0 (given the base that

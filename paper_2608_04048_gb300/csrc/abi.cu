@@ -242,7 +242,7 @@ rrq_status quantize_batch(const QView* items, int count, const Fmt& f, rrq_strea
   if (!items || count < 1) return RRQ_ERR_INVALID_ARG;
   const bool from_base = mode == kFromBase;
   if (from_base && f.n_stages < 2) return RRQ_ERR_INVALID_ARG;
-  if (mode != kBuild && f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
+  if (mode == kEmit && f.kind == rrq::kAsymBits) return RRQ_ERR_UNSUPPORTED;
   const int n_stages = f.n_stages;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (1 + 4 * n_stages));

@@ -292,8 +292,11 @@ __device__ __forceinline__ void store_words(uint8_t* codes, int64_t e0, const ui
   }
 }
 
-// Asymmetric grid with per-stage widths (values in natural order).
-template <int G>
+// Asymmetric grid with per-stage widths (values in natural order).  kBase:
+// stage 0 is given (Algorithm 1 with a base checkpoint): the lane reads its
+// bits[0] code words and the group's scale and zero, and the stages start
+// from R_0 = fl(x - fl(zero + fl(Q s))).
+template <int G, bool kBase>
 __device__ __forceinline__ void quantize_chunk_bits(const QuantizeBatch& p, const QuantizeItem& it,
                                                     int64_t e0, int lane, uint4 (&raw)[4]) {
   constexpr int L = G / 32;  // lanes per group
@@ -309,12 +312,33 @@ __device__ __forceinline__ void quantize_chunk_bits(const QuantizeBatch& p, cons
 #pragma unroll
     for (int m = 0; m < 4; ++m) v[4 * j + m] = pack2u(w4[m] << 16, w4[m] & 0xffff0000u);
   }
+  if constexpr (kBase) {
+    if (valid) {
+      const int b0 = p.bits[0];
+      const uint32_t* wp = reinterpret_cast<const uint32_t*>(it.codes[0]) + (e0 >> 5) * b0;
+      uint4 w = make_uint4(__ldg(wp), 0u, 0u, 0u);
+      if (b0 > 1) w.y = __ldg(wp + 1);
+      if (b0 > 2) w.z = __ldg(wp + 2);
+      if (b0 > 3) w.w = __ldg(wp + 3);
+      const float s0 = __ldg(static_cast<const float*>(it.scales[0]) + e0 / G);
+      const float z0 = __ldg(it.zeros[0] + e0 / G);
+      f32x2 l0[16];  // the base levels fl(zero + fl(Q s))
+      switch (b0) {
+        case 1: dequant_bits<1>(w, s0, z0, true, l0); break;
+        case 3: dequant_bits<3>(w, s0, z0, true, l0); break;
+        case 4: dequant_bits<4>(w, s0, z0, true, l0); break;
+        default: dequant_bits<2>(w, s0, z0, true, l0); break;
+      }
+#pragma unroll
+      for (int i = 0; i < 16; ++i) v[i] = sub2(v[i], l0[i]);  // R_0 = W - W_0
+    }
+  }
   float lo, hi;
   lane_minmax(v, lo, hi);
   group_minmax<L>(lo, hi);
 
 #pragma unroll 1
-  for (int k = 0; k < p.n_stages; ++k) {
+  for (int k = kBase ? 1 : 0; k < p.n_stages; ++k) {
     if (__any_sync(kFullMask, lo == 0.0f)) {  // a zero minimum is -0 if the group holds a -0
       uint32_t neg = 0;
       if (lo == 0.0f) {
@@ -689,7 +713,7 @@ __device__ __forceinline__ void quantize_chunk(const QuantizeBatch& p, const Qua
   if constexpr (F == kAsymF32)
     quantize_chunk_asym<G, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot, em);
   else if constexpr (F == kAsymBits)
-    quantize_chunk_bits<G>(p, it, e0, lane, raw);
+    quantize_chunk_bits<G, M == kModeBase>(p, it, e0, lane, raw);
   else
     quantize_chunk_sym<G, F == kSymF16, M>(p, it, e0, lane, raw, sel_lo, sel_hi, bw, ld_lo, ld_hi, rot, em);
 }
@@ -754,7 +778,8 @@ quantize_kernel(const __grid_constant__ QuantizeBatch p) {
   // base words of this warp's chunks, loaded one chunk ahead
   int m_base = 0;
   auto base_of = [&](int64_t chunk) -> BaseWords {
-    if (!kBase || chunk >= p.total_chunks) return BaseWords{make_uint2(0u, 0u), 0.0f, 0.0f};
+    // (per-stage widths read their base inside the chunk routine)
+    if (!kBase || F == kAsymBits || chunk >= p.total_chunks) return BaseWords{make_uint2(0u, 0u), 0.0f, 0.0f};
     const QuantizeItem& it = item_of(chunk, m_base);
     return load_base<G, F>(it, (chunk - it.chunk_begin) * kChunkElems + static_cast<int64_t>(lane) * kLaneElems);
   };
@@ -850,7 +875,7 @@ cudaError_t prepare_all() {
   if ((e = prepare_f<kAsymF32, M>())) return e;
   if ((e = prepare_f<kSymF32, M>())) return e;
   if ((e = prepare_f<kSymF16, M>())) return e;
-  if constexpr (M == kModeBuild) return prepare_f<kAsymBits, kModeBuild>();
+  if constexpr (M != kModeEmit) return prepare_f<kAsymBits, M>();
   return cudaSuccess;
 }
 
@@ -861,7 +886,7 @@ cudaError_t launch_all(int group, Format fmt, const QuantizeBatch& p, cudaStream
     case kSymF32: return launch_f<kSymF32, M>(group, p, stream, sms);
     case kSymF16: return launch_f<kSymF16, M>(group, p, stream, sms);
     case kAsymBits:
-      if constexpr (M == kModeBuild) return launch_f<kAsymBits, kModeBuild>(group, p, stream, sms);
+      if constexpr (M != kModeEmit) return launch_f<kAsymBits, M>(group, p, stream, sms);
       break;
   }
   return cudaErrorInvalidValue;

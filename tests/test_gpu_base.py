@@ -157,6 +157,54 @@ def test_batch_across_launches():
         _check(W, p, f"batch item {i}")
 
 
+BIT_SPLITS = [(1, 3), (3, 1), (4, 2, 1), (2, 4, 2, 1)]
+
+
+def _check_bits(W, pkg, bits, where):
+    """Stages 1.. of pkg against the oracle's base branch with widths, given
+    the package's own stage 0."""
+    codes, scales, zeros = _host(pkg)
+    rc, rs, rz = oracle.quantize_from_base_bits(bf16_bits(W), (codes[0], scales[0], zeros[0]), pkg.group,
+                                                list(bits))
+    for k in range(1, len(bits)):
+        assert np.array_equal(codes[k], rc[k]), f"{where} stage {k} codes"
+        assert np.array_equal(scales[k].view(np.uint32), rs[k].view(np.uint32)), f"{where} stage {k} scales"
+        assert np.array_equal(zeros[k].view(np.uint32), rz[k].view(np.uint32)), f"{where} stage {k} zeros"
+
+
+@pytest.mark.parametrize("group", GROUPS)
+@pytest.mark.parametrize("bits", BIT_SPLITS, ids=lambda b: "+".join(map(str, b)))
+def test_widths_random_base(bits, group):
+    """Per-stage widths: a random base (random codes, zero, subnormal and
+    huge scales) at width bits[0], stages 1.. bit for bit against the oracle."""
+    rows, cols = 67, 5 * group
+    W = workloads.generate(rows, cols, 40 + group, "t3_rowout", "cuda")
+    pkg = binding.Package.empty(rows, cols, group, len(bits), W.device, binding.GRID_ASYM, binding.SCALE_F32,
+                                bits=bits)
+    _random_base(pkg, seed=group + 10 * len(bits))
+    binding.rrq_quantize_from_base([W], [pkg])
+    _check_bits(W, pkg, bits, where=f"{bits} g{group}")
+    assert binding.rrq_get_device_status() == 0
+
+
+@pytest.mark.parametrize("bits", BIT_SPLITS, ids=lambda b: "+".join(map(str, b)))
+def test_widths_branches_agree(bits):
+    """Given the width package's own RTN stage 0, the base branch rebuilds the
+    same package on the device."""
+    W = workloads.generate(200, 1024, 55, "t3_rowout", "cuda")
+    (full,) = binding.rrq_quantize_ex([W], 128, len(bits), binding.GRID_ASYM, binding.SCALE_F32, bits=bits)
+    pkg = binding.Package.empty(200, 1024, 128, len(bits), W.device, binding.GRID_ASYM, binding.SCALE_F32, bits=bits)
+    pkg.codes[0].copy_(full.codes[0])
+    pkg.scales[0].copy_(full.scales[0])
+    pkg.zeros[0].copy_(full.zeros[0])
+    binding.rrq_quantize_from_base([W], [pkg])
+    torch.cuda.synchronize()
+    for k in range(len(bits)):
+        assert torch.equal(pkg.codes[k], full.codes[k]), f"{bits} stage {k} codes"
+        assert torch.equal(pkg.scales[k].view(torch.int32), full.scales[k].view(torch.int32)), f"{bits} stage {k}"
+        assert torch.equal(pkg.zeros[k].view(torch.int32), full.zeros[k].view(torch.int32)), f"{bits} stage {k}"
+
+
 def test_errors():
     W = workloads.generate(8, 256, 1, "normal", "cuda")
     pkg = binding.Package.empty(8, 256, 128, 1, W.device, binding.GRID_SYM, binding.SCALE_F16)

@@ -132,11 +132,8 @@ def test_unsupported_combinations():
     with pytest.raises(binding.RRQError) as e:   # width 5
         binding.rrq_quantize_ex([W], 128, 2, binding.GRID_ASYM, binding.SCALE_F32, bits=[5, 3])
     assert e.value.status == 1
-    (pkg,) = binding.rrq_quantize_ex([W], 128, 2, binding.GRID_ASYM, binding.SCALE_F32, bits=[1, 3])
-    with pytest.raises(binding.RRQError) as e:
-        binding.rrq_quantize_from_base([W], [pkg])
-    assert e.value.status == 2
-    # (the products take widths: tests/test_gpu_gemv.py, tests/test_gpu_prefill.py)
+    # (the base branch and the products take widths: tests/test_gpu_base.py,
+    # tests/test_gpu_gemv.py, tests/test_gpu_prefill.py)
 
 
 @pytest.mark.parametrize("group", GROUPS)
