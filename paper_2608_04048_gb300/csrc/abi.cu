@@ -398,10 +398,11 @@ rrq_status reconstruct_views(const ReconView* items, int count, const Fmt& f, in
 // ---------------------------------------------------------------------------
 // stage-wise product
 // ---------------------------------------------------------------------------
-rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k, int batch,
-                      rrq_stream_t stream) {
-  if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
-  if (batch < 1 || batch > rrq::kMaxGemvBatch) return RRQ_ERR_INVALID_ARG;
+// Checks shared by the two products: shapes, pointers, alignment, no output
+// overlapping an input or another output (act_rows activation rows per
+// matrix), and every pointer on the current device; returns the device state.
+rrq_status check_product_items(const rrq_gemv_desc* items, int count, const Fmt& f, int k, uint64_t act_rows,
+                               DeviceState** st_out) {
   const int group = f.group;
   std::vector<Range> ranges;
   ranges.reserve(static_cast<size_t>(count) * (2 + 3 * k));
@@ -415,8 +416,8 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
       if (!aligned(it.codes[j], 16) || !aligned(it.scales[j], 16) || (!f.sym() && !aligned(it.zeros[j], 16)))
         return RRQ_ERR_MISALIGNED;
     const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
-    ranges.push_back(range_of(it.A_bf16, 2 * static_cast<uint64_t>(batch) * it.cols, false));
-    ranges.push_back(range_of(it.Y, 4 * static_cast<uint64_t>(batch) * it.rows, true));
+    ranges.push_back(range_of(it.A_bf16, 2 * act_rows * it.cols, false));
+    ranges.push_back(range_of(it.Y, 4 * act_rows * it.rows, true));
     for (int j = 0; j < k; ++j) {
       ranges.push_back(range_of(it.codes[j], f.code_bytes(n, j), false));
       ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
@@ -436,6 +437,18 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
           (!f.sym() && !on_device(it.zeros[j], dev)))
         return RRQ_ERR_INVALID_ARG;
   }
+
+  *st_out = st;
+  return RRQ_OK;
+}
+
+rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k, int batch,
+                      rrq_stream_t stream) {
+  if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;
+  if (batch < 1 || batch > rrq::kMaxGemvBatch) return RRQ_ERR_INVALID_ARG;
+  const int group = f.group;
+  DeviceState* st = nullptr;
+  if (rrq_status rc = check_product_items(items, count, f, k, static_cast<uint64_t>(batch), &st)) return rc;
 
   int log2g = 0;
   while ((1 << log2g) < group) ++log2g;
@@ -556,40 +569,10 @@ rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, in
   if (tokens < 1 || tokens > RRQ_MAX_PREFILL_TOKENS) return RRQ_ERR_INVALID_ARG;
   const bool widths = f.kind == rrq::kAsymBits;
   const int group = f.group;
-  std::vector<Range> ranges;
-  ranges.reserve(static_cast<size_t>(count) * (2 + 3 * k));
-  for (int i = 0; i < count; ++i) {
-    const rrq_gemv_desc& it = items[i];
-    if (!shape_ok(it.rows, it.cols) || it.cols % group != 0 || !it.A_bf16 || !it.Y) return RRQ_ERR_INVALID_ARG;
-    if (it.cols > (int64_t{1} << 31) - rrq::kPrefillBK) return RRQ_ERR_INVALID_ARG;
-    for (int j = 0; j < k; ++j)
-      if (!it.codes[j] || !it.scales[j] || (!f.sym() && !it.zeros[j])) return RRQ_ERR_INVALID_ARG;
-    if (!aligned(it.A_bf16, 16) || !aligned(it.Y, 16)) return RRQ_ERR_MISALIGNED;
-    for (int j = 0; j < k; ++j)
-      if (!aligned(it.codes[j], 16) || !aligned(it.scales[j], 16) || (!f.sym() && !aligned(it.zeros[j], 16)))
-        return RRQ_ERR_MISALIGNED;
-    const uint64_t n = static_cast<uint64_t>(it.rows * it.cols);
-    ranges.push_back(range_of(it.A_bf16, 2 * static_cast<uint64_t>(tokens) * it.cols, false));
-    ranges.push_back(range_of(it.Y, 4 * static_cast<uint64_t>(tokens) * it.rows, true));
-    for (int j = 0; j < k; ++j) {
-      ranges.push_back(range_of(it.codes[j], f.code_bytes(n, j), false));
-      ranges.push_back(range_of(it.scales[j], f.scale_bytes() * (n / group), false));
-      if (!f.sym()) ranges.push_back(range_of(it.zeros[j], 4 * (n / group), false));
-    }
-  }
-  if (!ranges_disjoint(ranges)) return RRQ_ERR_INVALID_ARG;
-
-  int dev = 0;
+  for (int i = 0; i < count; ++i)
+    if (items[i].cols > (int64_t{1} << 31) - rrq::kPrefillBK) return RRQ_ERR_INVALID_ARG;  // TMA coordinates
   DeviceState* st = nullptr;
-  if (rrq_status rc = current_device(&dev, &st)) return rc;
-  for (int i = 0; i < count; ++i) {
-    const rrq_gemv_desc& it = items[i];
-    if (!on_device(it.A_bf16, dev) || !on_device(it.Y, dev)) return RRQ_ERR_INVALID_ARG;
-    for (int j = 0; j < k; ++j)
-      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) ||
-          (!f.sym() && !on_device(it.zeros[j], dev)))
-        return RRQ_ERR_INVALID_ARG;
-  }
+  if (rrq_status rc = check_product_items(items, count, f, k, static_cast<uint64_t>(tokens), &st)) return rc;
 
   int log2g = 0;
   while ((1 << log2g) < group) ++log2g;
