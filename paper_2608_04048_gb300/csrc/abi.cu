@@ -476,27 +476,6 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
       max_cols = std::max(max_cols, it.cols);
     }
     p.total_blocks = blocks;
-    // one contiguous range of blocks per CTA, with equal shares of rows x cols
-    p.grid = static_cast<int>(std::min<int64_t>({blocks, st->sms, rrq::kMaxGemvGrid}));
-    {
-      int64_t total = 0;
-      for (int i = 0; i < m; ++i) total += items[base + i].rows * items[base + i].cols;
-      int c = 0;
-      int64_t done = 0, blk = 0;
-      p.cta_begin[0] = 0;
-      for (int i = 0; i < m && c < p.grid; ++i) {
-        const rrq_gemv_desc& it = items[base + i];
-        const int64_t nblk = (it.rows + rrq::kGemvRows - 1) / rrq::kGemvRows;
-        for (int64_t b = 0; b < nblk; ++b, ++blk) {
-          const int64_t r = std::min<int64_t>(rrq::kGemvRows, it.rows - b * rrq::kGemvRows);
-          done += r * it.cols;
-          // close CTA c's range once its share is reached
-          while (c + 1 < p.grid && done * p.grid >= (c + 1) * total) p.cta_begin[++c] = blk + 1;
-        }
-      }
-      while (c < p.grid) p.cta_begin[++c] = blocks;
-      p.cta_begin[p.grid] = blocks;
-    }
     // activation rows per launch: as many as shared memory holds
     const int per = rrq::gemv_rows_per_launch(f.kind, k, max_cols);
     if (per < 1) return RRQ_ERR_UNSUPPORTED;

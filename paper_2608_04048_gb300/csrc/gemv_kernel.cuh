@@ -5,33 +5,41 @@
 // with the stages summed per weight first (one multiply per weight and token
 // instead of one per stage), reading only the package -- k x (2 + 64/g) bits
 // per weight -- and never a bf16 copy of the weights.  Aimed at decoding
-// (1 to 8 activation rows), where the product is bound by weight movement.
+// (1 to 8 activation rows), where the product moves little data per weight
+// and its cost is the instructions that form each weight.
 //
 // Work decomposition: the rows of every matrix are cut into blocks of 16
 // rows; the blocks of all matrices of a launch form one sequence, cut into
-// one contiguous range per CTA of a persistent grid with equal shares of
-// rows x columns (so a CTA meets few matrices), each CTA taking its blocks in
-// order with 16 warps, one row of the block per warp.  A CTA keeps the activations of its current matrix in shared memory
-// as binary32 (converted once when the matrix changes, in a swizzled layout:
-// 16-byte piece P of a row stored at P ^ ((P >> 3) & 7), so that the eight
-// lanes of a quarter warp reading their piece q hit eight different bank
-// groups).  A warp walks its row in chunks of 1024 columns, lane l owning
-// columns 32l..32l+31; each lane copies its code words, scales and zeros of
-// every stage asynchronously (cp.async) into a per-warp ring of shared-memory
-// buffers, two chunks ahead across rows and blocks.  Per group of four
-// columns the lane forms the binary32 prefix weights exactly as the
-// reconstruction does and multiplies them with one 16-byte shared-memory read
-// of activations per activation row (packed fp32 fma's).  At the end of a row
+// one contiguous range per CTA of a persistent grid (as many CTAs as fit on
+// the multiprocessors) with equal shares of rows x columns, so that a CTA
+// meets few matrices.  The CTA's 16 warps take one row of each block each.
+// A warp walks its row in windows of 2048 columns, lane l owning the 64
+// columns 64l..64l+63 of the window (1024 and 32 when the group is 32, so that
+// a lane's columns share one group; with a larger group the row length is a
+// multiple of 64, so a lane's 64 columns are all in the row or all past its
+// end): per stage one 16-byte load of codes (8 bytes for 32 columns) and one
+// scale and zero, all loaded into registers one window ahead, across rows,
+// blocks and matrices.
+//
+// The CTA keeps the activations of its current matrix in shared memory as
+// binary32, converted once per matrix, stored transposed within each window:
+// the 16-byte piece j (columns 4j..4j+3 of a lane's columns) of lane l sits at
+// (window, j, l), so the 32 lanes reading their piece j touch 512 contiguous
+// bytes (no bank conflict) at an offset that is a constant per j.  Per four
+// columns a lane forms the binary32 prefix weights exactly as the
+// reconstruction does and multiplies them with one 16-byte read of
+// activations per activation row (packed fp32 fma's).  At the end of a row
 // the warp reduces by butterfly shuffles and lane 0 stores Y: a fixed order,
 // so results are deterministic, with no atomics and no workspace.
 //
 // Accuracy: every product W~ * a is exact inside its fma and each partial sum
-// is rounded once, so |Y - exact| <= gamma_n * sum_c |W~ a| (n = cols) for any
-// summation order; the parity tests use the tighter count of this kernel's
-// summation tree.
+// is rounded once.  A lane's two accumulators (even and odd columns of each
+// pair) each take at most 32 products per 2048 columns of the row (rounded
+// up), then the pair and 5 butterfly steps, so |Y - exact| <=
+// (32 ceil(cols/2048) + 6) * 2^-24 * sum_c |W~ a| to first order.
 //
-// This header holds the kernel template; gemv_asym_f32.cu, gemv_sym_f32.cu
-// and gemv_sym_f16.cu each instantiate one package format.
+// This header holds the kernel template; gemv_asym_f32.cu, gemv_sym_f32.cu,
+// gemv_sym_f16.cu and gemv_asym_bits.cu each instantiate one package format.
 #pragma once
 
 #include <cuda_fp16.h>
@@ -45,286 +53,290 @@ constexpr int kWarps = 16;
 constexpr int kThreads = kWarps * 32;
 constexpr int kRows = kGemvRows;       // rows per block (one per warp)
 static_assert(kRows == kWarps, "one row of a block per warp");
-// ring depth (chunks per warp in shared memory, two ahead of use)
-template <int K>
-__host__ __device__ constexpr int ring_depth() { return 3; }
-// one stage of one chunk: codes (256 B at 2 bits, up to 512 B with per-stage
-// widths: 16 B per lane) | scales 128 B | zeros 128 B
-template <int F>
-__host__ __device__ constexpr int code_area() { return F == kAsymBits ? 512 : 256; }
-template <int F>
-__host__ __device__ constexpr int stage_bytes() { return code_area<F>() + 256; }
+constexpr int kWinCols = 2048;         // columns of a warp's window (1024 when the group is 32)
 constexpr int kMaxSmem = 227 * 1024;
 constexpr float kTwo23 = 8388608.0f;
 
+// Read-once package loads: no L1 allocation, read-only path.
+__device__ __forceinline__ uint4 ld_nc16(const void* p) {
+  uint4 v;
+  asm("ld.global.nc.L1::no_allocate.v4.u32 {%0,%1,%2,%3}, [%4];"
+      : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint2 ld_nc8(const void* p) {
+  uint2 v;
+  asm("ld.global.nc.L1::no_allocate.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_nc4(const void* p) {
+  uint32_t v;
+  asm("ld.global.nc.L1::no_allocate.u32 %0, [%1];" : "=r"(v) : "l"(p));
+  return v;
+}
+__device__ __forceinline__ uint32_t ld_nc2(const void* p) {
+  unsigned short v;
+  asm("ld.global.nc.L1::no_allocate.u16 %0, [%1];" : "=h"(v) : "l"(p));
+  return v;
+}
+
+// A lane's package data of one window: per stage the codes of its 64 (or 32)
+// columns (16 bytes at 2 bits; up to 32 bytes with per-stage widths), and the
+// raw scale and zero of their group.
 template <int F, int K>
-__host__ __device__ constexpr int ring_bytes() { return kWarps * ring_depth<K>() * K * stage_bytes<F>(); }
-
-// swizzled position of 16-byte activation piece P of a row
-__device__ __forceinline__ uint32_t act_piece(uint32_t P) { return P ^ ((P >> 3) & 7u); }
-
-// Where a warp is in its stream: block, chunk of the row, and the row's start.
-struct Cursor {
-  int64_t blk;   // global block index (>= total_blocks: past the end)
-  int64_t e;     // element offset of the chunk's first column within its matrix
-  int ch, nch;
-  int m;
+struct Window {
+  static constexpr int kVecs = F == kAsymBits ? 2 : 1;
+  uint4 code[K][kVecs];
+  uint32_t s[K];  // binary32 bits, or binary16 bits in the low half
+  float z[K];
 };
 
+// Where a warp is in its sequence of windows.
+struct Pos {
+  int64_t blk;   // global block index (>= the CTA's end: no window)
+  int64_t rowe;  // element offset of the row's first column within its matrix
+  int m;         // matrix (item) index
+  int ch, nch;   // window of the row, windows per row
+};
+
+// Named barrier 1 over the whole CTA, in its non-aligned form: warps reach
+// it from different places of the loop (each warp passes the same matrix
+// changes in the same order, so the arrivals always pair up).
+__device__ __forceinline__ void cta_barrier() {
+  asm volatile("barrier.sync 1, %0;" ::"n"(kThreads) : "memory");
+}
+
 template <int F, int K, int B>
-__global__ void __launch_bounds__(kThreads, 1)
+__global__ void __launch_bounds__(kThreads, (K == 1 && B <= 2 && F != kAsymBits) ? 2 : 1)
 gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
-  constexpr int kStageBytes = stage_bytes<F>();
-  constexpr int kCA = code_area<F>();  // scales at kCA, zeros at kCA + 128
-  constexpr int kBuf = K * kStageBytes;
-  constexpr int kRing = ring_depth<K>();
-  extern __shared__ __align__(128) uint8_t smem[];
-  float* act = reinterpret_cast<float*>(smem + ring_bytes<F, K>());  // [B][act_floats], swizzled pieces
+  constexpr bool kBits = F == kAsymBits;
+  extern __shared__ __align__(16) float4 act4[];  // [B][act_floats / 4] pieces, transposed per window
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
-  uint8_t* ring = smem + warp * kRing * kBuf;
-  const uint32_t ring_s = smem_u32(ring);
-  const int lane_col = lane * kLaneElems;
-  // byte offsets of this lane's eight activation pieces within a chunk
-  uint32_t poff[8];
-#pragma unroll
-  for (int q = 0; q < 8; ++q) poff[q] = act_piece(static_cast<uint32_t>(lane * 8 + q)) * 16u;
-
-  auto item_of = [&](int64_t blk, int& m) -> const GemvItem& {
-    while (m + 1 < p.count && blk >= p.item[m + 1].blk_begin) ++m;
-    return p.item[m];
-  };
+  const int64_t blk_begin = p.cta_begin[blockIdx.x];
   const int64_t blk_end = p.cta_begin[blockIdx.x + 1];
-  // position the cursor on the first valid row of this warp at or after blk
-  auto start_block = [&](Cursor& c, int64_t blk) {
+  if (blk_begin >= blk_end) return;  // the whole CTA: no barrier is reached
+  const int log2g = p.log2g;
+  const int lc = log2g == 5 ? 32 : 64;  // columns of a lane in a window: within one group
+  const int wcols = 32 * lc;            // columns of a window
+  const int lsh = log2g == 5 ? 3 : 4;   // log2 of a lane's 16-byte pieces per window
+  const int wsh = lsh + 7;              // log2 of wcols
+  const int act_pieces = act_floats / 4;
+
+  auto item_index = [&](int64_t blk, int m) {
+    while (m + 1 < p.count && blk >= p.item[m + 1].blk_begin) ++m;
+    return m;
+  };
+  // activations of matrix m, bf16 -> binary32 (exact), piece P of window w,
+  // lane l, piece j of the lane stored at (w * lc/4 + j) * 32 + l
+  auto load_acts = [&](int m) {
+    const GemvItem& it = p.item[m];
+    const int pieces = static_cast<int>(it.cols / 4);
+    for (int b = 0; b < nb; ++b) {
+      const uint2* src = reinterpret_cast<const uint2*>(it.A + b * it.cols);
+      float4* dst = act4 + b * act_pieces;
+      for (int P = threadIdx.x; P < pieces; P += kThreads) {
+        const uint2 a = __ldg(src + P);
+        dst[(((P >> (lsh + 5)) << lsh) + (P & ((1 << lsh) - 1))) * 32 + ((P >> lsh) & 31)] =
+            make_float4(__uint_as_float(a.x << 16), __uint_as_float(a.x & 0xffff0000u),
+                        __uint_as_float(a.y << 16), __uint_as_float(a.y & 0xffff0000u));
+      }
+    }
+  };
+  const int m_first = item_index(blk_begin, 0);
+  const int m_last = item_index(blk_end - 1, m_first);
+  load_acts(m_first);
+  cta_barrier();
+  int m_act = m_first;
+  // every warp passes every matrix change of the CTA's range, in order:
+  // all warps done with the old activations, load, all loaded
+  auto switch_to = [&](int m) {
+    while (m_act < m) {
+      cta_barrier();
+      load_acts(++m_act);
+      cta_barrier();
+    }
+  };
+
+  // the first row of this warp at or after block blk
+  auto seek = [&](Pos& c, int64_t blk) {
     for (; blk < blk_end; ++blk) {
-      const GemvItem& it = item_of(blk, c.m);
+      c.m = item_index(blk, c.m);
+      const GemvItem& it = p.item[c.m];
       const int64_t r = (blk - it.blk_begin) * kRows + warp;
       if (r < it.rows) {
         c.blk = blk;
+        c.rowe = r * it.cols;
         c.ch = 0;
-        c.e = r * it.cols;
-        c.nch = static_cast<int>((it.cols + kChunkElems - 1) / kChunkElems);
+        c.nch = static_cast<int>((it.cols + wcols - 1) >> wsh);
         return;
       }
     }
     c.blk = blk_end;
   };
-  auto advance = [&](Cursor& c) {
+
+  // this lane's package data of window c, into registers
+  auto load = [&](const Pos& c, Window<F, K>& w) {
     if (c.blk >= blk_end) return;
-    if (++c.ch < c.nch) c.e += kChunkElems;
-    else start_block(c, c.blk + 1);
-  };
-  auto issue = [&](const Cursor& c, int buf) {
-    if (c.blk < blk_end) {
-      // every field read before the first copy (the copies clobber memory)
-      const GemvItem& it = p.item[c.m];
-      const char* cp[K];
-      const char* sp[K];
-      const char* zp[K];
+    const GemvItem& it = p.item[c.m];
+    const int64_t col = static_cast<int64_t>(c.ch) * wcols + lane * lc;
+    if (col >= it.cols) return;  // beyond the row: never used
+    const uint64_t e = static_cast<uint64_t>(c.rowe + col);
+    const uint64_t g0 = e >> log2g;
 #pragma unroll
-      for (int i = 0; i < K; ++i) {
-        cp[i] = reinterpret_cast<const char*>(it.codes[i]);
-        sp[i] = reinterpret_cast<const char*>(it.scales[i]);
-        zp[i] = kSym ? nullptr : reinterpret_cast<const char*>(it.zeros[i]);
-      }
-      const int64_t cols = it.cols;
-      const int col = c.ch * kChunkElems + lane_col;
-      const bool valid = col < cols;
-      const uint64_t e = static_cast<uint64_t>(c.e) + lane_col;
-      const uint64_t off_code = valid ? e >> 2 : 0;
-      const uint64_t gi = e >> p.log2g;
-      uint64_t off_meta = valid ? gi * 4 : 0;
-      uint32_t n_scale = valid ? 4u : 0u;
-      if (kF16) {  // the aligned 4-byte word holding this group's 2-byte scale
-        off_meta = valid ? (gi * 2) & ~uint64_t{3} : 0;
-        const uint64_t left = static_cast<uint64_t>((it.rows * cols) >> p.log2g) * 2 - off_meta;
-        n_scale = valid ? (left < 4 ? 2u : 4u) : 0u;
-      }
-      const uint32_t n8 = valid ? 8u : 0u, n4 = valid ? 4u : 0u;
-      const uint32_t base = ring_s + buf * kBuf;
+    for (int i = 0; i < K; ++i) {
+      if constexpr (kBits) {  // 8b bytes for 64 codes of width b, 4-byte aligned
+        const int b = p.bits[i];
+        const int words = lc == 64 ? 2 * b : b;
+        const uint32_t* src = reinterpret_cast<const uint32_t*>(it.codes[i]) + (e >> 5) * b;
+        uint32_t wd[8];
 #pragma unroll
-      for (int i = 0; i < K; ++i) {
-        if constexpr (F == kAsymBits) {  // 4b bytes of b-bit codes for the lane's 32 weights
-          const int b = p.bits[i];
-          const char* src = cp[i] + (valid ? (e >> 5) * 4 * static_cast<uint64_t>(b) : 0);
-          const uint32_t dst = base + i * kStageBytes + lane * 16;
-          if (b == 4) cp_async_16(dst, src, valid ? 16u : 0u);
-          else if (b == 2) cp_async_8(dst, src, n8);
-          else {
-            cp_async_4(dst, src, n4);
-            if (b == 3) {
-              cp_async_4(dst + 4, src + 4, n4);
-              cp_async_4(dst + 8, src + 8, n4);
-            }
-          }
+        for (int t = 0; t < 8; ++t) wd[t] = t < words ? ld_nc4(src + t) : 0u;
+        w.code[i][0] = make_uint4(wd[0], wd[1], wd[2], wd[3]);
+        w.code[i][kBits ? 1 : 0] = make_uint4(wd[4], wd[5], wd[6], wd[7]);
+      } else {
+        const uint8_t* src = it.codes[i] + (e >> 2);
+        if (lc == 64) {
+          w.code[i][0] = ld_nc16(src);
         } else {
-          cp_async_8(base + i * kStageBytes + lane * 8, cp[i] + off_code, n8);
+          const uint2 v = ld_nc8(src);
+          w.code[i][0] = make_uint4(v.x, v.y, 0u, 0u);
         }
-        cp_async_4(base + i * kStageBytes + kCA + lane * 4, sp[i] + off_meta, n_scale);
-        if (!kSym) cp_async_4(base + i * kStageBytes + kCA + 128 + lane * 4, zp[i] + off_meta, n4);
       }
+      if constexpr (kF16) w.s[i] = ld_nc2(static_cast<const uint16_t*>(it.scales[i]) + g0);
+      else w.s[i] = ld_nc4(static_cast<const uint32_t*>(it.scales[i]) + g0);
+      if constexpr (!kSym) w.z[i] = __uint_as_float(ld_nc4(it.zeros[i] + g0));
     }
-    cp_async_commit();
   };
 
-  Cursor ic{0, 0, 0, 0, 0};
-  start_block(ic, p.cta_begin[blockIdx.x]);
+  f32x2 acc[B];
 #pragma unroll
-  for (int j = 0; j < kRing - 1; ++j) {
-    issue(ic, j);
-    advance(ic);
-  }
+  for (int b = 0; b < B; ++b) acc[b] = pack2(0.0f, 0.0f);
 
-  int slot = 0, slot_issue = kRing - 1;  // ring buffer of this chunk / of the next copy
-  int m_work = 0, m_act = -1;
-  for (int64_t blk = p.cta_begin[blockIdx.x]; blk < blk_end; ++blk) {
-    const GemvItem& it = item_of(blk, m_work);
-    if (m_work != m_act) {
-      // a new matrix: every warp has finished with the old activations
-      __syncthreads();
-      const int pieces = static_cast<int>(it.cols / 4);
-      for (int b = 0; b < nb; ++b)
-        for (int P = threadIdx.x; P < pieces; P += kThreads) {
-          const uint2 a = __ldg(reinterpret_cast<const uint2*>(it.A + b * it.cols) + P);
-          const float4 f = make_float4(__uint_as_float(a.x << 16), __uint_as_float(a.x & 0xffff0000u),
-                                       __uint_as_float(a.y << 16), __uint_as_float(a.y & 0xffff0000u));
-          reinterpret_cast<float4*>(act + b * act_floats)[act_piece(static_cast<uint32_t>(P))] = f;
+  // the k-stage prefix weights of a lane's window and their products with
+  // the activations, four columns at a time
+  auto window_dot = [&](const Pos& c, const Window<F, K>& w) {
+    const GemvItem& it = p.item[c.m];
+    const int64_t col = static_cast<int64_t>(c.ch) * wcols + lane * lc;
+    if (col >= it.cols) return;  // beyond the row: nothing to add
+    const bool second = lc == 64;  // the lane's second 32 columns
+    const float4* ap = act4 + ((c.ch << lsh) << 5) + lane;  // piece j of row b: ap[b * act_pieces + j * 32]
+    auto dot = [&](int j, const f32x2& w01, const f32x2& w23) {
+#pragma unroll
+      for (int b = 0; b < B; ++b) {
+        if (b < nb) {
+          const float4 a = ap[b * act_pieces + j * 32];
+          acc[b] = fma2(w01, pack2(a.x, a.y), acc[b]);
+          acc[b] = fma2(w23, pack2(a.z, a.w), acc[b]);
         }
-      __syncthreads();
-      m_act = m_work;
-    }
-    const int64_t r = (blk - it.blk_begin) * kRows + warp;
-    if (r >= it.rows) continue;  // this warp has no row in the matrix's last block
-    const int cols = static_cast<int>(it.cols);
-    const int nch = (cols + kChunkElems - 1) / kChunkElems;
-
-    f32x2 acc[B];
+      }
+    };
+    if constexpr (kBits) {
+      // per-stage widths: the reconstruction's width-generic stage sum
 #pragma unroll
-    for (int b = 0; b < B; ++b) acc[b] = pack2(0.0f, 0.0f);
-
-    for (int ch = 0; ch < nch; ++ch) {
-      issue(ic, slot_issue);
-      advance(ic);
-      slot_issue = slot_issue == kRing - 1 ? 0 : slot_issue + 1;
-      cp_async_wait<kRing - 1>();  // this lane's copies of this chunk have landed
-
-      const int col = ch * kChunkElems + lane_col;
-      const uint8_t* buf = ring + slot * kBuf;
-      slot = slot == kRing - 1 ? 0 : slot + 1;
-      uint2 code[K];
-      float s[K], z[K];
+      for (int h = 0; h < 2; ++h) {
+        if (h == 1 && !second) break;
+        f32x2 v[16];
+#pragma unroll
+        for (int i = 0; i < K; ++i) {
+          const float s = __uint_as_float(w.s[i]), z = w.z[i];
+          const uint4 c0 = w.code[i][0], c1 = w.code[i][Window<F, K>::kVecs - 1];
+          switch (p.bits[i]) {  // half h: words [h b, h b + b) of the window's 2b
+            case 1: dequant_bits<1>(make_uint4(h ? c0.y : c0.x, 0u, 0u, 0u), s, z, i == 0, v); break;
+            case 3:
+              dequant_bits<3>(h ? make_uint4(c0.w, c1.x, c1.y, 0u) : make_uint4(c0.x, c0.y, c0.z, 0u), s, z, i == 0, v);
+              break;
+            case 4: dequant_bits<4>(h ? c1 : c0, s, z, i == 0, v); break;
+            default:
+              dequant_bits<2>(h ? make_uint4(c0.z, c0.w, 0u, 0u) : make_uint4(c0.x, c0.y, 0u, 0u), s, z, i == 0, v);
+              break;
+          }
+        }
+#pragma unroll
+        for (int q = 0; q < 8; ++q) dot(8 * h + q, v[2 * q], v[2 * q + 1]);
+      }
+    } else {
+      // code j of a byte (bits 2j, 2j+1) left in place under the exponent of
+      // 2^(23-2j): t = 2^(23-2j) + Q exactly, and fma(t, s, -2^(23-2j) s)
+      // gives fl(Q s) with one rounding (2^(23-2j) s exact: prescale_ok)
+      f32x2 S[K], C01[K], C23[K], Z[K];
       bool fast = true;
 #pragma unroll
       for (int i = 0; i < K; ++i) {
-        code[i] = F == kAsymBits ? make_uint2(0u, 0u) : *reinterpret_cast<const uint2*>(buf + i * kStageBytes + lane * 8);
-        if (kF16) {
-          const uint32_t word = *reinterpret_cast<const uint32_t*>(buf + i * kStageBytes + kCA + lane * 4);
-          const uint64_t gi = static_cast<uint64_t>(r * cols + col) >> p.log2g;
-          const uint32_t h = (gi & 1) ? (word >> 16) : (word & 0xffffu);
-          s[i] = __half2float(__ushort_as_half(static_cast<unsigned short>(h)));
-        } else {
-          s[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + kCA + lane * 4);
-          fast = fast && prescale_ok(s[i]);
-        }
-        z[i] = kSym ? 0.0f : *reinterpret_cast<const float*>(buf + i * kStageBytes + kCA + 128 + lane * 4);
+        const float s = kF16 ? __half2float(__ushort_as_half(static_cast<unsigned short>(w.s[i])))
+                             : __uint_as_float(w.s[i]);
+        if (!kF16) fast = fast && prescale_ok(s);  // binary16 scales always are
+        S[i] = pack2(s, s);
+        C01[i] = mul2(S[i], pack2(-0x1p23f, -0x1p21f));
+        C23[i] = mul2(S[i], pack2(-0x1p19f, -0x1p17f));
+        Z[i] = kSym ? pack2(0.0f, 0.0f) : pack2(w.z[i], w.z[i]);
       }
-      if (col >= cols) continue;  // beyond the row's last column: nothing to add
-      const uint8_t* abase = reinterpret_cast<const uint8_t*>(act) + static_cast<uint32_t>(ch) * (kChunkElems * 4);
-
-      // four columns at a time: the k-stage prefix weights, then w . a
-      auto dot = [&](int q, const f32x2& w01, const f32x2& w23) {
+      // symmetric levels: t - (2^(23-2j) + 2) = Q - 2 exactly
+      const f32x2 K01 = pack2(0x1p23f + 2.0f, 0x1p21f + 2.0f), K23 = pack2(0x1p19f + 2.0f, 0x1p17f + 2.0f);
 #pragma unroll
-        for (int b = 0; b < B; ++b) {
-          if (b < nb) {
-            const float4 a = *reinterpret_cast<const float4*>(abase + b * act_floats * 4 + poff[q]);
-            acc[b] = fma2(w01, pack2(a.x, a.y), acc[b]);
-            acc[b] = fma2(w23, pack2(a.z, a.w), acc[b]);
-          }
-        }
-      };
-      if constexpr (F == kAsymBits) {
-        // per-stage widths: the reconstruction's width-generic stage sum
-        f32x2 w[16];
+      for (int h = 0; h < 2; ++h) {
+        if (h == 1 && !second) break;
+        if (fast) {
 #pragma unroll
-        for (int i = 0; i < K; ++i) {
-          const uint4 w4 = *reinterpret_cast<const uint4*>(buf + i * kStageBytes + lane * 16);
-          switch (p.bits[i]) {
-            case 1: dequant_bits<1>(w4, s[i], z[i], i == 0, w); break;
-            case 3: dequant_bits<3>(w4, s[i], z[i], i == 0, w); break;
-            case 4: dequant_bits<4>(w4, s[i], z[i], i == 0, w); break;
-            default: dequant_bits<2>(w4, s[i], z[i], i == 0, w); break;
-          }
-        }
+          for (int q = 0; q < 8; ++q) {
+            f32x2 w01, w23;
 #pragma unroll
-        for (int q = 0; q < 8; ++q) dot(q, w[2 * q], w[2 * q + 1]);
-      } else if (fast) {
-        // t = 2^23 + Q*4^j exactly; s*4^-j exact (see reconstruct_kernel.cuh)
-        f32x2 S01[K], S23[K], C01[K], C23[K], Z[K];
-#pragma unroll
-        for (int i = 0; i < K; ++i) {
-          S01[i] = pack2(s[i], __fmul_rn(s[i], 0x1p-2f));
-          S23[i] = pack2(__fmul_rn(s[i], 0x1p-4f), __fmul_rn(s[i], 0x1p-6f));
-          C01[i] = pack2(__fmul_rn(s[i], -0x1p23f), __fmul_rn(s[i], -0x1p21f));
-          C23[i] = pack2(__fmul_rn(s[i], -0x1p19f), __fmul_rn(s[i], -0x1p17f));
-          Z[i] = pack2(z[i], z[i]);
-        }
-        const f32x2 K01 = pack2(kTwo23 + 2.0f, kTwo23 + 8.0f), K23 = pack2(kTwo23 + 32.0f, kTwo23 + 128.0f);
-#pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          f32x2 w01, w23;
-#pragma unroll
-          for (int i = 0; i < K; ++i) {
-            const uint32_t word = q < 4 ? code[i].x : code[i].y;
-            const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
-            const f32x2 t01 = pack2u(0x4B000000u | (b8 & 0x03u), 0x4B000000u | (b8 & 0x0Cu));
-            const f32x2 t23 = pack2u(0x4B000000u | (b8 & 0x30u), 0x4B000000u | (b8 & 0xC0u));
-            if (kSym) {  // (Q - 2) s, exact; summed by one fma
-              const f32x2 u01 = sub2(t01, K01), u23 = sub2(t23, K23);
-              w01 = (i == 0) ? mul2(u01, S01[i]) : fma2(u01, S01[i], w01);
-              w23 = (i == 0) ? mul2(u23, S23[i]) : fma2(u23, S23[i], w23);
-            } else {     // fl(zero + fl(Q s))
-              const f32x2 l01 = add2(Z[i], fma2(t01, S01[i], C01[i]));
-              const f32x2 l23 = add2(Z[i], fma2(t23, S23[i], C23[i]));
-              w01 = (i == 0) ? l01 : add2(w01, l01);
-              w23 = (i == 0) ? l23 : add2(w23, l23);
+            for (int i = 0; i < K; ++i) {
+              const uint4 cw = w.code[i][0];
+              const uint32_t word = h == 0 ? (q < 4 ? cw.x : cw.y) : (q < 4 ? cw.z : cw.w);
+              const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
+              const f32x2 t01 = pack2u(field_or<0x03u>(b8, 0x4B000000u), field_or<0x0Cu>(b8, 0x4A000000u));
+              const f32x2 t23 = pack2u(field_or<0x30u>(b8, 0x49000000u), field_or<0xC0u>(b8, 0x48000000u));
+              if (kSym) {  // (Q - 2) s, exact; summed by one fma
+                const f32x2 u01 = sub2(t01, K01), u23 = sub2(t23, K23);
+                w01 = (i == 0) ? mul2(u01, S[i]) : fma2(u01, S[i], w01);
+                w23 = (i == 0) ? mul2(u23, S[i]) : fma2(u23, S[i], w23);
+              } else {     // fl(zero + fl(Q s))
+                const f32x2 l01 = add2(Z[i], fma2(t01, S[i], C01[i]));
+                const f32x2 l23 = add2(Z[i], fma2(t23, S[i], C23[i]));
+                w01 = (i == 0) ? l01 : add2(w01, l01);
+                w23 = (i == 0) ? l23 : add2(w23, l23);
+              }
             }
+            dot(8 * h + q, w01, w23);
           }
-          dot(q, w01, w23);
-        }
-      } else {
-        // a scale outside [2^-100, 2^100]: unscaled codes, plain (t - 2^23) s
-        const f32x2 T = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f), K2 = pack2(kTwo23 + 2.0f, kTwo23 + 2.0f);
+        } else {
+          // a scale outside [2^-100, 2^100]: unscaled codes, plain (t - 2^23) s
+          const f32x2 T = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f), K2 = pack2(kTwo23 + 2.0f, kTwo23 + 2.0f);
 #pragma unroll
-        for (int q = 0; q < 8; ++q) {
-          f32x2 w01, w23;
+          for (int q = 0; q < 8; ++q) {
+            f32x2 w01, w23;
 #pragma unroll
-          for (int i = 0; i < K; ++i) {
-            const uint32_t word = q < 4 ? code[i].x : code[i].y;
-            const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
-            const f32x2 t01 = pack2u(0x4B000000u | (b8 & 3u), 0x4B000000u | ((b8 >> 2) & 3u));
-            const f32x2 t23 = pack2u(0x4B000000u | ((b8 >> 4) & 3u), 0x4B000000u | ((b8 >> 6) & 3u));
-            const f32x2 S = pack2(s[i], s[i]);
-            if (kSym) {
-              const f32x2 u01 = sub2(t01, K2), u23 = sub2(t23, K2);
-              w01 = (i == 0) ? mul2(u01, S) : fma2(u01, S, w01);
-              w23 = (i == 0) ? mul2(u23, S) : fma2(u23, S, w23);
-            } else {
-              const f32x2 Z = pack2(z[i], z[i]);
-              const f32x2 l01 = add2(Z, fma2(sub2(t01, T), S, Z0));
-              const f32x2 l23 = add2(Z, fma2(sub2(t23, T), S, Z0));
-              w01 = (i == 0) ? l01 : add2(w01, l01);
-              w23 = (i == 0) ? l23 : add2(w23, l23);
+            for (int i = 0; i < K; ++i) {
+              const uint4 cw = w.code[i][0];
+              const uint32_t word = h == 0 ? (q < 4 ? cw.x : cw.y) : (q < 4 ? cw.z : cw.w);
+              const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
+              const f32x2 t01 = pack2u(magic23<3u>(b8), magic23<3u>(b8 >> 2));
+              const f32x2 t23 = pack2u(magic23<3u>(b8 >> 4), magic23<3u>(b8 >> 6));
+              if (kSym) {
+                const f32x2 u01 = sub2(t01, K2), u23 = sub2(t23, K2);
+                w01 = (i == 0) ? mul2(u01, S[i]) : fma2(u01, S[i], w01);
+                w23 = (i == 0) ? mul2(u23, S[i]) : fma2(u23, S[i], w23);
+              } else {
+                const f32x2 l01 = add2(Z[i], fma2(sub2(t01, T), S[i], Z0));
+                const f32x2 l23 = add2(Z[i], fma2(sub2(t23, T), S[i], Z0));
+                w01 = (i == 0) ? l01 : add2(w01, l01);
+                w23 = (i == 0) ? l23 : add2(w23, l23);
+              }
             }
+            dot(8 * h + q, w01, w23);
           }
-          dot(q, w01, w23);
         }
       }
     }
+  };
 
-    // end of the row: reduce over the warp in a fixed order and store
+  // end of a row: reduce over the warp in a fixed order and store
+  auto finish_row = [&](const Pos& c) {
+    const GemvItem& it = p.item[c.m];
+    const int64_t r = (c.blk - it.blk_begin) * kRows + warp;
 #pragma unroll
     for (int b = 0; b < B; ++b) {
       float x, y;
@@ -333,37 +345,76 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
 #pragma unroll
       for (int off = 16; off > 0; off >>= 1) t = __fadd_rn(t, __shfl_xor_sync(kFullMask, t, off));
       if (lane == 0 && b < nb) it.Y[b * it.rows + r] = t;
+      acc[b] = pack2(0.0f, 0.0f);
     }
+  };
+
+  // two windows in registers, loaded one ahead of use
+  Pos pa{0, 0, m_first, 0, 0}, pb{0, 0, m_first, 0, 0};
+  Window<F, K> wa{}, wb{};
+  seek(pa, blk_begin);
+  load(pa, wa);
+  auto step = [&](const Pos& pc, const Window<F, K>& wc, Pos& pn, Window<F, K>& wn) -> bool {
+    if (pc.blk >= blk_end) return false;
+    pn = pc;
+    if (++pn.ch >= pn.nch) seek(pn, pc.blk + 1);
+    load(pn, wn);
+    switch_to(pc.m);
+    window_dot(pc, wc);
+    if (pc.ch == pc.nch - 1) finish_row(pc);
+    return true;
+  };
+  while (step(pa, wa, pb, wb) && step(pb, wb, pa, wa)) {
   }
-  cp_async_wait<0>();
+  switch_to(m_last);
 }
 
-// activation rows a launch can hold for matrices of up to max_cols columns
+// activation floats per row a launch keeps for matrices of up to max_cols columns
 inline int64_t act_floats_of(int64_t max_cols) {
-  return ((max_cols + kChunkElems - 1) / kChunkElems) * kChunkElems;
+  return ((max_cols + kWinCols - 1) / kWinCols) * kWinCols;
 }
-template <int F, int K>
-int tokens_per_launch(int64_t max_cols) {
-  const int64_t t = (kMaxSmem - ring_bytes<F, K>()) / (act_floats_of(max_cols) * 4);
+inline int tokens_per_launch(int64_t max_cols) {
+  const int64_t t = kMaxSmem / (act_floats_of(max_cols) * 4);
   return static_cast<int>(t < kMaxGemvBatch ? t : kMaxGemvBatch);
 }
 
+constexpr int kMaxDevices = 64;
+
 template <int F, int K, int B>
-cudaError_t launch_fkb(const GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
-  static int attr_bytes = 0;  // largest dynamic shared memory enabled so far (same for every device)
+cudaError_t launch_fkb(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
+  // per device: the largest dynamic shared memory enabled so far, and the
+  // resident CTAs per multiprocessor at the last size asked
+  static int attr_bytes[kMaxDevices] = {};
+  static int occ_smem[kMaxDevices] = {};
+  static int occ[kMaxDevices] = {};
+  int dev = 0;
+  cudaError_t e = cudaGetDevice(&dev);
+  if (e != cudaSuccess) return e;
+  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
   const int act_floats = static_cast<int>(act_floats_of(max_cols));
-  const int smem = ring_bytes<F, K>() + nb * act_floats * 4;
-  if (smem > attr_bytes) {
-    cudaError_t e = cudaFuncSetAttribute(gemv_kernel<F, K, B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+  const int smem = nb * act_floats * 4;
+  if (smem > attr_bytes[dev]) {
+    e = cudaFuncSetAttribute(gemv_kernel<F, K, B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
     if (e != cudaSuccess) return e;
-    attr_bytes = smem;
+    attr_bytes[dev] = smem;
   }
+  if (occ[dev] == 0 || occ_smem[dev] != smem) {
+    int n = 0;
+    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<F, K, B>, kThreads, smem);
+    if (e != cudaSuccess) return e;
+    occ[dev] = n < 1 ? 1 : n;
+    occ_smem[dev] = smem;
+  }
+  int64_t grid = static_cast<int64_t>(sms) * occ[dev];
+  if (grid > kMaxGemvGrid) grid = kMaxGemvGrid;
+  if (grid > p.total_blocks) grid = p.total_blocks;
+  gemv_split(p, static_cast<int>(grid));
   gemv_kernel<F, K, B><<<p.grid, kThreads, smem, stream>>>(p, nb, act_floats);
   return cudaGetLastError();
 }
 
 template <int F, int K>
-cudaError_t launch_fk(int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms) {
+cudaError_t launch_fk(int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms) {
   if (nb <= 1) return launch_fkb<F, K, 1>(p, nb, max_cols, stream, sms);
   if (nb <= 2) return launch_fkb<F, K, 2>(p, nb, max_cols, stream, sms);
   if (nb <= 4) return launch_fkb<F, K, 4>(p, nb, max_cols, stream, sms);
@@ -372,7 +423,7 @@ cudaError_t launch_fk(int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t
 
 // Launch of one format (instantiated by one translation unit each).
 template <int F>
-cudaError_t launch_format(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms) {
+cudaError_t launch_format(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms) {
   switch (k) {
     case 1: return launch_fk<F, 1>(nb, max_cols, p, stream, sms);
     case 2: return launch_fk<F, 2>(nb, max_cols, p, stream, sms);

@@ -282,8 +282,8 @@ __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32
       for (int j = 0; j < NW / 4; ++j) {  // byte j: weights 4j..4j+3 (pairs 2j, 2j+1)
         const uint32_t word = j < 4 ? w.cw[i].x : w.cw[i].y;
         const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-        const f32x2 t01 = pack2u(0x4B000000u | (b & 0x03u), 0x4B000000u | (b & 0x0Cu));
-        const f32x2 t23 = pack2u(0x4B000000u | (b & 0x30u), 0x4B000000u | (b & 0xC0u));
+        const f32x2 t01 = pack2u(magic23<0x03u>(b), magic23<0x0Cu>(b));
+        const f32x2 t23 = pack2u(magic23<0x30u>(b), magic23<0xC0u>(b));
         if constexpr (kSym) {  // 4^j (Q - 2), exact; times s / 4^j exact
           const f32x2 u01 = sub2(t01, K01), u23 = sub2(t23, K23);
           acc[2 * j] = (i == 0) ? mul2(u01, S01) : fma2(u01, S01, acc[2 * j]);
@@ -303,7 +303,7 @@ __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32
       for (int m = 0; m < NW / 2; ++m) {
         const uint32_t word = m < 8 ? w.cw[i].x : w.cw[i].y;
         const int sh = 4 * (m & 7);
-        const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+        const f32x2 t = pack2u(magic23<3u>(word >> sh), magic23<3u>(word >> (sh + 2)));
         if constexpr (kSym) {
           const f32x2 u = sub2(t, K2);  // Q - 2, exact
           acc[m] = (i == 0) ? mul2(u, S) : fma2(u, S, acc[m]);

@@ -434,7 +434,7 @@ __device__ __forceinline__ void subtract_base(f32x2 (&v)[16], const BaseWords& b
     for (int i = 0; i < 16; ++i) {
       const uint32_t word = i < 8 ? w0 : w1;
       const int sh = 4 * (i & 7);
-      const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+      const f32x2 t = pack2u(magic23<3u>(word >> sh), magic23<3u>(word >> (sh + 2)));
       const f32x2 qs = scaled_ok ? fma2(t, S, C) : fma2(sub2(t, T23), S, Z0);
       v[i] = sub2(v[i], add2(Z, qs));
     }
@@ -445,7 +445,7 @@ __device__ __forceinline__ void subtract_base(f32x2 (&v)[16], const BaseWords& b
     for (int i = 0; i < 16; ++i) {
       const uint32_t word = i < 8 ? w0 : w1;
       const int sh = 4 * (i & 7);
-      const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+      const f32x2 t = pack2u(magic23<3u>(word >> sh), magic23<3u>(word >> (sh + 2)));
       v[i] = fma2(sub2(t, K2), NS, v[i]);
     }
   }

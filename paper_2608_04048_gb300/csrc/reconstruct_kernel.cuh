@@ -226,8 +226,8 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
           for (int j = 0; j < 8; ++j) {
             const uint32_t word = j < 4 ? w0 : w1;
             const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-            const f32x2 u01 = sub2(pack2u(0x4B000000u | (b & 0x03u), 0x4B000000u | (b & 0x0Cu)), K01);
-            const f32x2 u23 = sub2(pack2u(0x4B000000u | (b & 0x30u), 0x4B000000u | (b & 0xC0u)), K23);
+            const f32x2 u01 = sub2(pack2u(magic23<0x03u>(b), magic23<0x0Cu>(b)), K01);
+            const f32x2 u23 = sub2(pack2u(magic23<0x30u>(b), magic23<0xC0u>(b)), K23);
             acc[2 * j] = (i == 0) ? mul2(u01, S01) : fma2(u01, S01, acc[2 * j]);
             acc[2 * j + 1] = (i == 0) ? mul2(u23, S23) : fma2(u23, S23, acc[2 * j + 1]);
           }
@@ -237,7 +237,7 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
           for (int m = 0; m < 16; ++m) {
             const uint32_t word = m < 8 ? w0 : w1;
             const int sh = 4 * (m & 7);
-            const f32x2 u = sub2(pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u)), K2);
+            const f32x2 u = sub2(pack2u(magic23<3u>(word >> sh), magic23<3u>(word >> (sh + 2))), K2);
             acc[m] = (i == 0) ? mul2(u, S) : fma2(u, S, acc[m]);
           }
         }
@@ -251,8 +251,8 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
         for (int j = 0; j < 8; ++j) {  // byte j: elements 4j..4j+3 (pairs 2j, 2j+1)
           const uint32_t word = j < 4 ? w0 : w1;
           const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-          const f32x2 t01 = pack2u(0x4B000000u | (b & 0x03u), 0x4B000000u | (b & 0x0Cu));
-          const f32x2 t23 = pack2u(0x4B000000u | (b & 0x30u), 0x4B000000u | (b & 0xC0u));
+          const f32x2 t01 = pack2u(magic23<0x03u>(b), magic23<0x0Cu>(b));
+          const f32x2 t23 = pack2u(magic23<0x30u>(b), magic23<0xC0u>(b));
           const f32x2 l01 = add2(LO, fma2(t01, S01, C01));
           const f32x2 l23 = add2(LO, fma2(t23, S23, C23));
           acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
@@ -265,7 +265,7 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
         for (int m = 0; m < 16; ++m) {
           const uint32_t word = m < 8 ? w0 : w1;
           const int sh = 4 * (m & 7);
-          const f32x2 t = pack2u(0x4B000000u | ((word >> sh) & 3u), 0x4B000000u | ((word >> (sh + 2)) & 3u));
+          const f32x2 t = pack2u(magic23<3u>(word >> sh), magic23<3u>(word >> (sh + 2)));
           // RN(Q*s) through an fma with a zero addend (the compiler would fuse
           // a separate multiply into the following add)
           const f32x2 level = add2(LO, fma2(sub2(t, T23), S, Z));

@@ -142,6 +142,22 @@ __device__ __forceinline__ f32x2 pack2u(uint32_t lo, uint32_t hi) {
   asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(lo), "r"(hi));
   return r;
 }
+// (x & M) | e in one three-input logic instruction, with e in a register: a
+// code field masked in place under a float exponent (the code-to-float step
+// of every dequantisation).  Written out because the two constants of the
+// plain C form otherwise become an AND and an OR.
+template <uint32_t M>
+__device__ __forceinline__ uint32_t field_or(uint32_t x, uint32_t e) {
+  uint32_t r;
+  asm("lop3.b32 %0, %1, %2, %3, 0xEA;" : "=r"(r) : "r"(x), "n"(M), "r"(e));
+  return r;
+}
+// the float (2^23 + Q 2^k) for the field of x at bits k, k+1 (mask M = 3 << k)
+template <uint32_t M>
+__device__ __forceinline__ uint32_t magic23(uint32_t x) {
+  return field_or<M>(x, 0x4B000000u);
+}
+
 __device__ __forceinline__ void unpack2(f32x2 v, float& a, float& b) {
   asm("mov.b64 {%0, %1}, %2;" : "=f"(a), "=f"(b) : "l"(v));
 }
@@ -183,16 +199,16 @@ __device__ __forceinline__ float max3(float a, float b, float c) {
 template <int B>
 __device__ __forceinline__ void dequant_bits(const uint4& w4, float s, float z, bool first, f32x2 (&acc)[16]) {
   const uint32_t w[4] = {w4.x, w4.y, w4.z, w4.w};
-  auto code = [&](int j) -> uint32_t {
+  auto code = [&](int j) -> uint32_t {  // bits B*j.. of the code, unmasked above
     const int bit = B * j, i = bit >> 5, sh = bit & 31;
     uint32_t c = w[i] >> sh;
     if (sh + B > 32) c |= w[i + 1] << (32 - sh);
-    return c & ((1u << B) - 1u);
+    return c;
   };
   const f32x2 S = pack2(s, s), Z = pack2(z, z), T23 = pack2(8388608.0f, 8388608.0f), Z0 = pack2(0.0f, 0.0f);
 #pragma unroll
   for (int m = 0; m < 16; ++m) {
-    const f32x2 t = pack2u(0x4B000000u | code(2 * m), 0x4B000000u | code(2 * m + 1));
+    const f32x2 t = pack2u(magic23<(1u << B) - 1u>(code(2 * m)), magic23<(1u << B) - 1u>(code(2 * m + 1)));
     const f32x2 level = add2(Z, fma2(sub2(t, T23), S, Z0));  // fl(zero + fl(Q s))
     acc[m] = first ? level : add2(acc[m], level);
   }

@@ -82,7 +82,7 @@ struct GemvItem {
   int64_t blk_begin;
 };
 
-constexpr int kMaxGemvGrid = 256;  // CTAs of one launch (at most one per multiprocessor)
+constexpr int kMaxGemvGrid = 512;  // CTAs of one launch
 
 struct GemvBatch {
   int count;
@@ -95,6 +95,29 @@ struct GemvBatch {
 };
 
 constexpr int kGemvRows = 16;      // rows per block
+
+// Cuts the launch's blocks into `grid` contiguous ranges (one per CTA) with
+// equal shares of rows x columns; sets p.grid and p.cta_begin.
+inline void gemv_split(GemvBatch& p, int grid) {
+  p.grid = grid;
+  int64_t total = 0;
+  for (int i = 0; i < p.count; ++i) total += p.item[i].rows * p.item[i].cols;
+  int c = 0;
+  int64_t done = 0, blk = 0;
+  p.cta_begin[0] = 0;
+  for (int i = 0; i < p.count && c < grid; ++i) {
+    const GemvItem& it = p.item[i];
+    const int64_t nblk = (it.rows + kGemvRows - 1) / kGemvRows;
+    for (int64_t b = 0; b < nblk; ++b, ++blk) {
+      const int64_t r = it.rows - b * kGemvRows < kGemvRows ? it.rows - b * kGemvRows : kGemvRows;
+      done += r * it.cols;
+      // close CTA c's range once its share is reached
+      while (c + 1 < grid && done * grid >= (c + 1) * total) p.cta_begin[++c] = blk + 1;
+    }
+  }
+  while (c < grid) p.cta_begin[++c] = p.total_blocks;
+  p.cta_begin[grid] = p.total_blocks;
+}
 
 constexpr int kMaxGemvBatch = 8;   // activation rows (tokens) per call
 
@@ -211,12 +234,12 @@ cudaError_t reconstruct_launch_asym_bits(int group, int k, bool all_prefixes, co
 int gemv_rows_per_launch(Format fmt, int k, int64_t max_cols);
 // nb activation rows (1..kMaxGemvBatch, within gemv_rows_per_launch); one
 // translation unit per format.
-cudaError_t gemv_launch_asym_f32(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
-cudaError_t gemv_launch_sym_f32(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
-cudaError_t gemv_launch_sym_f16(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
-cudaError_t gemv_launch_asym_bits(int k, int nb, int64_t max_cols, const GemvBatch& p, cudaStream_t stream, int sms);
+cudaError_t gemv_launch_asym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms);
+cudaError_t gemv_launch_sym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms);
+cudaError_t gemv_launch_sym_f16(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms);
+cudaError_t gemv_launch_asym_bits(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms);
 
-inline cudaError_t gemv_launch(Format fmt, int k, int nb, int64_t max_cols, const GemvBatch& p,
+inline cudaError_t gemv_launch(Format fmt, int k, int nb, int64_t max_cols, GemvBatch& p,
                                cudaStream_t stream, int sms) {
   switch (fmt) {
     case kAsymF32: return gemv_launch_asym_f32(k, nb, max_cols, p, stream, sms);

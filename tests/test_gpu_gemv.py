@@ -3,11 +3,12 @@ Appendix C): Y = A W~^T from the package alone, against the oracle's binary64
 product of the same binary32 prefix weights.
 
 Tolerance, from the kernel's arithmetic: every product W~ a is exact inside
-its fma and every partial sum is rounded once; a lane sums its 32 columns of
-each 1024-column chunk into two accumulators (16 columns each, chunks in
-turn), then adds the two and the warp adds 32 lanes in 5 butterfly steps, so
-no term passes through more than d = cols/64 + 8 roundings and
-|Y - exact| <= d * 2^-24 * sum_c |W~ a| (first order).  sum_c |W~ a| is
+its fma and every partial sum is rounded once; a lane sums its 64 columns of
+each 2048-column window (32 of 1024 when the group is 32) into two
+accumulators (32 columns each, windows in turn), then adds the two and the
+warp adds 32 lanes in 5 butterfly steps, so no term passes through more than
+d = 32 ceil(cols/2048) + 8 roundings and |Y - exact| <= d * 2^-24 *
+sum_c |W~ a| (first order).  sum_c |W~ a| is
 bounded with the bf16 reconstruction: |W~| <= |bf16(W~)| (1 + 2^-8)."""
 import numpy as np
 import pytest
@@ -30,6 +31,11 @@ def lib():
     build.build()
     binding.load_library()
     binding.rrq_set_debug_flags(0)
+
+
+def _depth(cols):
+    """Roundings a term of a row of `cols` columns passes through at most."""
+    return 32 * -(-cols // 2048) + 8
 
 
 def _host_pkg(pkg, rows_idx=None):
@@ -63,7 +69,7 @@ def _check(pkg, A, Y, k, rows_idx=None, where=""):
         rec = oracle.reconstruct(codes, scales, zeros, nr, pkg.cols, pkg.group, k)
     recf = np.abs((rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
     Af = np.abs((Ab.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
-    d = pkg.cols // 64 + 8
+    d = _depth(pkg.cols)
     tol = d * 2.0 ** -24 * (Af @ recf.T) * (1 + 2.0 ** -8) + 1e-30
     got = Y.cpu().numpy().astype(np.float64)
     if rows_idx is not None:
@@ -166,7 +172,7 @@ def test_widths(batch, bits, group):
         want = oracle.product_bits(codes, scales, zeros, rows, cols, group, k, bits, Ab, False)
         rec = oracle.reconstruct_bits(codes, scales, zeros, rows, cols, group, k, bits)
         recf = np.abs((rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
-        d = cols // 64 + 8
+        d = _depth(cols)
         tol = d * 2.0 ** -24 * (Af @ recf.T) * (1 + 2.0 ** -8) + 1e-30
         err = np.abs(Y.cpu().numpy().astype(np.float64) - want)
         assert not np.any(err > tol), f"{bits} g{group} B{batch} k{k}: {int((err > tol).sum())} outputs beyond the bound"
