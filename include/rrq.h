@@ -308,6 +308,7 @@ typedef struct {
 } rrq_gemv_desc;
 
 #define RRQ_MAX_GEMV_BATCH 8
+#define RRQ_MAX_GEMV_COLS 57344
 
 /* Product of activations with the prefix-k weights, without materialising
  * them (Appendix C: A W~_(t) = A W^_0 + sum_k A R^_k):
@@ -320,8 +321,12 @@ typedef struct {
  * sum_c |W~ A|).  For decoding: 1 <= batch <= RRQ_MAX_GEMV_BATCH activation
  * rows; 1 <= k <= fmt->n_stages.  Per-stage widths (fmt->bits, asymmetric
  * grid) are taken with the reconstruction's stage sum of that format.  Y must
- * not overlap any input or another Y.  One launch per 64 matrices; other
- * rules as for rrq_reconstruct_ex. */
+ * not overlap any input or another Y.  The activation rows of a launch are
+ * held in shared memory as binary32, padded to a multiple of 2048 columns:
+ * a launch takes as many of the batch's rows as fit in 227 KiB, so the
+ * widest matrix of a call may have at most RRQ_MAX_GEMV_COLS columns
+ * (RRQ_ERR_UNSUPPORTED beyond).  One launch per 64 matrices and per such
+ * share of the batch; other rules as for rrq_reconstruct_ex. */
 rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
                     rrq_stream_t stream);
 

@@ -13,13 +13,14 @@
 // one contiguous range per CTA of a persistent grid (as many CTAs as fit on
 // the multiprocessors) with equal shares of rows x columns, so that a CTA
 // meets few matrices.  The CTA's 16 warps take one row of each block each.
-// A warp walks its row in windows of 2048 columns, lane l owning the 64
-// columns 64l..64l+63 of the window (1024 and 32 when the group is 32, so that
-// a lane's columns share one group; with a larger group the row length is a
-// multiple of 64, so a lane's 64 columns are all in the row or all past its
-// end): per stage one 16-byte load of codes (8 bytes for 32 columns) and one
-// scale and zero, all loaded into registers one window ahead, across rows,
-// blocks and matrices.
+// A warp walks its row in windows of 32 x lc columns, lane l owning the lc
+// columns lc*l .. lc*l + lc-1 of the window: lc = 128 for k <= 2 and up to
+// 2 activation rows (64 otherwise, where registers are scarcer), never more
+// than the group, so that a lane's columns share one group (the row length
+// is a multiple of the group, so a lane's columns are all in the row or all
+// past its end).  Per stage the lane loads lc/4 bytes of codes (16-byte
+// loads; 8 bytes for 32 columns) and one scale and zero, all into registers
+// one window ahead, across rows, blocks and matrices.
 //
 // The CTA keeps the activations of its current matrix in shared memory as
 // binary32, converted once per matrix, stored transposed within each window:
@@ -34,9 +35,9 @@
 //
 // Accuracy: every product W~ * a is exact inside its fma and each partial sum
 // is rounded once.  A lane's two accumulators (even and odd columns of each
-// pair) each take at most 32 products per 2048 columns of the row (rounded
+// pair) each take at most 64 products per 4096 columns of the row (rounded
 // up), then the pair and 5 butterfly steps, so |Y - exact| <=
-// (32 ceil(cols/2048) + 6) * 2^-24 * sum_c |W~ a| to first order.
+// (64 ceil(cols/4096) + 6) * 2^-24 * sum_c |W~ a| to first order.
 //
 // This header holds the kernel template; gemv_asym_f32.cu, gemv_sym_f32.cu,
 // gemv_sym_f16.cu and gemv_asym_bits.cu each instantiate one package format.
@@ -44,6 +45,7 @@
 
 #include <cuda_fp16.h>
 
+#include "rrq.h"  // RRQ_MAX_GEMV_COLS
 #include "rrq_device.cuh"
 
 namespace rrq {
@@ -53,7 +55,13 @@ constexpr int kWarps = 16;
 constexpr int kThreads = kWarps * 32;
 constexpr int kRows = kGemvRows;       // rows per block (one per warp)
 static_assert(kRows == kWarps, "one row of a block per warp");
-constexpr int kWinCols = 2048;         // columns of a warp's window (1024 when the group is 32)
+constexpr int kWinCols = 4096;         // columns of the widest warp window (activation padding)
+
+// Columns a lane owns in a window at most: 128 at k <= 2 with 1 or 2
+// activation rows (more weights per window's fixed cost), else 64
+// (registers).
+template <int F, int K, int B>
+__host__ __device__ constexpr int lane_cols_max() { return (F != kAsymBits && K <= 2 && B <= 2) ? 128 : 64; }
 constexpr int kMaxSmem = 227 * 1024;
 constexpr float kTwo23 = 8388608.0f;
 
@@ -83,9 +91,9 @@ __device__ __forceinline__ uint32_t ld_nc2(const void* p) {
 // A lane's package data of one window: per stage the codes of its 64 (or 32)
 // columns (16 bytes at 2 bits; up to 32 bytes with per-stage widths), and the
 // raw scale and zero of their group.
-template <int F, int K>
+template <int F, int K, int B>
 struct Window {
-  static constexpr int kVecs = F == kAsymBits ? 2 : 1;
+  static constexpr int kVecs = F == kAsymBits ? 2 : lane_cols_max<F, K, B>() / 64;
   uint4 code[K][kVecs];
   uint32_t s[K];  // binary32 bits, or binary16 bits in the low half
   float z[K];
@@ -119,10 +127,13 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
   const int64_t blk_end = p.cta_begin[blockIdx.x + 1];
   if (blk_begin >= blk_end) return;  // the whole CTA: no barrier is reached
   const int log2g = p.log2g;
-  const int lc = log2g == 5 ? 32 : 64;  // columns of a lane in a window: within one group
-  const int wcols = 32 * lc;            // columns of a window
-  const int lsh = log2g == 5 ? 3 : 4;   // log2 of a lane's 16-byte pieces per window
-  const int wsh = lsh + 7;              // log2 of wcols
+  constexpr int kLCM = lane_cols_max<F, K, B>();
+  // columns of a lane in a window: within one group
+  const int lc = (1 << log2g) < kLCM ? (1 << log2g) : kLCM;
+  const int wcols = 32 * lc;                          // columns of a window
+  const int lsh = lc == 32 ? 3 : (lc == 64 ? 4 : 5);  // log2 of a lane's 16-byte pieces per window
+  const int wsh = lsh + 7;                            // log2 of wcols
+  const int nh = lc >> 5;                             // 32-column parts of a lane's window
   const int act_pieces = act_floats / 4;
 
   auto item_index = [&](int64_t blk, int m) {
@@ -178,7 +189,7 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
   };
 
   // this lane's package data of window c, into registers
-  auto load = [&](const Pos& c, Window<F, K>& w) {
+  auto load = [&](const Pos& c, Window<F, K, B>& w) {
     if (c.blk >= blk_end) return;
     const GemvItem& it = p.item[c.m];
     const int64_t col = static_cast<int64_t>(c.ch) * wcols + lane * lc;
@@ -189,7 +200,7 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
     for (int i = 0; i < K; ++i) {
       if constexpr (kBits) {  // 8b bytes for 64 codes of width b, 4-byte aligned
         const int b = p.bits[i];
-        const int words = lc == 64 ? 2 * b : b;
+        const int words = nh * b;
         const uint32_t* src = reinterpret_cast<const uint32_t*>(it.codes[i]) + (e >> 5) * b;
         uint32_t wd[8];
 #pragma unroll
@@ -198,8 +209,10 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
         w.code[i][kBits ? 1 : 0] = make_uint4(wd[4], wd[5], wd[6], wd[7]);
       } else {
         const uint8_t* src = it.codes[i] + (e >> 2);
-        if (lc == 64) {
+        if (lc >= 64) {
           w.code[i][0] = ld_nc16(src);
+          if constexpr (Window<F, K, B>::kVecs > 1)
+            if (lc == 128) w.code[i][Window<F, K, B>::kVecs - 1] = ld_nc16(src + 16);
         } else {
           const uint2 v = ld_nc8(src);
           w.code[i][0] = make_uint4(v.x, v.y, 0u, 0u);
@@ -217,11 +230,10 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
 
   // the k-stage prefix weights of a lane's window and their products with
   // the activations, four columns at a time
-  auto window_dot = [&](const Pos& c, const Window<F, K>& w) {
+  auto window_dot = [&](const Pos& c, const Window<F, K, B>& w) {
     const GemvItem& it = p.item[c.m];
     const int64_t col = static_cast<int64_t>(c.ch) * wcols + lane * lc;
     if (col >= it.cols) return;  // beyond the row: nothing to add
-    const bool second = lc == 64;  // the lane's second 32 columns
     const float4* ap = act4 + ((c.ch << lsh) << 5) + lane;  // piece j of row b: ap[b * act_pieces + j * 32]
     auto dot = [&](int j, const f32x2& w01, const f32x2& w23) {
 #pragma unroll
@@ -237,12 +249,12 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
       // per-stage widths: the reconstruction's width-generic stage sum
 #pragma unroll
       for (int h = 0; h < 2; ++h) {
-        if (h == 1 && !second) break;
+        if (h >= nh) break;
         f32x2 v[16];
 #pragma unroll
         for (int i = 0; i < K; ++i) {
           const float s = __uint_as_float(w.s[i]), z = w.z[i];
-          const uint4 c0 = w.code[i][0], c1 = w.code[i][Window<F, K>::kVecs - 1];
+          const uint4 c0 = w.code[i][0], c1 = w.code[i][Window<F, K, B>::kVecs - 1];
           switch (p.bits[i]) {  // half h: words [h b, h b + b) of the window's 2b
             case 1: dequant_bits<1>(make_uint4(h ? c0.y : c0.x, 0u, 0u, 0u), s, z, i == 0, v); break;
             case 3:
@@ -276,16 +288,16 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
       // symmetric levels: t - (2^(23-2j) + 2) = Q - 2 exactly
       const f32x2 K01 = pack2(0x1p23f + 2.0f, 0x1p21f + 2.0f), K23 = pack2(0x1p19f + 2.0f, 0x1p17f + 2.0f);
 #pragma unroll
-      for (int h = 0; h < 2; ++h) {
-        if (h == 1 && !second) break;
+      for (int h = 0; h < kLCM / 32; ++h) {
+        if (h >= nh) break;
         if (fast) {
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
             f32x2 w01, w23;
 #pragma unroll
             for (int i = 0; i < K; ++i) {
-              const uint4 cw = w.code[i][0];
-              const uint32_t word = h == 0 ? (q < 4 ? cw.x : cw.y) : (q < 4 ? cw.z : cw.w);
+              const uint4 cw = w.code[i][h >> 1];
+              const uint32_t word = (h & 1) == 0 ? (q < 4 ? cw.x : cw.y) : (q < 4 ? cw.z : cw.w);
               const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
               const f32x2 t01 = pack2u(field_or<0x03u>(b8, 0x4B000000u), field_or<0x0Cu>(b8, 0x4A000000u));
               const f32x2 t23 = pack2u(field_or<0x30u>(b8, 0x49000000u), field_or<0xC0u>(b8, 0x48000000u));
@@ -310,8 +322,8 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
             f32x2 w01, w23;
 #pragma unroll
             for (int i = 0; i < K; ++i) {
-              const uint4 cw = w.code[i][0];
-              const uint32_t word = h == 0 ? (q < 4 ? cw.x : cw.y) : (q < 4 ? cw.z : cw.w);
+              const uint4 cw = w.code[i][h >> 1];
+              const uint32_t word = (h & 1) == 0 ? (q < 4 ? cw.x : cw.y) : (q < 4 ? cw.z : cw.w);
               const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
               const f32x2 t01 = pack2u(magic23<3u>(b8), magic23<3u>(b8 >> 2));
               const f32x2 t23 = pack2u(magic23<3u>(b8 >> 4), magic23<3u>(b8 >> 6));
@@ -351,10 +363,10 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
 
   // two windows in registers, loaded one ahead of use
   Pos pa{0, 0, m_first, 0, 0}, pb{0, 0, m_first, 0, 0};
-  Window<F, K> wa{}, wb{};
+  Window<F, K, B> wa{}, wb{};
   seek(pa, blk_begin);
   load(pa, wa);
-  auto step = [&](const Pos& pc, const Window<F, K>& wc, Pos& pn, Window<F, K>& wn) -> bool {
+  auto step = [&](const Pos& pc, const Window<F, K, B>& wc, Pos& pn, Window<F, K, B>& wn) -> bool {
     if (pc.blk >= blk_end) return false;
     pn = pc;
     if (++pn.ch >= pn.nch) seek(pn, pc.blk + 1);
@@ -370,9 +382,12 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
 }
 
 // activation floats per row a launch keeps for matrices of up to max_cols columns
-inline int64_t act_floats_of(int64_t max_cols) {
+constexpr int64_t act_floats_of(int64_t max_cols) {
   return ((max_cols + kWinCols - 1) / kWinCols) * kWinCols;
 }
+static_assert(act_floats_of(RRQ_MAX_GEMV_COLS) * 4 <= kMaxSmem &&
+                  act_floats_of(RRQ_MAX_GEMV_COLS + 32) * 4 > kMaxSmem,
+              "RRQ_MAX_GEMV_COLS is the widest row one activation row of a launch holds");
 inline int tokens_per_launch(int64_t max_cols) {
   const int64_t t = kMaxSmem / (act_floats_of(max_cols) * 4);
   return static_cast<int>(t < kMaxGemvBatch ? t : kMaxGemvBatch);

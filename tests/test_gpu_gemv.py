@@ -3,12 +3,12 @@ Appendix C): Y = A W~^T from the package alone, against the oracle's binary64
 product of the same binary32 prefix weights.
 
 Tolerance, from the kernel's arithmetic: every product W~ a is exact inside
-its fma and every partial sum is rounded once; a lane sums its 64 columns of
-each 2048-column window (32 of 1024 when the group is 32) into two
-accumulators (32 columns each, windows in turn), then adds the two and the
-warp adds 32 lanes in 5 butterfly steps, so no term passes through more than
-d = 32 ceil(cols/2048) + 8 roundings and |Y - exact| <= d * 2^-24 *
-sum_c |W~ a| (first order).  sum_c |W~ a| is
+its fma and every partial sum is rounded once; a lane sums its lc columns of
+each 32 lc-column window (lc = 128 at k <= 2 and batch <= 2, else 64, never
+more than the group) into two accumulators (lc/2 columns each, windows in turn), then
+adds the two and the warp adds 32 lanes in 5 butterfly steps, so no term
+passes through more than d = 64 ceil(cols/4096) + 8 roundings and
+|Y - exact| <= d * 2^-24 * sum_c |W~ a| (first order).  sum_c |W~ a| is
 bounded with the bf16 reconstruction: |W~| <= |bf16(W~)| (1 + 2^-8)."""
 import numpy as np
 import pytest
@@ -35,7 +35,7 @@ def lib():
 
 def _depth(cols):
     """Roundings a term of a row of `cols` columns passes through at most."""
-    return 32 * -(-cols // 2048) + 8
+    return 64 * -(-cols // 4096) + 8
 
 
 def _host_pkg(pkg, rows_idx=None):
@@ -176,6 +176,29 @@ def test_widths(batch, bits, group):
         tol = d * 2.0 ** -24 * (Af @ recf.T) * (1 + 2.0 ** -8) + 1e-30
         err = np.abs(Y.cpu().numpy().astype(np.float64) - want)
         assert not np.any(err > tol), f"{bits} g{group} B{batch} k{k}: {int((err > tol).sum())} outputs beyond the bound"
+
+
+def test_widest_rows_and_batch_split():
+    """The widest supported rows (RRQ_MAX_GEMV_COLS columns, one activation
+    row per launch's shared memory at most) and a batch of 8 at 28672 columns
+    (two activation rows per launch: four launches over the same package)."""
+    for rows, cols, batch in ((3, 57344, 1), (5, 28672, 8)):
+        W = workloads.generate(rows, cols, cols + batch, "t3_rowout", "cuda")
+        (pkg,) = binding.rrq_quantize_ex([W], 128, 4, binding.GRID_ASYM, binding.SCALE_F32)
+        A = _acts(batch, cols, seed=rows)
+        for k in (1, 4):
+            (Y,) = binding.rrq_gemv([pkg], [A], k)
+            _check(pkg, A, Y, k, where=f"{rows}x{cols} B{batch} k{k}")
+
+
+def test_too_wide():
+    cols = 57344 + 128
+    W = workloads.generate(1, cols, 9, "normal", "cuda")
+    pkg = binding.rrq_quantize(W, 128, 1)
+    A = _acts(1, cols, seed=3)
+    with pytest.raises(binding.RRQError) as e:
+        binding.rrq_gemv([pkg], [A], 1)
+    assert e.value.status == 2
 
 
 def test_errors():
