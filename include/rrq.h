@@ -323,10 +323,13 @@ typedef struct {
  * grid) are taken with the reconstruction's stage sum of that format.  Y must
  * not overlap any input or another Y.  The activation rows of a launch are
  * held in shared memory as binary32, padded to a multiple of 2048 columns:
- * a launch takes as many of the batch's rows as fit in 227 KiB, so the
- * widest matrix of a call may have at most RRQ_MAX_GEMV_COLS columns
- * (RRQ_ERR_UNSUPPORTED beyond).  One launch per 64 matrices and per such
- * share of the batch; other rules as for rrq_reconstruct_ex. */
+ * a launch takes as many of the batch's rows as fit in 227 KiB (at most 4
+ * at k = 4), so every
+ * matrix of a call may have at most RRQ_MAX_GEMV_COLS columns
+ * (RRQ_ERR_UNSUPPORTED beyond, before anything is launched).  Matrices
+ * that take the same number of rows per launch are launched together, up to
+ * 64 per launch, once per such share of the batch; other rules as for
+ * rrq_reconstruct_ex. */
 rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
                     rrq_stream_t stream);
 

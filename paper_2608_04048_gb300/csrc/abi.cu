@@ -450,18 +450,33 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
   DeviceState* st = nullptr;
   if (rrq_status rc = check_product_items(items, count, f, k, static_cast<uint64_t>(batch), &st)) return rc;
 
+  // activation rows one launch holds for each matrix (shared memory); the
+  // matrices that take the same number go together, so that a wide matrix
+  // does not split the batch of the narrower ones
+  std::vector<int> per(count), order(count);
+  for (int i = 0; i < count; ++i) {
+    const int cap = rrq::gemv_rows_per_launch(f.kind, k, items[i].cols);
+    if (cap < 1) return RRQ_ERR_UNSUPPORTED;
+    per[i] = std::min(cap, batch);
+    order[i] = i;
+  }
+  std::stable_sort(order.begin(), order.end(), [&](int a, int b) { return per[a] > per[b]; });
+
   int log2g = 0;
   while ((1 << log2g) < group) ++log2g;
   static thread_local rrq::GemvBatch p;
-  for (int base = 0; base < count; base += rrq::kMaxBatch) {
-    const int m = std::min(rrq::kMaxBatch, count - base);
+  for (int base = 0; base < count;) {
+    // up to kMaxBatch matrices with the same rows per launch
+    int m = 1;
+    while (m < rrq::kMaxBatch && base + m < count && per[order[base + m]] == per[order[base]]) ++m;
+    const int rows_per = per[order[base]];
     std::memset(&p, 0, sizeof p);
     p.count = m;
     p.log2g = log2g;
     for (int j = 0; j < rrq::kMaxStages; ++j) p.bits[j] = f.bits[j];
     int64_t blocks = 0, max_cols = 0;
     for (int i = 0; i < m; ++i) {
-      const rrq_gemv_desc& it = items[base + i];
+      const rrq_gemv_desc& it = items[order[base + i]];
       rrq::GemvItem& q = p.item[i];
       for (int j = 0; j < rrq::kMaxStages; ++j) {
         const int jj = j < k ? j : k - 1;
@@ -476,19 +491,17 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
       max_cols = std::max(max_cols, it.cols);
     }
     p.total_blocks = blocks;
-    // activation rows per launch: as many as shared memory holds
-    const int per = rrq::gemv_rows_per_launch(f.kind, k, max_cols);
-    if (per < 1) return RRQ_ERR_UNSUPPORTED;
-    for (int b0 = 0; b0 < batch; b0 += per) {
-      const int nb = std::min(per, batch - b0);
+    for (int b0 = 0; b0 < batch; b0 += rows_per) {
+      const int nb = std::min(rows_per, batch - b0);
       for (int i = 0; i < m; ++i) {
-        const rrq_gemv_desc& it = items[base + i];
+        const rrq_gemv_desc& it = items[order[base + i]];
         p.item[i].A = it.A_bf16 + static_cast<int64_t>(b0) * it.cols;
         p.item[i].Y = it.Y + static_cast<int64_t>(b0) * it.rows;
       }
       cudaError_t e = rrq::gemv_launch(f.kind, k, nb, max_cols, p, reinterpret_cast<cudaStream_t>(stream), st->sms);
       if (e != cudaSuccess) return fail_cuda(e);
     }
+    base += m;
   }
   return RRQ_OK;
 }

@@ -7,7 +7,7 @@ cudaError_t gemv_launch_asym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, 
   return launch_format<kAsymF32>(k, nb, max_cols, p, stream, sms);
 }
 
-// activation rows that fit in shared memory (the same for every format and k)
-int gemv_rows_per_launch(Format, int, int64_t max_cols) { return tokens_per_launch(max_cols); }
+// activation rows one launch takes (the same for every format)
+int gemv_rows_per_launch(Format, int k, int64_t max_cols) { return tokens_per_launch(max_cols, k); }
 
 }  // namespace rrq

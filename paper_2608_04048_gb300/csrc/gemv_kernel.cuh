@@ -115,7 +115,7 @@ __device__ __forceinline__ void cta_barrier() {
 }
 
 template <int F, int K, int B>
-__global__ void __launch_bounds__(kThreads, (K == 1 && B <= 2 && F != kAsymBits) ? 2 : 1)
+__global__ void __launch_bounds__(kThreads, (K == 1 && B == 1 && F != kAsymBits) ? 2 : 1)
 gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
@@ -388,9 +388,13 @@ constexpr int64_t act_floats_of(int64_t max_cols) {
 static_assert(act_floats_of(RRQ_MAX_GEMV_COLS) * 4 <= kMaxSmem &&
                   act_floats_of(RRQ_MAX_GEMV_COLS + 32) * 4 > kMaxSmem,
               "RRQ_MAX_GEMV_COLS is the widest row one activation row of a launch holds");
-inline int tokens_per_launch(int64_t max_cols) {
+// activation rows one launch takes: as many as shared memory holds, and at
+// most 4 at k = 4 (with 8 rows the k = 4 kernel runs out of registers; two
+// launches of 4 are faster)
+constexpr int max_rows_per_launch(int k) { return k == 4 ? 4 : kMaxGemvBatch; }
+inline int tokens_per_launch(int64_t max_cols, int k) {
   const int64_t t = kMaxSmem / (act_floats_of(max_cols) * 4);
-  return static_cast<int>(t < kMaxGemvBatch ? t : kMaxGemvBatch);
+  return static_cast<int>(t < max_rows_per_launch(k) ? t : max_rows_per_launch(k));
 }
 
 constexpr int kMaxDevices = 64;
@@ -430,10 +434,12 @@ cudaError_t launch_fkb(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stre
 
 template <int F, int K>
 cudaError_t launch_fk(int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms) {
+  if (nb > max_rows_per_launch(K)) return cudaErrorInvalidValue;
   if (nb <= 1) return launch_fkb<F, K, 1>(p, nb, max_cols, stream, sms);
   if (nb <= 2) return launch_fkb<F, K, 2>(p, nb, max_cols, stream, sms);
   if (nb <= 4) return launch_fkb<F, K, 4>(p, nb, max_cols, stream, sms);
-  return launch_fkb<F, K, 8>(p, nb, max_cols, stream, sms);
+  if constexpr (max_rows_per_launch(K) > 4) return launch_fkb<F, K, 8>(p, nb, max_cols, stream, sms);
+  return cudaErrorInvalidValue;
 }
 
 // Launch of one format (instantiated by one translation unit each).

@@ -191,6 +191,20 @@ def test_widest_rows_and_batch_split():
             _check(pkg, A, Y, k, where=f"{rows}x{cols} B{batch} k{k}")
 
 
+def test_mixed_widths_batch_8():
+    """One call at batch 8 over matrices that hold 8, 4, 2 and 1 activation
+    rows per launch (4096, 12288, 28672 and 57344 columns): each width class
+    is launched on its own share of the batch, in any order of the items."""
+    shapes = [(5, 28672), (7, 4096), (3, 57344), (17, 12288), (2, 4096)]
+    mats = [workloads.generate(r, c, 300 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+    pkgs = binding.rrq_quantize_ex(mats, 128, 2, binding.GRID_ASYM, binding.SCALE_F32)
+    acts = [_acts(8, c, seed=40 + i) for i, (r, c) in enumerate(shapes)]
+    for k in (1, 2):
+        ys = binding.rrq_gemv(pkgs, acts, k)
+        for i, (p, A, Y) in enumerate(zip(pkgs, acts, ys)):
+            _check(p, A, Y, k, where=f"item {i} {shapes[i]} k{k}")
+
+
 def test_too_wide():
     cols = 57344 + 128
     W = workloads.generate(1, cols, 9, "normal", "cuda")
