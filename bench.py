@@ -164,7 +164,8 @@ def time_gemv(pkgs, specs, stream, batch: int = 1, reps: int = 5) -> dict:
                   for sp in specs)
         out[f"k{k}"] = {"s_per_stack": round(t, 6), "alg_gbs": round(alg / t / 1e9, 1),
                         "frac_of_measured_hbm": round(alg / t / 1e9 / hbm, 4),
-                        "weights_per_s": round(sum(sp.numel for sp in specs) / t, 1)}
+                        "weights_per_s": round(sum(sp.numel for sp in specs) / t, 1),
+                        "weight_row_products_per_s": round(sum(sp.numel for sp in specs) * batch / t, 1)}
     return out
 
 
@@ -479,6 +480,9 @@ def run_gpu(args, world, rank, local) -> dict | None:
     sym = time_sym_f16(mats, p_outs, specs, stream) if not args.no_sym else None
     from_base = time_from_base(mats, pkgs, specs, stream) if not args.no_sym else None
     gemv = time_gemv(pkgs, specs, stream) if not args.no_sym else None
+    batches = [int(x) for x in args.gemv_batches.split(",") if x.strip()]
+    gemv_batches = {f"batch{b}": time_gemv(pkgs, specs, stream, batch=b) for b in batches if b != 1} \
+        if not args.no_sym and any(b != 1 for b in batches) else None
     prefill = time_prefill(pkgs, specs, stream) if not args.no_sym else None
     bits = {"+".join(map(str, b)): time_bits(mats, p_outs, specs, stream, b) for b in ((1, 3), (3, 1))} \
         if not args.no_sym else None
@@ -547,6 +551,7 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "sym_f16": sym,
             "from_base": from_base,
             "gemv_decode": gemv,
+            "gemv_decode_batches": gemv_batches,
             "prefill": prefill,
             "widths": bits,
             "group_pmr": pmr,
@@ -775,6 +780,8 @@ def main(argv=None):
     ap.add_argument("--no-sym", action="store_true",
                     help="skip the symmetric binary16, base-checkpoint and product breakdown")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--gemv-batches", default="1",
+                    help="comma-separated activation-row counts for the decode-product breakdown (1..8)")
     args = ap.parse_args(argv)
 
     world, rank, local = dist_env()
