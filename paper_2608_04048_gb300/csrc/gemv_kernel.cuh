@@ -270,23 +270,16 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
         for (int q = 0; q < 8; ++q) dot(8 * h + q, v[2 * q], v[2 * q + 1]);
       }
     } else {
-      // code j of a byte (bits 2j, 2j+1) left in place under the exponent of
-      // 2^(23-2j): t = 2^(23-2j) + Q exactly, and fma(t, s, -2^(23-2j) s)
-      // gives fl(Q s) with one rounding (2^(23-2j) s exact: prescale_ok)
-      f32x2 S[K], C01[K], C23[K], Z[K];
+      // the stage levels of each byte's four codes (asym_levels, sym_offsets)
+      StageConsts c[K];
       bool fast = true;
 #pragma unroll
       for (int i = 0; i < K; ++i) {
         const float s = kF16 ? __half2float(__ushort_as_half(static_cast<unsigned short>(w.s[i])))
                              : __uint_as_float(w.s[i]);
-        if (!kF16) fast = fast && prescale_ok(s);  // binary16 scales always are
-        S[i] = pack2(s, s);
-        C01[i] = mul2(S[i], pack2(-0x1p23f, -0x1p21f));
-        C23[i] = mul2(S[i], pack2(-0x1p19f, -0x1p17f));
-        Z[i] = kSym ? pack2(0.0f, 0.0f) : pack2(w.z[i], w.z[i]);
+        if (!kSym) fast = fast && prescale_ok(s);  // symmetric levels need no condition
+        c[i] = stage_consts(s, kSym ? 0.0f : w.z[i]);
       }
-      // symmetric levels: t - (2^(23-2j) + 2) = Q - 2 exactly
-      const f32x2 K01 = pack2(0x1p23f + 2.0f, 0x1p21f + 2.0f), K23 = pack2(0x1p19f + 2.0f, 0x1p17f + 2.0f);
 #pragma unroll
       for (int h = 0; h < kLCM / 32; ++h) {
         if (h >= nh) break;
@@ -299,24 +292,24 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
               const uint4 cw = w.code[i][h >> 1];
               const uint32_t word = (h & 1) == 0 ? (q < 4 ? cw.x : cw.y) : (q < 4 ? cw.z : cw.w);
               const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
-              const f32x2 t01 = pack2u(field_or<0x03u>(b8, 0x4B000000u), field_or<0x0Cu>(b8, 0x4A000000u));
-              const f32x2 t23 = pack2u(field_or<0x30u>(b8, 0x49000000u), field_or<0xC0u>(b8, 0x48000000u));
               if (kSym) {  // (Q - 2) s, exact; summed by one fma
-                const f32x2 u01 = sub2(t01, K01), u23 = sub2(t23, K23);
-                w01 = (i == 0) ? mul2(u01, S[i]) : fma2(u01, S[i], w01);
-                w23 = (i == 0) ? mul2(u23, S[i]) : fma2(u23, S[i], w23);
+                f32x2 u01, u23;
+                sym_offsets(b8, u01, u23);
+                w01 = (i == 0) ? mul2(u01, c[i].S) : fma2(u01, c[i].S, w01);
+                w23 = (i == 0) ? mul2(u23, c[i].S) : fma2(u23, c[i].S, w23);
               } else {     // fl(zero + fl(Q s))
-                const f32x2 l01 = add2(Z[i], fma2(t01, S[i], C01[i]));
-                const f32x2 l23 = add2(Z[i], fma2(t23, S[i], C23[i]));
+                f32x2 l01, l23;
+                asym_levels(b8, c[i], l01, l23);
                 w01 = (i == 0) ? l01 : add2(w01, l01);
                 w23 = (i == 0) ? l23 : add2(w23, l23);
               }
             }
             dot(8 * h + q, w01, w23);
           }
-        } else {
-          // a scale outside [2^-100, 2^100]: unscaled codes, plain (t - 2^23) s
-          const f32x2 T = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f), K2 = pack2(kTwo23 + 2.0f, kTwo23 + 2.0f);
+        } else if constexpr (!kSym) {
+          // an asymmetric scale outside [2^-100, 2^100]: unscaled codes,
+          // fl(Q s) as a plain (t - 2^23) s
+          const f32x2 T = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f);
 #pragma unroll
           for (int q = 0; q < 8; ++q) {
             f32x2 w01, w23;
@@ -327,16 +320,10 @@ gemv_kernel(const __grid_constant__ GemvBatch p, int nb, int act_floats) {
               const uint32_t b8 = (q & 3) == 0 ? word : (word >> (8 * (q & 3)));
               const f32x2 t01 = pack2u(magic23<3u>(b8), magic23<3u>(b8 >> 2));
               const f32x2 t23 = pack2u(magic23<3u>(b8 >> 4), magic23<3u>(b8 >> 6));
-              if (kSym) {
-                const f32x2 u01 = sub2(t01, K2), u23 = sub2(t23, K2);
-                w01 = (i == 0) ? mul2(u01, S[i]) : fma2(u01, S[i], w01);
-                w23 = (i == 0) ? mul2(u23, S[i]) : fma2(u23, S[i], w23);
-              } else {
-                const f32x2 l01 = add2(Z[i], fma2(sub2(t01, T), S[i], Z0));
-                const f32x2 l23 = add2(Z[i], fma2(sub2(t23, T), S[i], Z0));
-                w01 = (i == 0) ? l01 : add2(w01, l01);
-                w23 = (i == 0) ? l23 : add2(w23, l23);
-              }
+              const f32x2 l01 = add2(c[i].Z, fma2(sub2(t01, T), c[i].S, Z0));
+              const f32x2 l23 = add2(c[i].Z, fma2(sub2(t23, T), c[i].S, Z0));
+              w01 = (i == 0) ? l01 : add2(w01, l01);
+              w23 = (i == 0) ? l23 : add2(w23, l23);
             }
             dot(8 * h + q, w01, w23);
           }

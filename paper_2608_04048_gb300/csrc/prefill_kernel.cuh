@@ -264,6 +264,9 @@ __device__ __forceinline__ void load_scales(const PrefillItem& it, int64_t g, Pk
 // bits: with prescale_ok(s) each code stays in its bit field (value 4^j Q
 // for the j-th code of a byte) and one fma with s / 4^j and -2^23 s / 4^j
 // rounds Q s once; otherwise the code is shifted down and fma(Q, s, 0).
+// (The decode product and the reconstruction use the other placement of the
+// same trick, asym_levels: one exponent per code position and one scale.  In
+// this kernel the form here measured 1 % faster at k = 2..4.)
 template <int F, int K, int NW>
 __device__ __forceinline__ void prefix_weights_bf16(const PkgWords<K>& w, uint32_t (&h)[NW / 2]) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;

@@ -13,16 +13,16 @@
 // a chunk is staged in shared memory and written by a 1-D bulk copy (TMA
 // store), double-buffered per warp.
 //
-// fl(Q*s) is one fused multiply-add: with t the float whose bits are
-// 0x4B000000 | (Q << 2j), t = 2^23 + Q*4^j exactly, and
-// fma(t, s*4^-j, -2^23*s*4^-j) = RN(Q*s) because the scalings by powers of
-// two are exact for s in [2^-100, 2^100].  So four codes of one byte need one
-// shift and one logic operation each, no shift per code.  Groups with a scale
-// outside that range use the plain form RN((t - 2^23) * s).
+// fl(Q*s) is one fused multiply-add: code j of a byte stays in its bit field
+// under the exponent of 2^(23-2j), so that the float t = 2^(23-2j) + Q
+// exactly, and fma(t, s, -2^(23-2j) s) = RN(Q*s) because the scaling by a
+// power of two is exact for s in [2^-100, 2^100] (asym_levels).  So the four
+// codes of one byte need one shift per byte and one logic operation per code.
+// Groups with a scale outside that range use the plain form RN((t - 2^23) s).
 //
 // Symmetric grid (implicit zero-point 2): L_i = (Q_i - 2) * s_i, exact in
 // binary32, so acc + L_i is one fma(u, s, acc) with u = Q - 2 taken exactly
-// as t - (2^23 + 2*4^j) from the same prescaled t; the base stage is the
+// from the same t (sym_offsets), for every scale; the base stage is the
 // exact product u * s.  binary16 scales are read as the 4-byte word holding
 // the lane's scale and its neighbour's (the copy is cut to 2 bytes at the end
 // of an array with an odd number of groups) and widened exactly.
@@ -164,7 +164,7 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
         scale[i] = *reinterpret_cast<const float*>(buf + i * kStageBytes + kCB + lane * 4);
       }
       zero[i] = kSym ? 0.0f : *reinterpret_cast<const float*>(buf + i * kStageBytes + kCB + 128 + lane * 4);
-      ok = ok && prescale_ok(scale[i]);
+      ok = ok && (kSym || prescale_ok(scale[i]));  // symmetric levels need no condition
     }
 
     const bool all_ok = __all_sync(kFullMask, ok);
@@ -215,46 +215,25 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
           default: dequant_bits<2>(w4, scale[i], zero[i], i == 0, acc); break;
         }
       } else if (kSym) {
-        // u = Q - 2 (times 4^j in the prescaled form), exact; L = u * s exact
-        const float s = scale[i];
-        if (all_ok) {
-          const f32x2 S01 = pack2(s, __fmul_rn(s, 0x1p-2f));
-          const f32x2 S23 = pack2(__fmul_rn(s, 0x1p-4f), __fmul_rn(s, 0x1p-6f));
-          const f32x2 K01 = pack2(kTwo23 + 2.0f, kTwo23 + 8.0f);
-          const f32x2 K23 = pack2(kTwo23 + 32.0f, kTwo23 + 128.0f);
+        // u = Q - 2 and L = u s, both exact (sym_offsets)
+        const f32x2 S = pack2(scale[i], scale[i]);
 #pragma unroll
-          for (int j = 0; j < 8; ++j) {
-            const uint32_t word = j < 4 ? w0 : w1;
-            const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-            const f32x2 u01 = sub2(pack2u(magic23<0x03u>(b), magic23<0x0Cu>(b)), K01);
-            const f32x2 u23 = sub2(pack2u(magic23<0x30u>(b), magic23<0xC0u>(b)), K23);
-            acc[2 * j] = (i == 0) ? mul2(u01, S01) : fma2(u01, S01, acc[2 * j]);
-            acc[2 * j + 1] = (i == 0) ? mul2(u23, S23) : fma2(u23, S23, acc[2 * j + 1]);
-          }
-        } else {
-          const f32x2 K2 = pack2(kTwo23 + 2.0f, kTwo23 + 2.0f), S = pack2(s, s);
-#pragma unroll
-          for (int m = 0; m < 16; ++m) {
-            const uint32_t word = m < 8 ? w0 : w1;
-            const int sh = 4 * (m & 7);
-            const f32x2 u = sub2(pack2u(magic23<3u>(word >> sh), magic23<3u>(word >> (sh + 2))), K2);
-            acc[m] = (i == 0) ? mul2(u, S) : fma2(u, S, acc[m]);
-          }
+        for (int j = 0; j < 8; ++j) {
+          const uint32_t word = j < 4 ? w0 : w1;
+          const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
+          f32x2 u01, u23;
+          sym_offsets(b, u01, u23);
+          acc[2 * j] = (i == 0) ? mul2(u01, S) : fma2(u01, S, acc[2 * j]);
+          acc[2 * j + 1] = (i == 0) ? mul2(u23, S) : fma2(u23, S, acc[2 * j + 1]);
         }
       } else if (all_ok) {
-        const float s = scale[i];
-        const f32x2 S01 = pack2(s, __fmul_rn(s, 0x1p-2f));
-        const f32x2 S23 = pack2(__fmul_rn(s, 0x1p-4f), __fmul_rn(s, 0x1p-6f));
-        const f32x2 C01 = pack2(__fmul_rn(s, -0x1p23f), __fmul_rn(s, -0x1p21f));
-        const f32x2 C23 = pack2(__fmul_rn(s, -0x1p19f), __fmul_rn(s, -0x1p17f));
+        const StageConsts c = stage_consts(scale[i], zero[i]);
 #pragma unroll
         for (int j = 0; j < 8; ++j) {  // byte j: elements 4j..4j+3 (pairs 2j, 2j+1)
           const uint32_t word = j < 4 ? w0 : w1;
           const uint32_t b = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-          const f32x2 t01 = pack2u(magic23<0x03u>(b), magic23<0x0Cu>(b));
-          const f32x2 t23 = pack2u(magic23<0x30u>(b), magic23<0xC0u>(b));
-          const f32x2 l01 = add2(LO, fma2(t01, S01, C01));
-          const f32x2 l23 = add2(LO, fma2(t23, S23, C23));
+          f32x2 l01, l23;
+          asym_levels(b, c, l01, l23);
           acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
           acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
         }

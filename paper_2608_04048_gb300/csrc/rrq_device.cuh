@@ -214,11 +214,50 @@ __device__ __forceinline__ void dequant_bits(const uint4& w4, float s, float z, 
   }
 }
 
-// A scale for which s/4, s/16, s/64 and s * 2^23 are exact binary32 values,
-// so that a code left in its bit field (value 4^j Q) times s / 4^j, minus
-// 2^23 s / 4^j, gives Q s with a single rounding inside one fma.
+// A scale for which 2^17 s .. 2^23 s (and s / 64) are exact binary32
+// values, so that a code left in its bit field gives Q s with a single
+// rounding inside one fma (see asym_levels; a conservative range).
 __device__ __forceinline__ bool prescale_ok(float s) {
   return s == 0.0f || (s >= 0x1p-100f && s <= 0x1p+100f);
+}
+
+// ---------------------------------------------------------------------------
+// stage levels of 2-bit codes, four to a byte (code j at bits 2j, 2j+1)
+// ---------------------------------------------------------------------------
+// Code j stays in place under the float exponent of 2^(23-2j), so that
+// t_j = 2^(23-2j) + Q exactly (one logic op).  Asymmetric level
+// fl(zero + fl(Q s)): fma(t_j, s, -2^(23-2j) s) rounds Q s once when
+// 2^(23-2j) s is exact (prescale_ok(s)), then one add.  Symmetric level
+// (Q - 2) s: t_j - (2^(23-2j) + 2) = Q - 2 exactly, and its product with s is
+// exact (or overflows exactly as the definition's does) for every s.
+struct StageConsts {
+  f32x2 S;    // (s, s)
+  f32x2 C01;  // (-2^23 s, -2^21 s)
+  f32x2 C23;  // (-2^19 s, -2^17 s)
+  f32x2 Z;    // (zero, zero)
+};
+
+__device__ __forceinline__ StageConsts stage_consts(float s, float zero) {
+  const f32x2 S = pack2(s, s);
+  return {S, mul2(S, pack2(-0x1p23f, -0x1p21f)), mul2(S, pack2(-0x1p19f, -0x1p17f)), pack2(zero, zero)};
+}
+// (t_0, t_1) and (t_2, t_3) of byte b
+__device__ __forceinline__ f32x2 code_t01(uint32_t b) {
+  return pack2u(field_or<0x03u>(b, 0x4B000000u), field_or<0x0Cu>(b, 0x4A000000u));
+}
+__device__ __forceinline__ f32x2 code_t23(uint32_t b) {
+  return pack2u(field_or<0x30u>(b, 0x49000000u), field_or<0xC0u>(b, 0x48000000u));
+}
+// asymmetric levels fl(zero + fl(Q s)) of codes 0,1 and 2,3 of byte b
+// (prescale_ok(s) required)
+__device__ __forceinline__ void asym_levels(uint32_t b, const StageConsts& c, f32x2& l01, f32x2& l23) {
+  l01 = add2(c.Z, fma2(code_t01(b), c.S, c.C01));
+  l23 = add2(c.Z, fma2(code_t23(b), c.S, c.C23));
+}
+// Q - 2 of codes 0,1 and 2,3 of byte b (exact)
+__device__ __forceinline__ void sym_offsets(uint32_t b, f32x2& u01, f32x2& u23) {
+  u01 = sub2(code_t01(b), pack2(0x1p23f + 2.0f, 0x1p21f + 2.0f));
+  u23 = sub2(code_t23(b), pack2(0x1p19f + 2.0f, 0x1p17f + 2.0f));
 }
 
 // min and max over 16 packed pairs (32 values) held by one lane
