@@ -57,6 +57,7 @@ class GemvDesc(ctypes.Structure):
 
 
 MAX_GEMV_BATCH = 8
+MAX_GEMV_COLS = 57344   # widest matrix rrq_gemv takes (RRQ_MAX_GEMV_COLS)
 
 
 class PmrDesc(ctypes.Structure):
@@ -478,7 +479,8 @@ def gemv_descs(pkgs, acts, ys, k) -> ctypes.Array:
 
 def rrq_gemv(pkgs, acts, k: int, ys=None, stream=None, items=None):
     """Y_i = A_i W~_i^T for each package i at prefix k (Appendix C), A_i bf16
-    [batch, cols] with 1 <= batch <= 8; returns float32 [batch, rows] each."""
+    [batch, cols] with 1 <= batch <= 8 and cols <= MAX_GEMV_COLS; returns
+    float32 [batch, rows] each."""
     lib = load_library()
     batch = acts[0].shape[0]
     if any(not 1 <= k <= p.n_stages for p in pkgs):

@@ -30,6 +30,13 @@ def test_header_declares_the_boundary():
     assert set(names) == set(binding.EXPORTS)
 
 
+def test_binding_limits_match_the_header():
+    defines = dict(re.findall(r"#define\s+(RRQ_[A-Z_0-9]+)\s+\(?([0-9]+)", open(HEADER).read()))
+    assert int(defines["RRQ_MAX_STAGES"]) == binding.MAX_STAGES
+    assert int(defines["RRQ_MAX_GEMV_BATCH"]) == binding.MAX_GEMV_BATCH
+    assert int(defines["RRQ_MAX_GEMV_COLS"]) == binding.MAX_GEMV_COLS
+
+
 def test_every_declared_symbol_is_exported(lib):
     for name in declared_functions():
         assert hasattr(lib, name), name
