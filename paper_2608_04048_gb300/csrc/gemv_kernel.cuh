@@ -14,9 +14,9 @@
 // the multiprocessors) with equal shares of rows x columns, so that a CTA
 // meets few matrices.  The CTA's 16 warps take one row of each block each.
 // A warp walks its row in windows of 32 x lc columns, lane l owning the lc
-// columns lc*l .. lc*l + lc-1 of the window: lc = 128 for k <= 2 and up to
-// 2 activation rows (64 otherwise, where registers are scarcer), never more
-// than the group, so that a lane's columns share one group (the row length
+// columns lc*l .. lc*l + lc-1 of the window: lc = 128 at k = 1, and at k = 2
+// with up to 2 activation rows (64 otherwise, where registers are scarcer),
+// never more than the group, so that a lane's columns share one group (the row length
 // is a multiple of the group, so a lane's columns are all in the row or all
 // past its end).  Per stage the lane loads lc/4 bytes of codes (16-byte
 // loads; 8 bytes for 32 columns) and one scale and zero, all into registers
@@ -57,11 +57,13 @@ constexpr int kRows = kGemvRows;       // rows per block (one per warp)
 static_assert(kRows == kWarps, "one row of a block per warp");
 constexpr int kWinCols = 4096;         // columns of the widest warp window (activation padding)
 
-// Columns a lane owns in a window at most: 128 at k <= 2 with 1 or 2
-// activation rows (more weights per window's fixed cost), else 64
+// Columns a lane owns in a window at most: 128 at k = 1, and at k = 2 with 1
+// or 2 activation rows (more weights per window's fixed cost), else 64
 // (registers).
 template <int F, int K, int B>
-__host__ __device__ constexpr int lane_cols_max() { return (F != kAsymBits && K <= 2 && B <= 2) ? 128 : 64; }
+__host__ __device__ constexpr int lane_cols_max() {
+  return (F != kAsymBits && (K == 1 || (K == 2 && B <= 2))) ? 128 : 64;
+}
 constexpr int kMaxSmem = 227 * 1024;
 constexpr float kTwo23 = 8388608.0f;
 

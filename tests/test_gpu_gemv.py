@@ -4,8 +4,8 @@ product of the same binary32 prefix weights.
 
 Tolerance, from the kernel's arithmetic: every product W~ a is exact inside
 its fma and every partial sum is rounded once; a lane sums its lc columns of
-each 32 lc-column window (lc = 128 at k <= 2 and batch <= 2, else 64, never
-more than the group) into two accumulators (lc/2 columns each, windows in turn), then
+each 32 lc-column window (lc = 128 at k = 1 and at k = 2 with batch <= 2,
+else 64, never more than the group) into two accumulators (lc/2 columns each, windows in turn), then
 adds the two and the warp adds 32 lanes in 5 butterfly steps, so no term
 passes through more than d = 64 ceil(cols/4096) + 8 roundings and
 |Y - exact| <= d * 2^-24 * sum_c |W~ a| (first order).  sum_c |W~ a| is
