@@ -148,3 +148,24 @@ def check_sampled_sym(W: torch.Tensor, pkg, idx: np.ndarray, outs=None, where=""
         got = bf16_bits(o.reshape(-1, g).index_select(0, it))
         want = oracle.reconstruct_sym(rc, rs, idx.size, g, g, j + 1, f16)
         _cmp_bytes(got, want, f"{where} sampled prefix {j + 1}")
+
+
+SENTINEL = 0x7FA5A5A5  # a NaN pattern no kernel writes
+
+
+def guarded_outputs(shapes, batch, guard=1024):
+    """float32 [batch, rows] outputs, each inside a buffer with `guard`
+    sentinel floats (4 KiB) on both sides; 16-byte aligned."""
+    bufs, ys = [], []
+    for rows, _cols in shapes:
+        buf = torch.empty((batch * rows + 2 * guard,), dtype=torch.float32, device="cuda")
+        buf.view(torch.int32).fill_(SENTINEL)
+        bufs.append(buf)
+        ys.append(buf[guard:guard + batch * rows].view(batch, rows))
+    return bufs, ys, guard
+
+
+def bands_intact(bufs, guard) -> bool:
+    torch.cuda.synchronize()
+    return all(bool((b.view(torch.int32)[:guard] == SENTINEL).all()) and
+               bool((b.view(torch.int32)[-guard:] == SENTINEL).all()) for b in bufs)

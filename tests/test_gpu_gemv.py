@@ -16,7 +16,7 @@ import torch
 
 import oracle
 from paper_2608_04048_gb300 import binding, build, workloads
-from gpu_helpers import bf16_bits
+from gpu_helpers import bands_intact, bf16_bits, guarded_outputs
 
 pytestmark = pytest.mark.gpu
 
@@ -229,3 +229,21 @@ def test_errors():
     with pytest.raises(binding.RRQError) as e:
         binding.rrq_gemv([pkg], [A2], 1, ys=[Yover])
     assert e.value.status == 1
+
+
+def test_guard_bands_untouched():
+    """Outputs inside 4 KiB sentinel bands: ragged shapes (rows not a
+    multiple of 16, a group of 32, a partial window) at batches 1 and 3 and
+    every k write inside their [batch, rows] only."""
+    shapes = [(45, 384), (3, 4096 + 128), (17, 1152)]
+    mats = [workloads.generate(r, c, 500 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+    for group in (32, 128):
+        pkgs = [binding.rrq_quantize_ex([W], group, 4, binding.GRID_ASYM, binding.SCALE_F32)[0] for W in mats]
+        for batch in (1, 3):
+            acts = [_acts(batch, c, seed=60 + i) for i, (r, c) in enumerate(shapes)]
+            for k in (1, 4):
+                bufs, ys, guard = guarded_outputs(shapes, batch)
+                binding.rrq_gemv(pkgs, acts, k, ys)
+                assert bands_intact(bufs, guard), f"g{group} batch {batch} k {k}: a sentinel band changed"
+                for i, (p, A, Y) in enumerate(zip(pkgs, acts, ys)):
+                    _check(p, A, Y, k, where=f"guarded item {i} g{group} B{batch} k{k}")

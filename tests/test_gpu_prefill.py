@@ -17,7 +17,7 @@ import torch
 
 import oracle
 from paper_2608_04048_gb300 import binding, build, workloads
-from gpu_helpers import bf16_bits
+from gpu_helpers import bands_intact, bf16_bits, guarded_outputs
 
 pytestmark = pytest.mark.gpu
 
@@ -284,3 +284,19 @@ def test_bounded_waits_report_timeout():
     (Y,) = binding.rrq_prefill([pkg], [A], 4)
     _check(pkg, A, Y, 4, where="after timeout")
     _status_ok()
+
+
+def test_guard_bands_untouched():
+    """Outputs inside 4 KiB sentinel bands: a ragged row tile, a ragged token
+    tile and a half stage, at k = 1 and 4 (one and four-CTA clusters)."""
+    shapes = [(45, 288), (130, 4096 + 128)]
+    mats = [workloads.generate(r, c, 700 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+    pkgs = [binding.rrq_quantize_ex([W], 32, 4, binding.GRID_ASYM, binding.SCALE_F32)[0] for W in mats]
+    tokens = 1100
+    acts = [_acts(tokens, c, seed=80 + i) for i, (r, c) in enumerate(shapes)]
+    for k in (1, 4):
+        bufs, ys, guard = guarded_outputs(shapes, tokens)
+        binding.rrq_prefill(pkgs, acts, k, ys)
+        assert bands_intact(bufs, guard), f"k {k}: a sentinel band changed"
+        for i, (p, A, Y) in enumerate(zip(pkgs, acts, ys)):
+            _check(p, A, Y, k, where=f"guarded item {i} k{k}")
