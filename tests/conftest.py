@@ -27,3 +27,14 @@ def pytest_collection_modifyitems(config, items):
     for item in items:
         if "gpu" in item.keywords:
             item.add_marker(skip)
+
+
+def pytest_terminal_summary(terminalreporter, exitstatus, config):
+    """Whole-workload parity checks report their size, wall time and the
+    host cores the oracle ran on."""
+    mod = sys.modules.get("full_parity")
+    lines = getattr(mod, "REPORT", None) if mod else None
+    if lines:
+        terminalreporter.section("whole-workload parity against the oracle")
+        for line in lines:
+            terminalreporter.write_line(line)

@@ -1,8 +1,9 @@
 """GPU parity for the build with prefixes (rrq_quantize_prefixes: Algorithm 1
-and Eq. 8 at every prefix in one pass): for every format the package equals
-rrq_quantize_ex's and every bf16 prefix equals rrq_reconstruct_ex's on it, bit
-for bit (both of which the other parity tests tie to the CPU oracle), and a
-direct comparison with the oracle."""
+and Eq. 8 at every prefix in one pass): for every format and group size the
+package and every bf16 prefix equal the CPU oracle's on ragged shapes, bit for
+bit; and they equal rrq_quantize_ex's package and rrq_reconstruct_ex's
+prefixes on it (the two-call path).  The whole-workload checks of the same
+call are in test_gpu_full_size.py."""
 import numpy as np
 import pytest
 import torch
@@ -79,6 +80,47 @@ def test_edge_groups_and_forced_exact(group):
             check([Wf], group, 4, fmt, where=f"forced exact g{group} {fmt}")
     finally:
         binding.rrq_set_debug_flags(0)
+
+
+def _oracle_package(W, group, S, fmt):
+    """(codes, scales as stored, zeros or None) and the prefixes 1..S."""
+    bits = bf16_bits(W)
+    rows, cols = W.shape
+    if fmt[0] == binding.GRID_ASYM:
+        codes, scales, zeros = oracle.quantize(bits, group, S)
+        pre = [oracle.reconstruct(codes, scales, zeros, rows, cols, group, k) for k in range(1, S + 1)]
+    else:
+        f16 = fmt[1] == binding.SCALE_F16
+        codes, scales = oracle.quantize_sym(bits, group, S, f16)
+        zeros = None
+        pre = [oracle.reconstruct_sym(codes, scales, rows, cols, group, k, f16) for k in range(1, S + 1)]
+    return codes, scales, zeros, pre
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FMT_IDS)
+@pytest.mark.parametrize("group", GROUPS)
+def test_each_format_against_the_oracle(group, fmt):
+    """Every output of rrq_quantize_prefixes against the oracle directly:
+    ragged shapes (a single group, chunk tails that end mid-warp, a matrix of
+    many chunks), heavy tails and outliers, 4 and 3 stages."""
+    shapes = [(1, group), (7, 3 * group), (33, 5 * group), (130, 2 * group), (5, 4096 // group * group)]
+    for S in (4, 3):
+        mats = [workloads.generate(r, c, 70 + 3 * i + S, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
+        pkgs, outs = binding.rrq_quantize_prefixes(mats, group, S, *fmt)
+        torch.cuda.synchronize()
+        assert binding.rrq_get_device_status() == 0
+        for i, (W, p) in enumerate(zip(mats, pkgs)):
+            codes, scales, zeros, pre = _oracle_package(W, group, S, fmt)
+            where = f"g{group} S{S} {shapes[i]}"
+            for k in range(S):
+                assert np.array_equal(p.codes[k].cpu().numpy(), codes[k]), f"{where} stage {k} codes"
+                got = p.scales[k].cpu().numpy()
+                assert np.array_equal(got.view(np.uint8), np.ascontiguousarray(scales[k]).view(np.uint8)), \
+                    f"{where} stage {k} scales"
+                if zeros is not None:
+                    assert np.array_equal(p.zeros[k].cpu().numpy().view(np.uint32), zeros[k].view(np.uint32)), \
+                        f"{where} stage {k} zeros"
+                assert np.array_equal(bf16_bits(outs[i][k]), pre[k]), f"{where} prefix {k + 1}"
 
 
 def test_against_oracle_and_across_launches():
