@@ -1,23 +1,33 @@
-"""Benchmark of the RRQ hot path on GB300: package construction (rrq_quantize)
-and prefix reconstruction (rrq_reconstruct, k = 1..4) over a synthetic
-Qwen3-8B-shaped linear stack (36 layers x {q,k,v,o,gate,up,down}, 6.95e9
-bf16 weights, Student-t(3) weights with 0.1% +-20 sigma outliers per row,
-group 128, four 2-bit stages).
+"""Benchmark of the RRQ hot path on GB300: package construction (Algorithm 1)
+and prefix reconstruction (Eq. 8, k = 1..4) over synthetic weight stacks
+shaped like the paper's models.
 
-One step = rrq_quantize of every matrix of the stack, then rrq_reconstruct of
-every matrix at k = 1, 2, 3, 4.  The metric is bf16 weight bytes of the stack
-processed per second of step time (GB/s).  Inputs (13.9 GB) are far larger
-than L2, so no L2 flush is needed between steps.
+Default workload: a Qwen3-8B-shaped linear stack (36 layers x {q,k,v,o,gate,
+up,down}, 6.95e9 bf16 weights, Student-t(3) weights with 0.1% +-20 sigma
+outliers per row, group 128, four 2-bit stages).  Other workloads
+(--workload): single_4096, qwen3_8b_layer, sweep_8192 (four distributions x
+groups 32/64/128/256) and qwen3_32b_stack.
 
-    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+One step = rrq_quantize_prefixes over every matrix of the workload: the
+package and the bf16 reconstructions at k = 1, 2, 3, 4 of every matrix, from
+one read of W.  The metric is bf16 weight bytes processed per second of step
+time (GB/s).  The stacks' inputs are far larger than L2; the smaller
+workloads flush L2 before every timed call.  The breakdown times the package
+alone (rrq_quantize), every prefix from the package and each prefix by its
+own call, with a roofline entry for each.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
+                    [--split] [--impl reference]
 
 Under torchrun every rank builds and processes its own stack (independent
 matrices, no data-path collective): weak scaling, value = all ranks' bytes /
-max over ranks of the timed region.  Rank 0 prints one JSON line.
+max over ranks of the timed region.  With --split the ranks share ONE stack,
+each taking a disjoint set of its matrices (strong scaling).  Rank 0 prints
+one JSON line.
 
 --impl reference times the CPU oracle (the plain C implementation in oracle/,
-as it stands, single-threaded) on a bounded sample of the same workload; it is
-the slow reference arm, not a target.
+as it stands, in one process per host core over row ranges) on a bounded
+sample of the same workload; it is the slow reference arm, not a target.
 """
 from __future__ import annotations
 
@@ -379,14 +389,168 @@ def barrier(world: int):
 # ---------------------------------------------------------------------------
 # the GPU arm
 # ---------------------------------------------------------------------------
-def build_stack(specs, device, seed_offset: int):
-    from paper_2608_04048_gb300 import binding, workloads
-    mats, pkgs = [], []
-    for sp in specs:
-        W = workloads.generate(sp.rows, sp.cols, sp.seed + seed_offset, sp.dist, device)
-        mats.append(W)
-        pkgs.append(binding.Package.empty(sp.rows, sp.cols, GROUP, STAGES, device))
-    return mats, pkgs
+L2_BYTES = 126 * 2**20
+FLUSH_WORKLOADS = ("single_4096", "qwen3_8b_layer", "sweep_8192")   # inputs near or below L2
+
+
+def shard_matrices(specs, world: int, rank: int) -> list:
+    """Indices of the matrices rank `rank` takes when one stack is split over
+    `world` ranks: largest first, each to the rank with the fewest weights so
+    far (ties to the lower rank); every matrix goes to exactly one rank."""
+    load = [0] * world
+    owner = {}
+    for i in sorted(range(len(specs)), key=lambda i: (-specs[i].numel, i)):
+        r = min(range(world), key=lambda j: (load[j], j))
+        owner[i] = r
+        load[r] += specs[i].numel
+    return [i for i in range(len(specs)) if owner[i] == rank]
+
+
+class L2Flush:
+    """Writes a buffer twice the size of L2 (between timed calls of
+    workloads whose inputs would otherwise stay resident)."""
+
+    def __init__(self, device):
+        self.buf = torch.empty(2 * L2_BYTES // 4, dtype=torch.int32, device=device)
+        self.n = 0
+
+    def __call__(self):
+        self.n += 1
+        self.buf.fill_(self.n)
+
+
+def time_calls(calls, stream, reps: int, flush=None) -> float:
+    """Mean seconds of one pass over `calls` (after one untimed pass).
+    With `flush`, L2 is flushed before every call and only the calls are
+    timed (CUDA events around each); otherwise one event pair brackets the
+    passes."""
+    for c in calls:
+        c()
+    if flush is None:
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        for _ in range(reps):
+            for c in calls:
+                c()
+        b.record(stream)
+        torch.cuda.synchronize()
+        return a.elapsed_time(b) / reps / 1e3
+    evs = []
+    for _ in range(reps):
+        for c in calls:
+            flush()
+            a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            a.record(stream)
+            c()
+            b.record(stream)
+            evs.append((a, b))
+    torch.cuda.synchronize()
+    return sum(a.elapsed_time(b) for a, b in evs) / reps / 1e3
+
+
+class Workload:
+    """The device side of one named workload: inputs, packages, prefix
+    outputs, and the calls that make up a step and its breakdown parts.
+
+    The calls group matrices that share a group size.  If every matrix's
+    four bf16 prefixes fit in HBM beside the stack they get their own
+    outputs; otherwise (the Qwen3-32B-shaped stack) the matrices go in
+    layers of 7 that write their prefixes into one set of buffers, reused
+    by every layer."""
+
+    def __init__(self, specs, device, seed_offset: int, stream):
+        from paper_2608_04048_gb300 import binding, workloads
+        self.specs, self.stream, self.device = specs, stream, device
+        self.n_total = sum(sp.numel for sp in specs)
+        cache = {}
+        self.mats = []
+        for sp in specs:  # the sweep's group sizes share one input per distribution
+            key = (sp.rows, sp.cols, sp.seed, sp.dist)
+            if key not in cache:
+                cache[key] = workloads.generate(sp.rows, sp.cols, sp.seed + seed_offset, sp.dist, device)
+            self.mats.append(cache[key])
+        self.pkgs = [binding.Package.empty(sp.rows, sp.cols, sp.group, STAGES, device) for sp in specs]
+        pkg_bytes = sum(p.nbytes() for p in self.pkgs)
+        free, _ = torch.cuda.mem_get_info(device)
+        own = len(KS) * 2 * self.n_total
+        self.own_outputs = own + 4 * 2**30 < free
+        # units: matrices that go together in one call (same group; a layer
+        # of 7 when the outputs are shared)
+        per = None if self.own_outputs else 7
+        self.units = []
+        for g in sorted({sp.group for sp in specs}):
+            idx = [i for i, sp in enumerate(specs) if sp.group == g]
+            if per is None:
+                self.units.append(idx)
+            else:
+                self.units += [idx[i:i + per] for i in range(0, len(idx), per)]
+        if self.own_outputs:
+            self.p_outs = [[torch.empty((sp.rows, sp.cols), dtype=torch.bfloat16, device=device) for _ in KS]
+                           for sp in specs]
+        else:
+            shared = [[torch.empty((specs[i].rows, specs[i].cols), dtype=torch.bfloat16, device=device) for _ in KS]
+                      for i in self.units[0]]
+            self.p_outs = [shared[j % len(shared)] for j in range(len(specs))]
+            for u in self.units:
+                assert all((specs[i].rows, specs[i].cols) == (specs[self.units[0][j]].rows,
+                                                              specs[self.units[0][j]].cols)
+                           for j, i in enumerate(u))
+        self.pkg_bytes = pkg_bytes
+
+    def group_of(self, unit) -> int:
+        return self.specs[unit[0]].group
+
+    def step_calls(self):
+        """rrq_quantize_prefixes per unit: the package and every prefix."""
+        from paper_2608_04048_gb300 import binding
+        calls = []
+        for u in self.units:
+            mats, pkgs, outs = [self.mats[i] for i in u], [self.pkgs[i] for i in u], [self.p_outs[i] for i in u]
+            items = binding.quantize_prefixes_descs(mats, pkgs, outs)
+            g = self.group_of(u)
+            calls.append(lambda mats=mats, pkgs=pkgs, outs=outs, items=items, g=g: binding.rrq_quantize_prefixes(
+                mats, g, STAGES, binding.GRID_ASYM, binding.SCALE_F32, pkgs, outs, self.stream, items))
+        return calls
+
+    def quantize_calls(self):
+        """rrq_quantize_batch per group size (the package only, Algorithm 1)."""
+        from paper_2608_04048_gb300 import binding
+        calls = []
+        for g in sorted({sp.group for sp in self.specs}):
+            idx = [i for i, sp in enumerate(self.specs) if sp.group == g]
+            mats, pkgs = [self.mats[i] for i in idx], [self.pkgs[i] for i in idx]
+            items = binding.quantize_items(mats, pkgs)
+            calls.append(lambda mats=mats, pkgs=pkgs, items=items, g=g: binding.rrq_quantize_batch(
+                mats, pkgs, g, STAGES, stream=self.stream, items=items))
+        return calls
+
+    def reconstruct_calls(self, k: int | None):
+        """rrq_reconstruct_batch at prefix k (k given) or
+        rrq_reconstruct_prefixes_batch of every prefix (k None), per unit."""
+        from paper_2608_04048_gb300 import binding
+        calls = []
+        for u in self.units:
+            pkgs, outs = [self.pkgs[i] for i in u], [self.p_outs[i] for i in u]
+            if k is None:
+                items = binding.prefixes_items(pkgs, outs, len(KS))
+                calls.append(lambda pkgs=pkgs, outs=outs, items=items: binding.rrq_reconstruct_prefixes_batch(
+                    pkgs, len(KS), outs, stream=self.stream, items=items))
+            else:
+                one = [o[k - 1] for o in outs]
+                items = binding.reconstruct_items(pkgs, one)
+                calls.append(lambda pkgs=pkgs, one=one, items=items, k=k: binding.rrq_reconstruct_batch(
+                    pkgs, k, one, stream=self.stream, items=items))
+        return calls
+
+
+def roofline_entry(kernel: str, alg_bytes: float, seconds: float, peak: float, launches: int,
+                   traffic_key: str | None) -> dict:
+    achieved = alg_bytes / seconds / 1e9
+    traffic = recorded_traffic(traffic_key, alg_bytes / launches, alg_bytes / launches) if traffic_key else None
+    return {"kernel": kernel, "bound": "hbm", "achieved": round(achieved, 1), "peak": peak, "unit": "GB/s",
+            "frac": round(achieved / peak, 4), "frac_of_nominal_8tbs": round(achieved / 8000.0, 4),
+            "alg_bytes_per_launch": round(alg_bytes / launches), "s_per_pass": round(seconds, 6),
+            "traffic": traffic}
 
 
 def run_gpu(args, world, rank, local) -> dict | None:
@@ -394,38 +558,25 @@ def run_gpu(args, world, rank, local) -> dict | None:
     build.build()
     torch.cuda.set_device(local)
     device = torch.device("cuda", local)
-    specs = workloads.config_matrices(args.workload)
-    n_total = sum(sp.numel for sp in specs)
-    mats, pkgs = build_stack(specs, device, shard_seed_offset(rank))
-    # one bf16 output per matrix (13.9 GB): a batch may not write overlapping outputs
-    outs = [torch.empty((sp.rows, sp.cols), dtype=torch.bfloat16, device=device) for sp in specs]
+    specs_all = workloads.config_matrices(args.workload)
+    if args.split:  # one stack over all ranks (strong scaling)
+        specs = [specs_all[i] for i in shard_matrices(specs_all, world, rank)]
+        seed_offset = 0
+    else:           # a stack per rank (weak scaling)
+        specs = specs_all
+        seed_offset = shard_seed_offset(rank)
     stream = torch.cuda.current_stream(device)
     binding.rrq_get_device_status()
-
-    # one bf16 output per matrix and prefix (4 x 13.9 GB)
-    p_outs = [[torch.empty((sp.rows, sp.cols), dtype=torch.bfloat16, device=device) for _ in KS]
-              for sp in specs]
-    q_items = binding.quantize_items(mats, pkgs)
-    r_items = binding.reconstruct_items(pkgs, outs)
-    p_items = binding.prefixes_items(pkgs, p_outs, len(KS))
-
-    def quantize_all():
-        binding.rrq_quantize_batch(mats, pkgs, GROUP, STAGES, stream=stream, items=q_items)
-
-    def reconstruct_all():
-        # every prefix k = 1..4 of every matrix in one pass over the package
-        binding.rrq_reconstruct_prefixes_batch(pkgs, len(KS), p_outs, stream=stream, items=p_items)
-
-    def reconstruct_each_k():
-        for k in KS:
-            binding.rrq_reconstruct_batch(pkgs, k, outs, stream=stream, items=r_items)
-
-    f_items = binding.quantize_prefixes_descs(mats, pkgs, p_outs)
+    wl = Workload(specs, device, seed_offset, stream)
+    n_total = wl.n_total
+    flush = L2Flush(device) if args.workload in FLUSH_WORKLOADS else None
+    steps_calls = wl.step_calls()
 
     def step():
-        # the package and its 2/4/6/8-bit reconstructions in one pass over W
-        binding.rrq_quantize_prefixes(mats, GROUP, STAGES, binding.GRID_ASYM, binding.SCALE_F32,
-                                      pkgs, p_outs, stream, f_items)
+        for c in steps_calls:
+            if flush is not None:
+                flush()
+            c()
 
     for _ in range(args.warmup):
         step()
@@ -433,81 +584,98 @@ def run_gpu(args, world, rank, local) -> dict | None:
     if binding.rrq_get_device_status() != 0:
         raise RuntimeError("a kernel reported a timeout during warm-up")
 
-    ev = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(args.steps)]
+    # the timed region: events around every call when L2 is flushed between
+    # calls (the flushes are not timed), else around each step
+    per_call = flush is not None
+    ev = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+           for _ in (steps_calls if per_call else [None])] for _ in range(args.steps)]
     barrier(world)
     torch.cuda.synchronize()
     with ClockSampler(local) as clocks:
         t0 = torch.cuda.Event(enable_timing=True)
         t1 = torch.cuda.Event(enable_timing=True)
         t0.record(stream)
-        for a, b in ev:
-            a.record(stream)
-            step()
-            b.record(stream)
+        for s in range(args.steps):
+            if per_call:
+                for (a, b), c in zip(ev[s], steps_calls):
+                    flush()
+                    a.record(stream)
+                    c()
+                    b.record(stream)
+            else:
+                a, b = ev[s][0]
+                a.record(stream)
+                step()
+                b.record(stream)
         t1.record(stream)
         torch.cuda.synchronize()
     barrier(world)
     status = binding.rrq_get_device_status()
     if status != 0:
         raise RuntimeError(f"kernel status {status} in the timed region")
-    elapsed_ms = t0.elapsed_time(t1)
-    f_ms = [a.elapsed_time(b) for a, b in ev]
+    f_ms = [sum(a.elapsed_time(b) for a, b in evs) for evs in ev]
+    elapsed_ms = sum(f_ms) if per_call else t0.elapsed_time(t1)
     elapsed_ms = max_over_ranks(elapsed_ms, world)
 
-    # the same outputs by two calls (package, then every prefix): breakdown only
-    def timed(fn, reps=3):
-        fn()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(stream)
-        for _ in range(reps):
-            fn()
-        b.record(stream)
-        torch.cuda.synchronize()
-        return a.elapsed_time(b) / reps
-    q_ms = [timed(quantize_all)]
-    r_ms = [timed(reconstruct_all)]
-
-    # separate rrq_reconstruct calls per k (context for the breakdown, not the step)
-    reconstruct_each_k()
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(stream)
-    for _ in range(2):
-        reconstruct_each_k()
-    b.record(stream)
+    # breakdown: the package alone (rrq_quantize), every prefix from the
+    # package, and each prefix by its own call
+    q_s = time_calls(wl.quantize_calls(), stream, 3, flush)
+    r_s = time_calls(wl.reconstruct_calls(None), stream, 3, flush)
+    each_k = {k: time_calls(wl.reconstruct_calls(k), stream, 2, flush) for k in KS}
     torch.cuda.synchronize()
-    each_k_s = a.elapsed_time(b) / 2 / 1e3
+    if binding.rrq_get_device_status() != 0:
+        raise RuntimeError("a kernel reported a timeout in the breakdown")
 
-    sym = time_sym_f16(mats, p_outs, specs, stream) if not args.no_sym else None
-    from_base = time_from_base(mats, pkgs, specs, stream) if not args.no_sym else None
-    gemv = time_gemv(pkgs, specs, stream) if not args.no_sym else None
+    stack = args.workload == "qwen3_8b_stack" and wl.own_outputs and not args.no_sym
+    mats, pkgs, p_outs = wl.mats, wl.pkgs, wl.p_outs
+    sym = time_sym_f16(mats, p_outs, specs, stream) if stack else None
+    from_base = time_from_base(mats, pkgs, specs, stream) if stack else None
+    gemv = time_gemv(pkgs, specs, stream) if stack else None
     batches = [int(x) for x in args.gemv_batches.split(",") if x.strip()]
     gemv_batches = {f"batch{b}": time_gemv(pkgs, specs, stream, batch=b) for b in batches if b != 1} \
-        if not args.no_sym and any(b != 1 for b in batches) else None
-    prefill = time_prefill(pkgs, specs, stream) if not args.no_sym else None
+        if stack and any(b != 1 for b in batches) else None
+    prefill = time_prefill(pkgs, specs, stream) if stack else None
     bits = {"+".join(map(str, b)): time_bits(mats, p_outs, specs, stream, b) for b in ((1, 3), (3, 1))} \
-        if not args.no_sym else None
-    pmr = time_pmr(mats, specs, stream) if not args.no_sym else None
-    e2e = run_e2e(args, mats, pkgs, p_outs, specs, stream, world) if not args.no_e2e else None
+        if stack else None
+    pmr = time_pmr(mats, specs, stream) if stack else None
+    e2e = run_e2e(args, mats, pkgs, p_outs, specs, stream, world) \
+        if not args.no_e2e and wl.own_outputs and len(wl.units) == 1 else None
     if rank != 0:
         return None
 
     peaks = measured_peaks()
+    hbm = peaks["hbm_gbs"]
     clock_summary = clocks.summary()
     step_s = elapsed_ms / 1e3 / args.steps
     bytes_bf16 = 2.0 * n_total
-    value = world * bytes_bf16 / step_s / 1e9
-    q_s = statistics.mean(q_ms) / 1e3
-    r_s = statistics.mean(r_ms) / 1e3
+    total_bf16 = 2.0 * sum(sp.numel for sp in specs_all) if args.split else world * bytes_bf16
+    value = total_bf16 / step_s / 1e9
     f_s = statistics.mean(f_ms) / 1e3
-    f_alg = sum(alg_bytes_quantize(sp.numel) + STAGES * 2 * sp.numel for sp in specs)
-    q_alg = sum(alg_bytes_quantize(sp.numel) for sp in specs)
-    r_alg = sum(alg_bytes_prefixes(sp.numel, len(KS)) for sp in specs)
-    r_each_alg = sum(alg_bytes_reconstruct(sp.numel, k) for sp in specs for k in KS)
-    q_gbs = q_alg / q_s / 1e9
-    r_gbs = r_alg / r_s / 1e9
+    g_of = lambda sp: sp.group
+    f_alg = sum(alg_bytes_quantize(sp.numel, g_of(sp)) + STAGES * 2 * sp.numel for sp in specs)
+    q_alg = sum(alg_bytes_quantize(sp.numel, g_of(sp)) for sp in specs)
+    r_alg = sum(alg_bytes_prefixes(sp.numel, len(KS), g_of(sp)) for sp in specs)
+    k_alg = {k: sum(alg_bytes_reconstruct(sp.numel, k, g_of(sp)) for sp in specs) for k in KS}
     per_launch = 64  # matrices per kernel launch of the batch entry points
-    launches = math.ceil(len(specs) / per_launch)
-    traffic = recorded_traffic("rrq_quantize_prefixes", f_alg / launches, f_alg / launches)
+    launches = sum(math.ceil(len(u) / per_launch) for u in wl.units)
+    q_launches = sum(math.ceil(sum(1 for sp in specs if sp.group == g) / per_launch)
+                     for g in {sp.group for sp in specs})
+    traffic = recorded_traffic("rrq_quantize_prefixes", f_alg / launches, f_alg / launches) \
+        if args.workload in TRAFFIC_WORKLOADS else None
+    rooflines = {
+        "rrq_quantize": roofline_entry("quantize_kernel<g,0,0>: rrq_quantize_batch, the package only", q_alg, q_s,
+                                       hbm, q_launches,
+                                       "rrq_quantize" if args.workload in TRAFFIC_WORKLOADS else None),
+        "rrq_reconstruct_prefixes": roofline_entry(
+            "reconstruct_kernel<g,4,1,0>: rrq_reconstruct_prefixes_batch, every prefix 1..4 from the package",
+            r_alg, r_s, hbm, launches, "rrq_reconstruct_prefixes" if args.workload in TRAFFIC_WORKLOADS else None),
+    }
+    for k in KS:
+        rooflines[f"rrq_reconstruct_k{k}"] = roofline_entry(
+            f"reconstruct_kernel<g,{k},0,0>: rrq_reconstruct_batch at prefix k={k}", k_alg[k], each_k[k], hbm,
+            launches, None)
+    l2_text = (f"L2 flushed ({2 * L2_BYTES // 2**20} MiB write) before every timed call" if flush is not None else
+               f"inputs {2 * n_total / 1e9:.2f} GB per rank, larger than the {L2_BYTES // 2**20} MiB L2; no flush")
     line = {
         "metric": METRIC,
         "value": round(value, 2),
@@ -517,36 +685,37 @@ def run_gpu(args, world, rank, local) -> dict | None:
         "warmup": args.warmup,
         "ms_per_step": round(elapsed_ms / args.steps, 3),
         "higher_is_better": True,
-        "scaling": "weak",
+        "scaling": "strong" if args.split else "weak",
         "vs_baseline": None,
         "dtype": "f32",
         "data": "synthetic",
         "config": {
             "workload": WORKLOAD_TEXT.get(args.workload, args.workload),
-            "step": f"rrq_quantize_prefixes on all {len(specs)} matrices: the package and the "
-                    f"k=1,2,3,4 bf16 reconstructions of every matrix in one pass",
+            "step": (f"rrq_quantize_prefixes on all {len(specs)} matrices ({len(steps_calls)} call(s)): the "
+                     f"package and the k=1,2,3,4 bf16 reconstructions of every matrix in one pass"
+                     + ("" if wl.own_outputs else "; the prefixes of each layer of 7 go to one set of "
+                        "buffers reused by every layer (the four prefixes of the stack do not fit in HBM)")),
             "weights_per_rank": n_total,
-            "l2": f"inputs {2 * n_total / 1e9:.2f} GB per rank, larger than the 126 MB L2; no flush",
-            "parallelism": f"{world} independent rank(s), one stack each",
+            "l2": l2_text,
+            "parallelism": (f"one stack split over {world} rank(s) by matrices (largest first to the least "
+                            f"loaded rank)" if args.split else f"{world} independent rank(s), one stack each"),
         },
         "breakdown": {
             "step_alg_gbs": round(f_alg / f_s / 1e9, 1),
-            "step_frac_of_measured_hbm": round(f_alg / f_s / 1e9 / peaks["hbm_gbs"], 4),
+            "step_frac_of_measured_hbm": round(f_alg / f_s / 1e9 / hbm, 4),
             "two_calls_s_per_stack": round(q_s + r_s, 6),
             "two_calls_bf16_gbs": round(bytes_bf16 / (q_s + r_s) / 1e9, 2),
-            "quantize_alu_frac": round(n_total * STAGES * FP32_OPS_PER_WEIGHT_STAGE / q_s / 1e12
-                                       / fp32_peak_tops(clock_summary.get("sm_mhz")), 4),
             "quantize_s_per_stack": round(q_s, 6),
-            "quantize_alg_gbs": round(q_gbs, 1),
+            "quantize_alg_gbs": round(q_alg / q_s / 1e9, 1),
             "quantize_bf16_in_gbs": round(bytes_bf16 / q_s / 1e9, 1),
             "quantize_weights_per_s": round(n_total / q_s, 1),
+            "quantize_frac_of_measured_hbm": round(q_alg / q_s / 1e9 / hbm, 4),
+            "quantize_frac_of_nominal_8tbs": round(q_alg / q_s / 1e9 / 8000.0, 4),
             "reconstruct_prefixes_k1to4_s": round(r_s, 6),
-            "reconstruct_prefixes_alg_gbs": round(r_gbs, 1),
-            "reconstruct_separate_k1to4_s": round(each_k_s, 6),
-            "reconstruct_separate_alg_gbs": round(r_each_alg / each_k_s / 1e9, 1),
-            "quantize_frac_of_measured_hbm": round(q_gbs / peaks["hbm_gbs"], 4),
-            "reconstruct_frac_of_measured_hbm": round(r_gbs / peaks["hbm_gbs"], 4),
-            "quantize_frac_of_nominal_8tbs": round(q_gbs / 8000.0, 4),
+            "reconstruct_prefixes_alg_gbs": round(r_alg / r_s / 1e9, 1),
+            "reconstruct_frac_of_measured_hbm": round(r_alg / r_s / 1e9 / hbm, 4),
+            "reconstruct_separate_k1to4_s": round(sum(each_k.values()), 6),
+            "reconstruct_separate_alg_gbs": round(sum(k_alg.values()) / sum(each_k.values()) / 1e9, 1),
             "paper_context_s": {"full_all_rtn_package_qwen3_8b_a100": 1293, "four_rtn_passes_a100": 412},
             "sym_f16": sym,
             "from_base": from_base,
@@ -557,26 +726,24 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "group_pmr": pmr,
         },
         "roofline": {"kernel": "rrq_quantize_prefixes (quantize_kernel, build with prefixes)",
-                     "bound": "hbm", "achieved": round(f_alg / f_s / 1e9, 1), "peak": peaks["hbm_gbs"],
+                     "bound": "hbm", "achieved": round(f_alg / f_s / 1e9, 1), "peak": hbm,
                      "peak_source": f"{peaks['source']} copy bandwidth (MEASURED_PEAKS.json hbm_gbs)",
-                     "unit": "GB/s", "frac": round(f_alg / f_s / 1e9 / peaks["hbm_gbs"], 4),
-                     "alg_bytes_per_weight": 3.25 + 2 * STAGES, "traffic": traffic},
+                     "unit": "GB/s", "frac": round(f_alg / f_s / 1e9 / hbm, 4),
+                     "alg_bytes_per_weight": round(f_alg / n_total, 4), "traffic": traffic},
+        "rooflines": rooflines,
         "clocks": clock_summary,
         "gpu_launches": launches * args.steps,
         "e2e": e2e,
     }
+    if args.cpu_seconds > 0 and world == 1:  # the host's cores, once (rank 0 at N=1)
+        samples = [(specs[i].name, wl.mats[i]) for i in range(len(specs))]
+        line["cpu_baseline"] = cpu_baseline(samples, args.cpu_seconds)
     return line
 
 
-# operations of the definition per weight and stage: v - lo, / s, rhe, Q * s,
-# lo + Q s, v - L, and the min and max that give the next stage's range
-FP32_OPS_PER_WEIGHT_STAGE = 8
-
-
-def fp32_peak_tops(sm_mhz: float | None) -> float:
-    """fp32 pipe peak in tera-operations/s: 152 SMs x 128 fp32 lanes x SM clock
-    (125 per SM per clock measured with a packed-fma throughput loop)."""
-    return 152 * 128 * (sm_mhz or 2070.0) * 1e6 / 1e12
+# workloads whose DRAM traffic per algorithmic byte the committed ncu capture
+# (one Qwen3-8B-shaped layer) represents: the same shapes and group size
+TRAFFIC_WORKLOADS = ("qwen3_8b_stack", "qwen3_8b_layer")
 
 
 def recorded_traffic(kernel: str, q_bytes_per_launch: float, r_bytes_per_launch: float):
@@ -697,54 +864,86 @@ def run_e2e(args, mats, pkgs, p_outs, specs, stream, world) -> dict:
 # ---------------------------------------------------------------------------
 # CPU oracle: baseline leg and the --impl reference arm
 # ---------------------------------------------------------------------------
-def oracle_sample(seconds_target: float, seed_offset: int = 0):
-    """Times the single-threaded C oracle on whole matrices of the stack's
-    first layer (quantize plus reconstruct at k=1..4), adding matrices until
-    about `seconds_target` of CPU work; returns (bf16 bytes, seconds, names)."""
-    import oracle
-    from paper_2608_04048_gb300 import workloads
-    specs = workloads.config_matrices(WORKLOAD)
-    order = [1, 2, 0, 3, 6, 4, 5]  # k, v, q, o, down, gate, up of layer 0
-    done_bytes, spent, names = 0.0, 0.0, []
-    for i in order:
-        sp = specs[i]
-        W = workloads.generate(sp.rows, sp.cols, sp.seed + seed_offset, sp.dist, "cpu")
-        Wb = W.view(torch.int16).numpy().view(np.uint16)
-        t = time.perf_counter()
-        pkg = oracle.quantize(Wb, GROUP, STAGES)
-        for k in KS:
-            oracle.reconstruct(*pkg, sp.rows, sp.cols, GROUP, k)
-        spent += time.perf_counter() - t
-        done_bytes += 2.0 * sp.numel
-        names.append(f"{sp.name} {sp.rows}x{sp.cols}")
-        if spent >= seconds_target:
+ORACLE_WEIGHTS_PER_CORE_S = 2.0e7   # about what one host core's oracle does per second (sizes the sample)
+
+
+def oracle_pool_sample(samples, target_core_s: float, pool, region=None) -> dict:
+    """Times the oracle as it stands (quantize, then reconstruct at k =
+    1..4) on the host's cores.  Sampled matrices are taken in order until
+    they hold about `target_core_s` core-seconds of oracle work (at least
+    one), copied into shared memory (not timed), cut into about 4 row-range
+    tasks per process, and timed from the first submission to the last
+    result.  samples: (label, bf16 tensor) pairs."""
+    from oracle.pool import Layout, SharedRegion, Task
+    chosen, weights = [], 0
+    for label, W in samples:
+        chosen.append((label, W))
+        weights += W.numel()
+        if weights >= target_core_s * ORACLE_WEIGHTS_PER_CORE_S:
             break
-    return done_bytes, spent, names
+    lay = Layout()
+    offs = [lay.take(2 * W.numel()) for _, W in chosen]
+    own = region is None
+    reg = SharedRegion(lay.size) if own else region
+    try:
+        for (label, W), off in zip(chosen, offs):
+            reg.array(off, np.uint16, W.numel())[:] = W.contiguous().view(torch.int16).cpu().numpy().view(
+                np.uint16).reshape(-1)
+        per_task = max(1 << 16, weights // (4 * pool.processes))
+        tasks = []
+        for (label, W), off in zip(chosen, offs):
+            rows, cols = W.shape
+            tasks += Task(reg.name, label, "asym", GROUP, STAGES, rows, cols, off, check=False,
+                          oracle_prefixes=len(KS)).split(per_task)
+        t0 = time.perf_counter()
+        res = pool.run(tasks)
+        wall = time.perf_counter() - t0
+    finally:
+        if own:
+            reg.close()
+    core_s = sum(r["seconds"] for r in res)
+    names = [f"{label} {W.shape[0]}x{W.shape[1]}" for label, W in chosen]
+    return {"bytes": 2.0 * weights, "weights": weights, "wall_s": wall, "core_s": core_s, "names": names}
 
 
-def cpu_baseline(seconds_target: float) -> dict:
-    import oracle
-    oracle.build()
-    b, s, names = oracle_sample(seconds_target)
-    return {"value": round(b / s / 1e9, 5), "unit": "GB/s", "cores": 1, "kind": "oracle",
-            "sample": f"single-threaded C oracle, quantize + reconstruct k=1..4 of layer-0 matrices "
-                      f"{', '.join(names)} ({b / 2:.0f} weights, {s:.1f} s)",
-            "host_cpus": os.cpu_count()}
+def cpu_baseline(samples, target_core_s: float) -> dict:
+    from oracle.pool import OraclePool, host_description
+    host = host_description()
+    with OraclePool() as pool:
+        r = oracle_pool_sample(samples, target_core_s, pool)
+        procs = pool.processes
+    return {"value": round(r["bytes"] / r["wall_s"] / 1e9, 5), "unit": "GB/s", "cores": procs, "kind": "oracle",
+            "sample": f"the single-threaded C oracle, quantize + reconstruct k=1..4, in {procs} processes over "
+                      f"row ranges of {', '.join(r['names'])} ({r['weights']} weights, {r['wall_s']:.1f} s wall, "
+                      f"{r['core_s']:.1f} core-s)",
+            "per_core_gbs": round(r["bytes"] / r["core_s"] / 1e9, 5),
+            "weights_per_s_per_core": round(r["weights"] / r["core_s"], 1),
+            "cpu_model": host["cpu_model"], "host_cpus": host["cores"]}
+
+
+REFERENCE_SAMPLE = ("q_proj", "k_proj", "v_proj", "o_proj")   # of layer 0, per step
 
 
 def run_reference(args, world, rank):
     if rank != 0:
         return None
-    import oracle
-    oracle.build()
-    for _ in range(args.warmup):
-        oracle_sample(0.0)
-    total_b, total_s, names = 0.0, 0.0, None
-    for _ in range(args.steps):
-        b, s, names = oracle_sample(0.0)
-        total_b += b
-        total_s += s
+    from oracle.pool import OraclePool, host_description
+    from paper_2608_04048_gb300 import workloads
+    specs = [sp for sp in workloads.config_matrices(WORKLOAD)[:7] if sp.name.split(".")[-1] in REFERENCE_SAMPLE]
+    samples = [(sp.name, workloads.generate(sp.rows, sp.cols, sp.seed, sp.dist, "cpu")) for sp in specs]
+    host = host_description()
+    with OraclePool() as pool:
+        for _ in range(args.warmup):
+            oracle_pool_sample(samples, float("inf"), pool)
+        total_b, total_s, core_s = 0.0, 0.0, 0.0
+        for _ in range(args.steps):
+            r = oracle_pool_sample(samples, float("inf"), pool)
+            total_b += r["bytes"]
+            total_s += r["wall_s"]
+            core_s += r["core_s"]
+        procs = pool.processes
     value = total_b / total_s / 1e9
+    names = ", ".join(f"{sp.name} {sp.rows}x{sp.cols}" for sp in specs)
     return {
         "impl": "reference",
         "metric": METRIC,
@@ -753,16 +952,18 @@ def run_reference(args, world, rank):
         "n_gpus": world,
         "steps": args.steps,
         "warmup": args.warmup,
-        "ms_per_step": round(total_s / args.steps * 1e3, 3),
+        "ms_per_step": round(total_s / max(1, args.steps) * 1e3, 3),
         "higher_is_better": True,
         "scaling": "weak",
         "vs_baseline": None,
         "dtype": "f32",
         "data": "synthetic",
-        "config": {"workload": f"{WORKLOAD}: bounded sample of the same stack, {', '.join(names)}",
-                   "step": "oracle quantize + reconstruct k=1..4 of the sampled matrix on the host"},
-        "cpu_baseline": {"value": round(value, 5), "unit": "GB/s", "cores": 1, "kind": "oracle",
-                         "sample": f"{', '.join(names)} per step"},
+        "config": {"workload": f"{WORKLOAD}: bounded sample of the same stack, {names}",
+                   "step": f"oracle quantize + reconstruct k=1..4 of the sampled matrices on {procs} host "
+                           f"processes (row ranges)"},
+        "cpu_baseline": {"value": round(value, 5), "unit": "GB/s", "cores": procs, "kind": "oracle",
+                         "sample": f"{names} per step", "per_core_gbs": round(total_b / core_s / 1e9, 5),
+                         "cpu_model": host["cpu_model"]},
         "e2e": {"value": round(value, 5), "unit": "GB/s", "h2d_bytes_per_step": 0,
                 "d2h_bytes_per_step": 0},
     }
@@ -774,12 +975,16 @@ def main(argv=None):
     ap.add_argument("--steps", type=int, default=5)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
-    ap.add_argument("--workload", default=WORKLOAD)
+    ap.add_argument("--workload", default=WORKLOAD,
+                    help="single_4096, qwen3_8b_layer, qwen3_8b_stack (default), sweep_8192, qwen3_32b_stack")
+    ap.add_argument("--split", action="store_true",
+                    help="under torchrun: split ONE stack's matrices over the ranks (strong scaling)")
     ap.add_argument("--e2e-steps", type=int, default=2)
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-sym", action="store_true",
                     help="skip the symmetric binary16, base-checkpoint and product breakdown")
-    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--cpu-seconds", type=float, default=20.0,
+                    help="core-seconds of oracle work in the CPU baseline (0 skips it)")
     ap.add_argument("--gemv-batches", default="1",
                     help="comma-separated activation-row counts for the decode-product breakdown (1..8)")
     args = ap.parse_args(argv)
@@ -798,8 +1003,6 @@ def main(argv=None):
             if not torch.cuda.is_available():
                 raise SystemExit("bench.py needs a CUDA device (use --impl reference for the CPU oracle)")
             line = run_gpu(args, world, rank, local)
-            if line is not None:
-                line["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
         if line is not None:
             print(json.dumps(line), flush=True)
     finally:

@@ -72,3 +72,50 @@ def test_reference_arm_under_torchrun_two_ranks():
     assert line["impl"] == "reference" and line["n_gpus"] == 2
     assert line["value"] > 0 and line["e2e"]["h2d_bytes_per_step"] == 0
     assert line["cpu_baseline"]["kind"] == "oracle"
+
+
+def _shard_worker(rank, world, port, q):
+    import torch
+    import torch.distributed as dist
+    os.environ.update(MASTER_ADDR="127.0.0.1", MASTER_PORT=str(port), RANK=str(rank),
+                      WORLD_SIZE=str(world), LOCAL_RANK=str(rank))
+    sys.path.insert(0, ROOT)
+    import bench
+    from paper_2608_04048_gb300 import workloads
+    dist.init_process_group("gloo", rank=rank, world_size=world)
+    try:
+        out = {}
+        for name in ("qwen3_8b_stack", "qwen3_32b_stack", "qwen3_8b_layer"):
+            specs = workloads.config_matrices(name)
+            mine = bench.shard_matrices(specs, world, rank)
+            got = [None] * world
+            dist.all_gather_object(got, mine)
+            out[name] = got
+        q.put((rank, out))
+    finally:
+        dist.destroy_process_group()
+
+
+@pytest.mark.parametrize("world", [2, 3])
+def test_split_stack_covers_every_matrix_once(world):
+    """--split: each rank computes its own share of ONE stack; gathered over
+    gloo ranks, the shares cover every matrix exactly once and balance the
+    weights to within one matrix."""
+    from paper_2608_04048_gb300 import workloads
+    ctx = mp.get_context("spawn")
+    q = ctx.Queue()
+    port = _free_port()
+    procs = [ctx.Process(target=_shard_worker, args=(r, world, port, q)) for r in range(world)]
+    for p in procs:
+        p.start()
+    for p in procs:
+        p.join(180)
+        assert p.exitcode == 0
+    res = dict(q.get(timeout=10) for _ in range(world))
+    for name, shares in res[0].items():
+        assert all(res[r][name] == shares for r in range(world))  # every rank computes the same split
+        specs = workloads.config_matrices(name)
+        flat = sorted(i for s in shares for i in s)
+        assert flat == list(range(len(specs))), name
+        load = [sum(specs[i].numel for i in s) for s in shares]
+        assert max(load) - min(load) <= max(sp.numel for sp in specs), (name, load)
