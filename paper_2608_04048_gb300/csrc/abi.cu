@@ -555,6 +555,22 @@ bool encode_codes(CUtensorMap* map, const uint8_t* codes, int64_t rows, int64_t 
             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+}  // namespace
+
+bool rrq::encode_lane_tiles(CUtensorMap* map, const uint16_t* W, int64_t n, int lw) {
+  EncodeTiledFn fn = encode_tiled();
+  if (!fn || (lw != 32 && lw != 64) || n % lw != 0 || n / lw >= (int64_t{1} << 31)) return false;
+  const cuuint64_t dim[2] = {static_cast<cuuint64_t>(lw), static_cast<cuuint64_t>(n / lw)};
+  const cuuint64_t stride[1] = {static_cast<cuuint64_t>(lw) * 2};
+  const cuuint32_t box[2] = {static_cast<cuuint32_t>(lw), 32};
+  const cuuint32_t estride[2] = {1, 1};
+  return fn(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<uint16_t*>(W), dim, stride, box, estride,
+            CU_TENSOR_MAP_INTERLEAVE_NONE, lw == 64 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B,
+            CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+namespace {
+
 rrq_status prefill_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k, int64_t tokens,
                          rrq_stream_t stream) {
   if (!items || count < 1 || k < 1 || k > f.n_stages) return RRQ_ERR_INVALID_ARG;

@@ -50,6 +50,21 @@ struct QuantizeBatch {
   QuantizeItem item[kMaxBatch];
 };
 
+// The wide-lane build (quantize_tile_kernel.cuh): the launch's matrices as
+// 2-D tensor maps [n / LW, LW] of bf16 (one 32-row box = one warp chunk of
+// 32 * LW weights), and the batch with chunk_begin / total_chunks counted in
+// those chunks.
+struct QuantizeTileBatch {
+  CUtensorMap w[kMaxBatch];
+  QuantizeBatch b;
+};
+
+// Encodes W (n bf16 weights, n % lw == 0, n / lw < 2^31) as the 2-D tensor
+// map [n / lw, lw] with 32-row boxes and the 128-byte (lw = 64) or 64-byte
+// (lw = 32) swizzle; false if the driver's encoder is unavailable or rejects
+// it.
+bool encode_lane_tiles(CUtensorMap* map, const uint16_t* W, int64_t n, int lw);
+
 struct ReconstructItem {
   const uint8_t* codes[kMaxStages];
   const void* scales[kMaxStages];  // float or binary16
