@@ -40,7 +40,10 @@
  * default stream).  Outputs are valid once the stream reaches the call.  The
  * library never allocates, frees or synchronizes in these calls; only
  * rrq_get_device_status synchronizes.  A bad argument returns an error code
- * synchronously and launches nothing.  Functions are thread-safe.
+ * synchronously and launches nothing.  A call that makes several launches
+ * (batches beyond one launch's matrices, decode products split over
+ * activation rows) and meets RRQ_ERR_CUDA after its first launch may leave
+ * its outputs partly written.  Functions are thread-safe.
  */
 #ifndef RRQ_H
 #define RRQ_H
@@ -395,10 +398,24 @@ size_t rrq_meta_count(int64_t rows, int64_t cols, int group);
 size_t rrq_package_bytes(int64_t rows, int64_t cols, int group, int n_stages);
 
 /* Synchronizes `stream`, then reads and clears the current device's status
- * word.  Returns RRQ_ERR_TIMEOUT if a kernel on this device gave up on a
- * bounded wait since the last call (its outputs are then incomplete),
- * RRQ_ERR_CUDA if the synchronization failed, RRQ_OK otherwise. */
+ * word in one atomic exchange (a one-thread kernel on `stream`).  Returns
+ * RRQ_ERR_TIMEOUT if a kernel on this device gave up on a bounded wait since
+ * the last call (its outputs are then incomplete), RRQ_ERR_CUDA if the
+ * synchronization or the exchange failed, RRQ_OK otherwise.  The word is
+ * per device: kernels still running on other streams may set it after the
+ * exchange, and the next call reports them. */
 rrq_status rrq_get_device_status(rrq_stream_t stream);
+
+/* Whether [p, p + bytes) lies in device memory of the current device (or
+ * in managed memory): RRQ_OK if the driver reports every byte of it as part
+ * of such allocations, RRQ_ERR_INVALID_ARG otherwise (a null, host, freed or
+ * other device's pointer, or a length that runs past the allocation;
+ * bytes == 0 checks the first byte).  Every entry point applies this check
+ * to each of its buffers before launching anything.  Looks up the driver's
+ * pointer attributes on every call (nothing is remembered between calls),
+ * launches nothing and does not synchronize.  Paper: no counterpart (it is
+ * the library's argument guard). */
+rrq_status rrq_check_buffer(const void* p, size_t bytes);
 
 /* Longest time a kernel waits for one of its own bulk copies before it
  * records RRQ_ERR_TIMEOUT and returns (default 1,000,000 us).  0 makes every

@@ -26,7 +26,7 @@ EXPORTS = ["rrq_quantize", "rrq_reconstruct", "rrq_quantize_batch", "rrq_reconst
            "rrq_stage_codes_bytes", "rrq_group_pmr", "rrq_quantize_prefixes", "rrq_scales_bytes", "rrq_package_bytes_ex",
            "rrq_codes_bytes", "rrq_meta_count",
            "rrq_package_bytes", "rrq_get_device_status", "rrq_set_wait_limit_us",
-           "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error"]
+           "rrq_set_debug_flags", "rrq_status_string", "rrq_last_cuda_error", "rrq_check_buffer"]
 
 
 MAX_STAGES = 4
@@ -174,6 +174,8 @@ def load_library():
     lib.rrq_set_debug_flags.restype = None
     lib.rrq_status_string.argtypes = [i32]
     lib.rrq_status_string.restype = ctypes.c_char_p
+    lib.rrq_check_buffer.argtypes = [vp, ctypes.c_size_t]
+    lib.rrq_check_buffer.restype = i32
     lib.rrq_last_cuda_error.argtypes = []
     lib.rrq_last_cuda_error.restype = i32
     _LIB = lib
@@ -604,6 +606,12 @@ def rrq_package_bytes(rows: int, cols: int, group: int, n_stages: int) -> int:
 def rrq_get_device_status(stream=None) -> int:
     """Synchronizes the stream; returns 0 (RRQ_OK) or a status code."""
     return int(load_library().rrq_get_device_status(_stream_handle(stream)))
+
+
+def rrq_check_buffer(ptr: int, nbytes: int) -> int:
+    """Status of the library's device-buffer check for [ptr, ptr + nbytes)
+    (0 = device memory of the current device; launches nothing)."""
+    return int(load_library().rrq_check_buffer(ptr, nbytes))
 
 
 def rrq_set_wait_limit_us(us: int) -> None:

@@ -16,6 +16,12 @@
 // Per-device status word: bit kStatusTimeout is set by a kernel that gave up
 // on a bounded wait.  Read and cleared by rrq_get_device_status.
 __device__ unsigned int rrq_device_status;
+// The value rrq_get_device_status took out of the status word.
+__device__ unsigned int rrq_device_status_taken;
+
+// Reads and clears the status word in one atomic step, so that a bit set by
+// a kernel on another stream in the meantime is kept for the next read.
+__global__ void rrq_take_status_kernel() { rrq_device_status_taken = atomicExch(&rrq_device_status, 0u); }
 
 namespace {
 
@@ -55,6 +61,7 @@ rrq_status current_device(int* dev_out, DeviceState** state) {
     if ((e = rrq::quantize_prepare_base())) return fail_cuda(e);
     if ((e = rrq::quantize_prepare_emit())) return fail_cuda(e);
     if ((e = rrq::reconstruct_prepare())) return fail_cuda(e);
+    if ((e = rrq::gemv_prepare())) return fail_cuda(e);
     d.ready = true;
   }
   *dev_out = dev;
@@ -71,32 +78,75 @@ bool shape_ok(int64_t rows, int64_t cols) {
 
 bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) & (a - 1)) == 0; }
 
-// Device (or managed) memory of the current device.  With unified virtual
-// addressing a 2 MiB page of device virtual memory never holds host memory,
-// so answers are cached per page (a direct-mapped table of recent pages).
-struct PageCache {
-  static constexpr int kSlots = 4096;
-  std::atomic<uint64_t> slot[kSlots];  // (page << 8) | (device + 1), 0 = empty
-  PageCache() {
-    for (auto& s : slot) s.store(0, std::memory_order_relaxed);
-  }
-};
-PageCache g_pages;
+// The driver's cuPointerGetAttributes, looked up once through the runtime
+// (no link against the driver library).
+using PointerAttrsFn = CUresult (*)(unsigned int, CUpointer_attribute*, void**, CUdeviceptr);
 
-bool on_device(const void* p, int dev) {
-  const uint64_t page = reinterpret_cast<uintptr_t>(p) >> 21;
-  const uint64_t tag = (page << 8) | static_cast<uint64_t>(dev + 1);
-  std::atomic<uint64_t>& s = g_pages.slot[page % PageCache::kSlots];
-  if (s.load(std::memory_order_relaxed) == tag) return true;
-  cudaPointerAttributes a;
-  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
-    cudaGetLastError();  // clear the error of an unknown pointer
+PointerAttrsFn pointer_attrs() {
+  static PointerAttrsFn fn = [] {
+    void* ptr = nullptr;
+    cudaDriverEntryPointQueryResult q{};
+    if (cudaGetDriverEntryPointByVersion("cuPointerGetAttributes", &ptr, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
+        q != cudaDriverEntryPointSuccess)
+      return static_cast<PointerAttrsFn>(nullptr);
+    return reinterpret_cast<PointerAttrsFn>(ptr);
+  }();
+  return fn;
+}
+
+// Whether byte ranges lie in device memory of device `dev` (or in managed
+// memory): every byte of [lo, hi) must belong to allocations the driver
+// reports as such, walked allocation by allocation (a buffer may span
+// several contiguously mapped allocations).  Answers are kept for the
+// length of one call only: memory freed and reused between calls is looked
+// up again.
+class BufferCheck {
+ public:
+  explicit BufferCheck(int dev) : dev_(dev) {}
+
+  bool ok(uintptr_t lo, uintptr_t hi) {
+    if (hi < lo) return false;
+    while (lo < hi) {
+      uintptr_t end = 0;
+      if (!known(lo, &end) && !lookup(lo, &end)) return false;
+      lo = end;
+    }
+    return true;
+  }
+
+ private:
+  bool known(uintptr_t a, uintptr_t* end) const {
+    for (const auto& r : seen_)
+      if (a >= r.first && a < r.second) {
+        *end = r.second;
+        return true;
+      }
     return false;
   }
-  const bool ok = (a.type == cudaMemoryTypeDevice && a.device == dev) || a.type == cudaMemoryTypeManaged;
-  if (ok && a.type == cudaMemoryTypeDevice) s.store(tag, std::memory_order_relaxed);
-  return ok;
-}
+  bool lookup(uintptr_t a, uintptr_t* end) {
+    PointerAttrsFn fn = pointer_attrs();
+    if (!fn) return false;
+    unsigned int type = 0;
+    int ordinal = -1, managed = 0;
+    CUdeviceptr start = 0;
+    size_t size = 0;
+    CUpointer_attribute attrs[5] = {CU_POINTER_ATTRIBUTE_MEMORY_TYPE, CU_POINTER_ATTRIBUTE_DEVICE_ORDINAL,
+                                    CU_POINTER_ATTRIBUTE_IS_MANAGED, CU_POINTER_ATTRIBUTE_RANGE_START_ADDR,
+                                    CU_POINTER_ATTRIBUTE_RANGE_SIZE};
+    void* data[5] = {&type, &ordinal, &managed, &start, &size};
+    if (fn(5, attrs, data, static_cast<CUdeviceptr>(a)) != CUDA_SUCCESS) return false;
+    const bool device = managed || (type == CU_MEMORYTYPE_DEVICE && ordinal == dev_);
+    const uintptr_t s = static_cast<uintptr_t>(start), e = s + size;
+    if (!device || size == 0 || a < s || a >= e) return false;
+    seen_.push_back({s, e});
+    *end = e;
+    return true;
+  }
+
+  int dev_;
+  std::vector<std::pair<uintptr_t, uintptr_t>> seen_;
+};
 
 // Byte ranges touched by a call; outputs may not overlap anything else.
 struct Range {
@@ -113,6 +163,14 @@ bool ranges_disjoint(std::vector<Range>& r) {
     max_hi_any = std::max(max_hi_any, x.hi);
     if (x.output) max_hi_out = std::max(max_hi_out, x.hi);
   }
+  return true;
+}
+
+// Every non-empty range of a call in device memory of the current device.
+bool ranges_on_device(const std::vector<Range>& r, int dev) {
+  BufferCheck check(dev);
+  for (const Range& x : r)
+    if (x.hi != x.lo && !check.ok(x.lo, x.hi)) return false;
   return true;
 }
 
@@ -255,17 +313,7 @@ rrq_status quantize_batch(const QView* items, int count, const Fmt& f, rrq_strea
   int dev = 0;
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
-  for (int i = 0; i < count; ++i) {
-    const QView& it = items[i];
-    if (!on_device(it.W_bf16, dev)) return RRQ_ERR_INVALID_ARG;
-    if (mode == kEmit)
-      for (int k = 0; k < n_stages; ++k)
-        if (!on_device(it.out[k], dev)) return RRQ_ERR_INVALID_ARG;
-    for (int k = 0; k < n_stages; ++k)
-      if (!on_device(it.codes[k], dev) || !on_device(it.scales[k], dev) ||
-          (!f.sym() && !on_device(it.zeros[k], dev)))
-        return RRQ_ERR_INVALID_ARG;
-  }
+  if (!ranges_on_device(ranges, dev)) return RRQ_ERR_INVALID_ARG;
 
   static thread_local rrq::QuantizeBatch p;  // ~8 KiB: kept off the stack
   for (int base = 0; base < count; base += rrq::kMaxBatch) {
@@ -354,15 +402,7 @@ rrq_status reconstruct_views(const ReconView* items, int count, const Fmt& f, in
   int dev = 0;
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
-  for (int i = 0; i < count; ++i) {
-    const ReconView& it = items[i];
-    for (int j = 0; j < n_out; ++j)
-      if (!on_device(it.out[j], dev)) return RRQ_ERR_INVALID_ARG;
-    for (int j = 0; j < k; ++j)
-      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) ||
-          (!f.sym() && !on_device(it.zeros[j], dev)))
-        return RRQ_ERR_INVALID_ARG;
-  }
+  if (!ranges_on_device(ranges, dev)) return RRQ_ERR_INVALID_ARG;
 
   static thread_local rrq::ReconstructBatch p;
   for (int base = 0; base < count; base += rrq::kMaxBatch) {
@@ -429,14 +469,7 @@ rrq_status check_product_items(const rrq_gemv_desc* items, int count, const Fmt&
   int dev = 0;
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
-  for (int i = 0; i < count; ++i) {
-    const rrq_gemv_desc& it = items[i];
-    if (!on_device(it.A_bf16, dev) || !on_device(it.Y, dev)) return RRQ_ERR_INVALID_ARG;
-    for (int j = 0; j < k; ++j)
-      if (!on_device(it.codes[j], dev) || !on_device(it.scales[j], dev) ||
-          (!f.sym() && !on_device(it.zeros[j], dev)))
-        return RRQ_ERR_INVALID_ARG;
-  }
+  if (!ranges_on_device(ranges, dev)) return RRQ_ERR_INVALID_ARG;
 
   *st_out = st;
   return RRQ_OK;
@@ -662,10 +695,7 @@ rrq_status pmr_batch(const rrq_pmr_desc* items, int count, int group, rrq_stream
   int dev = 0;
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
-  for (int i = 0; i < count; ++i)
-    if (!on_device(items[i].W_bf16, dev) || !on_device(items[i].pmr, dev) ||
-        (items[i].stats && !on_device(items[i].stats, dev)))
-      return RRQ_ERR_INVALID_ARG;
+  if (!ranges_on_device(ranges, dev)) return RRQ_ERR_INVALID_ARG;
   static thread_local rrq::PmrBatch p;
   for (int base = 0; base < count; base += rrq::kMaxBatch) {
     const int m = std::min(rrq::kMaxBatch, count - base);
@@ -880,15 +910,26 @@ rrq_status rrq_get_device_status(rrq_stream_t stream) {
   int dev = 0;
   DeviceState* st = nullptr;
   if (rrq_status rc = current_device(&dev, &st)) return rc;
-  cudaError_t e = cudaStreamSynchronize(reinterpret_cast<cudaStream_t>(stream));
+  const cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) return fail_cuda(e);
+  rrq_take_status_kernel<<<1, 1, 0, s>>>();
+  if ((e = cudaGetLastError())) return fail_cuda(e);
   unsigned word = 0;
-  if ((e = cudaMemcpyFromSymbol(&word, rrq_device_status, sizeof word))) return fail_cuda(e);
-  if (word != 0) {
-    const unsigned zero = 0;
-    if ((e = cudaMemcpyToSymbol(rrq_device_status, &zero, sizeof zero))) return fail_cuda(e);
-  }
+  if ((e = cudaMemcpyFromSymbolAsync(&word, rrq_device_status_taken, sizeof word, 0, cudaMemcpyDeviceToHost, s)))
+    return fail_cuda(e);
+  if ((e = cudaStreamSynchronize(s))) return fail_cuda(e);
   return (word & rrq::kStatusTimeout) ? RRQ_ERR_TIMEOUT : RRQ_OK;
+}
+
+rrq_status rrq_check_buffer(const void* p, size_t bytes) {
+  if (!p) return RRQ_ERR_INVALID_ARG;
+  int dev = 0;
+  DeviceState* st = nullptr;
+  if (rrq_status rc = current_device(&dev, &st)) return rc;
+  const uintptr_t a = reinterpret_cast<uintptr_t>(p);
+  BufferCheck check(dev);
+  return check.ok(a, a + (bytes ? bytes : 1)) ? RRQ_OK : RRQ_ERR_INVALID_ARG;
 }
 
 void rrq_set_wait_limit_us(uint32_t microseconds) {

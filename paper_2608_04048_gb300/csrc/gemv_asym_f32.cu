@@ -3,6 +3,8 @@
 
 namespace rrq {
 
+cudaError_t gemv_prepare_asym_f32() { return prepare_format<kAsymF32>(); }
+
 cudaError_t gemv_launch_asym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms) {
   return launch_format<kAsymF32>(k, nb, max_cols, p, stream, sms);
 }

@@ -386,39 +386,46 @@ inline int tokens_per_launch(int64_t max_cols, int k) {
   return static_cast<int>(t < max_rows_per_launch(k) ? t : max_rows_per_launch(k));
 }
 
-constexpr int kMaxDevices = 64;
-
 template <int F, int K, int B>
 cudaError_t launch_fkb(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
-  // per device: the largest dynamic shared memory enabled so far, and the
-  // resident CTAs per multiprocessor at the last size asked
-  static int attr_bytes[kMaxDevices] = {};
-  static int occ_smem[kMaxDevices] = {};
-  static int occ[kMaxDevices] = {};
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
-  if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
+  // the kernel's dynamic shared memory limit is raised once per device
+  // (prepare_format); the resident CTAs are asked for at this launch's size
   const int act_floats = static_cast<int>(act_floats_of(max_cols));
   const int smem = nb * act_floats * 4;
-  if (smem > attr_bytes[dev]) {
-    e = cudaFuncSetAttribute(gemv_kernel<F, K, B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
-    if (e != cudaSuccess) return e;
-    attr_bytes[dev] = smem;
-  }
-  if (occ[dev] == 0 || occ_smem[dev] != smem) {
-    int n = 0;
-    e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, gemv_kernel<F, K, B>, kThreads, smem);
-    if (e != cudaSuccess) return e;
-    occ[dev] = n < 1 ? 1 : n;
-    occ_smem[dev] = smem;
-  }
-  int64_t grid = static_cast<int64_t>(sms) * occ[dev];
+  int occ = 0;
+  cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&occ, gemv_kernel<F, K, B>, kThreads, smem);
+  if (e != cudaSuccess) return e;
+  int64_t grid = static_cast<int64_t>(sms) * (occ < 1 ? 1 : occ);
   if (grid > kMaxGemvGrid) grid = kMaxGemvGrid;
   if (grid > p.total_blocks) grid = p.total_blocks;
   gemv_split(p, static_cast<int>(grid));
   gemv_kernel<F, K, B><<<p.grid, kThreads, smem, stream>>>(p, nb, act_floats);
   return cudaGetLastError();
+}
+
+template <int F, int K, int B>
+cudaError_t prepare_fkb() {
+  return cudaFuncSetAttribute(gemv_kernel<F, K, B>, cudaFuncAttributeMaxDynamicSharedMemorySize, kMaxSmem);
+}
+
+template <int F, int K>
+cudaError_t prepare_fk() {
+  cudaError_t e;
+  if ((e = prepare_fkb<F, K, 1>())) return e;
+  if ((e = prepare_fkb<F, K, 2>())) return e;
+  if ((e = prepare_fkb<F, K, 4>())) return e;
+  if constexpr (max_rows_per_launch(K) > 4) return prepare_fkb<F, K, 8>();
+  return cudaSuccess;
+}
+
+// Once per device: every kernel of one format may take up to kMaxSmem bytes.
+template <int F>
+cudaError_t prepare_format() {
+  cudaError_t e;
+  if ((e = prepare_fk<F, 1>())) return e;
+  if ((e = prepare_fk<F, 2>())) return e;
+  if ((e = prepare_fk<F, 3>())) return e;
+  return prepare_fk<F, 4>();
 }
 
 template <int F, int K>

@@ -3,6 +3,8 @@
 
 namespace rrq {
 
+cudaError_t gemv_prepare_sym_f32() { return prepare_format<kSymF32>(); }
+
 cudaError_t gemv_launch_sym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms) {
   return launch_format<kSymF32>(k, nb, max_cols, p, stream, sms);
 }

@@ -78,7 +78,10 @@ constexpr int kPfBarOffset = kPfCOffset + kPfCStages * kPfCStageBytes;
 // full_w, empty_w per weight stage; full_a, empty_a per activation stage;
 // full_c, empty_c per code stage; acc_full; drain; share_done per weight stage
 constexpr int kPfBars = 2 * kPfWStages + 2 * kPfAStages + 2 * kPfCStages + 2 + kPfWStages;
-constexpr int kPfSmemBytes = kPfBarOffset + 8 * kPfBars + 16 + 1024;  // + TMEM address, alignment slack
+// after the barriers: the TMEM address (16 bytes), then for clusters the
+// stages each CTA sent to this one [4] and the stages this CTA's MMA thread
+// consumed (32 bytes), and alignment slack
+constexpr int kPfSmemBytes = kPfBarOffset + 8 * kPfBars + 16 + 32 + 1024;
 
 // Instruction descriptor of tcgen05.mma .kind::f16: D binary32 (bits 4-5),
 // A and B bf16 (bits 7-9, 10-12), both K-major (bits 15, 16 clear),
@@ -129,6 +132,16 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
 }
 __device__ __forceinline__ void mbar_arrive(uint32_t bar) {
   asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+// Counts `bytes` of the barrier's current phase as arrived without a copy
+// (settles an expectation that no copy will meet).
+__device__ __forceinline__ void mbar_complete_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.complete_tx.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+// 32-bit store into the shared memory of a CTA of the cluster (address from
+// cluster_addr).
+__device__ __forceinline__ void st_cluster_u32(uint32_t addr, uint32_t v) {
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(addr), "r"(v) : "memory");
 }
 // Cluster forms: the address of the same shared-memory offset in CTA `rank`
 // of the cluster, an MMA commit that arrives on the barrier at the same
@@ -350,6 +363,11 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   const uint32_t drain = acc_full + 8;
   const uint32_t slot_s = bar_s + 8 * kPfBars;  // (after share_done)
   const volatile uint32_t* slot = reinterpret_cast<const volatile uint32_t*>(base + kPfBarOffset + 8 * kPfBars);
+  // clusters: sent_in[d] = stages CTA d sent into this CTA's weight ring
+  // (written by d's share warp at its end), sent_in[4] = stages this CTA's
+  // MMA thread consumed
+  volatile uint32_t* const sent_in = reinterpret_cast<volatile uint32_t*>(base + kPfBarOffset + 8 * kPfBars + 16);
+  const uint32_t sent_in_s = slot_s + 16;
   auto full_w = [&](int s) { return bar_s + 8 * s; };
   auto empty_w = [&](int s) { return bar_s + 8 * (kPfWStages + s); };
   auto full_a = [&](int s) { return bar_s + 8 * (2 * kPfWStages + s); };
@@ -396,6 +414,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     }
     mbar_init(acc_full, 1);
     mbar_init(drain, 1);
+    for (int d = 0; d < 5; ++d) sent_in[d] = 0u;
     fence_mbarrier_init();
   }
   if (warp == kPfMmaWarp) {
@@ -459,6 +478,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   } else if (warp == kPfMmaWarp) {
     if (lane == 0) {
       bool ok = true;
+      int consumed = 0;  // weight stages whose full barrier this thread passed
       for (int kb = 0; kb < nk; ++kb) {
         const int sw = kb % kPfWStages, sa = kb % kPfAStages;
         if ((active && !pf_wait(full_a(sa), (kb / kPfAStages) & 1, p.wait_limit_us)) ||
@@ -466,6 +486,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
           ok = false;
           break;
         }
+        consumed = kb + 1;
         tc_fence_after();
         if (active) {
           const uint32_t wa = w_s + sw * kPfWTileBytes, aa = a_s + sa * kPfATileBytes;
@@ -482,6 +503,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
         else mma_commit(empty_w(sw));
         if (active) mma_commit(empty_a(sa));
       }
+      if constexpr (CS > 1) sent_in[4] = static_cast<uint32_t>(consumed);
       if (ok) {
         if (active) mma_commit(acc_full);
       } else {  // no MMA may be in flight when the tensor memory is freed
@@ -498,6 +520,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
     if constexpr (CS > 1) {
       if (lane == 0) {
         constexpr uint32_t kBytes = kRows * 128;  // contiguous rows of the swizzled tile
+        uint32_t sent = 0;
         for (int kb = 0; kb < nk; ++kb) {
           const int s = kb % kPfWStages;
           if (!pf_wait(share_done(s), (kb / kPfWStages) & 1, p.wait_limit_us)) {
@@ -509,7 +532,12 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
           for (int d = 0; d < CS; ++d)
             if (d != rank) bulk_copy_cluster(cluster_addr(src, d), src, kBytes, cluster_addr(full_w(s), d));
           mbar_arrive_expect_tx(full_w(s), (CS - 1) * kBytes);
+          sent = static_cast<uint32_t>(kb + 1);
         }
+        // every CTA learns how many stages went into it (read after the
+        // first of the two final cluster barriers)
+#pragma unroll
+        for (int d = 0; d < CS; ++d) st_cluster_u32(cluster_addr(sent_in_s + 4 * rank, d), sent);
       }
     }
     __syncwarp();
@@ -680,7 +708,37 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   }
   tc_fence_before();
   __syncthreads();
-  if constexpr (CS > 1) cluster_sync();  // no CTA leaves while another may still write into it
+  if constexpr (CS > 1) {
+    cluster_sync();  // every CTA's sent counts are in place
+    // After a timeout, the other CTAs may have sent weight rows into stages
+    // this CTA's MMA thread never consumed; their bulk copies complete on
+    // this CTA's full barriers.  Settle each such stage's expected bytes to
+    // what was actually sent (this CTA's share warp expected every other
+    // CTA's rows for the stages it sent itself), then wait (bounded) for
+    // the phase, so that no copy lands after this CTA has left.  Pending
+    // stages span fewer than kPfWStages (a CTA sends stage kb only after
+    // every MMA thread of the cluster consumed kb - kPfWStages), so each
+    // slot has at most one open phase.
+    if (threadIdx.x == 0 && sent_in[4] < static_cast<uint32_t>(nk)) {
+      constexpr uint32_t kBytes = kRows * 128;
+      const uint32_t own = sent_in[rank];
+      uint32_t most = own;
+      for (int d = 0; d < CS; ++d) most = sent_in[d] > most ? sent_in[d] : most;
+      for (uint32_t kb = sent_in[4]; kb < most; ++kb) {
+        uint32_t m = 0;  // other CTAs that sent stage kb
+        for (int d = 0; d < CS; ++d) m += (d != rank && sent_in[d] > kb) ? 1u : 0u;
+        const uint32_t bar = full_w(static_cast<int>(kb % kPfWStages));
+        if (kb < own) {
+          if (m < CS - 1) mbar_complete_tx(bar, (CS - 1 - m) * kBytes);
+        } else {
+          if (m == 0) continue;  // nothing was sent into this stage
+          mbar_arrive_expect_tx(bar, m * kBytes);
+        }
+        mbar_wait(bar, (kb / kPfWStages) & 1, kDrainLimitUs);
+      }
+    }
+    cluster_sync();  // no CTA leaves while another may still write into it
+  }
   if (warp == kPfMmaWarp) {
     tc_fence_after();
     tmem_dealloc(tmem, kPfTmemCols);

@@ -91,6 +91,8 @@
 // quantize_emit.cu the build that also writes every prefix.
 #pragma once
 
+#include <atomic>
+
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -832,12 +834,16 @@ __host__ __device__ constexpr int smem_bytes() {
 
 template <int G, int F, int M>
 cudaError_t launch_gf(const QuantizeBatch& p, cudaStream_t stream, int sms) {
-  static int blocks_per_sm = 0;  // same for every device of this build
+  // resident CTAs per multiprocessor: the same for every device of this
+  // build, asked once (an atomic: any thread may launch)
+  static std::atomic<int> cached{0};
+  int blocks_per_sm = cached.load(std::memory_order_relaxed);
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
         &blocks_per_sm, quantize_kernel<G, F, M>, kThreads, smem_bytes<M>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
+    cached.store(blocks_per_sm, std::memory_order_relaxed);
   }
   const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;

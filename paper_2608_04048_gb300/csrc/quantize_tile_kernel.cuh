@@ -23,6 +23,8 @@
 // matrix descriptor.
 #pragma once
 
+#include <atomic>
+
 #include "quantize_kernel.cuh"
 
 namespace rrq {
@@ -457,13 +459,17 @@ __global__ void __launch_bounds__(kTileThreads, RRQ_TILE_CTAS_PER_SM) quantize_t
 
 template <int G, int F, int LW>
 cudaError_t tile_launch_gf(const QuantizeTileBatch& p, cudaStream_t stream, int sms) {
-  static int blocks_per_sm = 0;  // same for every device of this build
+  // resident CTAs per multiprocessor: the same for every device of this
+  // build, asked once (an atomic: any thread may launch)
+  static std::atomic<int> cached{0};
+  int blocks_per_sm = cached.load(std::memory_order_relaxed);
   if (blocks_per_sm == 0) {
     int n = 0;
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, quantize_tile_kernel<G, F, LW>, kTileThreads,
                                                                   tile_smem_bytes<LW>());
     if (e != cudaSuccess) return e;
     blocks_per_sm = n < 1 ? 1 : n;
+    cached.store(blocks_per_sm, std::memory_order_relaxed);
   }
   const int64_t want = (p.b.total_chunks + kTileWarps - 1) / kTileWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;

@@ -37,6 +37,8 @@
 // each instantiate one package format (they compile in parallel).
 #pragma once
 
+#include <atomic>
+
 #include <cuda_bf16.h>
 #include <cuda_fp16.h>
 
@@ -261,12 +263,16 @@ __global__ void __launch_bounds__(kThreads, 2) reconstruct_kernel(const __grid_c
 
 template <int G, int K, bool A, int F>
 cudaError_t launch_gk(const ReconstructBatch& p, cudaStream_t stream, int sms) {
-  static int blocks_per_sm = 0;
+  // resident CTAs per multiprocessor: the same for every device of this
+  // build, asked once (an atomic: any thread may launch)
+  static std::atomic<int> cached{0};
+  int blocks_per_sm = cached.load(std::memory_order_relaxed);
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(
         &blocks_per_sm, reconstruct_kernel<G, K, A, F>, kThreads, smem_bytes<K, F>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
+    cached.store(blocks_per_sm, std::memory_order_relaxed);
   }
   const int64_t want = (p.total_chunks + kWarps - 1) / kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;

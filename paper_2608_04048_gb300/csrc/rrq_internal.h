@@ -254,6 +254,21 @@ cudaError_t gemv_launch_sym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, c
 cudaError_t gemv_launch_sym_f16(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms);
 cudaError_t gemv_launch_asym_bits(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms);
 
+// Once per device: the decode product's kernels may take the shared memory
+// their largest launch needs.
+cudaError_t gemv_prepare_asym_f32();
+cudaError_t gemv_prepare_sym_f32();
+cudaError_t gemv_prepare_sym_f16();
+cudaError_t gemv_prepare_asym_bits();
+
+inline cudaError_t gemv_prepare() {
+  cudaError_t e;
+  if ((e = gemv_prepare_asym_f32())) return e;
+  if ((e = gemv_prepare_sym_f32())) return e;
+  if ((e = gemv_prepare_sym_f16())) return e;
+  return gemv_prepare_asym_bits();
+}
+
 inline cudaError_t gemv_launch(Format fmt, int k, int nb, int64_t max_cols, GemvBatch& p,
                                cudaStream_t stream, int sms) {
   switch (fmt) {
