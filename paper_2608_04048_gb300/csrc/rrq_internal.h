@@ -87,6 +87,15 @@ struct ReconstructBatch {
 // weights of the package's first k stages.  Each matrix's rows are cut into
 // blocks of 16; the blocks of all matrices of a launch are numbered
 // consecutively and blk_begin is this matrix's first.
+// The wide-lane reconstruction at one prefix (reconstruct_tile_kernel.cuh):
+// each matrix's bf16 output as the 2-D tensor map [n / 64, 64] (one 32-row
+// box = one warp chunk of 2048 weights), and the batch with chunk_begin /
+// total_chunks counted in those chunks.
+struct ReconstructTileBatch {
+  CUtensorMap out[kMaxBatch];
+  ReconstructBatch b;
+};
+
 struct GemvItem {
   const uint8_t* codes[kMaxStages];
   const void* scales[kMaxStages];  // float or binary16

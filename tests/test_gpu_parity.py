@@ -155,21 +155,30 @@ def test_guard_bands_untouched():
 def test_timeout_path_reports_and_recovers():
     """A wait limit of 0 makes every bounded wait give up at once: the kernel
     records RRQ_ERR_TIMEOUT, drains its own copies and returns; the device
-    stays usable and the next call is exact again."""
-    W = workloads.generate(512, 1024, 21, "normal", "cuda")
+    stays usable and the next call is exact again.  Both builds (the 2-D
+    tile form and the 1-D ring form) and the one-prefix reconstruction of a
+    whole number of 2048-weight chunks wait on their bulk copies; the
+    reconstruction of other sizes has no bounded waits."""
+    W = workloads.generate(512, 1024, 21, "normal", "cuda")      # tile forms
+    V = workloads.generate(3, 1024 + 32, 22, "normal", "cuda")   # 1-D forms (n % 64 != 0)
     binding.rrq_get_device_status()  # clear
     pkg = binding.rrq_quantize(W, 128, 4)
+    pkv = binding.rrq_quantize(V, 32, 4)
     binding.rrq_set_wait_limit_us(0)
     try:
         binding.rrq_quantize(W, 128, 4)
         assert binding.rrq_get_device_status() == 5
-        # reconstruction has no bounded waits (its copies complete in hardware)
-        out = binding.rrq_reconstruct(pkg, 4)
+        binding.rrq_quantize(V, 32, 4)
+        assert binding.rrq_get_device_status() == 5
+        binding.rrq_reconstruct(pkg, 4)
+        assert binding.rrq_get_device_status() == 5
+        binding.rrq_reconstruct(pkv, 4)  # cp.async copies complete in hardware
         assert binding.rrq_get_device_status() == 0
     finally:
         binding.rrq_set_wait_limit_us(1_000_000)
     assert binding.rrq_get_device_status() == 0
     check_full(W, 128, 4, where="after timeout")
+    check_full(V, 32, 4, where="after timeout, 1-D forms")
 
 
 def test_bad_pointers_rejected_on_device():
