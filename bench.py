@@ -619,7 +619,10 @@ def run_gpu(args, world, rank, local) -> dict | None:
 
     # breakdown: the package alone (rrq_quantize), every prefix from the
     # package, and each prefix by its own call
-    q_s = time_calls(wl.quantize_calls(), stream, 3, flush)
+    q_calls = wl.quantize_calls()
+    q_s = time_calls(q_calls, stream, 3, flush)
+    groups = sorted({sp.group for sp in specs})
+    q_by_group = {g: time_calls([c], stream, 3, flush) for g, c in zip(groups, q_calls)} if len(groups) > 1 else None
     r_s = time_calls(wl.reconstruct_calls(None), stream, 3, flush)
     each_k = {k: time_calls(wl.reconstruct_calls(k), stream, 2, flush) for k in KS}
     torch.cuda.synchronize()
@@ -663,7 +666,8 @@ def run_gpu(args, world, rank, local) -> dict | None:
     traffic = recorded_traffic("rrq_quantize_prefixes", f_alg / launches, f_alg / launches) \
         if args.workload in TRAFFIC_WORKLOADS else None
     rooflines = {
-        "rrq_quantize": roofline_entry("quantize_kernel<g,0,0>: rrq_quantize_batch, the package only", q_alg, q_s,
+        "rrq_quantize": roofline_entry("quantize_tile_kernel<g,0,64> (n % 64 == 0; else quantize_kernel<g,0,0>): "
+                                       "rrq_quantize_batch, the package only", q_alg, q_s,
                                        hbm, q_launches,
                                        "rrq_quantize" if args.workload in TRAFFIC_WORKLOADS else None),
         "rrq_reconstruct_prefixes": roofline_entry(
@@ -672,8 +676,9 @@ def run_gpu(args, world, rank, local) -> dict | None:
     }
     for k in KS:
         rooflines[f"rrq_reconstruct_k{k}"] = roofline_entry(
-            f"reconstruct_kernel<g,{k},0,0>: rrq_reconstruct_batch at prefix k={k}", k_alg[k], each_k[k], hbm,
-            launches, None)
+            f"reconstruct_tile_kernel<g,{k},0> (whole 2048-weight chunks; else reconstruct_kernel<g,{k},0,0>): "
+            f"rrq_reconstruct_batch at prefix k={k}", k_alg[k], each_k[k], hbm, launches,
+            "rrq_reconstruct_k4" if k == 4 and args.workload in TRAFFIC_WORKLOADS else None)
     l2_text = (f"L2 flushed ({2 * L2_BYTES // 2**20} MiB write) before every timed call" if flush is not None else
                f"inputs {2 * n_total / 1e9:.2f} GB per rank, larger than the {L2_BYTES // 2**20} MiB L2; no flush")
     line = {
@@ -716,6 +721,11 @@ def run_gpu(args, world, rank, local) -> dict | None:
             "reconstruct_frac_of_measured_hbm": round(r_alg / r_s / 1e9 / hbm, 4),
             "reconstruct_separate_k1to4_s": round(sum(each_k.values()), 6),
             "reconstruct_separate_alg_gbs": round(sum(k_alg.values()) / sum(each_k.values()) / 1e9, 1),
+            "quantize_by_group": None if q_by_group is None else {
+                f"g{g}": {"s": round(t, 6), "alg_gbs": round(a / t / 1e9, 1), "frac_of_measured_hbm": round(a / t / 1e9 / hbm, 4),
+                          "frac_of_nominal_8tbs": round(a / t / 1e9 / 8000.0, 4)}
+                for g, t in q_by_group.items()
+                for a in [sum(alg_bytes_quantize(sp.numel, g) for sp in specs if sp.group == g)]},
             "paper_context_s": {"full_all_rtn_package_qwen3_8b_a100": 1293, "four_rtn_passes_a100": 412},
             "sym_f16": sym,
             "from_base": from_base,
@@ -766,14 +776,58 @@ def recorded_traffic(kernel: str, q_bytes_per_launch: float, r_bytes_per_launch:
 
 # the source files each recorded kernel is compiled from
 KERNEL_SOURCES = {
-    "rrq_quantize": ["quantize_kernel.cuh", "quantize.cu"],
-    "rrq_quantize_ex_sym_f16": ["quantize_kernel.cuh", "quantize.cu"],
-    "rrq_reconstruct_prefixes": ["reconstruct_kernel.cuh", "reconstruct_asym_f32.cu"],
-    "rrq_reconstruct_ex_sym_f16": ["reconstruct_kernel.cuh", "reconstruct_sym_f16.cu"],
+    "rrq_quantize": ["quantize_tile_kernel.cuh", "quantize_kernel.cuh", "quantize.cu"],
+    "rrq_quantize_ex_sym_f16": ["quantize_tile_kernel.cuh", "quantize_kernel.cuh", "quantize.cu"],
+    "rrq_reconstruct_prefixes": ["reconstruct_kernel.cuh", "reconstruct_tile_kernel.cuh", "reconstruct_asym_f32.cu"],
+    "rrq_reconstruct_k4": ["reconstruct_kernel.cuh", "reconstruct_tile_kernel.cuh", "reconstruct_asym_f32.cu"],
+    "rrq_reconstruct_ex_sym_f16": ["reconstruct_kernel.cuh", "reconstruct_tile_kernel.cuh", "reconstruct_sym_f16.cu"],
     "rrq_quantize_prefixes": ["quantize_kernel.cuh", "quantize_emit.cu"],
     "rrq_gemv_k1": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
     "rrq_gemv_k4": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
 }
+
+# the kernel (ncu demangled-name prefix) and algorithmic bytes per weight at
+# group 128 behind each recorded entry
+TRAFFIC_KERNELS = {
+    "rrq_quantize": ("quantize_tile_kernel<128, 0,", 3.25),
+    "rrq_quantize_ex_sym_f16": ("quantize_tile_kernel<128, 2,", 2 + 4 * (0.25 + 2 / 128)),
+    "rrq_reconstruct_prefixes": ("reconstruct_kernel<128, 4, 1, 0>", 9.25),
+    "rrq_reconstruct_k4": ("reconstruct_tile_kernel<128, 4, 0>", 3.25),
+    "rrq_quantize_prefixes": ("quantize_kernel<128, 0, 2>", 11.25),
+}
+
+
+def record_traffic(csv_path: str, workload: str = "qwen3_8b_layer"):
+    """Writes profiles/traffic.json from an ncu CSV (--metrics
+    dram__bytes_read.sum,dram__bytes_write.sum --csv --log-file) of a bench.py
+    run on `workload`: for each recorded kernel its first launch's DRAM bytes,
+    the algorithmic bytes of one launch over the workload, and the SHA-256 of
+    its sources."""
+    import csv
+    from paper_2608_04048_gb300 import workloads
+    n = sum(sp.numel for sp in workloads.config_matrices(workload))
+    rows = list(csv.DictReader(line for line in open(csv_path) if line.startswith('"')))
+    launches = {}
+    for r in rows:
+        key = (r["ID"], r["Kernel Name"])
+        launches.setdefault(key, {})[r["Metric Name"]] = (float(r["Metric Value"].replace(",", "")), r["Metric Unit"])
+    unit = {"byte": 1, "Kbyte": 1e3, "Mbyte": 1e6, "Gbyte": 1e9}
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    rec = json.load(open(path)) if os.path.exists(path) else {}
+    for name, (prefix, per_weight) in TRAFFIC_KERNELS.items():
+        for (lid, kname), m in sorted(launches.items(), key=lambda x: int(x[0][0])):
+            if prefix in kname:
+                dram = sum(v * unit[u] for k, (v, u) in m.items() if k in ("dram__bytes_read.sum", "dram__bytes_write.sum"))
+                rec[name] = {"dram_bytes": int(dram), "alg_bytes": int(per_weight * n),
+                             "capture": f"{kname.split('(rrq')[0].replace('void rrq::<unnamed>::', '').strip()}: "
+                                        f"launch {lid} of bench.py --workload "
+                                        f"{workload} ({n:,} weights), ncu dram__bytes_read.sum + dram__bytes_write.sum",
+                             "source_sha256": kernel_source_hash(name),
+                             "dram_over_alg": round(dram / (per_weight * n), 4)}
+                break
+    with open(path, "w") as f:
+        json.dump(rec, f, indent=1)
+        f.write("\n")
 
 
 def kernel_source_hash(kernel: str) -> str:
@@ -985,9 +1039,14 @@ def main(argv=None):
                     help="skip the symmetric binary16, base-checkpoint and product breakdown")
     ap.add_argument("--cpu-seconds", type=float, default=20.0,
                     help="core-seconds of oracle work in the CPU baseline (0 skips it)")
+    ap.add_argument("--traffic-from", default=None,
+                    help="write profiles/traffic.json from this ncu CSV of a qwen3_8b_layer run, and exit")
     ap.add_argument("--gemv-batches", default="1",
                     help="comma-separated activation-row counts for the decode-product breakdown (1..8)")
     args = ap.parse_args(argv)
+    if args.traffic_from:
+        record_traffic(args.traffic_from)
+        return
 
     world, rank, local = dist_env()
     if world > 1:
