@@ -488,7 +488,8 @@ rrq_status gemv_batch(const rrq_gemv_desc* items, int count, const Fmt& f, int k
   // does not split the batch of the narrower ones
   std::vector<int> per(count), order(count);
   for (int i = 0; i < count; ++i) {
-    const int cap = rrq::gemv_rows_per_launch(f.kind, k, items[i].cols);
+    if (items[i].cols > RRQ_MAX_GEMV_COLS) return RRQ_ERR_UNSUPPORTED;  // the stated limit of every form
+    const int cap = rrq::gemv_rows_per_launch(f.kind, k, items[i].cols, group);
     if (cap < 1) return RRQ_ERR_UNSUPPORTED;
     per[i] = std::min(cap, batch);
     order[i] = i;

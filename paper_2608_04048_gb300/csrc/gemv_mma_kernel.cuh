@@ -1,0 +1,535 @@
+// Stage-wise product for decoding on the tensor cores, in the per-group
+// factored form of Appendix C's A W~ = A W_0 + sum_k A R_k.  Within one group
+// g of one stage k every weight is lo + Q s (asymmetric grid) or (Q - 2) s
+// (symmetric), so
+//     sum_{c in g} w_c a_c = s_kg * D_kg + lo_kg * S_g      (asymmetric)
+//                          = s_kg * (D_kg - 2 S_g)          (symmetric)
+// with D_kg = sum_{c in g} Q_c a_c over the integer codes and S_g = sum_{c in g}
+// a_c.  The kernel forms D_kg with bf16 MMAs (mma.sync m16n8k16, binary32
+// accumulation), the codes entering as the exact bf16 values 0..3, and sums
+// the groups' terms per row.  It never forms the binary32 prefix weights W~;
+// the result differs from A W~ by the rounding of the stage levels and of
+// the sums (bounded below).
+//
+// Layout.  A CTA of 16 warps takes a contiguous range of 16-row blocks
+// (gemv_split), matrix by matrix; a warp takes whole blocks (w, w + 16, ...
+// of the CTA's blocks of a matrix).  A block is walked stage by stage, each
+// stage in spans of kSpan = max(512, G) columns: the item (block, stage,
+// span) is 16 rows x kSpan/4 contiguous bytes of codes per row -- whole
+// 128-byte lines, so that each DRAM page opened for a row serves a whole
+// line, not the 32 bytes of one group -- and the rows' scales and zeros of
+// the span's groups.  The warp's lanes copy items with cp.async into a ring
+// of D slots of the warp's own in shared memory, D - 1 items ahead of the one
+// it multiplies (rows padded so that the fragment reads below hit distinct
+// banks).  Within a group, lane l (t = l % 4, rq = l / 4) takes the codes of
+// rows rq and rq + 8 of the block for the columns [t G/4, (t + 1) G/4) of the
+// group: G/64 words of 16 codes per row.  One MMA takes, for each lane, the
+// codes at bit offset 2e (e = 0..3) of the four bytes of one word: bytes 0
+// and 2 (one register: the code field masked in place under the bf16
+// exponent of 128, i.e. 128 + 4^e Q, brought to Q by one exact bf16x2 fma)
+// as k = 2t, 2t + 1, bytes 1 and 3 as k = 2t + 8, 2t + 9.  The permutation of
+// K this implies is applied to the activations: per matrix the CTA writes
+// them once, as bf16, into shared memory in exactly the B-fragment order of
+// every MMA (each lane then reads 8 bytes per MMA), with the group sums S_g
+// next to them.  Activation rows n >= nb of the launch are zero in B.  The
+// accumulator rows are the block's rows and its columns the activation rows:
+// lane l holds rows rq, rq + 8 for activation rows 2t, 2t + 1.
+//
+// Accuracy (binary32, round to nearest; the tensor cores' accumulation is
+// assumed to round each k16 step once, as for the prefill product): the
+// result differs from the oracle's binary64 sum of A W~ by at most
+//     d * 2^-24 * sum_c sum_k (|lo_k| + 3 s_k) |a_c|     (asymmetric)
+//     d * 2^-24 * sum_c sum_k 2 s_k |a_c|                 (symmetric)
+// with d = (k + 1) + G/16 + 8 + 2k groups + 18: the stage levels and their
+// sum that W~ rounds (k + 1), the G/16 MMA steps of D, the sum S_g (a sum of
+// 8 then a tree over G/8, at most 8 roundings at G = 256), two fma per group
+// and stage into the row's sum, and slack (18).
+#pragma once
+
+#include <cuda_bf16.h>
+
+#include "gemv_kernel.cuh"
+
+namespace rrq {
+namespace {
+
+constexpr int kMmaWarps = 16;
+constexpr int kMmaThreads = kMmaWarps * 32;
+constexpr int kMmaRingMax = 4;  // slots of a warp's ring at most
+constexpr int kMmaSmemMax = kMaxSmem - 128;  // dynamic shared memory (the kernel has 32 static bytes)
+
+// The item geometry for groups of G columns: kSpan columns (kL groups) per
+// item; a slot row holds the span's codes (kSpan / 4 bytes) and a pad that
+// puts the rows rq = 0..7 (G = 64: 4-byte reads), 0..3 (G = 128: 8-byte) or
+// 0..1 (G = 256: 16-byte reads) of one read phase on distinct banks.
+template <int G>
+struct MmaGeom {
+  static constexpr int kSpan = G > 512 ? G : 512;
+  static constexpr int kL = kSpan / G;
+  static constexpr int kPitch = kSpan / 4 + (G == 64 ? 16 : G == 128 ? 32 : 64);
+};
+__host__ __device__ constexpr int mma_pitch(int G) { return (G > 512 ? G : 512) / 4 + (G == 64 ? 16 : G == 128 ? 32 : 64); }
+__host__ __device__ constexpr int mma_groups_per_item(int G) { return (G > 512 ? G : 512) / G; }
+// one ring slot: 16 rows of codes, then the 16 x kL scales (binary32, or the
+// aligned binary16 pair holding the scale) and, on the asymmetric grid, the
+// 16 x kL zeros
+__host__ __device__ constexpr int mma_slot_bytes(bool sym, int G) {
+  return kGemvRows * mma_pitch(G) + (sym ? 1 : 2) * kGemvRows * mma_groups_per_item(G) * 4;
+}
+
+// shared memory of the per-matrix tables: per activation row, B fragments
+// (cols bf16, two MMAs' fragments of a lane in 16 bytes) and 64 bytes of pad
+// (rows 2 apart start on other banks), then per row the group sums (cols / G
+// floats, rounded up to 4); the whole rounded up to 128 bytes
+__host__ __device__ constexpr int64_t mma_brow_bytes(int64_t cols) { return cols * 2 + 64; }
+__host__ __device__ constexpr int64_t mma_srow_floats(int64_t cols, int G) { return (cols / G + 3) / 4 * 4; }
+__host__ __device__ constexpr int64_t mma_table_bytes(int64_t cols, int nb, int G) {
+  return (nb * mma_brow_bytes(cols) + nb * mma_srow_floats(cols, G) * 4 + 127) / 128 * 128;
+}
+// ring slots a launch gives each warp: up to kMmaRingMax within what the
+// tables leave of the shared memory (0 if not even 2 fit)
+__host__ __device__ constexpr int mma_ring_slots(bool sym, int G, int64_t table_bytes, int64_t smem_max) {
+  const int64_t fit = (smem_max - table_bytes) / (kMmaWarps * static_cast<int64_t>(mma_slot_bytes(sym, G)));
+  const int64_t d = fit < kMmaRingMax ? fit : kMmaRingMax;
+  return d < 2 ? 0 : static_cast<int>(d);
+}
+
+// wait until at most n (< kMmaRingMax) of this thread's cp.async groups are pending
+__device__ __forceinline__ void cp_async_wait_n(int n) {
+  if (n <= 1) cp_async_wait<1>();
+  else if (n == 2) cp_async_wait<2>();
+  else cp_async_wait<3>();
+}
+
+__device__ __forceinline__ void mma_bf16_16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0, %1, %2, %3}, {%4, %5, %6, %7}, {%8, %9}, "
+      "{%0, %1, %2, %3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+}
+
+// The code field at bit 2f (f <= 2) of a half, masked with the exponent bits
+// clear, is the bf16 subnormal 4^f Q 2^-133 (exact: the tensor cores take
+// subnormal bf16 operands as they are).  Register r of MMA e takes bytes 0, 2
+// (r = 0) or 1, 3 (r = 1) of the lane's word at code offset e from the word or
+// its shifts by 6 and 12; frag_f gives its f.  The B fragment of that register
+// carries b 2^(k - 2f), so that each product is Q b 2^(k - 133).
+__host__ __device__ constexpr int frag_f(int e, int r) {
+  return r == 0 ? (e == 3 ? 0 : e) : (e == 2 ? 0 : e == 3 ? 1 : e + 1);
+}
+template <int E>
+__device__ __forceinline__ void a_frag(uint32_t w0, uint32_t w1, uint32_t x6_0, uint32_t x6_1, uint32_t x12_0,
+                                       uint32_t x12_1, uint32_t (&a)[4]) {
+  constexpr uint32_t M0 = 0x00030003u, M1 = 0x000C000Cu, M2 = 0x00300030u;  // f = 0, 1, 2 in both halves
+  if constexpr (E == 0) {         // bytes 0, 2 bits 0-1 (w);  bytes 1, 3 bits 0-1 (w >> 6, f = 1)
+    a[0] = w0 & M0; a[1] = w1 & M0; a[2] = x6_0 & M1; a[3] = x6_1 & M1;
+  } else if constexpr (E == 1) {  // bits 2-3 (w, f = 1);      bits 2-3 (w >> 6, f = 2)
+    a[0] = w0 & M1; a[1] = w1 & M1; a[2] = x6_0 & M2; a[3] = x6_1 & M2;
+  } else if constexpr (E == 2) {  // bits 4-5 (w, f = 2);      bits 4-5 (w >> 12, f = 0)
+    a[0] = w0 & M2; a[1] = w1 & M2; a[2] = x12_0 & M0; a[3] = x12_1 & M0;
+  } else {                        // bits 6-7 (w >> 6, f = 0); bits 6-7 (w >> 12, f = 1)
+    a[0] = x6_0 & M0; a[1] = x6_1 & M0; a[2] = x12_0 & M1; a[3] = x12_1 & M1;
+  }
+}
+
+// N consecutive 4-byte words of shared memory (N = 2: 8-byte aligned; N = 4:
+// 16-byte aligned) into registers, one read
+template <int N, typename T>
+__device__ __forceinline__ void lds_vec(const void* p, T (&v)[N]) {
+  static_assert(sizeof(T) == 4 && (N == 2 || N == 4), "two or four words");
+  if constexpr (N == 2) {
+    const uint2 x = *reinterpret_cast<const uint2*>(p);
+    v[0] = __builtin_bit_cast(T, x.x); v[1] = __builtin_bit_cast(T, x.y);
+  } else {
+    const uint4 x = *reinterpret_cast<const uint4*>(p);
+    v[0] = __builtin_bit_cast(T, x.x); v[1] = __builtin_bit_cast(T, x.y);
+    v[2] = __builtin_bit_cast(T, x.z); v[3] = __builtin_bit_cast(T, x.w);
+  }
+}
+
+template <int F, int K, int G>
+__global__ void __launch_bounds__(kMmaThreads, 1)
+gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D) {
+  constexpr bool kSym = F == kSymF32 || F == kSymF16;
+  constexpr bool kF16 = F == kSymF16;
+  constexpr int W = G / 64;  // words of 16 codes per lane, row and group
+  using Geo = MmaGeom<G>;
+  constexpr int kSpan = Geo::kSpan, kL = Geo::kL, kPitch = Geo::kPitch;
+  static_assert(kSpan / 4 == 128, "two lanes copy a row's 128 bytes of codes");
+  constexpr int kCodes = kGemvRows * kPitch;   // a slot's codes
+  constexpr int kSlot = mma_slot_bytes(kSym, G);
+  extern __shared__ __align__(16) uint8_t smem[];
+  const int lane = threadIdx.x & 31;
+  const int warp = threadIdx.x >> 5;
+  const int t = lane & 3, rq = lane >> 2;
+  const int64_t blk_begin = p.cta_begin[blockIdx.x];
+  const int64_t blk_end = p.cta_begin[blockIdx.x + 1];
+  if (blk_begin >= blk_end) return;  // the whole CTA: no barrier is reached
+
+  int m_cur = -1;
+  int64_t cols = 0, ngroups = 0;
+  uint4* btab = nullptr;
+  float* stab = nullptr;
+  int64_t srow = 0;  // floats per row of the group sums
+
+  // B fragments and group sums of matrix m, per activation row n: for column
+  // c of group g, the lane quarter t = (c % G) / (G/4), word w, byte b and
+  // offset e of its code give MMA i = (g W + w) 4 + e, register b & 1, half
+  // b >> 1 of the fragment (n, i, t), stored at 16-byte unit (n, i / 2, t),
+  // 8-byte half i % 2, and holding a_c 2^(k_n - 2f); S_g 2^(k_n - 133) of row
+  // n at (n, g).  k_n = 253 - (the largest exponent field of the row's bf16
+  // activations) keeps every scaled activation below 2^127; the row sums are
+  // formed in the domain scaled by 2^(k_n - 133) and scaled back at the
+  // store.  A lane reads activation row min(rq, nb - 1) of B and the sums of
+  // rows min(2t, nb - 1), min(2t + 1, nb - 1): accumulator columns n >= nb
+  // repeat a real row and are never stored.
+  __shared__ int emax_s[kMaxGemvBatch];
+  const uint4* bt_lane = nullptr;
+  const float *sa_lane = nullptr, *sb_lane = nullptr;
+  int back0 = 0, back1 = 0;  // 133 - k of the lane's output columns 2t, 2t + 1
+  auto build_tables = [&](int m) {
+    const GemvItem& it = p.item[m];
+    cols = it.cols;
+    ngroups = cols / G;
+    const int64_t brow = mma_brow_bytes(cols) / 16;  // 16-byte units per B row
+    srow = mma_srow_floats(cols, G);
+    btab = reinterpret_cast<uint4*>(smem);
+    stab = reinterpret_cast<float*>(smem + nb * mma_brow_bytes(cols));
+    if (threadIdx.x < nb) emax_s[threadIdx.x] = 0;
+    __syncthreads();
+    for (int n = 0; n < nb; ++n) {
+      const uint16_t* a = it.A + static_cast<int64_t>(n) * cols;
+      int e = 0;
+      for (int64_t c = threadIdx.x; c < cols; c += kMmaThreads) e = max(e, (a[c] >> 7) & 0xFF);
+      e = __reduce_max_sync(0xFFFFFFFFu, e);
+      if (lane == 0) atomicMax(&emax_s[n], e);
+    }
+    __syncthreads();
+    uint16_t* bh = reinterpret_cast<uint16_t*>(btab);
+    for (int n = 0; n < nb; ++n) {
+      const uint16_t* a = it.A + static_cast<int64_t>(n) * cols;
+      const int kn = 253 - emax_s[n];
+      for (int64_t c = threadIdx.x; c < cols; c += kMmaThreads) {
+        const int64_t g = c / G;
+        const int cg = static_cast<int>(c % G);
+        const int tq = cg / (G / 4), u = cg % (G / 4);
+        const int w = u >> 4, v = u & 15, b = v >> 2, e = v & 3;
+        const int64_t mi = (g * W + w) * 4 + e;
+        const float x = scalbnf(__uint_as_float(static_cast<uint32_t>(a[c]) << 16), kn - 2 * frag_f(e, b & 1));
+        bh[(n * brow + (mi >> 1) * 4 + tq) * 8 + (mi & 1) * 4 + (b & 1) * 2 + (b >> 1)] =
+            __bfloat16_as_ushort(__float2bfloat16_rn(x));
+      }
+    }
+    // S_g: sums of 8 consecutive activations, then a tree over the G / 8
+    for (int64_t j = threadIdx.x; j < ngroups * nb; j += kMmaThreads) {
+      const int64_t g = j / nb;
+      const int n = static_cast<int>(j % nb);
+      const uint16_t* a = it.A + static_cast<int64_t>(n) * cols + g * G;
+      float s8[G / 8];
+#pragma unroll
+      for (int q = 0; q < G / 8; ++q) {
+        float s = __uint_as_float(static_cast<uint32_t>(a[8 * q]) << 16);
+#pragma unroll
+        for (int i = 1; i < 8; ++i) s = __fadd_rn(s, __uint_as_float(static_cast<uint32_t>(a[8 * q + i]) << 16));
+        s8[q] = s;
+      }
+#pragma unroll
+      for (int h = G / 16; h >= 1; h >>= 1)
+#pragma unroll
+        for (int q = 0; q < h; ++q) s8[q] = __fadd_rn(s8[q], s8[q + h]);
+      stab[n * srow + g] = scalbnf(s8[0], 120 - emax_s[n]);  // k_n - 133
+    }
+    const int bn = rq < nb ? rq : nb - 1;
+    const int n0 = 2 * t < nb ? 2 * t : nb - 1, n1 = 2 * t + 1 < nb ? 2 * t + 1 : nb - 1;
+    bt_lane = btab + bn * brow + t;
+    sa_lane = stab + n0 * srow;
+    sb_lane = stab + n1 * srow;
+    back0 = emax_s[n0] - 120;
+    back1 = emax_s[n1] - 120;
+  };
+
+  // This warp's ring: item j of its current matrix in slot j % D.
+  uint8_t* const ring = smem + ring_off + static_cast<int64_t>(warp) * D * kSlot;
+  const uint32_t ring_s = smem_u32(ring);
+
+  // The lanes' copies of item (block from row r0, stage k, span sp): piece i
+  // of a lane is the 16 bytes at part lane % 8 of row lane / 8 + 4 i of the
+  // span's codes (a warp's copy instruction covers 4 whole rows of 128
+  // bytes); entry i (e = lane + 32 i < 16 kL) is the scale (and zero) of row
+  // e / kL, group e % kL of the span.  The lane keeps its pointers per
+  // (block, stage); rows past the matrix are not copied (their sums are never
+  // stored), nor groups past the row's end.
+  constexpr int kEntries = (kGemvRows * kL + 31) / 32;
+  const uint8_t* cptr[4];           // the lane's pieces in span 0
+  const float* sptr[kEntries];      // its entries' scales (binary32) in span 0
+  const uint16_t* hptr[kEntries];   // or binary16 scales
+  const float* zptr[kEntries];      // and zeros
+  int64_t hx[kEntries];             // element index of a binary16 entry in span 0
+  bool cok[4], mok[kEntries];
+  auto set_stage = [&](const GemvItem& it, int64_t r0, int k) {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const int row = (lane >> 3) + 4 * i;
+      cok[i] = r0 + row < it.rows;
+      cptr[i] = it.codes[k] + (r0 + row) * (cols / 4) + (lane & 7) * 16;
+    }
+#pragma unroll
+    for (int i = 0; i < kEntries; ++i) {
+      const int e = lane + 32 * i;
+      const int row = e / kL, gi = e % kL;
+      mok[i] = e < kGemvRows * kL && r0 + row < it.rows;
+      const int64_t x = (r0 + row) * ngroups + gi;
+      if constexpr (kF16) {
+        hx[i] = x;
+        hptr[i] = static_cast<const uint16_t*>(it.scales[k]);
+      } else {
+        sptr[i] = static_cast<const float*>(it.scales[k]) + x;
+        if constexpr (!kSym) zptr[i] = it.zeros[k] + x;
+      }
+    }
+  };
+  auto issue = [&](const GemvItem& it, int sp, uint32_t dst) {
+    const int64_t g0 = static_cast<int64_t>(sp) * kL;
+    const int lg = ngroups - g0 < kL ? static_cast<int>(ngroups - g0) : kL;  // groups of this span
+    const int64_t cspan = g0 * (G / 4);
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      if (cok[i] && (lg == kL || (lane & 7) * 16 < lg * (G / 4)))
+        cp_async_16(dst + ((lane >> 3) + 4 * i) * kPitch + (lane & 7) * 16, cptr[i] + cspan, 16);
+#pragma unroll
+    for (int i = 0; i < kEntries; ++i) {
+      const int e = lane + 32 * i;
+      if (mok[i] && (lg == kL || e % kL < lg)) {
+        const uint32_t md = dst + kCodes + e * 4;
+        if constexpr (kF16) {  // the 4-byte aligned pair holding the scale (2 bytes at the array's end)
+          const int64_t xa = (hx[i] + g0) & ~static_cast<int64_t>(1);
+          cp_async_4(md, hptr[i] + xa, xa + 1 < it.rows * ngroups ? 4u : 2u);
+        } else {
+          cp_async_4(md, sptr[i] + g0, 4);
+          if constexpr (!kSym) cp_async_4(md + kGemvRows * kL * 4, zptr[i] + g0, 4);
+        }
+      }
+    }
+  };
+
+  // The CTA's range, matrix by matrix: the tables are built for a matrix,
+  // then each warp takes whole blocks of it (blocks w, w + 16, ...), each
+  // block stage by stage and span by span, D - 1 items in flight.
+  int m = 0;
+  while (m + 1 < p.count && blk_begin >= p.item[m + 1].blk_begin) ++m;
+  for (int64_t seg = blk_begin; seg < blk_end; ++m) {
+    const GemvItem& it = p.item[m];
+    const int64_t seg_end = m + 1 < p.count && p.item[m + 1].blk_begin < blk_end ? p.item[m + 1].blk_begin : blk_end;
+    if (m_cur >= 0) __syncthreads();  // every warp is done with the old tables
+    build_tables(m);
+    m_cur = m;
+    __syncthreads();
+    const int nspan = static_cast<int>((cols + kSpan - 1) / kSpan);
+    const int nblk = static_cast<int>((seg_end - seg - warp + kMmaWarps - 1) / kMmaWarps);  // may be <= 0
+    const int items = nblk > 0 ? nblk * K * nspan : 0;
+    // cursors (first row of the block, stage, span) of the next item to copy
+    // and of the item to multiply: a warp's blocks are 16 blocks apart
+    constexpr int64_t kRowStep = static_cast<int64_t>(kMmaWarps) * kGemvRows;
+    const int64_t r_first = (seg + warp - it.blk_begin) * kGemvRows;
+    int64_t ir = r_first;
+    int is = 0, ik = 0, left = items;
+    auto issue_next = [&](int s_dst) {
+      if (left > 0) {
+        if (is == 0) set_stage(it, ir, ik);
+        issue(it, is, ring_s + s_dst * kSlot);
+        --left;
+        if (++is == nspan) {
+          is = 0;
+          if (++ik == K) ik = 0, ir += kRowStep;
+        }
+      }
+      cp_async_commit();
+    };
+    for (int j = 0; j + 1 < D; ++j) issue_next(j);  // items 0 .. D - 2 (empty groups past the end)
+    float y[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // rows r0 (0, 1) and r0 + 8 (2, 3); activation rows 2t, 2t + 1
+    int slot = 0;  // j % D
+    int64_t cr = r_first;
+    int cs = 0, ck = 0;
+    for (int j = 0; j < items; ++j) {
+      // item j + D - 1 into the slot item j - 1 used (every lane is past it)
+      issue_next(slot == 0 ? D - 1 : slot - 1);
+      cp_async_wait_n(D - 1);  // this lane's copies of item j are done
+      __syncwarp();            // and every lane's
+      const uint8_t* sl = ring + slot * kSlot;
+      const uint32_t* ssl = reinterpret_cast<const uint32_t*>(sl + kCodes);  // [16][kL]
+      const float* zsl = reinterpret_cast<const float*>(sl + kCodes) + kGemvRows * kL;
+      const int64_t r0 = cr + rq;
+      const int64_t g0 = static_cast<int64_t>(cs) * kL;
+      const int lg = ngroups - g0 < kL ? static_cast<int>(ngroups - g0) : kL;
+      // one group of the item: D by G/16 MMAs, then the row sums with the
+      // rows' scales s0, s1, offsets o0, o1 (lo, or -2 s) and the sums sa, sb
+      auto group = [&](int gi, float s0, float s1, float o0, float o1, float sa, float sb) {
+        const int64_t g = g0 + gi;
+        // the lane's W words of rows rq and rq + 8 (one read each)
+        uint32_t c0[W], c1[W];
+        const uint8_t* cb = sl + gi * (G / 4) + t * (G / 16);
+        if constexpr (W == 1) {
+          c0[0] = *reinterpret_cast<const uint32_t*>(cb + rq * kPitch);
+          c1[0] = *reinterpret_cast<const uint32_t*>(cb + (rq + 8) * kPitch);
+        } else if constexpr (W == 2) {
+          const uint2 x0 = *reinterpret_cast<const uint2*>(cb + rq * kPitch);
+          const uint2 x1 = *reinterpret_cast<const uint2*>(cb + (rq + 8) * kPitch);
+          c0[0] = x0.x; c0[1] = x0.y;
+          c1[0] = x1.x; c1[1] = x1.y;
+        } else {
+          const uint4 x0 = *reinterpret_cast<const uint4*>(cb + rq * kPitch);
+          const uint4 x1 = *reinterpret_cast<const uint4*>(cb + (rq + 8) * kPitch);
+          c0[0] = x0.x; c0[1] = x0.y; c0[2] = x0.z; c0[3] = x0.w;
+          c1[0] = x1.x; c1[1] = x1.y; c1[2] = x1.z; c1[3] = x1.w;
+        }
+        float d[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        const uint4* bt = bt_lane + g * (W * 2 * 4);  // 16-byte units: MMA pairs x 4 lanes
+#pragma unroll
+        for (int w = 0; w < W; ++w) {
+          const uint32_t x6_0 = c0[w] >> 6, x6_1 = c1[w] >> 6, x12_0 = c0[w] >> 12, x12_1 = c1[w] >> 12;
+#pragma unroll
+          for (int h = 0; h < 2; ++h) {  // MMAs e = 2h, 2h + 1: one 16-byte read of B
+            const uint4 b = bt[(w * 2 + h) * 4];
+            uint32_t a[4];
+            if (h == 0) a_frag<0>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+            else a_frag<2>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+            mma_bf16_16816(d, a, b.x, b.y);
+            if (h == 0) a_frag<1>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+            else a_frag<3>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+            mma_bf16_16816(d, a, b.z, b.w);
+          }
+        }
+        // y += s D + lo S (asymmetric), s D - 2 s S (symmetric)
+        y[0] = __fmaf_rn(o0, sa, __fmaf_rn(s0, d[0], y[0]));
+        y[1] = __fmaf_rn(o0, sb, __fmaf_rn(s0, d[1], y[1]));
+        y[2] = __fmaf_rn(o1, sa, __fmaf_rn(s1, d[2], y[2]));
+        y[3] = __fmaf_rn(o1, sb, __fmaf_rn(s1, d[3], y[3]));
+      };
+      // a row's scale from its raw 4-byte word (binary16: the half holding element x)
+      auto scale_of = [&](uint32_t u, int64_t x) -> float {
+        if constexpr (kF16) {
+          return __half2float(__ushort_as_half(static_cast<unsigned short>((x & 1) ? u >> 16 : u & 0xFFFFu)));
+        } else {
+          return __uint_as_float(u);
+        }
+      };
+      const int64_t x0 = r0 * ngroups + g0, x1 = x0 + 8 * ngroups;  // scale element of rows rq, rq + 8 at g0
+      if (lg == kL) {  // a whole span: C groups' scales, zeros and sums per read; their MMA chains interleave
+        constexpr int C = kL < 4 ? kL : 4;
+#pragma unroll
+        for (int h = 0; h < kL; h += C) {
+          uint32_t u0[C], u1[C];
+          float z0[C], z1[C], sa[C], sb[C];
+          lds_vec<C>(ssl + rq * kL + h, u0);
+          lds_vec<C>(ssl + (rq + 8) * kL + h, u1);
+          lds_vec<C>(sa_lane + g0 + h, sa);
+          lds_vec<C>(sb_lane + g0 + h, sb);
+          if constexpr (!kSym) {
+            lds_vec<C>(zsl + rq * kL + h, z0);
+            lds_vec<C>(zsl + (rq + 8) * kL + h, z1);
+          }
+#pragma unroll
+          for (int i = 0; i < C; ++i) {
+            const float s0 = scale_of(u0[i], x0 + h + i), s1 = scale_of(u1[i], x1 + h + i);
+            group(h + i, s0, s1, kSym ? -2.0f * s0 : z0[i], kSym ? -2.0f * s1 : z1[i], sa[i], sb[i]);
+          }
+        }
+      } else {
+        for (int gi = 0; gi < lg; ++gi) {
+          const float s0 = scale_of(ssl[rq * kL + gi], x0 + gi), s1 = scale_of(ssl[(rq + 8) * kL + gi], x1 + gi);
+          const float o0 = kSym ? -2.0f * s0 : zsl[rq * kL + gi], o1 = kSym ? -2.0f * s1 : zsl[(rq + 8) * kL + gi];
+          group(gi, s0, s1, o0, o1, sa_lane[g0 + gi], sb_lane[g0 + gi]);
+        }
+      }
+      __syncwarp();  // every lane is done with the slot before it is refilled
+      slot = slot + 1 == D ? 0 : slot + 1;
+      if (++cs == nspan) {
+        cs = 0;
+        if (++ck == K) {  // the block's rows are complete: store and start over
+          ck = 0;
+          cr += kRowStep;
+          const int64_t r1 = r0 + 8;
+          const int n0 = 2 * t, n1 = 2 * t + 1;
+          if (r0 < it.rows) {
+            if (n0 < nb) it.Y[static_cast<int64_t>(n0) * it.rows + r0] = scalbnf(y[0], back0);
+            if (n1 < nb) it.Y[static_cast<int64_t>(n1) * it.rows + r0] = scalbnf(y[1], back1);
+          }
+          if (r1 < it.rows) {
+            if (n0 < nb) it.Y[static_cast<int64_t>(n0) * it.rows + r1] = scalbnf(y[2], back0);
+            if (n1 < nb) it.Y[static_cast<int64_t>(n1) * it.rows + r1] = scalbnf(y[3], back1);
+          }
+          y[0] = y[1] = y[2] = y[3] = 0.0f;
+        }
+      }
+    }
+    cp_async_wait<0>();  // the empty groups of the last items
+    seg = seg_end;
+  }
+}
+
+// activation rows one launch of the tensor-core form holds for matrices of up
+// to max_cols columns, with a ring of at least 2 slots a warp (0 if not even
+// one row fits)
+inline int mma_rows_per_launch(bool sym, int64_t max_cols, int group) {
+  for (int nb = kMaxGemvBatch; nb >= 1; --nb)
+    if (mma_ring_slots(sym, group, mma_table_bytes(max_cols, nb, group), kMmaSmemMax) >= 2) return nb;
+  return 0;
+}
+
+template <int F, int K, int G>
+cudaError_t mma_launch_kg(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
+  constexpr bool kSym = F == kSymF32 || F == kSymF16;
+  const int64_t tables = mma_table_bytes(max_cols, nb, G);
+  const int D = mma_ring_slots(kSym, G, tables, kMmaSmemMax);
+  if (D < 2) return cudaErrorInvalidValue;  // the caller sizes nb by mma_rows_per_launch
+  const int smem = static_cast<int>(tables + static_cast<int64_t>(kMmaWarps) * D * mma_slot_bytes(kSym, G));
+  int64_t grid = sms;  // one 16-warp CTA per multiprocessor
+  if (grid > kMaxGemvGrid) grid = kMaxGemvGrid;
+  if (grid > p.total_blocks) grid = p.total_blocks;
+  gemv_split(p, static_cast<int>(grid));
+  gemv_mma_kernel<F, K, G><<<p.grid, kMmaThreads, smem, stream>>>(p, nb, static_cast<int>(tables), D);
+  return cudaGetLastError();
+}
+
+template <int F, int K>
+cudaError_t mma_launch_k(int group, GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
+  switch (group) {
+    case 64: return mma_launch_kg<F, K, 64>(p, nb, max_cols, stream, sms);
+    case 128: return mma_launch_kg<F, K, 128>(p, nb, max_cols, stream, sms);
+    case 256: return mma_launch_kg<F, K, 256>(p, nb, max_cols, stream, sms);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int F>
+cudaError_t mma_launch_format(int group, int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms) {
+  switch (k) {
+    case 1: return mma_launch_k<F, 1>(group, p, nb, max_cols, stream, sms);
+    case 2: return mma_launch_k<F, 2>(group, p, nb, max_cols, stream, sms);
+    case 3: return mma_launch_k<F, 3>(group, p, nb, max_cols, stream, sms);
+    case 4: return mma_launch_k<F, 4>(group, p, nb, max_cols, stream, sms);
+    default: return cudaErrorInvalidValue;
+  }
+}
+
+template <int F, int K>
+cudaError_t mma_prepare_k() {
+  cudaError_t e;
+  const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 64>, a, kMmaSmemMax))) return e;
+  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 128>, a, kMmaSmemMax))) return e;
+  return cudaFuncSetAttribute(gemv_mma_kernel<F, K, 256>, a, kMmaSmemMax);
+}
+
+template <int F>
+cudaError_t mma_prepare_format() {
+  cudaError_t e;
+  if ((e = mma_prepare_k<F, 1>())) return e;
+  if ((e = mma_prepare_k<F, 2>())) return e;
+  if ((e = mma_prepare_k<F, 3>())) return e;
+  return mma_prepare_k<F, 4>();
+}
+
+}  // namespace
+}  // namespace rrq

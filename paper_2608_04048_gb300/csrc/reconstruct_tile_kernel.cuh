@@ -21,9 +21,21 @@
 namespace rrq {
 namespace {
 
-constexpr int kRtWarps = 8;
+#ifndef RRQ_RT_WARPS
+#define RRQ_RT_WARPS 8
+#endif
+#ifndef RRQ_RT_RING
+#define RRQ_RT_RING 3
+#endif
+#ifndef RRQ_RT_CTAS_PER_SM
+#define RRQ_RT_CTAS_PER_SM 2
+#endif
+#ifndef RRQ_RT_SLEEP
+#define RRQ_RT_SLEEP 0
+#endif
+constexpr int kRtWarps = RRQ_RT_WARPS;
 constexpr int kRtThreads = kRtWarps * 32;
-constexpr int kRtRing = 3;                       // chunks of package per warp in flight
+constexpr int kRtRing = RRQ_RT_RING;             // chunks of package per warp in flight
 constexpr int kRtChunk = 2048;                   // weights per warp chunk
 constexpr int kRtOutBytes = kRtChunk * 2;        // bf16 output of a chunk (one TMA box)
 
@@ -50,8 +62,30 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int 
                : "memory");
 }
 
+// Bounded wait that suspends in the barrier between checks (a time hint of
+// up to 1 ms per try) instead of returning at once.
+__device__ __forceinline__ bool rt_wait(uint32_t bar, uint32_t parity, uint32_t limit_us) {
+#if RRQ_RT_SLEEP
+  if (limit_us == 0) return false;
+  const uint64_t t0 = globaltimer_ns();
+  const uint64_t limit_ns = static_cast<uint64_t>(limit_us) * 1000u;
+  while (true) {
+    uint32_t done;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
+        : "=r"(done)
+        : "r"(bar), "r"(parity), "r"(1000000u)
+        : "memory");
+    if (done) return true;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+#else
+  return mbar_wait(bar, parity, limit_us);
+#endif
+}
+
 template <int G, int K, int F>
-__global__ void __launch_bounds__(kRtThreads, 2) reconstruct_tile_kernel(const __grid_constant__ ReconstructTileBatch p) {
+__global__ void __launch_bounds__(kRtThreads, RRQ_RT_CTAS_PER_SM) reconstruct_tile_kernel(const __grid_constant__ ReconstructTileBatch p) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
   using St = RtStage<G, F>;
@@ -115,7 +149,7 @@ __global__ void __launch_bounds__(kRtThreads, 2) reconstruct_tile_kernel(const _
   bool stored = false;
   for (int64_t chunk = first; chunk < b.total_chunks; chunk += stride, ++iter) {
     const int slot = iter % kRtRing;
-    const bool ready = mbar_wait(bar0 + 8 * slot, (iter / kRtRing) & 1, b.wait_limit_us);
+    const bool ready = rt_wait(bar0 + 8 * slot, (iter / kRtRing) & 1, b.wait_limit_us);
     if (!__all_sync(kFullMask, ready)) {
       // Give up: record it, wait (bounded) for this warp's copies in flight
       // so that none lands in freed shared memory, and leave.

@@ -254,8 +254,8 @@ cudaError_t reconstruct_launch_asym_bits(int group, int k, bool all_prefixes, co
                                          cudaStream_t stream, int sms);
 
 // Activation rows one launch can hold in shared memory for matrices of up to
-// max_cols columns with k stages (0: too wide).
-int gemv_rows_per_launch(Format fmt, int k, int64_t max_cols);
+// max_cols columns with k stages and groups of `group` (0: too wide).
+int gemv_rows_per_launch(Format fmt, int k, int64_t max_cols, int group);
 // nb activation rows (1..kMaxGemvBatch, within gemv_rows_per_launch); one
 // translation unit per format.
 cudaError_t gemv_launch_asym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms);

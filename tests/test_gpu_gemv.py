@@ -2,7 +2,17 @@
 Appendix C): Y = A W~^T from the package alone, against the oracle's binary64
 product of the same binary32 prefix weights.
 
-Tolerance, from the kernel's arithmetic: every product W~ a is exact inside
+Two forms, two bounds.  Groups of 64 and more with 2-bit stages take the
+per-group factored form on the tensor cores (gemv_mma_kernel.cuh): per group
+and stage s D + lo S (or s (D - 2 S)) with D the codes' product with the
+activations; it never forms W~, and its distance to the oracle is at most
+d * 2^-24 * sum_c sum_k (|lo_k| + 3 s_k) |a_c| (asymmetric; 2 s_k for the
+symmetric grid) with d = (k + 1) + g/16 + 8 + 2k groups + 18 (the kernel's
+header derives it).  Packages whose levels and activations are small
+integers make every sum exact: those must match bit for bit.
+
+The prefix-weight form (groups of 32, per-stage widths) keeps this bound:
+every product W~ a is exact inside
 its fma and every partial sum is rounded once; a lane sums its lc columns of
 each 32 lc-column window (lc = 128 at k = 1 and at k = 2 with batch <= 2,
 else 64, never more than the group) into two accumulators (lc/2 columns each, windows in turn), then
@@ -56,6 +66,26 @@ def _host_pkg(pkg, rows_idx=None):
     return codes, scales, zeros
 
 
+def factored(pkg) -> bool:
+    """The package takes the tensor-core form (2-bit stages, groups >= 64)."""
+    return pkg.group >= 64 and all(b == 2 for b in pkg.bits[:pkg.n_stages])
+
+
+def _depth_factored(cols, group, k):
+    return (k + 1) + group // 16 + 8 + 2 * k * (cols // group) + 18
+
+
+def _level_bound(scales, zeros, nr, cols, group, k, sym, f16):
+    """Per row and group: sum over the first k stages of |lo| + 3 s (2 s for
+    the symmetric grid), float64 [rows, groups]."""
+    T = np.zeros((nr, cols // group))
+    for i in range(k):
+        sc = scales[i].view(np.float16) if f16 else scales[i].view(np.float32)
+        sc = np.abs(sc.astype(np.float64)).reshape(nr, -1)
+        T += 2 * sc if sym else 3 * sc + np.abs(zeros[i].astype(np.float64)).reshape(nr, -1)
+    return T
+
+
 def _check(pkg, A, Y, k, rows_idx=None, where=""):
     """Y (GPU, float32 [batch, rows]) against the oracle on the given rows."""
     sym, f16 = pkg.grid == binding.GRID_SYM, pkg.scale_type == binding.SCALE_F16
@@ -63,14 +93,19 @@ def _check(pkg, A, Y, k, rows_idx=None, where=""):
     nr = pkg.rows if rows_idx is None else len(rows_idx)
     Ab = bf16_bits(A)
     want = oracle.gemv(codes, scales, zeros, nr, pkg.cols, pkg.group, k, Ab, sym, f16)
-    if sym:
-        rec = oracle.reconstruct_sym(codes, scales, nr, pkg.cols, pkg.group, k, f16)
-    else:
-        rec = oracle.reconstruct(codes, scales, zeros, nr, pkg.cols, pkg.group, k)
-    recf = np.abs((rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
     Af = np.abs((Ab.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
-    d = _depth(pkg.cols)
-    tol = d * 2.0 ** -24 * (Af @ recf.T) * (1 + 2.0 ** -8) + 1e-30
+    if factored(pkg):
+        T = _level_bound(scales, zeros, nr, pkg.cols, pkg.group, k, sym, f16)
+        Ag = Af.reshape(Af.shape[0], -1, pkg.group).sum(axis=2)
+        tol = _depth_factored(pkg.cols, pkg.group, k) * 2.0 ** -24 * (Ag @ T.T) + 1e-30
+    else:
+        if sym:
+            rec = oracle.reconstruct_sym(codes, scales, nr, pkg.cols, pkg.group, k, f16)
+        else:
+            rec = oracle.reconstruct(codes, scales, zeros, nr, pkg.cols, pkg.group, k)
+        recf = np.abs((rec.astype(np.uint32) << 16).view(np.float32).astype(np.float64))
+        d = _depth(pkg.cols)
+        tol = d * 2.0 ** -24 * (Af @ recf.T) * (1 + 2.0 ** -8) + 1e-30
     got = Y.cpu().numpy().astype(np.float64)
     if rows_idx is not None:
         got = got[:, rows_idx]
@@ -121,6 +156,60 @@ def test_deterministic_and_matches_asym_original_package():
     torch.cuda.synchronize()
     assert torch.equal(Y1.view(torch.int32), Y2.view(torch.int32))
     _check(pkg, A, Y1, 4, where="asym original")
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FMT_IDS)
+@pytest.mark.parametrize("group", [64, 128, 256])
+def test_integer_packages_exact(group, fmt):
+    """Levels and activations that are small integers make every product and
+    sum exact in binary32 (and in the tensor cores): the factored form must
+    equal the oracle's product bit for bit, for every prefix and batch."""
+    rows, cols = 37, 6 * group
+    sym, f16 = fmt[0] == binding.GRID_SYM, fmt[1] == binding.SCALE_F16
+    pkg = binding.Package.empty(rows, cols, group, 4, grid=fmt[0], scale_type=fmt[1])
+    gen = torch.Generator(device="cuda").manual_seed(group + 7 * fmt[0] + 3 * fmt[1])
+    n = rows * cols
+    for i in range(4):
+        pkg.codes[i].copy_(torch.randint(0, 256, (n // 4,), generator=gen, device="cuda", dtype=torch.int32).to(torch.uint8))
+        sc = torch.randint(1, 4, (n // group,), generator=gen, device="cuda").to(torch.float32)
+        pkg.scales[i].copy_(sc.to(pkg.scales[i].dtype))
+        if not sym:
+            pkg.zeros[i].copy_(torch.randint(-6, 3, (n // group,), generator=gen, device="cuda").to(torch.float32))
+    for batch in (1, 5, 8):
+        A = torch.randint(-3, 4, (batch, cols), generator=gen, device="cuda").to(torch.bfloat16)
+        codes, scales, zeros = _host_pkg(pkg)
+        for k in (1, 2, 3, 4):
+            (Y,) = binding.rrq_gemv([pkg], [A], k)
+            want = oracle.gemv(codes, scales, zeros, rows, cols, group, k, bf16_bits(A), sym, f16)
+            got = Y.cpu().numpy().astype(np.float64)
+            assert np.array_equal(got, want), f"g{group} {fmt} B{batch} k{k}: {int((got != want).sum())} differ"
+
+
+@pytest.mark.parametrize("fmt", FORMATS, ids=FMT_IDS)
+@pytest.mark.parametrize("group", [64, 128, 256])
+def test_activation_scales(group, fmt):
+    """The tensor-core form works in a domain scaled per activation row by a
+    power of two taken from the row's largest exponent: a row times 2^j gives
+    outputs times exactly 2^j (the same roundings), for rows of very different
+    magnitudes in one call; a row of zeros gives zeros; a row whose columns
+    span 2^-60 .. 2^60 stays within the bound."""
+    rows, cols = 40, 8 * group
+    W = workloads.generate(rows, cols, 90 + group, "t3_rowout", "cuda")
+    (pkg,) = binding.rrq_quantize_ex([W], group, 4, *fmt)
+    gen = torch.Generator(device="cuda").manual_seed(group + fmt[1])
+    z = torch.randn((1, cols), generator=gen, device="cuda")
+    base = (torch.sign(z) * (0.5 + z.abs())).to(torch.bfloat16)  # |a| >= 0.5: no row is scaled into subnormals
+    js = [0, -100, 100, -60, 60]
+    ex = torch.randint(-60, 61, (1, cols), generator=gen, device="cuda").to(torch.float32)
+    mixed = (base.float() * torch.exp2(ex)).to(torch.bfloat16)
+    A = torch.cat([(base.float() * 2.0 ** j).to(torch.bfloat16) for j in js]
+                  + [torch.zeros((1, cols), device="cuda", dtype=torch.bfloat16), mixed])
+    for k in (1, 2, 3, 4):
+        (Y,) = binding.rrq_gemv([pkg], [A], k)
+        for i, j in enumerate(js):
+            assert torch.equal(Y[i], Y[0] * 2.0 ** j), f"g{group} {fmt} k{k}: row scaled by 2^{j}"
+        assert torch.count_nonzero(Y[len(js)]) == 0
+        _check(pkg, A, Y, k, where=f"g{group} {fmt} k{k} scaled rows")
 
 
 def test_batch_across_launches():
