@@ -198,48 +198,62 @@ gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D
     stab = reinterpret_cast<float*>(smem + nb * mma_brow_bytes(cols));
     if (threadIdx.x < nb) emax_s[threadIdx.x] = 0;
     __syncthreads();
-    for (int n = 0; n < nb; ++n) {
-      const uint16_t* a = it.A + static_cast<int64_t>(n) * cols;
+    // The activations in 16-byte chunks of 8 columns, chunk q = n cols/8 +
+    // (column / 8) at thread q % 512: a group's G/8 chunks are consecutive
+    // lanes of one warp, in one row (cols / 8 is a multiple of G / 8).
+    // Pass 1: the row's largest exponent field, and S_g
+    // as the sums of 8 consecutive activations (left to right) added by a
+    // tree over the G / 8 (lane q + h into lane q, h = G/16 .. 1).
+    const int64_t cpr = cols / 8;  // chunks per row
+    const int64_t nch = cpr * nb;
+    for (int64_t q0 = threadIdx.x - lane; q0 < nch; q0 += kMmaThreads) {  // warp-uniform
+      const int64_t q = q0 + lane;
+      const bool ok = q < nch;
+      const int n = static_cast<int>((ok ? q : q0) / cpr);
+      uint4 v = make_uint4(0u, 0u, 0u, 0u);
+      if (ok) v = *reinterpret_cast<const uint4*>(it.A + static_cast<int64_t>(n) * cols + (q - n * cpr) * 8);
+      const uint32_t h[8] = {v.x & 0xFFFFu, v.x >> 16, v.y & 0xFFFFu, v.y >> 16,
+                             v.z & 0xFFFFu, v.z >> 16, v.w & 0xFFFFu, v.w >> 16};
       int e = 0;
-      for (int64_t c = threadIdx.x; c < cols; c += kMmaThreads) e = max(e, (a[c] >> 7) & 0xFF);
-      e = __reduce_max_sync(0xFFFFFFFFu, e);
-      if (lane == 0) atomicMax(&emax_s[n], e);
+      float sum = __uint_as_float(h[0] << 16);
+#pragma unroll
+      for (int i = 0; i < 8; ++i) e = max(e, static_cast<int>((h[i] >> 7) & 0xFF));
+#pragma unroll
+      for (int i = 1; i < 8; ++i) sum = __fadd_rn(sum, __uint_as_float(h[i] << 16));
+#pragma unroll
+      for (int hh = G / 16; hh >= 1; hh >>= 1) {
+        sum = __fadd_rn(sum, __shfl_down_sync(kFullMask, sum, hh, G / 8));
+        e = max(e, __shfl_down_sync(kFullMask, e, hh, G / 8));
+      }
+      if (ok && (lane % (G / 8)) == 0) {  // the group's first chunk
+        atomicMax(&emax_s[n], e);
+        stab[n * srow + (q - n * cpr) / (G / 8)] = sum;
+      }
     }
     __syncthreads();
+    // Pass 2: the B fragments a_c 2^(k_n - 2f), and S_g 2^(k_n - 133).
     uint16_t* bh = reinterpret_cast<uint16_t*>(btab);
-    for (int n = 0; n < nb; ++n) {
-      const uint16_t* a = it.A + static_cast<int64_t>(n) * cols;
+    for (int64_t q = threadIdx.x; q < nch; q += kMmaThreads) {
+      const int n = static_cast<int>(q / cpr);
+      const int64_t c0 = (q - n * cpr) * 8;
       const int kn = 253 - emax_s[n];
-      for (int64_t c = threadIdx.x; c < cols; c += kMmaThreads) {
-        const int64_t g = c / G;
-        const int cg = static_cast<int>(c % G);
+      const uint4 v = *reinterpret_cast<const uint4*>(it.A + static_cast<int64_t>(n) * cols + c0);
+      const uint32_t h[8] = {v.x & 0xFFFFu, v.x >> 16, v.y & 0xFFFFu, v.y >> 16,
+                             v.z & 0xFFFFu, v.z >> 16, v.w & 0xFFFFu, v.w >> 16};
+      const int64_t g = c0 / G;
+#pragma unroll
+      for (int i = 0; i < 8; ++i) {
+        const int cg = static_cast<int>((c0 + i) % G);
         const int tq = cg / (G / 4), u = cg % (G / 4);
-        const int w = u >> 4, v = u & 15, b = v >> 2, e = v & 3;
+        const int w = u >> 4, vv = u & 15, b = vv >> 2, e = vv & 3;
         const int64_t mi = (g * W + w) * 4 + e;
-        const float x = scalbnf(__uint_as_float(static_cast<uint32_t>(a[c]) << 16), kn - 2 * frag_f(e, b & 1));
+        const float x = scalbnf(__uint_as_float(h[i] << 16), kn - 2 * frag_f(e, b & 1));
         bh[(n * brow + (mi >> 1) * 4 + tq) * 8 + (mi & 1) * 4 + (b & 1) * 2 + (b >> 1)] =
             __bfloat16_as_ushort(__float2bfloat16_rn(x));
       }
+      if (c0 % G == 0) stab[n * srow + g] = scalbnf(stab[n * srow + g], kn - 133);
     }
-    // S_g: sums of 8 consecutive activations, then a tree over the G / 8
-    for (int64_t j = threadIdx.x; j < ngroups * nb; j += kMmaThreads) {
-      const int64_t g = j / nb;
-      const int n = static_cast<int>(j % nb);
-      const uint16_t* a = it.A + static_cast<int64_t>(n) * cols + g * G;
-      float s8[G / 8];
-#pragma unroll
-      for (int q = 0; q < G / 8; ++q) {
-        float s = __uint_as_float(static_cast<uint32_t>(a[8 * q]) << 16);
-#pragma unroll
-        for (int i = 1; i < 8; ++i) s = __fadd_rn(s, __uint_as_float(static_cast<uint32_t>(a[8 * q + i]) << 16));
-        s8[q] = s;
-      }
-#pragma unroll
-      for (int h = G / 16; h >= 1; h >>= 1)
-#pragma unroll
-        for (int q = 0; q < h; ++q) s8[q] = __fadd_rn(s8[q], s8[q + h]);
-      stab[n * srow + g] = scalbnf(s8[0], 120 - emax_s[n]);  // k_n - 133
-    }
+    __syncthreads();
     const int bn = rq < nb ? rq : nb - 1;
     const int n0 = 2 * t < nb ? 2 * t : nb - 1, n1 = 2 * t + 1 < nb ? 2 * t + 1 : nb - 1;
     bt_lane = btab + bn * brow + t;

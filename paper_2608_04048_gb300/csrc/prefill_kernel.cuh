@@ -130,9 +130,6 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
   asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
                : "memory");
 }
-__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
-  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
-}
 // Counts `bytes` of the barrier's current phase as arrived without a copy
 // (settles an expectation that no copy will meet).
 __device__ __forceinline__ void mbar_complete_tx(uint32_t bar, uint32_t bytes) {
@@ -189,23 +186,9 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&v)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
-// Bounded wait that sleeps in the barrier instead of spinning: each try
-// suspends the thread until the phase completes or about a millisecond
-// passes, so waiting warps take no issue slots from the working ones.
+// Bounded wait that sleeps in the barrier (rrq_device.cuh).
 __device__ __forceinline__ bool pf_wait(uint32_t bar, uint32_t parity, uint32_t limit_us) {
-  if (limit_us == 0) return false;
-  const uint64_t t0 = globaltimer_ns();
-  const uint64_t limit_ns = static_cast<uint64_t>(limit_us) * 1000u;
-  while (true) {
-    uint32_t done;
-    asm volatile(
-        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
-        : "=r"(done)
-        : "r"(bar), "r"(parity), "r"(1000000u)
-        : "memory");
-    if (done) return true;
-    if (globaltimer_ns() - t0 > limit_ns) return false;
-  }
+  return mbar_wait_sleep(bar, parity, limit_us);
 }
 
 // Package words of the 32 consecutive weights (one group) a thread forms in

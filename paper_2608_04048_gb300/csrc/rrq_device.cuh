@@ -62,6 +62,29 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, uint32_
   }
 }
 
+// Bounded wait that sleeps in the barrier instead of spinning: each try
+// suspends the thread until the phase completes or about a millisecond
+// passes, so waiting warps take no issue slots from the working ones.
+__device__ __forceinline__ bool mbar_wait_sleep(uint32_t bar, uint32_t parity, uint32_t limit_us) {
+  if (limit_us == 0) return false;
+  const uint64_t t0 = globaltimer_ns();
+  const uint64_t limit_ns = static_cast<uint64_t>(limit_us) * 1000u;
+  while (true) {
+    uint32_t done;
+    asm volatile(
+        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
+        : "=r"(done)
+        : "r"(bar), "r"(parity), "r"(1000000u)
+        : "memory");
+    if (done) return true;
+    if (globaltimer_ns() - t0 > limit_ns) return false;
+  }
+}
+
+__device__ __forceinline__ void mbar_arrive(uint32_t bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+
 // Orders this thread's generic-proxy shared-memory accesses before later
 // bulk-copy (async-proxy) accesses of the same memory.
 __device__ __forceinline__ void fence_proxy_async_smem() {
