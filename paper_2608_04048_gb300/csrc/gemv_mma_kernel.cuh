@@ -58,23 +58,17 @@ constexpr int kMmaThreads = kMmaWarps * 32;
 constexpr int kMmaRingMax = 4;  // slots of a warp's ring at most
 constexpr int kMmaSmemMax = kMaxSmem - 128;  // dynamic shared memory (the kernel has 32 static bytes)
 
-// The item geometry for groups of G columns: kSpan columns (kL groups) per
-// item; a slot row holds the span's codes (kSpan / 4 bytes) and a pad that
-// puts the rows rq = 0..7 (G = 64: 4-byte reads), 0..3 (G = 128: 8-byte) or
-// 0..1 (G = 256: 16-byte reads) of one read phase on distinct banks.
-template <int G>
-struct MmaGeom {
-  static constexpr int kSpan = G > 512 ? G : 512;
-  static constexpr int kL = kSpan / G;
-  static constexpr int kPitch = kSpan / 4 + (G == 64 ? 16 : G == 128 ? 32 : 64);
-};
-__host__ __device__ constexpr int mma_pitch(int G) { return (G > 512 ? G : 512) / 4 + (G == 64 ? 16 : G == 128 ? 32 : 64); }
-__host__ __device__ constexpr int mma_groups_per_item(int G) { return (G > 512 ? G : 512) / G; }
+// The item geometry for groups of G columns and spans of S columns (512
+// or 1024, at least G): kL = S / G groups per item; a slot row holds the
+// span's codes (S / 4 bytes) and a pad that puts the rows rq = 0..7 (G = 64:
+// 4-byte reads), 0..3 (G = 128: 8-byte) or 0..1 (G = 256: 16-byte reads) of
+// one read phase on distinct banks.
+__host__ __device__ constexpr int mma_pitch(int G, int S) { return S / 4 + (G == 64 ? 16 : G == 128 ? 32 : 64); }
 // one ring slot: 16 rows of codes, then the 16 x kL scales (binary32, or the
 // aligned binary16 pair holding the scale) and, on the asymmetric grid, the
 // 16 x kL zeros
-__host__ __device__ constexpr int mma_slot_bytes(bool sym, int G) {
-  return kGemvRows * mma_pitch(G) + (sym ? 1 : 2) * kGemvRows * mma_groups_per_item(G) * 4;
+__host__ __device__ constexpr int mma_slot_bytes(bool sym, int G, int S) {
+  return kGemvRows * mma_pitch(G, S) + (sym ? 1 : 2) * kGemvRows * (S / G) * 4;
 }
 
 // shared memory of the per-matrix tables: per activation row, B fragments
@@ -88,8 +82,8 @@ __host__ __device__ constexpr int64_t mma_table_bytes(int64_t cols, int nb, int 
 }
 // ring slots a launch gives each warp: up to kMmaRingMax within what the
 // tables leave of the shared memory (0 if not even 2 fit)
-__host__ __device__ constexpr int mma_ring_slots(bool sym, int G, int64_t table_bytes, int64_t smem_max) {
-  const int64_t fit = (smem_max - table_bytes) / (kMmaWarps * static_cast<int64_t>(mma_slot_bytes(sym, G)));
+__host__ __device__ constexpr int mma_ring_slots(bool sym, int G, int S, int64_t table_bytes, int64_t smem_max) {
+  const int64_t fit = (smem_max - table_bytes) / (kMmaWarps * static_cast<int64_t>(mma_slot_bytes(sym, G, S)));
   const int64_t d = fit < kMmaRingMax ? fit : kMmaRingMax;
   return d < 2 ? 0 : static_cast<int>(d);
 }
@@ -148,17 +142,18 @@ __device__ __forceinline__ void lds_vec(const void* p, T (&v)[N]) {
   }
 }
 
-template <int F, int K, int G>
+template <int F, int K, int G, int S>
 __global__ void __launch_bounds__(kMmaThreads, 1)
 gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
   constexpr int W = G / 64;  // words of 16 codes per lane, row and group
-  using Geo = MmaGeom<G>;
-  constexpr int kSpan = Geo::kSpan, kL = Geo::kL, kPitch = Geo::kPitch;
-  static_assert(kSpan / 4 == 128, "two lanes copy a row's 128 bytes of codes");
+  constexpr int kSpan = S, kL = S / G, kPitch = mma_pitch(G, S);
+  constexpr int kP = S / 64;                   // 16-byte pieces of a row's codes in a span
+  constexpr int kCopies = kGemvRows * kP / 32;  // pieces a lane copies per item
+  static_assert(S % G == 0 && kP <= 32, "a span is whole groups, a row at most one warp's pieces");
   constexpr int kCodes = kGemvRows * kPitch;   // a slot's codes
-  constexpr int kSlot = mma_slot_bytes(kSym, G);
+  constexpr int kSlot = mma_slot_bytes(kSym, G, S);
   extern __shared__ __align__(16) uint8_t smem[];
   const int lane = threadIdx.x & 31;
   const int warp = threadIdx.x >> 5;
@@ -268,60 +263,50 @@ gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D
   const uint32_t ring_s = smem_u32(ring);
 
   // The lanes' copies of item (block from row r0, stage k, span sp): piece i
-  // of a lane is the 16 bytes at part lane % 8 of row lane / 8 + 4 i of the
-  // span's codes (a warp's copy instruction covers 4 whole rows of 128
+  // of a lane is the 16 bytes at part lane % kP of row lane / kP + (32 / kP) i
+  // of the span's codes (a warp's copy instruction covers whole rows of S / 4
   // bytes); entry i (e = lane + 32 i < 16 kL) is the scale (and zero) of row
-  // e / kL, group e % kL of the span.  The lane keeps its pointers per
-  // (block, stage); rows past the matrix are not copied (their sums are never
-  // stored), nor groups past the row's end.
+  // lane / kL + (32 / kL) i, group lane % kL of the span.  The lane keeps its
+  // first piece and entry per (block, stage); rows past the matrix are not
+  // copied (their sums are never stored), nor groups past the row's end.
   constexpr int kEntries = (kGemvRows * kL + 31) / 32;
-  const uint8_t* cptr[4];           // the lane's pieces in span 0
-  const float* sptr[kEntries];      // its entries' scales (binary32) in span 0
-  const uint16_t* hptr[kEntries];   // or binary16 scales
-  const float* zptr[kEntries];      // and zeros
-  int64_t hx[kEntries];             // element index of a binary16 entry in span 0
-  bool cok[4], mok[kEntries];
+  static_assert(32 % kL == 0, "a lane's entries are one group of rows 32 / kL apart");
+  const uint8_t* cbase = nullptr;  // the lane's first piece in span 0
+  const void* sbase = nullptr;     // its first entry's scale (binary32 or binary16) in group 0
+  const float* zbase = nullptr;    // and zero
+  int64_t xbase = 0;               // element index of the first entry in group 0
+  int vrows = 0;                   // rows of the block in the matrix
   auto set_stage = [&](const GemvItem& it, int64_t r0, int k) {
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const int row = (lane >> 3) + 4 * i;
-      cok[i] = r0 + row < it.rows;
-      cptr[i] = it.codes[k] + (r0 + row) * (cols / 4) + (lane & 7) * 16;
-    }
-#pragma unroll
-    for (int i = 0; i < kEntries; ++i) {
-      const int e = lane + 32 * i;
-      const int row = e / kL, gi = e % kL;
-      mok[i] = e < kGemvRows * kL && r0 + row < it.rows;
-      const int64_t x = (r0 + row) * ngroups + gi;
-      if constexpr (kF16) {
-        hx[i] = x;
-        hptr[i] = static_cast<const uint16_t*>(it.scales[k]);
-      } else {
-        sptr[i] = static_cast<const float*>(it.scales[k]) + x;
-        if constexpr (!kSym) zptr[i] = it.zeros[k] + x;
-      }
-    }
+    vrows = it.rows - r0 < kGemvRows ? static_cast<int>(it.rows - r0) : kGemvRows;
+    cbase = it.codes[k] + (r0 + lane / kP) * (cols / 4) + (lane % kP) * 16;
+    xbase = (r0 + lane / kL) * ngroups + lane % kL;
+    sbase = it.scales[k];
+    zbase = it.zeros[k];
   };
   auto issue = [&](const GemvItem& it, int sp, uint32_t dst) {
     const int64_t g0 = static_cast<int64_t>(sp) * kL;
     const int lg = ngroups - g0 < kL ? static_cast<int>(ngroups - g0) : kL;  // groups of this span
-    const int64_t cspan = g0 * (G / 4);
+    const uint8_t* src = cbase + g0 * (G / 4);
+    const int64_t cstep = (32 / kP) * (cols / 4);  // bytes between a lane's pieces
 #pragma unroll
-    for (int i = 0; i < 4; ++i)
-      if (cok[i] && (lg == kL || (lane & 7) * 16 < lg * (G / 4)))
-        cp_async_16(dst + ((lane >> 3) + 4 * i) * kPitch + (lane & 7) * 16, cptr[i] + cspan, 16);
+    for (int i = 0; i < kCopies; ++i, src += cstep) {
+      const int row = lane / kP + (32 / kP) * i;
+      if (row < vrows && (lg == kL || (lane % kP) * 16 < lg * (G / 4)))
+        cp_async_16(dst + row * kPitch + (lane % kP) * 16, src, 16);
+    }
+    int64_t x = xbase + g0;
 #pragma unroll
-    for (int i = 0; i < kEntries; ++i) {
+    for (int i = 0; i < kEntries; ++i, x += (32 / kL) * ngroups) {
       const int e = lane + 32 * i;
-      if (mok[i] && (lg == kL || e % kL < lg)) {
+      const int row = lane / kL + (32 / kL) * i;
+      if (e < kGemvRows * kL && row < vrows && (lg == kL || lane % kL < lg)) {
         const uint32_t md = dst + kCodes + e * 4;
         if constexpr (kF16) {  // the 4-byte aligned pair holding the scale (2 bytes at the array's end)
-          const int64_t xa = (hx[i] + g0) & ~static_cast<int64_t>(1);
-          cp_async_4(md, hptr[i] + xa, xa + 1 < it.rows * ngroups ? 4u : 2u);
+          const int64_t xa = x & ~static_cast<int64_t>(1);
+          cp_async_4(md, static_cast<const uint16_t*>(sbase) + xa, xa + 1 < it.rows * ngroups ? 4u : 2u);
         } else {
-          cp_async_4(md, sptr[i] + g0, 4);
-          if constexpr (!kSym) cp_async_4(md + kGemvRows * kL * 4, zptr[i] + g0, 4);
+          cp_async_4(md, static_cast<const float*>(sbase) + x, 4);
+          if constexpr (!kSym) cp_async_4(md + kGemvRows * kL * 4, zbase + x, 4);
         }
       }
     }
@@ -483,27 +468,42 @@ gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D
 }
 
 // activation rows one launch of the tensor-core form holds for matrices of up
-// to max_cols columns, with a ring of at least 2 slots a warp (0 if not even
-// one row fits)
+// to max_cols columns, with a ring of at least 2 slots of 512-column spans a
+// warp (0 if not even one row fits)
 inline int mma_rows_per_launch(bool sym, int64_t max_cols, int group) {
+  const int span = group > 512 ? group : 512;
   for (int nb = kMaxGemvBatch; nb >= 1; --nb)
-    if (mma_ring_slots(sym, group, mma_table_bytes(max_cols, nb, group), kMmaSmemMax) >= 2) return nb;
+    if (mma_ring_slots(sym, group, span, mma_table_bytes(max_cols, nb, group), kMmaSmemMax) >= 2) return nb;
   return 0;
 }
 
-template <int F, int K, int G>
-cudaError_t mma_launch_kg(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
+template <int F, int K, int G, int S>
+cudaError_t mma_launch_kgs(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms, int D) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   const int64_t tables = mma_table_bytes(max_cols, nb, G);
-  const int D = mma_ring_slots(kSym, G, tables, kMmaSmemMax);
-  if (D < 2) return cudaErrorInvalidValue;  // the caller sizes nb by mma_rows_per_launch
-  const int smem = static_cast<int>(tables + static_cast<int64_t>(kMmaWarps) * D * mma_slot_bytes(kSym, G));
+  const int smem = static_cast<int>(tables + static_cast<int64_t>(kMmaWarps) * D * mma_slot_bytes(kSym, G, S));
   int64_t grid = sms;  // one 16-warp CTA per multiprocessor
   if (grid > kMaxGemvGrid) grid = kMaxGemvGrid;
   if (grid > p.total_blocks) grid = p.total_blocks;
   gemv_split(p, static_cast<int>(grid));
-  gemv_mma_kernel<F, K, G><<<p.grid, kMmaThreads, smem, stream>>>(p, nb, static_cast<int>(tables), D);
+  gemv_mma_kernel<F, K, G, S><<<p.grid, kMmaThreads, smem, stream>>>(p, nb, static_cast<int>(tables), D);
   return cudaGetLastError();
+}
+
+// spans of 1024 columns where groups of 128 or more leave room for a ring of
+// at least 2 of them (half the per-item costs), else 512 (G = 64: 512 only)
+template <int F, int K, int G>
+cudaError_t mma_launch_kg(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
+  constexpr bool kSym = F == kSymF32 || F == kSymF16;
+  const int64_t tables = mma_table_bytes(max_cols, nb, G);
+  if constexpr (G >= 128) {
+    const int d = mma_ring_slots(kSym, G, 1024, tables, kMmaSmemMax);
+    if (d >= 2) return mma_launch_kgs<F, K, G, 1024>(p, nb, max_cols, stream, sms, d);
+  }
+  constexpr int S0 = G > 512 ? G : 512;
+  const int d = mma_ring_slots(kSym, G, S0, tables, kMmaSmemMax);
+  if (d < 2) return cudaErrorInvalidValue;  // the caller sizes nb by mma_rows_per_launch
+  return mma_launch_kgs<F, K, G, S0>(p, nb, max_cols, stream, sms, d);
 }
 
 template <int F, int K>
@@ -531,9 +531,11 @@ template <int F, int K>
 cudaError_t mma_prepare_k() {
   cudaError_t e;
   const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 64>, a, kMmaSmemMax))) return e;
-  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 128>, a, kMmaSmemMax))) return e;
-  return cudaFuncSetAttribute(gemv_mma_kernel<F, K, 256>, a, kMmaSmemMax);
+  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 64, 512>, a, kMmaSmemMax))) return e;
+  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 128, 512>, a, kMmaSmemMax))) return e;
+  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 128, 1024>, a, kMmaSmemMax))) return e;
+  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 256, 512>, a, kMmaSmemMax))) return e;
+  return cudaFuncSetAttribute(gemv_mma_kernel<F, K, 256, 1024>, a, kMmaSmemMax);
 }
 
 template <int F>
