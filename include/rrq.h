@@ -317,22 +317,30 @@ typedef struct {
  * them (Appendix C: A W~_(t) = A W^_0 + sum_k A R^_k):
  *     Y[b][r] = sum_c W~[r][c] * A[b][c],   b < batch, r < rows
  * where W~[r][c] is the binary32 prefix sum of the first k stages (acc = L_0;
- * acc = fl(acc + L_i), the value rrq_reconstruct rounds to bf16).  The kernel
- * reads only the package (k x (2 + 64/g) bits per weight for RRQ_GRID_ASYM,
- * k x (2 + 16/g) for the binary16 symmetric format) and sums each row in a
- * fixed order in binary32 (deterministic; |Y - exact| <= gamma_cols *
- * sum_c |W~ A|).  For decoding: 1 <= batch <= RRQ_MAX_GEMV_BATCH activation
- * rows; 1 <= k <= fmt->n_stages.  Per-stage widths (fmt->bits, asymmetric
- * grid) are taken with the reconstruction's stage sum of that format.  Y must
- * not overlap any input or another Y.  The activation rows of a launch are
- * held in shared memory as binary32, padded to a multiple of 2048 columns:
- * a launch takes as many of the batch's rows as fit in 227 KiB (at most 4
- * at k = 4), so every
- * matrix of a call may have at most RRQ_MAX_GEMV_COLS columns
- * (RRQ_ERR_UNSUPPORTED beyond, before anything is launched).  Matrices
- * that take the same number of rows per launch are launched together, up to
- * 64 per launch, once per such share of the batch; other rules as for
- * rrq_reconstruct_ex. */
+ * acc = fl(acc + L_i), the value rrq_reconstruct rounds to bf16).  The kernels
+ * read only the package (k x (2 + 64/g) bits per weight for RRQ_GRID_ASYM,
+ * k x (2 + 16/g) for the binary16 symmetric format) and sum in binary32 in a
+ * fixed order (deterministic: two calls give the same bits).  Two forms:
+ *   - groups of 64 and more with 2-bit stages: Appendix C's stage-wise form
+ *     per group and stage, s D + lo S_g (s (D - 2 S_g) on the symmetric
+ *     grid), D = sum Q a over the group's codes on the tensor cores and S_g
+ *     = sum a; |Y - sum W~ a| <= d 2^-24 sum_c sum_k (|lo_k| + 3 s_k) |a_c|
+ *     (2 s_k symmetric) with d = (k + 1) + g/16 + 8 + 2k (cols/g) + 18.
+ *     The activations are held in shared memory as bf16 fragments, 2 bytes
+ *     per column and row plus the group sums;
+ *   - groups of 32 and per-stage widths (fmt->bits, asymmetric grid, with
+ *     the reconstruction's stage sum of that format): the prefix weights
+ *     formed per weight, |Y - exact| <= (64 ceil(cols/4096) + 8) 2^-24
+ *     sum_c |W~ A|.  The activations are held in shared memory as binary32,
+ *     padded to a multiple of 2048 columns (at most 4 rows at k = 4).
+ * For decoding: 1 <= batch <= RRQ_MAX_GEMV_BATCH activation rows;
+ * 1 <= k <= fmt->n_stages.  Y must not overlap any input or another Y.  A
+ * launch takes as many of the batch's rows as fit in 227 KiB of shared
+ * memory, so every matrix of a call may have at most RRQ_MAX_GEMV_COLS
+ * columns (RRQ_ERR_UNSUPPORTED beyond, before anything is launched).
+ * Matrices that take the same number of rows per launch are launched
+ * together, up to 64 per launch, once per such share of the batch; other
+ * rules as for rrq_reconstruct_ex. */
 rrq_status rrq_gemv(const rrq_gemv_desc* items, int count, const rrq_format* fmt, int k, int batch,
                     rrq_stream_t stream);
 

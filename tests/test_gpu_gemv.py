@@ -1,6 +1,6 @@
-"""GPU parity for the stage-wise product with the prefix weights (rrq_gemv,
-Appendix C): Y = A W~^T from the package alone, against the oracle's binary64
-product of the same binary32 prefix weights.
+"""GPU parity for the stage-wise product (rrq_gemv, Appendix C): Y = A W~^T
+from the package alone, against the oracle's binary64 product of the same
+binary32 prefix weights W~.
 
 Two forms, two bounds.  Groups of 64 and more with 2-bit stages take the
 per-group factored form on the tensor cores (gemv_mma_kernel.cuh): per group
@@ -268,9 +268,10 @@ def test_widths(batch, bits, group):
 
 
 def test_widest_rows_and_batch_split():
-    """The widest supported rows (RRQ_MAX_GEMV_COLS columns, one activation
-    row per launch's shared memory at most) and a batch of 8 at 28672 columns
-    (two activation rows per launch: four launches over the same package)."""
+    """The widest supported rows (RRQ_MAX_GEMV_COLS columns: one activation
+    row fits a launch's shared memory) and a batch of 8 at 28672 columns (two
+    activation rows per launch in the tensor-core form at group 128: four
+    launches over the same package)."""
     for rows, cols, batch in ((3, 57344, 1), (5, 28672, 8)):
         W = workloads.generate(rows, cols, cols + batch, "t3_rowout", "cuda")
         (pkg,) = binding.rrq_quantize_ex([W], 128, 4, binding.GRID_ASYM, binding.SCALE_F32)
@@ -281,9 +282,10 @@ def test_widest_rows_and_batch_split():
 
 
 def test_mixed_widths_batch_8():
-    """One call at batch 8 over matrices that hold 8, 4, 2 and 1 activation
-    rows per launch (4096, 12288, 28672 and 57344 columns): each width class
-    is launched on its own share of the batch, in any order of the items."""
+    """One call at batch 8 over matrices of 4096, 12288, 28672 and 57344
+    columns, which hold different numbers of activation rows per launch (8,
+    5, 2 and 1 in the tensor-core form at group 128): each width class is
+    launched on its own share of the batch, in any order of the items."""
     shapes = [(5, 28672), (7, 4096), (3, 57344), (17, 12288), (2, 4096)]
     mats = [workloads.generate(r, c, 300 + i, "t3_rowout", "cuda") for i, (r, c) in enumerate(shapes)]
     pkgs = binding.rrq_quantize_ex(mats, 128, 2, binding.GRID_ASYM, binding.SCALE_F32)
