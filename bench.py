@@ -630,14 +630,16 @@ def run_gpu(args, world, rank, local) -> dict | None:
         raise RuntimeError("a kernel reported a timeout in the breakdown")
 
     stack = args.workload == "qwen3_8b_stack" and wl.own_outputs and not args.no_sym
+    # the two products also on one layer (the size their ncu captures take)
+    products = stack or (args.workload == "qwen3_8b_layer" and wl.own_outputs and not args.no_sym)
     mats, pkgs, p_outs = wl.mats, wl.pkgs, wl.p_outs
     sym = time_sym_f16(mats, p_outs, specs, stream) if stack else None
     from_base = time_from_base(mats, pkgs, specs, stream) if stack else None
-    gemv = time_gemv(pkgs, specs, stream) if stack else None
+    gemv = time_gemv(pkgs, specs, stream) if products else None
     batches = [int(x) for x in args.gemv_batches.split(",") if x.strip()]
     gemv_batches = {f"batch{b}": time_gemv(pkgs, specs, stream, batch=b) for b in batches if b != 1} \
-        if stack and any(b != 1 for b in batches) else None
-    prefill = time_prefill(pkgs, specs, stream) if stack else None
+        if products and any(b != 1 for b in batches) else None
+    prefill = time_prefill(pkgs, specs, stream) if products else None
     bits = {"+".join(map(str, b)): time_bits(mats, p_outs, specs, stream, b) for b in ((1, 3), (3, 1))} \
         if stack else None
     pmr = time_pmr(mats, specs, stream) if stack else None
