@@ -88,6 +88,11 @@ __host__ __device__ constexpr int mma_ring_slots(bool sym, int G, int S, int64_t
   return d < 2 ? 0 : static_cast<int>(d);
 }
 
+// named barrier `id` over `count` threads (whole warps)
+__device__ __forceinline__ void named_barrier(int id, int count) {
+  asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
 // wait until at most n (< kMmaRingMax) of this thread's cp.async groups are pending
 __device__ __forceinline__ void cp_async_wait_n(int n) {
   if (n <= 1) cp_async_wait<1>();
@@ -142,9 +147,11 @@ __device__ __forceinline__ void lds_vec(const void* p, T (&v)[N]) {
   }
 }
 
-template <int F, int K, int G, int S>
+// kGrp: blocks shared by groups of P > 1 warps (else P = 1, compiled out)
+template <int F, int K, int G, int S, bool kGrp>
 __global__ void __launch_bounds__(kMmaThreads, 1)
-gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D) {
+gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D, int P_arg, int red_off) {
+  const int P = kGrp ? P_arg : 1;
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
   constexpr int W = G / 64;  // words of 16 codes per lane, row and group
@@ -313,8 +320,115 @@ gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D
   };
 
   // The CTA's range, matrix by matrix: the tables are built for a matrix,
-  // then each warp takes whole blocks of it (blocks w, w + 16, ...), each
-  // block stage by stage and span by span, D - 1 items in flight.
+  // then each warp (P = 1), or each group of P warps, takes whole blocks of
+  // it (blocks q, q + 16/P, ... for group q).  A block is walked item by item
+  // (item i: stage i / nspan, span i % nspan); warp j of a group takes items
+  // j, j + P, ..., D - 1 items in flight.  With P > 1 the group's warps sum
+  // their parts of a block's rows in shared memory, in warp order, behind
+  // named barrier 1 + q.
+  const int ngrp = kMmaWarps / P;
+  const int grp = warp / P, wj = warp % P;
+  // the item in slot `sl`: span sp of rows r0 (= block row + rq), r0 + 8 of a
+  // stage, into the row sums y (rows r0 (0, 1) and r0 + 8 (2, 3); activation
+  // rows 2t, 2t + 1)
+  auto item = [&](float (&y)[4], const uint8_t* sl, int64_t r0, int sp) {
+    const uint32_t* ssl = reinterpret_cast<const uint32_t*>(sl + kCodes);  // [16][kL]
+    const float* zsl = reinterpret_cast<const float*>(sl + kCodes) + kGemvRows * kL;
+    const int64_t g0 = static_cast<int64_t>(sp) * kL;
+    const int lg = ngroups - g0 < kL ? static_cast<int>(ngroups - g0) : kL;
+    // one group of the item: D by G/16 MMAs, then the row sums with the
+    // rows' scales s0, s1, offsets o0, o1 (lo, or -2 s) and the sums sa, sb
+    auto group = [&](int gi, float s0, float s1, float o0, float o1, float sa, float sb) {
+      const int64_t g = g0 + gi;
+      // the lane's W words of rows rq and rq + 8 (one read each)
+      uint32_t c0[W], c1[W];
+      const uint8_t* cb = sl + gi * (G / 4) + t * (G / 16);
+      if constexpr (W == 1) {
+        c0[0] = *reinterpret_cast<const uint32_t*>(cb + rq * kPitch);
+        c1[0] = *reinterpret_cast<const uint32_t*>(cb + (rq + 8) * kPitch);
+      } else if constexpr (W == 2) {
+        const uint2 x0 = *reinterpret_cast<const uint2*>(cb + rq * kPitch);
+        const uint2 x1 = *reinterpret_cast<const uint2*>(cb + (rq + 8) * kPitch);
+        c0[0] = x0.x; c0[1] = x0.y;
+        c1[0] = x1.x; c1[1] = x1.y;
+      } else {
+        const uint4 x0 = *reinterpret_cast<const uint4*>(cb + rq * kPitch);
+        const uint4 x1 = *reinterpret_cast<const uint4*>(cb + (rq + 8) * kPitch);
+        c0[0] = x0.x; c0[1] = x0.y; c0[2] = x0.z; c0[3] = x0.w;
+        c1[0] = x1.x; c1[1] = x1.y; c1[2] = x1.z; c1[3] = x1.w;
+      }
+      float d[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      const uint4* bt = bt_lane + g * (W * 2 * 4);  // 16-byte units: MMA pairs x 4 lanes
+#pragma unroll
+      for (int w = 0; w < W; ++w) {
+        const uint32_t x6_0 = c0[w] >> 6, x6_1 = c1[w] >> 6, x12_0 = c0[w] >> 12, x12_1 = c1[w] >> 12;
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {  // MMAs e = 2h, 2h + 1: one 16-byte read of B
+          const uint4 b = bt[(w * 2 + h) * 4];
+          uint32_t a[4];
+          if (h == 0) a_frag<0>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+          else a_frag<2>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+          mma_bf16_16816(d, a, b.x, b.y);
+          if (h == 0) a_frag<1>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+          else a_frag<3>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
+          mma_bf16_16816(d, a, b.z, b.w);
+        }
+      }
+      // y += s D + lo S (asymmetric), s D - 2 s S (symmetric)
+      y[0] = __fmaf_rn(o0, sa, __fmaf_rn(s0, d[0], y[0]));
+      y[1] = __fmaf_rn(o0, sb, __fmaf_rn(s0, d[1], y[1]));
+      y[2] = __fmaf_rn(o1, sa, __fmaf_rn(s1, d[2], y[2]));
+      y[3] = __fmaf_rn(o1, sb, __fmaf_rn(s1, d[3], y[3]));
+    };
+    // a row's scale from its raw 4-byte word (binary16: the half holding element x)
+    auto scale_of = [&](uint32_t u, int64_t x) -> float {
+      if constexpr (kF16) {
+        return __half2float(__ushort_as_half(static_cast<unsigned short>((x & 1) ? u >> 16 : u & 0xFFFFu)));
+      } else {
+        return __uint_as_float(u);
+      }
+    };
+    const int64_t x0 = r0 * ngroups + g0, x1 = x0 + 8 * ngroups;  // scale element of rows rq, rq + 8 at g0
+    if (lg == kL) {  // a whole span: C groups' scales, zeros and sums per read; their MMA chains interleave
+      constexpr int C = kL < 4 ? kL : 4;
+#pragma unroll
+      for (int h = 0; h < kL; h += C) {
+        uint32_t u0[C], u1[C];
+        float z0[C], z1[C], sa[C], sb[C];
+        lds_vec<C>(ssl + rq * kL + h, u0);
+        lds_vec<C>(ssl + (rq + 8) * kL + h, u1);
+        lds_vec<C>(sa_lane + g0 + h, sa);
+        lds_vec<C>(sb_lane + g0 + h, sb);
+        if constexpr (!kSym) {
+          lds_vec<C>(zsl + rq * kL + h, z0);
+          lds_vec<C>(zsl + (rq + 8) * kL + h, z1);
+        }
+#pragma unroll
+        for (int i = 0; i < C; ++i) {
+          const float s0 = scale_of(u0[i], x0 + h + i), s1 = scale_of(u1[i], x1 + h + i);
+          group(h + i, s0, s1, kSym ? -2.0f * s0 : z0[i], kSym ? -2.0f * s1 : z1[i], sa[i], sb[i]);
+        }
+      }
+    } else {
+      for (int gi = 0; gi < lg; ++gi) {
+        const float s0 = scale_of(ssl[rq * kL + gi], x0 + gi), s1 = scale_of(ssl[(rq + 8) * kL + gi], x1 + gi);
+        const float o0 = kSym ? -2.0f * s0 : zsl[rq * kL + gi], o1 = kSym ? -2.0f * s1 : zsl[(rq + 8) * kL + gi];
+        group(gi, s0, s1, o0, o1, sa_lane[g0 + gi], sb_lane[g0 + gi]);
+      }
+    }
+  };
+  auto store = [&](const float (&y)[4], const GemvItem& it, int64_t r0) {
+    const int64_t r1 = r0 + 8;
+    const int n0 = 2 * t, n1 = 2 * t + 1;
+    if (r0 < it.rows) {
+      if (n0 < nb) it.Y[static_cast<int64_t>(n0) * it.rows + r0] = scalbnf(y[0], back0);
+      if (n1 < nb) it.Y[static_cast<int64_t>(n1) * it.rows + r0] = scalbnf(y[1], back1);
+    }
+    if (r1 < it.rows) {
+      if (n0 < nb) it.Y[static_cast<int64_t>(n0) * it.rows + r1] = scalbnf(y[2], back0);
+      if (n1 < nb) it.Y[static_cast<int64_t>(n1) * it.rows + r1] = scalbnf(y[3], back1);
+    }
+  };
   int m = 0;
   while (m + 1 < p.count && blk_begin >= p.item[m + 1].blk_begin) ++m;
   for (int64_t seg = blk_begin; seg < blk_end; ++m) {
@@ -325,141 +439,110 @@ gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D
     m_cur = m;
     __syncthreads();
     const int nspan = static_cast<int>((cols + kSpan - 1) / kSpan);
-    const int nblk = static_cast<int>((seg_end - seg - warp + kMmaWarps - 1) / kMmaWarps);  // may be <= 0
-    const int items = nblk > 0 ? nblk * K * nspan : 0;
-    // cursors (first row of the block, stage, span) of the next item to copy
-    // and of the item to multiply: a warp's blocks are 16 blocks apart
-    constexpr int64_t kRowStep = static_cast<int64_t>(kMmaWarps) * kGemvRows;
-    const int64_t r_first = (seg + warp - it.blk_begin) * kGemvRows;
-    int64_t ir = r_first;
-    int is = 0, ik = 0, left = items;
-    auto issue_next = [&](int s_dst) {
-      if (left > 0) {
-        if (is == 0) set_stage(it, ir, ik);
-        issue(it, is, ring_s + s_dst * kSlot);
-        --left;
-        if (++is == nspan) {
-          is = 0;
-          if (++ik == K) ik = 0, ir += kRowStep;
+    const int ipb = K * nspan;                                                    // items per block
+    const int nblk = static_cast<int>((seg_end - seg - grp + ngrp - 1) / ngrp);  // may be <= 0
+    const int64_t row_step = static_cast<int64_t>(ngrp) * kGemvRows;
+    const int64_t r_first = (seg + grp - it.blk_begin) * kGemvRows;
+    if constexpr (!kGrp) {
+      // one warp per block: cursors (first row of the block, stage, span) of
+      // the next item to copy and of the item to multiply
+      const int items = nblk > 0 ? nblk * ipb : 0;
+      int64_t ir = r_first;
+      int is = 0, ik = 0, left = items;
+      auto issue_next = [&](int s_dst) {
+        if (left > 0) {
+          if (is == 0) set_stage(it, ir, ik);
+          issue(it, is, ring_s + s_dst * kSlot);
+          --left;
+          if (++is == nspan) {
+            is = 0;
+            if (++ik == K) ik = 0, ir += row_step;
+          }
+        }
+        cp_async_commit();
+      };
+      for (int j = 0; j + 1 < D; ++j) issue_next(j);  // items 0 .. D - 2 (empty groups past the end)
+      float y[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      int slot = 0;  // j % D
+      int64_t cr = r_first;
+      int cs = 0, ck = 0;
+      for (int j = 0; j < items; ++j) {
+        // item j + D - 1 into the slot item j - 1 used (every lane is past it)
+        issue_next(slot == 0 ? D - 1 : slot - 1);
+        cp_async_wait_n(D - 1);  // this lane's copies of item j are done
+        __syncwarp();            // and every lane's
+        item(y, ring + slot * kSlot, cr + rq, cs);
+        __syncwarp();  // every lane is done with the slot before it is refilled
+        slot = slot + 1 == D ? 0 : slot + 1;
+        if (++cs == nspan) {
+          cs = 0;
+          if (++ck == K) {  // the block's rows are complete: store and start over
+            ck = 0;
+            store(y, it, cr + rq);
+            y[0] = y[1] = y[2] = y[3] = 0.0f;
+            cr += row_step;
+          }
         }
       }
-      cp_async_commit();
-    };
-    for (int j = 0; j + 1 < D; ++j) issue_next(j);  // items 0 .. D - 2 (empty groups past the end)
-    float y[4] = {0.0f, 0.0f, 0.0f, 0.0f};  // rows r0 (0, 1) and r0 + 8 (2, 3); activation rows 2t, 2t + 1
-    int slot = 0;  // j % D
-    int64_t cr = r_first;
-    int cs = 0, ck = 0;
-    for (int j = 0; j < items; ++j) {
-      // item j + D - 1 into the slot item j - 1 used (every lane is past it)
-      issue_next(slot == 0 ? D - 1 : slot - 1);
-      cp_async_wait_n(D - 1);  // this lane's copies of item j are done
-      __syncwarp();            // and every lane's
-      const uint8_t* sl = ring + slot * kSlot;
-      const uint32_t* ssl = reinterpret_cast<const uint32_t*>(sl + kCodes);  // [16][kL]
-      const float* zsl = reinterpret_cast<const float*>(sl + kCodes) + kGemvRows * kL;
-      const int64_t r0 = cr + rq;
-      const int64_t g0 = static_cast<int64_t>(cs) * kL;
-      const int lg = ngroups - g0 < kL ? static_cast<int>(ngroups - g0) : kL;
-      // one group of the item: D by G/16 MMAs, then the row sums with the
-      // rows' scales s0, s1, offsets o0, o1 (lo, or -2 s) and the sums sa, sb
-      auto group = [&](int gi, float s0, float s1, float o0, float o1, float sa, float sb) {
-        const int64_t g = g0 + gi;
-        // the lane's W words of rows rq and rq + 8 (one read each)
-        uint32_t c0[W], c1[W];
-        const uint8_t* cb = sl + gi * (G / 4) + t * (G / 16);
-        if constexpr (W == 1) {
-          c0[0] = *reinterpret_cast<const uint32_t*>(cb + rq * kPitch);
-          c1[0] = *reinterpret_cast<const uint32_t*>(cb + (rq + 8) * kPitch);
-        } else if constexpr (W == 2) {
-          const uint2 x0 = *reinterpret_cast<const uint2*>(cb + rq * kPitch);
-          const uint2 x1 = *reinterpret_cast<const uint2*>(cb + (rq + 8) * kPitch);
-          c0[0] = x0.x; c0[1] = x0.y;
-          c1[0] = x1.x; c1[1] = x1.y;
-        } else {
-          const uint4 x0 = *reinterpret_cast<const uint4*>(cb + rq * kPitch);
-          const uint4 x1 = *reinterpret_cast<const uint4*>(cb + (rq + 8) * kPitch);
-          c0[0] = x0.x; c0[1] = x0.y; c0[2] = x0.z; c0[3] = x0.w;
-          c1[0] = x1.x; c1[1] = x1.y; c1[2] = x1.z; c1[3] = x1.w;
-        }
-        float d[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-        const uint4* bt = bt_lane + g * (W * 2 * 4);  // 16-byte units: MMA pairs x 4 lanes
-#pragma unroll
-        for (int w = 0; w < W; ++w) {
-          const uint32_t x6_0 = c0[w] >> 6, x6_1 = c1[w] >> 6, x12_0 = c0[w] >> 12, x12_1 = c1[w] >> 12;
-#pragma unroll
-          for (int h = 0; h < 2; ++h) {  // MMAs e = 2h, 2h + 1: one 16-byte read of B
-            const uint4 b = bt[(w * 2 + h) * 4];
-            uint32_t a[4];
-            if (h == 0) a_frag<0>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
-            else a_frag<2>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
-            mma_bf16_16816(d, a, b.x, b.y);
-            if (h == 0) a_frag<1>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
-            else a_frag<3>(c0[w], c1[w], x6_0, x6_1, x12_0, x12_1, a);
-            mma_bf16_16816(d, a, b.z, b.w);
-          }
-        }
-        // y += s D + lo S (asymmetric), s D - 2 s S (symmetric)
-        y[0] = __fmaf_rn(o0, sa, __fmaf_rn(s0, d[0], y[0]));
-        y[1] = __fmaf_rn(o0, sb, __fmaf_rn(s0, d[1], y[1]));
-        y[2] = __fmaf_rn(o1, sa, __fmaf_rn(s1, d[2], y[2]));
-        y[3] = __fmaf_rn(o1, sb, __fmaf_rn(s1, d[3], y[3]));
+    } else {
+      // groups of P warps: cursors (first row of the block, stage, span) of
+      // this warp's next item to copy and item to multiply; the block ends
+      // when the stage passes K
+      const int per = ipb > wj ? (ipb - wj + P - 1) / P : 0;  // this warp's items of a block
+      struct Cur {
+        int64_t r;
+        int k, s;
       };
-      // a row's scale from its raw 4-byte word (binary16: the half holding element x)
-      auto scale_of = [&](uint32_t u, int64_t x) -> float {
-        if constexpr (kF16) {
-          return __half2float(__ushort_as_half(static_cast<unsigned short>((x & 1) ? u >> 16 : u & 0xFFFFu)));
-        } else {
-          return __uint_as_float(u);
-        }
+      const int k_first = wj / nspan, s_first = wj % nspan;
+      auto advance = [&](Cur& c) {  // true if the stage or block changed
+        c.s += P;
+        if (c.s < nspan) return false;
+        do c.s -= nspan, ++c.k;
+        while (c.s >= nspan);
+        if (c.k >= K) c.k = k_first, c.s = s_first, c.r += row_step;
+        return true;
       };
-      const int64_t x0 = r0 * ngroups + g0, x1 = x0 + 8 * ngroups;  // scale element of rows rq, rq + 8 at g0
-      if (lg == kL) {  // a whole span: C groups' scales, zeros and sums per read; their MMA chains interleave
-        constexpr int C = kL < 4 ? kL : 4;
+      Cur ic{r_first, k_first, s_first};
+      int left = nblk > 0 ? nblk * per : 0;
+      bool fresh = true;  // the copy pointers are for another stage or block
+      auto issue_next = [&](int s_dst) {
+        if (left > 0) {
+          if (fresh) set_stage(it, ic.r, ic.k);
+          issue(it, ic.s, ring_s + s_dst * kSlot);
+          --left;
+          fresh = advance(ic);
+        }
+        cp_async_commit();
+      };
+      for (int j = 0; j + 1 < D; ++j) issue_next(j);
+      int slot = 0;
+      Cur cc{r_first, k_first, s_first};
+      float* red = reinterpret_cast<float*>(smem + red_off);  // [16 warps][32 lanes][4]
+      for (int b = 0; b < nblk; ++b) {
+        float y[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+        const int64_t r0 = cc.r + rq;
+        for (int u = 0; u < per; ++u) {
+          issue_next(slot == 0 ? D - 1 : slot - 1);
+          cp_async_wait_n(D - 1);
+          __syncwarp();
+          item(y, ring + slot * kSlot, cc.r + rq, cc.s);
+          __syncwarp();
+          slot = slot + 1 == D ? 0 : slot + 1;
+          advance(cc);
+        }
+        // the block's rows are complete: sum the group's parts in warp order and store
+        if (wj > 0) {
 #pragma unroll
-        for (int h = 0; h < kL; h += C) {
-          uint32_t u0[C], u1[C];
-          float z0[C], z1[C], sa[C], sb[C];
-          lds_vec<C>(ssl + rq * kL + h, u0);
-          lds_vec<C>(ssl + (rq + 8) * kL + h, u1);
-          lds_vec<C>(sa_lane + g0 + h, sa);
-          lds_vec<C>(sb_lane + g0 + h, sb);
-          if constexpr (!kSym) {
-            lds_vec<C>(zsl + rq * kL + h, z0);
-            lds_vec<C>(zsl + (rq + 8) * kL + h, z1);
-          }
+          for (int q = 0; q < 4; ++q) red[(warp * 32 + lane) * 4 + q] = y[q];
+        }
+        named_barrier(1 + grp, P * 32);
+        if (wj == 0) {
+          for (int j = 1; j < P; ++j)
 #pragma unroll
-          for (int i = 0; i < C; ++i) {
-            const float s0 = scale_of(u0[i], x0 + h + i), s1 = scale_of(u1[i], x1 + h + i);
-            group(h + i, s0, s1, kSym ? -2.0f * s0 : z0[i], kSym ? -2.0f * s1 : z1[i], sa[i], sb[i]);
-          }
+            for (int q = 0; q < 4; ++q) y[q] = __fadd_rn(y[q], red[((warp + j) * 32 + lane) * 4 + q]);
+          store(y, it, r0);
         }
-      } else {
-        for (int gi = 0; gi < lg; ++gi) {
-          const float s0 = scale_of(ssl[rq * kL + gi], x0 + gi), s1 = scale_of(ssl[(rq + 8) * kL + gi], x1 + gi);
-          const float o0 = kSym ? -2.0f * s0 : zsl[rq * kL + gi], o1 = kSym ? -2.0f * s1 : zsl[(rq + 8) * kL + gi];
-          group(gi, s0, s1, o0, o1, sa_lane[g0 + gi], sb_lane[g0 + gi]);
-        }
-      }
-      __syncwarp();  // every lane is done with the slot before it is refilled
-      slot = slot + 1 == D ? 0 : slot + 1;
-      if (++cs == nspan) {
-        cs = 0;
-        if (++ck == K) {  // the block's rows are complete: store and start over
-          ck = 0;
-          cr += kRowStep;
-          const int64_t r1 = r0 + 8;
-          const int n0 = 2 * t, n1 = 2 * t + 1;
-          if (r0 < it.rows) {
-            if (n0 < nb) it.Y[static_cast<int64_t>(n0) * it.rows + r0] = scalbnf(y[0], back0);
-            if (n1 < nb) it.Y[static_cast<int64_t>(n1) * it.rows + r0] = scalbnf(y[1], back1);
-          }
-          if (r1 < it.rows) {
-            if (n0 < nb) it.Y[static_cast<int64_t>(n0) * it.rows + r1] = scalbnf(y[2], back0);
-            if (n1 < nb) it.Y[static_cast<int64_t>(n1) * it.rows + r1] = scalbnf(y[3], back1);
-          }
-          y[0] = y[1] = y[2] = y[3] = 0.0f;
-        }
+        named_barrier(1 + grp, P * 32);  // the parts are read before the next block's
       }
     }
     cp_async_wait<0>();  // the empty groups of the last items
@@ -467,26 +550,46 @@ gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D
   }
 }
 
+// the group partial sums of a launch with more than one warp per block
+constexpr int kMmaRedBytes = kMmaWarps * 32 * 4 * 4;
+
 // activation rows one launch of the tensor-core form holds for matrices of up
 // to max_cols columns, with a ring of at least 2 slots of 512-column spans a
-// warp (0 if not even one row fits)
+// warp and the partial sums (0 if not even one row fits)
 inline int mma_rows_per_launch(bool sym, int64_t max_cols, int group) {
   const int span = group > 512 ? group : 512;
   for (int nb = kMaxGemvBatch; nb >= 1; --nb)
-    if (mma_ring_slots(sym, group, span, mma_table_bytes(max_cols, nb, group), kMmaSmemMax) >= 2) return nb;
+    if (mma_ring_slots(sym, group, span, mma_table_bytes(max_cols, nb, group) + kMmaRedBytes, kMmaSmemMax) >= 2)
+      return nb;
   return 0;
 }
 
+// Warps per block: 1 while every CTA holds at least 16 blocks; else the
+// smallest CTA's blocks (rounded down to a power of two) times P make 16, so
+// that each group of P warps has a block (launches over few rows, e.g. the
+// matrices of one layer).
+inline int mma_warps_per_block(const GemvBatch& p) {
+  int64_t least = p.total_blocks;
+  for (int c = 0; c < p.grid; ++c) {
+    const int64_t n = p.cta_begin[c + 1] - p.cta_begin[c];
+    if (n < least) least = n;
+  }
+  int P = 1;
+  while (P < kMmaWarps && least * P < kMmaWarps) P *= 2;
+  return P;
+}
+
 template <int F, int K, int G, int S>
-cudaError_t mma_launch_kgs(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms, int D) {
+cudaError_t mma_launch_kgs(GemvBatch& p, int nb, int64_t tables, int P, cudaStream_t stream, int D) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
-  const int64_t tables = mma_table_bytes(max_cols, nb, G);
-  const int smem = static_cast<int>(tables + static_cast<int64_t>(kMmaWarps) * D * mma_slot_bytes(kSym, G, S));
-  int64_t grid = sms;  // one 16-warp CTA per multiprocessor
-  if (grid > kMaxGemvGrid) grid = kMaxGemvGrid;
-  if (grid > p.total_blocks) grid = p.total_blocks;
-  gemv_split(p, static_cast<int>(grid));
-  gemv_mma_kernel<F, K, G, S><<<p.grid, kMmaThreads, smem, stream>>>(p, nb, static_cast<int>(tables), D);
+  const int64_t ring = static_cast<int64_t>(kMmaWarps) * D * mma_slot_bytes(kSym, G, S);
+  const int red = P > 1 ? kMmaRedBytes : 0;
+  const int smem = static_cast<int>(tables + ring + red);
+  const int ring_off = static_cast<int>(tables), red_off = static_cast<int>(tables + ring);
+  if (P > 1)
+    gemv_mma_kernel<F, K, G, S, true><<<p.grid, kMmaThreads, smem, stream>>>(p, nb, ring_off, D, P, red_off);
+  else
+    gemv_mma_kernel<F, K, G, S, false><<<p.grid, kMmaThreads, smem, stream>>>(p, nb, ring_off, D, 1, red_off);
   return cudaGetLastError();
 }
 
@@ -495,15 +598,21 @@ cudaError_t mma_launch_kgs(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t 
 template <int F, int K, int G>
 cudaError_t mma_launch_kg(GemvBatch& p, int nb, int64_t max_cols, cudaStream_t stream, int sms) {
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
+  int64_t grid = sms;  // one 16-warp CTA per multiprocessor
+  if (grid > kMaxGemvGrid) grid = kMaxGemvGrid;
+  if (grid > p.total_blocks) grid = p.total_blocks;
+  gemv_split(p, static_cast<int>(grid));
+  const int P = mma_warps_per_block(p);
   const int64_t tables = mma_table_bytes(max_cols, nb, G);
+  const int64_t fixed = tables + (P > 1 ? kMmaRedBytes : 0);
   if constexpr (G >= 128) {
-    const int d = mma_ring_slots(kSym, G, 1024, tables, kMmaSmemMax);
-    if (d >= 2) return mma_launch_kgs<F, K, G, 1024>(p, nb, max_cols, stream, sms, d);
+    const int d = mma_ring_slots(kSym, G, 1024, fixed, kMmaSmemMax);
+    if (d >= 2) return mma_launch_kgs<F, K, G, 1024>(p, nb, tables, P, stream, d);
   }
   constexpr int S0 = G > 512 ? G : 512;
-  const int d = mma_ring_slots(kSym, G, S0, tables, kMmaSmemMax);
+  const int d = mma_ring_slots(kSym, G, S0, fixed, kMmaSmemMax);
   if (d < 2) return cudaErrorInvalidValue;  // the caller sizes nb by mma_rows_per_launch
-  return mma_launch_kgs<F, K, G, S0>(p, nb, max_cols, stream, sms, d);
+  return mma_launch_kgs<F, K, G, S0>(p, nb, tables, P, stream, d);
 }
 
 template <int F, int K>
@@ -527,15 +636,22 @@ cudaError_t mma_launch_format(int group, int k, int nb, int64_t max_cols, GemvBa
   }
 }
 
+template <int F, int K, int G, int S>
+cudaError_t mma_prepare_kgs() {
+  cudaError_t e;
+  const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
+  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, G, S, false>, a, kMmaSmemMax))) return e;
+  return cudaFuncSetAttribute(gemv_mma_kernel<F, K, G, S, true>, a, kMmaSmemMax);
+}
+
 template <int F, int K>
 cudaError_t mma_prepare_k() {
   cudaError_t e;
-  const cudaFuncAttribute a = cudaFuncAttributeMaxDynamicSharedMemorySize;
-  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 64, 512>, a, kMmaSmemMax))) return e;
-  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 128, 512>, a, kMmaSmemMax))) return e;
-  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 128, 1024>, a, kMmaSmemMax))) return e;
-  if ((e = cudaFuncSetAttribute(gemv_mma_kernel<F, K, 256, 512>, a, kMmaSmemMax))) return e;
-  return cudaFuncSetAttribute(gemv_mma_kernel<F, K, 256, 1024>, a, kMmaSmemMax);
+  if ((e = mma_prepare_kgs<F, K, 64, 512>())) return e;
+  if ((e = mma_prepare_kgs<F, K, 128, 512>())) return e;
+  if ((e = mma_prepare_kgs<F, K, 128, 1024>())) return e;
+  if ((e = mma_prepare_kgs<F, K, 256, 512>())) return e;
+  return mma_prepare_kgs<F, K, 256, 1024>();
 }
 
 template <int F>

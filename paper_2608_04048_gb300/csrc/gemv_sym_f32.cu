@@ -1,17 +1,17 @@
 // Stage-wise product kernels for one package format (see gemv_kernel.cuh).
-#include "gemv_mma_kernel.cuh"
+#include "gemv_kernel.cuh"
 
 namespace rrq {
 
 cudaError_t gemv_prepare_sym_f32() {
   cudaError_t e = prepare_format<kSymF32>();
-  return e != cudaSuccess ? e : mma_prepare_format<kSymF32>();
+  return e != cudaSuccess ? e : gemv_mma_prepare_sym_f32();
 }
 
 cudaError_t gemv_launch_sym_f32(int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream, int sms) {
-  // groups of 64 and more: the factored form on the tensor cores
-  // (gemv_mma_kernel.cuh); groups of 32: the prefix-weight form
-  if (p.log2g >= 6) return mma_launch_format<kSymF32>(1 << p.log2g, k, nb, max_cols, p, stream, sms);
+  // groups of 64 and more: the stage-wise form on the tensor cores
+  // (gemv_mma_{format}.cu); groups of 32: the prefix-weight form
+  if (p.log2g >= 6) return gemv_mma_launch_sym_f32(1 << p.log2g, k, nb, max_cols, p, stream, sms);
   return launch_format<kSymF32>(k, nb, max_cols, p, stream, sms);
 }
 

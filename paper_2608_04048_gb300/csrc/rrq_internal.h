@@ -265,6 +265,16 @@ cudaError_t gemv_launch_asym_bits(int k, int nb, int64_t max_cols, GemvBatch& p,
 
 // Once per device: the decode product's kernels may take the shared memory
 // their largest launch needs.
+// the tensor-core form (groups of 64 and more, 2-bit stages), one unit per format
+cudaError_t gemv_mma_launch_asym_f32(int group, int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream,
+                                     int sms);
+cudaError_t gemv_mma_launch_sym_f32(int group, int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream,
+                                    int sms);
+cudaError_t gemv_mma_launch_sym_f16(int group, int k, int nb, int64_t max_cols, GemvBatch& p, cudaStream_t stream,
+                                    int sms);
+cudaError_t gemv_mma_prepare_asym_f32();
+cudaError_t gemv_mma_prepare_sym_f32();
+cudaError_t gemv_mma_prepare_sym_f16();
 cudaError_t gemv_prepare_asym_f32();
 cudaError_t gemv_prepare_sym_f32();
 cudaError_t gemv_prepare_sym_f16();
