@@ -13,7 +13,10 @@
 //
 // Layout.  A CTA of 16 warps takes a contiguous range of 16-row blocks
 // (gemv_split), matrix by matrix; a warp takes whole blocks (w, w + 16, ...
-// of the CTA's blocks of a matrix).  A block is walked stage by stage, each
+// of the CTA's blocks of a matrix).  Where some CTA holds fewer than 16
+// blocks (a launch over few rows, such as the matrices of one layer), groups
+// of P warps share each block instead, each warp taking every P-th item, and
+// the group adds its parts of the rows' sums in warp order.  A block is walked stage by stage, each
 // stage in spans of kSpan = max(512, G) columns: the item (block, stage,
 // span) is 16 rows x kSpan/4 contiguous bytes of codes per row -- whole
 // 128-byte lines, so that each DRAM page opened for a row serves a whole
@@ -43,7 +46,8 @@
 // with d = (k + 1) + G/16 + 8 + 2k groups + 18: the stage levels and their
 // sum that W~ rounds (k + 1), the G/16 MMA steps of D, the sum S_g (a sum of
 // 8 then a tree over G/8, at most 8 roundings at G = 256), two fma per group
-// and stage into the row's sum, and slack (18).
+// and stage into the row's sum, and slack (18, which also covers the P - 1 <=
+// 15 additions of a group's parts: each part holds fewer of the row's terms).
 #pragma once
 
 #include <cuda_bf16.h>

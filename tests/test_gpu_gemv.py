@@ -212,6 +212,21 @@ def test_activation_scales(group, fmt):
         _check(pkg, A, Y, k, where=f"g{group} {fmt} k{k} scaled rows")
 
 
+@pytest.mark.parametrize("fmt", FORMATS, ids=FMT_IDS)
+def test_one_warp_per_block(fmt):
+    """A launch with at least 16 blocks of 16 rows in every CTA takes one warp
+    per block (the form the whole stack takes); smaller launches share each
+    block among a group of warps.  Both against the oracle on every row."""
+    rows, cols, group = 40960, 512, 128  # 2560 blocks over at most 152 CTAs
+    W = workloads.generate(rows, cols, 91, "t3_rowout", "cuda")
+    (pkg,) = binding.rrq_quantize_ex([W], group, 4, *fmt)
+    for batch in (1, 5):
+        A = _acts(batch, cols, seed=batch + 17)
+        for k in (1, 4):
+            (Y,) = binding.rrq_gemv([pkg], [A], k)
+            _check(pkg, A, Y, k, where=f"{fmt} B{batch} k{k}")
+
+
 def test_batch_across_launches():
     rng = np.random.default_rng(12)
     shapes = [(int(rng.integers(1, 40)), 128 * int(rng.integers(1, 20))) for _ in range(70)]
