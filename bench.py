@@ -784,8 +784,8 @@ KERNEL_SOURCES = {
     "rrq_reconstruct_k4": ["reconstruct_kernel.cuh", "reconstruct_tile_kernel.cuh", "reconstruct_asym_f32.cu"],
     "rrq_reconstruct_ex_sym_f16": ["reconstruct_kernel.cuh", "reconstruct_tile_kernel.cuh", "reconstruct_sym_f16.cu"],
     "rrq_quantize_prefixes": ["quantize_kernel.cuh", "quantize_emit.cu"],
-    "rrq_gemv_k1": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
-    "rrq_gemv_k4": ["gemv_kernel.cuh", "gemv_asym_f32.cu"],
+    "rrq_gemv_k1": ["gemv_mma_kernel.cuh", "gemv_kernel.cuh", "gemv_mma_asym_f32.cu", "gemv_asym_f32.cu"],
+    "rrq_gemv_k4": ["gemv_mma_kernel.cuh", "gemv_kernel.cuh", "gemv_mma_asym_f32.cu", "gemv_asym_f32.cu"],
 }
 
 # the kernel (ncu demangled-name prefix) and algorithmic bytes per weight at
@@ -796,6 +796,8 @@ TRAFFIC_KERNELS = {
     "rrq_reconstruct_prefixes": ("reconstruct_kernel<128, 4, 1, 0>", 9.25),
     "rrq_reconstruct_k4": ("reconstruct_tile_kernel<128, 4, 0>", 3.25),
     "rrq_quantize_prefixes": ("quantize_kernel<128, 0, 2>", 11.25),
+    "rrq_gemv_k1": ("gemv_mma_kernel<0, 1, 128,", 0.25 + 8 / 128),
+    "rrq_gemv_k4": ("gemv_mma_kernel<0, 4, 128,", 4 * (0.25 + 8 / 128)),
 }
 
 
