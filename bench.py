@@ -630,10 +630,11 @@ def run_gpu(args, world, rank, local) -> dict | None:
         raise RuntimeError("a kernel reported a timeout in the breakdown")
 
     stack = args.workload == "qwen3_8b_stack" and wl.own_outputs and not args.no_sym
-    # the two products also on one layer (the size their ncu captures take)
+    # the symmetric binary16 format and the two products also on one layer
+    # (the size their ncu captures take)
     products = stack or (args.workload == "qwen3_8b_layer" and wl.own_outputs and not args.no_sym)
     mats, pkgs, p_outs = wl.mats, wl.pkgs, wl.p_outs
-    sym = time_sym_f16(mats, p_outs, specs, stream) if stack else None
+    sym = time_sym_f16(mats, p_outs, specs, stream) if products else None
     from_base = time_from_base(mats, pkgs, specs, stream) if stack else None
     gemv = time_gemv(pkgs, specs, stream) if products else None
     batches = [int(x) for x in args.gemv_batches.split(",") if x.strip()]
@@ -796,6 +797,7 @@ TRAFFIC_KERNELS = {
     "rrq_reconstruct_prefixes": ("reconstruct_kernel<128, 4, 1, 0>", 9.25),
     "rrq_reconstruct_k4": ("reconstruct_tile_kernel<128, 4, 0>", 3.25),
     "rrq_quantize_prefixes": ("quantize_kernel<128, 0, 2>", 11.25),
+    "rrq_reconstruct_ex_sym_f16": ("reconstruct_kernel<128, 4, 1, 2>", 4 * (0.25 + 2 / 128) + 8),
     "rrq_gemv_k1": ("gemv_mma_kernel<0, 1, 128,", 0.25 + 8 / 128),
     "rrq_gemv_k4": ("gemv_mma_kernel<0, 4, 128,", 4 * (0.25 + 8 / 128)),
 }
