@@ -7,7 +7,11 @@
 // Lane 0 brings the chunk's package into a per-warp ring with one 1-D bulk
 // copy per stage and array (codes 512 bytes, the 2048/g scales and zeros),
 // completing on the slot's mbarrier; each lane reads its 16 code bytes and
-// its group's scale and zero from there.  The bf16 result goes out through a
+// its group's scale and zero from there.  At k = 1 the lane forms its 64
+// levels and then converts them; for k >= 2 it sums 4 weights over all k
+// stages (in stage order, as Eq. 8 reads) before the next 4, converting as
+// it goes, which keeps few accumulators live and leaves room for 12 warps a
+// CTA (RtCfg).  The bf16 result goes out through a
 // 2-D TMA store of the matrix viewed as [n/64, 64] with the 128-byte swizzle:
 // a lane writes its 16-byte piece j at piece j ^ (l & 7) of its 128-byte row
 // (the eight lanes of a quarter warp hit eight bank groups) and the copy
@@ -21,21 +25,20 @@
 namespace rrq {
 namespace {
 
-#ifndef RRQ_RT_WARPS
-#define RRQ_RT_WARPS 8
-#endif
-#ifndef RRQ_RT_RING
-#define RRQ_RT_RING 3
-#endif
-#ifndef RRQ_RT_CTAS_PER_SM
-#define RRQ_RT_CTAS_PER_SM 2
-#endif
-#ifndef RRQ_RT_SLEEP
-#define RRQ_RT_SLEEP 0
-#endif
-constexpr int kRtWarps = RRQ_RT_WARPS;
-constexpr int kRtThreads = kRtWarps * 32;
-constexpr int kRtRing = RRQ_RT_RING;             // chunks of package per warp in flight
+// Launch shape by prefix.  At k = 1 a lane sums nothing: it keeps its 64
+// levels in registers and writes them after, 8 warps a CTA with three chunks
+// of package in flight per warp.  For k >= 2 a lane finishes 4 weights over
+// all k stages before the next 4 (few live accumulators), which leaves room
+// for 12 warps a CTA with two chunks in flight.  Two CTAs per multiprocessor
+// in both.
+template <int K>
+struct RtCfg {
+  static constexpr bool kOuter = K > 1;
+  static constexpr int kWarps = kOuter ? 12 : 8;
+  static constexpr int kThreads = kWarps * 32;
+  static constexpr int kRing = kOuter ? 2 : 3;  // chunks of package per warp in flight
+};
+constexpr int kRtCtasPerSm = 2;
 constexpr int kRtChunk = 2048;                   // weights per warp chunk
 constexpr int kRtOutBytes = kRtChunk * 2;        // bf16 output of a chunk (one TMA box)
 
@@ -51,9 +54,11 @@ struct RtStage {  // bytes of one stage of one chunk in the ring
 template <int G, int K, int F>
 __host__ __device__ constexpr int rt_slot_bytes() { return K * RtStage<G, F>::kBytes; }
 template <int G, int K, int F>
-__host__ __device__ constexpr int rt_warp_bytes() { return kRtRing * rt_slot_bytes<G, K, F>() + kRtOutBytes; }
+__host__ __device__ constexpr int rt_warp_bytes() { return RtCfg<K>::kRing * rt_slot_bytes<G, K, F>() + kRtOutBytes; }
 template <int G, int K, int F>
-__host__ __device__ constexpr int rt_smem_bytes() { return kRtWarps * rt_warp_bytes<G, K, F>() + kRtWarps * kRtRing * 8 + 1024; }
+__host__ __device__ constexpr int rt_smem_bytes() {
+  return RtCfg<K>::kWarps * (rt_warp_bytes<G, K, F>() + RtCfg<K>::kRing * 8) + 1024;
+}
 
 __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int y, uint32_t src) {
   asm volatile("cp.async.bulk.tensor.2d.global.shared::cta.tile.bulk_group [%0, {%1, %2}], [%3];" ::"l"(
@@ -62,30 +67,10 @@ __device__ __forceinline__ void tma_store_2d(const CUtensorMap* map, int x, int 
                : "memory");
 }
 
-// Bounded wait that suspends in the barrier between checks (a time hint of
-// up to 1 ms per try) instead of returning at once.
-__device__ __forceinline__ bool rt_wait(uint32_t bar, uint32_t parity, uint32_t limit_us) {
-#if RRQ_RT_SLEEP
-  if (limit_us == 0) return false;
-  const uint64_t t0 = globaltimer_ns();
-  const uint64_t limit_ns = static_cast<uint64_t>(limit_us) * 1000u;
-  while (true) {
-    uint32_t done;
-    asm volatile(
-        "{ .reg .pred p; mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3; selp.u32 %0, 1, 0, p; }"
-        : "=r"(done)
-        : "r"(bar), "r"(parity), "r"(1000000u)
-        : "memory");
-    if (done) return true;
-    if (globaltimer_ns() - t0 > limit_ns) return false;
-  }
-#else
-  return mbar_wait(bar, parity, limit_us);
-#endif
-}
-
 template <int G, int K, int F>
-__global__ void __launch_bounds__(kRtThreads, RRQ_RT_CTAS_PER_SM) reconstruct_tile_kernel(const __grid_constant__ ReconstructTileBatch p) {
+__global__ void __launch_bounds__(RtCfg<K>::kThreads, kRtCtasPerSm) reconstruct_tile_kernel(const __grid_constant__ ReconstructTileBatch p) {
+  constexpr int kRtWarps = RtCfg<K>::kWarps;
+  constexpr int kRtRing = RtCfg<K>::kRing;
   constexpr bool kSym = F == kSymF32 || F == kSymF16;
   constexpr bool kF16 = F == kSymF16;
   using St = RtStage<G, F>;
@@ -149,7 +134,7 @@ __global__ void __launch_bounds__(kRtThreads, RRQ_RT_CTAS_PER_SM) reconstruct_ti
   bool stored = false;
   for (int64_t chunk = first; chunk < b.total_chunks; chunk += stride, ++iter) {
     const int slot = iter % kRtRing;
-    const bool ready = rt_wait(bar0 + 8 * slot, (iter / kRtRing) & 1, b.wait_limit_us);
+    const bool ready = mbar_wait(bar0 + 8 * slot, (iter / kRtRing) & 1, b.wait_limit_us);
     if (!__all_sync(kFullMask, ready)) {
       // Give up: record it, wait (bounded) for this warp's copies in flight
       // so that none lands in freed shared memory, and leave.
@@ -193,69 +178,138 @@ __global__ void __launch_bounds__(kRtThreads, RRQ_RT_CTAS_PER_SM) reconstruct_ti
     const int m = item_of(chunk, m_work);
     const ReconstructItem& it = b.item[m];
 
-    f32x2 acc[32];
     const bool all_ok = __all_sync(kFullMask, ok);
+    if constexpr (RtCfg<K>::kOuter) {
+      if (stored && lane == 0) bulk_wait_read<0>();  // the previous chunk's store has read the buffer
+      __syncwarp();
+      uint8_t* row = out_stage + lane * 128;
+      // Weights in 16-byte output pieces: piece q holds code bytes 2q and 2q+1
+      // (8 weights), each summed over all k stages before the next, so that
+      // only a few accumulators are live.  form(i, h, b8, a01, a23) adds stage
+      // i's levels of the four codes of byte b8 (group half h) in stage order.
+      auto run = [&](auto form) {
 #pragma unroll
-    for (int i = 0; i < K; ++i) {
-      const uint32_t words[4] = {code[i].x, code[i].y, code[i].z, code[i].w};
+        for (int q = 0; q < 8; ++q) {
+          uint32_t hw[4];
 #pragma unroll
-      for (int h = 0; h < NH; ++h) {
-        constexpr int kBytesPerHalf = 16 / NH;
-        if (kSym) {
+          for (int jj = 0; jj < 2; ++jj) {
+            const int j = 2 * q + jj;
+            constexpr int kBytesPerHalf = 16 / NH;
+            const int h = j / kBytesPerHalf;
+            f32x2 a01, a23;
+#pragma unroll
+            for (int i = 0; i < K; ++i) {
+              const uint32_t w = (j >> 2) == 0 ? code[i].x : (j >> 2) == 1 ? code[i].y : (j >> 2) == 2 ? code[i].z : code[i].w;
+              const uint32_t b8 = (j & 3) == 0 ? w : (w >> (8 * (j & 3)));
+              form(i, h, b8, a01, a23);
+            }
+            float x, y;
+            unpack2(a01, x, y);
+            __nv_bfloat162 v = __floats2bfloat162_rn(x, y);
+            hw[2 * jj] = *reinterpret_cast<const uint32_t*>(&v);
+            unpack2(a23, x, y);
+            v = __floats2bfloat162_rn(x, y);
+            hw[2 * jj + 1] = *reinterpret_cast<const uint32_t*>(&v);
+          }
+          *reinterpret_cast<uint4*>(row + ((q ^ (lane & 7)) << 4)) = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+        }
+      };
+      if constexpr (kSym) {
+        run([&](int i, int h, uint32_t b8, f32x2& a01, f32x2& a23) {
           const f32x2 S = pack2(scale[i][h], scale[i][h]);
+          f32x2 u01, u23;
+          sym_offsets(b8, u01, u23);
+          a01 = (i == 0) ? mul2(u01, S) : fma2(u01, S, a01);
+          a23 = (i == 0) ? mul2(u23, S) : fma2(u23, S, a23);
+        });
+      } else if (all_ok) {
+        StageConsts cs[K][NH];
 #pragma unroll
-          for (int j = h * kBytesPerHalf; j < (h + 1) * kBytesPerHalf; ++j) {  // byte j: elements 4j..4j+3
-            const uint32_t word = words[j >> 2];
-            const uint32_t b8 = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-            f32x2 u01, u23;
-            sym_offsets(b8, u01, u23);
-            acc[2 * j] = (i == 0) ? mul2(u01, S) : fma2(u01, S, acc[2 * j]);
-            acc[2 * j + 1] = (i == 0) ? mul2(u23, S) : fma2(u23, S, acc[2 * j + 1]);
-          }
-        } else if (all_ok) {
-          const StageConsts c = stage_consts(scale[i][h], zero[i][h]);
+        for (int i = 0; i < K; ++i)
 #pragma unroll
-          for (int j = h * kBytesPerHalf; j < (h + 1) * kBytesPerHalf; ++j) {
-            const uint32_t word = words[j >> 2];
-            const uint32_t b8 = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-            f32x2 l01, l23;
-            asym_levels(b8, c, l01, l23);
-            acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
-            acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
-          }
-        } else {  // a scale outside [2^-100, 2^100] in the warp: fl(Q s) as a plain (t - 2^23) s
+          for (int h = 0; h < NH; ++h) cs[i][h] = stage_consts(scale[i][h], zero[i][h]);
+        run([&](int i, int h, uint32_t b8, f32x2& a01, f32x2& a23) {
+          f32x2 l01, l23;
+          asym_levels(b8, cs[i][h], l01, l23);
+          a01 = (i == 0) ? l01 : add2(a01, l01);
+          a23 = (i == 0) ? l23 : add2(a23, l23);
+        });
+      } else {  // a scale outside [2^-100, 2^100] in the warp: fl(Q s) as a plain (t - 2^23) s
+        run([&](int i, int h, uint32_t b8, f32x2& a01, f32x2& a23) {
           const f32x2 Z = pack2(zero[i][h], zero[i][h]), S = pack2(scale[i][h], scale[i][h]);
           const f32x2 T23 = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f);
+          const f32x2 t01 = pack2u(magic23<3u>(b8), magic23<3u>(b8 >> 2));
+          const f32x2 t23 = pack2u(magic23<3u>(b8 >> 4), magic23<3u>(b8 >> 6));
+          const f32x2 l01 = add2(Z, fma2(sub2(t01, T23), S, Z0));
+          const f32x2 l23 = add2(Z, fma2(sub2(t23, T23), S, Z0));
+          a01 = (i == 0) ? l01 : add2(a01, l01);
+          a23 = (i == 0) ? l23 : add2(a23, l23);
+        });
+      }
+    } else {
+      f32x2 acc[32];
 #pragma unroll
-          for (int j = h * kBytesPerHalf; j < (h + 1) * kBytesPerHalf; ++j) {
-            const uint32_t word = words[j >> 2];
-            const uint32_t b8 = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
-            const f32x2 t01 = pack2u(magic23<3u>(b8), magic23<3u>(b8 >> 2));
-            const f32x2 t23 = pack2u(magic23<3u>(b8 >> 4), magic23<3u>(b8 >> 6));
-            const f32x2 l01 = add2(Z, fma2(sub2(t01, T23), S, Z0));
-            const f32x2 l23 = add2(Z, fma2(sub2(t23, T23), S, Z0));
-            acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
-            acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
+      for (int i = 0; i < K; ++i) {
+        const uint32_t words[4] = {code[i].x, code[i].y, code[i].z, code[i].w};
+#pragma unroll
+        for (int h = 0; h < NH; ++h) {
+          constexpr int kBytesPerHalf = 16 / NH;
+          if (kSym) {
+            const f32x2 S = pack2(scale[i][h], scale[i][h]);
+#pragma unroll
+            for (int j = h * kBytesPerHalf; j < (h + 1) * kBytesPerHalf; ++j) {  // byte j: elements 4j..4j+3
+              const uint32_t word = words[j >> 2];
+              const uint32_t b8 = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
+              f32x2 u01, u23;
+              sym_offsets(b8, u01, u23);
+              acc[2 * j] = (i == 0) ? mul2(u01, S) : fma2(u01, S, acc[2 * j]);
+              acc[2 * j + 1] = (i == 0) ? mul2(u23, S) : fma2(u23, S, acc[2 * j + 1]);
+            }
+          } else if (all_ok) {
+            const StageConsts c = stage_consts(scale[i][h], zero[i][h]);
+#pragma unroll
+            for (int j = h * kBytesPerHalf; j < (h + 1) * kBytesPerHalf; ++j) {
+              const uint32_t word = words[j >> 2];
+              const uint32_t b8 = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
+              f32x2 l01, l23;
+              asym_levels(b8, c, l01, l23);
+              acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
+              acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
+            }
+          } else {  // a scale outside [2^-100, 2^100] in the warp: fl(Q s) as a plain (t - 2^23) s
+            const f32x2 Z = pack2(zero[i][h], zero[i][h]), S = pack2(scale[i][h], scale[i][h]);
+            const f32x2 T23 = pack2(kTwo23, kTwo23), Z0 = pack2(0.0f, 0.0f);
+#pragma unroll
+            for (int j = h * kBytesPerHalf; j < (h + 1) * kBytesPerHalf; ++j) {
+              const uint32_t word = words[j >> 2];
+              const uint32_t b8 = (j & 3) == 0 ? word : (word >> (8 * (j & 3)));
+              const f32x2 t01 = pack2u(magic23<3u>(b8), magic23<3u>(b8 >> 2));
+              const f32x2 t23 = pack2u(magic23<3u>(b8 >> 4), magic23<3u>(b8 >> 6));
+              const f32x2 l01 = add2(Z, fma2(sub2(t01, T23), S, Z0));
+              const f32x2 l23 = add2(Z, fma2(sub2(t23, T23), S, Z0));
+              acc[2 * j] = (i == 0) ? l01 : add2(acc[2 * j], l01);
+              acc[2 * j + 1] = (i == 0) ? l23 : add2(acc[2 * j + 1], l23);
+            }
           }
         }
       }
-    }
 
-    // bf16 round-to-nearest-even into this lane's swizzled 128-byte row
-    uint32_t h[32];
+      // bf16 round-to-nearest-even into this lane's swizzled 128-byte row
+      uint32_t h[32];
 #pragma unroll
-    for (int q = 0; q < 32; ++q) {
-      float x, y;
-      unpack2(acc[q], x, y);
-      const __nv_bfloat162 v = __floats2bfloat162_rn(x, y);
-      h[q] = *reinterpret_cast<const uint32_t*>(&v);
+      for (int q = 0; q < 32; ++q) {
+        float x, y;
+        unpack2(acc[q], x, y);
+        const __nv_bfloat162 v = __floats2bfloat162_rn(x, y);
+        h[q] = *reinterpret_cast<const uint32_t*>(&v);
+      }
+      if (stored && lane == 0) bulk_wait_read<0>();  // the previous chunk's store has read the buffer
+      __syncwarp();
+      uint8_t* row = out_stage + lane * 128;
+#pragma unroll
+      for (int j = 0; j < 8; ++j)
+        *reinterpret_cast<uint4*>(row + ((j ^ (lane & 7)) << 4)) = make_uint4(h[4 * j], h[4 * j + 1], h[4 * j + 2], h[4 * j + 3]);
     }
-    if (stored && lane == 0) bulk_wait_read<0>();  // the previous chunk's store has read the buffer
-    __syncwarp();
-    uint8_t* row = out_stage + lane * 128;
-#pragma unroll
-    for (int j = 0; j < 8; ++j)
-      *reinterpret_cast<uint4*>(row + ((j ^ (lane & 7)) << 4)) = make_uint4(h[4 * j], h[4 * j + 1], h[4 * j + 2], h[4 * j + 3]);
     fence_proxy_async_smem();
     __syncwarp();
     if (lane == 0) {
@@ -296,15 +350,15 @@ cudaError_t rt_launch_gk(const ReconstructTileBatch& p, cudaStream_t stream, int
   int blocks_per_sm = cached.load(std::memory_order_relaxed);
   if (blocks_per_sm == 0) {
     cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&blocks_per_sm, reconstruct_tile_kernel<G, K, F>,
-                                                                  kRtThreads, rt_smem_bytes<G, K, F>());
+                                                                  RtCfg<K>::kThreads, rt_smem_bytes<G, K, F>());
     if (e != cudaSuccess) return e;
     if (blocks_per_sm < 1) blocks_per_sm = 1;
     cached.store(blocks_per_sm, std::memory_order_relaxed);
   }
-  const int64_t want = (p.b.total_chunks + kRtWarps - 1) / kRtWarps;
+  const int64_t want = (p.b.total_chunks + RtCfg<K>::kWarps - 1) / RtCfg<K>::kWarps;
   const int64_t cap = static_cast<int64_t>(sms) * blocks_per_sm;
   const int grid = static_cast<int>(want < cap ? want : cap);
-  reconstruct_tile_kernel<G, K, F><<<grid, kRtThreads, rt_smem_bytes<G, K, F>(), stream>>>(p);
+  reconstruct_tile_kernel<G, K, F><<<grid, RtCfg<K>::kThreads, rt_smem_bytes<G, K, F>(), stream>>>(p);
   return cudaGetLastError();
 }
 
