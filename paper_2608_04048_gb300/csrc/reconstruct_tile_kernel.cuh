@@ -4,10 +4,11 @@
 // round-to-nearest-even, with L_i formed by asym_levels / sym_offsets).
 //
 // A warp owns a chunk of 2048 consecutive weights; lane l owns 64 of them.
-// Lane 0 brings the chunk's package into a per-warp ring with one 1-D bulk
-// copy per stage and array (codes 512 bytes, the 2048/g scales and zeros),
-// completing on the slot's mbarrier; each lane reads its 16 code bytes and
-// its group's scale and zero from there.  At k = 1 the lane forms its 64
+// The chunk's package (per stage: codes 512 bytes, the 2048/g scales and
+// zeros) comes into a per-warp ring of shared-memory slots, completing on the
+// slot's mbarrier: by one bulk copy per stage and array from lane 0 up to
+// k = 2, by per-lane 16-byte cp.async copies from k = 3 (RtCfg).  Each lane
+// reads its 16 code bytes and its group's scale and zero from there.  At k = 1 the lane forms its 64
 // levels and then converts them; for k >= 2 it sums 4 weights over all k
 // stages (in stage order, as Eq. 8 reads) before the next 4, converting as
 // it goes, which keeps few accumulators live and leaves room for 12 warps a
@@ -30,10 +31,15 @@ namespace {
 // of package in flight per warp.  For k >= 2 a lane finishes 4 weights over
 // all k stages before the next 4 (few live accumulators), which leaves room
 // for 12 warps a CTA with two chunks in flight.  Two CTAs per multiprocessor
-// in both.
+// in both.  Up to k = 2 lane 0 brings a chunk in with one bulk copy per
+// array; from k = 3 on (3k copies, most of them of 64 bytes) every lane
+// copies its own 16-byte units with cp.async instead, and the warp index is
+// taken by a broadcast so that the copy and store operands are known to be
+// warp-uniform.
 template <int K>
 struct RtCfg {
   static constexpr bool kOuter = K > 1;
+  static constexpr bool kLaneCopies = K > 2;
   static constexpr int kWarps = kOuter ? 12 : 8;
   static constexpr int kThreads = kWarps * 32;
   static constexpr int kRing = kOuter ? 2 : 3;  // chunks of package per warp in flight
@@ -79,7 +85,8 @@ __global__ void __launch_bounds__(RtCfg<K>::kThreads, kRtCtasPerSm) reconstruct_
   uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
   const ReconstructBatch& b = p.b;
   const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
+  const int warp = RtCfg<K>::kLaneCopies ? __shfl_sync(kFullMask, static_cast<int>(threadIdx.x >> 5), 0)
+                                         : static_cast<int>(threadIdx.x >> 5);
   uint8_t* out_stage = smem + warp * kRtOutBytes;                                      // 4 KiB, 1024-aligned
   uint8_t* ring = smem + kRtWarps * kRtOutBytes + warp * kRtRing * rt_slot_bytes<G, K, F>();
   const uint32_t ring_s = smem_u32(ring);
@@ -91,7 +98,7 @@ __global__ void __launch_bounds__(RtCfg<K>::kThreads, kRtCtasPerSm) reconstruct_
 
   if (lane == 0) {
 #pragma unroll
-    for (int i = 0; i < kRtRing; ++i) mbar_init(bar0 + 8 * i, 1);
+    for (int i = 0; i < kRtRing; ++i) mbar_init(bar0 + 8 * i, RtCfg<K>::kLaneCopies ? 32 : 1);
     fence_mbarrier_init();
   }
   __syncwarp();
@@ -118,11 +125,45 @@ __global__ void __launch_bounds__(RtCfg<K>::kThreads, kRtCtasPerSm) reconstruct_
                   reinterpret_cast<const uint8_t*>(it.zeros[i]) + c * St::kZeros, St::kZeros, bar);
     }
   };
-  if (lane == 0) {
+  // (from k = 3) every lane copies its 16-byte units of the slot (the slot
+  // holds the K code arrays, then the K scale arrays, then the K zero
+  // arrays, each unit at its own index) and arrives on the slot's barrier
+  // when they land
+  auto issue_all = [&](int64_t chunk, int slot) {
+    const int m = item_of(chunk, m_issue);
+    const ReconstructItem& it = b.item[m];
+    const int64_t c = chunk - it.chunk_begin;
+    constexpr int kCodeU = St::kCodes / 16, kScaleU = St::kScales / 16, kZeroU = St::kZeros / 16;
+    constexpr int kUnits = K * (kCodeU + kScaleU + kZeroU);
+    static_assert(kCodeU == 32, "one code unit per lane and stage");
+    const uint32_t dst = ring_s + slot * rt_slot_bytes<G, K, F>() + lane * 16;
 #pragma unroll
-    for (int i = 0; i < kRtRing; ++i) {
-      const int64_t c = first + i * stride;
-      if (c < b.total_chunks) issue(c, i);
+    for (int t = 0; t < (kUnits + 31) / 32; ++t) {
+      const int u = t * 32 + lane;
+      if (t < K) {
+        cp_async_16(dst + t * 512, it.codes[t] + c * St::kCodes + lane * 16, 16);
+      } else if (u < kUnits) {
+        const int v = u - K * kCodeU;
+        const uint8_t* src;
+        constexpr int kZeroD = kZeroU > 0 ? kZeroU : 1;  // no zeros on the symmetric grid
+        if (kZeroU == 0 || v < K * kScaleU)
+          src = static_cast<const uint8_t*>(it.scales[v / kScaleU]) + c * St::kScales + (v % kScaleU) * 16;
+        else
+          src = reinterpret_cast<const uint8_t*>(it.zeros[(v - K * kScaleU) / kZeroD]) + c * St::kZeros +
+                ((v - K * kScaleU) % kZeroD) * 16;
+        cp_async_16(dst + t * 512, src, 16);
+      }
+    }
+    cp_async_mbar_arrive_noinc(bar0 + 8 * slot);
+  };
+#pragma unroll
+  for (int i = 0; i < kRtRing; ++i) {
+    const int64_t c = first + i * stride;
+    if (c >= b.total_chunks) break;
+    if constexpr (RtCfg<K>::kLaneCopies) {
+      issue_all(c, i);
+    } else if (lane == 0) {
+      issue(c, i);
     }
   }
 
@@ -138,6 +179,10 @@ __global__ void __launch_bounds__(RtCfg<K>::kThreads, kRtCtasPerSm) reconstruct_
     if (!__all_sync(kFullMask, ready)) {
       // Give up: record it, wait (bounded) for this warp's copies in flight
       // so that none lands in freed shared memory, and leave.
+      if constexpr (RtCfg<K>::kLaneCopies) {  // this lane's copies landed
+        cp_async_commit();
+        cp_async_wait<0>();
+      }
       if (lane == 0) {
         atomicOr(b.status, kStatusTimeout);
         for (int j = 0; j < kRtRing; ++j) {
@@ -169,11 +214,17 @@ __global__ void __launch_bounds__(RtCfg<K>::kThreads, kRtCtasPerSm) reconstruct_
         ok = ok && (kSym || prescale_ok(scale[i][h]));
       }
     }
-    fence_proxy_async_smem();  // this lane's reads before the next async write of the slot
-    __syncwarp();
-    if (lane == 0) {
+    if constexpr (RtCfg<K>::kLaneCopies) {
+      __syncwarp();  // every lane's reads of the slot before its refill
       const int64_t next = chunk + kRtRing * stride;
-      if (next < b.total_chunks) issue(next, slot);
+      if (next < b.total_chunks) issue_all(next, slot);
+    } else {
+      fence_proxy_async_smem();  // this lane's reads before the next async write of the slot
+      __syncwarp();
+      if (lane == 0) {
+        const int64_t next = chunk + kRtRing * stride;
+        if (next < b.total_chunks) issue(next, slot);
+      }
     }
     const int m = item_of(chunk, m_work);
     const ReconstructItem& it = b.item[m];

@@ -148,6 +148,12 @@ template <int N>
 __device__ __forceinline__ void cp_async_wait() {
   asm volatile("cp.async.wait_group %0;" ::"n"(N) : "memory");
 }
+// Arrives on `bar` once every earlier cp.async of this thread has landed,
+// without raising the barrier's expected count (the count given at init
+// includes this arrival).
+__device__ __forceinline__ void cp_async_mbar_arrive_noinc(uint32_t bar) {
+  asm volatile("cp.async.mbarrier.arrive.noinc.shared::cta.b64 [%0];" ::"r"(bar) : "memory");
+}
 
 // ---------------------------------------------------------------------------
 // packed fp32x2 arithmetic (one instruction, two independent IEEE binary32

@@ -157,8 +157,9 @@ def test_timeout_path_reports_and_recovers():
     records RRQ_ERR_TIMEOUT, drains its own copies and returns; the device
     stays usable and the next call is exact again.  Both builds (the 2-D
     tile form and the 1-D ring form) and the one-prefix reconstruction of a
-    whole number of 2048-weight chunks wait on their bulk copies; the
-    reconstruction of other sizes has no bounded waits."""
+    whole number of 2048-weight chunks wait on barriers: the builds and that
+    reconstruction up to k = 2 on bulk copies, from k = 3 on per-lane
+    copies; the reconstruction of other sizes has no bounded waits."""
     W = workloads.generate(512, 1024, 21, "normal", "cuda")      # tile forms
     V = workloads.generate(3, 1024 + 32, 22, "normal", "cuda")   # 1-D forms (n % 64 != 0)
     binding.rrq_get_device_status()  # clear
@@ -171,6 +172,8 @@ def test_timeout_path_reports_and_recovers():
         binding.rrq_quantize(V, 32, 4)
         assert binding.rrq_get_device_status() == 5
         binding.rrq_reconstruct(pkg, 4)
+        assert binding.rrq_get_device_status() == 5
+        binding.rrq_reconstruct(pkg, 2)
         assert binding.rrq_get_device_status() == 5
         binding.rrq_reconstruct(pkv, 4)  # cp.async copies complete in hardware
         assert binding.rrq_get_device_status() == 0
