@@ -728,7 +728,9 @@ quantize_kernel(const __grid_constant__ QuantizeBatch p) {
   constexpr bool kBase = M == kModeBase;
   extern __shared__ __align__(128) uint8_t smem[];
   const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
+  // the warp index by broadcast: the compiler then knows it (and every copy
+  // and store operand derived from it) to be warp-uniform
+  const int warp = __shfl_sync(kFullMask, static_cast<int>(threadIdx.x >> 5), 0);
   uint8_t* ring = smem + warp * (kRing * kChunkBytes);
   const uint32_t ring_s = smem_u32(ring);
   const uint32_t bar0 = smem_u32(smem + kWarps * kRing * kChunkBytes) + warp * kRing * 8;
