@@ -167,7 +167,9 @@ gemv_mma_kernel(const __grid_constant__ GemvBatch p, int nb, int ring_off, int D
   constexpr int kSlot = mma_slot_bytes(kSym, G, S);
   extern __shared__ __align__(16) uint8_t smem[];
   const int lane = threadIdx.x & 31;
-  const int warp = threadIdx.x >> 5;
+  // the warp index by broadcast: the compiler then treats it, and the item
+  // and copy addresses derived from it, as warp-uniform
+  const int warp = __shfl_sync(kFullMask, static_cast<int>(threadIdx.x >> 5), 0);
   const int t = lane & 3, rq = lane >> 2;
   const int64_t blk_begin = p.cta_begin[blockIdx.x];
   const int64_t blk_end = p.cta_begin[blockIdx.x + 1];

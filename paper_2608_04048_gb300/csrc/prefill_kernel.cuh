@@ -360,7 +360,9 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   auto share_done = [&](int s) { return drain + 8 + 8 * s; };
   const bool codes_tma = p.codes_tma != 0;
 
-  const int warp = threadIdx.x >> 5;
+  // warp index and tensor-memory address by broadcast: the compiler then
+  // treats the copy and MMA operands derived from them as warp-uniform
+  const int warp = __shfl_sync(kFullMask, static_cast<int>(threadIdx.x >> 5), 0);
   const int lane = threadIdx.x & 31;
 
   // this CTA's tile: clusters in token-tile-major order, rank = token tile
@@ -407,7 +409,7 @@ __global__ void __launch_bounds__(kPfThreads, 1) prefill_kernel(const __grid_con
   tc_fence_before();
   __syncthreads();
   tc_fence_after();
-  const uint32_t tmem = *slot;
+  const uint32_t tmem = __shfl_sync(kFullMask, *slot, 0);
   if constexpr (CS > 1) cluster_sync();  // every CTA's barriers exist before any remote access
 
   if (warp == kPfTmaWarp) {
