@@ -14,7 +14,9 @@ one read of W.  The metric is bf16 weight bytes processed per second of step
 time (GB/s).  The stacks' inputs are far larger than L2; the smaller
 workloads flush L2 before every timed call.  The breakdown times the package
 alone (rrq_quantize), every prefix from the package and each prefix by its
-own call, with a roofline entry for each.
+own call, with a roofline entry for each; on the stacks it also replays the
+step's launches from one CUDA graph (`step_cuda_graph`) beside the eager
+timing.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME]
                     [--split] [--impl reference]
@@ -419,6 +421,34 @@ class L2Flush:
         self.buf.fill_(self.n)
 
 
+def time_graph(wl, calls, reps: int):
+    """Seconds per pass of `calls` replayed from one CUDA graph that holds
+    their launches (captured once on a side stream, relaxed capture mode),
+    after one untimed replay; (None, reason) if the capture is refused."""
+    old = wl.stream
+    side = torch.cuda.Stream(device=wl.device)
+    graph = torch.cuda.CUDAGraph()
+    try:
+        side.wait_stream(old)
+        wl.stream = side
+        with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
+            for c in calls:
+                c()
+    except Exception as e:  # reported in the breakdown, never a silent fallback
+        return None, f"{type(e).__name__}: {e}"[:200]
+    finally:
+        wl.stream = old
+    with torch.cuda.stream(side):
+        graph.replay()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(side)
+        for _ in range(reps):
+            graph.replay()
+        b.record(side)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps / 1e3, None
+
+
 def time_calls(calls, stream, reps: int, flush=None) -> float:
     """Mean seconds of one pass over `calls` (after one untimed pass).
     With `flush`, L2 is flushed before every call and only the calls are
@@ -625,6 +655,9 @@ def run_gpu(args, world, rank, local) -> dict | None:
     q_by_group = {g: time_calls([c], stream, 3, flush) for g, c in zip(groups, q_calls)} if len(groups) > 1 else None
     r_s = time_calls(wl.reconstruct_calls(None), stream, 3, flush)
     each_k = {k: time_calls(wl.reconstruct_calls(k), stream, 2, flush) for k in KS}
+    # the step's launches replayed from a CUDA graph (stacks: no L2 flush
+    # between calls), beside the eager timing above
+    graph_s, graph_err = time_graph(wl, steps_calls, args.steps) if flush is None else (None, None)
     torch.cuda.synchronize()
     if binding.rrq_get_device_status() != 0:
         raise RuntimeError("a kernel reported a timeout in the breakdown")
@@ -710,6 +743,14 @@ def run_gpu(args, world, rank, local) -> dict | None:
         },
         "breakdown": {
             "step_alg_gbs": round(f_alg / f_s / 1e9, 1),
+            "step_cuda_graph": None if flush is not None else (
+                {"error": graph_err} if graph_s is None else {
+                    "ms_per_step": round(graph_s * 1e3, 3),
+                    "bf16_gbs": round(bytes_bf16 / graph_s / 1e9, 2),
+                    "frac_of_measured_hbm": round(f_alg / graph_s / 1e9 / hbm, 4),
+                    "api_calls_per_step": len(steps_calls),
+                    "kernel_launches_per_step": launches,
+                    "eager_ms_per_step": round(elapsed_ms / args.steps, 3)}),
             "step_frac_of_measured_hbm": round(f_alg / f_s / 1e9 / hbm, 4),
             "two_calls_s_per_stack": round(q_s + r_s, 6),
             "two_calls_bf16_gbs": round(bytes_bf16 / (q_s + r_s) / 1e9, 2),

@@ -5,6 +5,7 @@
 #include <atomic>
 #include <cstdint>
 #include <cstring>
+#include <map>
 #include <mutex>
 #include <vector>
 
@@ -117,12 +118,12 @@ class BufferCheck {
 
  private:
   bool known(uintptr_t a, uintptr_t* end) const {
-    for (const auto& r : seen_)
-      if (a >= r.first && a < r.second) {
-        *end = r.second;
-        return true;
-      }
-    return false;
+    auto it = seen_.upper_bound(a);  // the first allocation starting after a
+    if (it == seen_.begin()) return false;
+    --it;
+    if (a >= it->second) return false;
+    *end = it->second;
+    return true;
   }
   bool lookup(uintptr_t a, uintptr_t* end) {
     PointerAttrsFn fn = pointer_attrs();
@@ -139,13 +140,13 @@ class BufferCheck {
     const bool device = managed || (type == CU_MEMORYTYPE_DEVICE && ordinal == dev_);
     const uintptr_t s = static_cast<uintptr_t>(start), e = s + size;
     if (!device || size == 0 || a < s || a >= e) return false;
-    seen_.push_back({s, e});
+    seen_[s] = e;
     *end = e;
     return true;
   }
 
   int dev_;
-  std::vector<std::pair<uintptr_t, uintptr_t>> seen_;
+  std::map<uintptr_t, uintptr_t> seen_;  // allocation start -> end (disjoint)
 };
 
 // Byte ranges touched by a call; outputs may not overlap anything else.
