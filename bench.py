@@ -163,7 +163,7 @@ def time_gemv(pkgs, specs, stream, batch: int = 1, reps: int = 5) -> dict:
     out = {"call": f"rrq_gemv over all {len(specs)} matrices, batch {batch} (asymmetric binary32 package)"}
     for k in KS:
         items = binding.gemv_descs(pkgs, acts, ys, k)
-        run = lambda: binding.rrq_gemv(pkgs, acts, k, ys, stream, items)
+        run = lambda st=stream: binding.rrq_gemv(pkgs, acts, k, ys, st, items)
         run()
         a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         a.record(stream)
@@ -178,7 +178,34 @@ def time_gemv(pkgs, specs, stream, batch: int = 1, reps: int = 5) -> dict:
                         "frac_of_measured_hbm": round(alg / t / 1e9 / hbm, 4),
                         "weights_per_s": round(sum(sp.numel for sp in specs) / t, 1),
                         "weight_row_products_per_s": round(sum(sp.numel for sp in specs) * batch / t, 1)}
+        if batch == 1:  # the same call's launches replayed from a CUDA graph (no host work per pass)
+            tg, err = graph_seconds(run, stream, reps)
+            out[f"k{k}"]["cuda_graph"] = {"error": err} if tg is None else {
+                "s_per_stack": round(tg, 6), "frac_of_measured_hbm": round(alg / tg / 1e9 / hbm, 4)}
     return out
+
+
+def graph_seconds(run, stream, reps: int):
+    """Seconds per pass of run(stream) replayed from one CUDA graph captured
+    on a side stream (relaxed capture mode), after one untimed replay;
+    (None, reason) if the capture is refused."""
+    side = torch.cuda.Stream(device=stream.device)
+    graph = torch.cuda.CUDAGraph()
+    try:
+        side.wait_stream(stream)
+        with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
+            run(side)
+    except Exception as e:  # reported in the breakdown, never a silent fallback
+        return None, f"{type(e).__name__}: {e}"[:200]
+    with torch.cuda.stream(side):
+        graph.replay()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(side)
+        for _ in range(reps):
+            graph.replay()
+        b.record(side)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps / 1e3, None
 
 
 def time_prefill(pkgs, specs, stream, tokens: int = 2048, reps: int = 2) -> dict:
@@ -422,31 +449,18 @@ class L2Flush:
 
 
 def time_graph(wl, calls, reps: int):
-    """Seconds per pass of `calls` replayed from one CUDA graph that holds
-    their launches (captured once on a side stream, relaxed capture mode),
-    after one untimed replay; (None, reason) if the capture is refused."""
+    """Seconds per pass of `calls` (the workload's calls, which launch on
+    wl.stream) replayed from one CUDA graph; see graph_seconds."""
     old = wl.stream
-    side = torch.cuda.Stream(device=wl.device)
-    graph = torch.cuda.CUDAGraph()
-    try:
-        side.wait_stream(old)
+
+    def run(side):
         wl.stream = side
-        with torch.cuda.graph(graph, stream=side, capture_error_mode="relaxed"):
+        try:
             for c in calls:
                 c()
-    except Exception as e:  # reported in the breakdown, never a silent fallback
-        return None, f"{type(e).__name__}: {e}"[:200]
-    finally:
-        wl.stream = old
-    with torch.cuda.stream(side):
-        graph.replay()
-        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-        a.record(side)
-        for _ in range(reps):
-            graph.replay()
-        b.record(side)
-    torch.cuda.synchronize()
-    return a.elapsed_time(b) / reps / 1e3, None
+        finally:
+            wl.stream = old
+    return graph_seconds(run, old, reps)
 
 
 def time_calls(calls, stream, reps: int, flush=None) -> float:
