@@ -160,3 +160,15 @@ def test_ex_argument_checks_run_before_cuda(lib):
     r.out_bf16[0] = base + 0x10004
     items = (binding.ReconstructDesc * 1)(r)
     assert lib.rrq_reconstruct_ex(items, 1, ctypes.byref(_fmt(n_stages=1)), 1, 0, None) == 3
+
+
+def test_missing_library_fails_loudly(monkeypatch, tmp_path):
+    """Without the built library every entry point raises: there is no CPU
+    fallback to take its place."""
+    import torch
+    monkeypatch.setattr(binding, "_LIB", None)
+    monkeypatch.setattr(binding, "library_path", lambda: str(tmp_path / "librrq.so"))
+    with pytest.raises(RuntimeError, match="missing"):
+        binding.load_library()
+    with pytest.raises((RuntimeError, TypeError)):
+        binding.rrq_quantize(torch.zeros(4, 128, dtype=torch.bfloat16))
